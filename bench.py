@@ -1,0 +1,453 @@
+#!/usr/bin/env python
+"""Benchmark of the cached Picard solver step on GB300.
+
+Workload (default): SD-v1.5-shaped cached Picard DDIM -- T=100, window 100,
+batch 1, 4x64x64 fp32 latents, 16-component mixture denoiser, tol 1e-3,
+tau_cache 0.05 (synthetic seeded inputs). One bench step = one complete
+generation (every Picard iteration until t = T). ``value`` is Picard solver
+steps (iterations) per second, whole job: the iterations all ranks ran divided
+by the slowest rank's device time, measured with CUDA events around every
+iteration (gather, mixture denoiser, update, decision). L2 (129 MB) is flushed
+before every iteration by writing a 256 MiB buffer, outside the timed events,
+because the whole working set (~35 MB) would otherwise stay L2-resident.
+
+Also reported: the roofline of the dominant kernel (the Picard update), the
+end-to-end rate through the public API with host buffers (``e2e``), the fp64
+oracle timed on the host cores (``cpu_baseline``), NFE and hit rate.
+
+``--impl reference`` times the fp64 CPU oracle (the only reference this
+method has: the paper ships no code) on the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import workload as W  # noqa: E402
+
+METRIC = "Picard+cache solver steps/s and HBM GB/s vs peak at T=100, 4x64x64; NFE"
+UNIT = "solver steps/s"
+FLUSH_BYTES = 256 << 20
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+# ncu DRAM bytes of the update kernel per launch, keyed by the sha256 of its
+# source file at capture time (profiles/ has the capture); reported as null
+# when the kernel source has changed since.
+NCU_TRAFFIC = {}
+
+
+def parse_args(argv=None):
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=sorted(W.ALL), default="sd15")
+    ap.add_argument("--no-flush", action="store_true", help="do not flush L2 between iterations")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--update-kernel", type=int, default=None, choices=[0, 1])
+    ap.add_argument("--oracle-sample", type=float, default=None, help=argparse.SUPPRESS)
+    return ap.parse_args(argv)
+
+
+# ---------------------------------------------------------------- ranks ----
+
+def rank_info():
+    env = os.environ
+    return (int(env.get("RANK", 0)), int(env.get("WORLD_SIZE", 1)), int(env.get("LOCAL_RANK", 0)))
+
+
+def rank_workload(w: W.Workload, rank: int) -> W.Workload:
+    """Weak scaling: rank r runs its own trajectories, seeds offset by r * batch."""
+    return w.with_(seed=w.seed + rank * w.batch)
+
+
+def aggregate(units_local, seconds_local, group=None):
+    """(sum of units over ranks, max seconds over ranks) -- host-side timing only."""
+    import torch
+    import torch.distributed as dist
+    if not (dist.is_available() and dist.is_initialized()):
+        return float(units_local), float(seconds_local)
+    dev = "cuda" if dist.get_backend(group) == "nccl" else "cpu"
+    u = torch.tensor([float(units_local)], dtype=torch.float64, device=dev)
+    s = torch.tensor([float(seconds_local)], dtype=torch.float64, device=dev)
+    dist.all_reduce(u, op=dist.ReduceOp.SUM, group=group)
+    dist.all_reduce(s, op=dist.ReduceOp.MAX, group=group)
+    return float(u.item()), float(s.item())
+
+
+def barrier():
+    import torch.distributed as dist
+    if dist.is_available() and dist.is_initialized():
+        dist.barrier()
+
+
+# -------------------------------------------------------------- helpers ----
+
+def measured_hbm_gbs():
+    try:
+        with open(PEAKS_PATH) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def kernel_source_sha():
+    import hashlib
+    p = os.path.join(ROOT, "paper_2609_36522_gb300", "csrc", "k_update_bulk.cu")
+    return hashlib.sha256(open(p, "rb").read()).hexdigest()[:16]
+
+
+def iteration_bytes(log, w: W.Workload):
+    """Algorithmic bytes per Picard iteration, from the solver's iteration log.
+
+    Per trajectory with window start t, p points, m misses, frontier e and h1
+    hits at positions >= 1 (rows of D fp32 values):
+      update : x_t, the p - lazy materialised old states, p eps rows, m ehat
+               and m xhat writes, h1 xhat reads (next distances), p new states
+      gather : m reads + m writes;  denoiser: m reads + m writes (+ K means)
+    """
+    row = w.D * 4
+    upd, other = [], []
+    for k in range(log.shape[0]):
+        u = o = 0
+        for b in range(log.shape[1]):
+            t, p, m, stride, e, h1 = (int(v) for v in log[k, b, :6])
+            if p == 0:
+                continue
+            lazy = max(0, t + p - e)
+            u += (1 + (p - lazy) + p + 2 * m + h1 + p) * row
+            o += 4 * m * row
+        upd.append(u)
+        other.append(o + w.K * row)
+    return np.array(upd, dtype=np.float64), np.array(other, dtype=np.float64)
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 100 ms."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        os.unlink(self.path)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None,
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# --------------------------------------------------------- oracle timing ----
+
+def oracle_sample(workload_name, budget_s):
+    """Time the fp64 oracle on whole generations of the workload for about
+    budget_s seconds (at least one generation). Runs in a fresh process."""
+    from oracle import run_picard
+    from oracle.gmm import make_eps_fn
+    w = W.ALL[workload_name]
+    a, x0, mu = W.inputs(w)
+    f = make_eps_fn(a, mu, w.gmm_std)
+    iters = gens = 0
+    t0 = time.perf_counter()
+    while True:
+        r = run_picard(a, x0, f, w.window, w.tol, w.cache_thresh, record=False)
+        iters += r.iters
+        gens += 1
+        if time.perf_counter() - t0 >= budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"iters": iters, "generations": gens, "seconds": dt, "nfe_per_gen": r.nfe,
+            "iters_per_gen": r.iters}
+
+
+def time_oracle_subprocess(workload_name, budget_s):
+    env = dict(os.environ)
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[k] = "1"
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", workload_name,
+                        "--oracle-sample", str(budget_s)], capture_output=True, text=True, env=env)
+    if r.returncode != 0:
+        raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
+    return json.loads(r.stdout.strip().splitlines()[-1])
+
+
+def cpu_baseline(workload_name, budget_s=12.0):
+    s = time_oracle_subprocess(workload_name, budget_s)
+    return {"value": s["iters"] / s["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"{s['generations']} full generation(s) of the workload "
+                      f"({s['iters']} Picard iterations, {s['seconds']:.1f} s) by the fp64 NumPy "
+                      f"oracle, single-threaded (BLAS/OpenMP threads = 1)"}
+
+
+# ------------------------------------------------------------ reference ----
+
+def run_reference(args):
+    rank, world, _ = rank_info()
+    if rank != 0:
+        return 0
+    w = W.ALL[args.workload]
+    # each step: one whole generation by the oracle, in its own process
+    for _ in range(args.warmup):
+        time_oracle_subprocess(args.workload, 0.0)
+    iters = 0
+    secs = 0.0
+    for _ in range(args.steps):
+        s = time_oracle_subprocess(args.workload, 0.0)
+        iters += s["iters"]
+        secs += s["seconds"]
+    value = iters / secs
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000.0 * secs / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": w.name, "step": "one full cached-Picard generation",
+                   "global_batch": w.batch, "seq_len": w.T, "window": w.window},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
+                         "sample": f"{args.steps} full generation(s), fp64 NumPy oracle, "
+                                   f"single-threaded"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ------------------------------------------------------------------ ours ----
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+    from paper_2609_36522_gb300 import abi
+    from paper_2609_36522_gb300 import build as pa_build
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+
+    rank, world, local = rank_info()
+    if world > 1:
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    if local == 0 or world == 1:
+        pa_build.build()
+    barrier()
+    w = rank_workload(W.ALL[args.workload], rank)
+    a, x0, mu = W.inputs(w)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.current_stream()
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=stream)
+    if args.update_kernel is not None:
+        s.set_update_kernel(args.update_kernel)
+    max_rows = w.batch * s.window
+    g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows, stream=stream)
+    eps = torch.empty(max_rows, w.D, dtype=torch.float32, device=dev)
+    x_dev = torch.from_numpy(x0).to(dev)
+    flush = None if args.no_flush else torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def generation_async(n_iters, ev=None):
+        s.init(x_dev)
+        for it in range(n_iters):
+            if flush is not None:
+                flush.zero_()
+            if ev is not None:
+                ev[it][0].record(stream)
+            bx, mb, nm = s.step_async()
+            g.eps(bx, mb, nm, eps)
+            s.submit_eps(eps)
+            if ev is not None:
+                ev[it][1].record(stream)
+
+    # learn the iteration count with the synchronous API (also a warm-up)
+    s.init(x_dev)
+    n_iters = 0
+    while True:
+        out = s.step()
+        if out is None:
+            break
+        n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
+        g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+        s.submit_eps(eps)
+        n_iters += 1
+    st0 = s.stats()
+    log = s.iter_log()
+    nfe, hits = st0["nfe"], st0["hits"]
+    upd_bytes, other_bytes = iteration_bytes(log, w)
+
+    for _ in range(args.warmup):
+        generation_async(n_iters)
+    assert s.poll() == 0, "solver did not finish within the learned iteration count"
+    torch.cuda.synchronize()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    events = [[[torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)]
+               for _ in range(n_iters)] for _ in range(args.steps)]
+    abi.pa_set_kernel_timing(s.h, True)
+    abi.pa_kernel_timing(s.h)  # reset
+    launches0 = s.stats()["launches"] + g.launches()
+    barrier()
+    torch.cuda.synchronize()
+    wall0 = time.perf_counter()
+    for k in range(args.steps):
+        generation_async(n_iters, events[k])
+    torch.cuda.synchronize()
+    barrier()
+    wall = time.perf_counter() - wall0
+    upd_ms, upd_n = abi.pa_kernel_timing(s.h)
+    abi.pa_set_kernel_timing(s.h, False)
+    launches = s.stats()["launches"] + g.launches() - launches0
+    assert s.poll() == 0
+    st1 = s.stats()
+    assert st1["iters"] == n_iters and st1["nfe"] == nfe, (st1, n_iters, nfe)
+    dev_ms = sum(events[k][it][0].elapsed_time(events[k][it][1])
+                 for k in range(args.steps) for it in range(n_iters))
+    time.sleep(0.2)
+    clk = clocks.stop()
+
+    units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
+    value = units / secs
+    gb_step = (upd_bytes.sum() + other_bytes.sum()) * args.steps / (dev_ms / 1000.0) / 1e9
+
+    # roofline of the dominant kernel (Picard update)
+    peak, peak_kind = measured_hbm_gbs()
+    achieved = upd_bytes.sum() * args.steps / (upd_ms / 1000.0) / 1e9
+    sha = kernel_source_sha()
+    traffic = NCU_TRAFFIC.get(sha)
+    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak, "traffic": traffic,
+                "kernel": "Picard update (" + ("bulk-copy pipeline" if st1["update_kernel"] == 1
+                                               else "plain loads") + ")",
+                "peak_kind": f"{peak_kind} HBM copy bandwidth",
+                "alg_bytes_per_launch": float(upd_bytes.mean()),
+                "avg_launch_us": 1000.0 * upd_ms / max(upd_n, 1)}
+
+    # end to end through the public API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        x_host = torch.from_numpy(x0).pin_memory()
+        out_host = torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory()
+        ctl_reads = 0
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        reps = max(3, min(args.steps, 50))
+        e0.record(stream)
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            s.init(x_host)
+            while True:
+                out = s.step()
+                ctl_reads += 1
+                if out is None:
+                    break
+                n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
+                g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+                s.submit_eps(eps)
+            s.result(out_host)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_s = max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0)
+        units_e, secs_e = aggregate(reps * n_iters, e2e_s)
+        e2e = {"value": units_e / secs_e, "unit": UNIT,
+               "h2d_bytes_per_step": int(w.batch * w.D * 4),
+               "d2h_bytes_per_step": int(w.batch * w.D * 4 + (ctl_reads // reps) * 32),
+               "steps": reps}
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args.workload)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": dev_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": w.name, "step": "one full cached-Picard generation",
+                       "picard_iters_per_step": n_iters, "global_batch": w.batch * world,
+                       "seq_len": w.T, "window": w.window, "latent": "x".join(map(str, w.latent_shape)),
+                       "mixture_components": w.K, "tol": w.tol, "cache_thresh": w.cache_thresh,
+                       "parallelism": f"replicas x{world} (independent trajectories)",
+                       "l2": ("not flushed" if args.no_flush else
+                              "256 MiB write before every Picard iteration, outside the timed events"),
+                       "timing": "CUDA events around each Picard iteration on the launch stream"},
+            "nfe_per_step": nfe, "hits_per_step": hits,
+            "hit_rate": hits / max(1, hits + nfe),
+            "solver_step_gbps": gb_step,
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": int(launches),
+            "clocks": clk,
+            "wall_s_timed_region": wall,
+        }
+        print(json.dumps(line))
+    s.close()
+    g.close()
+    if world > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    args = parse_args(argv)
+    if args.oracle_sample is not None:
+        print(json.dumps(oracle_sample(args.workload, args.oracle_sample)))
+        return 0
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,214 @@
+/*
+ * paraanya.h -- C ABI of the GB300 (sm_103a) cached Picard solver step.
+ *
+ * The library implements one Picard iteration of sliding-window parallel DDIM
+ * sampling (ParaDiGMS-style) with ParaAnya's output cache:
+ *
+ *   Sec. 2.1, Eq. 1   Picard update  x_{t+j+1} <- x_t + sum_{i=t}^{t+j} s(x_i, eps_i)
+ *   Sec. 2.1, Eq. 2   convergence    (1/D) ||x^{k+1}_i - x^k_i||^2 <= tau
+ *   Sec. 2.2, Eq. 3   cache map      C: t -> (xhat_t, ehat_t)
+ *   Sec. 2.2, Eq. 4   cache distance delta_t = (1/D) ||x_t - xhat_t||_1
+ *   Sec. 2.2, Eq. 5   hit iff delta_t < tau_cache; first entry is a miss
+ *   Sec. 2.2, Eq. 6   eps_t = ehat_t (hit) or eps_theta(x_t, t) (miss)
+ *   Sec. 2.2, Eq. 7   cache update for misses only
+ *
+ * Call order:  pa_create -> pa_init -> ( pa_step -> denoise -> pa_submit_eps )*
+ *              -> pa_step returns PA_DONE -> pa_result -> pa_destroy.
+ * pa_step_async / pa_poll are the host-sync-free variant of pa_step for
+ * denoisers that read the miss count on the device (e.g. pa_gmm_eps).
+ * Any other order returns PA_ERR_STATE and changes nothing.
+ *
+ * Conventions
+ *  - Latents are fp32, contiguous, NCHW-flattened: one row of D = prod(shape)
+ *    floats per timestep.
+ *  - Sampling index 0 is the noisiest state (x_0 of Eq. 1 is the initial
+ *    noise); alphas_cumprod has T+1 entries and entry T is the clean end (1.0).
+ *  - Misses are ordered trajectory-major, then by ascending timestep; the
+ *    miss list holds int32 pairs (b, i): trajectory b, absolute timestep i.
+ *  - Device memory: the caller owns every buffer. The solver's internal state
+ *    lives in a caller-allocated device workspace of pa_workspace_bytes()
+ *    bytes (256-byte aligned); the library never calls cudaMalloc. Pointers
+ *    returned by pa_step stay valid until the next pa_submit_eps/pa_destroy.
+ *  - Streams: every kernel and copy of a solver is issued on the stream given
+ *    to pa_create (NULL = legacy default stream).
+ *  - Errors: every call returns a pa_status; nothing throws across the ABI.
+ *    Device-side failures (a bounded wait that ran out, an index check) are
+ *    recorded in a device status word and reported by the next call that
+ *    synchronises (pa_step, pa_poll, pa_result, pa_stats).
+ */
+#ifndef PARAANYA_H
+#define PARAANYA_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define PA_API __attribute__((visibility("default")))
+#else
+#define PA_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct pa_solver pa_solver;   /* opaque, owned by the library */
+typedef struct pa_gmm pa_gmm;         /* opaque, owned by the library */
+
+typedef enum {
+  PA_OK = 0,
+  PA_DONE = 1,           /* every trajectory reached t = T */
+  PA_ERR_ARG = -1,       /* bad argument (size, pointer, alignment) */
+  PA_ERR_STATE = -2,     /* call out of order */
+  PA_ERR_CUDA = -3,      /* a CUDA runtime call failed */
+  PA_ERR_WORKSPACE = -4, /* workspace too small or misaligned */
+  PA_ERR_TIMEOUT = -5,   /* a device-side bounded wait ran out */
+  PA_ERR_DEVICE = -6     /* a device-side consistency check failed */
+} pa_status;
+
+typedef struct {
+  int64_t iters;         /* Picard iterations completed (global loop count) */
+  int64_t nfe;           /* sum over iterations of misses (network evaluations) */
+  int64_t hits;          /* sum over iterations of cache hits */
+  int64_t launches;      /* kernels this handle launched since pa_create */
+  int32_t n_active;      /* trajectories with t < T */
+  int32_t n_miss;        /* misses planned for the next iteration */
+  int32_t device_status; /* 0, or the first device-side error code */
+  int32_t update_kernel; /* kernel of the last pa_submit_eps: 0 plain loads, 1 bulk-copy
+                            pipeline, -1 none yet */
+} pa_stats_t;
+
+/* ---- solver ------------------------------------------------------------ */
+
+/* Bytes of device workspace a solver of these sizes needs (0 on bad sizes).
+ * T: DDIM steps (>= 1); window: P, evaluation points per iteration (1..1024);
+ * D: latent size (>= 1); batch: independent trajectories (1..64). */
+PA_API size_t pa_workspace_bytes(int T, int window, int64_t D, int batch);
+
+/* Create a solver. latent_shape[ndim] gives D = prod(latent_shape).
+ * alphas_cumprod: HOST array, T+1 doubles, sampling order (see above), each in
+ *   (0, 1], non-decreasing not required. The DDIM drift coefficients of Sec. 2.1
+ *   are derived from it on the host in fp64 and stored in fp32.
+ * tol: tau of Eq. 2 (>= 0). cache_thresh: tau_cache of Eq. 5 (>= 0; 0 disables
+ *   hits because the comparison is strict).
+ * workspace_dev: device pointer, 256-byte aligned, >= pa_workspace_bytes().
+ * stream: a cudaStream_t (may be NULL). The handle is written to *out. */
+PA_API pa_status pa_create(pa_solver** out, int T, int window,
+                    const int64_t* latent_shape, int ndim,
+                    const double* alphas_cumprod, double tol, double cache_thresh,
+                    int batch, void* workspace_dev, size_t workspace_bytes,
+                    void* stream);
+
+/* Start a generation: x_init [batch][D] fp32, HOST or DEVICE pointer (the copy
+ * direction is inferred from the address). All states of the first window are
+ * x_init (Sec. 2.1 initial trajectory estimate); every first-window timestep is
+ * a first entry, hence a miss (Sec. 2.2). Clears the cache and counters.
+ * May be called again at any time to restart. */
+PA_API pa_status pa_init(pa_solver* s, const float* x_init);
+
+/* Plan the next iteration: returns in *n_miss the number of misses M
+ * (Eq. 5), in *batch_x_dev the contiguous batch [M][D] of their latents
+ * (gathered on the device), and in *miss_bt_dev the (b, i) list [M][2].
+ * Synchronises the solver's stream once (to read M). Returns PA_DONE (and
+ * M = 0) when every trajectory has finished. */
+PA_API pa_status pa_step(pa_solver* s, int* n_miss, const float** batch_x_dev,
+                  const int32_t** miss_bt_dev);
+
+/* As pa_step without synchronising: *n_miss_dev points to the device int32
+ * holding M. The batch has room for batch*window rows; rows >= M are stale.
+ * Iterating a finished solver is a no-op on the device. */
+PA_API pa_status pa_step_async(pa_solver* s, const float** batch_x_dev,
+                        const int32_t** miss_bt_dev, const int32_t** n_miss_dev);
+
+/* Device address of the int32 holding the planned miss count M (the value
+ * pa_step returns); valid for the solver's lifetime. NULL for a NULL solver. */
+PA_API const int32_t* pa_n_miss_dev(const pa_solver* s);
+
+/* Hand back eps_theta for the planned misses: batch_eps_dev [M][D] fp32,
+ * DEVICE pointer, 16-byte alignment for the bulk-copy pipeline (otherwise the
+ * plain-load kernel runs). Runs Eq. 6 (assembly), Eq. 7 (cache update),
+ * the drift and the Picard prefix sum (Eq. 1), the errors of Eq. 2, the window
+ * advance, and the cache distances / hit-miss plan of the next iteration
+ * (Eq. 4, Eq. 5). Asynchronous on the solver's stream. */
+PA_API pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev);
+
+/* Synchronise and report: *n_active = trajectories not yet at t = T.
+ * Returns PA_DONE when it is 0, or a device error status. */
+PA_API pa_status pa_poll(pa_solver* s, int* n_active);
+
+/* Final states x_T [batch][D] fp32 into a HOST or DEVICE pointer. Valid once
+ * pa_step/pa_poll returned PA_DONE; PA_ERR_STATE before. Synchronises. */
+PA_API pa_status pa_result(pa_solver* s, float* x_out);
+
+/* Network evaluations so far (sum of misses). Synchronises; -1 on error. */
+PA_API int64_t pa_nfe(pa_solver* s);
+
+/* Counters, see pa_stats_t. Synchronises. */
+PA_API pa_status pa_stats(pa_solver* s, pa_stats_t* out);
+
+/* Per-iteration log, HOST buffer out[max_iters][batch][8] int32:
+ * (window start t, evaluation points p, misses of trajectory b, stride,
+ *  evaluated frontier e before the iteration (states > e were lazy copies of
+ *  state e), hits among window positions 1..p-1, 0, 0).
+ * *n_iters receives the number of logged iterations. Synchronises. */
+PA_API pa_status pa_iter_log(pa_solver* s, int32_t* out, int max_iters, int* n_iters);
+
+/* The reductions of the most recent pa_submit_eps, HOST buffers [batch][window]
+ * fp32: err_out[b][j] is Eq. 2's error of state t+j+1 and delta_out[b][j] the
+ * Eq. 4 distance of timestep t+j+1 against its cache entry (valid for j < p-1).
+ * Either pointer may be NULL. Synchronises. */
+PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out);
+
+/* Select the Picard-update kernel: 0 = plain loads, 1 = bulk-copy pipeline
+ * (default when D % 4 == 0). Returns PA_ERR_ARG for an unknown value. */
+PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
+
+/* Enable (1) or disable (0) CUDA-event timing of every Picard-update kernel
+ * launch, recorded on the solver's stream directly around the launch. */
+PA_API pa_status pa_set_kernel_timing(pa_solver* s, int enable);
+
+/* Sum of the update-kernel durations in ms, and how many launches were timed,
+ * since the previous call (which resets both). Synchronises. */
+PA_API pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches);
+
+PA_API void pa_destroy(pa_solver* s);
+
+/* ---- synthetic denoiser: posterior-mean eps of an isotropic Gaussian mixture
+ * (stand-in for the SD v1.5 UNet of Sec. 3.2; not part of the paper's method).
+ * eps*(x) = sqrt(1-a)/v * (x - sqrt(a) * sum_k r_k mu_k),
+ * v = a s^2 + 1 - a, r = softmax_k(-||x - sqrt(a) mu_k||^2 / (2v)), equal weights.
+ * ------------------------------------------------------------------------ */
+
+/* Bytes of device workspace for K components (1..128), latent size D, at most
+ * max_rows rows per call and T sampling steps (0 on bad sizes). */
+PA_API size_t pa_gmm_workspace_bytes(int K, int64_t D, int max_rows, int T);
+
+/* means_dev: DEVICE [K][D] fp32, caller-owned, must outlive the handle.
+ * alphas_cumprod: HOST [T+1] doubles (same array as the solver's).
+ * max_rows: largest batch ever passed (the solver's batch * window). */
+PA_API pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* means_dev,
+                        double std, const double* alphas_cumprod, int T,
+                        int max_rows, void* workspace_dev, size_t workspace_bytes,
+                        void* stream);
+
+/* eps for rows r < *n_rows_dev (DEVICE int32) of batch_x_dev [max_rows][D]:
+ * the timestep of row r is miss_bt_dev[2r+1]. Writes batch_eps_dev [.][D].
+ * Asynchronous on the handle's stream. */
+PA_API pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32_t* miss_bt_dev,
+                     const int32_t* n_rows_dev, float* batch_eps_dev);
+
+/* Kernels launched by this handle since pa_gmm_create. */
+PA_API int64_t pa_gmm_launches(const pa_gmm* g);
+
+PA_API void pa_gmm_destroy(pa_gmm* g);
+
+/* ---- misc -------------------------------------------------------------- */
+
+PA_API const char* pa_status_string(int status);
+/* Last host-side error message of this thread ("" if none). */
+PA_API const char* pa_last_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PARAANYA_H */

@@ -1,0 +1,417 @@
+// Solver-step kernels for sm_103a: first-iteration plan, miss gather (a4),
+// plain-load Picard update (a6-a9, a11) and the decision kernel (a10, a2, a3).
+//
+// Data layout (fp32, one row = one timestep's latent of D floats):
+//   X    [B][P+1][D]  state ring, state i lives in slot i mod (P+1)
+//   Xhat [B][P][D]    cache inputs  xhat_i  (Eq. 3), slot i mod P
+//   Ehat [B][P][D]    cache outputs ehat_i  (Eq. 3), slot i mod P
+//   batch_x [B*P][D]  gathered latents of the misses, rank order
+#include "pa_internal.h"
+
+namespace pa {
+namespace {
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__device__ __forceinline__ void set_status(Ctl* c, int code) {
+  atomicCAS(&c->status, kDevOk, code);
+}
+
+// ---------------------------------------------------------------------------
+// First iteration (after pa_init): every timestep of every first window enters
+// for the first time, hence is a miss (Sec. 2.2). States 1..p are lazy copies
+// of state 0 = x_init, so the frontier e starts at 0.
+__global__ void k_init_plan(Dev d) {
+  const int p0 = min(d.P, d.T);
+  for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
+    Traj tr{};
+    tr.t = 0; tr.p = p0; tr.e = 0; tr.done = 0; tr.m = p0; tr.h1 = 0;
+    d.traj[b] = tr;
+  }
+  for (int q = threadIdx.x; q < d.B * d.P; q += blockDim.x) {
+    const int b = q / d.P, j = q % d.P;
+    if (j < p0) {
+      const int r = b * p0 + j;
+      d.rank[q] = r;
+      d.miss_bt[2 * r] = b;
+      d.miss_bt[2 * r + 1] = j;
+    } else {
+      d.rank[q] = -1;
+    }
+  }
+  if (threadIdx.x == 0) {
+    Ctl c{};
+    c.n_miss = d.B * p0;
+    c.n_active = d.B;
+    c.iter = 0;
+    c.status = kDevOk;
+    c.nfe = (long long)d.B * p0;
+    c.hits = 0;
+    *d.ctl = c;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// a4: batch_x[r] <- x_{miss[r]} for r < n_miss. A lazy state (i > e) reads
+// state e, the value every new tail state was initialised to.
+template <int VEC>
+__global__ void __launch_bounds__(256) k_gather(Dev d) {
+  const int n = d.ctl->n_miss;
+  const int64_t nvec = d.D / VEC;
+  for (int r = blockIdx.y; r < n; r += gridDim.y) {
+    const int b = d.miss_bt[2 * r], i = d.miss_bt[2 * r + 1];
+    const int src = min(i, d.traj[b].e);
+    const float* from = d.X + ((int64_t)b * (d.P + 1) + src % (d.P + 1)) * d.D;
+    float* to = d.batch_x + (int64_t)r * d.D;
+    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < nvec;
+         v += (int64_t)gridDim.x * blockDim.x) {
+      if constexpr (VEC == 4) {
+        reinterpret_cast<float4*>(to)[v] = __ldg(reinterpret_cast<const float4*>(from) + v);
+      } else {
+        to[v] = __ldg(from + v);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Plain-load Picard update. One CTA = one column chunk of one trajectory;
+// each thread owns VEC adjacent columns and walks the window sequentially,
+// which makes the window-axis prefix sum (Eq. 1) a register recurrence.
+// Per window position j (timestep i = t + j):
+//   eps_i  = batch_eps[rank] (miss) or ehat_i (hit)              Eq. 6
+//   miss:  ehat_i <- eps_i, xhat_i <- x_i                         Eq. 7
+//   d_i    = (c_i - 1) x_i + e_i eps_i                            drift
+//   x'_{i+1} = x_t + sum_{l<=j} d_{t+l}  (compensated)            Eq. 1
+//   err_j  partial of sum (x'_{i+1} - x_{i+1})^2                  Eq. 2
+//   del_j  partial of sum |x'_{i+1} - xhat_{i+1}| (next iteration) Eq. 4
+// Partials are reduced per CTA in a fixed order and written to
+// part_*[b][j][chunk]; the decision kernel finishes the reduction.
+template <int VEC>
+struct V;
+template <>
+struct V<1> {
+  float a[1];
+};
+template <>
+struct V<4> {
+  float a[4];
+};
+
+template <int VEC>
+__device__ __forceinline__ V<VEC> ldv(const float* p) {
+  V<VEC> r;
+  if constexpr (VEC == 4) {
+    float4 q = *reinterpret_cast<const float4*>(p);
+    r.a[0] = q.x; r.a[1] = q.y; r.a[2] = q.z; r.a[3] = q.w;
+  } else {
+    r.a[0] = *p;
+  }
+  return r;
+}
+
+template <int VEC>
+__device__ __forceinline__ void stv(float* p, const V<VEC>& v) {
+  if constexpr (VEC == 4) {
+    *reinterpret_cast<float4*>(p) = make_float4(v.a[0], v.a[1], v.a[2], v.a[3]);
+  } else {
+    *p = v.a[0];
+  }
+}
+
+constexpr int kPlainThreads = 128;
+
+template <int VEC>
+__global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const float* __restrict__ beps,
+                                                             int nchunk) {
+  extern __shared__ float red[];  // [2][nwarps][P]
+  const int b = blockIdx.y;
+  const Traj tr = d.traj[b];
+  if (tr.p == 0) return;
+  const int t = tr.t, p = tr.p, e = tr.e, P = d.P;
+  const int64_t D = d.D;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  constexpr int nw = kPlainThreads / 32;
+  const int64_t col = ((int64_t)blockIdx.x * kPlainThreads + threadIdx.x) * VEC;
+  const bool live = col < D;
+  float* Xb = d.X + (int64_t)b * (P + 1) * D + col;
+  float* Xh = d.Xhat + (int64_t)b * P * D + col;
+  float* Eh = d.Ehat + (int64_t)b * P * D + col;
+  const int32_t* rk = d.rank + b * P;
+  const int n_miss = d.ctl->n_miss;
+
+  V<VEC> xcur{}, acc{}, comp{}, xfill{};
+  if (live) xcur = ldv<VEC>(Xb + (int64_t)(t % (P + 1)) * D);
+  acc = xcur;
+  xfill = xcur;  // state e when e == t
+  for (int j = 0; j < p; ++j) {
+    const int i = t + j;
+    const int r = rk[j];
+    if (r >= n_miss) set_status(d.ctl, kDevBadRank);
+    const float cm1 = d.cm1[i], ec = d.ecoef[i];
+    const int slot = i % P;
+    float ev = 0.f, dv = 0.f;
+    if (live) {
+      V<VEC> eps = (r >= 0) ? ldv<VEC>(beps + (int64_t)r * D + col) : ldv<VEC>(Eh + (int64_t)slot * D);
+      if (r >= 0) {
+        stv<VEC>(Eh + (int64_t)slot * D, eps);
+        stv<VEC>(Xh + (int64_t)slot * D, xcur);
+      }
+      V<VEC> xo;
+      if (i + 1 <= e) {
+        xo = ldv<VEC>(Xb + (int64_t)((i + 1) % (P + 1)) * D);
+        if (i + 1 == e) xfill = xo;
+      } else {
+        xo = xfill;
+      }
+      V<VEC> xn;
+#pragma unroll
+      for (int v = 0; v < VEC; ++v) {
+        const float dr = cm1 * xcur.a[v] + ec * eps.a[v];
+        const float y = dr - comp.a[v];
+        const float s = acc.a[v] + y;
+        comp.a[v] = (s - acc.a[v]) - y;
+        acc.a[v] = s;
+        xn.a[v] = s;
+        const float df = xn.a[v] - xo.a[v];
+        ev += df * df;
+      }
+      stv<VEC>(Xb + (int64_t)((i + 1) % (P + 1)) * D, xn);
+      if (j + 1 < p) {
+        const int r1 = rk[j + 1];
+        V<VEC> xh = (r1 >= 0) ? xo : ldv<VEC>(Xh + (int64_t)((i + 1) % P) * D);
+#pragma unroll
+        for (int v = 0; v < VEC; ++v) dv += fabsf(xn.a[v] - xh.a[v]);
+      }
+      xcur = xo;
+    }
+    ev = warp_sum(ev);
+    dv = warp_sum(dv);
+    if (lane == 0) {
+      red[warp * P + j] = ev;
+      red[(nw + warp) * P + j] = dv;
+    }
+  }
+  __syncthreads();
+  for (int j = threadIdx.x; j < p; j += kPlainThreads) {
+    float se = 0.f, sd = 0.f;
+#pragma unroll
+    for (int w = 0; w < nw; ++w) {
+      se += red[w * P + j];
+      sd += red[(nw + w) * P + j];
+    }
+    const int64_t o = ((int64_t)b * P + j) * nchunk + blockIdx.x;
+    d.part_err[o] = se;
+    d.part_del[o] = sd;
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Decision kernel (one CTA of 1024 threads):
+//  1. finish the reductions: err[b][j] (Eq. 2) and delta of timestep t+j+1
+//     (Eq. 4), summing the chunk partials in a fixed order (deterministic);
+//  2. per trajectory: stride = min(p, 1 + #leading err_j <= tol), advance
+//     t, shrink p = min(P, T - t), frontier e = old t + p, done at t = T;
+//  3. plan the next iteration: a timestep of the new window with a cache
+//     entry (i < e) hits iff delta < tau_cache (strict, Eq. 5), everything
+//     else misses; misses are compacted trajectory-major into miss_bt with a
+//     block-wide prefix sum, and rank[b][j] records each miss's batch row.
+constexpr int kDecideThreads = 1024;
+
+__global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
+  __shared__ int s_t[kMaxBatch], s_p[kMaxBatch], s_e[kMaxBatch];
+  __shared__ int s_tn[kMaxBatch], s_pn[kMaxBatch], s_m[kMaxBatch], s_h1[kMaxBatch];
+  __shared__ int s_warp[kDecideThreads / 32];
+  __shared__ int s_total;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int nwarps = kDecideThreads / 32;
+  const int B = d.B, P = d.P, T = d.T;
+  if (d.ctl->n_active == 0) return;  // finished: iterating further is a no-op
+  const int iter = d.ctl->iter;
+
+  for (int b = tid; b < B; b += kDecideThreads) {
+    const Traj tr = d.traj[b];
+    s_t[b] = tr.t; s_p[b] = tr.p; s_e[b] = tr.e;
+    s_m[b] = 0;
+    s_h1[b] = 0;
+  }
+  __syncthreads();
+
+  // 1. reductions, one warp per (b, j)
+  for (int q = warp; q < B * P; q += nwarps) {
+    const int b = q / P, j = q % P;
+    if (j >= s_p[b]) continue;
+    const float* pe = d.part_err + (int64_t)q * nchunk;
+    const float* pd = d.part_del + (int64_t)q * nchunk;
+    float se = 0.f, sd = 0.f;
+    for (int c = lane; c < nchunk; c += 32) {
+      se += pe[c];
+      sd += pd[c];
+    }
+    se = warp_sum(se);
+    sd = warp_sum(sd);
+    if (lane == 0) {
+      d.red_err[q] = se / (float)d.D;
+      d.red_del[q] = sd / (float)d.D;
+    }
+  }
+  __syncthreads();
+
+  // 2. window advance, one warp per trajectory
+  for (int b = warp; b < B; b += nwarps) {
+    const int t = s_t[b], p = s_p[b];
+    if (p == 0) {
+      if (lane == 0) {
+        s_tn[b] = t; s_pn[b] = 0;
+        int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+        for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
+        lg[0] = t;
+      }
+      continue;
+    }
+    int lead = p;
+    for (int j0 = 0; j0 < p; j0 += 32) {
+      const int j = j0 + lane;
+      const bool fail = (j < p) && !((double)d.red_err[b * P + j] <= d.tol);
+      const unsigned m = __ballot_sync(0xffffffffu, fail);
+      if (m) {
+        lead = j0 + __ffs(m) - 1;
+        break;
+      }
+    }
+    if (lane == 0) {
+      const int stride = min(p, 1 + lead);
+      const int tn = t + stride;
+      s_tn[b] = tn;
+      s_pn[b] = min(P, T - tn);
+      const Traj old = d.traj[b];
+      int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+      lg[0] = t; lg[1] = p; lg[2] = old.m; lg[3] = stride;
+      lg[4] = old.e; lg[5] = old.h1; lg[6] = 0; lg[7] = 0;
+    }
+  }
+  __syncthreads();
+
+  // 3. hit/miss plan of the next iteration and its compaction
+  const int N = B * P;
+  const int per = (N + kDecideThreads - 1) / kDecideThreads;
+  const int q0 = tid * per, q1 = min(N, q0 + per);
+  auto is_miss = [&](int q) -> int {
+    const int b = q / P, j = q % P;
+    if (j >= s_pn[b]) return 0;
+    const int i = s_tn[b] + j;
+    const int en = s_t[b] + s_p[b];  // new frontier
+    if (i >= en) return 1;           // first entry
+    const int jo = i - s_t[b] - 1;   // delta of timestep i was computed at old position jo
+    return ((double)d.red_del[b * P + jo] < d.cache_thresh) ? 0 : 1;
+  };
+  int cnt = 0;
+  for (int q = q0; q < q1; ++q) cnt += is_miss(q);
+  // block exclusive scan of cnt
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_warp[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    int w = s_warp[lane];
+    int wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += v;
+    }
+    s_warp[lane] = wi - w;  // exclusive
+    if (lane == 31) s_total = wi;
+  }
+  __syncthreads();
+  int r = s_warp[warp] + incl - cnt;
+  for (int q = q0; q < q1; ++q) {
+    const int b = q / P, j = q % P;
+    if (is_miss(q)) {
+      d.rank[q] = r;
+      d.miss_bt[2 * r] = b;
+      d.miss_bt[2 * r + 1] = s_tn[b] + j;
+      atomicAdd(&s_m[b], 1);
+      ++r;
+    } else {
+      d.rank[q] = -1;
+      if (j >= 1 && j < s_pn[b]) atomicAdd(&s_h1[b], 1);
+    }
+  }
+  __syncthreads();
+  int pts = 0;
+  for (int b = 0; b < B; ++b) pts += s_pn[b];
+  for (int b = tid; b < B; b += kDecideThreads) {
+    Traj tr{};
+    tr.t = s_tn[b];
+    tr.p = s_pn[b];
+    tr.e = (s_p[b] > 0) ? s_t[b] + s_p[b] : s_e[b];
+    tr.done = (s_pn[b] == 0);
+    tr.m = s_m[b];
+    tr.h1 = s_h1[b];
+    if (tr.t > T || tr.e < tr.t) set_status(d.ctl, kDevBadState);
+    d.traj[b] = tr;
+  }
+  if (tid == 0) {
+    int act = 0;
+    for (int b = 0; b < B; ++b) act += (s_pn[b] > 0);
+    const int n = s_total;
+    d.ctl->n_miss = n;
+    d.ctl->n_active = act;
+    d.ctl->iter = iter + 1;
+    d.ctl->nfe += n;
+    d.ctl->hits += pts - n;
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_init_plan(const Dev& d, cudaStream_t st) {
+  k_init_plan<<<1, 256, 0, st>>>(d);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather(const Dev& d, cudaStream_t st) {
+  const int rows = min(d.B * d.P, 65535);
+  if (d.D % 4 == 0) {
+    const int64_t nvec = d.D / 4;
+    const int64_t want = (nvec + 255) / 256;
+    const int gx = (int)(want < 64 ? want : 64);
+    k_gather<4><<<dim3(gx, rows), 256, 0, st>>>(d);
+  } else {
+    const int64_t want = (d.D + 255) / 256;
+    const int gx = (int)(want < 256 ? want : 256);
+    k_gather<1><<<dim3(gx, rows), 256, 0, st>>>(d);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream_t st,
+                                int* nchunk_out) {
+  const size_t smem = (size_t)2 * (kPlainThreads / 32) * d.P * sizeof(float);
+  if (d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0) {
+    const int nchunk = (int)((d.D + kPlainThreads * 4 - 1) / (kPlainThreads * 4));
+    *nchunk_out = nchunk;
+    k_update_plain<4><<<dim3(nchunk, d.B), kPlainThreads, smem, st>>>(d, batch_eps, nchunk);
+  } else {
+    const int nchunk = (int)((d.D + kPlainThreads - 1) / kPlainThreads);
+    *nchunk_out = nchunk;
+    k_update_plain<1><<<dim3(nchunk, d.B), kPlainThreads, smem, st>>>(d, batch_eps, nchunk);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st) {
+  k_decide<<<1, kDecideThreads, 0, st>>>(d, nchunk);
+  return cudaGetLastError();
+}
+
+}  // namespace pa

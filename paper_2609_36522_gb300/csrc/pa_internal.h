@@ -1,0 +1,110 @@
+// Internal layout shared by the host state machine (pa_solver.cpp) and the
+// kernels (k_solver.cu, k_update_bulk.cu). Not part of the public ABI.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace pa {
+
+constexpr int kMaxWindow = 1024;
+constexpr int kMaxBatch = 64;
+constexpr int kMinChunk = 32;       // narrowest column chunk of any update kernel
+constexpr size_t kAlign = 256;
+
+// Device status codes written by kernels (first error wins, atomicCAS from 0).
+constexpr int kDevOk = 0;
+constexpr int kDevTimeout = 1;      // a bounded mbarrier wait ran out
+constexpr int kDevBadRank = 2;      // a miss rank outside [0, n_miss)
+constexpr int kDevBadState = 3;     // trajectory bookkeeping inconsistent
+
+// Per-trajectory window bookkeeping.
+//  t : window start (the converged state x_t, Sec. 2.1 sliding window)
+//  p : evaluation points t..t+p-1 this iteration (0 once t == T)
+//  e : evaluated frontier: timesteps < e have a cache entry (Eq. 3); states
+//      0..e hold real values in the state ring; states > e are "lazy" and
+//      equal state e (new tail states copy the last computed state).
+//  m : misses of trajectory b in the planned iteration (for the iteration log)
+//  h1: hits among window positions 1..p-1 of the planned iteration (their xhat
+//      rows are read for the next iteration's distances; for the byte count)
+struct Traj {
+  int32_t t, p, e, done, m, h1, pad0, pad1;
+};
+constexpr int kLogFields = 8;  // iteration log entry: t, p, misses, stride, e, h1, 0, 0
+
+struct Ctl {
+  int32_t n_miss;     // misses planned for the next iteration (Eq. 5)
+  int32_t n_active;   // trajectories with t < T
+  int32_t iter;       // iterations completed
+  int32_t status;     // kDev* code
+  long long nfe;
+  long long hits;
+};
+
+struct Layout {
+  size_t X, Xhat, Ehat, batch_x, coef, traj, ctl, rank, miss_bt;
+  size_t part_err, part_del, red_err, red_del, iter_log, total;
+  int64_t part_cap;   // floats per partial array
+};
+
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+inline Layout make_layout(int T, int P, int64_t D, int B) {
+  Layout L{};
+  size_t o = 0;
+  auto take = [&](size_t bytes) { size_t at = o; o = align_up(o + bytes, kAlign); return at; };
+  const size_t row = (size_t)D * sizeof(float);
+  L.X = take((size_t)B * (P + 1) * row);          // state ring, slot = i mod (P+1)
+  L.Xhat = take((size_t)B * P * row);             // cache inputs, slot = i mod P
+  L.Ehat = take((size_t)B * P * row);             // cache outputs, slot = i mod P
+  L.batch_x = take((size_t)B * P * row);          // gathered misses
+  L.coef = take((size_t)2 * T * sizeof(float));   // (c_i - 1, e_i)
+  L.traj = take((size_t)B * sizeof(Traj));
+  L.ctl = take(sizeof(Ctl));
+  L.rank = take((size_t)B * P * sizeof(int32_t));
+  L.miss_bt = take((size_t)B * P * 2 * sizeof(int32_t));
+  L.part_cap = (int64_t)B * P * ((D + kMinChunk - 1) / kMinChunk);
+  L.part_err = take((size_t)L.part_cap * sizeof(float));
+  L.part_del = take((size_t)L.part_cap * sizeof(float));
+  L.red_err = take((size_t)B * P * sizeof(float));
+  L.red_del = take((size_t)B * P * sizeof(float));
+  L.iter_log = take((size_t)(T + 1) * B * kLogFields * sizeof(int32_t));
+  L.total = o;
+  return L;
+}
+
+// Device views of one solver's workspace.
+struct Dev {
+  float* X;
+  float* Xhat;
+  float* Ehat;
+  float* batch_x;
+  const float* cm1;   // c_i - 1
+  const float* ecoef; // e_i
+  Traj* traj;
+  Ctl* ctl;
+  int32_t* rank;      // [B][P] rank of window position j among the misses, -1 = hit
+  int32_t* miss_bt;   // [B*P][2]
+  float* part_err;    // [B][P][nchunk]
+  float* part_del;
+  float* red_err;     // [B][P]
+  float* red_del;
+  int32_t* iter_log;  // [T+1][B][kLogFields]
+  int T, P, B;
+  int64_t D;
+  double tol, cache_thresh;   // compared against fp32 reductions promoted to double
+};
+
+// Kernel launchers (k_solver.cu). Each returns the launch error.
+cudaError_t launch_init_plan(const Dev& d, cudaStream_t st);
+cudaError_t launch_gather(const Dev& d, cudaStream_t st);
+cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream_t st,
+                                int* nchunk_out);
+cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st);
+// k_update_bulk.cu
+cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st,
+                               int* nchunk_out);
+bool update_bulk_supported(const Dev& d, const float* batch_eps);
+
+}  // namespace pa

@@ -1,0 +1,409 @@
+// Host side of the C ABI: argument checks, the call-order state machine,
+// workspace carving, DDIM drift coefficients and kernel dispatch.
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "../../include/paraanya.h"
+#include "pa_internal.h"
+
+namespace pa {
+
+static thread_local std::string g_err;
+void set_error(const std::string& msg) { g_err = msg; }
+
+}  // namespace pa
+
+namespace {
+
+enum class St { Created, Ready, Stepped, Done };
+
+}  // namespace
+
+struct pa_solver {
+  pa::Dev d;
+  pa::Layout L;
+  char* ws;
+  cudaStream_t st;
+  St state;
+  int update_kind;   // requested: 0 plain, 1 bulk pipeline
+  int last_kind;     // kernel the last pa_submit_eps actually launched (-1: none yet)
+  int last_nchunk;
+  int64_t launches;
+  pa::Ctl* host_ctl; // pinned mirror of the device Ctl
+  // optional CUDA-event timing of the Picard-update kernel
+  bool timing;
+  std::vector<cudaEvent_t> ev;  // pairs: [2k] before, [2k+1] after launch k
+  size_t ev_next;               // pairs recorded since the last read
+};
+
+namespace {
+
+pa_status cuda_fail(const char* where, cudaError_t e) {
+  pa::set_error(std::string(where) + ": " + cudaGetErrorString(e));
+  return PA_ERR_CUDA;
+}
+
+pa_status arg_fail(const std::string& msg) {
+  pa::set_error(msg);
+  return PA_ERR_ARG;
+}
+
+pa_status state_fail(const char* where) {
+  pa::set_error(std::string(where) + ": call out of order");
+  return PA_ERR_STATE;
+}
+
+bool sizes_ok(int T, int P, int64_t D, int B) {
+  return T >= 1 && P >= 1 && P <= pa::kMaxWindow && D >= 1 && B >= 1 && B <= pa::kMaxBatch &&
+         D <= ((int64_t)1 << 40);
+}
+
+// Copy the device Ctl into the pinned mirror and wait. Returns a status for
+// a CUDA failure or a device-side error.
+pa_status sync_ctl(pa_solver* s, const char* where) {
+  cudaError_t e = cudaMemcpyAsync(s->host_ctl, s->d.ctl, sizeof(pa::Ctl), cudaMemcpyDeviceToHost, s->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);
+  if (e != cudaSuccess) return cuda_fail(where, e);
+  const int ds = s->host_ctl->status;
+  if (ds == pa::kDevTimeout) {
+    pa::set_error(std::string(where) + ": a device-side bounded wait ran out");
+    return PA_ERR_TIMEOUT;
+  }
+  if (ds != pa::kDevOk) {
+    pa::set_error(std::string(where) + ": device-side check failed (code " + std::to_string(ds) + ")");
+    return PA_ERR_DEVICE;
+  }
+  return PA_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* pa_last_error(void) { return pa::g_err.c_str(); }
+
+const char* pa_status_string(int status) {
+  switch (status) {
+    case PA_OK: return "PA_OK";
+    case PA_DONE: return "PA_DONE";
+    case PA_ERR_ARG: return "PA_ERR_ARG";
+    case PA_ERR_STATE: return "PA_ERR_STATE";
+    case PA_ERR_CUDA: return "PA_ERR_CUDA";
+    case PA_ERR_WORKSPACE: return "PA_ERR_WORKSPACE";
+    case PA_ERR_TIMEOUT: return "PA_ERR_TIMEOUT";
+    case PA_ERR_DEVICE: return "PA_ERR_DEVICE";
+    default: return "PA_UNKNOWN";
+  }
+}
+
+size_t pa_workspace_bytes(int T, int window, int64_t D, int batch) {
+  if (!sizes_ok(T, window, D, batch)) return 0;
+  const int P = window < T ? window : T;
+  return pa::make_layout(T, P, D, batch).total;
+}
+
+pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_shape, int ndim,
+                    const double* alphas_cumprod, double tol, double cache_thresh, int batch,
+                    void* workspace_dev, size_t workspace_bytes, void* stream) {
+  if (!out) return arg_fail("pa_create: out is NULL");
+  *out = nullptr;
+  if (!latent_shape || ndim < 1 || ndim > 8) return arg_fail("pa_create: latent_shape/ndim invalid");
+  int64_t D = 1;
+  for (int k = 0; k < ndim; ++k) {
+    if (latent_shape[k] < 1) return arg_fail("pa_create: latent_shape entries must be >= 1");
+    D *= latent_shape[k];
+    if (D > ((int64_t)1 << 40)) return arg_fail("pa_create: latent too large");
+  }
+  if (!sizes_ok(T, window, D, batch))
+    return arg_fail("pa_create: need T >= 1, 1 <= window <= 1024, 1 <= batch <= 64");
+  if (!alphas_cumprod) return arg_fail("pa_create: alphas_cumprod is NULL");
+  for (int i = 0; i <= T; ++i) {
+    const double a = alphas_cumprod[i];
+    if (!(a > 0.0 && a <= 1.0)) return arg_fail("pa_create: alphas_cumprod entries must be in (0, 1]");
+  }
+  if (!(tol >= 0.0) || !std::isfinite(tol)) return arg_fail("pa_create: tol must be finite and >= 0");
+  if (!(cache_thresh >= 0.0) || std::isnan(cache_thresh))
+    return arg_fail("pa_create: cache_thresh must be >= 0");
+  const int P = window < T ? window : T;
+  const pa::Layout L = pa::make_layout(T, P, D, batch);
+  if (!workspace_dev || (reinterpret_cast<uintptr_t>(workspace_dev) % pa::kAlign) != 0 ||
+      workspace_bytes < L.total) {
+    pa::set_error("pa_create: workspace NULL, not 256-byte aligned, or smaller than pa_workspace_bytes()");
+    return PA_ERR_WORKSPACE;
+  }
+
+  pa_solver* s = new pa_solver{};
+  s->L = L;
+  s->ws = static_cast<char*>(workspace_dev);
+  s->st = static_cast<cudaStream_t>(stream);
+  s->state = St::Created;
+  s->launches = 0;
+  s->last_nchunk = 0;
+  s->last_kind = -1;
+  char* w = s->ws;
+  pa::Dev& d = s->d;
+  d.X = reinterpret_cast<float*>(w + L.X);
+  d.Xhat = reinterpret_cast<float*>(w + L.Xhat);
+  d.Ehat = reinterpret_cast<float*>(w + L.Ehat);
+  d.batch_x = reinterpret_cast<float*>(w + L.batch_x);
+  float* coef = reinterpret_cast<float*>(w + L.coef);
+  d.cm1 = coef;
+  d.ecoef = coef + T;
+  d.traj = reinterpret_cast<pa::Traj*>(w + L.traj);
+  d.ctl = reinterpret_cast<pa::Ctl*>(w + L.ctl);
+  d.rank = reinterpret_cast<int32_t*>(w + L.rank);
+  d.miss_bt = reinterpret_cast<int32_t*>(w + L.miss_bt);
+  d.part_err = reinterpret_cast<float*>(w + L.part_err);
+  d.part_del = reinterpret_cast<float*>(w + L.part_del);
+  d.red_err = reinterpret_cast<float*>(w + L.red_err);
+  d.red_del = reinterpret_cast<float*>(w + L.red_del);
+  d.iter_log = reinterpret_cast<int32_t*>(w + L.iter_log);
+  d.T = T; d.P = P; d.B = batch; d.D = D;
+  d.tol = tol;
+  d.cache_thresh = cache_thresh;
+  s->update_kind = (D % 4 == 0) ? 1 : 0;
+
+  // DDIM (eta = 0) step i -> i+1 written as x + s(x, eps) with
+  // s = (c_i - 1) x + e_i eps; c_i - 1 is formed without cancellation.
+  std::vector<float> hc(2 * (size_t)T);
+  for (int i = 0; i < T; ++i) {
+    const double a = alphas_cumprod[i], an = alphas_cumprod[i + 1];
+    const double r = an / a;
+    const double c = std::sqrt(r);
+    const double cm1 = (r - 1.0) / (c + 1.0);
+    const double e = std::sqrt(1.0 - an) - std::sqrt(an) * std::sqrt(1.0 - a) / std::sqrt(a);
+    hc[i] = (float)cm1;
+    hc[T + i] = (float)e;
+  }
+  cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), sizeof(pa::Ctl), cudaHostAllocDefault);
+  if (e != cudaSuccess) {
+    delete s;
+    return cuda_fail("pa_create: cudaHostAlloc", e);
+  }
+  std::memset(s->host_ctl, 0, sizeof(pa::Ctl));
+  e = cudaMemcpyAsync(coef, hc.data(), hc.size() * sizeof(float), cudaMemcpyHostToDevice, s->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(d.ctl, 0, sizeof(pa::Ctl), s->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);
+  if (e != cudaSuccess) {
+    cudaFreeHost(s->host_ctl);
+    delete s;
+    return cuda_fail("pa_create", e);
+  }
+  *out = s;
+  return PA_OK;
+}
+
+pa_status pa_init(pa_solver* s, const float* x_init) {
+  if (!s) return arg_fail("pa_init: solver is NULL");
+  if (!x_init) return arg_fail("pa_init: x_init is NULL");
+  const pa::Dev& d = s->d;
+  // state 0 of every trajectory <- x_init; the rest of the first window is lazy
+  cudaError_t e = cudaMemcpy2DAsync(d.X, (size_t)(d.P + 1) * d.D * sizeof(float), x_init,
+                                    (size_t)d.D * sizeof(float), (size_t)d.D * sizeof(float), d.B,
+                                    cudaMemcpyDefault, s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_init: copy x_init", e);
+  e = pa::launch_init_plan(d, s->st);
+  s->launches++;
+  if (e != cudaSuccess) return cuda_fail("pa_init: launch", e);
+  s->state = St::Ready;
+  return PA_OK;
+}
+
+pa_status pa_step_async(pa_solver* s, const float** batch_x_dev, const int32_t** miss_bt_dev,
+                        const int32_t** n_miss_dev) {
+  if (!s) return arg_fail("pa_step_async: solver is NULL");
+  if (s->state != St::Ready) return state_fail("pa_step_async");
+  const cudaError_t e = pa::launch_gather(s->d, s->st);
+  s->launches++;
+  if (e != cudaSuccess) return cuda_fail("pa_step_async: gather", e);
+  if (batch_x_dev) *batch_x_dev = s->d.batch_x;
+  if (miss_bt_dev) *miss_bt_dev = s->d.miss_bt;
+  if (n_miss_dev) *n_miss_dev = &s->d.ctl->n_miss;
+  s->state = St::Stepped;
+  return PA_OK;
+}
+
+pa_status pa_step(pa_solver* s, int* n_miss, const float** batch_x_dev, const int32_t** miss_bt_dev) {
+  if (!s) return arg_fail("pa_step: solver is NULL");
+  if (!n_miss) return arg_fail("pa_step: n_miss is NULL");
+  *n_miss = 0;
+  if (s->state == St::Done) return PA_DONE;
+  if (s->state != St::Ready) return state_fail("pa_step");
+  pa_status r = pa_step_async(s, batch_x_dev, miss_bt_dev, nullptr);
+  if (r != PA_OK) return r;
+  r = sync_ctl(s, "pa_step");
+  if (r != PA_OK) {
+    s->state = St::Ready;
+    return r;
+  }
+  if (s->host_ctl->n_active == 0) {
+    s->state = St::Done;
+    return PA_DONE;
+  }
+  *n_miss = s->host_ctl->n_miss;
+  return PA_OK;
+}
+
+const int32_t* pa_n_miss_dev(const pa_solver* s) { return s ? &s->d.ctl->n_miss : nullptr; }
+
+pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
+  if (!s) return arg_fail("pa_submit_eps: solver is NULL");
+  if (s->state != St::Stepped) return state_fail("pa_submit_eps");
+  if (!batch_eps_dev) return arg_fail("pa_submit_eps: batch_eps is NULL");
+  int nchunk = 0;
+  cudaError_t e = cudaSuccess;
+  if (s->timing) {
+    if (s->ev_next * 2 + 2 > s->ev.size()) {
+      for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
+        cudaEvent_t x;
+        e = cudaEventCreate(&x);
+        if (e == cudaSuccess) s->ev.push_back(x);
+      }
+    }
+    if (e == cudaSuccess) e = cudaEventRecord(s->ev[2 * s->ev_next], s->st);
+    if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
+  }
+  if (s->update_kind == 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
+    e = pa::launch_update_bulk(s->d, batch_eps_dev, s->st, &nchunk);
+    s->last_kind = 1;
+  } else {
+    e = pa::launch_update_plain(s->d, batch_eps_dev, s->st, &nchunk);
+    s->last_kind = 0;
+  }
+  s->launches++;
+  if (e != cudaSuccess) return cuda_fail("pa_submit_eps: update", e);
+  if (s->timing) {
+    e = cudaEventRecord(s->ev[2 * s->ev_next + 1], s->st);
+    if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
+    s->ev_next++;
+  }
+  s->last_nchunk = nchunk;
+  e = pa::launch_decide(s->d, nchunk, s->st);
+  s->launches++;
+  if (e != cudaSuccess) return cuda_fail("pa_submit_eps: decide", e);
+  s->state = St::Ready;
+  return PA_OK;
+}
+
+pa_status pa_poll(pa_solver* s, int* n_active) {
+  if (!s) return arg_fail("pa_poll: solver is NULL");
+  if (s->state == St::Created) return state_fail("pa_poll");
+  const pa_status r = sync_ctl(s, "pa_poll");
+  if (r != PA_OK) return r;
+  if (n_active) *n_active = s->host_ctl->n_active;
+  if (s->host_ctl->n_active == 0 && s->state == St::Ready) {
+    s->state = St::Done;
+  }
+  return (s->host_ctl->n_active == 0) ? PA_DONE : PA_OK;
+}
+
+pa_status pa_result(pa_solver* s, float* x_out) {
+  if (!s) return arg_fail("pa_result: solver is NULL");
+  if (!x_out) return arg_fail("pa_result: x_out is NULL");
+  if (s->state != St::Done) return state_fail("pa_result");
+  const pa::Dev& d = s->d;
+  const float* src = d.X + (int64_t)(d.T % (d.P + 1)) * d.D;
+  cudaError_t e = cudaMemcpy2DAsync(x_out, (size_t)d.D * sizeof(float), src,
+                                    (size_t)(d.P + 1) * d.D * sizeof(float), (size_t)d.D * sizeof(float),
+                                    d.B, cudaMemcpyDefault, s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_result", e);
+  return sync_ctl(s, "pa_result");
+}
+
+int64_t pa_nfe(pa_solver* s) {
+  if (!s || s->state == St::Created) return -1;
+  if (sync_ctl(s, "pa_nfe") != PA_OK) return -1;
+  return s->host_ctl->nfe;
+}
+
+pa_status pa_stats(pa_solver* s, pa_stats_t* out) {
+  if (!s || !out) return arg_fail("pa_stats: NULL argument");
+  std::memset(out, 0, sizeof(*out));
+  out->launches = s->launches;
+  out->update_kernel = s->last_kind;
+  if (s->state == St::Created) return PA_OK;
+  const pa_status r = sync_ctl(s, "pa_stats");
+  const pa::Ctl& c = *s->host_ctl;
+  out->iters = c.iter;
+  out->nfe = c.nfe;
+  out->hits = c.hits;
+  out->n_active = c.n_active;
+  out->n_miss = c.n_miss;
+  out->device_status = c.status;
+  return r;
+}
+
+pa_status pa_iter_log(pa_solver* s, int32_t* out, int max_iters, int* n_iters) {
+  if (!s || !out || !n_iters || max_iters < 0) return arg_fail("pa_iter_log: bad argument");
+  *n_iters = 0;
+  if (s->state == St::Created) return state_fail("pa_iter_log");
+  const pa_status r = sync_ctl(s, "pa_iter_log");
+  if (r != PA_OK) return r;
+  const int n = s->host_ctl->iter < max_iters ? s->host_ctl->iter : max_iters;
+  if (n > 0) {
+    const cudaError_t e = cudaMemcpy(out, s->d.iter_log,
+                                     (size_t)n * s->d.B * pa::kLogFields * sizeof(int32_t),
+                                     cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail("pa_iter_log", e);
+  }
+  *n_iters = n;
+  return PA_OK;
+}
+
+pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out) {
+  if (!s) return arg_fail("pa_last_reductions: solver is NULL");
+  if (s->state == St::Created) return state_fail("pa_last_reductions");
+  cudaError_t e = cudaStreamSynchronize(s->st);
+  const size_t bytes = (size_t)s->d.B * s->d.P * sizeof(float);
+  if (e == cudaSuccess && err_out) e = cudaMemcpy(err_out, s->d.red_err, bytes, cudaMemcpyDeviceToHost);
+  if (e == cudaSuccess && delta_out) e = cudaMemcpy(delta_out, s->d.red_del, bytes, cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail("pa_last_reductions", e);
+  return PA_OK;
+}
+
+pa_status pa_set_update_kernel(pa_solver* s, int kind) {
+  if (!s) return arg_fail("pa_set_update_kernel: solver is NULL");
+  if (kind != 0 && kind != 1) return arg_fail("pa_set_update_kernel: kind must be 0 or 1");
+  s->update_kind = kind;
+  return PA_OK;
+}
+
+pa_status pa_set_kernel_timing(pa_solver* s, int enable) {
+  if (!s) return arg_fail("pa_set_kernel_timing: solver is NULL");
+  s->timing = (enable != 0);
+  return PA_OK;
+}
+
+pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches) {
+  if (!s || !update_ms || !n_launches) return arg_fail("pa_kernel_timing: NULL argument");
+  *update_ms = 0.0;
+  *n_launches = 0;
+  cudaError_t e = cudaStreamSynchronize(s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_kernel_timing", e);
+  double tot = 0.0;
+  for (size_t k = 0; k < s->ev_next; ++k) {
+    float ms = 0.f;
+    e = cudaEventElapsedTime(&ms, s->ev[2 * k], s->ev[2 * k + 1]);
+    if (e != cudaSuccess) return cuda_fail("pa_kernel_timing: elapsed", e);
+    tot += ms;
+  }
+  *update_ms = tot;
+  *n_launches = (int64_t)s->ev_next;
+  s->ev_next = 0;
+  return PA_OK;
+}
+
+void pa_destroy(pa_solver* s) {
+  if (!s) return;
+  cudaStreamSynchronize(s->st);
+  for (cudaEvent_t x : s->ev) cudaEventDestroy(x);
+  if (s->host_ctl) cudaFreeHost(s->host_ctl);
+  delete s;
+}
+
+}  // extern "C"

@@ -1,0 +1,156 @@
+"""Thin torch-side handles over the C ABI.
+
+PyTorch provides device memory (the workspaces are ``torch.uint8`` CUDA
+tensors from the caching allocator) and the stream; every computation is a
+kernel of libparaanya.so. Device outputs of the library are exposed as views
+into the workspace, never copied.
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from collections import namedtuple
+
+from . import abi
+
+# One planned iteration: M misses, views of the gathered batch and the miss
+# list (both [M][...], empty when M == 0), and the raw device addresses (valid
+# even when M == 0, for device-side denoisers that read M themselves).
+Plan = namedtuple("Plan", "n_miss batch_x miss_bt batch_x_ptr miss_bt_ptr")
+
+
+def _stream_ptr(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream), stream
+
+
+class Solver:
+    """Cached sliding-window Picard DDIM solver of ``batch`` trajectories."""
+
+    def __init__(self, T, window, latent_shape, alphas_cumprod, tol, cache_thresh,
+                 batch=1, stream=None, device="cuda"):
+        if not torch.cuda.is_available():
+            raise RuntimeError("Solver needs a CUDA device; there is no CPU implementation")
+        self.T, self.batch = int(T), int(batch)
+        self.window = min(int(window), self.T)
+        self.latent_shape = tuple(int(v) for v in latent_shape)
+        self.D = int(np.prod(self.latent_shape))
+        self.stream_ptr, self.stream = _stream_ptr(stream)
+        nbytes = abi.pa_workspace_bytes(self.T, int(window), self.D, self.batch)
+        if nbytes == 0:
+            raise abi.PaError("pa_workspace_bytes", abi.PA_ERR_ARG, "unsupported sizes")
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=device)
+        self.h = abi.pa_create(self.T, int(window), self.latent_shape, list(alphas_cumprod),
+                               tol, cache_thresh, self.batch, self.workspace.data_ptr(),
+                               nbytes, self.stream_ptr)
+
+    # -- views into the workspace -------------------------------------------
+    def _view(self, ptr, n, dtype, shape):
+        off = int(ptr) - self.workspace.data_ptr()
+        nb = int(np.prod(shape)) * torch.tensor([], dtype=dtype).element_size()
+        return self.workspace[off: off + nb].view(dtype).view(*shape)
+
+    def init(self, x_init):
+        """x_init: [batch][D] fp32 tensor (CUDA or CPU, contiguous)."""
+        x = x_init if isinstance(x_init, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(x_init))
+        if x.dtype != torch.float32 or not x.is_contiguous() or x.numel() != self.batch * self.D:
+            raise ValueError("x_init must be a contiguous float32 [batch][D] tensor")
+        self._x_init_keepalive = x
+        abi.pa_init(self.h, x.data_ptr())
+
+    def step(self):
+        """-> None when done, else a Plan (M, batch_x [M][D], miss_bt [M][2], raw pointers)."""
+        st, n, bx, mb = abi.pa_step(self.h)
+        if st == abi.PA_DONE:
+            return None
+        return Plan(n, self._view(bx, n, torch.float32, (n, self.D)),
+                    self._view(mb, n, torch.int32, (n, 2)), bx, mb)
+
+    def step_async(self):
+        """-> (batch_x_ptr, miss_bt_ptr, n_miss_dev_ptr), no host synchronisation."""
+        return abi.pa_step_async(self.h)
+
+    def n_miss_dev(self):
+        """Device address of the planned miss count (for device-side denoisers)."""
+        return abi.pa_n_miss_dev(self.h)
+
+    def submit_eps(self, eps):
+        if isinstance(eps, torch.Tensor):
+            if eps.dtype != torch.float32 or not eps.is_cuda or not eps.is_contiguous():
+                raise ValueError("eps must be a contiguous CUDA float32 tensor")
+            eps = eps.data_ptr()
+        abi.pa_submit_eps(self.h, eps)
+
+    def poll(self):
+        st, n = abi.pa_poll(self.h)
+        return n
+
+    def result(self, out=None):
+        if out is None:
+            out = torch.empty(self.batch, self.D, dtype=torch.float32, device=self.workspace.device)
+        abi.pa_result(self.h, out.data_ptr())
+        return out
+
+    def nfe(self):
+        return abi.pa_nfe(self.h)
+
+    def stats(self):
+        return abi.pa_stats(self.h)
+
+    def iter_log(self):
+        return abi.pa_iter_log(self.h, self.T + 1, self.batch)
+
+    def last_reductions(self):
+        return abi.pa_last_reductions(self.h, self.batch, self.window)
+
+    def set_update_kernel(self, kind):
+        abi.pa_set_update_kernel(self.h, kind)
+
+    def close(self):
+        if getattr(self, "h", None) is not None:
+            abi.pa_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+class GmmDenoiser:
+    """Posterior-mean eps of an isotropic Gaussian mixture (synthetic eps_theta)."""
+
+    def __init__(self, means, std, alphas_cumprod, max_rows, stream=None):
+        if not isinstance(means, torch.Tensor) or not means.is_cuda or means.dtype != torch.float32:
+            raise ValueError("means must be a CUDA float32 [K][D] tensor")
+        self.means = means.contiguous()
+        self.K, self.D = self.means.shape
+        self.T = len(alphas_cumprod) - 1
+        self.max_rows = int(max_rows)
+        self.stream_ptr, self.stream = _stream_ptr(stream)
+        nbytes = abi.pa_gmm_workspace_bytes(self.K, self.D, self.max_rows, self.T)
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=self.means.device)
+        self.h = abi.pa_gmm_create(self.K, self.D, self.means.data_ptr(), std, list(alphas_cumprod),
+                                   self.T, self.max_rows, self.workspace.data_ptr(), nbytes,
+                                   self.stream_ptr)
+
+    def eps(self, batch_x_ptr, miss_bt_ptr, n_rows_dev_ptr, out):
+        abi.pa_gmm_eps(self.h, batch_x_ptr, miss_bt_ptr, n_rows_dev_ptr,
+                       out.data_ptr() if isinstance(out, torch.Tensor) else out)
+
+    def launches(self):
+        return abi.pa_gmm_launches(self.h)
+
+    def close(self):
+        if getattr(self, "h", None) is not None:
+            abi.pa_gmm_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

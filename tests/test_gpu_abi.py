@@ -1,0 +1,111 @@
+"""GPU-side ABI behaviour: call order, restart, counters, device status."""
+import numpy as np
+import pytest
+
+import workload as W
+from paper_2609_36522_gb300 import abi
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_36522_gb300 import build as pa_build
+    pa_build.build()
+
+
+def _solver(w=W.TINY, **kw):
+    import torch
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+    a, x0, mu = W.inputs(w)
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, **kw)
+    g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, w.batch * s.window, **kw)
+    eps = torch.empty(w.batch * s.window, w.D, dtype=torch.float32, device="cuda")
+    x0d = torch.from_numpy(x0).cuda()
+    torch.cuda.synchronize()
+    return s, g, eps, x0d
+
+
+def _run(s, g, eps):
+    while True:
+        out = s.step()
+        if out is None:
+            return
+        n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
+        g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+        s.submit_eps(eps)
+
+
+def test_call_order_is_enforced():
+    s, g, eps, x0 = _solver()
+    with pytest.raises(abi.PaError) as e:
+        s.submit_eps(eps)
+    assert e.value.status == abi.PA_ERR_STATE
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_step(s.h)
+    assert e.value.status == abi.PA_ERR_STATE
+    s.init(x0)
+    with pytest.raises(abi.PaError) as e:
+        s.result()
+    assert e.value.status == abi.PA_ERR_STATE
+    out = s.step()
+    assert out is not None and out[0] == W.TINY.window
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_step(s.h)                       # step twice without submitting
+    assert e.value.status == abi.PA_ERR_STATE
+    s.submit_eps(eps)
+    with pytest.raises(abi.PaError) as e:
+        s.submit_eps(eps)                      # submit twice
+    assert e.value.status == abi.PA_ERR_STATE
+    _run(s, g, eps)
+    assert s.step() is None                    # PA_DONE is sticky
+    s.result()
+    st = s.stats()
+    assert st["device_status"] == 0 and st["n_active"] == 0
+
+
+def test_restart_reproduces_bits_and_counters():
+    s, g, eps, x0 = _solver(W.BATCHED.with_(T=30))
+    s.init(x0)
+    _run(s, g, eps)
+    first = s.result().cpu().numpy()
+    n1, st1, log1 = s.nfe(), s.stats(), s.iter_log()
+    s.init(x0)
+    _run(s, g, eps)
+    assert np.array_equal(first, s.result().cpu().numpy())
+    assert s.nfe() == n1
+    assert np.array_equal(log1, s.iter_log())
+    assert s.stats()["iters"] == st1["iters"]
+
+
+def test_launch_counter_and_reductions():
+    s, g, eps, x0 = _solver()
+    s.init(x0)
+    _run(s, g, eps)
+    st = s.stats()
+    # init plan + per iteration (gather, update, decide) + the final gather
+    assert st["launches"] == 1 + 3 * st["iters"] + 1
+    err, dl = s.last_reductions()
+    assert np.isfinite(err).all() and np.isfinite(dl).all()
+
+
+def test_nonblocking_stream():
+    import torch
+    st = torch.cuda.Stream()
+    w = W.TINY
+    s, g, eps, x0 = _solver(w, stream=st)
+    with torch.cuda.stream(st):
+        s.init(x0)
+        while True:
+            out = s.step()
+            if out is None:
+                break
+            n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
+            abi.pa_gmm_eps(g.h, out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps.data_ptr())
+            s.submit_eps(eps)
+        a = s.result().cpu().numpy()
+    st.synchronize()
+    s2, g2, eps2, _ = _solver(w)
+    s2.init(x0)
+    _run(s2, g2, eps2)
+    assert np.array_equal(a, s2.result().cpu().numpy())

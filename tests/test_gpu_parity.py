@@ -1,0 +1,149 @@
+"""GPU parity: the CUDA solver (through the C ABI) against the fp64 oracle on
+the same seeded inputs.
+
+Bar (from the method's decisions and the fp32 state):
+* iteration count, per-iteration window start / size / stride, per-trajectory
+  miss counts, the canonical miss list (b, i) and NFE / hits: bit-exact;
+* final latents: max_d |x_gpu - x_oracle| / max_d |x_oracle| <= 1e-5 per
+  trajectory.
+Inputs pass the decision-margin guard (no oracle distance or error within
+1e-6 relative of its threshold) before they are compared.
+"""
+import numpy as np
+import pytest
+
+import workload as W
+from oracle.guard import margins_ok, decision_margins
+from oracle.gmm import gmm_eps
+from gpu_harness import oracle_run, gpu_run, compare
+
+pytestmark = pytest.mark.gpu
+
+REL_TOL = 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import torch
+    from paper_2609_36522_gb300 import build as pa_build
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    pa_build.build()
+
+
+def _check(w, cache_thresh=None, **kw):
+    thr = w.cache_thresh if cache_thresh is None else cache_thresh
+    orc = oracle_run(w, cache_thresh=thr)
+    assert margins_ok(orc, w.tol, thr, rel=1e-6), decision_margins(orc, w.tol, thr)
+    gpu = gpu_run(w, cache_thresh=thr, **kw)
+    rel = compare(w, orc, gpu)
+    assert rel.max() <= REL_TOL, rel
+    return orc, gpu
+
+
+def test_tiny():
+    _check(W.TINY)
+
+
+def test_tiny_with_oracle_eps():
+    """Solver kernels alone: eps of the gathered batch comes from the fp64 oracle."""
+    _check(W.TINY, eps_source="oracle")
+
+
+def test_sd15_full_size():
+    orc, gpu = _check(W.SD15)
+    assert gpu["stats"]["hits"] > 0
+
+
+def test_sd15_uncached_equals_oracle_uncached():
+    w = W.SD15
+    orc = oracle_run(w, cache_thresh=0.0, use_cache=False)
+    gpu = gpu_run(w, cache_thresh=0.0)
+    rel = compare(w, orc, gpu)
+    assert rel.max() <= REL_TOL
+    assert gpu["stats"]["hits"] == 0
+
+
+@pytest.mark.parametrize("thr", W.SWEEP_THRESHOLDS)
+def test_sd15_threshold_sweep(thr):
+    _check(W.SD15, cache_thresh=thr)
+
+
+def test_batched_eight_trajectories():
+    _check(W.BATCHED)
+
+
+def test_large_latent():
+    _check(W.LARGE)
+
+
+@pytest.mark.parametrize("w", [
+    W.Workload("ragged odd D", T=12, window=5, batch=3, latent_shape=(3, 5, 7), K=3,
+               tol=1e-3, cache_thresh=0.05, seed=3),
+    W.Workload("ragged D%4==0", T=14, window=6, batch=2, latent_shape=(4, 5, 7), K=5,
+               tol=1e-3, cache_thresh=0.05, seed=4),
+    W.Workload("window 1", T=9, window=1, batch=2, latent_shape=(4, 4, 4), K=2,
+               tol=1e-3, cache_thresh=0.05, seed=5),
+    W.Workload("window T", T=20, window=20, batch=1, latent_shape=(4, 8, 8), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=6),
+    W.Workload("window > T", T=7, window=32, batch=2, latent_shape=(4, 8, 8), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=7),
+    W.Workload("T 1", T=1, window=4, batch=2, latent_shape=(4, 8, 8), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=8),
+    W.Workload("multi-chunk", T=30, window=12, batch=3, latent_shape=(4, 24, 24), K=8,
+               tol=1e-3, cache_thresh=0.05, seed=9),
+    W.Workload("tight tol", T=24, window=10, batch=2, latent_shape=(4, 16, 16), K=6,
+               tol=1e-6, cache_thresh=0.02, seed=10),
+], ids=lambda w: w.name)
+def test_edge_shapes(w):
+    _check(w)
+
+
+def test_always_hit_cache_evaluates_each_timestep_once():
+    w = W.Workload("always hit", T=24, window=8, batch=2, latent_shape=(4, 8, 8), K=4,
+                   tol=1e-3, cache_thresh=1e30, seed=11)
+    orc, gpu = _check(w)
+    assert gpu["nfe"] == w.batch * w.T
+
+
+def test_async_equals_sync_and_is_deterministic():
+    w = W.BATCHED.with_(T=40)
+    a = gpu_run(w, mode="sync")
+    b = gpu_run(w, mode="async")
+    c = gpu_run(w, mode="async")
+    assert np.array_equal(a["x_final"], b["x_final"])
+    assert np.array_equal(b["x_final"], c["x_final"])
+    assert np.array_equal(a["log"], b["log"])
+    assert a["nfe"] == b["nfe"]
+
+
+def test_host_x_init_equals_device_x_init():
+    a = gpu_run(W.TINY)
+    b = gpu_run(W.TINY, x_init_host=True)
+    assert np.array_equal(a["x_final"], b["x_final"])
+
+
+def test_gmm_kernel_against_oracle():
+    """The mixture denoiser alone, on rows spread over the whole schedule."""
+    import torch
+    from paper_2609_36522_gb300.solver import GmmDenoiser
+    for w in (W.SD15, W.LARGE):
+        a, _, mu = W.inputs(w)
+        n = 48
+        rng = np.random.default_rng(0)
+        idx = np.linspace(0, w.T - 1, n).astype(np.int32)
+        comp = rng.integers(0, w.K, n)
+        x = (np.sqrt(a[idx])[:, None] * (mu[comp] + 0.5 * rng.standard_normal((n, w.D)))
+             + np.sqrt(1 - a[idx])[:, None] * rng.standard_normal((n, w.D))).astype(np.float32)
+        miss = np.stack([np.zeros(n, np.int32), idx], axis=1).astype(np.int32)
+        dev = torch.device("cuda")
+        g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, n)
+        xd = torch.from_numpy(x).to(dev)
+        md = torch.from_numpy(miss).to(dev)
+        nd = torch.tensor([n], dtype=torch.int32, device=dev)
+        out = torch.empty_like(xd)
+        g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), out)
+        got = out.cpu().numpy().astype(np.float64)
+        want = gmm_eps(x.astype(np.float64), a[idx], mu.astype(np.float64), w.gmm_std)
+        rel = np.abs(got - want).max(axis=1) / np.abs(want).max(axis=1)
+        assert rel.max() <= 2e-6, rel.max()
+        g.close()
