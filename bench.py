@@ -59,7 +59,7 @@ def parse_args(argv=None):
     ap.add_argument("--no-flush", action="store_true", help="do not flush L2 between iterations")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--update-kernel", type=int, default=None, choices=[0, 1])
+    ap.add_argument("--update-kernel", type=int, default=None)
     ap.add_argument("--oracle-sample", type=float, default=None, help=argparse.SUPPRESS)
     return ap.parse_args(argv)
 
@@ -283,7 +283,8 @@ def run_ours(args):
     w = rank_workload(W.ALL[args.workload], rank)
     a, x0, mu = W.inputs(w)
     dev = torch.device("cuda", local)
-    stream = torch.cuda.current_stream()
+    stream = torch.cuda.Stream(device=dev)
+    torch.cuda.set_stream(stream)
     s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=stream)
     if args.update_kernel is not None:
         s.set_update_kernel(args.update_kernel)
@@ -292,19 +293,12 @@ def run_ours(args):
     eps = torch.empty(max_rows, w.D, dtype=torch.float32, device=dev)
     x_dev = torch.from_numpy(x0).to(dev)
     flush = None if args.no_flush else torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+    stream.synchronize()
 
-    def generation_async(n_iters, ev=None):
-        s.init(x_dev)
-        for it in range(n_iters):
-            if flush is not None:
-                flush.zero_()
-            if ev is not None:
-                ev[it][0].record(stream)
-            bx, mb, nm = s.step_async()
-            g.eps(bx, mb, nm, eps)
-            s.submit_eps(eps)
-            if ev is not None:
-                ev[it][1].record(stream)
+    def one_iteration():
+        bx, mb, nm = s.step_async()
+        g.eps(bx, mb, nm, eps)
+        s.submit_eps(eps)
 
     # learn the iteration count with the synchronous API (also a warm-up)
     s.init(x_dev)
@@ -313,7 +307,6 @@ def run_ours(args):
         out = s.step()
         if out is None:
             break
-        n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
         g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
         s.submit_eps(eps)
         n_iters += 1
@@ -322,37 +315,62 @@ def run_ours(args):
     nfe, hits = st0["nfe"], st0["hits"]
     upd_bytes, other_bytes = iteration_bytes(log, w)
 
+    # One Picard iteration (gather, denoiser, update, decision: 6 kernels) as a
+    # CUDA graph; the update kernel's timing events are captured with it.
+    s.init(x_dev)
+    one_iteration()                       # eager warm-up of every launch path
+    stream.synchronize()
+    abi.pa_set_kernel_timing(s.h, True)
+    abi.pa_kernel_timing(s.h, reset=True)
+    graph = torch.cuda.CUDAGraph()
+    s.init(x_dev)
+    stream.synchronize()
+    with torch.cuda.graph(graph, stream=stream):
+        one_iteration()
+    kernels_per_iter = 6
+
+    def generation(timed):
+        s.init(x_dev)
+        it_ms = upd = 0.0
+        for _ in range(n_iters):
+            if flush is not None:
+                flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            graph.replay()
+            e1.record(stream)
+            if timed:
+                e1.synchronize()
+                it_ms += e0.elapsed_time(e1)
+                upd += abi.pa_kernel_timing(s.h, reset=False)[0]
+        return it_ms, upd
+
     for _ in range(args.warmup):
-        generation_async(n_iters)
+        generation(False)
+    stream.synchronize()
     assert s.poll() == 0, "solver did not finish within the learned iteration count"
-    torch.cuda.synchronize()
 
     clocks = ClockSampler(local)
     clocks.start()
     time.sleep(0.3)
-    events = [[[torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)]
-               for _ in range(n_iters)] for _ in range(args.steps)]
-    abi.pa_set_kernel_timing(s.h, True)
-    abi.pa_kernel_timing(s.h)  # reset
-    launches0 = s.stats()["launches"] + g.launches()
     barrier()
-    torch.cuda.synchronize()
+    stream.synchronize()
     wall0 = time.perf_counter()
-    for k in range(args.steps):
-        generation_async(n_iters, events[k])
-    torch.cuda.synchronize()
+    dev_ms = upd_ms = 0.0
+    for _ in range(args.steps):
+        a_ms, u_ms = generation(True)
+        dev_ms += a_ms
+        upd_ms += u_ms
+        assert s.poll() == 0
+    stream.synchronize()
     barrier()
     wall = time.perf_counter() - wall0
-    upd_ms, upd_n = abi.pa_kernel_timing(s.h)
-    abi.pa_set_kernel_timing(s.h, False)
-    launches = s.stats()["launches"] + g.launches() - launches0
-    assert s.poll() == 0
     st1 = s.stats()
     assert st1["iters"] == n_iters and st1["nfe"] == nfe, (st1, n_iters, nfe)
-    dev_ms = sum(events[k][it][0].elapsed_time(events[k][it][1])
-                 for k in range(args.steps) for it in range(n_iters))
+    abi.pa_set_kernel_timing(s.h, False)
     time.sleep(0.2)
     clk = clocks.stop()
+    launches = args.steps * (n_iters * kernels_per_iter + 1)   # + init plan per generation
 
     units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
     value = units / secs
@@ -360,27 +378,28 @@ def run_ours(args):
 
     # roofline of the dominant kernel (Picard update)
     peak, peak_kind = measured_hbm_gbs()
+    n_upd = args.steps * n_iters
     achieved = upd_bytes.sum() * args.steps / (upd_ms / 1000.0) / 1e9
     sha = kernel_source_sha()
     traffic = NCU_TRAFFIC.get(sha)
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "Picard update (" + ("bulk-copy pipeline" if st1["update_kernel"] == 1
-                                               else "plain loads") + ")",
-                "peak_kind": f"{peak_kind} HBM copy bandwidth",
+                "kernel": "Picard update (" + ("tile-parallel bulk-copy pipeline"
+                                               if st1["update_kernel"] == 1 else "plain loads") + ")",
+                "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
                 "alg_bytes_per_launch": float(upd_bytes.mean()),
-                "avg_launch_us": 1000.0 * upd_ms / max(upd_n, 1)}
+                "avg_launch_us": 1000.0 * upd_ms / max(n_upd, 1)}
 
-    # end to end through the public API with host buffers
+    # end to end through the public API with host buffers (no graph, no flush)
     e2e = None
     if not args.no_e2e:
         x_host = torch.from_numpy(x0).pin_memory()
         out_host = torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory()
         ctl_reads = 0
-        torch.cuda.synchronize()
+        stream.synchronize()
+        reps = max(3, min(args.steps, 50))
         e0 = torch.cuda.Event(enable_timing=True)
         e1 = torch.cuda.Event(enable_timing=True)
-        reps = max(3, min(args.steps, 50))
         e0.record(stream)
         t0 = time.perf_counter()
         for _ in range(reps):
@@ -390,12 +409,11 @@ def run_ours(args):
                 ctl_reads += 1
                 if out is None:
                     break
-                n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
                 g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
                 s.submit_eps(eps)
             s.result(out_host)
         e1.record(stream)
-        torch.cuda.synchronize()
+        stream.synchronize()
         e2e_s = max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0)
         units_e, secs_e = aggregate(reps * n_iters, e2e_s)
         e2e = {"value": units_e / secs_e, "unit": UNIT,
@@ -420,7 +438,8 @@ def run_ours(args):
                        "parallelism": f"replicas x{world} (independent trajectories)",
                        "l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every Picard iteration, outside the timed events"),
-                       "timing": "CUDA events around each Picard iteration on the launch stream"},
+                       "timing": "CUDA events around each Picard iteration (one CUDA-graph replay of "
+                                 "gather, denoiser, update, decision) on the launch stream"},
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
             "solver_step_gbps": gb_step,

@@ -160,16 +160,37 @@ PA_API pa_status pa_iter_log(pa_solver* s, int32_t* out, int max_iters, int* n_i
 PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out);
 
 /* Select the Picard-update kernel: 0 = plain loads, 1 = bulk-copy pipeline
- * (default when D % 4 == 0). Returns PA_ERR_ARG for an unknown value. */
+ * (default when D % 4 == 0; it falls back to plain loads for a batch_eps
+ * pointer that is not 16-byte aligned), 100 + n = bulk-copy pipeline with
+ * launch shape n (0..9; columns per lane, warps per CTA, pipeline depth --
+ * a tuning aid). Returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
 
+/* Benchmark hook: launch only the Picard-update kernel of the planned
+ * iteration, `repeats` times back to back on the solver's stream (between
+ * pa_step and pa_submit_eps). Each launch moves the same bytes as the real
+ * one but overwrites the window's states with values that are no longer the
+ * method's; call pa_init before using the solver's results again. */
+PA_API pa_status pa_bench_update_only(pa_solver* s, const float* batch_eps_dev, int repeats);
+
+/* Fault-handling test hook: the number of polls after which an mbarrier wait
+ * of the bulk-copy update kernel counts as timed out (default 2^24). With 0
+ * every such wait gives up at once: the kernel records PA_ERR_TIMEOUT (read by
+ * the next synchronising call), still drains its in-flight copies with the
+ * default bound, and leaves the solver's numbers meaningless until pa_init. */
+PA_API pa_status pa_debug_set_wait_limit(pa_solver* s, uint32_t polls);
+
 /* Enable (1) or disable (0) CUDA-event timing of every Picard-update kernel
- * launch, recorded on the solver's stream directly around the launch. */
+ * launch, recorded on the solver's stream directly around the launch. Inside
+ * a stream capture the records become event nodes of the graph, recorded
+ * again at every replay. */
 PA_API pa_status pa_set_kernel_timing(pa_solver* s, int enable);
 
 /* Sum of the update-kernel durations in ms, and how many launches were timed,
- * since the previous call (which resets both). Synchronises. */
-PA_API pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches);
+ * since the last reset. reset != 0 starts a new count. For a captured graph,
+ * read with reset = 0 after each replay: the captured records hold that
+ * replay's times. Synchronises. */
+PA_API pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches, int reset);
 
 PA_API void pa_destroy(pa_solver* s);
 

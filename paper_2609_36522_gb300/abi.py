@@ -59,8 +59,10 @@ _PROTOS = {
     "pa_iter_log": (C.c_int, [VP, C.POINTER(C.c_int32), C.c_int, C.POINTER(C.c_int)]),
     "pa_last_reductions": (C.c_int, [VP, VP, VP]),
     "pa_set_update_kernel": (C.c_int, [VP, C.c_int]),
+    "pa_bench_update_only": (C.c_int, [VP, VP, C.c_int]),
+    "pa_debug_set_wait_limit": (C.c_int, [VP, C.c_uint32]),
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
-    "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64)]),
+    "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.c_int]),
     "pa_destroy": (None, [VP]),
     "pa_gmm_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int64, C.c_int, C.c_int]),
     "pa_gmm_create": (C.c_int, [PVP, C.c_int, C.c_int64, VP, C.c_double,
@@ -205,15 +207,23 @@ def pa_set_update_kernel(h, kind):
     return _check("pa_set_update_kernel", lib().pa_set_update_kernel(h, int(kind)))
 
 
+def pa_bench_update_only(h, batch_eps_ptr, repeats):
+    return _check("pa_bench_update_only", lib().pa_bench_update_only(h, _dptr(batch_eps_ptr), int(repeats)))
+
+
+def pa_debug_set_wait_limit(h, polls):
+    return _check("pa_debug_set_wait_limit", lib().pa_debug_set_wait_limit(h, int(polls)))
+
+
 def pa_set_kernel_timing(h, enable):
     return _check("pa_set_kernel_timing", lib().pa_set_kernel_timing(h, int(bool(enable))))
 
 
-def pa_kernel_timing(h):
-    """-> (total update-kernel ms, launches timed) since the previous call."""
+def pa_kernel_timing(h, reset=True):
+    """-> (total update-kernel ms, launches timed) since the last reset."""
     ms = C.c_double()
     n = C.c_int64()
-    _check("pa_kernel_timing", lib().pa_kernel_timing(h, C.byref(ms), C.byref(n)))
+    _check("pa_kernel_timing", lib().pa_kernel_timing(h, C.byref(ms), C.byref(n), int(bool(reset))))
     return ms.value, n.value
 
 

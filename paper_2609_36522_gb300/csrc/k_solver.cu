@@ -221,45 +221,69 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 //     else misses; misses are compacted trajectory-major into miss_bt with a
 //     block-wide prefix sum, and rank[b][j] records each miss's batch row.
 constexpr int kDecideThreads = 1024;
+constexpr int kDecideSmemPairs = 6144;  // (b, j) pairs whose reductions stay in shared memory
 
 __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
   __shared__ int s_t[kMaxBatch], s_p[kMaxBatch], s_e[kMaxBatch];
   __shared__ int s_tn[kMaxBatch], s_pn[kMaxBatch], s_m[kMaxBatch], s_h1[kMaxBatch];
   __shared__ int s_warp[kDecideThreads / 32];
-  __shared__ int s_total;
+  __shared__ int s_total, s_active, s_iter;
+  extern __shared__ float s_red[];  // [2][B*P] when B*P <= kDecideSmemPairs
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kDecideThreads / 32;
   const int B = d.B, P = d.P, T = d.T;
-  if (d.ctl->n_active == 0) return;  // finished: iterating further is a no-op
-  const int iter = d.ctl->iter;
+  const bool in_smem = B * P <= kDecideSmemPairs;
+  float* red_e = in_smem ? s_red : d.red_err;
+  float* red_d = in_smem ? s_red + B * P : d.red_del;
 
+  // Every load of this prologue is independent of the others (one round trip):
+  // counters, window bookkeeping, and the chunk partials of every (b, j).
+  if (tid == 0) {
+    s_active = d.ctl->n_active;
+    s_iter = d.ctl->iter;
+  }
   for (int b = tid; b < B; b += kDecideThreads) {
     const Traj tr = d.traj[b];
     s_t[b] = tr.t; s_p[b] = tr.p; s_e[b] = tr.e;
     s_m[b] = 0;
     s_h1[b] = 0;
   }
-  __syncthreads();
-
-  // 1. reductions, one warp per (b, j)
+  // 1. reductions, one warp per (b, j), eight independent partial sums per
+  // lane combined in a fixed order (deterministic). Positions beyond a
+  // trajectory's window are reduced too (their values are never used).
   for (int q = warp; q < B * P; q += nwarps) {
-    const int b = q / P, j = q % P;
-    if (j >= s_p[b]) continue;
     const float* pe = d.part_err + (int64_t)q * nchunk;
     const float* pd = d.part_del + (int64_t)q * nchunk;
-    float se = 0.f, sd = 0.f;
-    for (int c = lane; c < nchunk; c += 32) {
-      se += pe[c];
-      sd += pd[c];
+    float se[8], sd[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) { se[u] = 0.f; sd[u] = 0.f; }
+    for (int c0 = 0; c0 < nchunk; c0 += 256) {
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int c = c0 + u * 32 + lane;
+        if (c < nchunk) {
+          se[u] += pe[c];
+          sd[u] += pd[c];
+        }
+      }
     }
-    se = warp_sum(se);
-    sd = warp_sum(sd);
+    float te = ((se[0] + se[1]) + (se[2] + se[3])) + ((se[4] + se[5]) + (se[6] + se[7]));
+    float td = ((sd[0] + sd[1]) + (sd[2] + sd[3])) + ((sd[4] + sd[5]) + (sd[6] + sd[7]));
+    te = warp_sum(te);
+    td = warp_sum(td);
     if (lane == 0) {
-      d.red_err[q] = se / (float)d.D;
-      d.red_del[q] = sd / (float)d.D;
+      const float ve = te / (float)d.D, vd = td / (float)d.D;
+      red_e[q] = ve;
+      red_d[q] = vd;
+      if (in_smem) {  // keep the global copy for pa_last_reductions
+        d.red_err[q] = ve;
+        d.red_del[q] = vd;
+      }
     }
   }
   __syncthreads();
+  if (s_active == 0) return;  // finished: iterating further is a no-op
+  const int iter = s_iter;
 
   // 2. window advance, one warp per trajectory
   for (int b = warp; b < B; b += nwarps) {
@@ -276,7 +300,7 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
     int lead = p;
     for (int j0 = 0; j0 < p; j0 += 32) {
       const int j = j0 + lane;
-      const bool fail = (j < p) && !((double)d.red_err[b * P + j] <= d.tol);
+      const bool fail = (j < p) && !((double)red_e[b * P + j] <= d.tol);
       const unsigned m = __ballot_sync(0xffffffffu, fail);
       if (m) {
         lead = j0 + __ffs(m) - 1;
@@ -307,7 +331,7 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
     const int en = s_t[b] + s_p[b];  // new frontier
     if (i >= en) return 1;           // first entry
     const int jo = i - s_t[b] - 1;   // delta of timestep i was computed at old position jo
-    return ((double)d.red_del[b * P + jo] < d.cache_thresh) ? 0 : 1;
+    return ((double)red_d[b * P + jo] < d.cache_thresh) ? 0 : 1;
   };
   int cnt = 0;
   for (int q = q0; q < q1; ++q) cnt += is_miss(q);
@@ -410,7 +434,9 @@ cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream
 }
 
 cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st) {
-  k_decide<<<1, kDecideThreads, 0, st>>>(d, nchunk);
+  const int pairs = d.B * d.P;
+  const size_t smem = pairs <= kDecideSmemPairs ? (size_t)2 * pairs * sizeof(float) : 0;
+  k_decide<<<1, kDecideThreads, smem, st>>>(d, nchunk);
   return cudaGetLastError();
 }
 

@@ -1,12 +1,476 @@
-// Bulk-copy pipelined Picard update (placeholder until the pipeline lands).
+// Tile-parallel Picard update with bulk-copy staging, for sm_103a.
+//
+// Same mathematics as the plain-load kernel (k_solver.cu): per window position
+// j (timestep i = t + j) Eq. 6 assembly, Eq. 7 cache update for misses, the
+// drift d_j = (c_i - 1) x_i + e_i eps_i at the current latent, the window
+// prefix sum of Eq. 1, the Eq. 2 error of state i+1 and the Eq. 4 distance of
+// timestep i+1 for the next iteration.
+//
+// Parallel structure. A CTA owns a strip of SEG = 32*V adjacent columns of one
+// trajectory and walks the window in tiles of TW = NW*S positions. The drifts
+// of different positions are independent; only their prefix sum couples them.
+// So within a tile warp w takes positions w*S .. w*S+S-1, forms its S drifts
+// and their local prefix, publishes its segment total, and after one CTA
+// barrier adds the carry (the running sum from x_t plus the totals of the
+// warps before it). All sums are carried as fp32 (hi, lo) pairs (TwoSum), so
+// the blocked order loses nothing against a sequential compensated sum.
+//
+// Staging. Rows of a tile (per position: the eps row segment, from batch_eps
+// for a miss or ehat_i for a hit; the old state x_{i+1} unless it is a lazy
+// tail copy; xhat_{i+1} when timestep i+1 is a hit) are fetched with
+// cp.async.bulk (TMA engine, global -> shared) into one of nbuf tile buffers;
+// completion is counted on the buffer's mbarrier. Warp 0 issues a whole tile
+// at once, one lane per position. When the whole window fits in shared memory
+// (nbuf >= number of tiles) every copy is in flight right after the prologue;
+// otherwise the buffers are refilled as tiles retire.
+//
+// Every mbarrier wait is bounded. A wait that runs out records kDevTimeout in
+// the solver's status word and stops further issues; the CTA finishes its
+// (now meaningless) arithmetic with in-bounds accesses only, drains the
+// copies already issued with bounded waits, and returns.
 #include "pa_internal.h"
 
 namespace pa {
+namespace {
 
-bool update_bulk_supported(const Dev&, const float*) { return false; }
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
 
-cudaError_t launch_update_bulk(const Dev&, const float*, cudaStream_t, int*) {
-  return cudaErrorNotSupported;
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_u32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_u32(dst)),
+      "l"(src), "r"(bytes), "r"(smem_u32(bar))
+      : "memory");
+}
+
+__device__ __forceinline__ void fence_barrier_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+// Bounded wait on one mbarrier phase; false when `limit` polls ran out.
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint32_t limit) {
+  for (uint32_t n = 0; n < limit; ++n) {
+    if (mbar_try_wait(bar, parity)) return true;
+  }
+  return false;
+}
+
+constexpr uint32_t kDrainLimit = 1u << 24;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// s = fl(a + b) and s + err == a + b exactly (Knuth's TwoSum).
+__device__ __forceinline__ void two_sum(float a, float b, float& s, float& err) {
+  s = a + b;
+  const float bb = s - a;
+  err = (a - (s - bb)) + (b - bb);
+}
+
+// (hi, lo) += v
+__device__ __forceinline__ void acc_add(float& hi, float& lo, float v) {
+  float s, e;
+  two_sum(hi, v, s, e);
+  hi = s;
+  lo += e;
+}
+
+// (hi, lo) += (h2, l2)
+__device__ __forceinline__ void acc_add2(float& hi, float& lo, float h2, float l2) {
+  float s, e;
+  two_sum(hi, h2, s, e);
+  hi = s;
+  lo += e + l2;
+}
+
+template <int V>
+struct Vec {
+  float a[V];
+};
+
+template <int V>
+__device__ __forceinline__ Vec<V> ldv(const float* p) {
+  Vec<V> r;
+  if constexpr (V == 2) {
+    const float2 q = *reinterpret_cast<const float2*>(p);
+    r.a[0] = q.x; r.a[1] = q.y;
+  } else {
+    r.a[0] = *p;
+  }
+  return r;
+}
+
+template <int V>
+__device__ __forceinline__ void stv(float* p, const Vec<V>& v) {
+  if constexpr (V == 2) {
+    *reinterpret_cast<float2*>(p) = make_float2(v.a[0], v.a[1]);
+  } else {
+    *p = v.a[0];
+  }
+}
+
+template <int V, int NW, int S>
+struct TileShape {
+  static constexpr int SEG = 32 * V;                  // columns per strip
+  static constexpr int TW = NW * S;                   // positions per tile
+  static_assert(2 * TW <= NW * 32, "two reductions per position need 2*TW threads");
+  static constexpr size_t kTileFloats = (size_t)TW * 3 * SEG;
+  static constexpr size_t kTileBytes = kTileFloats * sizeof(float);
+  static constexpr int kMaxBuf = 16;                  // mbarriers in the barrier area
+  static constexpr size_t kBarBytes = 128;
+  // per position: rank, c-1, e, cache slot, state-ring slot of the next state
+  __host__ __device__ static size_t meta_bytes(int P) { return ((size_t)P * 20 + 127) / 128 * 128; }
+  static constexpr size_t kTotBytes = (size_t)NW * SEG * 2 * sizeof(float);   // segment totals
+  static constexpr size_t kCarBytes = kTotBytes;                              // carries into warps
+  static constexpr size_t kRedBytes = ((size_t)2 * TW * 33 * sizeof(float) + 127) / 128 * 128;
+  __host__ __device__ static size_t smem_bytes(int P, int nbuf) {
+    return kBarBytes + meta_bytes(P) + kTotBytes + kCarBytes + kRedBytes + (size_t)nbuf * kTileBytes;
+  }
+};
+
+// nbuf tile buffers (<= 16); when nbuf >= ceil(p / TW) every copy of the
+// window is in flight right after the prologue.
+template <int V, int NW, int S>
+__global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __restrict__ beps,
+                                                         int nstrip, int nbuf, uint32_t wait_limit) {
+  using Sh = TileShape<V, NW, S>;
+  constexpr int SEG = Sh::SEG, TW = Sh::TW;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int P = d.P;
+  const int b = blockIdx.y;
+  const int64_t D = d.D;
+
+  // smem: barriers | per-position metadata | totals | carries | reductions | tiles
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem_raw);
+  unsigned char* q = smem_raw + Sh::kBarBytes;
+  int32_t* s_rank = reinterpret_cast<int32_t*>(q);
+  float* s_cm1 = reinterpret_cast<float*>(q + (size_t)P * 4);
+  float* s_ec = reinterpret_cast<float*>(q + (size_t)P * 8);
+  int32_t* s_slot = reinterpret_cast<int32_t*>(q + (size_t)P * 12);  // (t+j) mod P
+  int32_t* s_nxt = reinterpret_cast<int32_t*>(q + (size_t)P * 16);   // (t+j+1) mod (P+1)
+  q += Sh::meta_bytes(P);
+  float* s_tot = reinterpret_cast<float*>(q);   // [NW][SEG][2]
+  q += Sh::kTotBytes;
+  float* s_car = reinterpret_cast<float*>(q);   // [NW][SEG][2]
+  q += Sh::kCarBytes;
+  float* s_red = reinterpret_cast<float*>(q);   // [2][TW][33]
+  q += Sh::kRedBytes;
+  float* s_tile = reinterpret_cast<float*>(q);  // 128-byte aligned: all offsets above are
+
+  // round 1: independent loads of the bookkeeping and every rank of the window
+  const Traj tr = d.traj[b];
+  const int n_miss = d.ctl->n_miss;
+  for (int j = tid; j < P; j += NW * 32) s_rank[j] = d.rank[b * P + j];
+  if (tr.p == 0) return;
+  const int t = tr.t, p = tr.p, e = tr.e;
+  for (int j = tid; j < p; j += NW * 32) {
+    s_slot[j] = (t + j) % P;
+    s_nxt[j] = (t + j + 1) % (P + 1);
+    s_cm1[j] = d.cm1[t + j];
+    s_ec[j] = d.ecoef[t + j];
+  }
+  if (tid == 0) {
+    for (int k = 0; k < nbuf; ++k) mbar_init(&bar[k], 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  for (int j = tid; j < p; j += NW * 32) {
+    if (s_rank[j] >= n_miss) {  // never expected: keep every copy in bounds and report it
+      atomicCAS(&d.ctl->status, kDevOk, kDevBadRank);
+      s_rank[j] = -1;
+    }
+  }
+  __syncthreads();
+
+  const int strip = blockIdx.x;
+  const int64_t c0 = (int64_t)strip * SEG;
+  const int64_t ncol = (D - c0) < SEG ? (D - c0) : SEG;
+  const uint32_t seg_bytes = (uint32_t)ncol * sizeof(float);
+  const int64_t mycol = c0 + (int64_t)lane * V;
+  const bool live = mycol < D;
+  float* Xb = d.X + (int64_t)b * (P + 1) * D;
+  float* Xh = d.Xhat + (int64_t)b * P * D;
+  float* Eh = d.Ehat + (int64_t)b * P * D;
+  const int ntile = (p + TW - 1) / TW;
+
+  // Warp 0 issues tile k into buffer k % nbuf; lane l fetches positions
+  // k*TW + l, k*TW + l + 32, ... The whole tile's byte count is announced on
+  // the buffer's mbarrier before any of its copies is issued.
+  auto issue_tile = [&](int k) {
+    float* buf = s_tile + (size_t)(k % nbuf) * Sh::kTileFloats;
+    uint64_t* bk = &bar[k % nbuf];
+    uint32_t total = 0;
+    for (int qb = 0; qb < TW; qb += 32) {
+      const int qi = qb + lane;
+      const int j = k * TW + qi;
+      if (qi < TW && j < p) {
+        const uint32_t n = 1u + (((t + j + 1) <= e) ? 1u : 0u) +
+                           (((j + 1 < p) && (s_rank[j + 1] < 0)) ? 1u : 0u);
+        total += n * seg_bytes;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) total += __shfl_xor_sync(0xffffffffu, total, o);
+    if (lane == 0) mbar_arrive_expect_tx(bk, total);
+    __syncwarp();
+    for (int qb = 0; qb < TW; qb += 32) {
+      const int qi = qb + lane;
+      const int j = k * TW + qi;
+      if (qi < TW && j < p) {
+        float* rowp = buf + (size_t)qi * 3 * SEG;
+        const int r = s_rank[j];
+        const float* src_eps = (r >= 0) ? beps + (int64_t)r * D + c0 : Eh + (int64_t)s_slot[j] * D + c0;
+        bulk_g2s(rowp, src_eps, seg_bytes, bk);
+        if (t + j + 1 <= e) bulk_g2s(rowp + SEG, Xb + (int64_t)s_nxt[j] * D + c0, seg_bytes, bk);
+        if ((j + 1 < p) && (s_rank[j + 1] < 0))
+          bulk_g2s(rowp + 2 * SEG, Xh + (int64_t)s_slot[j + 1] * D + c0, seg_bytes, bk);
+      }
+    }
+  };
+
+  // round 2: every tile that has a buffer goes out now; meanwhile every warp
+  // loads the lazy fill value (old state e) and warp 0 the window start x_t
+  const int pre = ntile < nbuf ? ntile : nbuf;
+  if (warp == 0)
+    for (int k = 0; k < pre; ++k) issue_tile(k);
+  int issued = pre;  // tiles issued so far (same value in every thread)
+  Vec<V> xfill{}, xlast{};
+  if (live) {
+    xfill = ldv<V>(Xb + (int64_t)(e % (P + 1)) * D + mycol);
+    if (warp == 0) xlast = ldv<V>(Xb + (int64_t)(t % (P + 1)) * D + mycol);
+  }
+  // warp 0 keeps the running carry: x_t + every drift before the current tile
+  float chi[V], clo[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) { chi[v] = xlast.a[v]; clo[v] = 0.f; }
+
+  const int64_t pbase = (int64_t)b * P * nstrip + strip;
+  const int red_first = NW * 32 - 2 * TW;  // the last 2*TW threads finish the reductions
+  int my_fail = 0;   // this thread's wait ran out
+  int aborted = 0;   // some thread's wait ran out (CTA-uniform, from a barrier)
+  for (int k = 0; k < ntile; ++k) {
+    const int bi = k % nbuf;
+    const uint32_t parity = (uint32_t)((k / nbuf) & 1);
+    if (!my_fail && !aborted && !mbar_wait_bounded(&bar[bi], parity, wait_limit)) {
+      atomicCAS(&d.ctl->status, kDevOk, kDevTimeout);
+      my_fail = 1;
+    }
+    const float* buf = s_tile + (size_t)bi * Sh::kTileFloats;
+    const int tb = k * TW;
+    const int q0 = warp * S;
+
+    // phase 1: drifts of this warp's S positions and their local prefix
+    float phi[S][V], plo[S][V];
+    Vec<V> xo_s[S];
+    Vec<V> xc;
+    if (q0 == 0) {
+      xc = xlast;  // warp 0: old state at the tile's first position
+    } else if (tb + q0 < p && t + tb + q0 <= e) {
+      xc = ldv<V>(buf + (size_t)(q0 - 1) * 3 * SEG + SEG + lane * V);
+    } else {
+      xc = xfill;
+    }
+    float rh[V], rl[V];
+#pragma unroll
+    for (int v = 0; v < V; ++v) { rh[v] = 0.f; rl[v] = 0.f; }
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      const int qi = q0 + s;
+      const int j = tb + qi;
+      const float* rowp = buf + (size_t)qi * 3 * SEG;
+      Vec<V> xo = xfill;
+      if (j < p && live) {
+        const Vec<V> eps = ldv<V>(rowp + lane * V);
+        if (s_rank[j] >= 0) {  // Eq. 7: the cache takes (x_i, eps_i) of a miss
+          const int64_t o = (int64_t)s_slot[j] * D + mycol;
+          stv<V>(Eh + o, eps);
+          stv<V>(Xh + o, xc);
+        }
+        const float cm1 = s_cm1[j], ec = s_ec[j];
+#pragma unroll
+        for (int v = 0; v < V; ++v) acc_add(rh[v], rl[v], fmaf(cm1, xc.a[v], ec * eps.a[v]));
+        if (t + j + 1 <= e) xo = ldv<V>(rowp + SEG + lane * V);
+      }
+#pragma unroll
+      for (int v = 0; v < V; ++v) { phi[s][v] = rh[v]; plo[s][v] = rl[v]; }
+      xo_s[s] = xo;
+      xc = xo;
+    }
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const size_t o = ((size_t)warp * SEG + lane * V + v) * 2;
+      s_tot[o] = rh[v];
+      s_tot[o + 1] = rl[v];
+    }
+    __syncthreads();  // A: totals published
+
+    // warp 0: exclusive scan of the warp totals per column, on top of the
+    // running carry, and the running carry of the next tile
+    if (warp == 0) {
+#pragma unroll
+      for (int w = 0; w < NW; ++w) {
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          const size_t o = ((size_t)w * SEG + lane * V + v) * 2;
+          s_car[o] = chi[v];
+          s_car[o + 1] = clo[v];
+          acc_add2(chi[v], clo[v], s_tot[o], s_tot[o + 1]);
+        }
+      }
+    }
+    __syncthreads();  // B: carries published
+
+    // phase 2: new states, their Eq. 2 error and next-iteration Eq. 4 distance
+#pragma unroll
+    for (int s = 0; s < S; ++s) {
+      const int qi = q0 + s;
+      const int j = tb + qi;
+      const float* rowp = buf + (size_t)qi * 3 * SEG;
+      float ev = 0.f, dv = 0.f;
+      if (j < p && live) {
+        Vec<V> xn;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          const size_t o = ((size_t)warp * SEG + lane * V + v) * 2;
+          float h = s_car[o], l = s_car[o + 1];
+          acc_add2(h, l, phi[s][v], plo[s][v]);
+          xn.a[v] = h + l;
+          const float df = xn.a[v] - xo_s[s].a[v];
+          ev = fmaf(df, df, ev);
+        }
+        stv<V>(Xb + (int64_t)s_nxt[j] * D + mycol, xn);
+        if (j + 1 < p) {
+          const Vec<V> xh = (s_rank[j + 1] < 0) ? ldv<V>(rowp + 2 * SEG + lane * V) : xo_s[s];
+#pragma unroll
+          for (int v = 0; v < V; ++v) dv += fabsf(xn.a[v] - xh.a[v]);
+        }
+      }
+      s_red[(size_t)qi * 33 + lane] = ev;
+      s_red[(size_t)(TW + qi) * 33 + lane] = dv;
+    }
+    // the next tile's first state, read by warp 0 before it refills the buffer
+    if (warp == 0) {
+      const int jl = tb + TW - 1;
+      if (jl < p && live && t + jl + 1 <= e) {
+        xlast = ldv<V>(buf + (size_t)(TW - 1) * 3 * SEG + SEG + lane * V);
+      } else {
+        xlast = xfill;
+      }
+    }
+    // C: every warp is done with this buffer, the totals and the carries;
+    // stop issuing after a timeout
+    aborted = __syncthreads_or(my_fail);
+    if (!aborted && k + nbuf < ntile) {
+      if (warp == 0) issue_tile(k + nbuf);
+      issued = k + nbuf + 1;
+    }
+    // per-position partials of this strip: one thread sums one row of lanes
+    if (tid >= red_first) {
+      const int r = tid - red_first;  // 0 .. 2*TW-1
+      const int qi = r % TW;
+      const int j = tb + qi;
+      if (j < p) {
+        const float* row = s_red + (size_t)r * 33;
+        float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int c = 0; c < 32; c += 4) {
+          acc[0] += row[c];
+          acc[1] += row[c + 1];
+          acc[2] += row[c + 2];
+          acc[3] += row[c + 3];
+        }
+        const float sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+        float* dst = (r < TW) ? d.part_err : d.part_del;
+        dst[pbase + (int64_t)j * nstrip] = sum;
+      }
+    }
+  }
+  // after a timeout: wait (bounded) for the last issue of every buffer
+  if (tid == 0 && aborted) {
+    for (int k = (issued > nbuf ? issued - nbuf : 0); k < issued; ++k)
+      mbar_wait_bounded(&bar[k % nbuf], (uint32_t)((k / nbuf) & 1), kDrainLimit);
+  }
+}
+
+// Shared memory budget per CTA for the tile buffers: enough for the whole
+// window when it fits, so every copy is in flight from the start.
+constexpr size_t kSmemBudget = 112 * 1024;
+
+template <int V, int NW, int S>
+cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+  using Sh = TileShape<V, NW, S>;
+  const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
+  const int ntile_max = (d.P + Sh::TW - 1) / Sh::TW;
+  const size_t fixed = Sh::smem_bytes(d.P, 0);
+  int nbuf = ntile_max < Sh::kMaxBuf ? ntile_max : Sh::kMaxBuf;
+  while (nbuf > 2 && fixed + (size_t)nbuf * Sh::kTileBytes > kSmemBudget) --nbuf;
+  if (nbuf < 1) nbuf = 1;
+  const size_t smem = Sh::smem_bytes(d.P, nbuf);
+  auto kern = k_update_tile<V, NW, S>;
+  // largest dynamic shared memory granted so far, per device and instantiation
+  static size_t configured[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || smem > configured[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) configured[dev] = smem;
+  }
+  *nchunk_out = nstrip;
+  kern<<<dim3(nstrip, d.B), NW * 32, smem, st>>>(d, beps, nstrip, nbuf, d.wait_limit);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+bool update_bulk_supported(const Dev& d, const float* batch_eps) {
+  // 16-byte granularity of bulk copies: every row segment must start on a
+  // 16-byte boundary and be a multiple of 16 bytes long.
+  return d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0;
+}
+
+cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
+  switch (d.bulk_cfg) {
+    case 0: return launch_tile<2, 8, 4>(d, batch_eps, st, nchunk_out);
+    case 1: return launch_tile<1, 8, 4>(d, batch_eps, st, nchunk_out);
+    case 2: return launch_tile<1, 4, 8>(d, batch_eps, st, nchunk_out);
+    case 3: return launch_tile<2, 4, 8>(d, batch_eps, st, nchunk_out);
+    case 4: return launch_tile<2, 8, 2>(d, batch_eps, st, nchunk_out);
+    case 5: return launch_tile<2, 4, 4>(d, batch_eps, st, nchunk_out);
+    case 6: return launch_tile<1, 8, 8>(d, batch_eps, st, nchunk_out);
+    case 7: return launch_tile<2, 8, 8>(d, batch_eps, st, nchunk_out);
+    case 8: return launch_tile<1, 16, 2>(d, batch_eps, st, nchunk_out);
+    case 9: return launch_tile<2, 16, 2>(d, batch_eps, st, nchunk_out);
+    default: return launch_tile<2, 8, 4>(d, batch_eps, st, nchunk_out);
+  }
 }
 
 }  // namespace pa

@@ -12,6 +12,7 @@ constexpr int kMaxWindow = 1024;
 constexpr int kMaxBatch = 64;
 constexpr int kMinChunk = 32;       // narrowest column chunk of any update kernel
 constexpr size_t kAlign = 256;
+constexpr int kBulkConfigs = 10;    // launch shapes of the bulk-copy update kernel
 
 // Device status codes written by kernels (first error wins, atomicCAS from 0).
 constexpr int kDevOk = 0;
@@ -94,7 +95,10 @@ struct Dev {
   int T, P, B;
   int64_t D;
   double tol, cache_thresh;   // compared against fp32 reductions promoted to double
+  int bulk_cfg;               // launch shape of the bulk-copy update kernel
+  uint32_t wait_limit;        // polls before an mbarrier wait counts as timed out
 };
+constexpr uint32_t kWaitLimit = 1u << 24;
 
 // Kernel launchers (k_solver.cu). Each returns the launch error.
 cudaError_t launch_init_plan(const Dev& d, cudaStream_t st);

@@ -81,6 +81,16 @@ pa_status sync_ctl(pa_solver* s, const char* where) {
   return PA_OK;
 }
 
+// Inside a stream capture the event becomes an event-record node of the graph
+// (recorded again at every replay); outside it is an ordinary record.
+cudaError_t record_timing_event(cudaEvent_t ev, cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(st, &cs);
+  if (e != cudaSuccess) return e;
+  if (cs == cudaStreamCaptureStatusActive) return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
+  return cudaEventRecord(ev, st);
+}
+
 }  // namespace
 
 extern "C" {
@@ -166,6 +176,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.T = T; d.P = P; d.B = batch; d.D = D;
   d.tol = tol;
   d.cache_thresh = cache_thresh;
+  d.wait_limit = pa::kWaitLimit;
   s->update_kind = (D % 4 == 0) ? 1 : 0;
 
   // DDIM (eta = 0) step i -> i+1 written as x + s(x, eps) with
@@ -265,7 +276,7 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
         if (e == cudaSuccess) s->ev.push_back(x);
       }
     }
-    if (e == cudaSuccess) e = cudaEventRecord(s->ev[2 * s->ev_next], s->st);
+    if (e == cudaSuccess) e = record_timing_event(s->ev[2 * s->ev_next], s->st);
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
   }
   if (s->update_kind == 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
@@ -278,7 +289,7 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
   s->launches++;
   if (e != cudaSuccess) return cuda_fail("pa_submit_eps: update", e);
   if (s->timing) {
-    e = cudaEventRecord(s->ev[2 * s->ev_next + 1], s->st);
+    e = record_timing_event(s->ev[2 * s->ev_next + 1], s->st);
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
     s->ev_next++;
   }
@@ -368,8 +379,38 @@ pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out) {
 
 pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   if (!s) return arg_fail("pa_set_update_kernel: solver is NULL");
-  if (kind != 0 && kind != 1) return arg_fail("pa_set_update_kernel: kind must be 0 or 1");
-  s->update_kind = kind;
+  if (kind == 0 || kind == 1) {
+    s->update_kind = kind;
+    s->d.bulk_cfg = 0;
+  } else if (kind >= 100 && kind < 100 + pa::kBulkConfigs) {
+    s->update_kind = 1;
+    s->d.bulk_cfg = kind - 100;
+  } else {
+    return arg_fail("pa_set_update_kernel: kind must be 0, 1 or 100 + launch shape");
+  }
+  return PA_OK;
+}
+
+pa_status pa_bench_update_only(pa_solver* s, const float* batch_eps_dev, int repeats) {
+  if (!s || !batch_eps_dev || repeats < 1) return arg_fail("pa_bench_update_only: bad argument");
+  if (s->state != St::Stepped) return state_fail("pa_bench_update_only");
+  for (int r = 0; r < repeats; ++r) {
+    int nchunk = 0;
+    cudaError_t e;
+    if (s->update_kind == 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
+      e = pa::launch_update_bulk(s->d, batch_eps_dev, s->st, &nchunk);
+    } else {
+      e = pa::launch_update_plain(s->d, batch_eps_dev, s->st, &nchunk);
+    }
+    s->launches++;
+    if (e != cudaSuccess) return cuda_fail("pa_bench_update_only", e);
+  }
+  return PA_OK;
+}
+
+pa_status pa_debug_set_wait_limit(pa_solver* s, uint32_t polls) {
+  if (!s) return arg_fail("pa_debug_set_wait_limit: solver is NULL");
+  s->d.wait_limit = polls ? polls : 0u;
   return PA_OK;
 }
 
@@ -379,7 +420,7 @@ pa_status pa_set_kernel_timing(pa_solver* s, int enable) {
   return PA_OK;
 }
 
-pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches) {
+pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches, int reset) {
   if (!s || !update_ms || !n_launches) return arg_fail("pa_kernel_timing: NULL argument");
   *update_ms = 0.0;
   *n_launches = 0;
@@ -394,7 +435,7 @@ pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches)
   }
   *update_ms = tot;
   *n_launches = (int64_t)s->ev_next;
-  s->ev_next = 0;
+  if (reset) s->ev_next = 0;
   return PA_OK;
 }
 

@@ -109,3 +109,28 @@ def test_nonblocking_stream():
     s2.init(x0)
     _run(s2, g2, eps2)
     assert np.array_equal(a, s2.result().cpu().numpy())
+
+
+def test_bounded_wait_reports_timeout_and_context_survives():
+    """Force every mbarrier wait of the bulk-copy update kernel to give up at
+    once: the kernel records a timeout (no hang, no fault), drains its copies,
+    and the next synchronising call reports PA_ERR_TIMEOUT. After pa_init the
+    same solver reproduces a clean run bit for bit."""
+    w = W.SD15.with_(T=30, window=30)
+    s, g, eps, x0 = _solver(w)
+    s.init(x0)
+    _run(s, g, eps)
+    clean = s.result().cpu().numpy()
+    s.init(x0)
+    out = s.step()
+    g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+    abi.pa_debug_set_wait_limit(s.h, 0)
+    s.submit_eps(eps)
+    with pytest.raises(abi.PaError) as e:
+        s.step()
+    assert e.value.status == abi.PA_ERR_TIMEOUT
+    abi.pa_debug_set_wait_limit(s.h, 1 << 24)
+    s.init(x0)
+    _run(s, g, eps)
+    assert np.array_equal(clean, s.result().cpu().numpy())
+    assert s.stats()["device_status"] == 0

@@ -147,3 +147,20 @@ def test_gmm_kernel_against_oracle():
         rel = np.abs(got - want).max(axis=1) / np.abs(want).max(axis=1)
         assert rel.max() <= 2e-6, rel.max()
         g.close()
+
+
+@pytest.mark.parametrize("kind", [0, 1] + list(range(100, 110)))
+def test_update_kernels_agree(kind):
+    """Plain-load and tile-parallel bulk-copy update kernels (every launch
+    shape) take the same decisions and agree with the oracle; their states
+    differ only by the rounding of the compensated prefix sums."""
+    w = W.Workload("multi-strip", T=40, window=24, batch=3, latent_shape=(4, 20, 20), K=6,
+                   tol=1e-3, cache_thresh=0.05, seed=12)
+    orc = oracle_run(w)
+    ref = gpu_run(w, update_kernel=0)
+    got = gpu_run(w, update_kernel=kind)
+    assert got["stats"]["update_kernel"] == (0 if kind == 0 else 1)
+    assert compare(w, orc, got).max() <= REL_TOL
+    assert np.array_equal(ref["log"], got["log"])
+    scale = np.abs(ref["x_final"]).max()
+    assert np.abs(ref["x_final"] - got["x_final"]).max() <= 1e-6 * scale
