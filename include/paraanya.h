@@ -218,6 +218,10 @@ PA_API pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* mean
 PA_API pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32_t* miss_bt_dev,
                      const int32_t* n_rows_dev, float* batch_eps_dev);
 
+/* Synchronise the handle's stream and report a device-side failure of the
+ * denoiser kernels (a bounded bulk-copy wait that ran out): PA_ERR_TIMEOUT. */
+PA_API pa_status pa_gmm_check(pa_gmm* g);
+
 /* Kernels launched by this handle since pa_gmm_create. */
 PA_API int64_t pa_gmm_launches(const pa_gmm* g);
 

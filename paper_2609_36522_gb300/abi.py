@@ -68,6 +68,7 @@ _PROTOS = {
     "pa_gmm_create": (C.c_int, [PVP, C.c_int, C.c_int64, VP, C.c_double,
                                 C.POINTER(C.c_double), C.c_int, C.c_int, VP, C.c_size_t, VP]),
     "pa_gmm_eps": (C.c_int, [VP, VP, VP, VP, VP]),
+    "pa_gmm_check": (C.c_int, [VP]),
     "pa_gmm_launches": (C.c_int64, [VP]),
     "pa_gmm_destroy": (None, [VP]),
     "pa_status_string": (C.c_char_p, [C.c_int]),
@@ -248,6 +249,10 @@ def pa_gmm_create(K, D, means_ptr, std, alphas_cumprod, T, max_rows, workspace_p
 def pa_gmm_eps(g, batch_x_ptr, miss_bt_ptr, n_rows_dev_ptr, batch_eps_ptr):
     return _check("pa_gmm_eps", lib().pa_gmm_eps(g, _dptr(batch_x_ptr), _dptr(miss_bt_ptr),
                                                  _dptr(n_rows_dev_ptr), _dptr(batch_eps_ptr)))
+
+
+def pa_gmm_check(g):
+    return _check("pa_gmm_check", lib().pa_gmm_check(g))
 
 
 def pa_gmm_launches(g):

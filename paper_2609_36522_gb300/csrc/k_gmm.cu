@@ -6,19 +6,25 @@
 //   r = softmax(logit)   (the common -||x||^2 / (2 v) term cancels)
 //   eps = sqrt(1 - a) / v * (x - sqrt(a) sum_k r_k mu_k)
 //
-// Three kernels per call:
-//   k_gmm_dots     split-K partial contraction G = X M^T   [rows x K]
-//   k_gmm_softmax  fixed-order split sum, logits, softmax  (one warp per row)
-//   k_gmm_out      eps = a x - a sqrt(a) R M                [rows x D]
+// Three kernels per call, each with a single load phase:
+//   k_gmm_dots     split-K contraction G = X M^T: a CTA stages a tile of 16
+//                  rows and its D-chunk of every mean (bulk copies), one warp
+//                  per row accumulates 16 components per pass, partials go to
+//                  gpart[chunk][row][k]
+//   k_gmm_softmax  one CTA per row: fixed-order sum of the chunk partials,
+//                  logits, max-subtracted softmax
+//   k_gmm_out      a CTA stages a 16-row x 256-column tile of X and the same
+//                  columns of every mean, then eps = a x - a sqrt(a) R M
 // Per-timestep scalars (sqrt(a), 1/(2v), sqrt(1-a)/v) are computed on the
 // host in fp64 from alpha-bar and stored in fp32, so 1 - a never cancels in
-// fp32.
+// fp32. Reductions run in a fixed order: results are bitwise reproducible.
 #include <cmath>
 #include <cstring>
 #include <string>
 #include <vector>
 
 #include "../../include/paraanya.h"
+#include "pa_bulk.cuh"
 #include "pa_internal.h"
 
 namespace pa {
@@ -27,35 +33,46 @@ void set_error(const std::string& msg);  // pa_solver.cpp
 
 namespace {
 
+using pa::bulk_g2s;
+using pa::fence_barrier_init;
+using pa::mbar_arrive_expect_tx;
+using pa::mbar_init;
+using pa::mbar_wait_bounded;
+
 constexpr int kMaxK = 128;
-constexpr int kDotThreads = 256;
-constexpr int kDotRows = 16;     // rows per dots CTA
-constexpr int kDotTile = 64;     // columns staged per step
-constexpr int kOutCols = 128;    // columns per output CTA
-constexpr int kOutRows = 32;     // rows per output CTA
+constexpr int kThreads = 256;
+constexpr int kDotRows = 16;     // rows per dots CTA (two per warp)
+constexpr int kKTile = 16;       // components accumulated per pass
+constexpr int kOutRows = 16;     // rows per output CTA
+constexpr int kOutCols = 256;    // columns per output CTA (one per thread)
+constexpr size_t kDotSmemBudget = 96 * 1024;
 
 struct GmmLayout {
-  size_t coef, mnorm, gpart, R, rowc, total;
-  int nsplit;
-  int64_t split_len;
+  size_t coef, mnorm, gpart, R, rowc, status, total;
+  int nchunk;       // D-chunks of the dots kernel
+  int chunk;        // columns per chunk
 };
+
+int dots_chunk(int K, int64_t D) {
+  // largest of 512/256/128/64 columns whose (rows + K) row segments fit the budget
+  int c = 512;
+  while (c > 64 && (size_t)(kDotRows + K) * (c + 4) * sizeof(float) > kDotSmemBudget) c /= 2;
+  while (c > 64 && (int64_t)c >= 2 * D) c /= 2;
+  return c;
+}
 
 GmmLayout gmm_layout(int K, int64_t D, int max_rows, int T) {
   GmmLayout L{};
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t at = o; o = pa::align_up(o + bytes, pa::kAlign); return at; };
-  // split D so that the dots grid has a few waves even for small batches
-  int64_t split_len = 2048;
-  while (split_len > 256 && (D + split_len - 1) / split_len * ((max_rows + kDotRows - 1) / kDotRows) < 304)
-    split_len /= 2;
-  split_len = std::max<int64_t>(kDotTile, split_len);
-  L.split_len = split_len;
-  L.nsplit = (int)((D + split_len - 1) / split_len);
+  L.chunk = dots_chunk(K, D);
+  L.nchunk = (int)((D + L.chunk - 1) / L.chunk);
   L.coef = take((size_t)3 * T * sizeof(float));
   L.mnorm = take((size_t)K * sizeof(float));
-  L.gpart = take((size_t)L.nsplit * max_rows * K * sizeof(float));
+  L.gpart = take((size_t)L.nchunk * max_rows * K * sizeof(float));
   L.R = take((size_t)max_rows * K * sizeof(float));
   L.rowc = take((size_t)max_rows * 2 * sizeof(float));
+  L.status = take(sizeof(int32_t));
   L.total = o;
   return L;
 }
@@ -88,135 +105,177 @@ __global__ void __launch_bounds__(256) k_gmm_norms(const float* __restrict__ mu,
   }
 }
 
-// gpart[split][r][k] = sum over this split's columns of x[r][d] mu[k][d]
-__global__ void __launch_bounds__(kDotThreads) k_gmm_dots(const float* __restrict__ X,
-                                                          const float* __restrict__ mu,
-                                                          const int32_t* __restrict__ n_rows_dev,
-                                                          int K, int64_t D, int64_t split_len,
-                                                          int max_rows, float* __restrict__ gpart) {
-  __shared__ float xs[kDotRows][kDotTile + 1];
-  __shared__ float ms[kMaxK][kDotTile + 1];
+// Stage `nrows` row segments [c0, c0 + ncol) of a row-major matrix with row
+// length D into shared rows of stride `ld` floats: bulk copies counted on
+// `bar`, issued by thread 0 (after the caller announced the bytes), or plain
+// loads by every thread when `bulk` is false.
+__device__ __forceinline__ void stage_rows(float* dst, int ld, const float* src, int64_t D, int64_t c0,
+                                           int ncol, int nrows, bool bulk, uint64_t* bar) {
+  if (bulk) {
+    if (threadIdx.x == 0) {
+      const uint32_t seg = (uint32_t)ncol * sizeof(float);
+      for (int r = 0; r < nrows; ++r) bulk_g2s(dst + (size_t)r * ld, src + (int64_t)r * D + c0, seg, bar);
+    }
+    return;
+  }
+  for (int q = threadIdx.x; q < nrows * ncol; q += blockDim.x) {
+    const int r = q / ncol, c = q % ncol;
+    dst[(size_t)r * ld + c] = src[(int64_t)r * D + c0 + c];
+  }
+}
+
+// Wait for the bulk copies of a single-phase kernel. On a timeout: record it,
+// let the copies already issued land (bounded), and report false.
+__device__ __forceinline__ bool wait_staged(bool bulk, uint64_t* bar, int32_t* status) {
+  if (!bulk) return true;
+  if (mbar_wait_bounded(bar, 0, pa::kWaitLimit)) return true;
+  atomicCAS(status, 0, pa::kDevTimeout);
+  mbar_wait_bounded(bar, 0, pa::kDrainLimit);
+  return false;
+}
+
+// gpart[chunk][r][k] = sum over the chunk's columns of x[r][d] mu[k][d]
+__global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__ X,
+                                                       const float* __restrict__ mu,
+                                                       const int32_t* __restrict__ n_rows_dev,
+                                                       int K, int64_t D, int chunk, int max_rows,
+                                                       bool bulk, float* __restrict__ gpart,
+                                                       int32_t* status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bar;
   const int n_rows = min(*n_rows_dev, max_rows);
   const int r0 = blockIdx.y * kDotRows;
   if (r0 >= n_rows) return;
-  const int split = blockIdx.x;
-  const int64_t d0 = (int64_t)split * split_len;
-  const int64_t d1 = (D < d0 + split_len) ? D : d0 + split_len;
-  const int nout = kDotRows * K;  // <= 16 * 128 = 2048 -> 8 per thread
-  float acc[8];
+  const int nr = min(kDotRows, n_rows - r0);
+  const int64_t c0 = (int64_t)blockIdx.x * chunk;
+  const int ncol = (int)(((D - c0) < chunk) ? (D - c0) : chunk);
+  const int ld = chunk + 4;  // padded row stride, keeps 16-byte alignment
+  float* xs = reinterpret_cast<float*>(smem_raw);
+  float* ms = xs + (size_t)kDotRows * ld;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+    if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
+  }
+  __syncthreads();
+  stage_rows(xs, ld, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
+  stage_rows(ms, ld, mu, D, c0, ncol, K, bulk, &bar);
+  const bool ok = wait_staged(bulk, &bar, status);
+  __syncthreads();
+  if (!ok) return;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int rr = warp; rr < nr; rr += kThreads / 32) {
+    const float* xr = xs + (size_t)rr * ld;
+    for (int k0 = 0; k0 < K; k0 += kKTile) {
+      float acc[kKTile];
 #pragma unroll
-  for (int u = 0; u < 8; ++u) acc[u] = 0.f;
-  for (int64_t c0 = d0; c0 < d1; c0 += kDotTile) {
-    const int w = (int)((d1 - c0) < kDotTile ? (d1 - c0) : kDotTile);
-    for (int q = threadIdx.x; q < kDotRows * kDotTile; q += kDotThreads) {
-      const int rr = q / kDotTile, cc = q % kDotTile;
-      const int r = r0 + rr;
-      xs[rr][cc] = (r < n_rows && cc < w) ? X[(int64_t)r * D + c0 + cc] : 0.f;
-    }
-    for (int q = threadIdx.x; q < K * kDotTile; q += kDotThreads) {
-      const int k = q / kDotTile, cc = q % kDotTile;
-      ms[k][cc] = (cc < w) ? mu[(int64_t)k * D + c0 + cc] : 0.f;
-    }
-    __syncthreads();
+      for (int u = 0; u < kKTile; ++u) acc[u] = 0.f;
+      for (int c = lane; c < ncol; c += 32) {
+        const float xv = xr[c];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
-      const int o = threadIdx.x + u * kDotThreads;
-      if (o < nout) {
-        const int rr = o / K, k = o % K;
-        float a = acc[u];
-#pragma unroll 16
-        for (int cc = 0; cc < kDotTile; ++cc) a = fmaf(xs[rr][cc], ms[k][cc], a);
-        acc[u] = a;
+        for (int u = 0; u < kKTile; ++u)
+          if (k0 + u < K) acc[u] = fmaf(xv, ms[(size_t)(k0 + u) * ld + c], acc[u]);
+      }
+#pragma unroll
+      for (int u = 0; u < kKTile; ++u) acc[u] = warp_sum(acc[u]);
+      if (lane < kKTile && k0 + lane < K) {
+        float v = 0.f;
+#pragma unroll
+        for (int u = 0; u < kKTile; ++u) v = (lane == u) ? acc[u] : v;
+        gpart[((int64_t)blockIdx.x * max_rows + r0 + rr) * K + k0 + lane] = v;
       }
     }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int u = 0; u < 8; ++u) {
-    const int o = threadIdx.x + u * kDotThreads;
-    if (o < nout) {
-      const int rr = o / K, k = o % K;
-      const int r = r0 + rr;
-      if (r < n_rows) gpart[((int64_t)split * max_rows + r) * K + k] = acc[u];
-    }
   }
 }
 
-// One warp per row: dots (fixed-order split sum) -> logits -> softmax.
-__global__ void __launch_bounds__(256) k_gmm_softmax(const float* __restrict__ gpart,
-                                                     const float* __restrict__ mnorm,
-                                                     const float* __restrict__ coef, int T,
-                                                     const int32_t* __restrict__ miss_bt,
-                                                     const int32_t* __restrict__ n_rows_dev,
-                                                     int K, int nsplit, int max_rows,
-                                                     float* __restrict__ R,
-                                                     float* __restrict__ rowc) {
+// One CTA per row: dots (fixed-order chunk sum) -> logits -> softmax.
+__global__ void __launch_bounds__(kThreads) k_gmm_softmax(const float* __restrict__ gpart,
+                                                          const float* __restrict__ mnorm,
+                                                          const float* __restrict__ coef, int T,
+                                                          const int32_t* __restrict__ miss_bt,
+                                                          const int32_t* __restrict__ n_rows_dev,
+                                                          int K, int nchunk, int max_rows,
+                                                          float* __restrict__ R,
+                                                          float* __restrict__ rowc) {
+  __shared__ float s_part[kThreads];
+  __shared__ float s_logit[kMaxK];
   const int n_rows = min(*n_rows_dev, max_rows);
-  const int r = blockIdx.x * 8 + (threadIdx.x >> 5);
-  const int lane = threadIdx.x & 31;
+  const int r = blockIdx.x;
   if (r >= n_rows) return;
+  // thread -> (component k, chunk group g); groups take the chunks round robin
+  int KB = 1;
+  while (KB < K) KB <<= 1;
+  const int G = kThreads / KB;
+  const int k = threadIdx.x % KB, g = threadIdx.x / KB;
+  float part = 0.f;
+  if (k < K)
+    for (int s = g; s < nchunk; s += G) part += gpart[((int64_t)s * max_rows + r) * K + k];
+  s_part[threadIdx.x] = part;
   const int i = miss_bt[2 * r + 1];
   const float sa = coef[i], q = coef[T + i], ac = coef[2 * T + i];
-  float l[kMaxK / 32];
-  float mx = -INFINITY;
-#pragma unroll
-  for (int u = 0; u < kMaxK / 32; ++u) {
-    const int k = lane + 32 * u;
-    l[u] = -INFINITY;
-    if (k < K) {
-      float dot = 0.f;
-      for (int s = 0; s < nsplit; ++s) dot += gpart[((int64_t)s * max_rows + r) * K + k];
-      l[u] = (2.f * sa * dot - sa * sa * mnorm[k]) * q;
-      mx = fmaxf(mx, l[u]);
+  __syncthreads();
+  if (threadIdx.x < K) {
+    float dot = 0.f;
+    for (int gg = 0; gg < G; ++gg) dot += s_part[gg * KB + threadIdx.x];
+    s_logit[threadIdx.x] = (2.f * sa * dot - sa * sa * mnorm[threadIdx.x]) * q;
+  }
+  __syncthreads();
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    float mx = -INFINITY;
+    for (int kk = lane; kk < K; kk += 32) mx = fmaxf(mx, s_logit[kk]);
+    mx = warp_max(mx);
+    float sum = 0.f;
+    for (int kk = lane; kk < K; kk += 32) sum += expf(s_logit[kk] - mx);
+    sum = warp_sum(sum);
+    const float inv = 1.f / sum;
+    for (int kk = lane; kk < K; kk += 32) R[(int64_t)r * K + kk] = expf(s_logit[kk] - mx) * inv;
+    if (lane == 0) {
+      rowc[2 * r] = ac;
+      rowc[2 * r + 1] = ac * sa;
     }
-  }
-  mx = warp_max(mx);
-  float sum = 0.f;
-#pragma unroll
-  for (int u = 0; u < kMaxK / 32; ++u) {
-    const int k = lane + 32 * u;
-    l[u] = (k < K) ? expf(l[u] - mx) : 0.f;
-    sum += l[u];
-  }
-  sum = warp_sum(sum);
-  const float inv = 1.f / sum;
-#pragma unroll
-  for (int u = 0; u < kMaxK / 32; ++u) {
-    const int k = lane + 32 * u;
-    if (k < K) R[(int64_t)r * K + k] = l[u] * inv;
-  }
-  if (lane == 0) {
-    rowc[2 * r] = ac;
-    rowc[2 * r + 1] = ac * sa;
   }
 }
 
-// eps[r][d] = ac x[r][d] - ac sqrt(a) sum_k R[r][k] mu[k][d]
+// eps[r][c] = ac x[r][c] - ac sqrt(a) sum_k R[r][k] mu[k][c]
 __global__ void __launch_bounds__(kOutCols) k_gmm_out(const float* __restrict__ X,
                                                       const float* __restrict__ mu,
                                                       const float* __restrict__ R,
                                                       const float* __restrict__ rowc,
                                                       const int32_t* __restrict__ n_rows_dev,
-                                                      int K, int64_t D, int max_rows,
-                                                      float* __restrict__ eps) {
-  extern __shared__ float sm[];  // ms[K][kOutCols], rs[kOutRows][K]
-  float* ms = sm;
-  float* rs = sm + (size_t)K * kOutCols;
+                                                      int K, int64_t D, int max_rows, bool bulk,
+                                                      float* __restrict__ eps, int32_t* status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bar;
+  __shared__ float s_r[kOutRows * kMaxK];
+  __shared__ float s_c[kOutRows * 2];
   const int n_rows = min(*n_rows_dev, max_rows);
   const int r0 = blockIdx.y * kOutRows;
   if (r0 >= n_rows) return;
-  const int64_t c = (int64_t)blockIdx.x * kOutCols + threadIdx.x;
-  for (int k = 0; k < K; ++k) ms[k * kOutCols + threadIdx.x] = (c < D) ? mu[(int64_t)k * D + c] : 0.f;
   const int nr = min(kOutRows, n_rows - r0);
-  for (int q = threadIdx.x; q < nr * K; q += kOutCols) rs[q] = R[(int64_t)r0 * K + q];
+  const int64_t c0 = (int64_t)blockIdx.x * kOutCols;
+  const int ncol = (int)(((D - c0) < kOutCols) ? (D - c0) : kOutCols);
+  float* ms = reinterpret_cast<float*>(smem_raw);   // [K][kOutCols]
+  float* xs = ms + (size_t)K * kOutCols;            // [kOutRows][kOutCols]
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_barrier_init();
+    if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
+  }
   __syncthreads();
-  if (c >= D) return;
+  stage_rows(ms, kOutCols, mu, D, c0, ncol, K, bulk, &bar);
+  stage_rows(xs, kOutCols, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
+  for (int q = threadIdx.x; q < nr * K; q += kOutCols) s_r[q] = R[(int64_t)r0 * K + q];
+  for (int q = threadIdx.x; q < nr * 2; q += kOutCols) s_c[q] = rowc[2 * r0 + q];
+  const bool ok = wait_staged(bulk, &bar, status);
+  __syncthreads();
+  if (!ok) return;
+  const int c = threadIdx.x;
+  if (c >= ncol) return;
   for (int rr = 0; rr < nr; ++rr) {
-    const int r = r0 + rr;
     float m = 0.f;
-    for (int k = 0; k < K; ++k) m = fmaf(rs[rr * K + k], ms[k * kOutCols + threadIdx.x], m);
-    const float ac = rowc[2 * r], acs = rowc[2 * r + 1];
-    eps[(int64_t)r * D + c] = ac * X[(int64_t)r * D + c] - acs * m;
+    for (int k = 0; k < K; ++k) m = fmaf(s_r[rr * K + k], ms[(size_t)k * kOutCols + c], m);
+    eps[(int64_t)(r0 + rr) * D + c0 + c] = s_c[2 * rr] * xs[(size_t)rr * kOutCols + c] - s_c[2 * rr + 1] * m;
   }
 }
 
@@ -273,25 +332,23 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
   }
   cudaError_t e = cudaMemcpyAsync(g->ws + L.coef, coef.data(), coef.size() * sizeof(float),
                                   cudaMemcpyHostToDevice, g->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.status, 0, sizeof(int32_t), g->st);
   if (e == cudaSuccess) {
     k_gmm_norms<<<K, 256, 0, g->st>>>(means_dev, D, reinterpret_cast<float*>(g->ws + L.mnorm));
     g->launches++;
     e = cudaGetLastError();
   }
+  const size_t dots_smem = (size_t)(kDotRows + K) * (L.chunk + 4) * sizeof(float);
+  const size_t out_smem = (size_t)(K + kOutRows) * kOutCols * sizeof(float);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_gmm_dots, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dots_smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_gmm_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out_smem);
   if (e == cudaSuccess) e = cudaStreamSynchronize(g->st);
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_create: ") + cudaGetErrorString(e));
     delete g;
     return PA_ERR_CUDA;
-  }
-  const size_t out_smem = ((size_t)K * kOutCols + (size_t)kOutRows * K) * sizeof(float);
-  if (out_smem > 48 * 1024) {
-    e = cudaFuncSetAttribute(k_gmm_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out_smem);
-    if (e != cudaSuccess) {
-      pa::set_error(std::string("pa_gmm_create: ") + cudaGetErrorString(e));
-      delete g;
-      return PA_ERR_CUDA;
-    }
   }
   *out = g;
   return PA_OK;
@@ -309,22 +366,38 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
   float* gpart = reinterpret_cast<float*>(g->ws + L.gpart);
   float* R = reinterpret_cast<float*>(g->ws + L.R);
   float* rowc = reinterpret_cast<float*>(g->ws + L.rowc);
-  const int rb = (g->max_rows + kDotRows - 1) / kDotRows;
-  k_gmm_dots<<<dim3(L.nsplit, rb), kDotThreads, 0, g->st>>>(batch_x_dev, g->means, n_rows_dev,
-                                                           g->K, g->D, L.split_len, g->max_rows, gpart);
-  k_gmm_softmax<<<(g->max_rows + 7) / 8, 256, 0, g->st>>>(gpart, mnorm, coef, g->T, miss_bt_dev,
-                                                         n_rows_dev, g->K, L.nsplit, g->max_rows,
-                                                         R, rowc);
-  const size_t out_smem = ((size_t)g->K * kOutCols + (size_t)kOutRows * g->K) * sizeof(float);
+  int32_t* status = reinterpret_cast<int32_t*>(g->ws + L.status);
+  // bulk copies need 16-byte aligned rows: D % 4 == 0 and aligned base pointers
+  const bool bulk = g->D % 4 == 0 && ((reinterpret_cast<uintptr_t>(batch_x_dev) |
+                                       reinterpret_cast<uintptr_t>(g->means)) & 15) == 0;
+  const size_t dots_smem = (size_t)(kDotRows + g->K) * (L.chunk + 4) * sizeof(float);
+  const size_t out_smem = (size_t)(g->K + kOutRows) * kOutCols * sizeof(float);
+  k_gmm_dots<<<dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows), kThreads, dots_smem, g->st>>>(
+      batch_x_dev, g->means, n_rows_dev, g->K, g->D, L.chunk, g->max_rows, bulk, gpart, status);
+  k_gmm_softmax<<<g->max_rows, kThreads, 0, g->st>>>(gpart, mnorm, coef, g->T, miss_bt_dev, n_rows_dev,
+                                                     g->K, L.nchunk, g->max_rows, R, rowc);
   k_gmm_out<<<dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
               kOutCols, out_smem, g->st>>>(batch_x_dev, g->means, R, rowc, n_rows_dev, g->K, g->D,
-                                            g->max_rows, batch_eps_dev);
+                                            g->max_rows, bulk, batch_eps_dev, status);
   g->launches += 3;
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_eps: ") + cudaGetErrorString(e));
     return PA_ERR_CUDA;
   }
+  return PA_OK;
+}
+
+extern "C" pa_status pa_gmm_check(pa_gmm* g) {
+  if (!g) { pa::set_error("pa_gmm_check: NULL handle"); return PA_ERR_ARG; }
+  int32_t st = 0;
+  cudaError_t e = cudaMemcpyAsync(&st, g->ws + g->L.status, sizeof(st), cudaMemcpyDeviceToHost, g->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(g->st);
+  if (e != cudaSuccess) {
+    pa::set_error(std::string("pa_gmm_check: ") + cudaGetErrorString(e));
+    return PA_ERR_CUDA;
+  }
+  if (st == pa::kDevTimeout) { pa::set_error("pa_gmm_check: a bounded wait ran out"); return PA_ERR_TIMEOUT; }
   return PA_OK;
 }
 

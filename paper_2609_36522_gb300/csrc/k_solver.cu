@@ -248,38 +248,27 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
     s_m[b] = 0;
     s_h1[b] = 0;
   }
-  // 1. reductions, one warp per (b, j), eight independent partial sums per
-  // lane combined in a fixed order (deterministic). Positions beyond a
-  // trajectory's window are reduced too (their values are never used).
-  for (int q = warp; q < B * P; q += nwarps) {
-    const float* pe = d.part_err + (int64_t)q * nchunk;
-    const float* pd = d.part_del + (int64_t)q * nchunk;
-    float se[8], sd[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) { se[u] = 0.f; sd[u] = 0.f; }
-    for (int c0 = 0; c0 < nchunk; c0 += 256) {
-#pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        const int c = c0 + u * 32 + lane;
-        if (c < nchunk) {
-          se[u] += pe[c];
-          sd[u] += pd[c];
-        }
-      }
+  // 1. reductions: one thread per (quantity, b, j) sums the chunk partials in
+  // a fixed order (four interleaved accumulators), so every partial load of
+  // the kernel is issued in the first round. Positions beyond a trajectory's
+  // window are reduced too (their values are never used).
+  const int npair = B * P;
+  for (int q = tid; q < 2 * npair; q += kDecideThreads) {
+    const int which = q / npair, pr = q % npair;
+    const float* src = (which ? d.part_del : d.part_err) + (int64_t)pr * nchunk;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    int c = 0;
+#pragma unroll 8
+    for (; c + 4 <= nchunk; c += 4) {
+      acc[0] += src[c];
+      acc[1] += src[c + 1];
+      acc[2] += src[c + 2];
+      acc[3] += src[c + 3];
     }
-    float te = ((se[0] + se[1]) + (se[2] + se[3])) + ((se[4] + se[5]) + (se[6] + se[7]));
-    float td = ((sd[0] + sd[1]) + (sd[2] + sd[3])) + ((sd[4] + sd[5]) + (sd[6] + sd[7]));
-    te = warp_sum(te);
-    td = warp_sum(td);
-    if (lane == 0) {
-      const float ve = te / (float)d.D, vd = td / (float)d.D;
-      red_e[q] = ve;
-      red_d[q] = vd;
-      if (in_smem) {  // keep the global copy for pa_last_reductions
-        d.red_err[q] = ve;
-        d.red_del[q] = vd;
-      }
-    }
+    for (; c < nchunk; ++c) acc[0] += src[c];
+    const float v = ((acc[0] + acc[1]) + (acc[2] + acc[3])) / (float)d.D;
+    (which ? red_d : red_e)[pr] = v;
+    if (in_smem) (which ? d.red_del : d.red_err)[pr] = v;  // global copy for pa_last_reductions
   }
   __syncthreads();
   if (s_active == 0) return;  // finished: iterating further is a no-op

@@ -28,57 +28,20 @@
 // the solver's status word and stops further issues; the CTA finishes its
 // (now meaningless) arithmetic with in-bounds accesses only, drains the
 // copies already issued with bounded waits, and returns.
+#include <cooperative_groups.h>
+
+#include "pa_bulk.cuh"
 #include "pa_internal.h"
 
 namespace pa {
 namespace {
 
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
+namespace cg = cooperative_groups;
 
-__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
-  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(bar)), "r"(count) : "memory");
-}
+// CTAs per thread-block cluster: the strips of a cluster combine their
+// per-position partial sums through distributed shared memory.
+constexpr int kCluster = 8;
 
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
-  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(bar)), "r"(bytes)
-               : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-
-__device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
-  asm volatile(
-      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-          smem_u32(dst)),
-      "l"(src), "r"(bytes), "r"(smem_u32(bar))
-      : "memory");
-}
-
-__device__ __forceinline__ void fence_barrier_init() {
-  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-}
-
-// Bounded wait on one mbarrier phase; false when `limit` polls ran out.
-__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint32_t limit) {
-  for (uint32_t n = 0; n < limit; ++n) {
-    if (mbar_try_wait(bar, parity)) return true;
-  }
-  return false;
-}
-
-constexpr uint32_t kDrainLimit = 1u << 24;
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -144,8 +107,9 @@ struct TileShape {
   static constexpr size_t kTileBytes = kTileFloats * sizeof(float);
   static constexpr int kMaxBuf = 16;                  // mbarriers in the barrier area
   static constexpr size_t kBarBytes = 128;
-  // per position: rank, c-1, e, cache slot, state-ring slot of the next state
-  __host__ __device__ static size_t meta_bytes(int P) { return ((size_t)P * 20 + 127) / 128 * 128; }
+  // per position: rank, c-1, e, cache slot, state-ring slot of the next state,
+  // and this strip's two partial sums (err, distance)
+  __host__ __device__ static size_t meta_bytes(int P) { return ((size_t)P * 28 + 127) / 128 * 128; }
   static constexpr size_t kTotBytes = (size_t)NW * SEG * 2 * sizeof(float);   // segment totals
   static constexpr size_t kCarBytes = kTotBytes;                              // carries into warps
   static constexpr size_t kRedBytes = ((size_t)2 * TW * 33 * sizeof(float) + 127) / 128 * 128;
@@ -175,6 +139,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   float* s_ec = reinterpret_cast<float*>(q + (size_t)P * 8);
   int32_t* s_slot = reinterpret_cast<int32_t*>(q + (size_t)P * 12);  // (t+j) mod P
   int32_t* s_nxt = reinterpret_cast<int32_t*>(q + (size_t)P * 16);   // (t+j+1) mod (P+1)
+  float* s_pos = reinterpret_cast<float*>(q + (size_t)P * 20);        // [2][P] strip partials
   q += Sh::meta_bytes(P);
   float* s_tot = reinterpret_cast<float*>(q);   // [NW][SEG][2]
   q += Sh::kTotBytes;
@@ -195,6 +160,8 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
     s_nxt[j] = (t + j + 1) % (P + 1);
     s_cm1[j] = d.cm1[t + j];
     s_ec[j] = d.ecoef[t + j];
+    s_pos[j] = 0.f;
+    s_pos[P + j] = 0.f;
   }
   if (tid == 0) {
     for (int k = 0; k < nbuf; ++k) mbar_init(&bar[k], 1);
@@ -209,7 +176,8 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   }
   __syncthreads();
 
-  const int strip = blockIdx.x;
+  const int strip = blockIdx.x;          // the grid is padded to whole clusters
+  const bool active = strip < nstrip;
   const int64_t c0 = (int64_t)strip * SEG;
   const int64_t ncol = (D - c0) < SEG ? (D - c0) : SEG;
   const uint32_t seg_bytes = (uint32_t)ncol * sizeof(float);
@@ -218,7 +186,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   float* Xb = d.X + (int64_t)b * (P + 1) * D;
   float* Xh = d.Xhat + (int64_t)b * P * D;
   float* Eh = d.Ehat + (int64_t)b * P * D;
-  const int ntile = (p + TW - 1) / TW;
+  const int ntile = active ? (p + TW - 1) / TW : 0;
 
   // Warp 0 issues tile k into buffer k % nbuf; lane l fetches positions
   // k*TW + l, k*TW + l + 32, ... The whole tile's byte count is announced on
@@ -271,7 +239,6 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
 #pragma unroll
   for (int v = 0; v < V; ++v) { chi[v] = xlast.a[v]; clo[v] = 0.f; }
 
-  const int64_t pbase = (int64_t)b * P * nstrip + strip;
   const int red_first = NW * 32 - 2 * TW;  // the last 2*TW threads finish the reductions
   int my_fail = 0;   // this thread's wait ran out
   int aborted = 0;   // some thread's wait ran out (CTA-uniform, from a barrier)
@@ -406,9 +373,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
           acc[2] += row[c + 2];
           acc[3] += row[c + 3];
         }
-        const float sum = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-        float* dst = (r < TW) ? d.part_err : d.part_del;
-        dst[pbase + (int64_t)j * nstrip] = sum;
+        s_pos[(r < TW ? 0 : P) + j] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
       }
     }
   }
@@ -417,6 +382,24 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
     for (int k = (issued > nbuf ? issued - nbuf : 0); k < issued; ++k)
       mbar_wait_bounded(&bar[k % nbuf], (uint32_t)((k / nbuf) & 1), kDrainLimit);
   }
+  // Combine the strips of this cluster: CTA rank q sums positions j = q mod
+  // kCluster over the cluster's CTAs in rank order (distributed shared
+  // memory) and writes part[b][j][cluster]. The second cluster barrier keeps
+  // every CTA's shared memory alive until its peers have read it.
+  cg::cluster_group cluster = cg::this_cluster();
+  cluster.sync();
+  const int rank = (int)cluster.block_rank();
+  const int nclus = gridDim.x / kCluster;
+  const int64_t cbase = (int64_t)b * P * nclus + blockIdx.x / kCluster;
+  for (int q2 = tid; q2 < 2 * p; q2 += NW * 32) {
+    const int which = q2 / p, j = q2 % p;
+    if (j % kCluster != rank) continue;
+    float sum = 0.f;
+#pragma unroll
+    for (int r = 0; r < kCluster; ++r) sum += cluster.map_shared_rank(s_pos, r)[which * P + j];
+    (which == 0 ? d.part_err : d.part_del)[cbase + (int64_t)j * nclus] = sum;
+  }
+  cluster.sync();
 }
 
 // Shared memory budget per CTA for the tile buffers: enough for the whole
@@ -444,9 +427,21 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) configured[dev] = smem;
   }
-  *nchunk_out = nstrip;
-  kern<<<dim3(nstrip, d.B), NW * 32, smem, st>>>(d, beps, nstrip, nbuf, d.wait_limit);
-  return cudaGetLastError();
+  const int gx = (nstrip + kCluster - 1) / kCluster * kCluster;
+  *nchunk_out = gx / kCluster;  // one partial per cluster and position
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(gx, d.B, 1);
+  cfg.blockDim = dim3(NW * 32, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = kCluster;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, d, beps, nstrip, nbuf, d.wait_limit);
 }
 
 }  // namespace
