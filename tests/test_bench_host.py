@@ -1,0 +1,65 @@
+"""Host-side logic of bench.py's multi-rank path, on CPU with gloo (world size 2).
+
+Ranks run independent trajectories (weak scaling); the only collectives are the
+host-side timing reductions: iterations are summed and the slowest rank's time
+is taken.
+"""
+import os
+import socket
+
+import pytest
+import torch.multiprocessing as mp
+
+import workload as W
+
+
+def _free_port():
+    s = socket.socket()
+    s.bind(("127.0.0.1", 0))
+    port = s.getsockname()[1]
+    s.close()
+    return port
+
+
+def _worker(rank, world, port, out):
+    import torch.distributed as dist
+    import bench
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    units, secs = bench.aggregate(10 * (rank + 1), 0.5 + rank)
+    w = bench.rank_workload(W.BATCHED, rank)
+    out[rank] = (units, secs, w.seed, bench.rank_info())
+    dist.barrier()
+    dist.destroy_process_group()
+
+
+def test_aggregate_and_rank_seeds_gloo():
+    world = 2
+    port = _free_port()
+    mgr = mp.Manager()
+    out = mgr.dict()
+    mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
+    for r in range(world):
+        units, secs, seed, info = out[r]
+        assert units == 30.0 and secs == 1.5
+        assert seed == W.BATCHED.seed + r * W.BATCHED.batch
+        assert info == (r, world, r)
+
+
+def test_single_process_aggregate_is_identity():
+    import bench
+    assert bench.aggregate(7, 0.25) == (7.0, 0.25)
+
+
+def test_iteration_bytes_counts_rows():
+    import numpy as np
+    import bench
+    w = W.TINY
+    # one trajectory: t=0, p=8, 8 misses, stride 4, frontier 0 (all lazy), no hits
+    log = np.zeros((1, 1, 8), dtype=np.int32)
+    log[0, 0, :6] = (0, 8, 8, 4, 0, 0)
+    upd, other = bench.iteration_bytes(log, w)
+    row = w.D * 4
+    assert upd[0] == (1 + 0 + 8 + 16 + 0 + 8) * row
+    assert other[0] == (4 * 8 + w.K) * row
