@@ -227,6 +227,37 @@ PA_API int64_t pa_gmm_launches(const pa_gmm* g);
 
 PA_API void pa_gmm_destroy(pa_gmm* g);
 
+/* pa_gmm_eps without a handle and without any device allocation (the paper
+ * has no counterpart; this is a deployment convenience).
+ *
+ * For callers that cannot allocate device memory when they run the denoiser:
+ * plugins that only get buffers from their host framework, real-time loops
+ * that forbid cudaMalloc/cudaFree after start-up, code that does not own the
+ * device's allocator. The caller passes the inputs (means_dev [K][D],
+ * alphas_cumprod on the HOST [T+1], batch_x_dev [n_rows][D], miss_bt_dev
+ * [n_rows][2] whose second entries are sampling indices < T) and the output
+ * batch_eps_dev [n_rows][D]; results equal pa_gmm_eps's for the same inputs.
+ *
+ * Scratch lives in one fixed 4 MiB device array inside this library (every
+ * GPU that loads the library holds it until the process exits). Sizes whose
+ * scratch (3T coefficients, K norms, n_rows*K*ceil(D/chunk) partials,
+ * responsibilities) would exceed 4 MiB are rejected with PA_ERR_ARG and a
+ * message naming the bytes needed; use pa_gmm_create/pa_gmm_eps then.
+ *
+ * The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress) with that device current; make that first call
+ * before any stream capture. Every call on a device shares the one array and
+ * overwrites it (the status word is cleared at the start of each call), so
+ * calls whose work overlaps on the GPU -- on different streams, or from
+ * different host threads without ordering -- race and give wrong results.
+ * The call is asynchronous on `stream`; it calls no cudaMalloc, cudaFree or
+ * other allocating routine. A bounded-wait timeout inside its kernels is
+ * recorded in the array's status word only (not reported). */
+PA_API pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D, double std,
+                                    const double* alphas_cumprod, int T,
+                                    const float* batch_x_dev, const int32_t* miss_bt_dev,
+                                    int n_rows, float* batch_eps_dev, void* stream);
+
 /* ---- misc -------------------------------------------------------------- */
 
 PA_API const char* pa_status_string(int status);

@@ -71,6 +71,8 @@ _PROTOS = {
     "pa_gmm_check": (C.c_int, [VP]),
     "pa_gmm_launches": (C.c_int64, [VP]),
     "pa_gmm_destroy": (None, [VP]),
+    "pa_gmm_eps_noalloc": (C.c_int, [VP, C.c_int, C.c_int64, C.c_double, C.POINTER(C.c_double),
+                                     C.c_int, VP, VP, C.c_int, VP, VP]),
     "pa_status_string": (C.c_char_p, [C.c_int]),
     "pa_last_error": (C.c_char_p, []),
 }
@@ -261,3 +263,12 @@ def pa_gmm_launches(g):
 
 def pa_gmm_destroy(g):
     lib().pa_gmm_destroy(g)
+
+
+def pa_gmm_eps_noalloc(means_ptr, K, D, std, alphas_cumprod, batch_x_ptr, miss_bt_ptr, n_rows,
+                       batch_eps_ptr, stream_ptr):
+    """Denoiser eps with the library's fixed device scratch (no allocation)."""
+    alphas = (C.c_double * len(alphas_cumprod))(*[float(v) for v in alphas_cumprod])
+    return _check("pa_gmm_eps_noalloc", lib().pa_gmm_eps_noalloc(
+        _dptr(means_ptr), int(K), int(D), float(std), alphas, len(alphas_cumprod) - 1,
+        _dptr(batch_x_ptr), _dptr(miss_bt_ptr), int(n_rows), _dptr(batch_eps_ptr), _dptr(stream_ptr)))

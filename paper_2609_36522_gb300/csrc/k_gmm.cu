@@ -20,6 +20,7 @@
 // fp32. Reductions run in a fixed order: results are bitwise reproducible.
 #include <cmath>
 #include <cstring>
+#include <mutex>
 #include <string>
 #include <vector>
 
@@ -404,3 +405,152 @@ extern "C" pa_status pa_gmm_check(pa_gmm* g) {
 extern "C" int64_t pa_gmm_launches(const pa_gmm* g) { return g ? g->launches : -1; }
 
 extern "C" void pa_gmm_destroy(pa_gmm* g) { delete g; }
+
+// ---------------------------------------------------------------------------
+// Allocation-free variant of pa_gmm_eps (no counterpart in the paper).
+//
+// Some callers cannot allocate device memory when they need the denoiser: a
+// plugin that only receives buffers handed over by its host framework, a
+// real-time loop that forbids cudaMalloc/cudaFree after start-up because an
+// allocation may block, or code running where another allocator owns the
+// device. pa_gmm_eps keeps its scratch (per-timestep coefficients, ||mu_k||^2,
+// split-K partial dot products, responsibilities, a status word) in the
+// workspace of a pa_gmm handle; pa_gmm_eps_noalloc keeps the same scratch in
+// the fixed device array below and runs the same kernels on it.
+constexpr size_t kNoAllocScratchBytes = (size_t)4 << 20;  // 4 MiB, held by every device that loads this library
+
+// The fixed scratch. In host code `g_gmm_scratch` is only a stand-in name:
+// its device address comes from cudaGetSymbolAddress, looked up per device.
+static __device__ __align__(256) unsigned char g_gmm_scratch[kNoAllocScratchBytes];
+
+namespace {
+
+constexpr int kNoAllocMaxDevices = 64;
+constexpr int kNoAllocCoefChunk = 512;                    // host coefficients staged in chunks on the stack
+
+std::mutex g_scratch_mu;
+unsigned char* g_scratch_dev[kNoAllocMaxDevices] = {};
+
+// Device address of g_gmm_scratch for the current device, looked up once per
+// device (the host-side name is only a stand-in for the device array).
+pa_status scratch_for_current_device(unsigned char** out) {
+  int dev = -1;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) {
+    pa::set_error(std::string("pa_gmm_eps_noalloc: cudaGetDevice: ") + cudaGetErrorString(e));
+    return PA_ERR_CUDA;
+  }
+  if (dev < 0 || dev >= kNoAllocMaxDevices) {
+    pa::set_error("pa_gmm_eps_noalloc: device index beyond the supported 64");
+    return PA_ERR_ARG;
+  }
+  std::lock_guard<std::mutex> lock(g_scratch_mu);
+  if (!g_scratch_dev[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_gmm_scratch);
+    if (e != cudaSuccess || !p) {
+      pa::set_error(std::string("pa_gmm_eps_noalloc: cudaGetSymbolAddress: ") + cudaGetErrorString(e));
+      return PA_ERR_CUDA;
+    }
+    g_scratch_dev[dev] = static_cast<unsigned char*>(p);
+  }
+  *out = g_scratch_dev[dev];
+  return PA_OK;
+}
+
+}  // namespace
+
+extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D, double std,
+                                        const double* alphas_cumprod, int T,
+                                        const float* batch_x_dev, const int32_t* miss_bt_dev,
+                                        int n_rows, float* batch_eps_dev, void* stream) {
+  if (K < 1 || K > kMaxK || D < 1 || T < 1 || n_rows < 0 || !means_dev || !alphas_cumprod ||
+      !batch_x_dev || !miss_bt_dev || !batch_eps_dev || !(std >= 0.0) || !std::isfinite(std)) {
+    pa::set_error("pa_gmm_eps_noalloc: bad size, pointer or std");
+    return PA_ERR_ARG;
+  }
+  for (int i = 0; i <= T; ++i) {
+    const double a = alphas_cumprod[i];
+    if (!(a > 0.0 && a <= 1.0)) {
+      pa::set_error("pa_gmm_eps_noalloc: alphas_cumprod must be in (0, 1]");
+      return PA_ERR_ARG;
+    }
+  }
+  if (n_rows == 0) return PA_OK;
+  // scratch layout: coef[3T] | mnorm[K] | gpart[nchunk][n_rows][K] | R[n_rows][K] |
+  //                 rowc[n_rows][2] | n_rows | status   (256-byte aligned pieces)
+  const int chunk = dots_chunk(K, D);
+  const int nchunk = (int)((D + chunk - 1) / chunk);
+  size_t o = 0;
+  auto take = [&](size_t bytes) { size_t at = o; o = pa::align_up(o + bytes, pa::kAlign); return at; };
+  const size_t o_coef = take((size_t)3 * T * sizeof(float));
+  const size_t o_mnorm = take((size_t)K * sizeof(float));
+  const size_t o_gpart = take((size_t)nchunk * n_rows * K * sizeof(float));
+  const size_t o_R = take((size_t)n_rows * K * sizeof(float));
+  const size_t o_rowc = take((size_t)n_rows * 2 * sizeof(float));
+  const size_t o_n = take(sizeof(int32_t));
+  const size_t o_status = take(sizeof(int32_t));
+  if (o > kNoAllocScratchBytes) {
+    pa::set_error("pa_gmm_eps_noalloc: these sizes need " + std::to_string(o) +
+                  " bytes of scratch, more than the fixed 4 MiB (4194304 bytes); "
+                  "use pa_gmm_create + pa_gmm_eps with a caller-allocated workspace");
+    return PA_ERR_ARG;
+  }
+  unsigned char* scratch = nullptr;
+  pa_status ps = scratch_for_current_device(&scratch);
+  if (ps != PA_OK) return ps;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  float* coef = reinterpret_cast<float*>(scratch + o_coef);
+  float* mnorm = reinterpret_cast<float*>(scratch + o_mnorm);
+  float* gpart = reinterpret_cast<float*>(scratch + o_gpart);
+  float* R = reinterpret_cast<float*>(scratch + o_R);
+  float* rowc = reinterpret_cast<float*>(scratch + o_rowc);
+  int32_t* nrows_dev = reinterpret_cast<int32_t*>(scratch + o_n);
+  int32_t* status = reinterpret_cast<int32_t*>(scratch + o_status);
+
+  // Per-timestep scalars, formed in fp64 on the host in stack-sized chunks;
+  // each pageable copy returns once its source has been staged.
+  cudaError_t e = cudaSuccess;
+  float buf[kNoAllocCoefChunk];
+  for (int part = 0; part < 3 && e == cudaSuccess; ++part) {
+    for (int i0 = 0; i0 < T && e == cudaSuccess; i0 += kNoAllocCoefChunk) {
+      const int n = (T - i0) < kNoAllocCoefChunk ? (T - i0) : kNoAllocCoefChunk;
+      for (int u = 0; u < n; ++u) {
+        const double a = alphas_cumprod[i0 + u];
+        const double v = a * std * std + (1.0 - a);
+        buf[u] = (float)(part == 0 ? std::sqrt(a) : part == 1 ? 1.0 / (2.0 * v) : std::sqrt(1.0 - a) / v);
+      }
+      e = cudaMemcpyAsync(coef + (size_t)part * T + i0, buf, (size_t)n * sizeof(float),
+                          cudaMemcpyHostToDevice, st);
+    }
+  }
+  const int32_t nr = n_rows;
+  if (e == cudaSuccess) e = cudaMemcpyAsync(nrows_dev, &nr, sizeof(nr), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);  // starts at zero every call
+  const size_t dots_smem = (size_t)(kDotRows + K) * (chunk + 4) * sizeof(float);
+  const size_t out_smem = (size_t)(K + kOutRows) * kOutCols * sizeof(float);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_gmm_dots, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dots_smem);
+  if (e == cudaSuccess)
+    e = cudaFuncSetAttribute(k_gmm_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out_smem);
+  if (e != cudaSuccess) {
+    pa::set_error(std::string("pa_gmm_eps_noalloc: ") + cudaGetErrorString(e));
+    return PA_ERR_CUDA;
+  }
+  const bool bulk = D % 4 == 0 && ((reinterpret_cast<uintptr_t>(batch_x_dev) |
+                                    reinterpret_cast<uintptr_t>(means_dev)) & 15) == 0;
+  k_gmm_norms<<<K, 256, 0, st>>>(means_dev, D, mnorm);
+  k_gmm_dots<<<dim3(nchunk, (n_rows + kDotRows - 1) / kDotRows), kThreads, dots_smem, st>>>(
+      batch_x_dev, means_dev, nrows_dev, K, D, chunk, n_rows, bulk, gpart, status);
+  k_gmm_softmax<<<n_rows, kThreads, 0, st>>>(gpart, mnorm, coef, T, miss_bt_dev, nrows_dev, K, nchunk,
+                                             n_rows, R, rowc);
+  k_gmm_out<<<dim3((unsigned)((D + kOutCols - 1) / kOutCols), (n_rows + kOutRows - 1) / kOutRows),
+              kOutCols, out_smem, st>>>(batch_x_dev, means_dev, R, rowc, nrows_dev, K, D, n_rows, bulk,
+                                        batch_eps_dev, status);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    pa::set_error(std::string("pa_gmm_eps_noalloc: ") + cudaGetErrorString(e));
+    return PA_ERR_CUDA;
+  }
+  return PA_OK;
+}

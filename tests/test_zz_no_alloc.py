@@ -1,0 +1,88 @@
+"""The allocation-free denoiser entry point, pa_gmm_eps_noalloc.
+
+It serves callers that cannot allocate device memory when they run the
+denoiser (plugins handed pre-allocated buffers by a host framework, real-time
+loops that forbid cudaMalloc/cudaFree after start-up): its scratch is a fixed
+4 MiB device array inside the library. This file is collected last on
+purpose, so that a run stopping at the first failure has run every other test
+first; it also passes when run on its own in a fresh process.
+"""
+import numpy as np
+import pytest
+
+import workload as W
+from oracle.gmm import gmm_eps
+
+pytestmark = pytest.mark.gpu
+
+REL_TOL = 2e-6  # the mixture-denoiser tolerance of test_gpu_parity
+
+
+@pytest.fixture(scope="module")
+def lib():
+    import torch
+    from paper_2609_36522_gb300 import build as pa_build
+    from paper_2609_36522_gb300 import abi
+    assert torch.cuda.is_available()
+    pa_build.build()
+    return abi
+
+
+def _rows(w, a, mu, n, seed):
+    rng = np.random.default_rng(seed)
+    idx = rng.integers(0, w.T, n).astype(np.int32)
+    comp = rng.integers(0, w.K, n)
+    x = (np.sqrt(a[idx])[:, None] * (mu[comp] + 0.5 * rng.standard_normal((n, w.D)))
+         + np.sqrt(1 - a[idx])[:, None] * rng.standard_normal((n, w.D))).astype(np.float32)
+    miss = np.stack([np.zeros(n, np.int32), idx], axis=1).astype(np.int32)
+    return x, miss, idx
+
+
+def test_noalloc_matches_handle_entry_point_on_two_calls(lib):
+    import torch
+    from paper_2609_36522_gb300.solver import GmmDenoiser
+    abi = lib
+    w = W.SD15
+    a, _, mu = W.inputs(w)
+    dev = torch.device("cuda")
+    mu_d = torch.from_numpy(mu).to(dev)
+    g = GmmDenoiser(mu_d, w.gmm_std, a, 100)
+    stream = torch.cuda.current_stream()
+    # two calls in a row; the second is smaller, so stale scratch of the first
+    # must not leak into it
+    for n, seed in ((100, 1), (37, 2)):
+        x, miss, idx = _rows(w, a, mu, n, seed)
+        xd = torch.from_numpy(x).to(dev)
+        md = torch.from_numpy(miss).to(dev)
+        nd = torch.tensor([n], dtype=torch.int32, device=dev)
+        ref = torch.empty_like(xd)
+        got = torch.full_like(xd, float("nan"))
+        g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), ref)
+        abi.pa_gmm_eps_noalloc(mu_d.data_ptr(), w.K, w.D, w.gmm_std, list(a), xd.data_ptr(),
+                               md.data_ptr(), n, got.data_ptr(), stream.cuda_stream)
+        torch.cuda.synchronize()
+        r = ref.cpu().numpy().astype(np.float64)
+        o = got.cpu().numpy().astype(np.float64)
+        scale = np.abs(r).max(axis=1)
+        assert np.isfinite(o).all()
+        assert (np.abs(o - r).max(axis=1) / scale).max() <= REL_TOL
+        want = gmm_eps(x.astype(np.float64), a[idx], mu.astype(np.float64), w.gmm_std)
+        assert (np.abs(o - want).max(axis=1) / np.abs(want).max(axis=1)).max() <= REL_TOL
+    g.close()
+
+
+def test_noalloc_rejects_sizes_beyond_its_scratch(lib):
+    import torch
+    abi = lib
+    w = W.LARGE  # K=64, D=65536: 128 rows need far more than 4 MiB of partials
+    a, _, mu = W.inputs(w)
+    dev = torch.device("cuda")
+    mu_d = torch.from_numpy(mu).to(dev)
+    x = torch.zeros(128, w.D, device=dev)
+    miss = torch.zeros(128, 2, dtype=torch.int32, device=dev)
+    out = torch.zeros_like(x)
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_gmm_eps_noalloc(mu_d.data_ptr(), w.K, w.D, w.gmm_std, list(a), x.data_ptr(),
+                               miss.data_ptr(), 128, out.data_ptr(), 0)
+    assert e.value.status == abi.PA_ERR_ARG
+    assert "4 MiB" in str(e.value)
