@@ -211,64 +211,74 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 }
 
 // ---------------------------------------------------------------------------
-// Decision kernel (one CTA of 1024 threads):
-//  1. finish the reductions: err[b][j] (Eq. 2) and delta of timestep t+j+1
-//     (Eq. 4), summing the chunk partials in a fixed order (deterministic);
+// Decision kernel, one launch of many CTAs:
+//  1. every CTA finishes some of the reductions: one warp per (quantity, b, j)
+//     sums the chunk partials of err[b][j] (Eq. 2) or of the distance of
+//     timestep t+j+1 (Eq. 4) in a fixed order (deterministic), to red_*;
+//  the CTA that finishes last (atomic ticket after a fence; nobody waits) then
 //  2. per trajectory: stride = min(p, 1 + #leading err_j <= tol), advance
 //     t, shrink p = min(P, T - t), frontier e = old t + p, done at t = T;
-//  3. plan the next iteration: a timestep of the new window with a cache
+//  3. plans the next iteration: a timestep of the new window with a cache
 //     entry (i < e) hits iff delta < tau_cache (strict, Eq. 5), everything
 //     else misses; misses are compacted trajectory-major into miss_bt with a
 //     block-wide prefix sum, and rank[b][j] records each miss's batch row.
-constexpr int kDecideThreads = 1024;
-constexpr int kDecideSmemPairs = 6144;  // (b, j) pairs whose reductions stay in shared memory
+constexpr int kDecideThreads = 256;
+constexpr int kDecideSmemPairs = 6144;  // (b, j) pairs whose reductions are staged in shared memory
 
 __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
   __shared__ int s_t[kMaxBatch], s_p[kMaxBatch], s_e[kMaxBatch];
   __shared__ int s_tn[kMaxBatch], s_pn[kMaxBatch], s_m[kMaxBatch], s_h1[kMaxBatch];
+  __shared__ int s_om[kMaxBatch], s_oh1[kMaxBatch];
   __shared__ int s_warp[kDecideThreads / 32];
-  __shared__ int s_total, s_active, s_iter;
+  __shared__ int s_total, s_active, s_iter, s_last;
   extern __shared__ float s_red[];  // [2][B*P] when B*P <= kDecideSmemPairs
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kDecideThreads / 32;
   const int B = d.B, P = d.P, T = d.T;
-  const bool in_smem = B * P <= kDecideSmemPairs;
-  float* red_e = in_smem ? s_red : d.red_err;
-  float* red_d = in_smem ? s_red + B * P : d.red_del;
+  const int npair = B * P;
 
-  // Every load of this prologue is independent of the others (one round trip):
-  // counters, window bookkeeping, and the chunk partials of every (b, j).
+  // 1. reductions, one warp per item (positions beyond a trajectory's window
+  // are reduced too; their values are never used)
+  const int item = blockIdx.x * nwarps + warp;
+  if (item < 2 * npair) {
+    const int which = item / npair, pr = item % npair;
+    const float* src = (which ? d.part_del : d.part_err) + (int64_t)pr * nchunk;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+    for (int c = lane, u = 0; c < nchunk; c += 32, u = (u + 1) & 3) acc[u] += src[c];
+    float v = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+    v = warp_sum(v);
+    if (lane == 0) (which ? d.red_del : d.red_err)[pr] = v / (float)d.D;
+  }
+  __syncthreads();
   if (tid == 0) {
+    __threadfence();
+    const unsigned int k = atomicAdd(&d.ctl->ticket, 1u);
+    s_last = (k == gridDim.x - 1);
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();  // the other CTAs' reductions are visible from here on
+  const bool in_smem = npair <= kDecideSmemPairs;
+  float* red_e = in_smem ? s_red : d.red_err;
+  float* red_d = in_smem ? s_red + npair : d.red_del;
+  if (tid == 0) {
+    d.ctl->ticket = 0u;  // ready for the next launch
     s_active = d.ctl->n_active;
     s_iter = d.ctl->iter;
   }
   for (int b = tid; b < B; b += kDecideThreads) {
     const Traj tr = d.traj[b];
     s_t[b] = tr.t; s_p[b] = tr.p; s_e[b] = tr.e;
+    s_om[b] = tr.m; s_oh1[b] = tr.h1;
     s_m[b] = 0;
     s_h1[b] = 0;
   }
-  // 1. reductions: one thread per (quantity, b, j) sums the chunk partials in
-  // a fixed order (four interleaved accumulators), so every partial load of
-  // the kernel is issued in the first round. Positions beyond a trajectory's
-  // window are reduced too (their values are never used).
-  const int npair = B * P;
-  for (int q = tid; q < 2 * npair; q += kDecideThreads) {
-    const int which = q / npair, pr = q % npair;
-    const float* src = (which ? d.part_del : d.part_err) + (int64_t)pr * nchunk;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    int c = 0;
-#pragma unroll 8
-    for (; c + 4 <= nchunk; c += 4) {
-      acc[0] += src[c];
-      acc[1] += src[c + 1];
-      acc[2] += src[c + 2];
-      acc[3] += src[c + 3];
+  if (in_smem) {
+    for (int q = tid; q < npair; q += kDecideThreads) {
+      s_red[q] = __ldcg(d.red_err + q);
+      s_red[npair + q] = __ldcg(d.red_del + q);
     }
-    for (; c < nchunk; ++c) acc[0] += src[c];
-    const float v = ((acc[0] + acc[1]) + (acc[2] + acc[3])) / (float)d.D;
-    (which ? red_d : red_e)[pr] = v;
-    if (in_smem) (which ? d.red_del : d.red_err)[pr] = v;  // global copy for pa_last_reductions
   }
   __syncthreads();
   if (s_active == 0) return;  // finished: iterating further is a no-op
@@ -301,10 +311,9 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
       const int tn = t + stride;
       s_tn[b] = tn;
       s_pn[b] = min(P, T - tn);
-      const Traj old = d.traj[b];
       int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
-      lg[0] = t; lg[1] = p; lg[2] = old.m; lg[3] = stride;
-      lg[4] = old.e; lg[5] = old.h1; lg[6] = 0; lg[7] = 0;
+      lg[0] = t; lg[1] = p; lg[2] = s_om[b]; lg[3] = stride;
+      lg[4] = s_e[b]; lg[5] = s_oh1[b]; lg[6] = 0; lg[7] = 0;
     }
   }
   __syncthreads();
@@ -334,14 +343,15 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
   if (lane == 31) s_warp[warp] = incl;
   __syncthreads();
   if (warp == 0) {
-    int w = s_warp[lane];
+    static_assert(nwarps <= 32, "one warp scans the warp totals");
+    const int w = lane < nwarps ? s_warp[lane] : 0;
     int wi = w;
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
       const int v = __shfl_up_sync(0xffffffffu, wi, o);
       if (lane >= o) wi += v;
     }
-    s_warp[lane] = wi - w;  // exclusive
+    if (lane < nwarps) s_warp[lane] = wi - w;  // exclusive
     if (lane == 31) s_total = wi;
   }
   __syncthreads();
@@ -425,7 +435,9 @@ cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream
 cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st) {
   const int pairs = d.B * d.P;
   const size_t smem = pairs <= kDecideSmemPairs ? (size_t)2 * pairs * sizeof(float) : 0;
-  k_decide<<<1, kDecideThreads, smem, st>>>(d, nchunk);
+  const int nwarps = kDecideThreads / 32;
+  const int grid = (2 * pairs + nwarps - 1) / nwarps;
+  k_decide<<<grid, kDecideThreads, smem, st>>>(d, nchunk);
   return cudaGetLastError();
 }
 

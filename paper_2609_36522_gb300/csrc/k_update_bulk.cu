@@ -119,8 +119,11 @@ struct TileShape {
 };
 
 // nbuf tile buffers (<= 16); when nbuf >= ceil(p / TW) every copy of the
-// window is in flight right after the prologue.
-template <int V, int NW, int S>
+// window is in flight right after the prologue. CLUSTER: combine the strip
+// partials of kCluster CTAs through distributed shared memory (else one
+// partial per strip). WAIT_ALL: every thread polls the tile's mbarrier (else
+// warp 0 polls and the CTA barrier releases the others).
+template <int V, int NW, int S, bool CLUSTER, bool WAIT_ALL>
 __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __restrict__ beps,
                                                          int nstrip, int nbuf, uint32_t wait_limit) {
   using Sh = TileShape<V, NW, S>;
@@ -245,10 +248,14 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   for (int k = 0; k < ntile; ++k) {
     const int bi = k % nbuf;
     const uint32_t parity = (uint32_t)((k / nbuf) & 1);
-    if (!my_fail && !aborted && !mbar_wait_bounded(&bar[bi], parity, wait_limit)) {
+    // warp 0 watches the tile's mbarrier; the other warps sleep at the CTA
+    // barrier instead of polling (the barrier orders the landed data for them)
+    if ((WAIT_ALL || warp == 0) && !my_fail && !aborted &&
+        !mbar_wait_bounded(&bar[bi], parity, wait_limit)) {
       atomicCAS(&d.ctl->status, kDevOk, kDevTimeout);
       my_fail = 1;
     }
+    if (!WAIT_ALL) __syncthreads();
     const float* buf = s_tile + (size_t)bi * Sh::kTileFloats;
     const int tb = k * TW;
     const int q0 = warp * S;
@@ -315,6 +322,13 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
     __syncthreads();  // B: carries published
 
     // phase 2: new states, their Eq. 2 error and next-iteration Eq. 4 distance
+    float ch[V], cl[V];
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const size_t o = ((size_t)warp * SEG + lane * V + v) * 2;
+      ch[v] = s_car[o];
+      cl[v] = s_car[o + 1];
+    }
 #pragma unroll
     for (int s = 0; s < S; ++s) {
       const int qi = q0 + s;
@@ -325,8 +339,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
         Vec<V> xn;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-          const size_t o = ((size_t)warp * SEG + lane * V + v) * 2;
-          float h = s_car[o], l = s_car[o + 1];
+          float h = ch[v], l = cl[v];
           acc_add2(h, l, phi[s][v], plo[s][v]);
           xn.a[v] = h + l;
           const float df = xn.a[v] - xo_s[s].a[v];
@@ -382,31 +395,43 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
     for (int k = (issued > nbuf ? issued - nbuf : 0); k < issued; ++k)
       mbar_wait_bounded(&bar[k % nbuf], (uint32_t)((k / nbuf) & 1), kDrainLimit);
   }
-  // Combine the strips of this cluster: CTA rank q sums positions j = q mod
-  // kCluster over the cluster's CTAs in rank order (distributed shared
-  // memory) and writes part[b][j][cluster]. The second cluster barrier keeps
-  // every CTA's shared memory alive until its peers have read it.
-  cg::cluster_group cluster = cg::this_cluster();
-  cluster.sync();
-  const int rank = (int)cluster.block_rank();
-  const int nclus = gridDim.x / kCluster;
-  const int64_t cbase = (int64_t)b * P * nclus + blockIdx.x / kCluster;
-  for (int q2 = tid; q2 < 2 * p; q2 += NW * 32) {
-    const int which = q2 / p, j = q2 % p;
-    if (j % kCluster != rank) continue;
-    float sum = 0.f;
+  if constexpr (CLUSTER) {
+    // Combine the strips of this cluster: CTA rank q sums positions j = q mod
+    // kCluster over the cluster's CTAs in rank order (distributed shared
+    // memory) and writes part[b][j][cluster]. The second cluster barrier keeps
+    // every CTA's shared memory alive until its peers have read it.
+    cg::cluster_group cluster = cg::this_cluster();
+    cluster.sync();
+    const int rank = (int)cluster.block_rank();
+    const int nclus = gridDim.x / kCluster;
+    const int64_t cbase = (int64_t)b * P * nclus + blockIdx.x / kCluster;
+    for (int q2 = tid; q2 < 2 * p; q2 += NW * 32) {
+      const int which = q2 / p, j = q2 % p;
+      if (j % kCluster != rank) continue;
+      float sum = 0.f;
 #pragma unroll
-    for (int r = 0; r < kCluster; ++r) sum += cluster.map_shared_rank(s_pos, r)[which * P + j];
-    (which == 0 ? d.part_err : d.part_del)[cbase + (int64_t)j * nclus] = sum;
+      for (int r = 0; r < kCluster; ++r) sum += cluster.map_shared_rank(s_pos, r)[which * P + j];
+      (which == 0 ? d.part_err : d.part_del)[cbase + (int64_t)j * nclus] = sum;
+    }
+    cluster.sync();
+  } else {
+    // one partial per strip and position
+    __syncthreads();
+    if (active) {
+      const int64_t pbase = (int64_t)b * P * nstrip + strip;
+      for (int q2 = tid; q2 < 2 * p; q2 += NW * 32) {
+        const int which = q2 / p, j = q2 % p;
+        (which == 0 ? d.part_err : d.part_del)[pbase + (int64_t)j * nstrip] = s_pos[which * P + j];
+      }
+    }
   }
-  cluster.sync();
 }
 
 // Shared memory budget per CTA for the tile buffers: enough for the whole
 // window when it fits, so every copy is in flight from the start.
 constexpr size_t kSmemBudget = 112 * 1024;
 
-template <int V, int NW, int S>
+template <int V, int NW, int S, bool CLUSTER, bool WAIT_ALL>
 cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
   using Sh = TileShape<V, NW, S>;
   const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
@@ -416,7 +441,7 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
   while (nbuf > 2 && fixed + (size_t)nbuf * Sh::kTileBytes > kSmemBudget) --nbuf;
   if (nbuf < 1) nbuf = 1;
   const size_t smem = Sh::smem_bytes(d.P, nbuf);
-  auto kern = k_update_tile<V, NW, S>;
+  auto kern = k_update_tile<V, NW, S, CLUSTER, WAIT_ALL>;
   // largest dynamic shared memory granted so far, per device and instantiation
   static size_t configured[64] = {};
   int dev = 0;
@@ -427,8 +452,8 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) configured[dev] = smem;
   }
-  const int gx = (nstrip + kCluster - 1) / kCluster * kCluster;
-  *nchunk_out = gx / kCluster;  // one partial per cluster and position
+  const int gx = CLUSTER ? (nstrip + kCluster - 1) / kCluster * kCluster : nstrip;
+  *nchunk_out = CLUSTER ? gx / kCluster : nstrip;  // partials per position
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3(gx, d.B, 1);
   cfg.blockDim = dim3(NW * 32, 1, 1);
@@ -436,11 +461,11 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
   cfg.stream = st;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = kCluster;
+  attr[0].val.clusterDim.x = CLUSTER ? kCluster : 1;
   attr[0].val.clusterDim.y = 1;
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = CLUSTER ? 1 : 0;
   return cudaLaunchKernelEx(&cfg, kern, d, beps, nstrip, nbuf, d.wait_limit);
 }
 
@@ -454,17 +479,17 @@ bool update_bulk_supported(const Dev& d, const float* batch_eps) {
 
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
   switch (d.bulk_cfg) {
-    case 0: return launch_tile<2, 8, 4>(d, batch_eps, st, nchunk_out);
-    case 1: return launch_tile<1, 8, 4>(d, batch_eps, st, nchunk_out);
-    case 2: return launch_tile<1, 4, 8>(d, batch_eps, st, nchunk_out);
-    case 3: return launch_tile<2, 4, 8>(d, batch_eps, st, nchunk_out);
-    case 4: return launch_tile<2, 8, 2>(d, batch_eps, st, nchunk_out);
-    case 5: return launch_tile<2, 4, 4>(d, batch_eps, st, nchunk_out);
-    case 6: return launch_tile<1, 8, 8>(d, batch_eps, st, nchunk_out);
-    case 7: return launch_tile<2, 8, 8>(d, batch_eps, st, nchunk_out);
-    case 8: return launch_tile<1, 16, 2>(d, batch_eps, st, nchunk_out);
-    case 9: return launch_tile<2, 16, 2>(d, batch_eps, st, nchunk_out);
-    default: return launch_tile<2, 8, 4>(d, batch_eps, st, nchunk_out);
+    case 0: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 1: return launch_tile<2, 8, 4, false, false>(d, batch_eps, st, nchunk_out);
+    case 2: return launch_tile<2, 8, 4, true, true>(d, batch_eps, st, nchunk_out);
+    case 3: return launch_tile<2, 8, 4, true, false>(d, batch_eps, st, nchunk_out);
+    case 4: return launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
+    case 5: return launch_tile<1, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 6: return launch_tile<2, 8, 2, false, true>(d, batch_eps, st, nchunk_out);
+    case 7: return launch_tile<2, 16, 2, false, true>(d, batch_eps, st, nchunk_out);
+    case 8: return launch_tile<2, 8, 8, false, true>(d, batch_eps, st, nchunk_out);
+    case 9: return launch_tile<2, 4, 4, false, true>(d, batch_eps, st, nchunk_out);
+    default: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
   }
 }
 

@@ -41,6 +41,8 @@ struct Ctl {
   int32_t status;     // kDev* code
   long long nfe;
   long long hits;
+  uint32_t ticket;    // CTAs of the decision kernel that finished their reductions
+  int32_t pad;
 };
 
 struct Layout {
