@@ -34,6 +34,8 @@ void set_error(const std::string& msg);  // pa_solver.cpp
 
 namespace {
 
+using pa::pdl_trigger;
+using pa::pdl_wait;
 using pa::bulk_g2s;
 using pa::fence_barrier_init;
 using pa::mbar_arrive_expect_tx;
@@ -159,8 +161,9 @@ __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__
     if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
   }
   __syncthreads();
+  stage_rows(ms, ld, mu, D, c0, ncol, K, bulk, &bar);  // the means do not depend on the predecessor
+  pdl_wait();  // the rows come from the gather (or the caller) just before
   stage_rows(xs, ld, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
-  stage_rows(ms, ld, mu, D, c0, ncol, K, bulk, &bar);
   const bool ok = wait_staged(bulk, &bar, status);
   __syncthreads();
   if (!ok) return;
@@ -208,12 +211,13 @@ __global__ void __launch_bounds__(kThreads) k_gmm_softmax(const float* __restric
   while (KB < K) KB <<= 1;
   const int G = kThreads / KB;
   const int k = threadIdx.x % KB, g = threadIdx.x / KB;
+  const int i = miss_bt[2 * r + 1];
+  const float sa = coef[i], q = coef[T + i], ac = coef[2 * T + i];
+  pdl_wait();  // the partials come from the dot-product kernel
   float part = 0.f;
   if (k < K)
     for (int s = g; s < nchunk; s += G) part += gpart[((int64_t)s * max_rows + r) * K + k];
   s_part[threadIdx.x] = part;
-  const int i = miss_bt[2 * r + 1];
-  const float sa = coef[i], q = coef[T + i], ac = coef[2 * T + i];
   __syncthreads();
   if (threadIdx.x < K) {
     float dot = 0.f;
@@ -264,8 +268,10 @@ __global__ void __launch_bounds__(kOutCols) k_gmm_out(const float* __restrict__ 
     if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
   }
   __syncthreads();
+  // the means and the rows (written two kernels back) do not depend on the predecessor
   stage_rows(ms, kOutCols, mu, D, c0, ncol, K, bulk, &bar);
   stage_rows(xs, kOutCols, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
+  pdl_wait();  // the responsibilities come from the softmax kernel
   for (int q = threadIdx.x; q < nr * K; q += kOutCols) s_r[q] = R[(int64_t)r0 * K + q];
   for (int q = threadIdx.x; q < nr * 2; q += kOutCols) s_c[q] = rowc[2 * r0 + q];
   const bool ok = wait_staged(bulk, &bar, status);
@@ -373,15 +379,20 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
                                        reinterpret_cast<uintptr_t>(g->means)) & 15) == 0;
   const size_t dots_smem = (size_t)(kDotRows + g->K) * (L.chunk + 4) * sizeof(float);
   const size_t out_smem = (size_t)(g->K + kOutRows) * kOutCols * sizeof(float);
-  k_gmm_dots<<<dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows), kThreads, dots_smem, g->st>>>(
-      batch_x_dev, g->means, n_rows_dev, g->K, g->D, L.chunk, g->max_rows, bulk, gpart, status);
-  k_gmm_softmax<<<g->max_rows, kThreads, 0, g->st>>>(gpart, mnorm, coef, g->T, miss_bt_dev, n_rows_dev,
-                                                     g->K, L.nchunk, g->max_rows, R, rowc);
-  k_gmm_out<<<dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
-              kOutCols, out_smem, g->st>>>(batch_x_dev, g->means, R, rowc, n_rows_dev, g->K, g->D,
-                                            g->max_rows, bulk, batch_eps_dev, status);
+  cudaError_t e = pa::launch_ex(k_gmm_dots, dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows),
+                                dim3(kThreads), dots_smem, g->st, 0, batch_x_dev, g->means, n_rows_dev, g->K,
+                                g->D, L.chunk, g->max_rows, bulk, gpart, status);
+  if (e == cudaSuccess)
+    e = pa::launch_ex(k_gmm_softmax, dim3(g->max_rows), dim3(kThreads), 0, g->st, 0, (const float*)gpart,
+                      (const float*)mnorm, (const float*)coef, g->T, miss_bt_dev, n_rows_dev, g->K, L.nchunk,
+                      g->max_rows, R, rowc);
+  if (e == cudaSuccess)
+    e = pa::launch_ex(k_gmm_out,
+                      dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
+                      dim3(kOutCols), out_smem, g->st, 0, batch_x_dev, g->means, (const float*)R,
+                      (const float*)rowc, n_rows_dev, g->K, g->D, g->max_rows, bulk, batch_eps_dev, status);
   g->launches += 3;
-  const cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_eps: ") + cudaGetErrorString(e));
     return PA_ERR_CUDA;

@@ -60,6 +60,7 @@ __global__ void k_init_plan(Dev d) {
 // state e, the value every new tail state was initialised to.
 template <int VEC>
 __global__ void __launch_bounds__(256) k_gather(Dev d) {
+  pdl_wait();  // everything read here comes from the decision kernel
   const int n = d.ctl->n_miss;
   const int64_t nvec = d.D / VEC;
   for (int r = blockIdx.y; r < n; r += gridDim.y) {
@@ -130,6 +131,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
                                                              int nchunk) {
   extern __shared__ float red[];  // [2][nwarps][P]
   const int b = blockIdx.y;
+  pdl_wait();
   const Traj tr = d.traj[b];
   if (tr.p == 0) return;
   const int t = tr.t, p = tr.p, e = tr.e, P = d.P;
@@ -237,6 +239,7 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
   const int B = d.B, P = d.P, T = d.T;
   const int npair = B * P;
 
+  pdl_wait();  // the partials come from the update kernel
   // 1. reductions, one warp per item (positions beyond a trajectory's window
   // are reduced too; their values are never used)
   const int item = blockIdx.x * nwarps + warp;
@@ -408,11 +411,11 @@ cudaError_t launch_gather(const Dev& d, cudaStream_t st) {
     const int64_t nvec = d.D / 4;
     const int64_t want = (nvec + 255) / 256;
     const int gx = (int)(want < 64 ? want : 64);
-    k_gather<4><<<dim3(gx, rows), 256, 0, st>>>(d);
+    return launch_ex(k_gather<4>, dim3(gx, rows), dim3(256), 0, st, 0, d);
   } else {
     const int64_t want = (d.D + 255) / 256;
     const int gx = (int)(want < 256 ? want : 256);
-    k_gather<1><<<dim3(gx, rows), 256, 0, st>>>(d);
+    return launch_ex(k_gather<1>, dim3(gx, rows), dim3(256), 0, st, 0, d);
   }
   return cudaGetLastError();
 }
@@ -423,11 +426,13 @@ cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream
   if (d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0) {
     const int nchunk = (int)((d.D + kPlainThreads * 4 - 1) / (kPlainThreads * 4));
     *nchunk_out = nchunk;
-    k_update_plain<4><<<dim3(nchunk, d.B), kPlainThreads, smem, st>>>(d, batch_eps, nchunk);
+    return launch_ex(k_update_plain<4>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps,
+                     nchunk);
   } else {
     const int nchunk = (int)((d.D + kPlainThreads - 1) / kPlainThreads);
     *nchunk_out = nchunk;
-    k_update_plain<1><<<dim3(nchunk, d.B), kPlainThreads, smem, st>>>(d, batch_eps, nchunk);
+    return launch_ex(k_update_plain<1>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps,
+                     nchunk);
   }
   return cudaGetLastError();
 }
@@ -437,7 +442,7 @@ cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st) {
   const size_t smem = pairs <= kDecideSmemPairs ? (size_t)2 * pairs * sizeof(float) : 0;
   const int nwarps = kDecideThreads / 32;
   const int grid = (2 * pairs + nwarps - 1) / nwarps;
-  k_decide<<<grid, kDecideThreads, smem, st>>>(d, nchunk);
+  return launch_ex(k_decide, dim3(grid), dim3(kDecideThreads), smem, st, 0, d, nchunk);
   return cudaGetLastError();
 }
 

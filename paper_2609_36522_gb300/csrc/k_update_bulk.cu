@@ -178,6 +178,9 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
     }
   }
   __syncthreads();
+  // Everything above came from the decision kernel and earlier; the eps rows
+  // below come from the denoiser that ran just before this kernel.
+  pdl_wait();
 
   const int strip = blockIdx.x;          // the grid is padded to whole clusters
   const bool active = strip < nstrip;
@@ -427,6 +430,247 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   }
 }
 
+// ---------------------------------------------------------------------------
+// Segment-per-warp Picard update: used when the whole window of a strip fits
+// in shared memory. Warp w owns the contiguous window positions
+// [w*L, min(p, (w+1)*L)), L = ceil(p / NW), and issues their bulk copies
+// itself (one mbarrier per warp). Phase 1 forms the compensated sum of the
+// segment's drifts; after one CTA barrier every warp builds its carry
+// x_t + sum of the earlier segments' totals and walks its segment again,
+// recomputing the drifts from shared memory, to produce the new states, the
+// Eq. 2 errors and the next-iteration Eq. 4 distances. Per-lane err/distance
+// values go through a transposed shared-memory buffer; after a second barrier
+// one thread per (quantity, position) sums its row into the strip partial.
+// Two CTA barriers per launch in all.
+template <int V, int NW>
+struct SegShape {
+  static constexpr int SEG = 32 * V;
+  __host__ __device__ static size_t meta_bytes(int P) { return ((size_t)P * 20 + 127) / 128 * 128; }
+  __host__ __device__ static size_t rows_bytes(int P) { return (size_t)P * 3 * SEG * sizeof(float); }
+  __host__ __device__ static size_t red_bytes(int P) { return ((size_t)2 * P * 33 * sizeof(float) + 127) / 128 * 128; }
+  static constexpr size_t kTotBytes = (size_t)NW * SEG * 2 * sizeof(float);
+  static constexpr size_t kBarBytes = 128;  // NW <= 16 mbarriers
+  __host__ __device__ static size_t smem_bytes(int P) {
+    return kBarBytes + meta_bytes(P) + kTotBytes + red_bytes(P) + rows_bytes(P);
+  }
+};
+
+template <int V, int NW>
+__global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __restrict__ beps, int nstrip,
+                                                        uint32_t wait_limit) {
+  using Sh = SegShape<V, NW>;
+  constexpr int SEG = Sh::SEG;
+  static_assert(NW <= 16, "one mbarrier per warp in a 128-byte area");
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int P = d.P;
+  const int b = blockIdx.y;
+  const int64_t D = d.D;
+
+  uint64_t* bar = reinterpret_cast<uint64_t*>(smem_raw);
+  unsigned char* q = smem_raw + Sh::kBarBytes;
+  int32_t* s_rank = reinterpret_cast<int32_t*>(q);
+  float* s_cm1 = reinterpret_cast<float*>(q + (size_t)P * 4);
+  float* s_ec = reinterpret_cast<float*>(q + (size_t)P * 8);
+  int32_t* s_slot = reinterpret_cast<int32_t*>(q + (size_t)P * 12);  // (t+j) mod P
+  int32_t* s_nxt = reinterpret_cast<int32_t*>(q + (size_t)P * 16);   // (t+j+1) mod (P+1)
+  q += Sh::meta_bytes(P);
+  float* s_tot = reinterpret_cast<float*>(q);   // [NW][SEG][2]
+  q += Sh::kTotBytes;
+  float* s_red = reinterpret_cast<float*>(q);   // [2][P][33]
+  q += Sh::red_bytes(P);
+  float* s_rows = reinterpret_cast<float*>(q);  // [P][3][SEG]: eps, old x_{i+1}, xhat_{i+1}
+
+  const Traj tr = d.traj[b];
+  const int n_miss = d.ctl->n_miss;
+  for (int j = tid; j < P; j += NW * 32) s_rank[j] = d.rank[b * P + j];
+  if (tr.p == 0) return;
+  const int t = tr.t, p = tr.p, e = tr.e;
+  for (int j = tid; j < p; j += NW * 32) {
+    s_slot[j] = (t + j) % P;
+    s_nxt[j] = (t + j + 1) % (P + 1);
+    s_cm1[j] = d.cm1[t + j];
+    s_ec[j] = d.ecoef[t + j];
+  }
+  if (tid == 0) {
+    for (int k = 0; k < NW; ++k) mbar_init(&bar[k], 1);
+    fence_barrier_init();
+  }
+  __syncthreads();
+  for (int j = tid; j < p; j += NW * 32) {
+    if (s_rank[j] >= n_miss) {  // never expected: keep every copy in bounds and report it
+      atomicCAS(&d.ctl->status, kDevOk, kDevBadRank);
+      s_rank[j] = -1;
+    }
+  }
+  __syncthreads();
+  pdl_wait();  // the eps rows come from the denoiser that ran just before
+
+  const int strip = blockIdx.x;
+  const int64_t c0 = (int64_t)strip * SEG;
+  const int64_t ncol = (D - c0) < SEG ? (D - c0) : SEG;
+  const uint32_t seg_bytes = (uint32_t)ncol * sizeof(float);
+  const int64_t mycol = c0 + (int64_t)lane * V;
+  const bool live = mycol < D;
+  float* Xb = d.X + (int64_t)b * (P + 1) * D;
+  float* Xh = d.Xhat + (int64_t)b * P * D;
+  float* Eh = d.Ehat + (int64_t)b * P * D;
+  const int L = (p + NW - 1) / NW;
+  const int j0 = warp * L;
+  const int j1 = (j0 + L) < p ? (j0 + L) : p;
+
+  // this warp's copies: the whole byte count first, then one lane per position
+  {
+    uint32_t total = 0;
+    for (int j = j0 + lane; j < j1; j += 32) {
+      total += seg_bytes * (1u + ((t + j + 1 <= e) ? 1u : 0u) + (((j + 1 < p) && (s_rank[j + 1] < 0)) ? 1u : 0u));
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) total += __shfl_xor_sync(0xffffffffu, total, o);
+    if (lane == 0 && j0 < j1) mbar_arrive_expect_tx(&bar[warp], total);
+    __syncwarp();
+    for (int j = j0 + lane; j < j1; j += 32) {
+      float* rowp = s_rows + (size_t)j * 3 * SEG;
+      const int r = s_rank[j];
+      const float* src_eps = (r >= 0) ? beps + (int64_t)r * D + c0 : Eh + (int64_t)s_slot[j] * D + c0;
+      bulk_g2s(rowp, src_eps, seg_bytes, &bar[warp]);
+      if (t + j + 1 <= e) bulk_g2s(rowp + SEG, Xb + (int64_t)s_nxt[j] * D + c0, seg_bytes, &bar[warp]);
+      if ((j + 1 < p) && (s_rank[j + 1] < 0))
+        bulk_g2s(rowp + 2 * SEG, Xh + (int64_t)s_slot[j + 1] * D + c0, seg_bytes, &bar[warp]);
+    }
+  }
+  Vec<V> xstart{}, xfill{};
+  if (live) {
+    xstart = ldv<V>(Xb + (int64_t)(t % (P + 1)) * D + mycol);
+    xfill = ldv<V>(Xb + (int64_t)(e % (P + 1)) * D + mycol);
+  }
+  int my_fail = 0;
+  if (j0 < j1 && !mbar_wait_bounded(&bar[warp], 0, wait_limit)) my_fail = 1;
+  if (warp > 0 && j0 < j1 && !my_fail && !mbar_wait_bounded(&bar[warp - 1], 0, wait_limit)) my_fail = 1;
+  if (my_fail) atomicCAS(&d.ctl->status, kDevOk, kDevTimeout);
+
+  // old state at the segment's first position
+  Vec<V> xc0 = xfill;
+  if (j0 == 0) {
+    xc0 = xstart;
+  } else if (j0 < j1 && t + j0 <= e && live) {
+    xc0 = ldv<V>(s_rows + (size_t)(j0 - 1) * 3 * SEG + SEG + lane * V);
+  }
+
+  // phase 1: compensated sum of this segment's drifts
+  float rh[V], rl[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) { rh[v] = 0.f; rl[v] = 0.f; }
+  if (live) {
+    Vec<V> xc = xc0;
+    for (int j = j0; j < j1; ++j) {
+      const float* rowp = s_rows + (size_t)j * 3 * SEG;
+      const Vec<V> eps = ldv<V>(rowp + lane * V);
+      const float cm1 = s_cm1[j], ec = s_ec[j];
+#pragma unroll
+      for (int v = 0; v < V; ++v) acc_add(rh[v], rl[v], fmaf(cm1, xc.a[v], ec * eps.a[v]));
+      xc = (t + j + 1 <= e) ? ldv<V>(rowp + SEG + lane * V) : xfill;
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const size_t o = ((size_t)warp * SEG + lane * V + v) * 2;
+    s_tot[o] = rh[v];
+    s_tot[o + 1] = rl[v];
+  }
+  __syncthreads();
+
+  // phase 2: carry into this segment, then the new states, errors, distances
+  float ch[V], cl[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) { ch[v] = xstart.a[v]; cl[v] = 0.f; }
+  for (int w = 0; w < warp; ++w) {
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const size_t o = ((size_t)w * SEG + lane * V + v) * 2;
+      acc_add2(ch[v], cl[v], s_tot[o], s_tot[o + 1]);
+    }
+  }
+  {
+    Vec<V> xc = xc0;
+    for (int j = j0; j < j1; ++j) {
+      const float* rowp = s_rows + (size_t)j * 3 * SEG;
+      float ev = 0.f, dv = 0.f;
+      if (live) {
+        const Vec<V> eps = ldv<V>(rowp + lane * V);
+        if (s_rank[j] >= 0) {  // Eq. 7: the cache takes (x_i, eps_i) of a miss
+          const int64_t o = (int64_t)s_slot[j] * D + mycol;
+          stv<V>(Eh + o, eps);
+          stv<V>(Xh + o, xc);
+        }
+        const float cm1 = s_cm1[j], ec = s_ec[j];
+        const Vec<V> xo = (t + j + 1 <= e) ? ldv<V>(rowp + SEG + lane * V) : xfill;
+        Vec<V> xn;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          acc_add(ch[v], cl[v], fmaf(cm1, xc.a[v], ec * eps.a[v]));
+          xn.a[v] = ch[v] + cl[v];
+          const float df = xn.a[v] - xo.a[v];
+          ev = fmaf(df, df, ev);
+        }
+        stv<V>(Xb + (int64_t)s_nxt[j] * D + mycol, xn);
+        if (j + 1 < p) {
+          const Vec<V> xh = (s_rank[j + 1] < 0) ? ldv<V>(rowp + 2 * SEG + lane * V) : xo;
+#pragma unroll
+          for (int v = 0; v < V; ++v) dv += fabsf(xn.a[v] - xh.a[v]);
+        }
+        xc = xo;
+      }
+      s_red[(size_t)j * 33 + lane] = ev;
+      s_red[(size_t)(P + j) * 33 + lane] = dv;
+    }
+  }
+  __syncthreads();
+  // strip partials: one thread per (quantity, position) sums its row of lanes
+  const int64_t pbase = (int64_t)b * P * nstrip + strip;
+  for (int r = tid; r < 2 * p; r += NW * 32) {
+    const int which = r / p, j = r % p;
+    const float* row = s_red + (size_t)(which * P + j) * 33;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < 32; c += 4) {
+      acc[0] += row[c];
+      acc[1] += row[c + 1];
+      acc[2] += row[c + 2];
+      acc[3] += row[c + 3];
+    }
+    (which == 0 ? d.part_err : d.part_del)[pbase + (int64_t)j * nstrip] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  }
+  // after a timeout, let this warp's copies land before the CTA exits
+  if (my_fail && lane == 0 && j0 < j1) mbar_wait_bounded(&bar[warp], 0, kDrainLimit);
+}
+
+constexpr size_t kSegSmemMax = 200 * 1024;
+
+template <int V, int NW>
+bool seg_fits(const Dev& d) {
+  return SegShape<V, NW>::smem_bytes(d.P) <= kSegSmemMax;
+}
+
+template <int V, int NW>
+cudaError_t launch_seg(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+  using Sh = SegShape<V, NW>;
+  const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
+  const size_t smem = Sh::smem_bytes(d.P);
+  auto kern = k_update_seg<V, NW>;
+  static size_t configured[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || smem > configured[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) configured[dev] = smem;
+  }
+  *nchunk_out = nstrip;
+  return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, nstrip, d.wait_limit);
+}
+
 // Shared memory budget per CTA for the tile buffers: enough for the whole
 // window when it fits, so every copy is in flight from the start.
 constexpr size_t kSmemBudget = 112 * 1024;
@@ -454,19 +698,8 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
   }
   const int gx = CLUSTER ? (nstrip + kCluster - 1) / kCluster * kCluster : nstrip;
   *nchunk_out = CLUSTER ? gx / kCluster : nstrip;  // partials per position
-  cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(gx, d.B, 1);
-  cfg.blockDim = dim3(NW * 32, 1, 1);
-  cfg.dynamicSmemBytes = smem;
-  cfg.stream = st;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = CLUSTER ? kCluster : 1;
-  attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = 1;
-  cfg.attrs = attr;
-  cfg.numAttrs = CLUSTER ? 1 : 0;
-  return cudaLaunchKernelEx(&cfg, kern, d, beps, nstrip, nbuf, d.wait_limit);
+  return launch_ex(kern, dim3(gx, d.B, 1), dim3(NW * 32), smem, st, CLUSTER ? kCluster : 0, d, beps, nstrip,
+                   nbuf, d.wait_limit);
 }
 
 }  // namespace
@@ -479,16 +712,23 @@ bool update_bulk_supported(const Dev& d, const float* batch_eps) {
 
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
   switch (d.bulk_cfg) {
-    case 0: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 1: return launch_tile<2, 8, 4, false, false>(d, batch_eps, st, nchunk_out);
+    case 0:  // whole window in shared memory when it fits, else the tiled pipeline
+      if (seg_fits<2, 8>(d)) return launch_seg<2, 8>(d, batch_eps, st, nchunk_out);
+      return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 1: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
     case 2: return launch_tile<2, 8, 4, true, true>(d, batch_eps, st, nchunk_out);
-    case 3: return launch_tile<2, 8, 4, true, false>(d, batch_eps, st, nchunk_out);
-    case 4: return launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
-    case 5: return launch_tile<1, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 6: return launch_tile<2, 8, 2, false, true>(d, batch_eps, st, nchunk_out);
-    case 7: return launch_tile<2, 16, 2, false, true>(d, batch_eps, st, nchunk_out);
-    case 8: return launch_tile<2, 8, 8, false, true>(d, batch_eps, st, nchunk_out);
-    case 9: return launch_tile<2, 4, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 3: return launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
+    case 4: return seg_fits<2, 8>(d) ? launch_seg<2, 8>(d, batch_eps, st, nchunk_out)
+                                     : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 5: return seg_fits<2, 16>(d) ? launch_seg<2, 16>(d, batch_eps, st, nchunk_out)
+                                      : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 6: return seg_fits<1, 8>(d) ? launch_seg<1, 8>(d, batch_eps, st, nchunk_out)
+                                     : launch_tile<1, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 7: return seg_fits<1, 16>(d) ? launch_seg<1, 16>(d, batch_eps, st, nchunk_out)
+                                      : launch_tile<1, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 8: return seg_fits<2, 4>(d) ? launch_seg<2, 4>(d, batch_eps, st, nchunk_out)
+                                     : launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
+    case 9: return launch_tile<2, 8, 2, false, true>(d, batch_eps, st, nchunk_out);
     default: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
   }
 }

@@ -102,6 +102,48 @@ struct Dev {
 };
 constexpr uint32_t kWaitLimit = 1u << 24;
 
+// Programmatic dependent launch (PDL). Every kernel of an iteration is
+// launched with programmatic stream serialization, so it may be scheduled as
+// soon as its predecessor's CTAs have exited, before the predecessor's grid is
+// retired: it does the work that does not read the predecessor's output, then
+// executes pdl_wait() (predecessor complete, its writes visible). No kernel
+// triggers its successor early (pdl_trigger is available but unused: early
+// triggers let waiting CTAs hold shared memory the predecessor still needs),
+// so a kernel's prologue may read anything written two or more kernels back.
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+bool pdl_enabled();  // false when the environment sets PA_DISABLE_PDL=1
+
+// cudaLaunchKernelEx with the PDL attribute (when enabled) and an optional
+// cluster width along x (0 = no cluster attribute).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                      unsigned cluster_x, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[2];
+  unsigned n = 0;
+  if (pdl_enabled()) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  if (cluster_x > 0) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = cluster_x;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
+
 // Kernel launchers (k_solver.cu). Each returns the launch error.
 cudaError_t launch_init_plan(const Dev& d, cudaStream_t st);
 cudaError_t launch_gather(const Dev& d, cudaStream_t st);

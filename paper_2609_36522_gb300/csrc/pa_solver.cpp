@@ -4,6 +4,7 @@
 
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -15,6 +16,14 @@ namespace pa {
 
 static thread_local std::string g_err;
 void set_error(const std::string& msg) { g_err = msg; }
+
+bool pdl_enabled() {
+  static const bool on = [] {
+    const char* v = std::getenv("PA_DISABLE_PDL");
+    return !(v && v[0] == '1');
+  }();
+  return on;
+}
 
 }  // namespace pa
 
