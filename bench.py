@@ -325,9 +325,10 @@ def run_ours(args):
     graph = torch.cuda.CUDAGraph()
     s.init(x_dev)
     stream.synchronize()
+    gmm0 = g.launches()
     with torch.cuda.graph(graph, stream=stream):
         one_iteration()
-    kernels_per_iter = 6
+    kernels_per_iter = 3 + (g.launches() - gmm0)   # gather, update, decision + denoiser kernels
 
     def generation(timed):
         s.init(x_dev)
@@ -439,7 +440,7 @@ def run_ours(args):
                        "l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every Picard iteration, outside the timed events"),
                        "timing": "CUDA events around each Picard iteration (one CUDA-graph replay of "
-                                 "gather, denoiser, update, decision) on the launch stream"},
+                                 "gather, denoiser, update, decision kernels) on the launch stream"},
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
             "solver_step_gbps": gb_step,

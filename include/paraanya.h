@@ -240,7 +240,7 @@ PA_API void pa_gmm_destroy(pa_gmm* g);
  *
  * Scratch lives in one fixed 4 MiB device array inside this library (every
  * GPU that loads the library holds it until the process exits). Sizes whose
- * scratch (3T coefficients, K norms, n_rows*K*ceil(D/chunk) partials,
+ * scratch (3T coefficients, K norms, n_rows*K dot-product accumulators and
  * responsibilities) would exceed 4 MiB are rejected with PA_ERR_ARG and a
  * message naming the bytes needed; use pa_gmm_create/pa_gmm_eps then.
  *

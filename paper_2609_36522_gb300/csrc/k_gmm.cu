@@ -6,15 +6,13 @@
 //   r = softmax(logit)   (the common -||x||^2 / (2 v) term cancels)
 //   eps = sqrt(1 - a) / v * (x - sqrt(a) sum_k r_k mu_k)
 //
-// Three kernels per call, each with a single load phase:
-//   k_gmm_dots     split-K contraction G = X M^T: a CTA stages a tile of 16
-//                  rows and its D-chunk of every mean (bulk copies), one warp
-//                  per row accumulates 16 components per pass, partials go to
-//                  gpart[chunk][row][k]
-//   k_gmm_softmax  one CTA per row: fixed-order sum of the chunk partials,
-//                  logits, max-subtracted softmax
-//   k_gmm_out      a CTA stages a 16-row x 256-column tile of X and the same
-//                  columns of every mean, then eps = a x - a sqrt(a) R M
+// Two kernels per call, each with a single load phase:
+//   k_gmm_dots     split-K contraction G = X M^T over bulk-staged 16-row tiles
+//                  (register-tiled 4 rows x 8 components per thread); the last
+//                  CTA of each row block sums the chunks in a fixed order and
+//                  applies the logits and the max-subtracted softmax
+//   k_gmm_out      eps = a x - a sqrt(a) R M over bulk-staged 16-row x
+//                  256-column tiles (4 x 4 outputs per thread)
 // Per-timestep scalars (sqrt(a), 1/(2v), sqrt(1-a)/v) are computed on the
 // host in fp64 from alpha-bar and stored in fp32, so 1 - a never cancels in
 // fp32. Reductions run in a fixed order: results are bitwise reproducible.
@@ -47,14 +45,24 @@ constexpr int kThreads = 256;
 constexpr int kDotRows = 16;     // rows per dots CTA (two per warp)
 constexpr int kKTile = 16;       // components accumulated per pass
 constexpr int kOutRows = 16;     // rows per output CTA
-constexpr int kOutCols = 256;    // columns per output CTA (one per thread)
+constexpr int kOutCols = 256;    // columns per output CTA (four per thread)
 constexpr size_t kDotSmemBudget = 96 * 1024;
+constexpr float kDotScale = 4294967296.f;  // 2^32: fixed-point scale of the dot-product accumulators
 
 struct GmmLayout {
-  size_t coef, mnorm, gpart, R, rowc, status, total;
+  size_t coef, mnorm, gacc, R, rowc, tickets, status, total;
   int nchunk;       // D-chunks of the dots kernel
   int chunk;        // columns per chunk
 };
+
+size_t dots_smem_bytes(int K, int chunk) {
+  // the staged tiles, later reused for the column-split sums
+  int KG = 1;
+  while (KG * 8 < K) KG <<= 1;
+  const size_t tiles = (size_t)(kDotRows + K) * (chunk + 4) * sizeof(float);
+  const size_t red = (size_t)(kThreads / (4 * KG) + 1) * kDotRows * K * sizeof(float);
+  return tiles > red ? tiles : red;
+}
 
 int dots_chunk(int K, int64_t D) {
   // largest of 512/256/128/64 columns whose (rows + K) row segments fit the budget
@@ -72,9 +80,10 @@ GmmLayout gmm_layout(int K, int64_t D, int max_rows, int T) {
   L.nchunk = (int)((D + L.chunk - 1) / L.chunk);
   L.coef = take((size_t)3 * T * sizeof(float));
   L.mnorm = take((size_t)K * sizeof(float));
-  L.gpart = take((size_t)L.nchunk * max_rows * K * sizeof(float));
+  L.gacc = take((size_t)max_rows * K * sizeof(long long));
   L.R = take((size_t)max_rows * K * sizeof(float));
   L.rowc = take((size_t)max_rows * 2 * sizeof(float));
+  L.tickets = take((size_t)((max_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t));
   L.status = take(sizeof(int32_t));
   L.total = o;
   return L;
@@ -137,15 +146,33 @@ __device__ __forceinline__ bool wait_staged(bool bulk, uint64_t* bar, int32_t* s
   return false;
 }
 
-// gpart[chunk][r][k] = sum over the chunk's columns of x[r][d] mu[k][d]
+// Dot products and softmax, one kernel: a CTA stages 16 rows x `chunk`
+// columns of X and the same columns of every mean, each thread accumulates a
+// 4-row x 8-component block over a column split (register tiling: 12 shared
+// loads per 32 FMAs), and the column splits are summed in a fixed order
+// through shared memory. Chunks are combined by adding each CTA's sums,
+// rounded to fixed point (2^-32), into int64 accumulators gacc[r][k] with
+// atomics: integer addition is exact, so the result does not depend on the
+// order in which CTAs arrive. The CTA that finishes a row block last (atomic
+// ticket after a fence, nobody waits) reads the finished dot products, clears
+// the accumulators for the next call, and applies the logits and the
+// max-subtracted softmax -> R[r][k], rowc[r].
 __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__ X,
                                                        const float* __restrict__ mu,
                                                        const int32_t* __restrict__ n_rows_dev,
-                                                       int K, int64_t D, int chunk, int max_rows,
-                                                       bool bulk, float* __restrict__ gpart,
+                                                       int K, int64_t D, int chunk, int nchunk, int max_rows,
+                                                       bool bulk, long long* __restrict__ gacc,
+                                                       uint32_t* __restrict__ tickets,
+                                                       const float* __restrict__ coef, int T,
+                                                       const int32_t* __restrict__ miss_bt,
+                                                       const float* __restrict__ mnorm,
+                                                       float* __restrict__ R, float* __restrict__ rowc,
                                                        int32_t* status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t bar;
+  __shared__ int s_last;
+  __shared__ float s_logit[kDotRows * kMaxK];
+  __shared__ float s_sa[kDotRows], s_q[kDotRows], s_ac[kDotRows];
   const int n_rows = min(*n_rows_dev, max_rows);
   const int r0 = blockIdx.y * kDotRows;
   if (r0 >= n_rows) return;
@@ -155,11 +182,13 @@ __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__
   const int ld = chunk + 4;  // padded row stride, keeps 16-byte alignment
   float* xs = reinterpret_cast<float*>(smem_raw);
   float* ms = xs + (size_t)kDotRows * ld;
-  if (threadIdx.x == 0) {
+  const int tid = threadIdx.x;
+  if (tid == 0) {
     mbar_init(&bar, 1);
     fence_barrier_init();
     if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
   }
+  for (int q = tid; q < (kDotRows - nr) * ld; q += kThreads) xs[(size_t)nr * ld + q] = 0.f;  // rows past nr
   __syncthreads();
   stage_rows(ms, ld, mu, D, c0, ncol, K, bulk, &bar);  // the means do not depend on the predecessor
   pdl_wait();  // the rows come from the gather (or the caller) just before
@@ -167,88 +196,106 @@ __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__
   const bool ok = wait_staged(bulk, &bar, status);
   __syncthreads();
   if (!ok) return;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  for (int rr = warp; rr < nr; rr += kThreads / 32) {
-    const float* xr = xs + (size_t)rr * ld;
-    for (int k0 = 0; k0 < K; k0 += kKTile) {
-      float acc[kKTile];
-#pragma unroll
-      for (int u = 0; u < kKTile; ++u) acc[u] = 0.f;
-      for (int c = lane; c < ncol; c += 32) {
-        const float xv = xr[c];
-#pragma unroll
-        for (int u = 0; u < kKTile; ++u)
-          if (k0 + u < K) acc[u] = fmaf(xv, ms[(size_t)(k0 + u) * ld + c], acc[u]);
-      }
-#pragma unroll
-      for (int u = 0; u < kKTile; ++u) acc[u] = warp_sum(acc[u]);
-      if (lane < kKTile && k0 + lane < K) {
-        float v = 0.f;
-#pragma unroll
-        for (int u = 0; u < kKTile; ++u) v = (lane == u) ? acc[u] : v;
-        gpart[((int64_t)blockIdx.x * max_rows + r0 + rr) * K + k0 + lane] = v;
-      }
-    }
-  }
-}
 
-// One CTA per row: dots (fixed-order chunk sum) -> logits -> softmax.
-__global__ void __launch_bounds__(kThreads) k_gmm_softmax(const float* __restrict__ gpart,
-                                                          const float* __restrict__ mnorm,
-                                                          const float* __restrict__ coef, int T,
-                                                          const int32_t* __restrict__ miss_bt,
-                                                          const int32_t* __restrict__ n_rows_dev,
-                                                          int K, int nchunk, int max_rows,
-                                                          float* __restrict__ R,
-                                                          float* __restrict__ rowc) {
-  __shared__ float s_part[kThreads];
-  __shared__ float s_logit[kMaxK];
-  const int n_rows = min(*n_rows_dev, max_rows);
-  const int r = blockIdx.x;
-  if (r >= n_rows) return;
-  // thread -> (component k, chunk group g); groups take the chunks round robin
-  int KB = 1;
-  while (KB < K) KB <<= 1;
-  const int G = kThreads / KB;
-  const int k = threadIdx.x % KB, g = threadIdx.x / KB;
-  const int i = miss_bt[2 * r + 1];
-  const float sa = coef[i], q = coef[T + i], ac = coef[2 * T + i];
-  pdl_wait();  // the partials come from the dot-product kernel
-  float part = 0.f;
-  if (k < K)
-    for (int s = g; s < nchunk; s += G) part += gpart[((int64_t)s * max_rows + r) * K + k];
-  s_part[threadIdx.x] = part;
+  // thread -> (column split tcs, component group tkg, row group trg)
+  int KG = 1;
+  while (KG * 8 < K) KG <<= 1;          // component groups of 8 (power of two)
+  const int CS = kThreads / (4 * KG);   // column splits
+  const int tcs = tid % CS, tkg = (tid / CS) % KG, trg = tid / (CS * KG);
+  float acc[4][8];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int u = 0; u < 8; ++u) acc[i][u] = 0.f;
+  for (int c = tcs; c < ncol; c += CS) {
+    float xv[4], mv[8];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) xv[i] = xs[(size_t)(trg * 4 + i) * ld + c];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int k = tkg + KG * u;  // interleaved: neighbouring groups read neighbouring rows
+      mv[u] = (k < K) ? ms[(size_t)k * ld + c] : 0.f;
+    }
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int u = 0; u < 8; ++u) acc[i][u] = fmaf(xv[i], mv[u], acc[i][u]);
+  }
+  __syncthreads();  // the tiles are consumed: reuse their space for the split sums
+  float* red = xs;  // [kDotRows * K][CS + 1]: split index fastest (conflict-free both ways)
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int k = tkg + KG * u;
+      if (k < K) red[((size_t)(trg * 4 + i) * K + k) * (CS + 1) + tcs] = acc[i][u];
+    }
   __syncthreads();
-  if (threadIdx.x < K) {
-    float dot = 0.f;
-    for (int gg = 0; gg < G; ++gg) dot += s_part[gg * KB + threadIdx.x];
-    s_logit[threadIdx.x] = (2.f * sa * dot - sa * sa * mnorm[threadIdx.x]) * q;
+  for (int o = tid; o < nr * K; o += kThreads) {
+    float a4[4] = {0.f, 0.f, 0.f, 0.f};
+    const float* ro = red + (size_t)o * (CS + 1);
+    for (int cs = 0, u = 0; cs < CS; ++cs, u = (u + 1) & 3) a4[u] += ro[cs];
+    const float sum = (a4[0] + a4[1]) + (a4[2] + a4[3]);
+    atomicAdd(reinterpret_cast<unsigned long long*>(gacc + (int64_t)r0 * K + o),
+              static_cast<unsigned long long>(__float2ll_rn(sum * kDotScale)));
+  }
+  // the last CTA of this row block finishes the contraction and the softmax
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    const unsigned int k = atomicAdd(&tickets[blockIdx.y], 1u);
+    s_last = (k == gridDim.x - 1);
   }
   __syncthreads();
-  if (threadIdx.x < 32) {
-    const int lane = threadIdx.x;
+  if (!s_last) return;
+  __threadfence();
+  if (tid == 0) tickets[blockIdx.y] = 0u;  // ready for the next call
+  if (tid < nr) {
+    const int i = miss_bt[2 * (r0 + tid) + 1];
+    s_sa[tid] = coef[i];
+    s_q[tid] = coef[T + i];
+    s_ac[tid] = coef[2 * T + i];
+  }
+  __syncthreads();
+  for (int o = tid; o < nr * K; o += kThreads) {
+    const int rr = o / K, k = o % K;
+    long long* acc_p = gacc + (int64_t)(r0 + rr) * K + k;
+    const long long v = __ldcg(acc_p);
+    *acc_p = 0;  // ready for the next call
+    const float dot = (float)((double)v * (1.0 / (double)kDotScale));
+    const float sa = s_sa[rr];
+    s_logit[rr * K + k] = (2.f * sa * dot - sa * sa * mnorm[k]) * s_q[rr];
+  }
+  __syncthreads();
+  const int warp = tid >> 5, lane = tid & 31;
+  for (int rr = warp; rr < nr; rr += kThreads / 32) {
+    const float* l = s_logit + rr * K;
     float mx = -INFINITY;
-    for (int kk = lane; kk < K; kk += 32) mx = fmaxf(mx, s_logit[kk]);
+    for (int k = lane; k < K; k += 32) mx = fmaxf(mx, l[k]);
     mx = warp_max(mx);
     float sum = 0.f;
-    for (int kk = lane; kk < K; kk += 32) sum += expf(s_logit[kk] - mx);
+    for (int k = lane; k < K; k += 32) sum += expf(l[k] - mx);
     sum = warp_sum(sum);
     const float inv = 1.f / sum;
-    for (int kk = lane; kk < K; kk += 32) R[(int64_t)r * K + kk] = expf(s_logit[kk] - mx) * inv;
+    const int r = r0 + rr;
+    for (int k = lane; k < K; k += 32) R[(int64_t)r * K + k] = expf(l[k] - mx) * inv;
     if (lane == 0) {
-      rowc[2 * r] = ac;
-      rowc[2 * r + 1] = ac * sa;
+      rowc[2 * r] = s_ac[rr];
+      rowc[2 * r + 1] = s_ac[rr] * s_sa[rr];
     }
   }
 }
 
-// eps[r][c] = ac x[r][c] - ac sqrt(a) sum_k R[r][k] mu[k][c]
-__global__ void __launch_bounds__(kOutCols) k_gmm_out(const float* __restrict__ X,
+// eps[r][c] = ac x[r][c] - ac sqrt(a) sum_k R[r][k] mu[k][c]: a CTA stages a
+// 16-row x 256-column tile of X and the same columns of every mean; each
+// thread computes a 4-row x 4-column block (one 16-byte mean load and four
+// broadcast responsibility loads per 16 FMAs).
+__global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ X,
                                                       const float* __restrict__ mu,
                                                       const float* __restrict__ R,
                                                       const float* __restrict__ rowc,
                                                       const int32_t* __restrict__ n_rows_dev,
-                                                      int K, int64_t D, int max_rows, bool bulk,
+                                                      int K, int64_t D, int max_rows, bool bulk, bool vec_out,
                                                       float* __restrict__ eps, int32_t* status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t bar;
@@ -262,7 +309,8 @@ __global__ void __launch_bounds__(kOutCols) k_gmm_out(const float* __restrict__ 
   const int ncol = (int)(((D - c0) < kOutCols) ? (D - c0) : kOutCols);
   float* ms = reinterpret_cast<float*>(smem_raw);   // [K][kOutCols]
   float* xs = ms + (size_t)K * kOutCols;            // [kOutRows][kOutCols]
-  if (threadIdx.x == 0) {
+  const int tid = threadIdx.x;
+  if (tid == 0) {
     mbar_init(&bar, 1);
     fence_barrier_init();
     if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
@@ -271,18 +319,47 @@ __global__ void __launch_bounds__(kOutCols) k_gmm_out(const float* __restrict__ 
   // the means and the rows (written two kernels back) do not depend on the predecessor
   stage_rows(ms, kOutCols, mu, D, c0, ncol, K, bulk, &bar);
   stage_rows(xs, kOutCols, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
-  pdl_wait();  // the responsibilities come from the softmax kernel
-  for (int q = threadIdx.x; q < nr * K; q += kOutCols) s_r[q] = R[(int64_t)r0 * K + q];
-  for (int q = threadIdx.x; q < nr * 2; q += kOutCols) s_c[q] = rowc[2 * r0 + q];
+  pdl_wait();  // the responsibilities come from the dot-product kernel
+  for (int q = tid; q < kOutRows * K; q += kThreads) s_r[q] = (q < nr * K) ? R[(int64_t)r0 * K + q] : 0.f;
+  for (int q = tid; q < kOutRows * 2; q += kThreads) s_c[q] = (q < nr * 2) ? rowc[2 * r0 + q] : 0.f;
   const bool ok = wait_staged(bulk, &bar, status);
   __syncthreads();
   if (!ok) return;
-  const int c = threadIdx.x;
-  if (c >= ncol) return;
-  for (int rr = 0; rr < nr; ++rr) {
-    float m = 0.f;
-    for (int k = 0; k < K; ++k) m = fmaf(s_r[rr * K + k], ms[(size_t)k * kOutCols + c], m);
-    eps[(int64_t)(r0 + rr) * D + c0 + c] = s_c[2 * rr] * xs[(size_t)rr * kOutCols + c] - s_c[2 * rr + 1] * m;
+  const int cg = tid % (kOutCols / 4), rg = tid / (kOutCols / 4);  // 64 column groups x 4 row groups
+  const int cc = cg * 4;
+  if (cc >= ncol) return;
+  float acc[4][4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+  for (int k = 0; k < K; ++k) {
+    const float4 m = *reinterpret_cast<const float4*>(ms + (size_t)k * kOutCols + cc);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float rk = s_r[(rg * 4 + i) * K + k];
+      acc[i][0] = fmaf(rk, m.x, acc[i][0]);
+      acc[i][1] = fmaf(rk, m.y, acc[i][1]);
+      acc[i][2] = fmaf(rk, m.z, acc[i][2]);
+      acc[i][3] = fmaf(rk, m.w, acc[i][3]);
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const int rr = rg * 4 + i;
+    if (rr >= nr) break;
+    const float ac = s_c[2 * rr], acs = s_c[2 * rr + 1];
+    const float* xr = xs + (size_t)rr * kOutCols + cc;
+    float* er = eps + (int64_t)(r0 + rr) * D + c0 + cc;
+    if (vec_out && cc + 4 <= ncol) {
+      const float4 x = *reinterpret_cast<const float4*>(xr);
+      *reinterpret_cast<float4*>(er) = make_float4(ac * x.x - acs * acc[i][0], ac * x.y - acs * acc[i][1],
+                                                   ac * x.z - acs * acc[i][2], ac * x.w - acs * acc[i][3]);
+    } else {
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (cc + j < ncol) er[j] = ac * xr[j] - acs * acc[i][j];
+    }
   }
 }
 
@@ -340,12 +417,16 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
   cudaError_t e = cudaMemcpyAsync(g->ws + L.coef, coef.data(), coef.size() * sizeof(float),
                                   cudaMemcpyHostToDevice, g->st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.status, 0, sizeof(int32_t), g->st);
+  if (e == cudaSuccess)
+    e = cudaMemsetAsync(g->ws + L.tickets, 0, (size_t)((max_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t),
+                        g->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.gacc, 0, (size_t)max_rows * K * sizeof(long long), g->st);
   if (e == cudaSuccess) {
     k_gmm_norms<<<K, 256, 0, g->st>>>(means_dev, D, reinterpret_cast<float*>(g->ws + L.mnorm));
     g->launches++;
     e = cudaGetLastError();
   }
-  const size_t dots_smem = (size_t)(kDotRows + K) * (L.chunk + 4) * sizeof(float);
+  const size_t dots_smem = dots_smem_bytes(K, L.chunk);
   const size_t out_smem = (size_t)(K + kOutRows) * kOutCols * sizeof(float);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_gmm_dots, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dots_smem);
@@ -370,28 +451,28 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
   const GmmLayout& L = g->L;
   float* coef = reinterpret_cast<float*>(g->ws + L.coef);
   float* mnorm = reinterpret_cast<float*>(g->ws + L.mnorm);
-  float* gpart = reinterpret_cast<float*>(g->ws + L.gpart);
+  long long* gacc = reinterpret_cast<long long*>(g->ws + L.gacc);
   float* R = reinterpret_cast<float*>(g->ws + L.R);
   float* rowc = reinterpret_cast<float*>(g->ws + L.rowc);
   int32_t* status = reinterpret_cast<int32_t*>(g->ws + L.status);
   // bulk copies need 16-byte aligned rows: D % 4 == 0 and aligned base pointers
   const bool bulk = g->D % 4 == 0 && ((reinterpret_cast<uintptr_t>(batch_x_dev) |
                                        reinterpret_cast<uintptr_t>(g->means)) & 15) == 0;
-  const size_t dots_smem = (size_t)(kDotRows + g->K) * (L.chunk + 4) * sizeof(float);
+  uint32_t* tickets = reinterpret_cast<uint32_t*>(g->ws + L.tickets);
+  const bool vec_out = g->D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps_dev) & 15) == 0;
+  const size_t dots_smem = dots_smem_bytes(g->K, L.chunk);
   const size_t out_smem = (size_t)(g->K + kOutRows) * kOutCols * sizeof(float);
   cudaError_t e = pa::launch_ex(k_gmm_dots, dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows),
                                 dim3(kThreads), dots_smem, g->st, 0, batch_x_dev, g->means, n_rows_dev, g->K,
-                                g->D, L.chunk, g->max_rows, bulk, gpart, status);
-  if (e == cudaSuccess)
-    e = pa::launch_ex(k_gmm_softmax, dim3(g->max_rows), dim3(kThreads), 0, g->st, 0, (const float*)gpart,
-                      (const float*)mnorm, (const float*)coef, g->T, miss_bt_dev, n_rows_dev, g->K, L.nchunk,
-                      g->max_rows, R, rowc);
+                                g->D, L.chunk, L.nchunk, g->max_rows, bulk, gacc, tickets, (const float*)coef,
+                                g->T, miss_bt_dev, (const float*)mnorm, R, rowc, status);
   if (e == cudaSuccess)
     e = pa::launch_ex(k_gmm_out,
                       dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
                       dim3(kOutCols), out_smem, g->st, 0, batch_x_dev, g->means, (const float*)R,
-                      (const float*)rowc, n_rows_dev, g->K, g->D, g->max_rows, bulk, batch_eps_dev, status);
-  g->launches += 3;
+                      (const float*)rowc, n_rows_dev, g->K, g->D, g->max_rows, bulk, vec_out, batch_eps_dev,
+                      status);
+  g->launches += 2;
   if (e == cudaSuccess) e = cudaGetLastError();
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_eps: ") + cudaGetErrorString(e));
@@ -488,17 +569,18 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
     }
   }
   if (n_rows == 0) return PA_OK;
-  // scratch layout: coef[3T] | mnorm[K] | gpart[nchunk][n_rows][K] | R[n_rows][K] |
-  //                 rowc[n_rows][2] | n_rows | status   (256-byte aligned pieces)
+  // scratch layout: coef[3T] | mnorm[K] | gacc[n_rows][K] (int64) | R[n_rows][K] |
+  //                 rowc[n_rows][2] | tickets | n_rows | status   (256-byte aligned pieces)
   const int chunk = dots_chunk(K, D);
   const int nchunk = (int)((D + chunk - 1) / chunk);
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t at = o; o = pa::align_up(o + bytes, pa::kAlign); return at; };
   const size_t o_coef = take((size_t)3 * T * sizeof(float));
   const size_t o_mnorm = take((size_t)K * sizeof(float));
-  const size_t o_gpart = take((size_t)nchunk * n_rows * K * sizeof(float));
+  const size_t o_gacc = take((size_t)n_rows * K * sizeof(long long));
   const size_t o_R = take((size_t)n_rows * K * sizeof(float));
   const size_t o_rowc = take((size_t)n_rows * 2 * sizeof(float));
+  const size_t o_tick = take((size_t)((n_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t));
   const size_t o_n = take(sizeof(int32_t));
   const size_t o_status = take(sizeof(int32_t));
   if (o > kNoAllocScratchBytes) {
@@ -513,9 +595,10 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* coef = reinterpret_cast<float*>(scratch + o_coef);
   float* mnorm = reinterpret_cast<float*>(scratch + o_mnorm);
-  float* gpart = reinterpret_cast<float*>(scratch + o_gpart);
+  long long* gacc = reinterpret_cast<long long*>(scratch + o_gacc);
   float* R = reinterpret_cast<float*>(scratch + o_R);
   float* rowc = reinterpret_cast<float*>(scratch + o_rowc);
+  uint32_t* tickets = reinterpret_cast<uint32_t*>(scratch + o_tick);
   int32_t* nrows_dev = reinterpret_cast<int32_t*>(scratch + o_n);
   int32_t* status = reinterpret_cast<int32_t*>(scratch + o_status);
 
@@ -538,7 +621,10 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   const int32_t nr = n_rows;
   if (e == cudaSuccess) e = cudaMemcpyAsync(nrows_dev, &nr, sizeof(nr), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);  // starts at zero every call
-  const size_t dots_smem = (size_t)(kDotRows + K) * (chunk + 4) * sizeof(float);
+  if (e == cudaSuccess)  // the row-block tickets and the dot accumulators start at zero every call too
+    e = cudaMemsetAsync(tickets, 0, (size_t)((n_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(gacc, 0, (size_t)n_rows * K * sizeof(long long), st);
+  const size_t dots_smem = dots_smem_bytes(K, chunk);
   const size_t out_smem = (size_t)(K + kOutRows) * kOutCols * sizeof(float);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_gmm_dots, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dots_smem);
@@ -551,13 +637,13 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   const bool bulk = D % 4 == 0 && ((reinterpret_cast<uintptr_t>(batch_x_dev) |
                                     reinterpret_cast<uintptr_t>(means_dev)) & 15) == 0;
   k_gmm_norms<<<K, 256, 0, st>>>(means_dev, D, mnorm);
+  const bool vec_out = D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps_dev) & 15) == 0;
   k_gmm_dots<<<dim3(nchunk, (n_rows + kDotRows - 1) / kDotRows), kThreads, dots_smem, st>>>(
-      batch_x_dev, means_dev, nrows_dev, K, D, chunk, n_rows, bulk, gpart, status);
-  k_gmm_softmax<<<n_rows, kThreads, 0, st>>>(gpart, mnorm, coef, T, miss_bt_dev, nrows_dev, K, nchunk,
-                                             n_rows, R, rowc);
-  k_gmm_out<<<dim3((unsigned)((D + kOutCols - 1) / kOutCols), (n_rows + kOutRows - 1) / kOutRows),
-              kOutCols, out_smem, st>>>(batch_x_dev, means_dev, R, rowc, nrows_dev, K, D, n_rows, bulk,
-                                        batch_eps_dev, status);
+      batch_x_dev, means_dev, nrows_dev, K, D, chunk, nchunk, n_rows, bulk, gacc, tickets, coef, T, miss_bt_dev,
+      mnorm, R, rowc, status);
+  k_gmm_out<<<dim3((unsigned)((D + kOutCols - 1) / kOutCols), (n_rows + kOutRows - 1) / kOutRows), kOutCols,
+              out_smem, st>>>(batch_x_dev, means_dev, R, rowc, nrows_dev, K, D, n_rows, bulk, vec_out,
+                              batch_eps_dev, status);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_eps_noalloc: ") + cudaGetErrorString(e));

@@ -74,15 +74,16 @@ def test_noalloc_matches_handle_entry_point_on_two_calls(lib):
 def test_noalloc_rejects_sizes_beyond_its_scratch(lib):
     import torch
     abi = lib
-    w = W.LARGE  # K=64, D=65536: 128 rows need far more than 4 MiB of partials
-    a, _, mu = W.inputs(w)
+    # 4096 rows x 128 components need 4 MiB of int64 dot accumulators alone
+    K, D, n, T = 128, 256, 4096, 10
+    a = W.alphas_cumprod(T)
     dev = torch.device("cuda")
-    mu_d = torch.from_numpy(mu).to(dev)
-    x = torch.zeros(128, w.D, device=dev)
-    miss = torch.zeros(128, 2, dtype=torch.int32, device=dev)
+    mu_d = torch.randn(K, D, device=dev)
+    x = torch.zeros(n, D, device=dev)
+    miss = torch.zeros(n, 2, dtype=torch.int32, device=dev)
     out = torch.zeros_like(x)
     with pytest.raises(abi.PaError) as e:
-        abi.pa_gmm_eps_noalloc(mu_d.data_ptr(), w.K, w.D, w.gmm_std, list(a), x.data_ptr(),
-                               miss.data_ptr(), 128, out.data_ptr(), 0)
+        abi.pa_gmm_eps_noalloc(mu_d.data_ptr(), K, D, 0.5, list(a), x.data_ptr(),
+                               miss.data_ptr(), n, out.data_ptr(), 0)
     assert e.value.status == abi.PA_ERR_ARG
     assert "4 MiB" in str(e.value)
