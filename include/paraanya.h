@@ -173,8 +173,9 @@ PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
  * method's; call pa_init before using the solver's results again. */
 PA_API pa_status pa_bench_update_only(pa_solver* s, const float* batch_eps_dev, int repeats);
 
-/* Fault-handling test hook: the number of polls after which an mbarrier wait
- * of the bulk-copy update kernel counts as timed out (default 2^24). With 0
+/* Fault-handling test hook: the number of tries (each may suspend for about
+ * 10 us) after which an mbarrier wait of the bulk-copy update kernel counts
+ * as timed out (default 2^17, about a second). With 0
  * every such wait gives up at once: the kernel records PA_ERR_TIMEOUT (read by
  * the next synchronising call), still drains its in-flight copies with the
  * default bound, and leaves the solver's numbers meaningless until pa_init. */

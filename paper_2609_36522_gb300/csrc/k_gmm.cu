@@ -119,14 +119,15 @@ __global__ void __launch_bounds__(256) k_gmm_norms(const float* __restrict__ mu,
 
 // Stage `nrows` row segments [c0, c0 + ncol) of a row-major matrix with row
 // length D into shared rows of stride `ld` floats: bulk copies counted on
-// `bar`, issued by thread 0 (after the caller announced the bytes), or plain
-// loads by every thread when `bulk` is false.
+// `bar`, issued by the lanes of warp 0 (after the caller announced the bytes),
+// or plain loads by every thread when `bulk` is false.
 __device__ __forceinline__ void stage_rows(float* dst, int ld, const float* src, int64_t D, int64_t c0,
                                            int ncol, int nrows, bool bulk, uint64_t* bar) {
   if (bulk) {
-    if (threadIdx.x == 0) {
+    if (threadIdx.x < 32) {  // the lanes of warp 0 issue the rows in parallel
       const uint32_t seg = (uint32_t)ncol * sizeof(float);
-      for (int r = 0; r < nrows; ++r) bulk_g2s(dst + (size_t)r * ld, src + (int64_t)r * D + c0, seg, bar);
+      for (int r = threadIdx.x; r < nrows; r += 32)
+        bulk_g2s(dst + (size_t)r * ld, src + (int64_t)r * D + c0, seg, bar);
     }
     return;
   }

@@ -6,6 +6,8 @@
 //   Xhat [B][P][D]    cache inputs  xhat_i  (Eq. 3), slot i mod P
 //   Ehat [B][P][D]    cache outputs ehat_i  (Eq. 3), slot i mod P
 //   batch_x [B*P][D]  gathered latents of the misses, rank order
+#include <type_traits>
+
 #include "pa_internal.h"
 
 namespace pa {
@@ -57,23 +59,35 @@ __global__ void k_init_plan(Dev d) {
 
 // ---------------------------------------------------------------------------
 // a4: batch_x[r] <- x_{miss[r]} for r < n_miss. A lazy state (i > e) reads
-// state e, the value every new tail state was initialised to.
+// state e, the value every new tail state was initialised to. Each thread
+// moves kGatherUnroll vectors per row with all loads issued before the stores.
+constexpr int kGatherThreads = 256;
+constexpr int kGatherUnroll = 4;
+
 template <int VEC>
-__global__ void __launch_bounds__(256) k_gather(Dev d) {
+__global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d) {
+  using T = typename std::conditional<VEC == 4, float4, float>::type;
   pdl_wait();  // everything read here comes from the decision kernel
   const int n = d.ctl->n_miss;
   const int64_t nvec = d.D / VEC;
+  const int64_t stride = (int64_t)gridDim.x * kGatherThreads;
+  const int64_t base = (int64_t)blockIdx.x * kGatherThreads + threadIdx.x;
   for (int r = blockIdx.y; r < n; r += gridDim.y) {
     const int b = d.miss_bt[2 * r], i = d.miss_bt[2 * r + 1];
     const int src = min(i, d.traj[b].e);
-    const float* from = d.X + ((int64_t)b * (d.P + 1) + src % (d.P + 1)) * d.D;
-    float* to = d.batch_x + (int64_t)r * d.D;
-    for (int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; v < nvec;
-         v += (int64_t)gridDim.x * blockDim.x) {
-      if constexpr (VEC == 4) {
-        reinterpret_cast<float4*>(to)[v] = __ldg(reinterpret_cast<const float4*>(from) + v);
-      } else {
-        to[v] = __ldg(from + v);
+    const T* from = reinterpret_cast<const T*>(d.X + ((int64_t)b * (d.P + 1) + src % (d.P + 1)) * d.D);
+    T* to = reinterpret_cast<T*>(d.batch_x + (int64_t)r * d.D);
+    for (int64_t v0 = base; v0 < nvec; v0 += stride * kGatherUnroll) {
+      T buf[kGatherUnroll];
+#pragma unroll
+      for (int u = 0; u < kGatherUnroll; ++u) {
+        const int64_t v = v0 + u * stride;
+        if (v < nvec) buf[u] = __ldg(from + v);
+      }
+#pragma unroll
+      for (int u = 0; u < kGatherUnroll; ++u) {
+        const int64_t v = v0 + u * stride;
+        if (v < nvec) to[v] = buf[u];
       }
     }
   }
@@ -407,17 +421,12 @@ cudaError_t launch_init_plan(const Dev& d, cudaStream_t st) {
 
 cudaError_t launch_gather(const Dev& d, cudaStream_t st) {
   const int rows = min(d.B * d.P, 65535);
-  if (d.D % 4 == 0) {
-    const int64_t nvec = d.D / 4;
-    const int64_t want = (nvec + 255) / 256;
-    const int gx = (int)(want < 64 ? want : 64);
-    return launch_ex(k_gather<4>, dim3(gx, rows), dim3(256), 0, st, 0, d);
-  } else {
-    const int64_t want = (d.D + 255) / 256;
-    const int gx = (int)(want < 256 ? want : 256);
-    return launch_ex(k_gather<1>, dim3(gx, rows), dim3(256), 0, st, 0, d);
-  }
-  return cudaGetLastError();
+  const int vec = (d.D % 4 == 0) ? 4 : 1;
+  const int64_t nvec = d.D / vec;
+  const int64_t want = (nvec + kGatherThreads * kGatherUnroll - 1) / (kGatherThreads * kGatherUnroll);
+  const int gx = (int)(want < 64 ? want : 64);
+  if (vec == 4) return launch_ex(k_gather<4>, dim3(gx, rows), dim3(kGatherThreads), 0, st, 0, d);
+  return launch_ex(k_gather<1>, dim3(gx, rows), dim3(kGatherThreads), 0, st, 0, d);
 }
 
 cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream_t st,

@@ -22,19 +22,24 @@ __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t by
                : "memory");
 }
 
+// One try_wait with a suspend-time hint: the thread may sleep until the phase
+// completes (or about kWaitHintNs passes) instead of spinning.
+constexpr uint32_t kWaitHintNs = 10000;
+
 __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(smem_u32(bar)), "r"(parity)
+      : "r"(smem_u32(bar)), "r"(parity), "r"(kWaitHintNs)
       : "memory");
   return ok != 0;
 }
 
-// Bounded wait on one phase; false when `limit` polls ran out.
+// Bounded wait on one phase; false when `limit` tries ran out (each try may
+// suspend for up to about kWaitHintNs).
 __device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint32_t limit) {
   for (uint32_t n = 0; n < limit; ++n) {
     if (mbar_try_wait(bar, parity)) return true;
@@ -55,6 +60,6 @@ __device__ __forceinline__ void bulk_g2s(void* dst, const void* src, uint32_t by
       : "memory");
 }
 
-constexpr uint32_t kDrainLimit = 1u << 24;
+constexpr uint32_t kDrainLimit = 1u << 17;  // ~1.3 s at the suspend hint
 
 }  // namespace pa

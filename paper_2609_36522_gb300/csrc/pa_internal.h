@@ -100,7 +100,7 @@ struct Dev {
   int bulk_cfg;               // launch shape of the bulk-copy update kernel
   uint32_t wait_limit;        // polls before an mbarrier wait counts as timed out
 };
-constexpr uint32_t kWaitLimit = 1u << 24;
+constexpr uint32_t kWaitLimit = 1u << 17;  // tries of an mbarrier wait (~1.3 s with the suspend hint)
 
 // Programmatic dependent launch (PDL). Every kernel of an iteration is
 // launched with programmatic stream serialization, so it may be scheduled as

@@ -129,7 +129,7 @@ def test_bounded_wait_reports_timeout_and_context_survives():
     with pytest.raises(abi.PaError) as e:
         s.step()
     assert e.value.status == abi.PA_ERR_TIMEOUT
-    abi.pa_debug_set_wait_limit(s.h, 1 << 24)
+    abi.pa_debug_set_wait_limit(s.h, 1 << 17)
     s.init(x0)
     _run(s, g, eps)
     assert np.array_equal(clean, s.result().cpu().numpy())
