@@ -43,10 +43,15 @@ UNIT = "solver steps/s"
 FLUSH_BYTES = 256 << 20
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
-# ncu DRAM bytes of the update kernel per launch, keyed by the sha256 of its
-# source file at capture time (profiles/ has the capture); reported as null
-# when the kernel source has changed since.
-NCU_TRAFFIC = {}
+# ncu DRAM bytes (read + write) of the update kernel per launch, averaged over
+# one generation's launches, keyed by the sha256 of the kernel's source files at
+# capture time and the workload (profiles/ has the capture); reported as null when the kernel
+# source has changed since.
+NCU_TRAFFIC = {
+    ("9ce682d895630e3d", "sd15"): 6244928.0,
+    ("9ce682d895630e3d", "batched"): 24780757.0,
+    ("9ce682d895630e3d", "large"): 71603189.0,
+}
 
 
 def parse_args(argv=None):
@@ -106,10 +111,16 @@ def measured_hbm_gbs():
         return FALLBACK_HBM_GBS, "fallback"
 
 
+UPDATE_KERNEL_SOURCES = ("k_update_bulk.cu", "pa_bulk.cuh", "pa_internal.h")
+
+
 def kernel_source_sha():
     import hashlib
-    p = os.path.join(ROOT, "paper_2609_36522_gb300", "csrc", "k_update_bulk.cu")
-    return hashlib.sha256(open(p, "rb").read()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for name in UPDATE_KERNEL_SOURCES:
+        with open(os.path.join(ROOT, "paper_2609_36522_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def iteration_bytes(log, w: W.Workload):
@@ -382,11 +393,12 @@ def run_ours(args):
     n_upd = args.steps * n_iters
     achieved = upd_bytes.sum() * args.steps / (upd_ms / 1000.0) / 1e9
     sha = kernel_source_sha()
-    traffic = NCU_TRAFFIC.get(sha)
+    traffic = NCU_TRAFFIC.get((sha, args.workload))
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "Picard update (" + ("tile-parallel bulk-copy pipeline"
-                                               if st1["update_kernel"] == 1 else "plain loads") + ")",
+                "kernel": "Picard update (" + ("bulk-copy kernel" if st1["update_kernel"] == 1
+                                               else "plain loads") + ")",
+                "traffic_note": "ncu dram read+write bytes per launch, averaged over one generation",
                 "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
                 "alg_bytes_per_launch": float(upd_bytes.mean()),
                 "avg_launch_us": 1000.0 * upd_ms / max(n_upd, 1)}
