@@ -326,7 +326,7 @@ def run_ours(args):
     nfe, hits = st0["nfe"], st0["hits"]
     upd_bytes, other_bytes = iteration_bytes(log, w)
 
-    # One Picard iteration (gather, denoiser, update, decision: 6 kernels) as a
+    # One Picard iteration (gather, denoiser dots + out, update, decision: 5 kernels) as a
     # CUDA graph; the update kernel's timing events are captured with it.
     s.init(x_dev)
     one_iteration()                       # eager warm-up of every launch path
@@ -336,10 +336,11 @@ def run_ours(args):
     graph = torch.cuda.CUDAGraph()
     s.init(x_dev)
     stream.synchronize()
-    gmm0 = g.launches()
+    gmm0, sol0 = g.launches(), s.stats()["launches"]
     with torch.cuda.graph(graph, stream=stream):
         one_iteration()
-    kernels_per_iter = 3 + (g.launches() - gmm0)   # gather, update, decision + denoiser kernels
+    # gather, update, decision + denoiser kernels
+    kernels_per_iter = (s.stats()["launches"] - sol0) + (g.launches() - gmm0)
 
     def generation(timed):
         s.init(x_dev)
@@ -452,7 +453,7 @@ def run_ours(args):
                        "l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every Picard iteration, outside the timed events"),
                        "timing": "CUDA events around each Picard iteration (one CUDA-graph replay of "
-                                 "gather, denoiser, update, decision kernels) on the launch stream"},
+                                 "the gather, denoiser, update and decision kernels) on the launch stream"},
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
             "solver_step_gbps": gb_step,

@@ -166,13 +166,6 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
  * a tuning aid). Returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
 
-/* Benchmark hook: launch only the Picard-update kernel of the planned
- * iteration, `repeats` times back to back on the solver's stream (between
- * pa_step and pa_submit_eps). Each launch moves the same bytes as the real
- * one but overwrites the window's states with values that are no longer the
- * method's; call pa_init before using the solver's results again. */
-PA_API pa_status pa_bench_update_only(pa_solver* s, const float* batch_eps_dev, int repeats);
-
 /* Fault-handling test hook: the number of tries (each may suspend for about
  * 10 us) after which an mbarrier wait of the bulk-copy update kernel counts
  * as timed out (default 2^17, about a second). With 0

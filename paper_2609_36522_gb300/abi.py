@@ -59,7 +59,6 @@ _PROTOS = {
     "pa_iter_log": (C.c_int, [VP, C.POINTER(C.c_int32), C.c_int, C.POINTER(C.c_int)]),
     "pa_last_reductions": (C.c_int, [VP, VP, VP]),
     "pa_set_update_kernel": (C.c_int, [VP, C.c_int]),
-    "pa_bench_update_only": (C.c_int, [VP, VP, C.c_int]),
     "pa_debug_set_wait_limit": (C.c_int, [VP, C.c_uint32]),
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
     "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.c_int]),
@@ -208,10 +207,6 @@ def pa_last_reductions(h, batch, window):
 
 def pa_set_update_kernel(h, kind):
     return _check("pa_set_update_kernel", lib().pa_set_update_kernel(h, int(kind)))
-
-
-def pa_bench_update_only(h, batch_eps_ptr, repeats):
-    return _check("pa_bench_update_only", lib().pa_bench_update_only(h, _dptr(batch_eps_ptr), int(repeats)))
 
 
 def pa_debug_set_wait_limit(h, polls):

@@ -8,6 +8,7 @@
 //   batch_x [B*P][D]  gathered latents of the misses, rank order
 #include <type_traits>
 
+#include "pa_decide.cuh"
 #include "pa_internal.h"
 
 namespace pa {
@@ -227,42 +228,36 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 }
 
 // ---------------------------------------------------------------------------
-// Decision kernel, one launch of many CTAs:
-//  1. every CTA finishes some of the reductions: one warp per (quantity, b, j)
-//     sums the chunk partials of err[b][j] (Eq. 2) or of the distance of
-//     timestep t+j+1 (Eq. 4) in a fixed order (deterministic), to red_*;
-//  the CTA that finishes last (atomic ticket after a fence; nobody waits) then
-//  2. per trajectory: stride = min(p, 1 + #leading err_j <= tol), advance
-//     t, shrink p = min(P, T - t), frontier e = old t + p, done at t = T;
-//  3. plans the next iteration: a timestep of the new window with a cache
-//     entry (i < e) hits iff delta < tau_cache (strict, Eq. 5), everything
-//     else misses; misses are compacted trajectory-major into miss_bt with a
-//     block-wide prefix sum, and rank[b][j] records each miss's batch row.
+// Decision kernel for the update kernels that leave the reductions unfinished
+// (plain-load and tile forms), one launch of many CTAs: every CTA finishes
+// some of the reductions -- one warp per (quantity, b, j) sums the chunk
+// partials of err[b][j] (Eq. 2) or of the distance of timestep t+j+1 (Eq. 4)
+// in a fixed order (deterministic), to red_* -- and the CTA that finishes
+// last (atomic ticket after a fence; nobody waits) runs decide_plan.
 constexpr int kDecideThreads = 256;
 constexpr int kDecideSmemPairs = 6144;  // (b, j) pairs whose reductions are staged in shared memory
 
 __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
-  __shared__ int s_t[kMaxBatch], s_p[kMaxBatch], s_e[kMaxBatch];
-  __shared__ int s_tn[kMaxBatch], s_pn[kMaxBatch], s_m[kMaxBatch], s_h1[kMaxBatch];
-  __shared__ int s_om[kMaxBatch], s_oh1[kMaxBatch];
-  __shared__ int s_warp[kDecideThreads / 32];
-  __shared__ int s_total, s_active, s_iter, s_last;
+  __shared__ int s_last;
   extern __shared__ float s_red[];  // [2][B*P] when B*P <= kDecideSmemPairs
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kDecideThreads / 32;
-  const int B = d.B, P = d.P, T = d.T;
-  const int npair = B * P;
+  const int npair = d.B * d.P;
 
   pdl_wait();  // the partials come from the update kernel
-  // 1. reductions, one warp per item (positions beyond a trajectory's window
-  // are reduced too; their values are never used)
   const int item = blockIdx.x * nwarps + warp;
   if (item < 2 * npair) {
     const int which = item / npair, pr = item % npair;
     const float* src = (which ? d.part_del : d.part_err) + (int64_t)pr * nchunk;
     float acc[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll 4
-    for (int c = lane, u = 0; c < nchunk; c += 32, u = (u + 1) & 3) acc[u] += src[c];
+    int c = lane;
+    for (; c + 96 < nchunk; c += 128) {
+      acc[0] += src[c];
+      acc[1] += src[c + 32];
+      acc[2] += src[c + 64];
+      acc[3] += src[c + 96];
+    }
+    for (; c < nchunk; c += 32) acc[0] += src[c];
     float v = (acc[0] + acc[1]) + (acc[2] + acc[3]);
     v = warp_sum(v);
     if (lane == 0) (which ? d.red_del : d.red_err)[pr] = v / (float)d.D;
@@ -276,21 +271,8 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
   __syncthreads();
   if (!s_last) return;
   __threadfence();  // the other CTAs' reductions are visible from here on
+  if (tid == 0) d.ctl->ticket = 0u;  // ready for the next launch
   const bool in_smem = npair <= kDecideSmemPairs;
-  float* red_e = in_smem ? s_red : d.red_err;
-  float* red_d = in_smem ? s_red + npair : d.red_del;
-  if (tid == 0) {
-    d.ctl->ticket = 0u;  // ready for the next launch
-    s_active = d.ctl->n_active;
-    s_iter = d.ctl->iter;
-  }
-  for (int b = tid; b < B; b += kDecideThreads) {
-    const Traj tr = d.traj[b];
-    s_t[b] = tr.t; s_p[b] = tr.p; s_e[b] = tr.e;
-    s_om[b] = tr.m; s_oh1[b] = tr.h1;
-    s_m[b] = 0;
-    s_h1[b] = 0;
-  }
   if (in_smem) {
     for (int q = tid; q < npair; q += kDecideThreads) {
       s_red[q] = __ldcg(d.red_err + q);
@@ -298,118 +280,7 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
     }
   }
   __syncthreads();
-  if (s_active == 0) return;  // finished: iterating further is a no-op
-  const int iter = s_iter;
-
-  // 2. window advance, one warp per trajectory
-  for (int b = warp; b < B; b += nwarps) {
-    const int t = s_t[b], p = s_p[b];
-    if (p == 0) {
-      if (lane == 0) {
-        s_tn[b] = t; s_pn[b] = 0;
-        int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
-        for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
-        lg[0] = t;
-      }
-      continue;
-    }
-    int lead = p;
-    for (int j0 = 0; j0 < p; j0 += 32) {
-      const int j = j0 + lane;
-      const bool fail = (j < p) && !((double)red_e[b * P + j] <= d.tol);
-      const unsigned m = __ballot_sync(0xffffffffu, fail);
-      if (m) {
-        lead = j0 + __ffs(m) - 1;
-        break;
-      }
-    }
-    if (lane == 0) {
-      const int stride = min(p, 1 + lead);
-      const int tn = t + stride;
-      s_tn[b] = tn;
-      s_pn[b] = min(P, T - tn);
-      int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
-      lg[0] = t; lg[1] = p; lg[2] = s_om[b]; lg[3] = stride;
-      lg[4] = s_e[b]; lg[5] = s_oh1[b]; lg[6] = 0; lg[7] = 0;
-    }
-  }
-  __syncthreads();
-
-  // 3. hit/miss plan of the next iteration and its compaction
-  const int N = B * P;
-  const int per = (N + kDecideThreads - 1) / kDecideThreads;
-  const int q0 = tid * per, q1 = min(N, q0 + per);
-  auto is_miss = [&](int q) -> int {
-    const int b = q / P, j = q % P;
-    if (j >= s_pn[b]) return 0;
-    const int i = s_tn[b] + j;
-    const int en = s_t[b] + s_p[b];  // new frontier
-    if (i >= en) return 1;           // first entry
-    const int jo = i - s_t[b] - 1;   // delta of timestep i was computed at old position jo
-    return ((double)red_d[b * P + jo] < d.cache_thresh) ? 0 : 1;
-  };
-  int cnt = 0;
-  for (int q = q0; q < q1; ++q) cnt += is_miss(q);
-  // block exclusive scan of cnt
-  int incl = cnt;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int v = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += v;
-  }
-  if (lane == 31) s_warp[warp] = incl;
-  __syncthreads();
-  if (warp == 0) {
-    static_assert(nwarps <= 32, "one warp scans the warp totals");
-    const int w = lane < nwarps ? s_warp[lane] : 0;
-    int wi = w;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, wi, o);
-      if (lane >= o) wi += v;
-    }
-    if (lane < nwarps) s_warp[lane] = wi - w;  // exclusive
-    if (lane == 31) s_total = wi;
-  }
-  __syncthreads();
-  int r = s_warp[warp] + incl - cnt;
-  for (int q = q0; q < q1; ++q) {
-    const int b = q / P, j = q % P;
-    if (is_miss(q)) {
-      d.rank[q] = r;
-      d.miss_bt[2 * r] = b;
-      d.miss_bt[2 * r + 1] = s_tn[b] + j;
-      atomicAdd(&s_m[b], 1);
-      ++r;
-    } else {
-      d.rank[q] = -1;
-      if (j >= 1 && j < s_pn[b]) atomicAdd(&s_h1[b], 1);
-    }
-  }
-  __syncthreads();
-  int pts = 0;
-  for (int b = 0; b < B; ++b) pts += s_pn[b];
-  for (int b = tid; b < B; b += kDecideThreads) {
-    Traj tr{};
-    tr.t = s_tn[b];
-    tr.p = s_pn[b];
-    tr.e = (s_p[b] > 0) ? s_t[b] + s_p[b] : s_e[b];
-    tr.done = (s_pn[b] == 0);
-    tr.m = s_m[b];
-    tr.h1 = s_h1[b];
-    if (tr.t > T || tr.e < tr.t) set_status(d.ctl, kDevBadState);
-    d.traj[b] = tr;
-  }
-  if (tid == 0) {
-    int act = 0;
-    for (int b = 0; b < B; ++b) act += (s_pn[b] > 0);
-    const int n = s_total;
-    d.ctl->n_miss = n;
-    d.ctl->n_active = act;
-    d.ctl->iter = iter + 1;
-    d.ctl->nfe += n;
-    d.ctl->hits += pts - n;
-  }
+  decide_plan<kDecideThreads>(d, in_smem ? s_red : d.red_err, in_smem ? s_red + npair : d.red_del);
 }
 
 }  // namespace

@@ -1,0 +1,158 @@
+// The serial part of one Picard iteration's decision (a10, a2, a3), run by a
+// single CTA once every per-position reduction is finished (the last CTA of
+// the decision kernel in k_solver.cu).
+#pragma once
+
+#include "pa_internal.h"
+
+namespace pa {
+
+// red_e[b*P + j]: Eq. 2 error of window position j of trajectory b (already
+// divided by D); red_d[b*P + j]: Eq. 4 distance of timestep t+j+1 (divided by
+// D). Only positions j < p_b are read. With NT threads the CTA
+//  1. per trajectory: stride = min(p, 1 + #leading err_j <= tol) (warp
+//     ballots), advances t, shrinks p = min(P, T - t), sets the frontier
+//     e = old t + p, done at t = T, and writes the iteration log;
+//  2. plans the next iteration: a timestep of the new window with a cache
+//     entry (i < e) hits iff delta < tau_cache (strict, Eq. 5), everything else
+//     misses; misses are compacted trajectory-major into miss_bt with a
+//     block-wide prefix sum, and rank[b][j] records each miss's batch row;
+//  3. updates the counters (n_miss, n_active, iter, nfe, hits).
+template <int NT>
+__device__ void decide_plan(const Dev& d, const float* red_e, const float* red_d) {
+  __shared__ int s_t[kMaxBatch], s_p[kMaxBatch], s_e[kMaxBatch];
+  __shared__ int s_tn[kMaxBatch], s_pn[kMaxBatch], s_m[kMaxBatch], s_h1[kMaxBatch];
+  __shared__ int s_om[kMaxBatch], s_oh1[kMaxBatch];
+  __shared__ int s_warp[NT / 32];
+  __shared__ int s_total, s_active, s_iter;
+  constexpr int nwarps = NT / 32;
+  static_assert(nwarps <= 32, "one warp scans the warp totals");
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int B = d.B, P = d.P, T = d.T;
+  if (tid == 0) {
+    s_active = d.ctl->n_active;
+    s_iter = d.ctl->iter;
+  }
+  for (int b = tid; b < B; b += NT) {
+    const Traj tr = d.traj[b];
+    s_t[b] = tr.t; s_p[b] = tr.p; s_e[b] = tr.e;
+    s_om[b] = tr.m; s_oh1[b] = tr.h1;
+    s_m[b] = 0;
+    s_h1[b] = 0;
+  }
+  __syncthreads();
+  if (s_active == 0) return;  // finished: iterating further is a no-op
+  const int iter = s_iter;
+
+  // 1. window advance, one warp per trajectory
+  for (int b = warp; b < B; b += nwarps) {
+    const int t = s_t[b], p = s_p[b];
+    if (p == 0) {
+      if (lane == 0) {
+        s_tn[b] = t; s_pn[b] = 0;
+        int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+        for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
+        lg[0] = t;
+      }
+      continue;
+    }
+    int lead = p;
+    for (int j0 = 0; j0 < p; j0 += 32) {
+      const int j = j0 + lane;
+      const bool fail = (j < p) && !((double)red_e[b * P + j] <= d.tol);
+      const unsigned m = __ballot_sync(0xffffffffu, fail);
+      if (m) {
+        lead = j0 + __ffs(m) - 1;
+        break;
+      }
+    }
+    if (lane == 0) {
+      const int stride = min(p, 1 + lead);
+      const int tn = t + stride;
+      s_tn[b] = tn;
+      s_pn[b] = min(P, T - tn);
+      int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+      lg[0] = t; lg[1] = p; lg[2] = s_om[b]; lg[3] = stride;
+      lg[4] = s_e[b]; lg[5] = s_oh1[b]; lg[6] = 0; lg[7] = 0;
+    }
+  }
+  __syncthreads();
+
+  // 2. hit/miss plan of the next iteration and its compaction
+  const int N = B * P;
+  const int per = (N + NT - 1) / NT;
+  const int q0 = tid * per, q1 = min(N, q0 + per);
+  auto is_miss = [&](int q) -> int {
+    const int b = q / P, j = q % P;
+    if (j >= s_pn[b]) return 0;
+    const int i = s_tn[b] + j;
+    const int en = s_t[b] + s_p[b];  // new frontier
+    if (i >= en) return 1;           // first entry
+    const int jo = i - s_t[b] - 1;   // delta of timestep i was computed at old position jo
+    return ((double)red_d[b * P + jo] < d.cache_thresh) ? 0 : 1;
+  };
+  int cnt = 0;
+  for (int q = q0; q < q1; ++q) cnt += is_miss(q);
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_warp[warp] = incl;
+  __syncthreads();
+  if (warp == 0) {
+    const int w = lane < nwarps ? s_warp[lane] : 0;
+    int wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += v;
+    }
+    if (lane < nwarps) s_warp[lane] = wi - w;  // exclusive
+    if (lane == 31) s_total = wi;
+  }
+  __syncthreads();
+  int r = s_warp[warp] + incl - cnt;
+  for (int q = q0; q < q1; ++q) {
+    const int b = q / P, j = q % P;
+    if (is_miss(q)) {
+      d.rank[q] = r;
+      d.miss_bt[2 * r] = b;
+      d.miss_bt[2 * r + 1] = s_tn[b] + j;
+      atomicAdd(&s_m[b], 1);
+      ++r;
+    } else {
+      d.rank[q] = -1;
+      if (j >= 1 && j < s_pn[b]) atomicAdd(&s_h1[b], 1);
+    }
+  }
+  __syncthreads();
+
+  // 3. trajectories and counters
+  int pts = 0;
+  for (int b = 0; b < B; ++b) pts += s_pn[b];
+  for (int b = tid; b < B; b += NT) {
+    Traj tr{};
+    tr.t = s_tn[b];
+    tr.p = s_pn[b];
+    tr.e = (s_p[b] > 0) ? s_t[b] + s_p[b] : s_e[b];
+    tr.done = (s_pn[b] == 0);
+    tr.m = s_m[b];
+    tr.h1 = s_h1[b];
+    if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
+    d.traj[b] = tr;
+  }
+  if (tid == 0) {
+    int act = 0;
+    for (int b = 0; b < B; ++b) act += (s_pn[b] > 0);
+    const int n = s_total;
+    d.ctl->n_miss = n;
+    d.ctl->n_active = act;
+    d.ctl->iter = iter + 1;
+    d.ctl->nfe += n;
+    d.ctl->hits += pts - n;
+  }
+}
+
+}  // namespace pa

@@ -400,23 +400,6 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   return PA_OK;
 }
 
-pa_status pa_bench_update_only(pa_solver* s, const float* batch_eps_dev, int repeats) {
-  if (!s || !batch_eps_dev || repeats < 1) return arg_fail("pa_bench_update_only: bad argument");
-  if (s->state != St::Stepped) return state_fail("pa_bench_update_only");
-  for (int r = 0; r < repeats; ++r) {
-    int nchunk = 0;
-    cudaError_t e;
-    if (s->update_kind == 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
-      e = pa::launch_update_bulk(s->d, batch_eps_dev, s->st, &nchunk);
-    } else {
-      e = pa::launch_update_plain(s->d, batch_eps_dev, s->st, &nchunk);
-    }
-    s->launches++;
-    if (e != cudaSuccess) return cuda_fail("pa_bench_update_only", e);
-  }
-  return PA_OK;
-}
-
 pa_status pa_debug_set_wait_limit(pa_solver* s, uint32_t polls) {
   if (!s) return arg_fail("pa_debug_set_wait_limit: solver is NULL");
   s->d.wait_limit = polls ? polls : 0u;

@@ -122,30 +122,84 @@ def test_host_x_init_equals_device_x_init():
     assert np.array_equal(a["x_final"], b["x_final"])
 
 
-def test_gmm_kernel_against_oracle():
-    """The mixture denoiser alone, on rows spread over the whole schedule."""
+def _gmm_rows(w, n, seed=0):
+    a, _, mu = W.inputs(w)
+    rng = np.random.default_rng(seed)
+    idx = np.linspace(0, w.T - 1, n).astype(np.int32)
+    comp = rng.integers(0, w.K, n)
+    x = (np.sqrt(a[idx])[:, None] * (mu[comp] + 0.5 * rng.standard_normal((n, w.D)))
+         + np.sqrt(1 - a[idx])[:, None] * rng.standard_normal((n, w.D))).astype(np.float32)
+    miss = np.stack([np.zeros(n, np.int32), idx], axis=1).astype(np.int32)
+    return a, mu, idx, x, miss
+
+
+@pytest.mark.parametrize("wname,n,max_rows", [("sd15", 48, 48), ("sd15", 1, 100), ("sd15", 37, 100),
+                                              ("sd15", 100, 100), ("batched", 256, 256),
+                                              ("large", 48, 48), ("tiny", 5, 8)])
+def test_gmm_kernel_against_oracle(wname, n, max_rows):
+    """The mixture denoiser alone, on rows spread over the whole schedule, with
+    the device row count below the capacity, and over three calls in a row
+    (the fixed-point accumulators and the tickets are reused)."""
     import torch
     from paper_2609_36522_gb300.solver import GmmDenoiser
-    for w in (W.SD15, W.LARGE):
-        a, _, mu = W.inputs(w)
-        n = 48
-        rng = np.random.default_rng(0)
-        idx = np.linspace(0, w.T - 1, n).astype(np.int32)
-        comp = rng.integers(0, w.K, n)
-        x = (np.sqrt(a[idx])[:, None] * (mu[comp] + 0.5 * rng.standard_normal((n, w.D)))
-             + np.sqrt(1 - a[idx])[:, None] * rng.standard_normal((n, w.D))).astype(np.float32)
-        miss = np.stack([np.zeros(n, np.int32), idx], axis=1).astype(np.int32)
-        dev = torch.device("cuda")
-        g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, n)
+    w = W.ALL[wname]
+    a, mu, idx, x, miss = _gmm_rows(w, n)
+    dev = torch.device("cuda")
+    g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows)
+    xd = torch.zeros(max_rows, w.D, dtype=torch.float32, device=dev)
+    xd[:n] = torch.from_numpy(x).to(dev)
+    md = torch.zeros(max_rows, 2, dtype=torch.int32, device=dev)
+    md[:n] = torch.from_numpy(miss).to(dev)
+    nd = torch.tensor([n], dtype=torch.int32, device=dev)
+    outs = []
+    for _ in range(3):
+        out = torch.full_like(xd, float("nan"))
+        g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), out)
+        outs.append(out)
+    torch.cuda.synchronize()
+    from paper_2609_36522_gb300 import abi
+    abi.pa_gmm_check(g.h)
+    got = outs[0][:n].cpu().numpy().astype(np.float64)
+    want = gmm_eps(x.astype(np.float64), a[idx], mu.astype(np.float64), w.gmm_std)
+    rel = np.abs(got - want).max(axis=1) / np.abs(want).max(axis=1)
+    assert rel.max() <= 2e-6, rel.max()
+    for o in outs[1:]:
+        assert torch.equal(o[:n], outs[0][:n])       # bitwise reproducible
+    assert torch.isnan(outs[0][n:]).all()            # rows past the count are not written
+    g.close()
+
+
+def test_gmm_in_cuda_graph():
+    """The denoiser captured in a CUDA graph and replayed gives the eager
+    result (bitwise), with a device row count that changes between replays."""
+    import torch
+    from paper_2609_36522_gb300.solver import GmmDenoiser
+    w = W.SD15
+    n = 100
+    a, mu, idx, x, miss = _gmm_rows(w, n, seed=3)
+    dev = torch.device("cuda")
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, n, stream=st)
         xd = torch.from_numpy(x).to(dev)
         md = torch.from_numpy(miss).to(dev)
         nd = torch.tensor([n], dtype=torch.int32, device=dev)
-        out = torch.empty_like(xd)
-        g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), out)
-        got = out.cpu().numpy().astype(np.float64)
-        want = gmm_eps(x.astype(np.float64), a[idx], mu.astype(np.float64), w.gmm_std)
-        rel = np.abs(got - want).max(axis=1) / np.abs(want).max(axis=1)
-        assert rel.max() <= 2e-6, rel.max()
+        want = torch.empty_like(xd)
+        g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), want)
+        got = torch.empty_like(xd)
+        st.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=st):
+            g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), got)
+        for m in (n, 17, n):
+            nd.fill_(m)
+            got.fill_(float("nan"))
+            graph.replay()
+            st.synchronize()
+            assert torch.equal(got[:m], want[:m])
+            assert torch.isnan(got[m:]).all()
+        from paper_2609_36522_gb300 import abi
+        abi.pa_gmm_check(g.h)
         g.close()
 
 
