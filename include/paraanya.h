@@ -162,7 +162,7 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
 /* Select the Picard-update kernel: 0 = plain loads, 1 = bulk-copy pipeline
  * (default when D % 4 == 0; it falls back to plain loads for a batch_eps
  * pointer that is not 16-byte aligned), 100 + n = bulk-copy pipeline with
- * launch shape n (0..9; columns per lane, warps per CTA, pipeline depth --
+ * launch shape n (0..11; columns per lane, warps per CTA, pipeline depth --
  * a tuning aid). Returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
 

@@ -80,7 +80,10 @@ struct Vec {
 template <int V>
 __device__ __forceinline__ Vec<V> ldv(const float* p) {
   Vec<V> r;
-  if constexpr (V == 2) {
+  if constexpr (V == 4) {
+    const float4 q = *reinterpret_cast<const float4*>(p);
+    r.a[0] = q.x; r.a[1] = q.y; r.a[2] = q.z; r.a[3] = q.w;
+  } else if constexpr (V == 2) {
     const float2 q = *reinterpret_cast<const float2*>(p);
     r.a[0] = q.x; r.a[1] = q.y;
   } else {
@@ -91,7 +94,9 @@ __device__ __forceinline__ Vec<V> ldv(const float* p) {
 
 template <int V>
 __device__ __forceinline__ void stv(float* p, const Vec<V>& v) {
-  if constexpr (V == 2) {
+  if constexpr (V == 4) {
+    *reinterpret_cast<float4*>(p) = make_float4(v.a[0], v.a[1], v.a[2], v.a[3]);
+  } else if constexpr (V == 2) {
     *reinterpret_cast<float2*>(p) = make_float2(v.a[0], v.a[1]);
   } else {
     *p = v.a[0];
@@ -710,9 +715,30 @@ bool update_bulk_supported(const Dev& d, const float* batch_eps) {
   return d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0;
 }
 
+// Four columns per lane halve the per-element bookkeeping and the strip
+// partials, but quadruple the shared memory of a strip; they pay off while the
+// grid still fills the GPU in about one wave (window 100 at 4x64x64: 128 CTAs)
+// or several CTAs fit per SM (window 32), not for multi-wave grids of one CTA
+// per SM (window 64 at 4x128x128).
+bool prefer_wide_strips(const Dev& d) {
+  if (!seg_fits<4, 8>(d)) return false;
+  static int nsm[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (nsm[dev] == 0 && cudaDeviceGetAttribute(&nsm[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) {
+    nsm[dev] = 0;
+    return false;
+  }
+  const size_t smem = SegShape<4, 8>::smem_bytes(d.P) + 4096;  // + static shared memory and reserve
+  const int per_sm = (int)((size_t)(228 * 1024) / smem);
+  const int64_t grid = (int64_t)d.B * ((d.D + SegShape<4, 8>::SEG - 1) / SegShape<4, 8>::SEG);
+  return per_sm >= 2 || grid <= nsm[dev];
+}
+
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
   switch (d.bulk_cfg) {
     case 0:  // whole window in shared memory when it fits, else the tiled pipeline
+      if (prefer_wide_strips(d)) return launch_seg<4, 8>(d, batch_eps, st, nchunk_out);
       if (seg_fits<2, 8>(d)) return launch_seg<2, 8>(d, batch_eps, st, nchunk_out);
       return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
     case 1: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
@@ -729,6 +755,10 @@ cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_
     case 8: return seg_fits<2, 4>(d) ? launch_seg<2, 4>(d, batch_eps, st, nchunk_out)
                                      : launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
     case 9: return launch_tile<2, 8, 2, false, true>(d, batch_eps, st, nchunk_out);
+    case 10: return seg_fits<4, 8>(d) ? launch_seg<4, 8>(d, batch_eps, st, nchunk_out)
+                                      : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 11: return seg_fits<4, 4>(d) ? launch_seg<4, 4>(d, batch_eps, st, nchunk_out)
+                                      : launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
     default: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
   }
 }

@@ -203,7 +203,7 @@ def test_gmm_in_cuda_graph():
         g.close()
 
 
-@pytest.mark.parametrize("kind", [0, 1] + list(range(100, 110)))
+@pytest.mark.parametrize("kind", [0, 1] + list(range(100, 112)))
 def test_update_kernels_agree(kind):
     """Plain-load and tile-parallel bulk-copy update kernels (every launch
     shape) take the same decisions and agree with the oracle; their states
