@@ -65,6 +65,7 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-kernel", type=int, default=None)
+    ap.add_argument("--gmm-form", type=int, default=None, help="denoiser dot products: 1 tensor cores, 0 CUDA cores")
     ap.add_argument("--oracle-sample", type=float, default=None, help=argparse.SUPPRESS)
     return ap.parse_args(argv)
 
@@ -301,6 +302,8 @@ def run_ours(args):
         s.set_update_kernel(args.update_kernel)
     max_rows = w.batch * s.window
     g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows, stream=stream)
+    if args.gmm_form is not None:
+        g.set_form(args.gmm_form)
     eps = torch.empty(max_rows, w.D, dtype=torch.float32, device=dev)
     x_dev = torch.from_numpy(x0).to(dev)
     flush = None if args.no_flush else torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
@@ -449,6 +452,8 @@ def run_ours(args):
                        "picard_iters_per_step": n_iters, "global_batch": w.batch * world,
                        "seq_len": w.T, "window": w.window, "latent": "x".join(map(str, w.latent_shape)),
                        "mixture_components": w.K, "tol": w.tol, "cache_thresh": w.cache_thresh,
+                       "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
+                                                 if g.form() == 1 else "CUDA cores (fp32 FMA)"),
                        "parallelism": f"replicas x{world} (independent trajectories)",
                        "l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every Picard iteration, outside the timed events"),

@@ -219,6 +219,22 @@ PA_API pa_status pa_gmm_check(pa_gmm* g);
 /* Kernels launched by this handle since pa_gmm_create. */
 PA_API int64_t pa_gmm_launches(const pa_gmm* g);
 
+/* How pa_gmm_eps forms the dot products x . mu_k (a choice of this library;
+ * the paper has no counterpart). form 1: on the tensor cores (tcgen05,
+ * kind::tf32, every operand split into two tf32 parts and three products
+ * summed, which keeps fp32 accuracy), 128 rows x 128 columns per CTA;
+ * available when the GPU is of the sm_100 family, D % 4 == 0 and the means
+ * are 16-byte aligned, and selected by pa_gmm_create when also K > 16.
+ * form 0: fp32 FMA on the CUDA cores (the default for K <= 16, where the
+ * contraction is too small for the tensor cores to pay off). A
+ * call whose batch_x is not 16-byte aligned uses form 0. The forms agree to
+ * fp32 rounding; each is bitwise reproducible. Returns PA_ERR_ARG for form 1
+ * when it is not available. */
+PA_API pa_status pa_gmm_set_form(pa_gmm* g, int form);
+
+/* The form pa_gmm_eps uses: 1 or 0, -1 for NULL. */
+PA_API int pa_gmm_form(const pa_gmm* g);
+
 PA_API void pa_gmm_destroy(pa_gmm* g);
 
 /* pa_gmm_eps without a handle and without any device allocation (the paper
@@ -230,13 +246,15 @@ PA_API void pa_gmm_destroy(pa_gmm* g);
  * device's allocator. The caller passes the inputs (means_dev [K][D],
  * alphas_cumprod on the HOST [T+1], batch_x_dev [n_rows][D], miss_bt_dev
  * [n_rows][2] whose second entries are sampling indices < T) and the output
- * batch_eps_dev [n_rows][D]; results equal pa_gmm_eps's for the same inputs.
+ * batch_eps_dev [n_rows][D]; the dot products are formed on the CUDA cores
+ * (pa_gmm_set_form's form 0), and results agree with pa_gmm_eps's to fp32
+ * rounding.
  *
  * Scratch lives in one fixed 4 MiB device array inside this library (every
  * GPU that loads the library holds it until the process exits). Sizes whose
- * scratch (3T coefficients, K norms, n_rows*K dot-product accumulators and
- * responsibilities) would exceed 4 MiB are rejected with PA_ERR_ARG and a
- * message naming the bytes needed; use pa_gmm_create/pa_gmm_eps then.
+ * scratch (3T coefficients, K norms, two sets of n_rows*K int64 dot-product
+ * accumulators) would exceed 4 MiB are rejected with PA_ERR_ARG and a message
+ * naming the bytes needed; use pa_gmm_create/pa_gmm_eps then.
  *
  * The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress) with that device current; make that first call

@@ -69,6 +69,8 @@ _PROTOS = {
     "pa_gmm_eps": (C.c_int, [VP, VP, VP, VP, VP]),
     "pa_gmm_check": (C.c_int, [VP]),
     "pa_gmm_launches": (C.c_int64, [VP]),
+    "pa_gmm_set_form": (C.c_int, [VP, C.c_int]),
+    "pa_gmm_form": (C.c_int, [VP]),
     "pa_gmm_destroy": (None, [VP]),
     "pa_gmm_eps_noalloc": (C.c_int, [VP, C.c_int, C.c_int64, C.c_double, C.POINTER(C.c_double),
                                      C.c_int, VP, VP, C.c_int, VP, VP]),
@@ -254,6 +256,14 @@ def pa_gmm_check(g):
 
 def pa_gmm_launches(g):
     return int(lib().pa_gmm_launches(g))
+
+
+def pa_gmm_set_form(g, form):
+    return _check("pa_gmm_set_form", lib().pa_gmm_set_form(g, int(form)))
+
+
+def pa_gmm_form(g):
+    return int(lib().pa_gmm_form(g))
 
 
 def pa_gmm_destroy(g):

@@ -6,17 +6,31 @@
 //   r = softmax(logit)   (the common -||x||^2 / (2 v) term cancels)
 //   eps = sqrt(1 - a) / v * (x - sqrt(a) sum_k r_k mu_k)
 //
-// Two kernels per call, each with a single load phase:
-//   k_gmm_dots     split-K contraction G = X M^T over bulk-staged 16-row tiles
-//                  (register-tiled 4 rows x 8 components per thread); the last
-//                  CTA of each row block sums the chunks in a fixed order and
-//                  applies the logits and the max-subtracted softmax
-//   k_gmm_out      eps = a x - a sqrt(a) R M over bulk-staged 16-row x
-//                  256-column tiles (4 x 4 outputs per thread)
+// Two kernels per call:
+//   dot products   G = X M^T, split over column chunks of D, either on the
+//                  tensor cores (k_gmm_dots_tc: tcgen05, tf32 operands split
+//                  in two parts for fp32 accuracy) or on the CUDA cores
+//                  (k_gmm_dots: bulk-staged 16-row tiles, 4 rows x 8
+//                  components per thread); each CTA adds its chunk sums, in
+//                  2^-32 fixed point, into int64 accumulators with integer
+//                  atomics (exact: the order of arrival does not matter)
+//   k_gmm_out      per 16-row block: logits and max-subtracted softmax of its
+//                  rows from the accumulators, then eps = a x - a sqrt(a) R M
+//                  over bulk-staged 16-row x 256-column tiles (4 x 4 outputs
+//                  per thread)
+// The accumulators come in two sets used in turn. A call's dot-product kernel
+// reads the handle's epoch e, accumulates into set e mod 2, clears the other
+// set (read by the previous call's output kernel, which has completed) and
+// records e for the output kernel; the output kernel reads set e mod 2 and
+// advances the epoch. No kernel waits for another CTA, and the state lives on
+// the device, so a captured CUDA graph replays correctly.
 // Per-timestep scalars (sqrt(a), 1/(2v), sqrt(1-a)/v) are computed on the
 // host in fp64 from alpha-bar and stored in fp32, so 1 - a never cancels in
 // fp32. Reductions run in a fixed order: results are bitwise reproducible.
+#include <cooperative_groups.h>
+
 #include <cmath>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <string>
@@ -25,12 +39,15 @@
 #include "../../include/paraanya.h"
 #include "pa_bulk.cuh"
 #include "pa_internal.h"
+#include "pa_tcgen05.cuh"
 
 namespace pa {
 void set_error(const std::string& msg);  // pa_solver.cpp
 }
 
 namespace {
+
+namespace cg = cooperative_groups;
 
 using pa::pdl_trigger;
 using pa::pdl_wait;
@@ -39,20 +56,55 @@ using pa::fence_barrier_init;
 using pa::mbar_arrive_expect_tx;
 using pa::mbar_init;
 using pa::mbar_wait_bounded;
+using pa::smem_u32;
+using pa::tc_commit;
+using pa::tc_fence_after_sync;
+using pa::tc_fence_before_sync;
+using pa::tc_idesc_tf32;
+using pa::tc_mma_tf32;
+using pa::tc_smem_desc;
+using pa::tmem_alloc;
+using pa::tmem_dealloc;
+using pa::tmem_ld16;
+using pa::to_tf32;
+using pa::fence_proxy_async_smem;
 
 constexpr int kMaxK = 128;
 constexpr int kThreads = 256;
 constexpr int kDotRows = 16;     // rows per dots CTA (two per warp)
-constexpr int kKTile = 16;       // components accumulated per pass
 constexpr int kOutRows = 16;     // rows per output CTA
 constexpr int kOutCols = 256;    // columns per output CTA (four per thread)
 constexpr size_t kDotSmemBudget = 96 * 1024;
 constexpr float kDotScale = 4294967296.f;  // 2^32: fixed-point scale of the dot-product accumulators
 
+// tensor-core dot products: rows per CTA (the MMA's M), columns per CTA
+constexpr int kTcRows = 128;
+constexpr int kTcCols = 128;  // 16 MMA steps of 8
+constexpr int kTcThreads = 256;
+constexpr int kTcCluster = 8;            // column chunks per thread-block cluster ...
+constexpr int kTcClusterMinChunks = 256;  // ... when there are this many chunks (fewer atomics per accumulator)
+constexpr int kTcMinK = 16;               // tensor-core dot products by default above this many components
+
+// the MMA's N: K rounded up to 16, 32, 64 or 128 (padded means are zero)
+__host__ __device__ inline int tc_npad(int K) {
+  int n = 16;
+  while (n < K) n <<= 1;
+  return n;
+}
+// floats of one column chunk's means image: hi and lo, Kp rows each
+__host__ __device__ inline size_t tc_mu_chunk_floats(int K) { return (size_t)2 * tc_npad(K) * kTcCols; }
+
 struct GmmLayout {
-  size_t coef, mnorm, gacc, R, rowc, tickets, status, total;
-  int nchunk;       // D-chunks of the dots kernel
+  size_t coef, mnorm, gacc, epoch, status, mu_img, total;
+  int tc_chunks;    // column chunks of the tensor-core dot products (whole clusters)
+  int nchunk;       // D-chunks of the CUDA-core dots kernel
   int chunk;        // columns per chunk
+};
+
+// Which accumulator set a call uses (see the file comment).
+struct GmmEpoch {
+  uint32_t epoch;   // advanced by the output kernel
+  uint32_t cur;     // the epoch of the dot products just formed
 };
 
 size_t dots_smem_bytes(int K, int chunk) {
@@ -80,11 +132,11 @@ GmmLayout gmm_layout(int K, int64_t D, int max_rows, int T) {
   L.nchunk = (int)((D + L.chunk - 1) / L.chunk);
   L.coef = take((size_t)3 * T * sizeof(float));
   L.mnorm = take((size_t)K * sizeof(float));
-  L.gacc = take((size_t)max_rows * K * sizeof(long long));
-  L.R = take((size_t)max_rows * K * sizeof(float));
-  L.rowc = take((size_t)max_rows * 2 * sizeof(float));
-  L.tickets = take((size_t)((max_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t));
+  L.gacc = take((size_t)2 * max_rows * K * sizeof(long long));  // two sets, used in turn
+  L.epoch = take(sizeof(GmmEpoch));
   L.status = take(sizeof(int32_t));
+  L.tc_chunks = (int)((D + kTcCols - 1) / kTcCols + kTcCluster - 1) / kTcCluster * kTcCluster;  // whole clusters
+  L.mu_img = take((size_t)L.tc_chunks * tc_mu_chunk_floats(K) * sizeof(float));
   L.total = o;
   return L;
 }
@@ -147,34 +199,34 @@ __device__ __forceinline__ bool wait_staged(bool bulk, uint64_t* bar, int32_t* s
   return false;
 }
 
-// Dot products and softmax, one kernel: a CTA stages 16 rows x `chunk`
-// columns of X and the same columns of every mean, each thread accumulates a
-// 4-row x 8-component block over a column split (register tiling: 12 shared
-// loads per 32 FMAs), and the column splits are summed in a fixed order
-// through shared memory. Chunks are combined by adding each CTA's sums,
-// rounded to fixed point (2^-32), into int64 accumulators gacc[r][k] with
-// atomics: integer addition is exact, so the result does not depend on the
-// order in which CTAs arrive. The CTA that finishes a row block last (atomic
-// ticket after a fence, nobody waits) reads the finished dot products, clears
-// the accumulators for the next call, and applies the logits and the
-// max-subtracted softmax -> R[r][k], rowc[r].
+// Start of a dot-product kernel: the accumulator set of this call (epoch e),
+// the other set cleared by all CTAs together (every CTA, also those without
+// rows), and e recorded for the output kernel.
+__device__ __forceinline__ long long* begin_dots(long long* gacc2, GmmEpoch* ep, int64_t set_size) {
+  const uint32_t e = ep->epoch;  // advanced by the previous call's output kernel, long finished
+  long long* other = gacc2 + (int64_t)((e + 1u) & 1u) * set_size;
+  const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x;
+  const int64_t nthr = (int64_t)gridDim.x * gridDim.y * blockDim.x;
+  for (int64_t q = cta * blockDim.x + threadIdx.x; q < set_size; q += nthr) other[q] = 0;
+  if (cta == 0 && threadIdx.x == 0) ep->cur = e;
+  return gacc2 + (int64_t)(e & 1u) * set_size;
+}
+
+// Dot products on the CUDA cores: a CTA stages 16 rows x `chunk` columns of
+// X and the same columns of every mean, each thread accumulates a 4-row x
+// 8-component block over a column split (register tiling: 12 shared loads per
+// 32 FMAs), the column splits are summed in a fixed order through shared
+// memory, and the chunk sums go into the accumulators (file comment).
 __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__ X,
                                                        const float* __restrict__ mu,
                                                        const int32_t* __restrict__ n_rows_dev,
                                                        int K, int64_t D, int chunk, int nchunk, int max_rows,
-                                                       bool bulk, long long* __restrict__ gacc,
-                                                       uint32_t* __restrict__ tickets,
-                                                       const float* __restrict__ coef, int T,
-                                                       const int32_t* __restrict__ miss_bt,
-                                                       const float* __restrict__ mnorm,
-                                                       float* __restrict__ R, float* __restrict__ rowc,
-                                                       int32_t* status) {
+                                                       bool bulk, long long* __restrict__ gacc2,
+                                                       GmmEpoch* ep, int32_t* status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t bar;
-  __shared__ int s_last;
-  __shared__ float s_logit[kDotRows * kMaxK];
-  __shared__ float s_sa[kDotRows], s_q[kDotRows], s_ac[kDotRows];
-  const int n_rows = min(*n_rows_dev, max_rows);
+  long long* gacc = begin_dots(gacc2, ep, (int64_t)max_rows * K);
+  const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
   const int r0 = blockIdx.y * kDotRows;
   if (r0 >= n_rows) return;
   const int nr = min(kDotRows, n_rows - r0);
@@ -235,66 +287,33 @@ __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__
   for (int o = tid; o < nr * K; o += kThreads) {
     float a4[4] = {0.f, 0.f, 0.f, 0.f};
     const float* ro = red + (size_t)o * (CS + 1);
-    for (int cs = 0, u = 0; cs < CS; ++cs, u = (u + 1) & 3) a4[u] += ro[cs];
+    int cs = 0;
+    for (; cs + 3 < CS; cs += 4) {
+      a4[0] += ro[cs];
+      a4[1] += ro[cs + 1];
+      a4[2] += ro[cs + 2];
+      a4[3] += ro[cs + 3];
+    }
+    for (; cs < CS; ++cs) a4[0] += ro[cs];
     const float sum = (a4[0] + a4[1]) + (a4[2] + a4[3]);
     atomicAdd(reinterpret_cast<unsigned long long*>(gacc + (int64_t)r0 * K + o),
               static_cast<unsigned long long>(__float2ll_rn(sum * kDotScale)));
   }
-  // the last CTA of this row block finishes the contraction and the softmax
-  __syncthreads();
-  if (tid == 0) {
-    __threadfence();
-    const unsigned int k = atomicAdd(&tickets[blockIdx.y], 1u);
-    s_last = (k == gridDim.x - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  if (tid == 0) tickets[blockIdx.y] = 0u;  // ready for the next call
-  if (tid < nr) {
-    const int i = miss_bt[2 * (r0 + tid) + 1];
-    s_sa[tid] = coef[i];
-    s_q[tid] = coef[T + i];
-    s_ac[tid] = coef[2 * T + i];
-  }
-  __syncthreads();
-  for (int o = tid; o < nr * K; o += kThreads) {
-    const int rr = o / K, k = o % K;
-    long long* acc_p = gacc + (int64_t)(r0 + rr) * K + k;
-    const long long v = __ldcg(acc_p);
-    *acc_p = 0;  // ready for the next call
-    const float dot = (float)((double)v * (1.0 / (double)kDotScale));
-    const float sa = s_sa[rr];
-    s_logit[rr * K + k] = (2.f * sa * dot - sa * sa * mnorm[k]) * s_q[rr];
-  }
-  __syncthreads();
-  const int warp = tid >> 5, lane = tid & 31;
-  for (int rr = warp; rr < nr; rr += kThreads / 32) {
-    const float* l = s_logit + rr * K;
-    float mx = -INFINITY;
-    for (int k = lane; k < K; k += 32) mx = fmaxf(mx, l[k]);
-    mx = warp_max(mx);
-    float sum = 0.f;
-    for (int k = lane; k < K; k += 32) sum += expf(l[k] - mx);
-    sum = warp_sum(sum);
-    const float inv = 1.f / sum;
-    const int r = r0 + rr;
-    for (int k = lane; k < K; k += 32) R[(int64_t)r * K + k] = expf(l[k] - mx) * inv;
-    if (lane == 0) {
-      rowc[2 * r] = s_ac[rr];
-      rowc[2 * r + 1] = s_ac[rr] * s_sa[rr];
-    }
-  }
 }
 
-// eps[r][c] = ac x[r][c] - ac sqrt(a) sum_k R[r][k] mu[k][c]: a CTA stages a
-// 16-row x 256-column tile of X and the same columns of every mean; each
-// thread computes a 4-row x 4-column block (one 16-byte mean load and four
-// broadcast responsibility loads per 16 FMAs).
+// Output kernel. First the 16 rows' responsibilities: the finished dot
+// products (accumulator set of this call), the logits with ||mu_k||^2 and the
+// per-timestep scalars, and the max-subtracted softmax, while the row and mean
+// tiles are in flight. Then eps[r][c] = ac x[r][c] - ac sqrt(a) sum_k
+// R[r][k] mu[k][c] over a 16-row x 256-column tile: each thread computes a
+// 4-row x 4-column block (one 16-byte mean load and four broadcast
+// responsibility loads per 16 FMAs).
 __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ X,
                                                       const float* __restrict__ mu,
-                                                      const float* __restrict__ R,
-                                                      const float* __restrict__ rowc,
+                                                      const long long* __restrict__ gacc2,
+                                                      GmmEpoch* ep, const float* __restrict__ coef, int T,
+                                                      const int32_t* __restrict__ miss_bt,
+                                                      const float* __restrict__ mnorm,
                                                       const int32_t* __restrict__ n_rows_dev,
                                                       int K, int64_t D, int max_rows, bool bulk, bool vec_out,
                                                       float* __restrict__ eps, int32_t* status) {
@@ -302,7 +321,8 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   __shared__ __align__(8) uint64_t bar;
   __shared__ float s_r[kOutRows * kMaxK];
   __shared__ float s_c[kOutRows * 2];
-  const int n_rows = min(*n_rows_dev, max_rows);
+  __shared__ float s_sa[kOutRows], s_q[kOutRows];
+  const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
   const int r0 = blockIdx.y * kOutRows;
   if (r0 >= n_rows) return;
   const int nr = min(kOutRows, n_rows - r0);
@@ -310,7 +330,7 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   const int ncol = (int)(((D - c0) < kOutCols) ? (D - c0) : kOutCols);
   float* ms = reinterpret_cast<float*>(smem_raw);   // [K][kOutCols]
   float* xs = ms + (size_t)K * kOutCols;            // [kOutRows][kOutCols]
-  const int tid = threadIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   if (tid == 0) {
     mbar_init(&bar, 1);
     fence_barrier_init();
@@ -320,9 +340,41 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   // the means and the rows (written two kernels back) do not depend on the predecessor
   stage_rows(ms, kOutCols, mu, D, c0, ncol, K, bulk, &bar);
   stage_rows(xs, kOutCols, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
-  pdl_wait();  // the responsibilities come from the dot-product kernel
-  for (int q = tid; q < kOutRows * K; q += kThreads) s_r[q] = (q < nr * K) ? R[(int64_t)r0 * K + q] : 0.f;
-  for (int q = tid; q < kOutRows * 2; q += kThreads) s_c[q] = (q < nr * 2) ? rowc[2 * r0 + q] : 0.f;
+  for (int rr = tid; rr < nr; rr += kThreads) {
+    const int i = miss_bt[2 * (r0 + rr) + 1];
+    s_sa[rr] = coef[i];
+    s_q[rr] = coef[T + i];
+    s_c[2 * rr] = coef[2 * T + i];
+    s_c[2 * rr + 1] = coef[2 * T + i] * coef[i];
+  }
+  pdl_wait();  // the dot products come from the kernel just before
+  const uint32_t cur = ep->cur;
+  const long long* gacc = gacc2 + (int64_t)(cur & 1u) * max_rows * K;
+  __syncthreads();
+  for (int q = tid; q < kOutRows * K; q += kThreads) {
+    float l = 0.f;
+    if (q < nr * K) {
+      const int rr = q / K, k = q % K;
+      const float dot = __ll2float_rn(__ldcg(gacc + (int64_t)r0 * K + q)) * (1.f / kDotScale);  // exact scale
+      const float sa = s_sa[rr];
+      l = (2.f * sa * dot - sa * sa * mnorm[k]) * s_q[rr];
+    }
+    s_r[q] = l;
+  }
+  __syncthreads();
+  for (int rr = warp; rr < nr; rr += kThreads / 32) {
+    float* l = s_r + rr * K;
+    float mx = -INFINITY;
+    for (int k = lane; k < K; k += 32) mx = fmaxf(mx, l[k]);
+    mx = warp_max(mx);
+    float sum = 0.f;
+    for (int k = lane; k < K; k += 32) sum += expf(l[k] - mx);
+    sum = warp_sum(sum);
+    const float inv = 1.f / sum;
+    __syncwarp();
+    for (int k = lane; k < K; k += 32) l[k] = expf(l[k] - mx) * inv;
+  }
+  if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) ep->epoch = cur + 1u;  // the next call's set
   const bool ok = wait_staged(bulk, &bar, status);
   __syncthreads();
   if (!ok) return;
@@ -364,6 +416,194 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   }
 }
 
+// ---------------------------------------------------------------------------
+// Tensor-core form of the dot products (tcgen05, kind::tf32). G = X M^T is a
+// dense contraction over D: a CTA takes a block of 128 rows (M = 128, rows past
+// the count are zero) and a chunk of kTcCols columns, and computes the
+// 128 x Kp partial product (Kp = K rounded up to 16, 32, 64 or 128; padded
+// means are zero) in TMEM with single-thread tcgen05.mma issue. fp32 accuracy
+// from tf32 operands: every value is split as v = hi + lo with
+// hi = tf32(v), lo = tf32(v - hi), and the product summed as
+// hi*hi + hi*lo + lo*hi (the lo*lo term is below fp32 resolution). The rows are
+// split by the CTA's threads into core-matrix order in shared memory; the
+// means' split image is prepared once per handle (k_gmm_mu_image) and arrives
+// by one bulk copy. Chunk sums go into the fixed-point accumulators as in
+// k_gmm_dots (with a thread-block cluster of kTcCluster chunks, the cluster's
+// partial sums are first added through distributed shared memory, which cuts
+// the atomics on each accumulator by that factor).
+__host__ inline size_t tc_smem_bytes(int K) {
+  return ((size_t)2 * kTcRows * kTcCols + tc_mu_chunk_floats(K)) * sizeof(float);
+}
+// element (r, c) of a K-major tile with kTcCols columns, in core-matrix order:
+// 8-row groups of (kTcCols / 4) core matrices of 8 rows x 4 values
+__host__ __device__ inline int tc_off(int r, int c) {
+  return ((r >> 3) * (kTcCols / 4) + (c >> 2)) * 32 + (r & 7) * 4 + (c & 3);
+}
+
+// The means' split image, once per handle: chunk ch, part (0 hi, 1 lo), in
+// core-matrix order with Kp rows.
+__global__ void __launch_bounds__(256) k_gmm_mu_image(const float* __restrict__ mu, int K, int64_t D,
+                                                      float* __restrict__ img) {
+  const int Kp = tc_npad(K);
+  const int64_t ch = blockIdx.x;
+  float* out = img + ch * tc_mu_chunk_floats(K);
+  for (int q = threadIdx.x; q < Kp * kTcCols; q += 256) {
+    const int k = q / kTcCols, c = q % kTcCols;
+    const int64_t col = ch * kTcCols + c;
+    const float v = (k < K && col < D) ? mu[(int64_t)k * D + col] : 0.f;
+    const float hi = to_tf32(v);
+    out[tc_off(k, c)] = hi;
+    out[(size_t)Kp * kTcCols + tc_off(k, c)] = to_tf32(v - hi);
+  }
+}
+
+template <int CL>
+__global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restrict__ X,
+                                                            const float* __restrict__ mu_img,
+                                                            const int32_t* __restrict__ n_rows_dev, int K,
+                                                            int64_t D, int max_rows,
+                                                            long long* __restrict__ gacc2, GmmEpoch* ep,
+                                                            int32_t* status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bar_mu;
+  __shared__ __align__(8) uint64_t bar_mma;
+  __shared__ uint32_t s_taddr;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  long long* gacc = begin_dots(gacc2, ep, (int64_t)max_rows * K);
+  const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
+  const int r0 = blockIdx.y * kTcRows;
+  if (r0 >= n_rows) return;
+  const int nr = min(kTcRows, n_rows - r0);
+  const int Kp = tc_npad(K);
+  const uint32_t ncols = Kp < 32 ? 32u : (uint32_t)Kp;  // TMEM columns: a power of two >= 32
+  const int64_t c0 = (int64_t)blockIdx.x * kTcCols;
+  float* A_hi = reinterpret_cast<float*>(smem_raw);
+  float* A_lo = A_hi + kTcRows * kTcCols;
+  float* B_img = A_lo + kTcRows * kTcCols;  // hi then lo, Kp rows each
+  if (tid == 0) {
+    mbar_init(&bar_mu, 1);
+    mbar_init(&bar_mma, 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(&s_taddr, ncols);
+    tc_fence_before_sync();
+  }
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t taddr = s_taddr;
+  if (tid == 0) {  // the means image does not depend on the predecessor
+    const uint32_t bytes = (uint32_t)(tc_mu_chunk_floats(K) * sizeof(float));
+    mbar_arrive_expect_tx(&bar_mu, bytes);
+    bulk_g2s(B_img, mu_img + (size_t)blockIdx.x * tc_mu_chunk_floats(K), bytes, &bar_mu);
+  }
+  pdl_wait();  // the rows come from the gather just before
+
+  // rows -> (hi, lo) in core-matrix order: a warp step covers 8 rows x 16
+  // columns; lanes 8q..8q+7 write one 128-byte core matrix (conflict-free).
+  // All of a thread's loads are issued before the first conversion.
+  {
+    constexpr int kSteps = (kTcRows / 8) * (kTcCols / 16);
+    constexpr int kPer = kSteps / (kTcThreads / 32);
+    const int rin = lane & 7, kq = lane >> 3;
+    float4 v[kPer];
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int it = warp + u * (kTcThreads / 32);
+      const int g = it / (kTcCols / 16), kb = (it % (kTcCols / 16)) * 4 + kq;
+      const int r = g * 8 + rin, c = kb * 4;
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (r < nr && c0 + c < D) v[u] = __ldg(reinterpret_cast<const float4*>(X + (int64_t)(r0 + r) * D + c0 + c));
+    }
+#pragma unroll
+    for (int u = 0; u < kPer; ++u) {
+      const int it = warp + u * (kTcThreads / 32);
+      const int g = it / (kTcCols / 16), kb = (it % (kTcCols / 16)) * 4 + kq;
+      const int r = g * 8 + rin, c = kb * 4;
+      float4 hi, lo;
+      hi.x = to_tf32(v[u].x); lo.x = to_tf32(v[u].x - hi.x);
+      hi.y = to_tf32(v[u].y); lo.y = to_tf32(v[u].y - hi.y);
+      hi.z = to_tf32(v[u].z); lo.z = to_tf32(v[u].z - hi.z);
+      hi.w = to_tf32(v[u].w); lo.w = to_tf32(v[u].w - hi.w);
+      const int off = tc_off(r, c);
+      *reinterpret_cast<float4*>(A_hi + off) = hi;
+      *reinterpret_cast<float4*>(A_lo + off) = lo;
+    }
+  }
+  fence_proxy_async_smem();  // the tensor core reads what the threads wrote
+  // every decision below is taken by the whole CTA (__syncthreads_and)
+  bool ok = __syncthreads_and(mbar_wait_bounded(&bar_mu, 0, pa::kWaitLimit));
+  if (!ok) {
+    if (tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    mbar_wait_bounded(&bar_mu, 0, pa::kDrainLimit);  // the copy lands before the CTA moves on
+  }
+  if (tid == 0 && ok) {
+    tc_fence_after_sync();
+    const uint32_t idesc = tc_idesc_tf32(kTcRows, Kp);
+    const uint32_t a_hi = smem_u32(A_hi), a_lo = smem_u32(A_lo);
+    const uint32_t b_hi = smem_u32(B_img), b_lo = b_hi + (uint32_t)(Kp * kTcCols * sizeof(float));
+    const uint32_t sbo = (kTcCols / 4) * 128;  // next 8-row group
+    for (int ks = 0; ks < kTcCols / 8; ++ks) {
+      const uint32_t ko = (uint32_t)ks * 256;  // two core matrices along K per step
+      const uint64_t dah = tc_smem_desc(a_hi + ko, 128, sbo), dal = tc_smem_desc(a_lo + ko, 128, sbo);
+      const uint64_t dbh = tc_smem_desc(b_hi + ko, 128, sbo), dbl = tc_smem_desc(b_lo + ko, 128, sbo);
+      tc_mma_tf32(taddr, dah, dbh, idesc, ks > 0 ? 1u : 0u);
+      tc_mma_tf32(taddr, dah, dbl, idesc, 1u);
+      tc_mma_tf32(taddr, dal, dbh, idesc, 1u);
+    }
+    tc_commit(&bar_mma);
+  }
+  if (ok && !__syncthreads_and(mbar_wait_bounded(&bar_mma, 0, pa::kWaitLimit))) {
+    if (tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    mbar_wait_bounded(&bar_mma, 0, pa::kDrainLimit);  // let the MMAs finish before TMEM is freed
+    ok = false;
+  }
+  tc_fence_after_sync();
+  float* part = A_hi;  // [kTcRows][Kp]: this CTA's partial sums (the operands are consumed)
+  if (warp < 4 && ok) {  // warp w reads TMEM lanes (rows) 32w .. 32w + 31
+    const int row = warp * 32 + lane;
+    for (int cb = 0; cb < Kp; cb += 16) {
+      float v[16];
+      tmem_ld16(taddr + ((uint32_t)(warp * 32) << 16) + (uint32_t)cb, v);
+      if constexpr (CL > 1) {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) part[row * Kp + cb + u] = v[u];
+      } else if (row < nr) {
+#pragma unroll
+        for (int u = 0; u < 16; ++u) {
+          const int k = cb + u;
+          if (k < K)
+            atomicAdd(reinterpret_cast<unsigned long long*>(gacc + (int64_t)(r0 + row) * K + k),
+                      static_cast<unsigned long long>(__float2ll_rn(v[u] * kDotScale)));
+        }
+      }
+    }
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(taddr, ncols);
+  if constexpr (CL > 1) {
+    // the CL column chunks of a cluster are added through distributed shared
+    // memory in rank order; rank q then adds rows [q R, (q+1) R) to gacc
+    cg::cluster_group cluster = cg::this_cluster();
+    if (!ok)
+      for (int q = tid; q < kTcRows * Kp; q += kTcThreads) part[q] = 0.f;
+    cluster.sync();
+    const int rank = (int)cluster.block_rank();
+    constexpr int kRowsPer = kTcRows / CL;
+    for (int o = tid; o < kRowsPer * K; o += kTcThreads) {
+      const int rr = rank * kRowsPer + o / K, k = o % K;
+      if (rr < nr) {
+        float sum = 0.f;
+        for (int q = 0; q < CL; ++q) sum += cluster.map_shared_rank(part, q)[rr * Kp + k];
+        atomicAdd(reinterpret_cast<unsigned long long*>(gacc + (int64_t)(r0 + rr) * K + k),
+                  static_cast<unsigned long long>(__float2ll_rn(sum * kDotScale)));
+      }
+    }
+    cluster.sync();  // peers read this CTA's partial sums until here
+  }
+}
+
 }  // namespace
 
 struct pa_gmm {
@@ -374,6 +614,8 @@ struct pa_gmm {
   GmmLayout L;
   cudaStream_t st;
   int64_t launches;
+  bool tc_ok;   // the tensor-core dot products fit this device and these sizes
+  bool use_tc;  // ... and are selected
 };
 
 extern "C" size_t pa_gmm_workspace_bytes(int K, int64_t D, int max_rows, int T) {
@@ -418,10 +660,8 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
   cudaError_t e = cudaMemcpyAsync(g->ws + L.coef, coef.data(), coef.size() * sizeof(float),
                                   cudaMemcpyHostToDevice, g->st);
   if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.status, 0, sizeof(int32_t), g->st);
-  if (e == cudaSuccess)
-    e = cudaMemsetAsync(g->ws + L.tickets, 0, (size_t)((max_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t),
-                        g->st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.gacc, 0, (size_t)max_rows * K * sizeof(long long), g->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.epoch, 0, sizeof(GmmEpoch), g->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(g->ws + L.gacc, 0, (size_t)2 * max_rows * K * sizeof(long long), g->st);
   if (e == cudaSuccess) {
     k_gmm_norms<<<K, 256, 0, g->st>>>(means_dev, D, reinterpret_cast<float*>(g->ws + L.mnorm));
     g->launches++;
@@ -433,6 +673,32 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
     e = cudaFuncSetAttribute(k_gmm_dots, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)dots_smem);
   if (e == cudaSuccess)
     e = cudaFuncSetAttribute(k_gmm_out, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)out_smem);
+  // tensor-core dot products: sm_100-family tensor cores, 16-byte rows, and
+  // shared memory for the split rows and the means image of one chunk
+  int dev = 0, major = 0, optin = 0;
+  g->tc_ok = false;
+  if (e == cudaSuccess) e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (e == cudaSuccess && major == 10 && D % 4 == 0 && (reinterpret_cast<uintptr_t>(means_dev) & 15) == 0 &&
+      tc_smem_bytes(K) + 2048 <= (size_t)optin) {
+    e = cudaFuncSetAttribute(k_gmm_dots_tc<kTcCluster>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)tc_smem_bytes(K));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(k_gmm_dots_tc<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)tc_smem_bytes(K));
+    if (e == cudaSuccess) {
+      k_gmm_mu_image<<<L.tc_chunks, 256, 0, g->st>>>(means_dev, K, D, reinterpret_cast<float*>(g->ws + L.mu_img));
+      g->launches++;
+      e = cudaGetLastError();
+      g->tc_ok = e == cudaSuccess;
+    }
+  }
+  // Default: the tensor cores for K > 16. At K <= 16 the contraction is under
+  // a microsecond of CUDA-core FMA work per call and the CUDA-core kernel's
+  // shorter per-CTA chain wins (measured at 4x64x64: 46.9 vs 49.7 us per
+  // Picard iteration); at K = 64 the tensor cores win (172.2 vs 186.2 us at
+  // 4x128x128).
+  g->use_tc = g->tc_ok && K > kTcMinK;
   if (e == cudaSuccess) e = cudaStreamSynchronize(g->st);
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_create: ") + cudaGetErrorString(e));
@@ -450,28 +716,34 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
     return PA_ERR_ARG;
   }
   const GmmLayout& L = g->L;
-  float* coef = reinterpret_cast<float*>(g->ws + L.coef);
-  float* mnorm = reinterpret_cast<float*>(g->ws + L.mnorm);
-  long long* gacc = reinterpret_cast<long long*>(g->ws + L.gacc);
-  float* R = reinterpret_cast<float*>(g->ws + L.R);
-  float* rowc = reinterpret_cast<float*>(g->ws + L.rowc);
+  const float* coef = reinterpret_cast<const float*>(g->ws + L.coef);
+  const float* mnorm = reinterpret_cast<const float*>(g->ws + L.mnorm);
+  long long* gacc2 = reinterpret_cast<long long*>(g->ws + L.gacc);
+  GmmEpoch* ep = reinterpret_cast<GmmEpoch*>(g->ws + L.epoch);
   int32_t* status = reinterpret_cast<int32_t*>(g->ws + L.status);
   // bulk copies need 16-byte aligned rows: D % 4 == 0 and aligned base pointers
   const bool bulk = g->D % 4 == 0 && ((reinterpret_cast<uintptr_t>(batch_x_dev) |
                                        reinterpret_cast<uintptr_t>(g->means)) & 15) == 0;
-  uint32_t* tickets = reinterpret_cast<uint32_t*>(g->ws + L.tickets);
   const bool vec_out = g->D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps_dev) & 15) == 0;
-  const size_t dots_smem = dots_smem_bytes(g->K, L.chunk);
   const size_t out_smem = (size_t)(g->K + kOutRows) * kOutCols * sizeof(float);
-  cudaError_t e = pa::launch_ex(k_gmm_dots, dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows),
-                                dim3(kThreads), dots_smem, g->st, 0, batch_x_dev, g->means, n_rows_dev, g->K,
-                                g->D, L.chunk, L.nchunk, g->max_rows, bulk, gacc, tickets, (const float*)coef,
-                                g->T, miss_bt_dev, (const float*)mnorm, R, rowc, status);
+  const dim3 tc_grid(L.tc_chunks, (g->max_rows + kTcRows - 1) / kTcRows);
+  cudaError_t e;
+  if (g->use_tc && bulk && L.tc_chunks >= kTcClusterMinChunks)
+    e = pa::launch_ex(k_gmm_dots_tc<kTcCluster>, tc_grid, dim3(kTcThreads), tc_smem_bytes(g->K), g->st,
+                      kTcCluster, batch_x_dev, (const float*)(g->ws + L.mu_img), n_rows_dev, g->K, g->D,
+                      g->max_rows, gacc2, ep, status);
+  else if (g->use_tc && bulk)
+    e = pa::launch_ex(k_gmm_dots_tc<1>, tc_grid, dim3(kTcThreads), tc_smem_bytes(g->K), g->st, 0, batch_x_dev,
+                      (const float*)(g->ws + L.mu_img), n_rows_dev, g->K, g->D, g->max_rows, gacc2, ep, status);
+  else
+    e = pa::launch_ex(k_gmm_dots, dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows), dim3(kThreads),
+                      dots_smem_bytes(g->K, L.chunk), g->st, 0, batch_x_dev, g->means, n_rows_dev, g->K, g->D,
+                      L.chunk, L.nchunk, g->max_rows, bulk, gacc2, ep, status);
   if (e == cudaSuccess)
     e = pa::launch_ex(k_gmm_out,
                       dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
-                      dim3(kOutCols), out_smem, g->st, 0, batch_x_dev, g->means, (const float*)R,
-                      (const float*)rowc, n_rows_dev, g->K, g->D, g->max_rows, bulk, vec_out, batch_eps_dev,
+                      dim3(kOutCols), out_smem, g->st, 0, batch_x_dev, g->means, (const long long*)gacc2, ep, coef,
+                      g->T, miss_bt_dev, mnorm, n_rows_dev, g->K, g->D, g->max_rows, bulk, vec_out, batch_eps_dev,
                       status);
   g->launches += 2;
   if (e == cudaSuccess) e = cudaGetLastError();
@@ -496,6 +768,20 @@ extern "C" pa_status pa_gmm_check(pa_gmm* g) {
 }
 
 extern "C" int64_t pa_gmm_launches(const pa_gmm* g) { return g ? g->launches : -1; }
+
+extern "C" pa_status pa_gmm_set_form(pa_gmm* g, int form) {
+  if (!g) { pa::set_error("pa_gmm_set_form: NULL handle"); return PA_ERR_ARG; }
+  if (form != 0 && form != 1) { pa::set_error("pa_gmm_set_form: form must be 0 or 1"); return PA_ERR_ARG; }
+  if (form == 1 && !g->tc_ok) {
+    pa::set_error("pa_gmm_set_form: tensor-core dot products need an sm_100-family GPU, D % 4 == 0, "
+                  "16-byte aligned means and enough shared memory");
+    return PA_ERR_ARG;
+  }
+  g->use_tc = form == 1;
+  return PA_OK;
+}
+
+extern "C" int pa_gmm_form(const pa_gmm* g) { return g ? (g->use_tc ? 1 : 0) : -1; }
 
 extern "C" void pa_gmm_destroy(pa_gmm* g) { delete g; }
 
@@ -570,18 +856,16 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
     }
   }
   if (n_rows == 0) return PA_OK;
-  // scratch layout: coef[3T] | mnorm[K] | gacc[n_rows][K] (int64) | R[n_rows][K] |
-  //                 rowc[n_rows][2] | tickets | n_rows | status   (256-byte aligned pieces)
+  // scratch layout: coef[3T] | mnorm[K] | gacc[2][n_rows][K] (int64) | epoch |
+  //                 n_rows | status   (256-byte aligned pieces)
   const int chunk = dots_chunk(K, D);
   const int nchunk = (int)((D + chunk - 1) / chunk);
   size_t o = 0;
   auto take = [&](size_t bytes) { size_t at = o; o = pa::align_up(o + bytes, pa::kAlign); return at; };
   const size_t o_coef = take((size_t)3 * T * sizeof(float));
   const size_t o_mnorm = take((size_t)K * sizeof(float));
-  const size_t o_gacc = take((size_t)n_rows * K * sizeof(long long));
-  const size_t o_R = take((size_t)n_rows * K * sizeof(float));
-  const size_t o_rowc = take((size_t)n_rows * 2 * sizeof(float));
-  const size_t o_tick = take((size_t)((n_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t));
+  const size_t o_gacc = take((size_t)2 * n_rows * K * sizeof(long long));
+  const size_t o_epoch = take(sizeof(GmmEpoch));
   const size_t o_n = take(sizeof(int32_t));
   const size_t o_status = take(sizeof(int32_t));
   if (o > kNoAllocScratchBytes) {
@@ -596,10 +880,8 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   float* coef = reinterpret_cast<float*>(scratch + o_coef);
   float* mnorm = reinterpret_cast<float*>(scratch + o_mnorm);
-  long long* gacc = reinterpret_cast<long long*>(scratch + o_gacc);
-  float* R = reinterpret_cast<float*>(scratch + o_R);
-  float* rowc = reinterpret_cast<float*>(scratch + o_rowc);
-  uint32_t* tickets = reinterpret_cast<uint32_t*>(scratch + o_tick);
+  long long* gacc2 = reinterpret_cast<long long*>(scratch + o_gacc);
+  GmmEpoch* ep = reinterpret_cast<GmmEpoch*>(scratch + o_epoch);
   int32_t* nrows_dev = reinterpret_cast<int32_t*>(scratch + o_n);
   int32_t* status = reinterpret_cast<int32_t*>(scratch + o_status);
 
@@ -622,9 +904,9 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   const int32_t nr = n_rows;
   if (e == cudaSuccess) e = cudaMemcpyAsync(nrows_dev, &nr, sizeof(nr), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);  // starts at zero every call
-  if (e == cudaSuccess)  // the row-block tickets and the dot accumulators start at zero every call too
-    e = cudaMemsetAsync(tickets, 0, (size_t)((n_rows + kDotRows - 1) / kDotRows) * sizeof(uint32_t), st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(gacc, 0, (size_t)n_rows * K * sizeof(long long), st);
+  if (e == cudaSuccess)  // the epoch and both accumulator sets start at zero every call too
+    e = cudaMemsetAsync(ep, 0, sizeof(GmmEpoch), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(gacc2, 0, (size_t)2 * n_rows * K * sizeof(long long), st);
   const size_t dots_smem = dots_smem_bytes(K, chunk);
   const size_t out_smem = (size_t)(K + kOutRows) * kOutCols * sizeof(float);
   if (e == cudaSuccess)
@@ -640,11 +922,10 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   k_gmm_norms<<<K, 256, 0, st>>>(means_dev, D, mnorm);
   const bool vec_out = D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps_dev) & 15) == 0;
   k_gmm_dots<<<dim3(nchunk, (n_rows + kDotRows - 1) / kDotRows), kThreads, dots_smem, st>>>(
-      batch_x_dev, means_dev, nrows_dev, K, D, chunk, nchunk, n_rows, bulk, gacc, tickets, coef, T, miss_bt_dev,
-      mnorm, R, rowc, status);
+      batch_x_dev, means_dev, nrows_dev, K, D, chunk, nchunk, n_rows, bulk, gacc2, ep, status);
   k_gmm_out<<<dim3((unsigned)((D + kOutCols - 1) / kOutCols), (n_rows + kOutRows - 1) / kOutRows), kOutCols,
-              out_smem, st>>>(batch_x_dev, means_dev, R, rowc, nrows_dev, K, D, n_rows, bulk, vec_out,
-                              batch_eps_dev, status);
+              out_smem, st>>>(batch_x_dev, means_dev, gacc2, ep, coef, T, miss_bt_dev, mnorm, nrows_dev, K, D,
+                              n_rows, bulk, vec_out, batch_eps_dev, status);
   e = cudaGetLastError();
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_eps_noalloc: ") + cudaGetErrorString(e));

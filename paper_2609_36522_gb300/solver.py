@@ -144,6 +144,13 @@ class GmmDenoiser:
     def launches(self):
         return abi.pa_gmm_launches(self.h)
 
+    def set_form(self, form):
+        """1: dot products on the tensor cores; 0: on the CUDA cores."""
+        abi.pa_gmm_set_form(self.h, form)
+
+    def form(self):
+        return abi.pa_gmm_form(self.h)
+
     def close(self):
         if getattr(self, "h", None) is not None:
             abi.pa_gmm_destroy(self.h)

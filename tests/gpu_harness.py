@@ -17,7 +17,7 @@ def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True):
 
 
 def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=None,
-            mode="sync", x_init_host=False):
+            mode="sync", x_init_host=False, gmm_form=None):
     """Run one generation on the GPU.
 
     eps_source: "gmm" (the CUDA mixture kernel) or "oracle" (fp64 mixture
@@ -36,6 +36,8 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
     max_rows = w.batch * s.window
     means = torch.from_numpy(mu).to(dev)
     g = GmmDenoiser(means, w.gmm_std, a, max_rows)
+    if gmm_form is not None:
+        g.set_form(gmm_form)
     eps_buf = torch.empty(max_rows, w.D, dtype=torch.float32, device=dev)
     x_init = torch.from_numpy(x0)
     if x_init_host:

@@ -88,5 +88,7 @@ def test_null_handles_are_rejected(lib):
     L.pa_destroy(None)
     L.pa_gmm_destroy(None)
     assert L.pa_gmm_launches(None) == -1
+    assert L.pa_gmm_form(None) == -1
+    assert L.pa_gmm_set_form(None, 0) == abi.PA_ERR_ARG
     h = C.c_void_p()
     assert L.pa_gmm_create(C.byref(h), 0, 16, None, 0.5, None, 4, 4, None, 0, None) == abi.PA_ERR_ARG

@@ -133,19 +133,23 @@ def _gmm_rows(w, n, seed=0):
     return a, mu, idx, x, miss
 
 
+@pytest.mark.parametrize("form", [1, 0])
 @pytest.mark.parametrize("wname,n,max_rows", [("sd15", 48, 48), ("sd15", 1, 100), ("sd15", 37, 100),
                                               ("sd15", 100, 100), ("batched", 256, 256),
                                               ("large", 48, 48), ("tiny", 5, 8)])
-def test_gmm_kernel_against_oracle(wname, n, max_rows):
-    """The mixture denoiser alone, on rows spread over the whole schedule, with
-    the device row count below the capacity, and over three calls in a row
-    (the fixed-point accumulators and the tickets are reused)."""
+def test_gmm_kernel_against_oracle(wname, n, max_rows, form):
+    """The mixture denoiser alone, with the dot products on the tensor cores
+    (form 1) and on the CUDA cores (form 0), on rows spread over the whole
+    schedule, with the device row count below the capacity, and over three
+    calls in a row (the fixed-point accumulators and the tickets are reused)."""
     import torch
     from paper_2609_36522_gb300.solver import GmmDenoiser
     w = W.ALL[wname]
     a, mu, idx, x, miss = _gmm_rows(w, n)
     dev = torch.device("cuda")
     g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows)
+    assert g.form() == (1 if w.K > 16 else 0), "tensor cores by default above 16 components"
+    g.set_form(form)
     xd = torch.zeros(max_rows, w.D, dtype=torch.float32, device=dev)
     xd[:n] = torch.from_numpy(x).to(dev)
     md = torch.zeros(max_rows, 2, dtype=torch.int32, device=dev)
@@ -201,6 +205,13 @@ def test_gmm_in_cuda_graph():
         from paper_2609_36522_gb300 import abi
         abi.pa_gmm_check(g.h)
         g.close()
+
+
+def test_sd15_tensor_core_denoiser():
+    """Whole-pipeline parity with the denoiser's dot products on the tensor
+    cores (the default only above 16 components)."""
+    w = W.SD15
+    compare(w, oracle_run(w), gpu_run(w, gmm_form=1))
 
 
 @pytest.mark.parametrize("kind", [0, 1] + list(range(100, 112)))
