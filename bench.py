@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
 NCU_TRAFFIC = {
-    ("9ce682d895630e3d", "sd15"): 6244928.0,
-    ("9ce682d895630e3d", "batched"): 24780757.0,
-    ("9ce682d895630e3d", "large"): 71603189.0,
+    ("ec3eb38c7468b7b6", "sd15"): 6242688.0,
+    ("ec3eb38c7468b7b6", "batched"): 24668416.0,
+    ("ec3eb38c7468b7b6", "large"): 71628142.0,
 }
 
 

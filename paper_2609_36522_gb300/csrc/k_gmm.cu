@@ -348,14 +348,17 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
     s_c[2 * rr + 1] = coef[2 * T + i] * coef[i];
   }
   pdl_wait();  // the dot products come from the kernel just before
+  // both accumulator sets are read together with the set index (one round trip)
   const uint32_t cur = ep->cur;
-  const long long* gacc = gacc2 + (int64_t)(cur & 1u) * max_rows * K;
+  const int64_t set_size = (int64_t)max_rows * K;
   __syncthreads();
   for (int q = tid; q < kOutRows * K; q += kThreads) {
     float l = 0.f;
     if (q < nr * K) {
       const int rr = q / K, k = q % K;
-      const float dot = __ll2float_rn(__ldcg(gacc + (int64_t)r0 * K + q)) * (1.f / kDotScale);  // exact scale
+      const long long v0 = __ldcg(gacc2 + (int64_t)r0 * K + q);
+      const long long v1 = __ldcg(gacc2 + set_size + (int64_t)r0 * K + q);
+      const float dot = __ll2float_rn((cur & 1u) ? v1 : v0) * (1.f / kDotScale);  // exact scale
       const float sa = s_sa[rr];
       l = (2.f * sa * dot - sa * sa * mnorm[k]) * s_q[rr];
     }
