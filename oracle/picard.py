@@ -17,7 +17,8 @@ p = min(P, T - t) evaluation points t .. t+p-1:
 4.  Assembly (Eq. 6): eps_i = cached ehat_i for hits, fresh eps for misses.
 5.  Cache update (Eq. 7), misses only: (xhat_i, ehat_i) <- (x_i, eps_i).
 6.  Drift at the current latent (Sec. 2.2 last paragraph):
-    d_i = (c_i - 1) x_i + e_i eps_i.
+    d_i = (c_i - 1) x_i + e_i eps_i (+ sigma_i z_i for a stochastic step, with
+    the draw z_i fixed before sampling).
 7.  Picard update (Eq. 1, window form): x_{t+j+1} <- x_t + sum_{i=t}^{t+j} d_i.
 8.  Convergence error (Eq. 2): err_j = (1/D) || x^{new}_{t+j+1} - x^{old}_{t+j+1} ||^2.
 9.  Window advance: stride = min(p, 1 + number of leading j with err_j <= tau)
@@ -36,7 +37,7 @@ from typing import List, Optional
 
 import numpy as np
 
-from .ddim import drift_coefficients, drift
+from .ddim import drift, step_coefficients
 
 
 @dataclass
@@ -68,7 +69,7 @@ class PicardResult:
 
 
 def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
-               use_cache=True, max_iters=None, record=True):
+               use_cache=True, max_iters=None, record=True, eta=0.0, noise=None):
     """Cached (or uncached) sliding-window Picard sampling of B trajectories.
 
     alphas       : fp64 [T+1] sampling-order alpha-bar (alphas[T] == 1).
@@ -79,10 +80,18 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
     cache_thresh : tau_cache of Eq. 5 (hit iff delta < tau_cache).
     use_cache    : False gives the uncached sampler (every point evaluated).
     max_iters    : stop early after this many iterations (bounded samples).
+    eta, noise   : stochastic steps (eta > 0): noise [B][T][D] holds the draws
+                   z_i; the drift of step i gains sigma_i z_i (the same draw in
+                   every iteration).
     """
     a = np.asarray(alphas, dtype=np.float64)
     T = len(a) - 1
-    c, e = drift_coefficients(a)
+    c, e, sig = step_coefficients(a, eta)
+    Z = None
+    if eta != 0.0:
+        if noise is None:
+            raise ValueError("eta > 0 needs the noise draws")
+        Z = np.asarray(noise, dtype=np.float64)
     x0 = np.asarray(x_init, dtype=np.float64)
     B, D = x0.shape
     P = int(window)
@@ -157,7 +166,8 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
                         has_entry[b, i] = True
             # 6. drift at the current latents
             idx = np.arange(tb, tb + pb)
-            d = drift(X[b, idx], eps_w, c[idx][:, None], e[idx][:, None])
+            d = drift(X[b, idx], eps_w, c[idx][:, None], e[idx][:, None],
+                      sig[idx][:, None], None if Z is None else Z[b, idx])
             # 7. Picard update, window form of Eq. 1
             x_new = X[b, tb][None, :] + np.cumsum(d, axis=0)
             # 8. convergence error, Eq. 2

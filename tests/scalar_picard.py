@@ -17,6 +17,21 @@ def _ddim(x, eps, a, an):
     return out
 
 
+def _ddpm(x, eps, a, an, z):
+    """Ancestral DDPM step in the posterior form q(x_{t-1} | x_t, x0): the
+    mean (sqrt(an) beta / (1 - a)) x0 + (sqrt(alpha) (1 - an) / (1 - a)) x and
+    the variance (1 - an) / (1 - a) * beta, with beta = 1 - a / an."""
+    beta = 1.0 - a / an
+    alpha = 1.0 - beta
+    var = (1.0 - an) / (1.0 - a) * beta
+    out = []
+    for xd, ed, zd in zip(x, eps, z):
+        x0 = (xd - math.sqrt(1.0 - a) * ed) / math.sqrt(a)
+        mean = math.sqrt(an) * beta / (1.0 - a) * x0 + math.sqrt(alpha) * (1.0 - an) / (1.0 - a) * xd
+        out.append(mean + math.sqrt(var) * zd)
+    return out
+
+
 def _eps(x, a, means, std):
     K = len(means)
     v = a * std * std + 1.0 - a
@@ -37,8 +52,11 @@ def _eps(x, a, means, std):
     return out
 
 
-def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh):
-    """Returns (final states per trajectory, per-iteration (misses, strides, distances))."""
+def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh, noise=None):
+    """Returns (final states per trajectory, per-iteration (misses, strides, distances)).
+
+    noise: None for DDIM; else the draws noise[b][i] of every trajectory and
+    step, and every step is an ancestral DDPM step (eta = 1)."""
     T = len(alphas) - 1
     B = len(x_init)
     D = len(x_init[0])
@@ -101,7 +119,10 @@ def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh):
             run = list(states[b][t])
             for j in range(p):
                 i = t + j
-                stepped = _ddim(states[b][i], eps_of[i], alphas[i], alphas[i + 1])
+                if noise is None:
+                    stepped = _ddim(states[b][i], eps_of[i], alphas[i], alphas[i + 1])
+                else:
+                    stepped = _ddpm(states[b][i], eps_of[i], alphas[i], alphas[i + 1], noise[b][i])
                 drift = [s_ - x_ for s_, x_ in zip(stepped, states[b][i])]
                 run = [r + d for r, d in zip(run, drift)]
                 new[i + 1] = run

@@ -17,6 +17,8 @@ What it produces, per workload:
 * ``x_init`` -- initial noise N(0, 1), fp32, one row per trajectory.
 * ``means`` -- Gaussian-mixture component means N(0, 1), fp32, [K][D]; the
   mixture has equal weights and isotropic component std ``gmm_std``.
+* ``noise`` -- for stochastic steps (eta > 0) the draws z_i ~ N(0, 1) of every
+  trajectory and step, fp32 [B][T][D], fixed before sampling.
 
 The SD v1.5 latent shape 4x64x64 (512^2 images, Sec. 3.2) and the paper's
 cache tolerance 0.05 (Sec. 3.3) set the shapes and thresholds; COCO prompts and
@@ -34,6 +36,7 @@ BETA_START = 1e-4
 BETA_END = 0.02
 GMM_STD = 0.5
 MEANS_SEED_OFFSET = 1_000_000
+NOISE_SEED_OFFSET = 2_000_000
 
 
 @dataclass(frozen=True)
@@ -50,6 +53,7 @@ class Workload:
     cache_thresh: float         # tau_cache (Eq. 5)
     seed: int = 0               # trajectory b uses noise seed (seed + b)
     gmm_std: float = GMM_STD
+    eta: float = 0.0            # stochastic steps (eta = 1: DDPM); 0 = DDIM
     extra: dict = field(default_factory=dict, compare=False)
 
     @property
@@ -69,6 +73,10 @@ BATCHED = Workload("batched T100 P32 B8 4x64x64 K16", T=100, window=32, batch=8,
                    latent_shape=(4, 64, 64), K=16, tol=1e-3, cache_thresh=0.05)
 LARGE = Workload("large T200 P64 B2 4x128x128 K64", T=200, window=64, batch=2,
                  latent_shape=(4, 128, 128), K=64, tol=5e-4, cache_thresh=0.05)
+# Stochastic sampling (a next step beyond the DDIM workloads): DDPM, i.e. eta = 1
+# over the full 1000-step schedule, window 64 (Table 2's best DDPM window).
+DDPM = Workload("DDPM T1000 P64 B1 4x64x64 K16", T=1000, window=64, batch=1,
+                latent_shape=(4, 64, 64), K=16, tol=1e-3, cache_thresh=0.05, eta=1.0)
 SWEEP_THRESHOLDS = (0.0, 0.01, 0.02, 0.05, 0.1)
 
 
@@ -78,7 +86,7 @@ def sweep(base: Workload = SD15):
             for c in SWEEP_THRESHOLDS]
 
 
-ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE}
+ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM}
 
 
 def train_alphas_cumprod() -> np.ndarray:
@@ -112,6 +120,16 @@ def means(w: Workload) -> np.ndarray:
     """Mixture means, fp32 [K][D], from default_rng(1_000_000 + seed)."""
     rng = np.random.default_rng(MEANS_SEED_OFFSET + w.seed)
     return rng.standard_normal((w.K, w.D)).astype(np.float32)
+
+
+def noise(w: Workload) -> np.ndarray:
+    """The draws z_i of stochastic steps, fp32 [B][T][D]; trajectory b draws
+    from default_rng(2_000_000 + seed + b). None for eta = 0."""
+    if w.eta == 0.0:
+        return None
+    rows = [np.random.default_rng(NOISE_SEED_OFFSET + w.seed + b).standard_normal((w.T, w.D)).astype(np.float32)
+            for b in range(w.batch)]
+    return np.stack(rows, axis=0)
 
 
 def inputs(w: Workload):
