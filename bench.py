@@ -130,7 +130,8 @@ def iteration_bytes(log, w: W.Workload):
     Per trajectory with window start t, p points, m misses, frontier e and h1
     hits at positions >= 1 (rows of D fp32 values):
       update : x_t, the p - lazy materialised old states, p eps rows, m ehat
-               and m xhat writes, h1 xhat reads (next distances), p new states
+               and m xhat writes, h1 xhat reads (next distances), p new states,
+               and p draws z_i for stochastic steps (eta > 0)
       gather : m reads + m writes;  denoiser: m reads + m writes (+ K means)
     """
     row = w.D * 4
@@ -142,7 +143,7 @@ def iteration_bytes(log, w: W.Workload):
             if p == 0:
                 continue
             lazy = max(0, t + p - e)
-            u += (1 + (p - lazy) + p + 2 * m + h1 + p) * row
+            u += (1 + (p - lazy) + p + 2 * m + h1 + p + (p if w.eta != 0.0 else 0)) * row
             o += 4 * m * row
         upd.append(u)
         other.append(o + w.K * row)
@@ -213,7 +214,8 @@ def oracle_sample(workload_name, budget_s):
     iters = gens = 0
     t0 = time.perf_counter()
     while True:
-        r = run_picard(a, x0, f, w.window, w.tol, w.cache_thresh, record=False)
+        r = run_picard(a, x0, f, w.window, w.tol, w.cache_thresh, record=False,
+                       eta=w.eta, noise=W.noise(w))
         iters += r.iters
         gens += 1
         if time.perf_counter() - t0 >= budget_s:
@@ -300,6 +302,8 @@ def run_ours(args):
     s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=stream)
     if args.update_kernel is not None:
         s.set_update_kernel(args.update_kernel)
+    if w.eta != 0.0:  # stochastic steps: the draws stay resident on the device
+        s.set_noise(w.eta, torch.from_numpy(W.noise(w)).to(dev))
     max_rows = w.batch * s.window
     g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows, stream=stream)
     if args.gmm_form is not None:
@@ -452,6 +456,7 @@ def run_ours(args):
                        "picard_iters_per_step": n_iters, "global_batch": w.batch * world,
                        "seq_len": w.T, "window": w.window, "latent": "x".join(map(str, w.latent_shape)),
                        "mixture_components": w.K, "tol": w.tol, "cache_thresh": w.cache_thresh,
+                       "eta": w.eta,
                        "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
                                                  if g.form() == 1 else "CUDA cores (fp32 FMA)"),
                        "parallelism": f"replicas x{world} (independent trajectories)",

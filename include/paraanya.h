@@ -99,6 +99,25 @@ PA_API pa_status pa_create(pa_solver** out, int T, int window,
                     int batch, void* workspace_dev, size_t workspace_bytes,
                     void* stream);
 
+/* Stochastic steps (an extension beyond the paper's DDIM runs; eta = 1 over the
+ * full 1000-step schedule is DDPM, the sampler of Table 2). Step i becomes
+ * x_{i+1} = c_i x_i + e_i eps + sigma_i z_i with
+ * sigma_i = eta sqrt((1 - a_{i+1}) / (1 - a_i)) sqrt(1 - a_i / a_{i+1}) and
+ * e_i = sqrt(1 - a_{i+1} - sigma_i^2) - sqrt(a_{i+1} (1 - a_i) / a_i), so the
+ * Picard drift (Eq. 1) gains sigma_i z_i. The draws z_i are fixed before
+ * sampling (the paper is silent on stochastic samplers; this is the reading
+ * that keeps Eq. 1 a deterministic recursion): noise_dev is a DEVICE array
+ * [batch][T][D] fp32 of N(0, 1) draws, 16-byte aligned (else PA_ERR_ARG),
+ * caller-owned, read by every following
+ * iteration until the next pa_set_noise -- it must stay valid and unchanged
+ * that long. eta = 0 (noise_dev may be NULL) restores plain DDIM. eta must be
+ * in [0, 1]. Not allowed between pa_step and pa_submit_eps (PA_ERR_STATE);
+ * takes effect from the next iteration (call pa_init to restart cleanly).
+ * The bulk-copy update kernel stages the draws when D % 4 == 0 and the window
+ * fits its shared memory; otherwise the plain-load kernel runs.
+ * Synchronises the solver's stream. */
+PA_API pa_status pa_set_noise(pa_solver* s, double eta, const float* noise_dev);
+
 /* Start a generation: x_init [batch][D] fp32, HOST or DEVICE pointer (the copy
  * direction is inferred from the address). All states of the first window are
  * x_init (Sec. 2.1 initial trajectory estimate); every first-window timestep is

@@ -47,6 +47,7 @@ _PROTOS = {
     "pa_create": (C.c_int, [PVP, C.c_int, C.c_int, C.POINTER(C.c_int64), C.c_int,
                             C.POINTER(C.c_double), C.c_double, C.c_double, C.c_int,
                             VP, C.c_size_t, VP]),
+    "pa_set_noise": (C.c_int, [VP, C.c_double, VP]),
     "pa_init": (C.c_int, [VP, VP]),
     "pa_step": (C.c_int, [VP, C.POINTER(C.c_int), PVP, PVP]),
     "pa_step_async": (C.c_int, [VP, PVP, PVP, PVP]),
@@ -134,6 +135,10 @@ def pa_create(T, window, latent_shape, alphas_cumprod, tol, cache_thresh, batch,
                                         float(tol), float(cache_thresh), batch,
                                         _dptr(workspace_ptr), workspace_bytes, _dptr(stream_ptr)))
     return h
+
+
+def pa_set_noise(h, eta, noise_ptr):
+    return _check("pa_set_noise", lib().pa_set_noise(h, float(eta), _dptr(noise_ptr)))
 
 
 def pa_init(h, x_init_ptr):

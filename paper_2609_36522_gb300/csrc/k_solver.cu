@@ -101,7 +101,7 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d) {
 // Per window position j (timestep i = t + j):
 //   eps_i  = batch_eps[rank] (miss) or ehat_i (hit)              Eq. 6
 //   miss:  ehat_i <- eps_i, xhat_i <- x_i                         Eq. 7
-//   d_i    = (c_i - 1) x_i + e_i eps_i                            drift
+//   d_i    = (c_i - 1) x_i + e_i eps_i (+ sigma_i z_i)            drift
 //   x'_{i+1} = x_t + sum_{l<=j} d_{t+l}  (compensated)            Eq. 1
 //   err_j  partial of sum (x'_{i+1} - x_{i+1})^2                  Eq. 2
 //   del_j  partial of sum |x'_{i+1} - xhat_{i+1}| (next iteration) Eq. 4
@@ -170,6 +170,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
     const int r = rk[j];
     if (r >= n_miss) set_status(d.ctl, kDevBadRank);
     const float cm1 = d.cm1[i], ec = d.ecoef[i];
+    const float sg = d.noise ? d.sigma[i] : 0.f;
     const int slot = i % P;
     float ev = 0.f, dv = 0.f;
     if (live) {
@@ -185,10 +186,12 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
       } else {
         xo = xfill;
       }
+      V<VEC> zn{};
+      if (d.noise) zn = ldv<VEC>(d.noise + ((int64_t)b * d.T + i) * D + col);  // the draw z_i
       V<VEC> xn;
 #pragma unroll
       for (int v = 0; v < VEC; ++v) {
-        const float dr = cm1 * xcur.a[v] + ec * eps.a[v];
+        const float dr = fmaf(sg, zn.a[v], cm1 * xcur.a[v] + ec * eps.a[v]);
         const float y = dr - comp.a[v];
         const float s = acc.a[v] + y;
         comp.a[v] = (s - acc.a[v]) - y;
@@ -303,7 +306,11 @@ cudaError_t launch_gather(const Dev& d, cudaStream_t st) {
 cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream_t st,
                                 int* nchunk_out) {
   const size_t smem = (size_t)2 * (kPlainThreads / 32) * d.P * sizeof(float);
-  if (d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0) {
+  // float4 rows need every row base 16-byte aligned: D % 4 == 0 and aligned
+  // eps (and draws) pointers; the workspace arrays are 256-byte aligned
+  const bool aligned = (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0 &&
+                       (reinterpret_cast<uintptr_t>(d.noise) & 15) == 0;
+  if (d.D % 4 == 0 && aligned) {
     const int nchunk = (int)((d.D + kPlainThreads * 4 - 1) / (kPlainThreads * 4));
     *nchunk_out = nchunk;
     return launch_ex(k_update_plain<4>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps,

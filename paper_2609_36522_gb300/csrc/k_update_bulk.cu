@@ -446,12 +446,14 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
 // Eq. 2 errors and the next-iteration Eq. 4 distances. Per-lane err/distance
 // values go through a transposed shared-memory buffer; after a second barrier
 // one thread per (quantity, position) sums its row into the strip partial.
-// Two CTA barriers per launch in all.
-template <int V, int NW>
+// Two CTA barriers per launch in all. With NOISE (stochastic steps) every
+// position stages a fourth row, the draw z_i, and its drift gains sigma_i z_i.
+template <int V, int NW, bool NOISE = false>
 struct SegShape {
   static constexpr int SEG = 32 * V;
-  __host__ __device__ static size_t meta_bytes(int P) { return ((size_t)P * 20 + 127) / 128 * 128; }
-  __host__ __device__ static size_t rows_bytes(int P) { return (size_t)P * 3 * SEG * sizeof(float); }
+  static constexpr int NR = NOISE ? 4 : 3;  // staged rows per position
+  __host__ __device__ static size_t meta_bytes(int P) { return ((size_t)P * 24 + 127) / 128 * 128; }
+  __host__ __device__ static size_t rows_bytes(int P) { return (size_t)P * NR * SEG * sizeof(float); }
   __host__ __device__ static size_t red_bytes(int P) { return ((size_t)2 * P * 33 * sizeof(float) + 127) / 128 * 128; }
   static constexpr size_t kTotBytes = (size_t)NW * SEG * 2 * sizeof(float);
   static constexpr size_t kBarBytes = 128;  // NW <= 16 mbarriers
@@ -460,11 +462,12 @@ struct SegShape {
   }
 };
 
-template <int V, int NW>
+template <int V, int NW, bool NOISE>
 __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __restrict__ beps, int nstrip,
                                                         uint32_t wait_limit) {
-  using Sh = SegShape<V, NW>;
+  using Sh = SegShape<V, NW, NOISE>;
   constexpr int SEG = Sh::SEG;
+  constexpr int NR = Sh::NR;
   static_assert(NW <= 16, "one mbarrier per warp in a 128-byte area");
   extern __shared__ __align__(128) unsigned char smem_raw[];
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -479,12 +482,13 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   float* s_ec = reinterpret_cast<float*>(q + (size_t)P * 8);
   int32_t* s_slot = reinterpret_cast<int32_t*>(q + (size_t)P * 12);  // (t+j) mod P
   int32_t* s_nxt = reinterpret_cast<int32_t*>(q + (size_t)P * 16);   // (t+j+1) mod (P+1)
+  float* s_sig = reinterpret_cast<float*>(q + (size_t)P * 20);       // sigma_i (stochastic steps)
   q += Sh::meta_bytes(P);
   float* s_tot = reinterpret_cast<float*>(q);   // [NW][SEG][2]
   q += Sh::kTotBytes;
   float* s_red = reinterpret_cast<float*>(q);   // [2][P][33]
   q += Sh::red_bytes(P);
-  float* s_rows = reinterpret_cast<float*>(q);  // [P][3][SEG]: eps, old x_{i+1}, xhat_{i+1}
+  float* s_rows = reinterpret_cast<float*>(q);  // [P][NR][SEG]: eps, old x_{i+1}, xhat_{i+1} (, z_i)
 
   const Traj tr = d.traj[b];
   const int n_miss = d.ctl->n_miss;
@@ -496,6 +500,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
     s_nxt[j] = (t + j + 1) % (P + 1);
     s_cm1[j] = d.cm1[t + j];
     s_ec[j] = d.ecoef[t + j];
+    if (NOISE) s_sig[j] = d.sigma[t + j];
   }
   if (tid == 0) {
     for (int k = 0; k < NW; ++k) mbar_init(&bar[k], 1);
@@ -528,20 +533,22 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   {
     uint32_t total = 0;
     for (int j = j0 + lane; j < j1; j += 32) {
-      total += seg_bytes * (1u + ((t + j + 1 <= e) ? 1u : 0u) + (((j + 1 < p) && (s_rank[j + 1] < 0)) ? 1u : 0u));
+      total += seg_bytes * ((NOISE ? 2u : 1u) + ((t + j + 1 <= e) ? 1u : 0u) +
+                            (((j + 1 < p) && (s_rank[j + 1] < 0)) ? 1u : 0u));
     }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) total += __shfl_xor_sync(0xffffffffu, total, o);
     if (lane == 0 && j0 < j1) mbar_arrive_expect_tx(&bar[warp], total);
     __syncwarp();
     for (int j = j0 + lane; j < j1; j += 32) {
-      float* rowp = s_rows + (size_t)j * 3 * SEG;
+      float* rowp = s_rows + (size_t)j * NR * SEG;
       const int r = s_rank[j];
       const float* src_eps = (r >= 0) ? beps + (int64_t)r * D + c0 : Eh + (int64_t)s_slot[j] * D + c0;
       bulk_g2s(rowp, src_eps, seg_bytes, &bar[warp]);
       if (t + j + 1 <= e) bulk_g2s(rowp + SEG, Xb + (int64_t)s_nxt[j] * D + c0, seg_bytes, &bar[warp]);
       if ((j + 1 < p) && (s_rank[j + 1] < 0))
         bulk_g2s(rowp + 2 * SEG, Xh + (int64_t)s_slot[j + 1] * D + c0, seg_bytes, &bar[warp]);
+      if (NOISE) bulk_g2s(rowp + 3 * SEG, d.noise + ((int64_t)b * d.T + t + j) * D + c0, seg_bytes, &bar[warp]);
     }
   }
   Vec<V> xstart{}, xfill{};
@@ -559,7 +566,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   if (j0 == 0) {
     xc0 = xstart;
   } else if (j0 < j1 && t + j0 <= e && live) {
-    xc0 = ldv<V>(s_rows + (size_t)(j0 - 1) * 3 * SEG + SEG + lane * V);
+    xc0 = ldv<V>(s_rows + (size_t)(j0 - 1) * NR * SEG + SEG + lane * V);
   }
 
   // phase 1: compensated sum of this segment's drifts
@@ -569,11 +576,17 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   if (live) {
     Vec<V> xc = xc0;
     for (int j = j0; j < j1; ++j) {
-      const float* rowp = s_rows + (size_t)j * 3 * SEG;
+      const float* rowp = s_rows + (size_t)j * NR * SEG;
       const Vec<V> eps = ldv<V>(rowp + lane * V);
       const float cm1 = s_cm1[j], ec = s_ec[j];
+      Vec<V> zn{};
+      if (NOISE) zn = ldv<V>(rowp + 3 * SEG + lane * V);
 #pragma unroll
-      for (int v = 0; v < V; ++v) acc_add(rh[v], rl[v], fmaf(cm1, xc.a[v], ec * eps.a[v]));
+      for (int v = 0; v < V; ++v) {
+        float dr = fmaf(cm1, xc.a[v], ec * eps.a[v]);
+        if (NOISE) dr = fmaf(s_sig[j], zn.a[v], dr);
+        acc_add(rh[v], rl[v], dr);
+      }
       xc = (t + j + 1 <= e) ? ldv<V>(rowp + SEG + lane * V) : xfill;
     }
   }
@@ -599,7 +612,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   {
     Vec<V> xc = xc0;
     for (int j = j0; j < j1; ++j) {
-      const float* rowp = s_rows + (size_t)j * 3 * SEG;
+      const float* rowp = s_rows + (size_t)j * NR * SEG;
       float ev = 0.f, dv = 0.f;
       if (live) {
         const Vec<V> eps = ldv<V>(rowp + lane * V);
@@ -610,10 +623,14 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
         }
         const float cm1 = s_cm1[j], ec = s_ec[j];
         const Vec<V> xo = (t + j + 1 <= e) ? ldv<V>(rowp + SEG + lane * V) : xfill;
+        Vec<V> zn{};
+        if (NOISE) zn = ldv<V>(rowp + 3 * SEG + lane * V);
         Vec<V> xn;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-          acc_add(ch[v], cl[v], fmaf(cm1, xc.a[v], ec * eps.a[v]));
+          float dr = fmaf(cm1, xc.a[v], ec * eps.a[v]);
+          if (NOISE) dr = fmaf(s_sig[j], zn.a[v], dr);
+          acc_add(ch[v], cl[v], dr);
           xn.a[v] = ch[v] + cl[v];
           const float df = xn.a[v] - xo.a[v];
           ev = fmaf(df, df, ev);
@@ -652,17 +669,17 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
 
 constexpr size_t kSegSmemMax = 200 * 1024;
 
-template <int V, int NW>
+template <int V, int NW, bool NOISE = false>
 bool seg_fits(const Dev& d) {
-  return SegShape<V, NW>::smem_bytes(d.P) <= kSegSmemMax;
+  return SegShape<V, NW, NOISE>::smem_bytes(d.P) <= kSegSmemMax;
 }
 
-template <int V, int NW>
+template <int V, int NW, bool NOISE = false>
 cudaError_t launch_seg(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
-  using Sh = SegShape<V, NW>;
+  using Sh = SegShape<V, NW, NOISE>;
   const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
   const size_t smem = Sh::smem_bytes(d.P);
-  auto kern = k_update_seg<V, NW>;
+  auto kern = k_update_seg<V, NW, NOISE>;
   static size_t configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -711,8 +728,11 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
 
 bool update_bulk_supported(const Dev& d, const float* batch_eps) {
   // 16-byte granularity of bulk copies: every row segment must start on a
-  // 16-byte boundary and be a multiple of 16 bytes long.
-  return d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0;
+  // 16-byte boundary and be a multiple of 16 bytes long. Stochastic steps
+  // stage the draws too, in the segment form only.
+  const bool ok = d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0;
+  if (!d.noise) return ok;
+  return ok && (reinterpret_cast<uintptr_t>(d.noise) & 15) == 0 && seg_fits<2, 8, true>(d);
 }
 
 // Four columns per lane halve the per-element bookkeeping and the strip
@@ -720,8 +740,9 @@ bool update_bulk_supported(const Dev& d, const float* batch_eps) {
 // grid still fills the GPU in about one wave (window 100 at 4x64x64: 128 CTAs)
 // or several CTAs fit per SM (window 32), not for multi-wave grids of one CTA
 // per SM (window 64 at 4x128x128).
+template <bool NOISE>
 bool prefer_wide_strips(const Dev& d) {
-  if (!seg_fits<4, 8>(d)) return false;
+  if (!seg_fits<4, 8, NOISE>(d)) return false;
   static int nsm[64] = {};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
@@ -729,16 +750,20 @@ bool prefer_wide_strips(const Dev& d) {
     nsm[dev] = 0;
     return false;
   }
-  const size_t smem = SegShape<4, 8>::smem_bytes(d.P) + 4096;  // + static shared memory and reserve
+  const size_t smem = SegShape<4, 8, NOISE>::smem_bytes(d.P) + 4096;  // + static shared memory and reserve
   const int per_sm = (int)((size_t)(228 * 1024) / smem);
   const int64_t grid = (int64_t)d.B * ((d.D + SegShape<4, 8>::SEG - 1) / SegShape<4, 8>::SEG);
   return per_sm >= 2 || grid <= nsm[dev];
 }
 
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
+  if (d.noise) {  // stochastic steps: the segment form with the draws staged (update_bulk_supported)
+    if (prefer_wide_strips<true>(d)) return launch_seg<4, 8, true>(d, batch_eps, st, nchunk_out);
+    return launch_seg<2, 8, true>(d, batch_eps, st, nchunk_out);
+  }
   switch (d.bulk_cfg) {
     case 0:  // whole window in shared memory when it fits, else the tiled pipeline
-      if (prefer_wide_strips(d)) return launch_seg<4, 8>(d, batch_eps, st, nchunk_out);
+      if (prefer_wide_strips<false>(d)) return launch_seg<4, 8>(d, batch_eps, st, nchunk_out);
       if (seg_fits<2, 8>(d)) return launch_seg<2, 8>(d, batch_eps, st, nchunk_out);
       return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
     case 1: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);

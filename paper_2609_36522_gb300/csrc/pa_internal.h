@@ -62,7 +62,7 @@ inline Layout make_layout(int T, int P, int64_t D, int B) {
   L.Xhat = take((size_t)B * P * row);             // cache inputs, slot = i mod P
   L.Ehat = take((size_t)B * P * row);             // cache outputs, slot = i mod P
   L.batch_x = take((size_t)B * P * row);          // gathered misses
-  L.coef = take((size_t)2 * T * sizeof(float));   // (c_i - 1, e_i)
+  L.coef = take((size_t)3 * T * sizeof(float));   // (c_i - 1, e_i, sigma_i)
   L.traj = take((size_t)B * sizeof(Traj));
   L.ctl = take(sizeof(Ctl));
   L.rank = take((size_t)B * P * sizeof(int32_t));
@@ -85,6 +85,8 @@ struct Dev {
   float* batch_x;
   const float* cm1;   // c_i - 1
   const float* ecoef; // e_i
+  const float* sigma; // sigma_i of stochastic steps (0 for eta = 0)
+  const float* noise; // [B][T][D] draws z_i of stochastic steps, caller-owned; NULL for eta = 0
   Traj* traj;
   Ctl* ctl;
   int32_t* rank;      // [B][P] rank of window position j among the misses, -1 = hit

@@ -2,6 +2,7 @@
 // workspace carving, DDIM drift coefficients and kernel dispatch.
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -44,6 +45,8 @@ struct pa_solver {
   int last_nchunk;
   int64_t launches;
   pa::Ctl* host_ctl; // pinned mirror of the device Ctl
+  std::vector<double> alphas;  // the schedule, kept for pa_set_noise
+  double eta;
   // optional CUDA-event timing of the Picard-update kernel
   bool timing;
   std::vector<cudaEvent_t> ev;  // pairs: [2k] before, [2k+1] after launch k
@@ -51,6 +54,28 @@ struct pa_solver {
 };
 
 namespace {
+
+// DDIM step i -> i+1 with noise scale sigma_i = eta sqrt((1 - a') / (1 - a))
+// sqrt(1 - a / a'), written as x + s(x, eps, z) with
+// s = (c_i - 1) x + e_i eps + sigma_i z, c_i = sqrt(a' / a),
+// e_i = sqrt(1 - a' - sigma_i^2) - sqrt(a' (1 - a) / a); c_i - 1 is formed
+// without cancellation. fp64 on the host, stored as fp32 [3][T].
+std::vector<float> step_coefficients(const std::vector<double>& al, double eta) {
+  const int T = (int)al.size() - 1;
+  std::vector<float> hc(3 * (size_t)T);
+  for (int i = 0; i < T; ++i) {
+    const double a = al[i], an = al[i + 1];
+    const double r = an / a;
+    const double c = std::sqrt(r);
+    const double cm1 = (r - 1.0) / (c + 1.0);
+    const double sig = eta * std::sqrt((1.0 - an) / (1.0 - a)) * std::sqrt(1.0 - a / an);
+    const double e = std::sqrt(std::max(0.0, 1.0 - an - sig * sig)) - std::sqrt(an) * std::sqrt(1.0 - a) / std::sqrt(a);
+    hc[i] = (float)cm1;
+    hc[T + i] = (float)e;
+    hc[2 * (size_t)T + i] = (float)sig;
+  }
+  return hc;
+}
 
 pa_status cuda_fail(const char* where, cudaError_t e) {
   pa::set_error(std::string(where) + ": " + cudaGetErrorString(e));
@@ -173,6 +198,10 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   float* coef = reinterpret_cast<float*>(w + L.coef);
   d.cm1 = coef;
   d.ecoef = coef + T;
+  d.sigma = coef + 2 * (size_t)T;
+  d.noise = nullptr;
+  s->alphas.assign(alphas_cumprod, alphas_cumprod + T + 1);
+  s->eta = 0.0;
   d.traj = reinterpret_cast<pa::Traj*>(w + L.traj);
   d.ctl = reinterpret_cast<pa::Ctl*>(w + L.ctl);
   d.rank = reinterpret_cast<int32_t*>(w + L.rank);
@@ -188,18 +217,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.wait_limit = pa::kWaitLimit;
   s->update_kind = (D % 4 == 0) ? 1 : 0;
 
-  // DDIM (eta = 0) step i -> i+1 written as x + s(x, eps) with
-  // s = (c_i - 1) x + e_i eps; c_i - 1 is formed without cancellation.
-  std::vector<float> hc(2 * (size_t)T);
-  for (int i = 0; i < T; ++i) {
-    const double a = alphas_cumprod[i], an = alphas_cumprod[i + 1];
-    const double r = an / a;
-    const double c = std::sqrt(r);
-    const double cm1 = (r - 1.0) / (c + 1.0);
-    const double e = std::sqrt(1.0 - an) - std::sqrt(an) * std::sqrt(1.0 - a) / std::sqrt(a);
-    hc[i] = (float)cm1;
-    hc[T + i] = (float)e;
-  }
+  const std::vector<float> hc = step_coefficients(s->alphas, 0.0);  // DDIM (eta = 0)
   cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), sizeof(pa::Ctl), cudaHostAllocDefault);
   if (e != cudaSuccess) {
     delete s;
@@ -215,6 +233,23 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
     return cuda_fail("pa_create", e);
   }
   *out = s;
+  return PA_OK;
+}
+
+pa_status pa_set_noise(pa_solver* s, double eta, const float* noise_dev) {
+  if (!s) return arg_fail("pa_set_noise: solver is NULL");
+  if (s->state == St::Stepped) return state_fail("pa_set_noise");
+  if (!(eta >= 0.0 && eta <= 1.0)) return arg_fail("pa_set_noise: eta must be in [0, 1]");
+  if (eta > 0.0 && !noise_dev) return arg_fail("pa_set_noise: eta > 0 needs the draws (noise_dev)");
+  if (eta > 0.0 && (reinterpret_cast<uintptr_t>(noise_dev) & 15) != 0)
+    return arg_fail("pa_set_noise: noise_dev must be 16-byte aligned");
+  const std::vector<float> hc = step_coefficients(s->alphas, eta);
+  cudaError_t e = cudaMemcpyAsync(s->ws + s->L.coef, hc.data(), hc.size() * sizeof(float), cudaMemcpyHostToDevice,
+                                  s->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);  // hc is a local buffer
+  if (e != cudaSuccess) return cuda_fail("pa_set_noise", e);
+  s->eta = eta;
+  s->d.noise = eta > 0.0 ? noise_dev : nullptr;
   return PA_OK;
 }
 

@@ -52,6 +52,19 @@ class Solver:
         nb = int(np.prod(shape)) * torch.tensor([], dtype=dtype).element_size()
         return self.workspace[off: off + nb].view(dtype).view(*shape)
 
+    def set_noise(self, eta, noise=None):
+        """Stochastic steps: noise is a CUDA float32 [batch][T][D] tensor of
+        N(0, 1) draws (kept alive by this object); eta = 0 restores DDIM."""
+        if eta == 0.0:
+            self._noise_keepalive = None
+            abi.pa_set_noise(self.h, 0.0, None)
+            return
+        if (not isinstance(noise, torch.Tensor) or not noise.is_cuda or noise.dtype != torch.float32
+                or not noise.is_contiguous() or noise.numel() != self.batch * self.T * self.D):
+            raise ValueError("noise must be a contiguous CUDA float32 [batch][T][D] tensor")
+        self._noise_keepalive = noise
+        abi.pa_set_noise(self.h, eta, noise.data_ptr())
+
     def init(self, x_init):
         """x_init: [batch][D] fp32 tensor (CUDA or CPU, contiguous)."""
         x = x_init if isinstance(x_init, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(x_init))

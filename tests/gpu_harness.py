@@ -13,7 +13,7 @@ def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True):
     a, x0, mu = W.inputs(w)
     thr = w.cache_thresh if cache_thresh is None else cache_thresh
     return run_picard(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr,
-                      use_cache=use_cache)
+                      use_cache=use_cache, eta=w.eta, noise=W.noise(w))
 
 
 def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=None,
@@ -39,6 +39,12 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
     if gmm_form is not None:
         g.set_form(gmm_form)
     eps_buf = torch.empty(max_rows, w.D, dtype=torch.float32, device=dev)
+    noise_keep = None
+    if w.eta != 0.0:
+        z = torch.from_numpy(W.noise(w)).to(dev).reshape(-1)
+        noise_keep = z
+        from paper_2609_36522_gb300 import abi as _abi
+        _abi.pa_set_noise(s.h, w.eta, z.data_ptr())
     x_init = torch.from_numpy(x0)
     if x_init_host:
         x_init = x_init.pin_memory()

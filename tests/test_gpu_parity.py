@@ -229,3 +229,56 @@ def test_update_kernels_agree(kind):
     assert np.array_equal(ref["log"], got["log"])
     scale = np.abs(ref["x_final"]).max()
     assert np.abs(ref["x_final"] - got["x_final"]).max() <= 1e-6 * scale
+
+
+# ---- stochastic steps (eta > 0): DDPM over the full 1000-step schedule -------
+
+def test_ddpm_full_schedule():
+    """DDPM (eta = 1, T = 1000, window 64): decisions, miss lists and NFE
+    bit-exact, final latents within 1e-5 of the oracle."""
+    w = W.DDPM
+    rel = compare(w, oracle_run(w), gpu_run(w))
+    assert rel.max() <= 1e-5, rel
+
+
+@pytest.mark.parametrize("eta", [1.0, 0.5])
+@pytest.mark.parametrize("kind", [0, 1])
+def test_noisy_steps_small(eta, kind):
+    """Stochastic steps on small cases through both update kernels."""
+    w = W.TINY.with_(T=16, window=8, eta=eta)
+    rel = compare(w, oracle_run(w), gpu_run(w, update_kernel=kind))
+    assert rel.max() <= 1e-5, rel
+
+
+@pytest.mark.parametrize("shape,window", [((3, 7, 9), 5), ((4, 32, 32), 40), ((4, 16, 16), 128)])
+def test_noisy_steps_shapes(shape, window):
+    """Ragged D (plain kernel), a window past T, and a 128-point window."""
+    w = W.TINY.with_(T=100, window=window, latent_shape=shape, K=4, eta=1.0)
+    rel = compare(w, oracle_run(w), gpu_run(w))
+    assert rel.max() <= 1e-5, rel
+
+
+def test_noisy_misaligned_draws_rejected():
+    """Draws not 16-byte aligned are refused on the host (no kernel runs)."""
+    import torch
+    from paper_2609_36522_gb300 import abi
+    from paper_2609_36522_gb300.solver import Solver
+    w = W.TINY.with_(T=20, window=8, latent_shape=(4, 8, 8), eta=1.0)
+    a, x0, mu = W.inputs(w)
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch)
+    buf = torch.zeros(w.batch * w.T * w.D + 1, dtype=torch.float32, device="cuda")
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_set_noise(s.h, 1.0, buf[1:].data_ptr())
+    assert e.value.status == abi.PA_ERR_ARG
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_set_noise(s.h, 1.5, buf.data_ptr())
+    assert e.value.status == abi.PA_ERR_ARG
+    s.close()
+
+
+def test_eta_zero_restores_ddim():
+    """pa_set_noise(eta = 0) gives the DDIM run bit for bit."""
+    w = W.TINY.with_(T=30, window=10, latent_shape=(4, 16, 16))
+    plain = gpu_run(w)
+    again = gpu_run(w.with_(eta=0.0))
+    assert np.array_equal(plain["x_final"], again["x_final"])
