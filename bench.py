@@ -333,40 +333,71 @@ def run_ours(args):
     nfe, hits = st0["nfe"], st0["hits"]
     upd_bytes, other_bytes = iteration_bytes(log, w)
 
-    # One Picard iteration (gather, denoiser dots + out, update, decision: 5 kernels) as a
-    # CUDA graph; the update kernel's timing events are captured with it.
+    # One generation (n_iters Picard iterations: gather, denoiser, update and
+    # decision kernels each) as a CUDA graph. The timed graph also records CUDA
+    # events around every update-kernel launch (the roofline's kernel time); the
+    # plain graph has no event nodes and gives the iteration rate.
     s.init(x_dev)
     one_iteration()                       # eager warm-up of every launch path
     stream.synchronize()
-    abi.pa_set_kernel_timing(s.h, True)
-    abi.pa_kernel_timing(s.h, reset=True)
-    graph = torch.cuda.CUDAGraph()
-    s.init(x_dev)
-    stream.synchronize()
-    gmm0, sol0 = g.launches(), s.stats()["launches"]
-    with torch.cuda.graph(graph, stream=stream):
-        one_iteration()
-    # gather, update, decision + denoiser kernels
-    kernels_per_iter = (s.stats()["launches"] - sol0) + (g.launches() - gmm0)
 
-    def generation(timed):
+    def capture(timed):
+        abi.pa_set_kernel_timing(s.h, timed)
+        abi.pa_kernel_timing(s.h, reset=True)
         s.init(x_dev)
-        it_ms = upd = 0.0
-        for _ in range(n_iters):
-            if flush is not None:
-                flush.zero_()
-            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            e0.record(stream)
-            graph.replay()
-            e1.record(stream)
-            if timed:
+        stream.synchronize()
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=stream):
+            for _ in range(n_iters):
+                one_iteration()
+        abi.pa_set_kernel_timing(s.h, False)
+        return gr
+
+    gmm0, sol0 = g.launches(), s.stats()["launches"]
+    graph_plain = capture(False)
+    # gather, update, decision + denoiser kernels of one Picard iteration
+    kernels_per_iter = ((s.stats()["launches"] - sol0) + (g.launches() - gmm0)) // n_iters
+    graph_timed = capture(True)
+
+    def generation(gr, timed):
+        """L2 flushed, then one generation timed with one event pair."""
+        s.init(x_dev)
+        if flush is not None:
+            flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        gr.replay()
+        e1.record(stream)
+        e1.synchronize()
+        ms = e0.elapsed_time(e1)
+        upd = abi.pa_kernel_timing(s.h, reset=False)[0] if timed else 0.0
+        return ms, upd
+
+    def cold_iterations(reps):
+        """Per-iteration time with L2 flushed before every Picard iteration."""
+        single = torch.cuda.CUDAGraph()
+        s.init(x_dev)
+        stream.synchronize()
+        with torch.cuda.graph(single, stream=stream):
+            one_iteration()
+        tot, n = 0.0, 0
+        for _ in range(reps):
+            s.init(x_dev)
+            for _ in range(n_iters):
+                if flush is not None:
+                    flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                single.replay()
+                e1.record(stream)
                 e1.synchronize()
-                it_ms += e0.elapsed_time(e1)
-                upd += abi.pa_kernel_timing(s.h, reset=False)[0]
-        return it_ms, upd
+                tot += e0.elapsed_time(e1)
+                n += 1
+        return 1000.0 * tot / max(n, 1)
 
     for _ in range(args.warmup):
-        generation(False)
+        generation(graph_plain, False)
+        generation(graph_timed, True)
     stream.synchronize()
     assert s.poll() == 0, "solver did not finish within the learned iteration count"
 
@@ -376,10 +407,13 @@ def run_ours(args):
     barrier()
     stream.synchronize()
     wall0 = time.perf_counter()
-    dev_ms = upd_ms = 0.0
+    dev_ms = upd_ms = timed_ms = 0.0
     for _ in range(args.steps):
-        a_ms, u_ms = generation(True)
+        a_ms, _ = generation(graph_plain, False)
         dev_ms += a_ms
+        assert s.poll() == 0
+        t_ms, u_ms = generation(graph_timed, True)     # same work, update kernel bracketed by events
+        timed_ms += t_ms
         upd_ms += u_ms
         assert s.poll() == 0
     stream.synchronize()
@@ -387,10 +421,10 @@ def run_ours(args):
     wall = time.perf_counter() - wall0
     st1 = s.stats()
     assert st1["iters"] == n_iters and st1["nfe"] == nfe, (st1, n_iters, nfe)
-    abi.pa_set_kernel_timing(s.h, False)
     time.sleep(0.2)
     clk = clocks.stop()
-    launches = args.steps * (n_iters * kernels_per_iter + 1)   # + init plan per generation
+    launches = 2 * args.steps * (n_iters * kernels_per_iter + 1)   # both graphs; + init plan per generation
+    cold_us = cold_iterations(max(1, min(args.steps, 10)))
 
     units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
     value = units / secs
@@ -461,12 +495,18 @@ def run_ours(args):
                                                  if g.form() == 1 else "CUDA cores (fp32 FMA)"),
                        "parallelism": f"replicas x{world} (independent trajectories)",
                        "l2": ("not flushed" if args.no_flush else
-                              "256 MiB write before every Picard iteration, outside the timed events"),
-                       "timing": "CUDA events around each Picard iteration (one CUDA-graph replay of "
-                                 "the gather, denoiser, update and decision kernels) on the launch stream"},
+                              "256 MiB write before every generation (between timed steps), outside the "
+                              "timed events"),
+                       "timing": "CUDA events around each generation: one CUDA-graph replay of its Picard "
+                                 "iterations (gather, denoiser, update and decision kernels each) on the "
+                                 "launch stream; the update kernel's own events come from a second graph "
+                                 "of the same generation, replayed alternately"},
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
             "solver_step_gbps": gb_step,
+            "cold_iteration_us": cold_us,
+            "cold_iteration_note": "one Picard iteration with L2 flushed before every iteration, "
+                                   "CUDA events around each (conservative; includes one event pair per iteration)",
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,
