@@ -478,7 +478,7 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
   if (r0 >= n_rows) return;
   const int nr = min(kTcRows, n_rows - r0);
   const int Kp = tc_npad(K);
-  const uint32_t ncols = Kp < 32 ? 32u : (uint32_t)Kp;  // TMEM columns: a power of two >= 32
+  const uint32_t ncols = 2 * Kp < 32 ? 32u : (uint32_t)(2 * Kp);  // TMEM columns: a power of two >= 32
   const int64_t c0 = (int64_t)blockIdx.x * kTcCols;
   float* A_hi = reinterpret_cast<float*>(smem_raw);
   float* A_lo = A_hi + kTcRows * kTcCols;
@@ -542,17 +542,19 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
   }
   if (tid == 0 && ok) {
     tc_fence_after_sync();
-    const uint32_t idesc = tc_idesc_tf32(kTcRows, Kp);
+    // The means image's hi rows are directly followed by its lo rows, so one
+    // N = 2 Kp product gives hi*hi in columns [0, Kp) and hi*lo in [Kp, 2 Kp);
+    // lo*hi then accumulates into [0, Kp): two MMAs per k-step.
+    const uint32_t idesc2 = tc_idesc_tf32(kTcRows, 2 * Kp), idesc1 = tc_idesc_tf32(kTcRows, Kp);
     const uint32_t a_hi = smem_u32(A_hi), a_lo = smem_u32(A_lo);
-    const uint32_t b_hi = smem_u32(B_img), b_lo = b_hi + (uint32_t)(Kp * kTcCols * sizeof(float));
+    const uint32_t b_hi = smem_u32(B_img);
     const uint32_t sbo = (kTcCols / 4) * 128;  // next 8-row group
     for (int ks = 0; ks < kTcCols / 8; ++ks) {
       const uint32_t ko = (uint32_t)ks * 256;  // two core matrices along K per step
       const uint64_t dah = tc_smem_desc(a_hi + ko, 128, sbo), dal = tc_smem_desc(a_lo + ko, 128, sbo);
-      const uint64_t dbh = tc_smem_desc(b_hi + ko, 128, sbo), dbl = tc_smem_desc(b_lo + ko, 128, sbo);
-      tc_mma_tf32(taddr, dah, dbh, idesc, ks > 0 ? 1u : 0u);
-      tc_mma_tf32(taddr, dah, dbl, idesc, 1u);
-      tc_mma_tf32(taddr, dal, dbh, idesc, 1u);
+      const uint64_t db = tc_smem_desc(b_hi + ko, 128, sbo);
+      tc_mma_tf32(taddr, dah, db, idesc2, ks > 0 ? 1u : 0u);
+      tc_mma_tf32(taddr, dal, db, idesc1, 1u);
     }
     tc_commit(&bar_mma);
   }
@@ -566,8 +568,11 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
   if (warp < 4 && ok) {  // warp w reads TMEM lanes (rows) 32w .. 32w + 31
     const int row = warp * 32 + lane;
     for (int cb = 0; cb < Kp; cb += 16) {
-      float v[16];
+      float v[16], w[16];
       tmem_ld16(taddr + ((uint32_t)(warp * 32) << 16) + (uint32_t)cb, v);
+      tmem_ld16(taddr + ((uint32_t)(warp * 32) << 16) + (uint32_t)(Kp + cb), w);
+#pragma unroll
+      for (int u = 0; u < 16; ++u) v[u] += w[u];  // (hi*hi + lo*hi) + hi*lo
       if constexpr (CL > 1) {
 #pragma unroll
         for (int u = 0; u < 16; ++u) part[row * Kp + cb + u] = v[u];
@@ -698,8 +703,8 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
   }
   // Default: the tensor cores for K > 16. At K <= 16 the contraction is under
   // a microsecond of CUDA-core FMA work per call and the CUDA-core kernel's
-  // shorter per-CTA chain wins (measured at 4x64x64: 46.9 vs 49.7 us per
-  // Picard iteration); at K = 64 the tensor cores win (172.2 vs 186.2 us at
+  // shorter per-CTA chain wins (measured at 4x64x64: 30.1 vs 33.1 us per
+  // Picard iteration); at K = 64 the tensor cores win (151.9 vs 170.4 us at
   // 4x128x128).
   g->use_tc = g->tc_ok && K > kTcMinK;
   if (e == cudaSuccess) e = cudaStreamSynchronize(g->st);
