@@ -490,31 +490,28 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   q += Sh::red_bytes(P);
   float* s_rows = reinterpret_cast<float*>(q);  // [P][NR][SEG]: eps, old x_{i+1}, xhat_{i+1} (, z_i)
 
+  // Everything read before pdl_wait() was written two or more kernels back
+  // (the previous update and decision kernels); only the batch eps rows come
+  // from the denoiser just before.
   const Traj tr = d.traj[b];
   const int n_miss = d.ctl->n_miss;
-  for (int j = tid; j < P; j += NW * 32) s_rank[j] = d.rank[b * P + j];
   if (tr.p == 0) return;
   const int t = tr.t, p = tr.p, e = tr.e;
   for (int j = tid; j < p; j += NW * 32) {
+    int r = d.rank[b * P + j];
+    if (r >= n_miss) {  // never expected: keep every copy in bounds and report it
+      atomicCAS(&d.ctl->status, kDevOk, kDevBadRank);
+      r = -1;
+    }
+    s_rank[j] = r;
     s_slot[j] = (t + j) % P;
     s_nxt[j] = (t + j + 1) % (P + 1);
-    s_cm1[j] = d.cm1[t + j];
-    s_ec[j] = d.ecoef[t + j];
-    if (NOISE) s_sig[j] = d.sigma[t + j];
   }
   if (tid == 0) {
     for (int k = 0; k < NW; ++k) mbar_init(&bar[k], 1);
     fence_barrier_init();
   }
   __syncthreads();
-  for (int j = tid; j < p; j += NW * 32) {
-    if (s_rank[j] >= n_miss) {  // never expected: keep every copy in bounds and report it
-      atomicCAS(&d.ctl->status, kDevOk, kDevBadRank);
-      s_rank[j] = -1;
-    }
-  }
-  __syncthreads();
-  pdl_wait();  // the eps rows come from the denoiser that ran just before
 
   const int strip = blockIdx.x;
   const int64_t c0 = (int64_t)strip * SEG;
@@ -529,7 +526,9 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   const int j0 = warp * L;
   const int j1 = (j0 + L) < p ? (j0 + L) : p;
 
-  // this warp's copies: the whole byte count first, then one lane per position
+  // this warp's copies: the whole byte count first, then one lane per
+  // position; everything but the misses' batch eps rows goes out before
+  // pdl_wait() and overlaps the denoiser's tail
   {
     uint32_t total = 0;
     for (int j = j0 + lane; j < j1; j += 32) {
@@ -542,15 +541,25 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
     __syncwarp();
     for (int j = j0 + lane; j < j1; j += 32) {
       float* rowp = s_rows + (size_t)j * NR * SEG;
-      const int r = s_rank[j];
-      const float* src_eps = (r >= 0) ? beps + (int64_t)r * D + c0 : Eh + (int64_t)s_slot[j] * D + c0;
-      bulk_g2s(rowp, src_eps, seg_bytes, &bar[warp]);
+      if (s_rank[j] < 0) bulk_g2s(rowp, Eh + (int64_t)s_slot[j] * D + c0, seg_bytes, &bar[warp]);
       if (t + j + 1 <= e) bulk_g2s(rowp + SEG, Xb + (int64_t)s_nxt[j] * D + c0, seg_bytes, &bar[warp]);
       if ((j + 1 < p) && (s_rank[j + 1] < 0))
         bulk_g2s(rowp + 2 * SEG, Xh + (int64_t)s_slot[j + 1] * D + c0, seg_bytes, &bar[warp]);
       if (NOISE) bulk_g2s(rowp + 3 * SEG, d.noise + ((int64_t)b * d.T + t + j) * D + c0, seg_bytes, &bar[warp]);
     }
+    pdl_wait();  // the batch eps rows come from the denoiser that ran just before
+    for (int j = j0 + lane; j < j1; j += 32) {
+      const int r = s_rank[j];
+      if (r >= 0) bulk_g2s(s_rows + (size_t)j * NR * SEG, beps + (int64_t)r * D + c0, seg_bytes, &bar[warp]);
+    }
   }
+  // this warp's step coefficients (read by this warp only)
+  for (int j = j0 + lane; j < j1; j += 32) {
+    s_cm1[j] = d.cm1[t + j];
+    s_ec[j] = d.ecoef[t + j];
+    if (NOISE) s_sig[j] = d.sigma[t + j];
+  }
+  __syncwarp();
   Vec<V> xstart{}, xfill{};
   if (live) {
     xstart = ldv<V>(Xb + (int64_t)(t % (P + 1)) * D + mycol);
@@ -569,24 +578,32 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
     xc0 = ldv<V>(s_rows + (size_t)(j0 - 1) * NR * SEG + SEG + lane * V);
   }
 
-  // phase 1: compensated sum of this segment's drifts
+  // phase 1: the drifts (written over the eps rows, for phase 2), the cache
+  // update of the misses (Eq. 7), and the compensated sum of the segment
   float rh[V], rl[V];
 #pragma unroll
   for (int v = 0; v < V; ++v) { rh[v] = 0.f; rl[v] = 0.f; }
   if (live) {
     Vec<V> xc = xc0;
     for (int j = j0; j < j1; ++j) {
-      const float* rowp = s_rows + (size_t)j * NR * SEG;
+      float* rowp = s_rows + (size_t)j * NR * SEG;
       const Vec<V> eps = ldv<V>(rowp + lane * V);
+      if (s_rank[j] >= 0) {  // Eq. 7: the cache takes (x_i, eps_i) of a miss
+        const int64_t o = (int64_t)s_slot[j] * D + mycol;
+        stv<V>(Eh + o, eps);
+        stv<V>(Xh + o, xc);
+      }
       const float cm1 = s_cm1[j], ec = s_ec[j];
       Vec<V> zn{};
       if (NOISE) zn = ldv<V>(rowp + 3 * SEG + lane * V);
+      Vec<V> dr;
 #pragma unroll
       for (int v = 0; v < V; ++v) {
-        float dr = fmaf(cm1, xc.a[v], ec * eps.a[v]);
-        if (NOISE) dr = fmaf(s_sig[j], zn.a[v], dr);
-        acc_add(rh[v], rl[v], dr);
+        dr.a[v] = fmaf(cm1, xc.a[v], ec * eps.a[v]);
+        if (NOISE) dr.a[v] = fmaf(s_sig[j], zn.a[v], dr.a[v]);
+        acc_add(rh[v], rl[v], dr.a[v]);
       }
+      stv<V>(rowp + lane * V, dr);
       xc = (t + j + 1 <= e) ? ldv<V>(rowp + SEG + lane * V) : xfill;
     }
   }
@@ -610,27 +627,16 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
     }
   }
   {
-    Vec<V> xc = xc0;
     for (int j = j0; j < j1; ++j) {
       const float* rowp = s_rows + (size_t)j * NR * SEG;
       float ev = 0.f, dv = 0.f;
       if (live) {
-        const Vec<V> eps = ldv<V>(rowp + lane * V);
-        if (s_rank[j] >= 0) {  // Eq. 7: the cache takes (x_i, eps_i) of a miss
-          const int64_t o = (int64_t)s_slot[j] * D + mycol;
-          stv<V>(Eh + o, eps);
-          stv<V>(Xh + o, xc);
-        }
-        const float cm1 = s_cm1[j], ec = s_ec[j];
+        const Vec<V> dr = ldv<V>(rowp + lane * V);  // the drift, from phase 1
         const Vec<V> xo = (t + j + 1 <= e) ? ldv<V>(rowp + SEG + lane * V) : xfill;
-        Vec<V> zn{};
-        if (NOISE) zn = ldv<V>(rowp + 3 * SEG + lane * V);
         Vec<V> xn;
 #pragma unroll
         for (int v = 0; v < V; ++v) {
-          float dr = fmaf(cm1, xc.a[v], ec * eps.a[v]);
-          if (NOISE) dr = fmaf(s_sig[j], zn.a[v], dr);
-          acc_add(ch[v], cl[v], dr);
+          acc_add(ch[v], cl[v], dr.a[v]);
           xn.a[v] = ch[v] + cl[v];
           const float df = xn.a[v] - xo.a[v];
           ev = fmaf(df, df, ev);
@@ -641,7 +647,6 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
 #pragma unroll
           for (int v = 0; v < V; ++v) dv += fabsf(xn.a[v] - xh.a[v]);
         }
-        xc = xo;
       }
       s_red[(size_t)j * 33 + lane] = ev;
       s_red[(size_t)(P + j) * 33 + lane] = dv;
