@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
 NCU_TRAFFIC = {
-    ("ec3eb38c7468b7b6", "sd15"): 6242688.0,
-    ("ec3eb38c7468b7b6", "batched"): 24668416.0,
-    ("ec3eb38c7468b7b6", "large"): 71628142.0,
+    ("6a9f5cdb0de0680f", "sd15"): 6247488.0,
+    ("6a9f5cdb0de0680f", "batched"): 24649984.0,
+    ("6a9f5cdb0de0680f", "large"): 71753838.0,
 }
 
 
