@@ -207,6 +207,85 @@ PA_API pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_la
 
 PA_API void pa_destroy(pa_solver* s);
 
+/* ---- Parareal (SRDS-style) sampling with the same cache ------------------
+ * Sec. 2.1 names Parareal-based samplers (SRDS: a coarse solver initialises,
+ * fine solvers refine); Sec. 2.2 applies the output cache to their network
+ * evaluations and leaves the Parareal update unchanged. The paper states no
+ * more; this library's reading: blocks of s = ceil(sqrt(T)) DDIM steps
+ * (N = ceil(T / s) blocks); coarse solver G_n = one DDIM jump across block n
+ * from eps at its start; fine solver F_n = the block's DDIM steps;
+ * iteration 0: U_{n+1} = G_n(U_n); iteration k: F_n(U_n^{k-1}) for all n, then
+ * U_{n+1}^k = G_n(U_n^k) + F_n(U_n^{k-1}) - G_n(U_n^{k-1}) in block order;
+ * converged when max_n (1/D) ||U_n^k - U_n^{k-1}||^2 <= tol (Eq. 2 on the block
+ * boundaries) or k = N (Parareal is then exact); converged trajectories freeze.
+ * One cache entry per (trajectory, sampling index), shared by coarse and fine
+ * evaluations: hit iff an entry exists and its Eq. 4 distance < cache_thresh
+ * (Eq. 5); misses are evaluated and stored (Eq. 7). Each evaluation stage (a
+ * fine step of every block, or one coarse block) is one pa_srds_step /
+ * denoise / pa_srds_submit_eps round, with the same batch_x / miss_bt
+ * conventions as pa_step (misses trajectory-major, then by block).
+ * ------------------------------------------------------------------------ */
+typedef struct pa_srds pa_srds;
+
+typedef struct {
+  int64_t iters;         /* Parareal iterations completed (0 = coarse initialisation only) */
+  int64_t nfe;           /* network evaluations (misses) */
+  int64_t hits;          /* evaluations served by the cache */
+  int64_t launches;      /* kernels this handle launched */
+  int32_t n_active;      /* trajectories not yet converged */
+  int32_t n_miss;        /* misses of the current stage */
+  int32_t device_status;
+  int32_t blocks;        /* N */
+  int32_t block_steps;   /* s */
+  int32_t reserved;
+} pa_srds_stats_t;
+
+/* Device workspace bytes (0 on bad sizes; batch <= 64, batch * N <= 2048). */
+PA_API size_t pa_srds_workspace_bytes(int T, int64_t D, int batch);
+
+/* Same conventions as pa_create (alphas_cumprod HOST [T+1], sampling order;
+ * caller-owned 256-byte aligned DEVICE workspace; stream may be NULL). */
+PA_API pa_status pa_srds_create(pa_srds** out, int T, const int64_t* latent_shape, int ndim,
+                                const double* alphas_cumprod, double tol, double cache_thresh,
+                                int batch, void* workspace_dev, size_t workspace_bytes, void* stream);
+
+/* x_init [batch][D] fp32, HOST or DEVICE; clears the cache; restarts. */
+PA_API pa_status pa_srds_init(pa_srds* h, const float* x_init);
+
+/* Plan the next evaluation stage: cache test of its rows, compaction of the
+ * misses into batch_x [n_miss][D] (library-owned, valid until the next
+ * submit), miss_bt [n_miss][2] = (trajectory, sampling index). Synchronises
+ * to read n_miss; PA_DONE once every trajectory has converged. */
+PA_API pa_status pa_srds_step(pa_srds* h, int* n_miss, const float** batch_x, const int32_t** miss_bt);
+
+/* pa_srds_step without host synchronisation: *n_miss_dev is the device
+ * address of the miss count (for device-side denoisers such as pa_gmm_eps).
+ * Stages issued after the last trajectory converged do nothing. */
+PA_API pa_status pa_srds_step_async(pa_srds* h, const float** batch_x, const int32_t** miss_bt,
+                                    const int32_t** n_miss_dev);
+
+/* Device address of the current stage's miss count (NULL for a NULL handle). */
+PA_API const int32_t* pa_srds_n_miss_dev(const pa_srds* h);
+
+/* batch_eps [n_miss][D] fp32 DEVICE for the planned misses: applies the
+ * stage (fine steps or coarse jump + correction), and after the last stage of
+ * an iteration the convergence test. */
+PA_API pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps);
+
+/* Synchronise; *n_active = trajectories still refining; PA_DONE when none. */
+PA_API pa_status pa_srds_poll(pa_srds* h, int* n_active);
+
+/* x_out [batch][D] (HOST or DEVICE) = U_N; only after PA_DONE. Synchronises. */
+PA_API pa_status pa_srds_result(pa_srds* h, float* x_out);
+
+PA_API pa_status pa_srds_stats(pa_srds* h, pa_srds_stats_t* out);
+
+/* err_out [N][batch] fp32 HOST: the block-boundary error of every iteration
+ * (rows of iterations not run are unspecified). Synchronises. */
+PA_API pa_status pa_srds_errors(pa_srds* h, float* err_out);
+
+PA_API void pa_srds_destroy(pa_srds* h);
+
 /* ---- synthetic denoiser: posterior-mean eps of an isotropic Gaussian mixture
  * (stand-in for the SD v1.5 UNet of Sec. 3.2; not part of the paper's method).
  * eps*(x) = sqrt(1-a)/v * (x - sqrt(a) * sum_k r_k mu_k),

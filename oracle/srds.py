@@ -62,7 +62,7 @@ class SrdsResult:
     iters_per_traj: List[int]
     boundaries: List[np.ndarray] = field(default_factory=list)  # U after init and each iteration, [B][N+1][D]
     errs: List[List[float]] = field(default_factory=list)       # per iteration, per trajectory (None if frozen)
-    batches: List[list] = field(default_factory=list)           # per evaluation batch: list of (b, i, hit)
+    batches: List[list] = field(default_factory=list)           # per evaluation batch: (b, i, hit, delta)
 
 
 def run_srds(alphas, x_init, eps_fn, tol, cache_thresh, use_cache=True, max_iters=None):
@@ -91,10 +91,11 @@ def run_srds(alphas, x_init, eps_fn, tol, cache_thresh, use_cache=True, max_iter
         log = []
         for r, (b, i) in enumerate(zip(bs, idx)):
             hit = False
+            delta = None
             if use_cache and has[b, i]:
                 delta = float(np.sum(np.abs(rows[r] - xhat[b, i])) / D)
                 hit = delta < cache_thresh
-            log.append((int(b), int(i), hit))
+            log.append((int(b), int(i), hit, delta))
             if hit:
                 out[r] = ehat[b, i]
             else:

@@ -38,6 +38,16 @@ class PaStats(C.Structure):
         return {k: getattr(self, k) for k, _ in self._fields_}
 
 
+class PaSrdsStats(C.Structure):
+    _fields_ = [("iters", C.c_int64), ("nfe", C.c_int64), ("hits", C.c_int64),
+                ("launches", C.c_int64), ("n_active", C.c_int32), ("n_miss", C.c_int32),
+                ("device_status", C.c_int32), ("blocks", C.c_int32), ("block_steps", C.c_int32),
+                ("reserved", C.c_int32)]
+
+    def as_dict(self):
+        return {k: getattr(self, k) for k, _ in self._fields_ if k != "reserved"}
+
+
 _lib = None
 VP = C.c_void_p
 PVP = C.POINTER(C.c_void_p)
@@ -64,6 +74,19 @@ _PROTOS = {
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
     "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.c_int]),
     "pa_destroy": (None, [VP]),
+    "pa_srds_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int64, C.c_int]),
+    "pa_srds_create": (C.c_int, [PVP, C.c_int, C.POINTER(C.c_int64), C.c_int, C.POINTER(C.c_double),
+                                 C.c_double, C.c_double, C.c_int, VP, C.c_size_t, VP]),
+    "pa_srds_init": (C.c_int, [VP, VP]),
+    "pa_srds_step": (C.c_int, [VP, C.POINTER(C.c_int), PVP, PVP]),
+    "pa_srds_step_async": (C.c_int, [VP, PVP, PVP, PVP]),
+    "pa_srds_submit_eps": (C.c_int, [VP, VP]),
+    "pa_srds_n_miss_dev": (VP, [VP]),
+    "pa_srds_poll": (C.c_int, [VP, C.POINTER(C.c_int)]),
+    "pa_srds_result": (C.c_int, [VP, VP]),
+    "pa_srds_stats": (C.c_int, [VP, C.POINTER(PaSrdsStats)]),
+    "pa_srds_errors": (C.c_int, [VP, VP]),
+    "pa_srds_destroy": (None, [VP]),
     "pa_gmm_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int64, C.c_int, C.c_int]),
     "pa_gmm_create": (C.c_int, [PVP, C.c_int, C.c_int64, VP, C.c_double,
                                 C.POINTER(C.c_double), C.c_int, C.c_int, VP, C.c_size_t, VP]),
@@ -282,3 +305,72 @@ def pa_gmm_eps_noalloc(means_ptr, K, D, std, alphas_cumprod, batch_x_ptr, miss_b
     return _check("pa_gmm_eps_noalloc", lib().pa_gmm_eps_noalloc(
         _dptr(means_ptr), int(K), int(D), float(std), alphas, len(alphas_cumprod) - 1,
         _dptr(batch_x_ptr), _dptr(miss_bt_ptr), int(n_rows), _dptr(batch_eps_ptr), _dptr(stream_ptr)))
+
+
+# ---- Parareal (SRDS-style) sampler -----------------------------------------
+
+def pa_srds_workspace_bytes(T, D, batch):
+    return int(lib().pa_srds_workspace_bytes(T, D, batch))
+
+
+def pa_srds_create(T, latent_shape, alphas_cumprod, tol, cache_thresh, batch, workspace_ptr,
+                   workspace_bytes, stream_ptr):
+    shape = (C.c_int64 * len(latent_shape))(*[int(v) for v in latent_shape])
+    alphas = (C.c_double * len(alphas_cumprod))(*[float(v) for v in alphas_cumprod])
+    h = C.c_void_p()
+    _check("pa_srds_create", lib().pa_srds_create(C.byref(h), T, shape, len(latent_shape), alphas, float(tol),
+                                                  float(cache_thresh), batch, _dptr(workspace_ptr),
+                                                  workspace_bytes, _dptr(stream_ptr)))
+    return h
+
+
+def pa_srds_init(h, x_ptr):
+    return _check("pa_srds_init", lib().pa_srds_init(h, _dptr(x_ptr)))
+
+
+def pa_srds_step(h):
+    n = C.c_int(0)
+    bx, mb = C.c_void_p(), C.c_void_p()
+    st = _check("pa_srds_step", lib().pa_srds_step(h, C.byref(n), C.byref(bx), C.byref(mb)))
+    return st, n.value, bx.value, mb.value
+
+
+def pa_srds_step_async(h):
+    bx, mb, nm = C.c_void_p(), C.c_void_p(), C.c_void_p()
+    st = _check("pa_srds_step_async", lib().pa_srds_step_async(h, C.byref(bx), C.byref(mb), C.byref(nm)))
+    return st, bx.value, mb.value, nm.value
+
+
+def pa_srds_n_miss_dev(h):
+    return lib().pa_srds_n_miss_dev(h)
+
+
+def pa_srds_submit_eps(h, eps_ptr):
+    return _check("pa_srds_submit_eps", lib().pa_srds_submit_eps(h, _dptr(eps_ptr)))
+
+
+def pa_srds_poll(h):
+    n = C.c_int(0)
+    st = _check("pa_srds_poll", lib().pa_srds_poll(h, C.byref(n)))
+    return st, n.value
+
+
+def pa_srds_result(h, out_ptr):
+    return _check("pa_srds_result", lib().pa_srds_result(h, _dptr(out_ptr)))
+
+
+def pa_srds_stats(h):
+    out = PaSrdsStats()
+    _check("pa_srds_stats", lib().pa_srds_stats(h, C.byref(out)))
+    return out.as_dict()
+
+
+def pa_srds_errors(h, n_blocks, batch):
+    import numpy as _np
+    buf = _np.zeros((n_blocks, batch), dtype=_np.float32)
+    _check("pa_srds_errors", lib().pa_srds_errors(h, buf.ctypes.data_as(C.c_void_p)))
+    return buf
+
+
+def pa_srds_destroy(h):
+    lib().pa_srds_destroy(h)

@@ -1,0 +1,649 @@
+// Parareal (SRDS-style) DDIM sampling with ParaAnya's output cache on every
+// network evaluation (Sec. 2.1: Parareal-based samplers; Sec. 2.2: the cache
+// applies to the coarse and fine evaluations, the Parareal update unchanged).
+//
+// Blocks of s = ceil(sqrt(T)) sampling steps, N = ceil(T / s) blocks; block n
+// covers indices [n s, e_n), e_n = min((n + 1) s, T). Fine solver F_n: the
+// DDIM steps of block n. Coarse solver G_n: one DDIM jump from alpha-bar(n s)
+// to alpha-bar(e_n) with eps at (u, n s).
+//   iteration 0   U_0 = x_init, U_{n+1} = G_n(U_n)                 (coarse stages)
+//   iteration k   F_n(U_n^{k-1}) for all n                         (s fine stages)
+//                 U_{n+1}^k = G_n(U_n^k) + F_n(U_n^{k-1}) - G_n(U_n^{k-1})  (N coarse stages)
+//                 err = max_n (1/D) ||U_n^k - U_n^{k-1}||^2 <= tol => converged (Eq. 2 on the
+//                 block boundaries); a converged trajectory is frozen; Parareal is exact at k = N.
+// Every evaluation stage: cache distance of each live row against its index's
+// entry (Eq. 4), hit iff entry && delta < tau_cache (Eq. 5), misses compacted
+// trajectory-major (k_srds_plan) and gathered for the denoiser; then the step
+// (k_srds_apply) takes eps from the batch (miss, updating the entry, Eq. 7) or
+// from the cache (hit, Eq. 6).
+//
+// Data (rows of D): U, Up [B][N+1][D] fp64 boundaries now and before this
+// iteration; Y [B][N][D] fp64 fine states (F after the sweep); G [B][N][D]
+// fp64 coarse results; Xh [B][T][D] fp64 and Eh [B][T][D] fp32 the cache;
+// batch_x [B*N][D] fp32. The trajectory states are fp64: a sample passes
+// through about T steps plus N corrections, one rounding each, and fp32
+// states drift by ~1e-5 of the latent scale over T = 100 (measured); the
+// denoiser still sees fp32 rows and returns fp32 eps.
+#include <cmath>
+#include <string>
+#include <vector>
+
+#include "../../include/paraanya.h"
+#include "pa_internal.h"
+
+namespace pa {
+void set_error(const std::string& msg);  // pa_solver.cpp
+}
+
+namespace {
+
+constexpr int kSThreads = 256;
+constexpr int kSStrip = 4096;        // columns per distance / error CTA
+constexpr int kSMaxRows = 2048;      // B * N
+constexpr int kSPlanPer = kSMaxRows / kSThreads;
+
+enum StageKind : int32_t { kCoarseInit = 0, kFine = 1, kCoarse = 2 };
+
+struct SCtl {
+  int32_t n_miss, n_active, iter, status;
+  long long nfe, hits;
+};
+
+struct SDev {
+  int T, B, N, s, nstrip;
+  int64_t D;
+  double* U;
+  double* Up;
+  double* Y;
+  double* G;
+  double* Xh;
+  float* Eh;
+  int32_t* has;      // [B][T]
+  float* batch_x;    // [B*N][D]
+  int32_t* miss_bt;  // [B*N][2]
+  int32_t* rank;     // [B*N]: miss rank, -1 hit, -2 not live
+  double* part;      // [B*N][nstrip]
+  int32_t* active;   // [B]
+  int32_t* iters;    // [B]
+  float* err_log;    // [N][B]
+  const double* cm1;  // [T] single steps: c_i - 1
+  const double* e1;   // [T]
+  const double* cjm1; // [N] block jumps: c - 1
+  const double* ej;   // [N]
+  SCtl* ctl;
+  double tol, cache_thresh;
+};
+
+struct Stage {
+  int32_t kind, j, n, iter;  // fine: j; coarse: n
+};
+
+__device__ __forceinline__ int stage_rows(const SDev& d, const Stage& st) {
+  return st.kind == kFine ? d.B * d.N : d.B;
+}
+
+// Row r of a stage: trajectory b, sampling index i, its input row; false if
+// the row takes no part (frozen trajectory, or past the end of a short block).
+__device__ __forceinline__ bool row_info(const SDev& d, const Stage& st, int r, int& b, int& n, int& i,
+                                         double*& x) {
+  if (st.kind == kFine) {
+    b = r / d.N;
+    n = r % d.N;
+    i = n * d.s + st.j;
+    const int end = min((n + 1) * d.s, d.T);
+    x = d.Y + ((int64_t)b * d.N + n) * d.D;
+    return d.active[b] && i < end;
+  }
+  b = r;
+  n = st.n;
+  i = n * d.s;
+  x = d.U + ((int64_t)b * (d.N + 1) + n) * d.D;
+  return d.active[b] != 0;
+}
+
+__device__ __forceinline__ double block_sum(double v, double* s_w) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  if (lane == 0) s_w[warp] = v;
+  __syncthreads();
+  double t = 0.0;
+  if (threadIdx.x == 0)
+    for (int w = 0; w < kSThreads / 32; ++w) t += s_w[w];  // fixed order
+  return t;
+}
+
+// Eq. 4 partial sums: sum |x - xhat_i| over one strip of one row with an entry.
+__global__ void __launch_bounds__(kSThreads) k_srds_dist(SDev d, Stage st) {
+  __shared__ double s_w[kSThreads / 32];
+  const int r = blockIdx.y;
+  int b, n, i;
+  double* x;
+  if (!row_info(d, st, r, b, n, i, x) || !d.has[(int64_t)b * d.T + i]) return;
+  const double* xh = d.Xh + ((int64_t)b * d.T + i) * d.D;
+  const int64_t c0 = (int64_t)blockIdx.x * kSStrip;
+  const int64_t c1 = (c0 + kSStrip < d.D) ? c0 + kSStrip : d.D;
+  double acc = 0.0;
+  for (int64_t c = c0 + threadIdx.x; c < c1; c += kSThreads) acc += fabs(x[c] - xh[c]);
+  const double t = block_sum(acc, s_w);
+  if (threadIdx.x == 0) d.part[(int64_t)r * d.nstrip + blockIdx.x] = t;
+}
+
+// Hit/miss of every live row (Eq. 5, first entry = miss) and the compaction of
+// the misses in row order (trajectory-major), one CTA.
+__global__ void __launch_bounds__(kSThreads) k_srds_plan(SDev d, Stage st) {
+  __shared__ int s_warp[kSThreads / 32];
+  __shared__ int s_total, s_hits;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int rows = stage_rows(d, st);
+  if (tid == 0) s_hits = 0;
+  __syncthreads();
+  int flag[kSPlanPer];  // 1 miss, 0 hit, -1 not live
+  int cnt = 0, hits = 0;
+  const int q0 = tid * kSPlanPer;
+#pragma unroll
+  for (int u = 0; u < kSPlanPer; ++u) {
+    const int r = q0 + u;
+    flag[u] = -1;
+    if (r >= rows) continue;
+    int b, n, i;
+    double* x;
+    if (!row_info(d, st, r, b, n, i, x)) continue;
+    bool hit = false;
+    if (d.has[(int64_t)b * d.T + i]) {
+      double sum = 0.0;
+      for (int k = 0; k < d.nstrip; ++k) sum += d.part[(int64_t)r * d.nstrip + k];
+      hit = sum / (double)d.D < d.cache_thresh;
+    }
+    flag[u] = hit ? 0 : 1;
+    cnt += hit ? 0 : 1;
+    hits += hit ? 1 : 0;
+  }
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  if (lane == 31) s_warp[warp] = incl;
+  atomicAdd(&s_hits, hits);
+  __syncthreads();
+  if (warp == 0) {
+    const int w = lane < kSThreads / 32 ? s_warp[lane] : 0;
+    int wi = w;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, wi, o);
+      if (lane >= o) wi += v;
+    }
+    if (lane < kSThreads / 32) s_warp[lane] = wi - w;
+    if (lane == 31) s_total = wi;
+  }
+  __syncthreads();
+  int m = s_warp[warp] + incl - cnt;
+#pragma unroll
+  for (int u = 0; u < kSPlanPer; ++u) {
+    const int r = q0 + u;
+    if (r >= rows) continue;
+    if (flag[u] == 1) {
+      int b, n, i;
+      double* x;
+      row_info(d, st, r, b, n, i, x);
+      d.rank[r] = m;
+      d.miss_bt[2 * m] = b;
+      d.miss_bt[2 * m + 1] = i;
+      ++m;
+    } else {
+      d.rank[r] = flag[u] == 0 ? -1 : -2;
+    }
+  }
+  if (tid == 0) {
+    d.ctl->n_miss = s_total;
+    d.ctl->nfe += s_total;
+    d.ctl->hits += s_hits;
+  }
+}
+
+// batch_x[m] <- the input row of miss m.
+__global__ void __launch_bounds__(kSThreads) k_srds_gather(SDev d, Stage st) {
+  const int n_miss = d.ctl->n_miss;
+  for (int m = blockIdx.y; m < n_miss; m += gridDim.y) {
+    const int b = d.miss_bt[2 * m], i = d.miss_bt[2 * m + 1];
+    const int n = i / d.s;
+    const double* x = st.kind == kFine ? d.Y + ((int64_t)b * d.N + n) * d.D
+                                       : d.U + ((int64_t)b * (d.N + 1) + n) * d.D;
+    float* to = d.batch_x + (int64_t)m * d.D;
+    for (int64_t c = (int64_t)blockIdx.x * kSThreads + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * kSThreads)
+      to[c] = (float)x[c];
+  }
+}
+
+// The step of every live row: eps from the batch (miss: the entry becomes
+// (x, eps), Eq. 7) or the cache (hit, Eq. 6); then a fine step
+// Y <- Y + (c_i - 1) Y + e_i eps, or a coarse jump g = x + (c - 1) x + e eps
+// with U_{n+1} = g (iteration 0) or g + F_n - G_n (later), G_n <- g.
+__global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, const float* __restrict__ beps) {
+  const int r = blockIdx.y;
+  int b, n, i;
+  double* x;
+  if (!row_info(d, st, r, b, n, i, x)) return;
+  const int rk = d.rank[r];
+  const int64_t e_off = ((int64_t)b * d.T + i) * d.D;
+  const float* eps = rk >= 0 ? beps + (int64_t)rk * d.D : d.Eh + e_off;
+  if (rk >= 0 && blockIdx.x == 0 && threadIdx.x == 0) d.has[(int64_t)b * d.T + i] = 1;
+  const double cm1 = st.kind == kFine ? d.cm1[i] : d.cjm1[n];
+  const double ec = st.kind == kFine ? d.e1[i] : d.ej[n];
+  double* Un1 = d.U + ((int64_t)b * (d.N + 1) + n + 1) * d.D;
+  double* Gn = d.G + ((int64_t)b * d.N + n) * d.D;
+  const double* Fn = d.Y + ((int64_t)b * d.N + n) * d.D;
+  for (int64_t c = (int64_t)blockIdx.x * kSThreads + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * kSThreads) {
+    const double xv = x[c];
+    const float ev = eps[c];
+    if (rk >= 0) {
+      d.Xh[e_off + c] = xv;
+      d.Eh[e_off + c] = ev;
+    }
+    const double g = xv + fma(cm1, xv, ec * (double)ev);
+    if (st.kind == kFine) {
+      x[c] = g;
+    } else if (st.kind == kCoarseInit) {
+      Gn[c] = g;
+      Un1[c] = g;
+    } else {
+      Un1[c] = g + (Fn[c] - Gn[c]);
+      Gn[c] = g;
+    }
+  }
+}
+
+// End of an iteration: partial sums of (U_{n+1} - Up_{n+1})^2 per strip
+// (iterations >= 1), then Up <- U and Y_n <- U_n for the next fine sweep.
+__global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter) {
+  __shared__ double s_w[kSThreads / 32];
+  const int r = blockIdx.y, b = r / d.N, n = r % d.N;
+  if (!d.active[b]) return;
+  const int64_t c0 = (int64_t)blockIdx.x * kSStrip;
+  const int64_t c1 = (c0 + kSStrip < d.D) ? c0 + kSStrip : d.D;
+  double* u1 = d.U + ((int64_t)b * (d.N + 1) + n + 1) * d.D;
+  double* p1 = d.Up + ((int64_t)b * (d.N + 1) + n + 1) * d.D;
+  const double* u0 = d.U + ((int64_t)b * (d.N + 1) + n) * d.D;
+  double* y = d.Y + ((int64_t)b * d.N + n) * d.D;
+  double acc = 0.0;
+  for (int64_t c = c0 + threadIdx.x; c < c1; c += kSThreads) {
+    const double df = u1[c] - p1[c];
+    acc = fma(df, df, acc);
+    p1[c] = u1[c];
+    y[c] = u0[c];
+  }
+  const double t = block_sum(acc, s_w);
+  if (threadIdx.x == 0) d.part[(int64_t)r * d.nstrip + blockIdx.x] = iter > 0 ? t : 0.0;
+}
+
+// Convergence of every trajectory after iteration `iter` (one CTA).
+__global__ void __launch_bounds__(kSThreads) k_srds_finish(SDev d, int iter) {
+  __shared__ int s_act;
+  if (threadIdx.x == 0) s_act = 0;
+  __syncthreads();
+  for (int b = threadIdx.x; b < d.B; b += kSThreads) {
+    if (!d.active[b]) continue;
+    if (iter > 0) {
+      double err = 0.0;
+      for (int n = 0; n < d.N; ++n) {
+        double sum = 0.0;
+        const int r = b * d.N + n;
+        for (int k = 0; k < d.nstrip; ++k) sum += d.part[(int64_t)r * d.nstrip + k];
+        err = fmax(err, sum / (double)d.D);
+      }
+      d.iters[b] = iter;
+      d.err_log[(int64_t)(iter - 1) * d.B + b] = (float)err;
+      if (err <= d.tol || iter >= d.N) {
+        d.active[b] = 0;
+        continue;
+      }
+    }
+    atomicAdd(&s_act, 1);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    d.ctl->n_active = s_act;
+    d.ctl->iter = iter;
+  }
+}
+
+// fp32 rows (pitch D) -> fp64 rows of the boundary array (pitch (N+1) D), and back.
+__global__ void k_srds_load(SDev d, const float* __restrict__ src, int slot) {
+  const int b = blockIdx.y;
+  double* to = d.U + ((int64_t)b * (d.N + 1) + slot) * d.D;
+  double* to2 = d.Up + ((int64_t)b * (d.N + 1) + slot) * d.D;
+  for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * blockDim.x) {
+    to[c] = (double)src[(int64_t)b * d.D + c];
+    to2[c] = to[c];
+  }
+}
+
+__global__ void k_srds_store(SDev d, float* __restrict__ dst, int slot) {
+  const int b = blockIdx.y;
+  const double* from = d.U + ((int64_t)b * (d.N + 1) + slot) * d.D;
+  for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * blockDim.x)
+    dst[(int64_t)b * d.D + c] = (float)from[c];
+}
+
+__global__ void k_srds_reset(SDev d) {
+  for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
+    d.active[b] = 1;
+    d.iters[b] = 0;
+  }
+  for (int64_t q = threadIdx.x; q < (int64_t)d.B * d.T; q += blockDim.x) d.has[q] = 0;
+  if (threadIdx.x == 0) {
+    SCtl c{};
+    c.n_active = d.B;
+    *d.ctl = c;
+  }
+}
+
+struct SLayout {
+  size_t U, Up, Y, G, Xh, Eh, has, batch_x, miss_bt, rank, part, active, iters, err_log, coef, ctl, total;
+};
+
+SLayout s_layout(int T, int64_t D, int B, int N, int nstrip) {
+  SLayout L{};
+  size_t o = 0;
+  auto take = [&](size_t bytes) { size_t at = o; o = pa::align_up(o + bytes, pa::kAlign); return at; };
+  const size_t row = (size_t)D * sizeof(float), row64 = (size_t)D * sizeof(double);
+  L.U = take((size_t)B * (N + 1) * row64);
+  L.Up = take((size_t)B * (N + 1) * row64);
+  L.Y = take((size_t)B * N * row64);
+  L.G = take((size_t)B * N * row64);
+  L.Xh = take((size_t)B * T * row64);
+  L.Eh = take((size_t)B * T * row);
+  L.has = take((size_t)B * T * sizeof(int32_t));
+  L.batch_x = take((size_t)B * N * row);
+  L.miss_bt = take((size_t)B * N * 2 * sizeof(int32_t));
+  L.rank = take((size_t)B * N * sizeof(int32_t));
+  L.part = take((size_t)B * N * nstrip * sizeof(double));
+  L.active = take((size_t)B * sizeof(int32_t));
+  L.iters = take((size_t)B * sizeof(int32_t));
+  L.err_log = take((size_t)N * B * sizeof(float));
+  L.coef = take((size_t)(2 * T + 2 * N) * sizeof(double));
+  L.ctl = take(sizeof(SCtl));
+  L.total = o;
+  return L;
+}
+
+void s_blocks(int T, int* s, int* N) {
+  int v = 1;
+  while (v * v < T) ++v;
+  *s = v;
+  *N = (T + v - 1) / v;
+}
+
+}  // namespace
+
+struct pa_srds {
+  SDev d;
+  SLayout L;
+  char* ws;
+  cudaStream_t st;
+  int phase;      // -1 created, 0 ready for a step, 1 stepped (waiting for eps), 2 done
+  int iter;       // current iteration (0 = coarse initialisation)
+  int stage;      // index within the iteration: fine stages first (iter >= 1), then coarse
+  int64_t launches;
+  SCtl* host_ctl;
+};
+
+namespace {
+
+pa_status s_fail(const std::string& m, pa_status code) {
+  pa::set_error(m);
+  return code;
+}
+
+Stage current_stage(const pa_srds* h) {
+  Stage st{};
+  st.iter = h->iter;
+  const int nfine = h->iter == 0 ? 0 : h->d.s;
+  if (h->stage < nfine) {
+    st.kind = kFine;
+    st.j = h->stage;
+  } else {
+    st.kind = h->iter == 0 ? kCoarseInit : kCoarse;
+    st.n = h->stage - nfine;
+  }
+  return st;
+}
+
+cudaError_t s_sync_ctl(pa_srds* h) {
+  cudaError_t e = cudaMemcpyAsync(h->host_ctl, h->d.ctl, sizeof(SCtl), cudaMemcpyDeviceToHost, h->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+  return e;
+}
+
+}  // namespace
+
+extern "C" size_t pa_srds_workspace_bytes(int T, int64_t D, int batch) {
+  if (T < 1 || T > 100000 || D < 1 || batch < 1 || batch > pa::kMaxBatch) return 0;
+  int s, N;
+  s_blocks(T, &s, &N);
+  if ((int64_t)batch * N > kSMaxRows) return 0;
+  return s_layout(T, D, batch, N, (int)((D + kSStrip - 1) / kSStrip)).total;
+}
+
+extern "C" pa_status pa_srds_create(pa_srds** out, int T, const int64_t* latent_shape, int ndim,
+                                    const double* alphas_cumprod, double tol, double cache_thresh, int batch,
+                                    void* workspace_dev, size_t workspace_bytes, void* stream) {
+  if (!out) return s_fail("pa_srds_create: out is NULL", PA_ERR_ARG);
+  *out = nullptr;
+  if (T < 1 || T > 100000 || !latent_shape || ndim < 1 || ndim > 8 || !alphas_cumprod || batch < 1 ||
+      batch > pa::kMaxBatch || !(tol >= 0.0) || !(cache_thresh >= 0.0))
+    return s_fail("pa_srds_create: bad size, pointer or threshold", PA_ERR_ARG);
+  int64_t D = 1;
+  for (int k = 0; k < ndim; ++k) {
+    if (latent_shape[k] < 1) return s_fail("pa_srds_create: latent_shape entries must be >= 1", PA_ERR_ARG);
+    D *= latent_shape[k];
+  }
+  for (int i = 0; i <= T; ++i) {
+    const double a = alphas_cumprod[i];
+    if (!(a > 0.0 && a <= 1.0)) return s_fail("pa_srds_create: alphas_cumprod must be in (0, 1]", PA_ERR_ARG);
+  }
+  int s, N;
+  s_blocks(T, &s, &N);
+  if ((int64_t)batch * N > kSMaxRows) return s_fail("pa_srds_create: batch * blocks exceeds 2048", PA_ERR_ARG);
+  const int nstrip = (int)((D + kSStrip - 1) / kSStrip);
+  const SLayout L = s_layout(T, D, batch, N, nstrip);
+  if (!workspace_dev || (reinterpret_cast<uintptr_t>(workspace_dev) % pa::kAlign) != 0 || workspace_bytes < L.total)
+    return s_fail("pa_srds_create: workspace NULL, not 256-byte aligned, or smaller than pa_srds_workspace_bytes()",
+                  PA_ERR_WORKSPACE);
+  pa_srds* h = new pa_srds{};
+  h->L = L;
+  h->ws = static_cast<char*>(workspace_dev);
+  h->st = static_cast<cudaStream_t>(stream);
+  h->phase = -1;
+  char* w = h->ws;
+  SDev& d = h->d;
+  d.T = T; d.B = batch; d.N = N; d.s = s; d.nstrip = nstrip; d.D = D;
+  d.U = reinterpret_cast<double*>(w + L.U);
+  d.Up = reinterpret_cast<double*>(w + L.Up);
+  d.Y = reinterpret_cast<double*>(w + L.Y);
+  d.G = reinterpret_cast<double*>(w + L.G);
+  d.Xh = reinterpret_cast<double*>(w + L.Xh);
+  d.Eh = reinterpret_cast<float*>(w + L.Eh);
+  d.has = reinterpret_cast<int32_t*>(w + L.has);
+  d.batch_x = reinterpret_cast<float*>(w + L.batch_x);
+  d.miss_bt = reinterpret_cast<int32_t*>(w + L.miss_bt);
+  d.rank = reinterpret_cast<int32_t*>(w + L.rank);
+  d.part = reinterpret_cast<double*>(w + L.part);
+  d.active = reinterpret_cast<int32_t*>(w + L.active);
+  d.iters = reinterpret_cast<int32_t*>(w + L.iters);
+  d.err_log = reinterpret_cast<float*>(w + L.err_log);
+  double* coef = reinterpret_cast<double*>(w + L.coef);
+  d.cm1 = coef;
+  d.e1 = coef + T;
+  d.cjm1 = coef + 2 * T;
+  d.ej = coef + 2 * T + N;
+  d.ctl = reinterpret_cast<SCtl*>(w + L.ctl);
+  d.tol = tol;
+  d.cache_thresh = cache_thresh;
+  // DDIM (eta = 0) jump from a to a2: x + (c - 1) x + e eps with c = sqrt(a2 / a),
+  // e = sqrt(1 - a2) - sqrt(a2 (1 - a) / a); c - 1 formed without cancellation.
+  auto jump = [](double a, double a2, double* cm1, double* e) {
+    const double r = a2 / a, c = std::sqrt(r);
+    *cm1 = (r - 1.0) / (c + 1.0);
+    *e = std::sqrt(1.0 - a2) - std::sqrt(a2) * std::sqrt(1.0 - a) / std::sqrt(a);
+  };
+  std::vector<double> hc(2 * (size_t)T + 2 * (size_t)N);
+  for (int i = 0; i < T; ++i) jump(alphas_cumprod[i], alphas_cumprod[i + 1], &hc[i], &hc[T + i]);
+  for (int n = 0; n < N; ++n) {
+    const int a0 = n * s, a1 = (n + 1) * s < T ? (n + 1) * s : T;
+    jump(alphas_cumprod[a0], alphas_cumprod[a1], &hc[2 * T + n], &hc[2 * T + N + n]);
+  }
+  cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&h->host_ctl), sizeof(SCtl), cudaHostAllocDefault);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(coef, hc.data(), hc.size() * sizeof(double), cudaMemcpyHostToDevice, h->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(d.ctl, 0, sizeof(SCtl), h->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+  if (e != cudaSuccess) {
+    if (h->host_ctl) cudaFreeHost(h->host_ctl);
+    delete h;
+    return s_fail(std::string("pa_srds_create: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  }
+  *out = h;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_init(pa_srds* h, const float* x_init) {
+  if (!h || !x_init) return s_fail("pa_srds_init: NULL argument", PA_ERR_ARG);
+  const SDev& d = h->d;
+  // x_init (host or device) is staged in batch_x, then widened into U_0 and Up_0
+  cudaError_t e = cudaMemcpyAsync(d.batch_x, x_init, (size_t)d.B * d.D * sizeof(float), cudaMemcpyDefault, h->st);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_init: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  k_srds_load<<<dim3(32, d.B), 256, 0, h->st>>>(d, d.batch_x, 0);
+  k_srds_reset<<<1, 256, 0, h->st>>>(d);
+  h->launches += 2;
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_init: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  h->iter = 0;
+  h->stage = 0;
+  h->phase = 0;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_step_async(pa_srds* h, const float** batch_x, const int32_t** miss_bt,
+                                        const int32_t** n_miss_dev) {
+  if (!h) return s_fail("pa_srds_step_async: NULL handle", PA_ERR_ARG);
+  if (h->phase == 2) return PA_DONE;
+  if (h->phase != 0) return s_fail("pa_srds_step_async: call order (pa_srds_init, then step / submit)", PA_ERR_STATE);
+  const SDev& d = h->d;
+  const Stage st = current_stage(h);
+  const int rows = st.kind == kFine ? d.B * d.N : d.B;
+  k_srds_dist<<<dim3(d.nstrip, rows), kSThreads, 0, h->st>>>(d, st);
+  k_srds_plan<<<1, kSThreads, 0, h->st>>>(d, st);
+  const int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
+  k_srds_gather<<<dim3(gx < 32 ? gx : 32, rows), kSThreads, 0, h->st>>>(d, st);
+  h->launches += 3;
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_step_async: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  if (batch_x) *batch_x = d.batch_x;
+  if (miss_bt) *miss_bt = d.miss_bt;
+  if (n_miss_dev) *n_miss_dev = &d.ctl->n_miss;
+  h->phase = 1;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_step(pa_srds* h, int* n_miss, const float** batch_x, const int32_t** miss_bt) {
+  if (!h || !n_miss) return s_fail("pa_srds_step: NULL argument", PA_ERR_ARG);
+  if (h->phase == 2) return PA_DONE;
+  if (h->phase == 0 && h->stage == 0 && h->iter > 0) {  // a new iteration: anything left to refine?
+    cudaError_t e = s_sync_ctl(h);
+    if (e != cudaSuccess) return s_fail(std::string("pa_srds_step: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+    if (h->host_ctl->status != 0) return s_fail("pa_srds_step: device-side failure", PA_ERR_DEVICE);
+    if (h->host_ctl->n_active == 0) {
+      h->phase = 2;
+      return PA_DONE;
+    }
+  }
+  pa_status r = pa_srds_step_async(h, batch_x, miss_bt, nullptr);
+  if (r != PA_OK) return r;
+  const cudaError_t e = s_sync_ctl(h);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_step: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  *n_miss = h->host_ctl->n_miss;
+  return PA_OK;
+}
+
+extern "C" const int32_t* pa_srds_n_miss_dev(const pa_srds* h) { return h ? &h->d.ctl->n_miss : nullptr; }
+
+extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
+  if (!h || !batch_eps) return s_fail("pa_srds_submit_eps: NULL argument", PA_ERR_ARG);
+  if (h->phase != 1) return s_fail("pa_srds_submit_eps: no step to complete", PA_ERR_STATE);
+  const SDev& d = h->d;
+  const Stage st = current_stage(h);
+  const int rows = st.kind == kFine ? d.B * d.N : d.B;
+  const int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
+  k_srds_apply<<<dim3(gx < 32 ? gx : 32, rows), kSThreads, 0, h->st>>>(d, st, batch_eps);
+  h->launches++;
+  const int nstages = (h->iter == 0 ? 0 : d.s) + d.N;
+  if (++h->stage == nstages) {  // the iteration is complete
+    k_srds_err<<<dim3(d.nstrip, d.B * d.N), kSThreads, 0, h->st>>>(d, h->iter);
+    k_srds_finish<<<1, kSThreads, 0, h->st>>>(d, h->iter);
+    h->launches += 2;
+    h->stage = 0;
+    h->iter++;
+  }
+  const cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_submit_eps: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  h->phase = (h->iter > d.N) ? 2 : 0;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_poll(pa_srds* h, int* n_active) {
+  if (!h) return s_fail("pa_srds_poll: NULL handle", PA_ERR_ARG);
+  const cudaError_t e = s_sync_ctl(h);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_poll: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  const int act = h->host_ctl->n_active;
+  if (n_active) *n_active = act;
+  if (act == 0 && h->phase == 0) h->phase = 2;
+  return act == 0 ? PA_DONE : PA_OK;
+}
+
+extern "C" pa_status pa_srds_result(pa_srds* h, float* x_out) {
+  if (!h || !x_out) return s_fail("pa_srds_result: NULL argument", PA_ERR_ARG);
+  if (h->phase != 2) return s_fail("pa_srds_result: not finished", PA_ERR_STATE);
+  const SDev& d = h->d;
+  // U_N narrowed to fp32 in batch_x (free once sampling is done), then copied out
+  k_srds_store<<<dim3(32, d.B), 256, 0, h->st>>>(d, d.batch_x, d.N);
+  h->launches++;
+  cudaError_t e = cudaGetLastError();
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(x_out, d.batch_x, (size_t)d.B * d.D * sizeof(float), cudaMemcpyDefault, h->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_result: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_stats(pa_srds* h, pa_srds_stats_t* out) {
+  if (!h || !out) return s_fail("pa_srds_stats: NULL argument", PA_ERR_ARG);
+  const cudaError_t e = s_sync_ctl(h);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_stats: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  out->iters = h->host_ctl->iter;
+  out->nfe = h->host_ctl->nfe;
+  out->hits = h->host_ctl->hits;
+  out->launches = h->launches;
+  out->n_active = h->host_ctl->n_active;
+  out->n_miss = h->host_ctl->n_miss;
+  out->device_status = h->host_ctl->status;
+  out->blocks = h->d.N;
+  out->block_steps = h->d.s;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_errors(pa_srds* h, float* err_out) {
+  if (!h || !err_out) return s_fail("pa_srds_errors: NULL argument", PA_ERR_ARG);
+  const cudaError_t e = cudaMemcpy(err_out, h->d.err_log, (size_t)h->d.N * h->d.B * sizeof(float),
+                                   cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_errors: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  return PA_OK;
+}
+
+extern "C" void pa_srds_destroy(pa_srds* h) {
+  if (!h) return;
+  if (h->host_ctl) cudaFreeHost(h->host_ctl);
+  delete h;
+}

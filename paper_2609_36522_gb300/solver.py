@@ -174,3 +174,83 @@ class GmmDenoiser:
             self.close()
         except Exception:
             pass
+
+
+class SrdsSolver:
+    """Cached Parareal (SRDS-style) DDIM sampler through the C ABI; the same
+    denoiser interface as Solver (batch_x, miss_bt, device miss count)."""
+
+    def __init__(self, T, latent_shape, alphas_cumprod, tol, cache_thresh, batch=1, stream=None):
+        self.T, self.batch = int(T), int(batch)
+        self.latent_shape = tuple(int(v) for v in latent_shape)
+        self.D = int(np.prod(self.latent_shape))
+        self.stream_ptr, self.stream = _stream_ptr(stream)
+        nbytes = abi.pa_srds_workspace_bytes(self.T, self.D, self.batch)
+        if nbytes == 0:
+            raise ValueError("unsupported sizes for the Parareal sampler")
+        dev = torch.device("cuda", torch.cuda.current_device())
+        self.workspace = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+        self.h = abi.pa_srds_create(self.T, self.latent_shape, list(alphas_cumprod), tol, cache_thresh,
+                                    self.batch, self.workspace.data_ptr(), nbytes, self.stream_ptr)
+        st = abi.pa_srds_stats(self.h)
+        self.blocks, self.block_steps = st["blocks"], st["block_steps"]
+        self.max_rows = self.batch * self.blocks
+
+    def init(self, x_init):
+        x = x_init if isinstance(x_init, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(x_init))
+        if x.dtype != torch.float32 or not x.is_contiguous() or x.numel() != self.batch * self.D:
+            raise ValueError("x_init must be a contiguous float32 [batch][D] tensor")
+        self._x_init_keepalive = x
+        abi.pa_srds_init(self.h, x.data_ptr())
+
+    def _view(self, ptr, dtype, shape):
+        off = int(ptr) - self.workspace.data_ptr()
+        nb = int(np.prod(shape)) * torch.tensor([], dtype=dtype).element_size()
+        return self.workspace[off: off + nb].view(dtype).view(*shape)
+
+    def step(self):
+        """-> None when done, else a Plan of the next evaluation stage."""
+        st, n, bx, mb = abi.pa_srds_step(self.h)
+        if st == abi.PA_DONE:
+            return None
+        return Plan(n, self._view(bx, torch.float32, (n, self.D)), self._view(mb, torch.int32, (n, 2)), bx, mb)
+
+    def n_miss_dev(self):
+        return abi.pa_srds_n_miss_dev(self.h)
+
+    def step_async(self):
+        """-> None when done, else (batch_x_ptr, miss_bt_ptr, n_miss_dev_ptr)."""
+        st, bx, mb, nm = abi.pa_srds_step_async(self.h)
+        if st == abi.PA_DONE:
+            return None
+        return bx, mb, nm
+
+    def submit_eps(self, eps):
+        abi.pa_srds_submit_eps(self.h, eps.data_ptr() if isinstance(eps, torch.Tensor) else eps)
+
+    def poll(self):
+        st, n = abi.pa_srds_poll(self.h)
+        return n
+
+    def result(self, out=None):
+        if out is None:
+            out = torch.empty(self.batch, self.D, dtype=torch.float32, device=self.workspace.device)
+        abi.pa_srds_result(self.h, out.data_ptr())
+        return out
+
+    def stats(self):
+        return abi.pa_srds_stats(self.h)
+
+    def errors(self):
+        return abi.pa_srds_errors(self.h, self.blocks, self.batch)
+
+    def close(self):
+        if getattr(self, "h", None) is not None:
+            abi.pa_srds_destroy(self.h)
+            self.h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -1,0 +1,105 @@
+"""Parity of the CUDA Parareal (SRDS-style) sampler with the fp64 oracle:
+the per-stage miss lists, NFE, hits and iteration count exactly, final latents
+within 1e-5 (max-abs relative)."""
+import numpy as np
+import pytest
+
+import workload as W
+from oracle.gmm import make_eps_fn
+from oracle.ddim import serial_ddim
+from oracle.srds import run_srds
+
+pytestmark = pytest.mark.gpu
+
+
+def oracle_srds(w, tol=None, thresh=None):
+    a, x0, mu = W.inputs(w)
+    return run_srds(a, x0, make_eps_fn(a, mu, w.gmm_std), w.tol if tol is None else tol,
+                    w.cache_thresh if thresh is None else thresh)
+
+
+def gpu_srds(w, tol=None, thresh=None, mode="sync"):
+    import torch
+    from paper_2609_36522_gb300.solver import SrdsSolver, GmmDenoiser
+    a, x0, mu = W.inputs(w)
+    dev = torch.device("cuda")
+    s = SrdsSolver(w.T, w.latent_shape, a, w.tol if tol is None else tol,
+                   w.cache_thresh if thresh is None else thresh, batch=w.batch)
+    g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, s.max_rows)
+    eps = torch.empty(s.max_rows, w.D, dtype=torch.float32, device=dev)
+    s.init(torch.from_numpy(x0).to(dev))
+    stages = []
+    if mode == "sync":
+        while True:
+            out = s.step()
+            if out is None:
+                break
+            stages.append([tuple(int(v) for v in row) for row in out.miss_bt.cpu().numpy()])
+            g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+            s.submit_eps(eps)
+    else:
+        while True:
+            out = s.step_async()
+            if out is None:
+                break
+            bx, mb, nm = out
+            g.eps(bx, mb, nm, eps)
+            s.submit_eps(eps)
+    s.poll()
+    res = dict(x_final=s.result().cpu().numpy(), stats=s.stats(), stages=stages)
+    s.close()
+    g.close()
+    return res
+
+
+def compare_srds(w, orc, gpu):
+    misses = [[(b, i) for (b, i, hit, _) in batch if not hit] for batch in orc.batches]
+    assert gpu["stages"] == misses
+    st = gpu["stats"]
+    assert st["iters"] == orc.iters
+    assert st["nfe"] == orc.nfe and st["hits"] == orc.hits
+    scale = np.abs(orc.x_final).max(axis=1)
+    rel = np.abs(gpu["x_final"] - orc.x_final).max(axis=1) / scale
+    assert rel.max() <= 1e-5, rel
+    return rel
+
+
+def margins(orc, tol, thresh):
+    md = min((abs(dl - thresh) / max(thresh, 1e-30) for batch in orc.batches
+              for (_, _, _, dl) in batch if dl is not None), default=np.inf)
+    me = min((abs(e - tol) / max(tol, 1e-30) for errs in orc.errs for e in errs if e is not None),
+             default=np.inf)
+    return md, me
+
+
+@pytest.mark.parametrize("wname", ["srds", "srds_batched"])
+def test_srds_parity(wname):
+    w = W.ALL[wname]
+    orc = oracle_srds(w)
+    md, me = margins(orc, w.tol, w.cache_thresh)
+    assert md > 1e-6 and me > 1e-6, (md, me)
+    compare_srds(w, orc, gpu_srds(w))
+
+
+def test_srds_small_and_ragged():
+    w = W.TINY.with_(T=30, latent_shape=(3, 7, 9), K=4, sampler="srds", batch=3)
+    compare_srds(w, oracle_srds(w), gpu_srds(w))
+
+
+def test_srds_uncached_exact_after_n_iterations():
+    """tol = 0 and no cache hits: N iterations, and the serial DDIM result."""
+    w = W.SRDS.with_(latent_shape=(4, 16, 16))
+    a, x0, mu = W.inputs(w)
+    g = gpu_srds(w, tol=0.0, thresh=0.0)
+    assert g["stats"]["iters"] == g["stats"]["blocks"] and g["stats"]["hits"] == 0
+    serial = serial_ddim(a, x0, make_eps_fn(a, mu, w.gmm_std))[:, -1]
+    rel = np.abs(g["x_final"] - serial).max(axis=1) / np.abs(serial).max(axis=1)
+    assert rel.max() <= 1e-5, rel
+
+
+def test_srds_async_equals_sync():
+    w = W.SRDS.with_(latent_shape=(4, 16, 16))
+    a = gpu_srds(w)
+    b = gpu_srds(w, mode="async")
+    assert np.array_equal(a["x_final"], b["x_final"])
+    assert a["stats"]["nfe"] == b["stats"]["nfe"]

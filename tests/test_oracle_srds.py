@@ -84,10 +84,10 @@ def test_counting_invariants_and_first_entries():
     r = run_srds(a, x0, fn, 1e-4, 0.05)
     evals = sum(len(b) for b in r.batches)
     assert r.nfe + r.hits == evals
-    assert r.nfe == sum(1 for b in r.batches for (_, _, hit) in b if not hit)
+    assert r.nfe == sum(1 for b in r.batches for (_, _, hit, _) in b if not hit)
     seen = set()
     for batch in r.batches:
-        for (b, i, hit) in batch:
+        for (b, i, hit, _) in batch:
             if (b, i) not in seen:
                 assert not hit                 # first entry is a miss (Sec. 2.2)
             seen.add((b, i))

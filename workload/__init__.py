@@ -54,6 +54,7 @@ class Workload:
     seed: int = 0               # trajectory b uses noise seed (seed + b)
     gmm_std: float = GMM_STD
     eta: float = 0.0            # stochastic steps (eta = 1: DDPM); 0 = DDIM
+    sampler: str = "picard"     # "picard" (sliding window) or "srds" (Parareal blocks; window unused)
     extra: dict = field(default_factory=dict, compare=False)
 
     @property
@@ -77,6 +78,9 @@ LARGE = Workload("large T200 P64 B2 4x128x128 K64", T=200, window=64, batch=2,
 # over the full 1000-step schedule, window 64 (Table 2's best DDPM window).
 DDPM = Workload("DDPM T1000 P64 B1 4x64x64 K16", T=1000, window=64, batch=1,
                 latent_shape=(4, 64, 64), K=16, tol=1e-3, cache_thresh=0.05, eta=1.0)
+# Parareal (SRDS-style) sampling with the cache, on the SD-shaped and batched inputs.
+SRDS = SD15.with_(name="SRDS T100 B1 4x64x64 K16", sampler="srds")
+SRDS_BATCHED = BATCHED.with_(name="SRDS T100 B8 4x64x64 K16", sampler="srds")
 SWEEP_THRESHOLDS = (0.0, 0.01, 0.02, 0.05, 0.1)
 
 
@@ -86,7 +90,8 @@ def sweep(base: Workload = SD15):
             for c in SWEEP_THRESHOLDS]
 
 
-ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM}
+ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM,
+       "srds": SRDS, "srds_batched": SRDS_BATCHED}
 
 
 def train_alphas_cumprod() -> np.ndarray:
