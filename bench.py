@@ -207,7 +207,7 @@ class ClockSampler:
 def oracle_sample(workload_name, budget_s):
     """Time the fp64 oracle on whole generations of the workload for about
     budget_s seconds (at least one generation). Runs in a fresh process."""
-    from oracle import run_picard
+    from oracle import run_picard, run_srds
     from oracle.gmm import make_eps_fn
     w = W.ALL[workload_name]
     a, x0, mu = W.inputs(w)
@@ -215,9 +215,13 @@ def oracle_sample(workload_name, budget_s):
     iters = gens = 0
     t0 = time.perf_counter()
     while True:
-        r = run_picard(a, x0, f, w.window, w.tol, w.cache_thresh, record=False,
-                       eta=w.eta, noise=W.noise(w))
-        iters += r.iters
+        if w.sampler == "srds":   # a solver step is one evaluation stage
+            r = run_srds(a, x0, f, w.tol, w.cache_thresh)
+            iters += len(r.batches)
+        else:
+            r = run_picard(a, x0, f, w.window, w.tol, w.cache_thresh, record=False,
+                           eta=w.eta, noise=W.noise(w))
+            iters += r.iters
         gens += 1
         if time.perf_counter() - t0 >= budget_s:
             break
@@ -242,7 +246,7 @@ def cpu_baseline(workload_name, budget_s=12.0):
     s = time_oracle_subprocess(workload_name, budget_s)
     return {"value": s["iters"] / s["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
             "sample": f"{s['generations']} full generation(s) of the workload "
-                      f"({s['iters']} Picard iterations, {s['seconds']:.1f} s) by the fp64 NumPy "
+                      f"({s['iters']} solver steps, {s['seconds']:.1f} s) by the fp64 NumPy "
                       f"oracle, single-threaded (BLAS/OpenMP threads = 1)"}
 
 
@@ -268,7 +272,9 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000.0 * secs / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name, "step": "one full cached-Picard generation",
+        "config": {"workload": w.name,
+                   "step": ("one full cached Parareal generation (solver step = evaluation stage)"
+                            if w.sampler == "srds" else "one full cached-Picard generation"),
                    "global_batch": w.batch, "seq_len": w.T, "window": w.window},
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"{args.steps} full generation(s), fp64 NumPy oracle, "
@@ -296,6 +302,8 @@ def run_ours(args):
         pa_build.build()
     barrier()
     w = rank_workload(W.ALL[args.workload], rank)
+    if w.sampler == "srds":
+        return run_srds_bench(args, w)
     a, x0, mu = W.inputs(w)
     dev = torch.device("cuda", local)
     stream = torch.cuda.Stream(device=dev)
@@ -527,6 +535,163 @@ def run_ours(args):
     g.close()
     if world > 1:
         dist.destroy_process_group()
+    return 0
+
+
+def run_srds_bench(args, w):
+    """The Parareal (SRDS-style) sampler: a solver step is one evaluation stage
+    (a fine step of every block, or one coarse block, with its cache test,
+    compaction, denoiser call and update). One generation = every stage until
+    all trajectories converged, captured as one CUDA graph; L2 flushed between
+    generations; CUDA events around each replay."""
+    import torch
+    import torch.distributed as dist
+    from paper_2609_36522_gb300.solver import SrdsSolver, GmmDenoiser
+    rank, world, local = rank_info()
+    a, x0, mu = W.inputs(w)
+    dev = torch.device("cuda", local)
+    stream = torch.cuda.Stream(device=dev)
+    torch.cuda.set_stream(stream)
+    s = SrdsSolver(w.T, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=stream)
+    g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, s.max_rows, stream=stream)
+    if args.gmm_form is not None:
+        g.set_form(args.gmm_form)
+    eps = torch.empty(s.max_rows, w.D, dtype=torch.float32, device=dev)
+    x_dev = torch.from_numpy(x0).to(dev)
+    flush = None if args.no_flush else torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
+
+    def one_stage():
+        g.eps(*s.step_async(), eps)
+        s.submit_eps(eps)
+
+    s.init(x_dev)
+    n_stages = 0
+    while True:                         # the stage count, through the synchronous API
+        out = s.step()
+        if out is None:
+            break
+        g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+        s.submit_eps(eps)
+        n_stages += 1
+    st0 = s.stats()
+    nfe, hits, iters = st0["nfe"], st0["hits"], st0["iters"]
+    l_init = s.stats()["launches"]
+    s.init(x_dev)
+    stream.synchronize()
+    l0 = s.stats()["launches"] + g.launches()
+    l_init = s.stats()["launches"] - l_init
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=stream):
+        for _ in range(n_stages):
+            one_stage()
+    launches_per_gen = s.stats()["launches"] + g.launches() - l0
+
+    def generation():
+        if flush is not None:
+            flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        s.init(x_dev)
+        graph.replay()
+        e1.record(stream)
+        e1.synchronize()
+        return e0.elapsed_time(e1)
+
+    for _ in range(args.warmup):
+        generation()
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    barrier()
+    wall0 = time.perf_counter()
+    dev_ms = 0.0
+    for _ in range(args.steps):
+        dev_ms += generation()
+    stream.synchronize()
+    barrier()
+    wall = time.perf_counter() - wall0
+    st1 = s.stats()
+    assert st1["nfe"] == nfe and st1["n_active"] == 0, (st1, nfe)
+    time.sleep(0.2)
+    clk = clocks.stop()
+    units, secs = aggregate(args.steps * n_stages, dev_ms / 1000.0)
+    value = units / secs
+    # lower bound of the bytes every stage must move (fp64 states, fp32 eps):
+    # per evaluated row the distance (x, xhat: 16 B) and the update (x in and
+    # out, eps: 20 B); per miss the gather (12 B) and the cache entry (12 B)
+    row = w.D
+    alg = ((nfe + hits) * 36 + nfe * 24) * row
+    peak, peak_kind = measured_hbm_gbs()
+    achieved = alg * args.steps / (dev_ms / 1000.0) / 1e9
+    e2e = None
+    if not args.no_e2e:
+        x_host = torch.from_numpy(x0).pin_memory()
+        out_host = torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory()
+        polls = 0
+        reps = max(3, min(args.steps, 20))
+        stream.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            s.init(x_host)
+            done = False
+            while not done:
+                for _ in range(E2E_CHUNK):
+                    out = s.step_async()
+                    if out is None:
+                        done = True
+                        break
+                    g.eps(*out, eps)
+                    s.submit_eps(eps)
+                polls += 1
+                if not done and s.poll() == 0:
+                    done = True
+            s.result(out_host)
+        e1.record(stream)
+        stream.synchronize()
+        e2e_s = max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0)
+        units_e, secs_e = aggregate(reps * n_stages, e2e_s)
+        e2e = {"value": units_e / secs_e, "unit": UNIT, "h2d_bytes_per_step": int(w.batch * w.D * 4),
+               "d2h_bytes_per_step": int(w.batch * w.D * 4 + (polls // reps) * 24), "steps": reps,
+               "api": f"pa_srds_init (host x_init), pa_srds_step_async + pa_gmm_eps + pa_srds_submit_eps in "
+                      f"chunks of {E2E_CHUNK} stages, pa_srds_poll per chunk, pa_srds_result (host x_T)"}
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(args.workload)
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": dev_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64 states, f32 eps", "data": "synthetic",
+            "config": {"workload": w.name, "step": "one full cached Parareal generation",
+                       "solver_step_unit": "evaluation stage", "stages_per_step": n_stages,
+                       "parareal_iterations": iters, "blocks": s.blocks, "block_steps": s.block_steps,
+                       "global_batch": w.batch * world, "seq_len": w.T,
+                       "latent": "x".join(map(str, w.latent_shape)), "mixture_components": w.K,
+                       "tol": w.tol, "cache_thresh": w.cache_thresh,
+                       "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
+                                                 if g.form() == 1 else "CUDA cores (fp32 FMA)"),
+                       "parallelism": f"replicas x{world} (independent trajectories)",
+                       "l2": ("not flushed" if args.no_flush else
+                              "256 MiB write before every generation (between timed steps), outside the "
+                              "timed events"),
+                       "timing": "CUDA events around each generation (pa_srds_init, then one CUDA-graph "
+                                 "replay of its stages)"},
+            "nfe_per_step": nfe, "hits_per_step": hits, "hit_rate": hits / max(1, hits + nfe),
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                         "frac": achieved / peak, "traffic": None,
+                         "kernel": "whole evaluation stages (solver kernels and denoiser, one graph)",
+                         "traffic_note": "achieved = a lower bound of the stage bytes over the whole "
+                                         "generation time (latency-bound stages of B x N rows)",
+                         "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})"},
+            "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": int(args.steps * (launches_per_gen + l_init)),
+            "clocks": clk, "wall_s_timed_region": wall,
+        }
+        print(json.dumps(line))
+    s.close()
+    g.close()
     return 0
 
 
