@@ -182,7 +182,9 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
  * (default when D % 4 == 0; it falls back to plain loads for a batch_eps
  * pointer that is not 16-byte aligned), 100 + n = bulk-copy pipeline with
  * launch shape n (0..11; columns per lane, warps per CTA, pipeline depth --
- * a tuning aid). Returns PA_ERR_ARG for an unknown value. */
+ * a tuning aid), 112 = the register-resident form (rows loaded straight into
+ * registers; windows up to 104 points, 64 with stochastic steps, else the
+ * tiled pipeline). Returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
 
 /* Fault-handling test hook: the number of tries (each may suspend for about

@@ -242,11 +242,16 @@ constexpr int kDecideSmemPairs = 6144;  // (b, j) pairs whose reductions are sta
 
 __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
   __shared__ int s_last;
+  __shared__ DecideShared ds;
   extern __shared__ float s_red[];  // [2][B*P] when B*P <= kDecideSmemPairs
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   constexpr int nwarps = kDecideThreads / 32;
   const int npair = d.B * d.P;
 
+  // every CTA stages the trajectories and counters (written by the previous
+  // decision, several kernels back) before the dependency wait: whichever
+  // CTA finishes last then decides without another round trip to memory
+  decide_load<kDecideThreads>(d, ds);
   pdl_wait();  // the partials come from the update kernel
   const int item = blockIdx.x * nwarps + warp;
   if (item < 2 * npair) {
@@ -283,7 +288,7 @@ __global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
     }
   }
   __syncthreads();
-  decide_plan<kDecideThreads>(d, in_smem ? s_red : d.red_err, in_smem ? s_red + npair : d.red_del);
+  decide_run<kDecideThreads>(d, ds, in_smem ? s_red : d.red_err, in_smem ? s_red + npair : d.red_del);
 }
 
 }  // namespace

@@ -698,6 +698,248 @@ cudaError_t launch_seg(const Dev& d, const float* beps, cudaStream_t st, int* nc
   return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, nstrip, d.wait_limit);
 }
 
+// ---------------------------------------------------------------------------
+// Register-resident segment update. The same segmentation and arithmetic as
+// k_update_seg (warp w owns positions [w*L, min(p, (w+1)*L)), L = ceil(p/NW);
+// two passes joined by one CTA barrier; per-lane err/distance terms reduced
+// through a transposed shared-memory buffer), so its results are bit-identical
+// to that kernel's. Rows are not staged in shared memory: every lane loads its
+// V columns of each of its positions' rows (eps, old state, next cache input,
+// draw) straight into registers with 16-byte loads, all issued before the
+// first is used, and both passes run on registers. Each row crosses the SM's
+// load/store path once (in) and the results once (out), against four times
+// for the staged form (bulk copy in, a read in each pass, the drift written
+// and read back). LMAX bounds the positions per warp (registers: about
+// 3-4 rows x V x LMAX floats per thread). No waits of any kind.
+template <int V, int NW>
+struct RegShape {
+  static constexpr int SEG = 32 * V;
+  __host__ __device__ static size_t rank_bytes(int P) { return ((size_t)P * 4 + 127) / 128 * 128; }
+  static constexpr size_t kTotBytes = (size_t)NW * SEG * 2 * sizeof(float);
+  __host__ __device__ static size_t red_bytes(int P) { return ((size_t)2 * P * 33 * sizeof(float) + 127) / 128 * 128; }
+  __host__ __device__ static size_t smem_bytes(int P) { return rank_bytes(P) + kTotBytes + red_bytes(P); }
+};
+
+template <int V, int NW, int LMAX, bool NOISE>
+__global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* __restrict__ beps, int nstrip) {
+  using Sh = RegShape<V, NW>;
+  constexpr int SEG = Sh::SEG;
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int P = d.P;
+  const int b = blockIdx.y;
+  const int64_t D = d.D;
+  int32_t* s_rank = reinterpret_cast<int32_t*>(smem_raw);
+  float* s_tot = reinterpret_cast<float*>(smem_raw + Sh::rank_bytes(P));              // [NW][SEG][2]
+  float* s_red = reinterpret_cast<float*>(smem_raw + Sh::rank_bytes(P) + Sh::kTotBytes);  // [2][P][33]
+
+  // Everything read before pdl_wait() was written two or more kernels back
+  // (the previous update and decision kernels); only the batch eps rows come
+  // from the denoiser just before. The ranks do not depend on the window, so
+  // they are fetched together with it.
+  const Traj tr = d.traj[b];
+  const int n_miss = d.ctl->n_miss;
+  for (int j = tid; j < P; j += NW * 32) {
+    int r = d.rank[b * P + j];
+    if (r >= n_miss) {  // never expected: keep every load in bounds and report it
+      atomicCAS(&d.ctl->status, kDevOk, kDevBadRank);
+      r = -1;
+    }
+    s_rank[j] = r;
+  }
+  if (tr.p == 0) return;
+  __syncthreads();
+  const int t = tr.t, p = tr.p, e = tr.e;
+  const int strip = blockIdx.x;
+  const int64_t mycol = (int64_t)strip * SEG + (int64_t)lane * V;
+  const bool live = mycol < D;
+  float* Xb = d.X + (int64_t)b * (P + 1) * D;
+  float* Xh = d.Xhat + (int64_t)b * P * D;
+  float* Eh = d.Ehat + (int64_t)b * P * D;
+  const int L = (p + NW - 1) / NW;  // <= LMAX (launcher)
+  const int j0 = warp * L;
+  const int nj = (j0 + L < p ? j0 + L : p) - j0;  // positions of this warp (may be <= 0)
+
+  int rk[LMAX + 1];
+#pragma unroll
+  for (int g = 0; g <= LMAX; ++g) rk[g] = (g <= nj && j0 + g < p) ? s_rank[j0 + g] : -1;
+  const int sl0 = nj > 0 ? (t + j0) % P : 0;        // cache slot of position j0
+  const int nx0 = nj > 0 ? (t + j0 + 1) % (P + 1) : 0;  // state-ring slot of x_{t+j0+1}
+
+  Vec<V> eps[LMAX], xo[LMAX], xh[LMAX], zn[LMAX];
+  float cm1[LMAX], ec[LMAX], sg[LMAX];
+  Vec<V> xstart{}, xfill{}, xc0{};
+  if (live) {
+    xstart = ldv<V>(Xb + (int64_t)(t % (P + 1)) * D + mycol);
+    xfill = ldv<V>(Xb + (int64_t)(e % (P + 1)) * D + mycol);
+    if (nj > 0 && j0 > 0 && t + j0 <= e) xc0 = ldv<V>(Xb + (int64_t)((t + j0) % (P + 1)) * D + mycol);
+  }
+#pragma unroll
+  for (int g = 0; g < LMAX; ++g) {
+    if (g < nj) {
+      const int j = j0 + g;
+      cm1[g] = d.cm1[t + j];
+      ec[g] = d.ecoef[t + j];
+      if (NOISE) sg[g] = d.sigma[t + j];
+      if (live) {
+        int sl = sl0 + g;
+        if (sl >= P) sl -= P;
+        int sl1 = sl + 1;
+        if (sl1 >= P) sl1 -= P;
+        int nx = nx0 + g;
+        if (nx >= P + 1) nx -= P + 1;
+        if (rk[g] < 0) eps[g] = ldv<V>(Eh + (int64_t)sl * D + mycol);
+        if (t + j + 1 <= e) xo[g] = ldv<V>(Xb + (int64_t)nx * D + mycol);
+        if (j + 1 < p && rk[g + 1] < 0) xh[g] = ldv<V>(Xh + (int64_t)sl1 * D + mycol);
+        if (NOISE) zn[g] = ldv<V>(d.noise + ((int64_t)b * d.T + t + j) * D + mycol);
+      }
+    }
+  }
+  pdl_wait();  // the batch eps rows come from the denoiser that ran just before
+  if (live) {
+#pragma unroll
+    for (int g = 0; g < LMAX; ++g)
+      if (g < nj && rk[g] >= 0) eps[g] = ldv<V>(beps + (int64_t)rk[g] * D + mycol);
+  }
+
+  // phase 1: the drifts (kept in eps), the cache update of the misses
+  // (Eq. 7), and the compensated sum of the segment
+  float rh[V], rl[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) { rh[v] = 0.f; rl[v] = 0.f; }
+  if (live) {
+    Vec<V> xc = j0 == 0 ? xstart : ((t + j0 <= e) ? xc0 : xfill);
+#pragma unroll
+    for (int g = 0; g < LMAX; ++g) {
+      if (g < nj) {
+        const int j = j0 + g;
+        if (rk[g] >= 0) {  // Eq. 7: the cache takes (x_i, eps_i) of a miss
+          int sl = sl0 + g;
+          if (sl >= P) sl -= P;
+          const int64_t o = (int64_t)sl * D + mycol;
+          stv<V>(Eh + o, eps[g]);
+          stv<V>(Xh + o, xc);
+        }
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          float dr = fmaf(cm1[g], xc.a[v], ec[g] * eps[g].a[v]);
+          if (NOISE) dr = fmaf(sg[g], zn[g].a[v], dr);
+          acc_add(rh[v], rl[v], dr);
+          eps[g].a[v] = dr;
+        }
+        xc = (t + j + 1 <= e) ? xo[g] : xfill;
+      }
+    }
+  }
+#pragma unroll
+  for (int v = 0; v < V; ++v) {
+    const size_t o = ((size_t)warp * SEG + lane * V + v) * 2;
+    s_tot[o] = rh[v];
+    s_tot[o + 1] = rl[v];
+  }
+  __syncthreads();
+
+  // phase 2: carry into this segment, then the new states, errors, distances
+  float ch[V], cl[V];
+#pragma unroll
+  for (int v = 0; v < V; ++v) { ch[v] = xstart.a[v]; cl[v] = 0.f; }
+  for (int w = 0; w < warp; ++w) {
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      const size_t o = ((size_t)w * SEG + lane * V + v) * 2;
+      acc_add2(ch[v], cl[v], s_tot[o], s_tot[o + 1]);
+    }
+  }
+#pragma unroll
+  for (int g = 0; g < LMAX; ++g) {
+    if (g < nj) {
+      const int j = j0 + g;
+      float ev = 0.f, dv = 0.f;
+      if (live) {
+        const Vec<V> xold = (t + j + 1 <= e) ? xo[g] : xfill;
+        Vec<V> xn;
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          acc_add(ch[v], cl[v], eps[g].a[v]);
+          xn.a[v] = ch[v] + cl[v];
+          const float df = xn.a[v] - xold.a[v];
+          ev = fmaf(df, df, ev);
+        }
+        int nx = nx0 + g;
+        if (nx >= P + 1) nx -= P + 1;
+        stv<V>(Xb + (int64_t)nx * D + mycol, xn);
+        if (j + 1 < p) {
+          // the next timestep's cache input: its entry if it is a hit, else
+          // this iteration's x_{i+1} (the entry it is about to receive)
+          const Vec<V> xc1 = rk[g + 1] < 0 ? xh[g] : xold;
+#pragma unroll
+          for (int v = 0; v < V; ++v) dv += fabsf(xn.a[v] - xc1.a[v]);
+        }
+      }
+      s_red[(size_t)j * 33 + lane] = ev;
+      s_red[(size_t)(P + j) * 33 + lane] = dv;
+    }
+  }
+  __syncthreads();
+  // strip partials: one thread per (quantity, position) sums its row of lanes
+  const int64_t pbase = (int64_t)b * P * nstrip + strip;
+  for (int r = tid; r < 2 * p; r += NW * 32) {
+    const int which = r / p, j = r % p;
+    const float* row = s_red + (size_t)(which * P + j) * 33;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+    for (int c = 0; c < 32; c += 4) {
+      acc[0] += row[c];
+      acc[1] += row[c + 1];
+      acc[2] += row[c + 2];
+      acc[3] += row[c + 3];
+    }
+    (which == 0 ? d.part_err : d.part_del)[pbase + (int64_t)j * nstrip] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+  }
+}
+
+template <int V, int NW, int LMAX, bool NOISE>
+cudaError_t launch_reg(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+  using Sh = RegShape<V, NW>;
+  const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
+  const size_t smem = Sh::smem_bytes(d.P);
+  auto kern = k_update_reg<V, NW, LMAX, NOISE>;
+  static size_t configured[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64 || smem > configured[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64) configured[dev] = smem;
+  }
+  *nchunk_out = nstrip;
+  return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, nstrip);
+}
+
+// Positions per warp that the register-resident form holds for a window of P
+// (8 warps): 0 when it does not apply.
+constexpr int kRegMaxL = 13;       // deterministic steps: 3 rows x 4 x 13 floats per thread
+constexpr int kRegMaxLNoise = 8;   // stochastic steps: 4 rows x 4 x 8
+int reg_lmax(const Dev& d) {
+  const int L = (d.P + 7) / 8;
+  if (L <= 4) return 4;
+  if (L <= 8) return 8;
+  if (L <= kRegMaxL && !d.noise) return kRegMaxL;
+  return 0;
+}
+
+cudaError_t launch_reg_auto(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+  const int lm = reg_lmax(d);
+  if (d.noise) {
+    if (lm == 4) return launch_reg<4, 8, 4, true>(d, beps, st, nchunk_out);
+    return launch_reg<4, 8, kRegMaxLNoise, true>(d, beps, st, nchunk_out);
+  }
+  if (lm == 4) return launch_reg<4, 8, 4, false>(d, beps, st, nchunk_out);
+  if (lm == 8) return launch_reg<4, 8, 8, false>(d, beps, st, nchunk_out);
+  return launch_reg<4, 8, kRegMaxL, false>(d, beps, st, nchunk_out);
+}
+
 // Shared memory budget per CTA for the tile buffers: enough for the whole
 // window when it fits, so every copy is in flight from the start.
 constexpr size_t kSmemBudget = 112 * 1024;
@@ -762,6 +1004,7 @@ bool prefer_wide_strips(const Dev& d) {
 }
 
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
+  if (d.bulk_cfg == 12 && reg_lmax(d)) return launch_reg_auto(d, batch_eps, st, nchunk_out);
   if (d.noise) {  // stochastic steps: the segment form with the draws staged (update_bulk_supported)
     if (prefer_wide_strips<true>(d)) return launch_seg<4, 8, true>(d, batch_eps, st, nchunk_out);
     return launch_seg<2, 8, true>(d, batch_eps, st, nchunk_out);
@@ -789,6 +1032,8 @@ cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_
                                       : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
     case 11: return seg_fits<4, 4>(d) ? launch_seg<4, 4>(d, batch_eps, st, nchunk_out)
                                       : launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
+    case 12: return reg_lmax(d) ? launch_reg_auto(d, batch_eps, st, nchunk_out)
+                                : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
     default: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
   }
 }

@@ -18,31 +18,48 @@ namespace pa {
 //     misses; misses are compacted trajectory-major into miss_bt with a
 //     block-wide prefix sum, and rank[b][j] records each miss's batch row;
 //  3. updates the counters (n_miss, n_active, iter, nfe, hits).
+// Shared state of one decision (static shared memory of the calling kernel).
+struct DecideShared {
+  int t[kMaxBatch], p[kMaxBatch], e[kMaxBatch];
+  int tn[kMaxBatch], pn[kMaxBatch], m[kMaxBatch], h1[kMaxBatch];
+  int om[kMaxBatch], oh1[kMaxBatch];
+  int warp_tot[32];
+  int total, active, iter;
+};
+
+// The trajectories and counters a decision starts from. They were written by
+// the previous decision, several kernels back, so a kernel may read them
+// before its dependency wait. No barrier.
 template <int NT>
-__device__ void decide_plan(const Dev& d, const float* red_e, const float* red_d) {
-  __shared__ int s_t[kMaxBatch], s_p[kMaxBatch], s_e[kMaxBatch];
-  __shared__ int s_tn[kMaxBatch], s_pn[kMaxBatch], s_m[kMaxBatch], s_h1[kMaxBatch];
-  __shared__ int s_om[kMaxBatch], s_oh1[kMaxBatch];
-  __shared__ int s_warp[NT / 32];
-  __shared__ int s_total, s_active, s_iter;
+__device__ void decide_load(const Dev& d, DecideShared& sh) {
+  const int tid = threadIdx.x;
+  if (tid == 0) {
+    sh.active = d.ctl->n_active;
+    sh.iter = d.ctl->iter;
+  }
+  for (int b = tid; b < d.B; b += NT) {
+    const Traj tr = d.traj[b];
+    sh.t[b] = tr.t; sh.p[b] = tr.p; sh.e[b] = tr.e;
+    sh.om[b] = tr.m; sh.oh1[b] = tr.h1;
+    sh.m[b] = 0;
+    sh.h1[b] = 0;
+  }
+}
+
+// Steps 1-3 above on the state decide_load staged; starts with a barrier.
+template <int NT>
+__device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, const float* red_d) {
+  int* s_t = sh.t; int* s_p = sh.p; int* s_e = sh.e;
+  int* s_tn = sh.tn; int* s_pn = sh.pn; int* s_m = sh.m; int* s_h1 = sh.h1;
+  int* s_om = sh.om; int* s_oh1 = sh.oh1; int* s_warp = sh.warp_tot;
   constexpr int nwarps = NT / 32;
   static_assert(nwarps <= 32, "one warp scans the warp totals");
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int B = d.B, P = d.P, T = d.T;
-  if (tid == 0) {
-    s_active = d.ctl->n_active;
-    s_iter = d.ctl->iter;
-  }
-  for (int b = tid; b < B; b += NT) {
-    const Traj tr = d.traj[b];
-    s_t[b] = tr.t; s_p[b] = tr.p; s_e[b] = tr.e;
-    s_om[b] = tr.m; s_oh1[b] = tr.h1;
-    s_m[b] = 0;
-    s_h1[b] = 0;
-  }
   __syncthreads();
+  const int s_active = sh.active;
   if (s_active == 0) return;  // finished: iterating further is a no-op
-  const int iter = s_iter;
+  const int iter = sh.iter;
 
   // 1. window advance, one warp per trajectory
   for (int b = warp; b < B; b += nwarps) {
@@ -110,7 +127,7 @@ __device__ void decide_plan(const Dev& d, const float* red_e, const float* red_d
       if (lane >= o) wi += v;
     }
     if (lane < nwarps) s_warp[lane] = wi - w;  // exclusive
-    if (lane == 31) s_total = wi;
+    if (lane == 31) sh.total = wi;
   }
   __syncthreads();
   int r = s_warp[warp] + incl - cnt;
@@ -146,13 +163,19 @@ __device__ void decide_plan(const Dev& d, const float* red_e, const float* red_d
   if (tid == 0) {
     int act = 0;
     for (int b = 0; b < B; ++b) act += (s_pn[b] > 0);
-    const int n = s_total;
+    const int n = sh.total;
     d.ctl->n_miss = n;
     d.ctl->n_active = act;
     d.ctl->iter = iter + 1;
     d.ctl->nfe += n;
     d.ctl->hits += pts - n;
   }
+}
+
+template <int NT>
+__device__ void decide_plan(const Dev& d, DecideShared& sh, const float* red_e, const float* red_d) {
+  decide_load<NT>(d, sh);
+  decide_run<NT>(d, sh, red_e, red_d);
 }
 
 }  // namespace pa

@@ -12,7 +12,7 @@ constexpr int kMaxWindow = 1024;
 constexpr int kMaxBatch = 64;
 constexpr int kMinChunk = 32;       // narrowest column chunk of any update kernel
 constexpr size_t kAlign = 256;
-constexpr int kBulkConfigs = 12;    // launch shapes of the bulk-copy update kernel
+constexpr int kBulkConfigs = 13;    // launch shapes of the bulk-copy update kernel
 
 // Device status codes written by kernels (first error wins, atomicCAS from 0).
 constexpr int kDevOk = 0;

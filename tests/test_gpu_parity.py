@@ -214,7 +214,7 @@ def test_sd15_tensor_core_denoiser():
     compare(w, oracle_run(w), gpu_run(w, gmm_form=1))
 
 
-@pytest.mark.parametrize("kind", [0, 1] + list(range(100, 112)))
+@pytest.mark.parametrize("kind", [0, 1] + list(range(100, 113)))
 def test_update_kernels_agree(kind):
     """Plain-load and tile-parallel bulk-copy update kernels (every launch
     shape) take the same decisions and agree with the oracle; their states
@@ -229,6 +229,21 @@ def test_update_kernels_agree(kind):
     assert np.array_equal(ref["log"], got["log"])
     scale = np.abs(ref["x_final"]).max()
     assert np.abs(ref["x_final"] - got["x_final"]).max() <= 1e-6 * scale
+
+
+@pytest.mark.parametrize("window,eta", [(24, 0.0), (64, 0.0), (100, 0.0), (64, 1.0), (32, 0.5)])
+def test_register_update_matches_staged(window, eta):
+    """The register-resident update (launch shape 12) performs the staged
+    segment kernel's arithmetic (4 columns per lane, 8 warps) in the same
+    order: decisions and final latents bit-identical, on a ragged last strip."""
+    w = W.Workload("reg-vs-staged", T=100, window=window, batch=2, latent_shape=(4, 20, 20), K=6,
+                   tol=1e-3, cache_thresh=0.05, seed=5, eta=eta)
+    orc = oracle_run(w)
+    staged = gpu_run(w, update_kernel=110)
+    reg = gpu_run(w, update_kernel=112)
+    assert np.array_equal(staged["log"], reg["log"])
+    assert np.array_equal(staged["x_final"], reg["x_final"])
+    assert compare(w, orc, reg).max() <= REL_TOL
 
 
 # ---- stochastic steps (eta > 0): DDPM over the full 1000-step schedule -------
