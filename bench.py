@@ -342,8 +342,9 @@ def run_ours(args):
     nfe, hits = st0["nfe"], st0["hits"]
     upd_bytes, other_bytes = iteration_bytes(log, w)
 
-    # One generation (n_iters Picard iterations: gather, denoiser, update and
-    # decision kernels each) as a CUDA graph. The timed graph also records CUDA
+    # One generation (n_iters Picard iterations: denoiser, update and planning
+    # kernels each -- the planning kernel decides and gathers the next batch;
+    # pa_init gathers the first) as a CUDA graph. The timed graph also records CUDA
     # events around every update-kernel launch (the roofline's kernel time); the
     # plain graph has no event nodes and gives the iteration rate.
     s.init(x_dev)
@@ -351,26 +352,27 @@ def run_ours(args):
     stream.synchronize()
 
     def capture(timed):
+        """-> (graph, kernels launched per iteration inside it)"""
         abi.pa_set_kernel_timing(s.h, timed)
         abi.pa_kernel_timing(s.h, reset=True)
-        s.init(x_dev)
         stream.synchronize()
+        l0 = s.stats()["launches"] + g.launches()
         gr = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gr, stream=stream):
+            s.init(x_dev)                 # x_init copy, sums cleared, first plan and its gather
             for _ in range(n_iters):
                 one_iteration()
         abi.pa_set_kernel_timing(s.h, False)
-        return gr
+        l1 = s.stats()["launches"] + g.launches()
+        return gr, (l1 - l0 - init_launches) // n_iters
 
-    gmm0, sol0 = g.launches(), s.stats()["launches"]
-    graph_plain = capture(False)
-    # gather, update, decision + denoiser kernels of one Picard iteration
-    kernels_per_iter = ((s.stats()["launches"] - sol0) + (g.launches() - gmm0)) // n_iters
-    graph_timed = capture(True)
+    # denoiser, update and planning (decision + next gather) kernels of one iteration
+    init_launches = 2                     # pa_init: first plan and its gather
+    graph_plain, kernels_per_iter = capture(False)
+    graph_timed, _ = capture(True)
 
     def generation(gr, timed):
-        """L2 flushed, then one generation timed with one event pair."""
-        s.init(x_dev)
+        """L2 flushed, then one generation (pa_init included) timed with one event pair."""
         if flush is not None:
             flush.zero_()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -383,21 +385,24 @@ def run_ours(args):
         return ms, upd
 
     def cold_iterations(reps):
-        """Per-iteration time with L2 flushed before every Picard iteration."""
-        single = torch.cuda.CUDAGraph()
+        """Per-iteration time with L2 flushed before every Picard iteration.
+        Iterations alternate between the two copies of the plan, so an even
+        and an odd iteration are captured and replayed in turn."""
+        single = [torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()]
         s.init(x_dev)
         stream.synchronize()
-        with torch.cuda.graph(single, stream=stream):
-            one_iteration()
+        for k in range(2):
+            with torch.cuda.graph(single[k], stream=stream):
+                one_iteration()
         tot, n = 0.0, 0
         for _ in range(reps):
             s.init(x_dev)
-            for _ in range(n_iters):
+            for it in range(n_iters):
                 if flush is not None:
                     flush.zero_()
                 e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
                 e0.record(stream)
-                single.replay()
+                single[it % 2].replay()
                 e1.record(stream)
                 e1.synchronize()
                 tot += e0.elapsed_time(e1)
@@ -432,7 +437,7 @@ def run_ours(args):
     assert st1["iters"] == n_iters and st1["nfe"] == nfe, (st1, n_iters, nfe)
     time.sleep(0.2)
     clk = clocks.stop()
-    launches = 2 * args.steps * (n_iters * kernels_per_iter + 1)   # both graphs; + init plan per generation
+    launches = 2 * args.steps * (n_iters * kernels_per_iter + init_launches)   # both graphs, pa_init each
     cold_us = cold_iterations(max(1, min(args.steps, 10)))
 
     units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
@@ -513,8 +518,9 @@ def run_ours(args):
                        "l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every generation (between timed steps), outside the "
                               "timed events"),
-                       "timing": "CUDA events around each generation: one CUDA-graph replay of its Picard "
-                                 "iterations (gather, denoiser, update and decision kernels each) on the "
+                       "timing": "CUDA events around each generation: pa_init outside, then one CUDA-graph "
+                                 "replay of its Picard iterations (denoiser, update and planning kernels each; "
+                                 "the planning kernel decides and gathers the next batch) on the "
                                  "launch stream; the update kernel's own events come from a second graph "
                                  "of the same generation, replayed alternately"},
             "nfe_per_step": nfe, "hits_per_step": hits,

@@ -1,5 +1,6 @@
 // Solver-step kernels for sm_103a: first-iteration plan, miss gather (a4),
-// plain-load Picard update (a6-a9, a11) and the decision kernel (a10, a2, a3).
+// plain-load Picard update (a6-a9, a11) and the planning kernel that takes
+// the decision after an update (a10, a2, a3) and gathers the next batch (a4).
 //
 // Data layout (fp32, one row = one timestep's latent of D floats):
 //   X    [B][P+1][D]  state ring, state i lives in slot i mod (P+1)
@@ -33,7 +34,7 @@ __global__ void k_init_plan(Dev d) {
   for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
     Traj tr{};
     tr.t = 0; tr.p = p0; tr.e = 0; tr.done = 0; tr.m = p0; tr.h1 = 0;
-    d.traj[b] = tr;
+    d.traj[b] = tr;  // copy 0: the plan of iteration 0
   }
   for (int q = threadIdx.x; q < d.B * d.P; q += blockDim.x) {
     const int b = q / d.P, j = q % d.P;
@@ -55,6 +56,12 @@ __global__ void k_init_plan(Dev d) {
     c.nfe = (long long)d.B * p0;
     c.hits = 0;
     *d.ctl = c;
+    PlanCtr pc;
+    pc.n_active = c.n_active;
+    pc.iter = 0;
+    pc.nfe = c.nfe;
+    pc.hits = 0;
+    d.pc[0] = pc;
   }
 }
 
@@ -66,31 +73,38 @@ constexpr int kGatherThreads = 256;
 constexpr int kGatherUnroll = 4;
 
 template <int VEC>
-__global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d) {
+__device__ __forceinline__ void copy_row(const Dev& d, int b, int src_state, int r) {
   using T = typename std::conditional<VEC == 4, float4, float>::type;
-  pdl_wait();  // everything read here comes from the decision kernel
-  const int n = d.ctl->n_miss;
   const int64_t nvec = d.D / VEC;
   const int64_t stride = (int64_t)gridDim.x * kGatherThreads;
   const int64_t base = (int64_t)blockIdx.x * kGatherThreads + threadIdx.x;
+  const T* from = reinterpret_cast<const T*>(d.X + ((int64_t)b * (d.P + 1) + src_state % (d.P + 1)) * d.D);
+  T* to = reinterpret_cast<T*>(d.batch_x + (int64_t)r * d.D);
+  for (int64_t v0 = base; v0 < nvec; v0 += stride * kGatherUnroll) {
+    T buf[kGatherUnroll];
+#pragma unroll
+    for (int u = 0; u < kGatherUnroll; ++u) {
+      const int64_t v = v0 + u * stride;
+      if (v < nvec) buf[u] = __ldg(from + v);
+    }
+#pragma unroll
+    for (int u = 0; u < kGatherUnroll; ++u) {
+      const int64_t v = v0 + u * stride;
+      if (v < nvec) to[v] = buf[u];
+    }
+  }
+}
+
+// The gather of a plan already in memory (copy par): after the first plan,
+// and after the one-CTA planner.
+template <int VEC>
+__global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d, int par) {
+  pdl_wait();  // everything read here comes from the kernel that planned
+  const int n = d.ctl->n_miss;
+  const Traj* tr = d.traj + par * d.B;
   for (int r = blockIdx.y; r < n; r += gridDim.y) {
     const int b = d.miss_bt[2 * r], i = d.miss_bt[2 * r + 1];
-    const int src = min(i, d.traj[b].e);
-    const T* from = reinterpret_cast<const T*>(d.X + ((int64_t)b * (d.P + 1) + src % (d.P + 1)) * d.D);
-    T* to = reinterpret_cast<T*>(d.batch_x + (int64_t)r * d.D);
-    for (int64_t v0 = base; v0 < nvec; v0 += stride * kGatherUnroll) {
-      T buf[kGatherUnroll];
-#pragma unroll
-      for (int u = 0; u < kGatherUnroll; ++u) {
-        const int64_t v = v0 + u * stride;
-        if (v < nvec) buf[u] = __ldg(from + v);
-      }
-#pragma unroll
-      for (int u = 0; u < kGatherUnroll; ++u) {
-        const int64_t v = v0 + u * stride;
-        if (v < nvec) to[v] = buf[u];
-      }
-    }
+    copy_row<VEC>(d, b, min(i, tr[b].e), r);
   }
 }
 
@@ -105,8 +119,8 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d) {
 //   x'_{i+1} = x_t + sum_{l<=j} d_{t+l}  (compensated)            Eq. 1
 //   err_j  partial of sum (x'_{i+1} - x_{i+1})^2                  Eq. 2
 //   del_j  partial of sum |x'_{i+1} - xhat_{i+1}| (next iteration) Eq. 4
-// Partials are reduced per CTA in a fixed order and written to
-// part_*[b][j][chunk]; the decision kernel finishes the reduction.
+// Partials are reduced per CTA in a fixed order and added into the
+// iteration's fp64 accumulators (red_add); the planning kernel reads the sums.
 template <int VEC>
 struct V;
 template <>
@@ -142,12 +156,11 @@ __device__ __forceinline__ void stv(float* p, const V<VEC>& v) {
 constexpr int kPlainThreads = 128;
 
 template <int VEC>
-__global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const float* __restrict__ beps,
-                                                             int nchunk) {
+__global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const float* __restrict__ beps, int par) {
   extern __shared__ float red[];  // [2][nwarps][P]
   const int b = blockIdx.y;
   pdl_wait();
-  const Traj tr = d.traj[b];
+  const Traj tr = d.traj[par * d.B + b];
   if (tr.p == 0) return;
   const int t = tr.t, p = tr.p, e = tr.e, P = d.P;
   const int64_t D = d.D;
@@ -224,71 +237,91 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
       se += red[w * P + j];
       sd += red[(nw + w) * P + j];
     }
-    const int64_t o = ((int64_t)b * P + j) * nchunk + blockIdx.x;
-    d.part_err[o] = se;
-    d.part_del[o] = sd;
+    red_add(d, par, 0, b * P + j, se);
+    red_add(d, par, 1, b * P + j, sd);
   }
 }
 
 // ---------------------------------------------------------------------------
-// Decision kernel for the update kernels that leave the reductions unfinished
-// (plain-load and tile forms), one launch of many CTAs: every CTA finishes
-// some of the reductions -- one warp per (quantity, b, j) sums the chunk
-// partials of err[b][j] (Eq. 2) or of the distance of timestep t+j+1 (Eq. 4)
-// in a fixed order (deterministic), to red_* -- and the CTA that finishes
-// last (atomic ticket after a fence; nobody waits) runs decide_plan.
-constexpr int kDecideThreads = 256;
-constexpr int kDecideSmemPairs = 6144;  // (b, j) pairs whose reductions are staged in shared memory
+// Planning kernel (a10, a2, a3 after iteration k, then a4 of iteration k+1),
+// one launch. The update kernel left complete fp64 sums of the Eq. 2 errors
+// and Eq. 4 distances; every CTA reads them (B*P of each), divides by D and
+// takes the whole decision in shared memory -- the same inputs and the same
+// arithmetic give the same plan in every CTA -- then copies the column range
+// blockIdx.x of batch row blockIdx.y, if that row holds a miss. CTA (0, 0)
+// also publishes the plan (copy par ^ 1 of the trajectories and counters,
+// ranks, miss list, iteration log, the reductions for the host) and clears
+// the accumulator set of iteration k+1. Nobody waits for anybody: the other
+// CTAs read copy par of the plan, which no CTA writes in this launch.
+constexpr int kPlanThreads = 256;
+constexpr int kFusedMaxPairs = 1024;  // B*P planned in every CTA; beyond, one CTA plans
 
-__global__ void __launch_bounds__(kDecideThreads) k_decide(Dev d, int nchunk) {
-  __shared__ int s_last;
+struct RedShared {
+  const double* e;
+  const double* dl;
+  __device__ double err(int q) const { return e[q]; }
+  __device__ double del(int q) const { return dl[q]; }
+};
+
+struct RedSums {
+  const double* e;
+  const double* dl;
+  double inv_d;
+  __device__ double err(int q) const { return __ldcg(e + q) * inv_d; }
+  __device__ double del(int q) const { return __ldcg(dl + q) * inv_d; }
+};
+
+template <int VEC>
+__global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
   __shared__ DecideShared ds;
-  extern __shared__ float s_red[];  // [2][B*P] when B*P <= kDecideSmemPairs
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int nwarps = kDecideThreads / 32;
+  __shared__ double s_e[kFusedMaxPairs], s_d[kFusedMaxPairs];
+  const int tid = threadIdx.x;
+  const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
   const int npair = d.B * d.P;
+  decide_load<kPlanThreads>(d, ds, par);
+  pdl_wait();  // the sums and the new states come from the update kernel
+  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair;
+  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair;
+  const double inv_d = 1.0 / (double)d.D;
+  for (int q = tid; q < npair; q += kPlanThreads) {
+    const double ve = __ldcg(acc_e + q) * inv_d, vd = __ldcg(acc_d + q) * inv_d;
+    s_e[q] = ve;
+    s_d[q] = vd;
+    if (publish) {
+      d.red_err[q] = (float)ve;
+      d.red_del[q] = (float)vd;
+      double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair;  // iteration k+1 adds into these
+      nxt[q] = 0.0;
+      nxt[npair + q] = 0.0;
+    }
+  }
+  decide_run<kPlanThreads>(d, ds, RedShared{s_e, s_d}, par, publish, (int)blockIdx.y);
+  if ((int)blockIdx.y < ds.total && ds.target_b >= 0) {
+    const int b = ds.target_b;
+    copy_row<VEC>(d, b, min(ds.target_i, ds.en[b]), blockIdx.y);
+  }
+}
 
-  // every CTA stages the trajectories and counters (written by the previous
-  // decision, several kernels back) before the dependency wait: whichever
-  // CTA finishes last then decides without another round trip to memory
-  decide_load<kDecideThreads>(d, ds);
-  pdl_wait();  // the partials come from the update kernel
-  const int item = blockIdx.x * nwarps + warp;
-  if (item < 2 * npair) {
-    const int which = item / npair, pr = item % npair;
-    const float* src = (which ? d.part_del : d.part_err) + (int64_t)pr * nchunk;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
-    int c = lane;
-    for (; c + 96 < nchunk; c += 128) {
-      acc[0] += src[c];
-      acc[1] += src[c + 32];
-      acc[2] += src[c + 64];
-      acc[3] += src[c + 96];
-    }
-    for (; c < nchunk; c += 32) acc[0] += src[c];
-    float v = (acc[0] + acc[1]) + (acc[2] + acc[3]);
-    v = warp_sum(v);
-    if (lane == 0) (which ? d.red_del : d.red_err)[pr] = v / (float)d.D;
+// One-CTA planner for B*P beyond kFusedMaxPairs: reads the sums from memory;
+// a separate gather follows.
+constexpr int kPlanOneThreads = 1024;
+
+__global__ void __launch_bounds__(kPlanOneThreads) k_plan_one(Dev d, int par) {
+  __shared__ DecideShared ds;
+  const int npair = d.B * d.P;
+  decide_load<kPlanOneThreads>(d, ds, par);
+  pdl_wait();  // the sums come from the update kernel
+  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair;
+  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair;
+  const RedSums red{acc_e, acc_d, 1.0 / (double)d.D};
+  decide_run<kPlanOneThreads>(d, ds, red, par, true, -1);
+  double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair;
+  for (int q = threadIdx.x; q < npair; q += kPlanOneThreads) {
+    d.red_err[q] = (float)red.err(q);
+    d.red_del[q] = (float)red.del(q);
+    nxt[q] = 0.0;
+    nxt[npair + q] = 0.0;
   }
-  __syncthreads();
-  if (tid == 0) {
-    __threadfence();
-    const unsigned int k = atomicAdd(&d.ctl->ticket, 1u);
-    s_last = (k == gridDim.x - 1);
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();  // the other CTAs' reductions are visible from here on
-  if (tid == 0) d.ctl->ticket = 0u;  // ready for the next launch
-  const bool in_smem = npair <= kDecideSmemPairs;
-  if (in_smem) {
-    for (int q = tid; q < npair; q += kDecideThreads) {
-      s_red[q] = __ldcg(d.red_err + q);
-      s_red[npair + q] = __ldcg(d.red_del + q);
-    }
-  }
-  __syncthreads();
-  decide_run<kDecideThreads>(d, ds, in_smem ? s_red : d.red_err, in_smem ? s_red + npair : d.red_del);
 }
 
 }  // namespace
@@ -298,18 +331,49 @@ cudaError_t launch_init_plan(const Dev& d, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_gather(const Dev& d, cudaStream_t st) {
+namespace {
+dim3 gather_grid(const Dev& d) {
   const int rows = min(d.B * d.P, 65535);
   const int vec = (d.D % 4 == 0) ? 4 : 1;
   const int64_t nvec = d.D / vec;
   const int64_t want = (nvec + kGatherThreads * kGatherUnroll - 1) / (kGatherThreads * kGatherUnroll);
-  const int gx = (int)(want < 64 ? want : 64);
-  if (vec == 4) return launch_ex(k_gather<4>, dim3(gx, rows), dim3(kGatherThreads), 0, st, 0, d);
-  return launch_ex(k_gather<1>, dim3(gx, rows), dim3(kGatherThreads), 0, st, 0, d);
+  return dim3((int)(want < 64 ? want : 64), rows);
+}
+}  // namespace
+
+cudaError_t launch_gather(const Dev& d, int par, cudaStream_t st) {
+  const dim3 g = gather_grid(d);
+  if (d.D % 4 == 0) return launch_ex(k_gather<4>, g, dim3(kGatherThreads), 0, st, 0, d, par);
+  return launch_ex(k_gather<1>, g, dim3(kGatherThreads), 0, st, 0, d, par);
 }
 
-cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream_t st,
-                                int* nchunk_out) {
+cudaError_t launch_plan(const Dev& d, int par, cudaStream_t st, int* launches) {
+  if (d.B * d.P <= kFusedMaxPairs) {
+    *launches = 1;
+    // every CTA plans, so fewer and longer CTAs: about two per SM in all,
+    // each copying a longer part of its row
+    static int nsm[64] = {};
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev >= 0 && dev < 64 && nsm[dev] == 0) {
+      e = cudaDeviceGetAttribute(&nsm[dev], cudaDevAttrMultiProcessorCount, dev);
+      if (e != cudaSuccess) return e;
+    }
+    const int sms = (dev >= 0 && dev < 64 && nsm[dev] > 0) ? nsm[dev] : 148;
+    dim3 g = gather_grid(d);
+    const int gx = (2 * sms + (int)g.y - 1) / (int)g.y;
+    if (gx < (int)g.x) g.x = gx < 1 ? 1 : gx;
+    if (d.D % 4 == 0) return launch_ex(k_plan_gather<4>, g, dim3(kPlanThreads), 0, st, 0, d, par);
+    return launch_ex(k_plan_gather<1>, g, dim3(kPlanThreads), 0, st, 0, d, par);
+  }
+  *launches = 2;
+  cudaError_t e = launch_ex(k_plan_one, dim3(1), dim3(kPlanOneThreads), 0, st, 0, d, par);
+  if (e != cudaSuccess) return e;
+  return launch_gather(d, par ^ 1, st);
+}
+
+cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, int par, cudaStream_t st) {
   const size_t smem = (size_t)2 * (kPlainThreads / 32) * d.P * sizeof(float);
   // float4 rows need every row base 16-byte aligned: D % 4 == 0 and aligned
   // eps (and draws) pointers; the workspace arrays are 256-byte aligned
@@ -317,25 +381,10 @@ cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream
                        (reinterpret_cast<uintptr_t>(d.noise) & 15) == 0;
   if (d.D % 4 == 0 && aligned) {
     const int nchunk = (int)((d.D + kPlainThreads * 4 - 1) / (kPlainThreads * 4));
-    *nchunk_out = nchunk;
-    return launch_ex(k_update_plain<4>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps,
-                     nchunk);
-  } else {
-    const int nchunk = (int)((d.D + kPlainThreads - 1) / kPlainThreads);
-    *nchunk_out = nchunk;
-    return launch_ex(k_update_plain<1>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps,
-                     nchunk);
+    return launch_ex(k_update_plain<4>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
   }
-  return cudaGetLastError();
-}
-
-cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st) {
-  const int pairs = d.B * d.P;
-  const size_t smem = pairs <= kDecideSmemPairs ? (size_t)2 * pairs * sizeof(float) : 0;
-  const int nwarps = kDecideThreads / 32;
-  const int grid = (2 * pairs + nwarps - 1) / nwarps;
-  return launch_ex(k_decide, dim3(grid), dim3(kDecideThreads), smem, st, 0, d, nchunk);
-  return cudaGetLastError();
+  const int nchunk = (int)((d.D + kPlainThreads - 1) / kPlainThreads);
+  return launch_ex(k_update_plain<1>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
 }
 
 }  // namespace pa

@@ -130,7 +130,7 @@ struct TileShape {
 // warp 0 polls and the CTA barrier releases the others).
 template <int V, int NW, int S, bool CLUSTER, bool WAIT_ALL>
 __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __restrict__ beps,
-                                                         int nstrip, int nbuf, uint32_t wait_limit) {
+                                                         int nstrip, int nbuf, uint32_t wait_limit, int par) {
   using Sh = TileShape<V, NW, S>;
   constexpr int SEG = Sh::SEG, TW = Sh::TW;
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -158,7 +158,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   float* s_tile = reinterpret_cast<float*>(q);  // 128-byte aligned: all offsets above are
 
   // round 1: independent loads of the bookkeeping and every rank of the window
-  const Traj tr = d.traj[b];
+  const Traj tr = d.traj[par * d.B + b];
   const int n_miss = d.ctl->n_miss;
   for (int j = tid; j < P; j += NW * 32) s_rank[j] = d.rank[b * P + j];
   if (tr.p == 0) return;
@@ -406,30 +406,27 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   if constexpr (CLUSTER) {
     // Combine the strips of this cluster: CTA rank q sums positions j = q mod
     // kCluster over the cluster's CTAs in rank order (distributed shared
-    // memory) and writes part[b][j][cluster]. The second cluster barrier keeps
+    // memory) and adds it into the iteration's sums. The second cluster barrier keeps
     // every CTA's shared memory alive until its peers have read it.
     cg::cluster_group cluster = cg::this_cluster();
     cluster.sync();
     const int rank = (int)cluster.block_rank();
-    const int nclus = gridDim.x / kCluster;
-    const int64_t cbase = (int64_t)b * P * nclus + blockIdx.x / kCluster;
     for (int q2 = tid; q2 < 2 * p; q2 += NW * 32) {
       const int which = q2 / p, j = q2 % p;
       if (j % kCluster != rank) continue;
       float sum = 0.f;
 #pragma unroll
       for (int r = 0; r < kCluster; ++r) sum += cluster.map_shared_rank(s_pos, r)[which * P + j];
-      (which == 0 ? d.part_err : d.part_del)[cbase + (int64_t)j * nclus] = sum;
+      red_add(d, par, which, b * P + j, sum);
     }
     cluster.sync();
   } else {
-    // one partial per strip and position
+    // one partial per strip and position, added into the iteration's sums
     __syncthreads();
     if (active) {
-      const int64_t pbase = (int64_t)b * P * nstrip + strip;
       for (int q2 = tid; q2 < 2 * p; q2 += NW * 32) {
         const int which = q2 / p, j = q2 % p;
-        (which == 0 ? d.part_err : d.part_del)[pbase + (int64_t)j * nstrip] = s_pos[which * P + j];
+        red_add(d, par, which, b * P + j, s_pos[which * P + j]);
       }
     }
   }
@@ -463,8 +460,8 @@ struct SegShape {
 };
 
 template <int V, int NW, bool NOISE>
-__global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __restrict__ beps, int nstrip,
-                                                        uint32_t wait_limit) {
+__global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __restrict__ beps,
+                                                        uint32_t wait_limit, int par) {
   using Sh = SegShape<V, NW, NOISE>;
   constexpr int SEG = Sh::SEG;
   constexpr int NR = Sh::NR;
@@ -493,7 +490,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   // Everything read before pdl_wait() was written two or more kernels back
   // (the previous update and decision kernels); only the batch eps rows come
   // from the denoiser just before.
-  const Traj tr = d.traj[b];
+  const Traj tr = d.traj[par * d.B + b];
   const int n_miss = d.ctl->n_miss;
   if (tr.p == 0) return;
   const int t = tr.t, p = tr.p, e = tr.e;
@@ -654,7 +651,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   }
   __syncthreads();
   // strip partials: one thread per (quantity, position) sums its row of lanes
-  const int64_t pbase = (int64_t)b * P * nstrip + strip;
+  // and adds it into the iteration's sums
   for (int r = tid; r < 2 * p; r += NW * 32) {
     const int which = r / p, j = r % p;
     const float* row = s_red + (size_t)(which * P + j) * 33;
@@ -666,7 +663,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
       acc[2] += row[c + 2];
       acc[3] += row[c + 3];
     }
-    (which == 0 ? d.part_err : d.part_del)[pbase + (int64_t)j * nstrip] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+    red_add(d, par, which, b * P + j, (acc[0] + acc[1]) + (acc[2] + acc[3]));
   }
   // after a timeout, let this warp's copies land before the CTA exits
   if (my_fail && lane == 0 && j0 < j1) mbar_wait_bounded(&bar[warp], 0, kDrainLimit);
@@ -680,7 +677,7 @@ bool seg_fits(const Dev& d) {
 }
 
 template <int V, int NW, bool NOISE = false>
-cudaError_t launch_seg(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+cudaError_t launch_seg(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = SegShape<V, NW, NOISE>;
   const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
   const size_t smem = Sh::smem_bytes(d.P);
@@ -694,8 +691,7 @@ cudaError_t launch_seg(const Dev& d, const float* beps, cudaStream_t st, int* nc
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) configured[dev] = smem;
   }
-  *nchunk_out = nstrip;
-  return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, nstrip, d.wait_limit);
+  return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, d.wait_limit, par);
 }
 
 // ---------------------------------------------------------------------------
@@ -721,7 +717,7 @@ struct RegShape {
 };
 
 template <int V, int NW, int LMAX, bool NOISE>
-__global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* __restrict__ beps, int nstrip) {
+__global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* __restrict__ beps, int par) {
   using Sh = RegShape<V, NW>;
   constexpr int SEG = Sh::SEG;
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -737,7 +733,7 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
   // (the previous update and decision kernels); only the batch eps rows come
   // from the denoiser just before. The ranks do not depend on the window, so
   // they are fetched together with it.
-  const Traj tr = d.traj[b];
+  const Traj tr = d.traj[par * d.B + b];
   const int n_miss = d.ctl->n_miss;
   for (int j = tid; j < P; j += NW * 32) {
     int r = d.rank[b * P + j];
@@ -882,7 +878,7 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
   }
   __syncthreads();
   // strip partials: one thread per (quantity, position) sums its row of lanes
-  const int64_t pbase = (int64_t)b * P * nstrip + strip;
+  // and adds it into the iteration's sums
   for (int r = tid; r < 2 * p; r += NW * 32) {
     const int which = r / p, j = r % p;
     const float* row = s_red + (size_t)(which * P + j) * 33;
@@ -894,12 +890,12 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
       acc[2] += row[c + 2];
       acc[3] += row[c + 3];
     }
-    (which == 0 ? d.part_err : d.part_del)[pbase + (int64_t)j * nstrip] = (acc[0] + acc[1]) + (acc[2] + acc[3]);
+    red_add(d, par, which, b * P + j, (acc[0] + acc[1]) + (acc[2] + acc[3]));
   }
 }
 
 template <int V, int NW, int LMAX, bool NOISE>
-cudaError_t launch_reg(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+cudaError_t launch_reg(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = RegShape<V, NW>;
   const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
   const size_t smem = Sh::smem_bytes(d.P);
@@ -913,8 +909,7 @@ cudaError_t launch_reg(const Dev& d, const float* beps, cudaStream_t st, int* nc
     if (e != cudaSuccess) return e;
     if (dev >= 0 && dev < 64) configured[dev] = smem;
   }
-  *nchunk_out = nstrip;
-  return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, nstrip);
+  return launch_ex(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, d, beps, par);
 }
 
 // Positions per warp that the register-resident form holds for a window of P
@@ -929,15 +924,15 @@ int reg_lmax(const Dev& d) {
   return 0;
 }
 
-cudaError_t launch_reg_auto(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+cudaError_t launch_reg_auto(const Dev& d, const float* beps, int par, cudaStream_t st) {
   const int lm = reg_lmax(d);
   if (d.noise) {
-    if (lm == 4) return launch_reg<4, 8, 4, true>(d, beps, st, nchunk_out);
-    return launch_reg<4, 8, kRegMaxLNoise, true>(d, beps, st, nchunk_out);
+    if (lm == 4) return launch_reg<4, 8, 4, true>(d, beps, par, st);
+    return launch_reg<4, 8, kRegMaxLNoise, true>(d, beps, par, st);
   }
-  if (lm == 4) return launch_reg<4, 8, 4, false>(d, beps, st, nchunk_out);
-  if (lm == 8) return launch_reg<4, 8, 8, false>(d, beps, st, nchunk_out);
-  return launch_reg<4, 8, kRegMaxL, false>(d, beps, st, nchunk_out);
+  if (lm == 4) return launch_reg<4, 8, 4, false>(d, beps, par, st);
+  if (lm == 8) return launch_reg<4, 8, 8, false>(d, beps, par, st);
+  return launch_reg<4, 8, kRegMaxL, false>(d, beps, par, st);
 }
 
 // Shared memory budget per CTA for the tile buffers: enough for the whole
@@ -945,7 +940,7 @@ cudaError_t launch_reg_auto(const Dev& d, const float* beps, cudaStream_t st, in
 constexpr size_t kSmemBudget = 112 * 1024;
 
 template <int V, int NW, int S, bool CLUSTER, bool WAIT_ALL>
-cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* nchunk_out) {
+cudaError_t launch_tile(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = TileShape<V, NW, S>;
   const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
   const int ntile_max = (d.P + Sh::TW - 1) / Sh::TW;
@@ -966,9 +961,8 @@ cudaError_t launch_tile(const Dev& d, const float* beps, cudaStream_t st, int* n
     if (dev >= 0 && dev < 64) configured[dev] = smem;
   }
   const int gx = CLUSTER ? (nstrip + kCluster - 1) / kCluster * kCluster : nstrip;
-  *nchunk_out = CLUSTER ? gx / kCluster : nstrip;  // partials per position
   return launch_ex(kern, dim3(gx, d.B, 1), dim3(NW * 32), smem, st, CLUSTER ? kCluster : 0, d, beps, nstrip,
-                   nbuf, d.wait_limit);
+                   nbuf, d.wait_limit, par);
 }
 
 }  // namespace
@@ -1003,38 +997,45 @@ bool prefer_wide_strips(const Dev& d) {
   return per_sm >= 2 || grid <= nsm[dev];
 }
 
-cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st, int* nchunk_out) {
-  if (d.bulk_cfg == 12 && reg_lmax(d)) return launch_reg_auto(d, batch_eps, st, nchunk_out);
-  if (d.noise) {  // stochastic steps: the segment form with the draws staged (update_bulk_supported)
-    if (prefer_wide_strips<true>(d)) return launch_seg<4, 8, true>(d, batch_eps, st, nchunk_out);
-    return launch_seg<2, 8, true>(d, batch_eps, st, nchunk_out);
+cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, int par, cudaStream_t st) {
+  if (d.bulk_cfg == 12 && reg_lmax(d)) return launch_reg_auto(d, batch_eps, par, st);
+  if (d.noise) {  // stochastic steps: the segment forms with the draws (update_bulk_supported)
+    if (prefer_wide_strips<true>(d)) {
+      if (d.bulk_cfg == 0 && reg_lmax(d)) return launch_reg_auto(d, batch_eps, par, st);
+      return launch_seg<4, 8, true>(d, batch_eps, par, st);
+    }
+    return launch_seg<2, 8, true>(d, batch_eps, par, st);
   }
   switch (d.bulk_cfg) {
-    case 0:  // whole window in shared memory when it fits, else the tiled pipeline
-      if (prefer_wide_strips<false>(d)) return launch_seg<4, 8>(d, batch_eps, st, nchunk_out);
-      if (seg_fits<2, 8>(d)) return launch_seg<2, 8>(d, batch_eps, st, nchunk_out);
-      return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 1: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 2: return launch_tile<2, 8, 4, true, true>(d, batch_eps, st, nchunk_out);
-    case 3: return launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
-    case 4: return seg_fits<2, 8>(d) ? launch_seg<2, 8>(d, batch_eps, st, nchunk_out)
-                                     : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 5: return seg_fits<2, 16>(d) ? launch_seg<2, 16>(d, batch_eps, st, nchunk_out)
-                                      : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 6: return seg_fits<1, 8>(d) ? launch_seg<1, 8>(d, batch_eps, st, nchunk_out)
-                                     : launch_tile<1, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 7: return seg_fits<1, 16>(d) ? launch_seg<1, 16>(d, batch_eps, st, nchunk_out)
-                                      : launch_tile<1, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 8: return seg_fits<2, 4>(d) ? launch_seg<2, 4>(d, batch_eps, st, nchunk_out)
-                                     : launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
-    case 9: return launch_tile<2, 8, 2, false, true>(d, batch_eps, st, nchunk_out);
-    case 10: return seg_fits<4, 8>(d) ? launch_seg<4, 8>(d, batch_eps, st, nchunk_out)
-                                      : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    case 11: return seg_fits<4, 4>(d) ? launch_seg<4, 4>(d, batch_eps, st, nchunk_out)
-                                      : launch_tile<2, 4, 8, false, true>(d, batch_eps, st, nchunk_out);
-    case 12: return reg_lmax(d) ? launch_reg_auto(d, batch_eps, st, nchunk_out)
-                                : launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
-    default: return launch_tile<2, 8, 4, false, true>(d, batch_eps, st, nchunk_out);
+    case 0:  // four columns per lane in registers (or staged) when the grid suits
+             // them, else the staged window in shared memory, else the tiled pipeline
+      if (prefer_wide_strips<false>(d)) {
+        if (reg_lmax(d)) return launch_reg_auto(d, batch_eps, par, st);
+        return launch_seg<4, 8>(d, batch_eps, par, st);
+      }
+      if (seg_fits<2, 8>(d)) return launch_seg<2, 8>(d, batch_eps, par, st);
+      return launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
+    case 1: return launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
+    case 2: return launch_tile<2, 8, 4, true, true>(d, batch_eps, par, st);
+    case 3: return launch_tile<2, 4, 8, false, true>(d, batch_eps, par, st);
+    case 4: return seg_fits<2, 8>(d) ? launch_seg<2, 8>(d, batch_eps, par, st)
+                                     : launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
+    case 5: return seg_fits<2, 16>(d) ? launch_seg<2, 16>(d, batch_eps, par, st)
+                                      : launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
+    case 6: return seg_fits<1, 8>(d) ? launch_seg<1, 8>(d, batch_eps, par, st)
+                                     : launch_tile<1, 8, 4, false, true>(d, batch_eps, par, st);
+    case 7: return seg_fits<1, 16>(d) ? launch_seg<1, 16>(d, batch_eps, par, st)
+                                      : launch_tile<1, 8, 4, false, true>(d, batch_eps, par, st);
+    case 8: return seg_fits<2, 4>(d) ? launch_seg<2, 4>(d, batch_eps, par, st)
+                                     : launch_tile<2, 4, 8, false, true>(d, batch_eps, par, st);
+    case 9: return launch_tile<2, 8, 2, false, true>(d, batch_eps, par, st);
+    case 10: return seg_fits<4, 8>(d) ? launch_seg<4, 8>(d, batch_eps, par, st)
+                                      : launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
+    case 11: return seg_fits<4, 4>(d) ? launch_seg<4, 4>(d, batch_eps, par, st)
+                                      : launch_tile<2, 4, 8, false, true>(d, batch_eps, par, st);
+    case 12: return reg_lmax(d) ? launch_reg_auto(d, batch_eps, par, st)
+                                : launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
+    default: return launch_tile<2, 8, 4, false, true>(d, batch_eps, par, st);
   }
 }
 

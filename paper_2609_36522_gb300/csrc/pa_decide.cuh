@@ -1,44 +1,44 @@
-// The serial part of one Picard iteration's decision (a10, a2, a3), run by a
-// single CTA once every per-position reduction is finished (the last CTA of
-// the decision kernel in k_solver.cu).
+// The decision that ends one Picard iteration (a10, a2, a3), as a CTA-wide
+// device function. Every CTA of the planning kernel runs it on the same
+// inputs and reaches the same plan; one of them (publish) writes the plan to
+// memory, the others keep what they need in shared memory (the batch row
+// they gather).
 #pragma once
 
 #include "pa_internal.h"
 
 namespace pa {
 
-// red_e[b*P + j]: Eq. 2 error of window position j of trajectory b (already
-// divided by D); red_d[b*P + j]: Eq. 4 distance of timestep t+j+1 (divided by
-// D). Only positions j < p_b are read. With NT threads the CTA
-//  1. per trajectory: stride = min(p, 1 + #leading err_j <= tol) (warp
-//     ballots), advances t, shrinks p = min(P, T - t), sets the frontier
-//     e = old t + p, done at t = T, and writes the iteration log;
-//  2. plans the next iteration: a timestep of the new window with a cache
-//     entry (i < e) hits iff delta < tau_cache (strict, Eq. 5), everything else
-//     misses; misses are compacted trajectory-major into miss_bt with a
-//     block-wide prefix sum, and rank[b][j] records each miss's batch row;
-//  3. updates the counters (n_miss, n_active, iter, nfe, hits).
 // Shared state of one decision (static shared memory of the calling kernel).
 struct DecideShared {
   int t[kMaxBatch], p[kMaxBatch], e[kMaxBatch];
-  int tn[kMaxBatch], pn[kMaxBatch], m[kMaxBatch], h1[kMaxBatch];
+  int tn[kMaxBatch], pn[kMaxBatch], en[kMaxBatch], m[kMaxBatch], h1[kMaxBatch];
   int om[kMaxBatch], oh1[kMaxBatch];
   int warp_tot[32];
   int total, active, iter;
+  long long nfe, hits;
+  int target_b, target_i;  // the miss of the requested batch row, if any
 };
 
-// The trajectories and counters a decision starts from. They were written by
-// the previous decision, several kernels back, so a kernel may read them
-// before its dependency wait. No barrier.
+// The plan of iteration k (copy par = k mod 2). It was written by the previous
+// decision, several kernels back, so it may be read before the dependency
+// wait. No barrier.
 template <int NT>
-__device__ void decide_load(const Dev& d, DecideShared& sh) {
+__device__ void decide_load(const Dev& d, DecideShared& sh, int par) {
   const int tid = threadIdx.x;
   if (tid == 0) {
-    sh.active = d.ctl->n_active;
-    sh.iter = d.ctl->iter;
+    const PlanCtr c = d.pc[par];
+    sh.active = c.n_active;
+    sh.iter = c.iter;
+    sh.nfe = c.nfe;
+    sh.hits = c.hits;
+    sh.total = 0;
+    sh.target_b = -1;
+    sh.target_i = 0;
   }
+  const Traj* tr0 = d.traj + par * d.B;
   for (int b = tid; b < d.B; b += NT) {
-    const Traj tr = d.traj[b];
+    const Traj tr = tr0[b];
     sh.t[b] = tr.t; sh.p[b] = tr.p; sh.e[b] = tr.e;
     sh.om[b] = tr.m; sh.oh1[b] = tr.h1;
     sh.m[b] = 0;
@@ -46,9 +46,23 @@ __device__ void decide_load(const Dev& d, DecideShared& sh) {
   }
 }
 
-// Steps 1-3 above on the state decide_load staged; starts with a barrier.
-template <int NT>
-__device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, const float* red_d) {
+// red_e[b*P + j]: Eq. 2 error of window position j of trajectory b (divided
+// by D); red_d[b*P + j]: Eq. 4 distance of timestep t+j+1 (divided by D).
+// Only positions j < p_b are read. With NT threads the CTA
+//  1. per trajectory: stride = min(p, 1 + #leading err_j <= tol) (warp
+//     ballots), advances t, shrinks p = min(P, T - t), sets the frontier
+//     e = old t + p, done at t = T, and (publish) writes the iteration log;
+//  2. plans the next iteration: a timestep of the new window with a cache
+//     entry (i < e) hits iff delta < tau_cache (strict, Eq. 5), everything else
+//     misses; misses are compacted trajectory-major with a block-wide prefix
+//     sum; publish writes rank[b][j] (each miss's batch row) and miss_bt, and
+//     every CTA notes the miss of batch row `target` (target_b, target_i);
+//  3. publish writes the new trajectories and counters to copy par ^ 1 and
+//     the host-visible counters.
+// When no trajectory is active the plan is carried over unchanged. Starts
+// with a barrier (after decide_load) and ends with one.
+template <int NT, typename Red>
+__device__ void decide_run(const Dev& d, DecideShared& sh, const Red& red, int par, bool publish, int target) {
   int* s_t = sh.t; int* s_p = sh.p; int* s_e = sh.e;
   int* s_tn = sh.tn; int* s_pn = sh.pn; int* s_m = sh.m; int* s_h1 = sh.h1;
   int* s_om = sh.om; int* s_oh1 = sh.oh1; int* s_warp = sh.warp_tot;
@@ -56,9 +70,18 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, c
   static_assert(nwarps <= 32, "one warp scans the warp totals");
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int B = d.B, P = d.P, T = d.T;
+  Traj* out_traj = d.traj + (par ^ 1) * B;
   __syncthreads();
-  const int s_active = sh.active;
-  if (s_active == 0) return;  // finished: iterating further is a no-op
+  if (sh.active == 0) {  // finished: iterating further changes nothing
+    if (publish) {
+      const Traj* in_traj = d.traj + par * B;
+      for (int b = tid; b < B; b += NT) out_traj[b] = in_traj[b];
+      if (tid == 0) d.pc[par ^ 1] = d.pc[par];
+    }
+    for (int b = tid; b < B; b += NT) sh.en[b] = s_e[b];
+    __syncthreads();
+    return;
+  }
   const int iter = sh.iter;
 
   // 1. window advance, one warp per trajectory
@@ -67,16 +90,18 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, c
     if (p == 0) {
       if (lane == 0) {
         s_tn[b] = t; s_pn[b] = 0;
-        int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
-        for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
-        lg[0] = t;
+        if (publish) {
+          int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+          for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
+          lg[0] = t;
+        }
       }
       continue;
     }
     int lead = p;
     for (int j0 = 0; j0 < p; j0 += 32) {
       const int j = j0 + lane;
-      const bool fail = (j < p) && !((double)red_e[b * P + j] <= d.tol);
+      const bool fail = (j < p) && !(red.err(b * P + j) <= d.tol);
       const unsigned m = __ballot_sync(0xffffffffu, fail);
       if (m) {
         lead = j0 + __ffs(m) - 1;
@@ -88,9 +113,11 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, c
       const int tn = t + stride;
       s_tn[b] = tn;
       s_pn[b] = min(P, T - tn);
-      int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
-      lg[0] = t; lg[1] = p; lg[2] = s_om[b]; lg[3] = stride;
-      lg[4] = s_e[b]; lg[5] = s_oh1[b]; lg[6] = 0; lg[7] = 0;
+      if (publish) {
+        int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+        lg[0] = t; lg[1] = p; lg[2] = s_om[b]; lg[3] = stride;
+        lg[4] = s_e[b]; lg[5] = s_oh1[b]; lg[6] = 0; lg[7] = 0;
+      }
     }
   }
   __syncthreads();
@@ -106,7 +133,7 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, c
     const int en = s_t[b] + s_p[b];  // new frontier
     if (i >= en) return 1;           // first entry
     const int jo = i - s_t[b] - 1;   // delta of timestep i was computed at old position jo
-    return ((double)red_d[b * P + jo] < d.cache_thresh) ? 0 : 1;
+    return (red.del(b * P + jo) < d.cache_thresh) ? 0 : 1;
   };
   int cnt = 0;
   for (int q = q0; q < q1; ++q) cnt += is_miss(q);
@@ -131,51 +158,67 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const float* red_e, c
   }
   __syncthreads();
   int r = s_warp[warp] + incl - cnt;
-  for (int q = q0; q < q1; ++q) {
-    const int b = q / P, j = q % P;
-    if (is_miss(q)) {
-      d.rank[q] = r;
-      d.miss_bt[2 * r] = b;
-      d.miss_bt[2 * r + 1] = s_tn[b] + j;
-      atomicAdd(&s_m[b], 1);
-      ++r;
-    } else {
-      d.rank[q] = -1;
-      if (j >= 1 && j < s_pn[b]) atomicAdd(&s_h1[b], 1);
+  if (target >= r && target < r + cnt) {  // the requested batch row is one of this thread's misses
+    int rr = r;
+    for (int q = q0; q < q1; ++q) {
+      if (!is_miss(q)) continue;
+      if (rr == target) {
+        sh.target_b = q / P;
+        sh.target_i = s_tn[q / P] + q % P;
+      }
+      ++rr;
     }
   }
+  if (publish) {
+    for (int q = q0; q < q1; ++q) {
+      const int b = q / P, j = q % P;
+      if (is_miss(q)) {
+        d.rank[q] = r;
+        d.miss_bt[2 * r] = b;
+        d.miss_bt[2 * r + 1] = s_tn[b] + j;
+        atomicAdd(&s_m[b], 1);
+        ++r;
+      } else {
+        d.rank[q] = -1;
+        if (j >= 1 && j < s_pn[b]) atomicAdd(&s_h1[b], 1);
+      }
+    }
+  }
+  for (int b = tid; b < B; b += NT) sh.en[b] = (s_p[b] > 0) ? s_t[b] + s_p[b] : s_e[b];
   __syncthreads();
 
-  // 3. trajectories and counters
-  int pts = 0;
-  for (int b = 0; b < B; ++b) pts += s_pn[b];
-  for (int b = tid; b < B; b += NT) {
-    Traj tr{};
-    tr.t = s_tn[b];
-    tr.p = s_pn[b];
-    tr.e = (s_p[b] > 0) ? s_t[b] + s_p[b] : s_e[b];
-    tr.done = (s_pn[b] == 0);
-    tr.m = s_m[b];
-    tr.h1 = s_h1[b];
-    if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
-    d.traj[b] = tr;
+  // 3. trajectories and counters of the next iteration
+  if (publish) {
+    int pts = 0;
+    for (int b = 0; b < B; ++b) pts += s_pn[b];
+    for (int b = tid; b < B; b += NT) {
+      Traj tr{};
+      tr.t = s_tn[b];
+      tr.p = s_pn[b];
+      tr.e = sh.en[b];
+      tr.done = (s_pn[b] == 0);
+      tr.m = s_m[b];
+      tr.h1 = s_h1[b];
+      if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
+      out_traj[b] = tr;
+    }
+    if (tid == 0) {
+      int act = 0;
+      for (int b = 0; b < B; ++b) act += (s_pn[b] > 0);
+      const int n = sh.total;
+      PlanCtr c;
+      c.n_active = act;
+      c.iter = iter + 1;
+      c.nfe = sh.nfe + n;
+      c.hits = sh.hits + (pts - n);
+      d.pc[par ^ 1] = c;
+      d.ctl->n_miss = n;
+      d.ctl->n_active = act;
+      d.ctl->iter = c.iter;
+      d.ctl->nfe = c.nfe;
+      d.ctl->hits = c.hits;
+    }
   }
-  if (tid == 0) {
-    int act = 0;
-    for (int b = 0; b < B; ++b) act += (s_pn[b] > 0);
-    const int n = sh.total;
-    d.ctl->n_miss = n;
-    d.ctl->n_active = act;
-    d.ctl->iter = iter + 1;
-    d.ctl->nfe += n;
-    d.ctl->hits += pts - n;
-  }
-}
-
-template <int NT>
-__device__ void decide_plan(const Dev& d, DecideShared& sh, const float* red_e, const float* red_d) {
-  decide_load<NT>(d, sh);
-  decide_run<NT>(d, sh, red_e, red_d);
 }
 
 }  // namespace pa

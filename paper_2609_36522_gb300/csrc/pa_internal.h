@@ -10,7 +10,6 @@ namespace pa {
 
 constexpr int kMaxWindow = 1024;
 constexpr int kMaxBatch = 64;
-constexpr int kMinChunk = 32;       // narrowest column chunk of any update kernel
 constexpr size_t kAlign = 256;
 constexpr int kBulkConfigs = 13;    // launch shapes of the bulk-copy update kernel
 
@@ -34,6 +33,8 @@ struct Traj {
 };
 constexpr int kLogFields = 8;  // iteration log entry: t, p, misses, stride, e, h1, 0, 0
 
+// Counters read by the host (one copy, written by whichever kernel publishes
+// a plan) and by the denoiser (n_miss, through its device pointer).
 struct Ctl {
   int32_t n_miss;     // misses planned for the next iteration (Eq. 5)
   int32_t n_active;   // trajectories with t < T
@@ -41,14 +42,20 @@ struct Ctl {
   int32_t status;     // kDev* code
   long long nfe;
   long long hits;
-  uint32_t ticket;    // CTAs of the decision kernel that finished their reductions
-  int32_t pad;
+};
+
+// The counters a decision starts from. Kept in two copies, like the
+// trajectories: the plan of iteration k lives in copy k mod 2, so the kernel
+// that decides iteration k+1 reads copy k mod 2 in all of its CTAs while one
+// of them writes copy (k+1) mod 2.
+struct PlanCtr {
+  int32_t n_active, iter;
+  long long nfe, hits;
 };
 
 struct Layout {
-  size_t X, Xhat, Ehat, batch_x, coef, traj, ctl, rank, miss_bt;
-  size_t part_err, part_del, red_err, red_del, iter_log, total;
-  int64_t part_cap;   // floats per partial array
+  size_t X, Xhat, Ehat, batch_x, coef, traj, pc, ctl, rank, miss_bt;
+  size_t acc, red_err, red_del, iter_log, total;
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -63,13 +70,12 @@ inline Layout make_layout(int T, int P, int64_t D, int B) {
   L.Ehat = take((size_t)B * P * row);             // cache outputs, slot = i mod P
   L.batch_x = take((size_t)B * P * row);          // gathered misses
   L.coef = take((size_t)3 * T * sizeof(float));   // (c_i - 1, e_i, sigma_i)
-  L.traj = take((size_t)B * sizeof(Traj));
+  L.traj = take((size_t)2 * B * sizeof(Traj));     // two copies (plan parity)
+  L.pc = take(2 * sizeof(PlanCtr));
   L.ctl = take(sizeof(Ctl));
   L.rank = take((size_t)B * P * sizeof(int32_t));
   L.miss_bt = take((size_t)B * P * 2 * sizeof(int32_t));
-  L.part_cap = (int64_t)B * P * ((D + kMinChunk - 1) / kMinChunk);
-  L.part_err = take((size_t)L.part_cap * sizeof(float));
-  L.part_del = take((size_t)L.part_cap * sizeof(float));
+  L.acc = take((size_t)2 * 2 * B * P * sizeof(double));  // [set][err, dist][B][P]
   L.red_err = take((size_t)B * P * sizeof(float));
   L.red_del = take((size_t)B * P * sizeof(float));
   L.iter_log = take((size_t)(T + 1) * B * kLogFields * sizeof(int32_t));
@@ -87,18 +93,18 @@ struct Dev {
   const float* ecoef; // e_i
   const float* sigma; // sigma_i of stochastic steps (0 for eta = 0)
   const float* noise; // [B][T][D] draws z_i of stochastic steps, caller-owned; NULL for eta = 0
-  Traj* traj;
+  Traj* traj;         // [2][B]: copy k mod 2 holds the plan of iteration k
+  PlanCtr* pc;        // [2]
   Ctl* ctl;
   int32_t* rank;      // [B][P] rank of window position j among the misses, -1 = hit
   int32_t* miss_bt;   // [B*P][2]
-  float* part_err;    // [B][P][nchunk]
-  float* part_del;
-  float* red_err;     // [B][P]
+  double* acc;        // [2][2][B][P]: sums of Eq. 2 and Eq. 4 terms; set k mod 2 in iteration k
+  float* red_err;     // [B][P] the last decision's reductions (divided by D), for the host
   float* red_del;
   int32_t* iter_log;  // [T+1][B][kLogFields]
   int T, P, B;
   int64_t D;
-  double tol, cache_thresh;   // compared against fp32 reductions promoted to double
+  double tol, cache_thresh;   // compared against the fp64 sums divided by D
   int bulk_cfg;               // launch shape of the bulk-copy update kernel
   uint32_t wait_limit;        // polls before an mbarrier wait counts as timed out
 };
@@ -146,15 +152,24 @@ cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem
   return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
 }
 
-// Kernel launchers (k_solver.cu). Each returns the launch error.
+// One CTA's share of the Eq. 2 error (which = 0) or Eq. 4 distance (which =
+// 1) of window position q = b*P + j, added into the accumulator set of the
+// iteration's parity. fp64 sums of fp32 CTA partials: the rounding of the
+// order in which CTAs arrive is far below the fp32 partials' own.
+__device__ __forceinline__ void red_add(const Dev& d, int par, int which, int q, float v) {
+  atomicAdd(d.acc + ((size_t)(par * 2 + which) * d.B * d.P + q), (double)v);
+}
+
+// Kernel launchers (k_solver.cu). Each returns the launch error. par = k mod 2
+// for iteration k: the copy of the plan the kernel reads (and the accumulator
+// set the update kernels add into).
 cudaError_t launch_init_plan(const Dev& d, cudaStream_t st);
-cudaError_t launch_gather(const Dev& d, cudaStream_t st);
-cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, cudaStream_t st,
-                                int* nchunk_out);
-cudaError_t launch_decide(const Dev& d, int nchunk, cudaStream_t st);
+cudaError_t launch_gather(const Dev& d, int par, cudaStream_t st);
+cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, int par, cudaStream_t st);
+// the decision after iteration k (par = k mod 2) and the gather of iteration k+1
+cudaError_t launch_plan(const Dev& d, int par, cudaStream_t st, int* launches);
 // k_update_bulk.cu
-cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, cudaStream_t st,
-                               int* nchunk_out);
+cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, int par, cudaStream_t st);
 bool update_bulk_supported(const Dev& d, const float* batch_eps);
 
 }  // namespace pa

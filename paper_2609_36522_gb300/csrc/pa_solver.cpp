@@ -42,7 +42,7 @@ struct pa_solver {
   St state;
   int update_kind;   // requested: 0 plain, 1 bulk pipeline
   int last_kind;     // kernel the last pa_submit_eps actually launched (-1: none yet)
-  int last_nchunk;
+  int64_t k;         // pa_submit_eps calls since pa_init: the plan of iteration k is copy k mod 2
   int64_t launches;
   pa::Ctl* host_ctl; // pinned mirror of the device Ctl
   std::vector<double> alphas;  // the schedule, kept for pa_set_noise
@@ -187,7 +187,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   s->st = static_cast<cudaStream_t>(stream);
   s->state = St::Created;
   s->launches = 0;
-  s->last_nchunk = 0;
+  s->k = 0;
   s->last_kind = -1;
   char* w = s->ws;
   pa::Dev& d = s->d;
@@ -203,11 +203,11 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   s->alphas.assign(alphas_cumprod, alphas_cumprod + T + 1);
   s->eta = 0.0;
   d.traj = reinterpret_cast<pa::Traj*>(w + L.traj);
+  d.pc = reinterpret_cast<pa::PlanCtr*>(w + L.pc);
   d.ctl = reinterpret_cast<pa::Ctl*>(w + L.ctl);
   d.rank = reinterpret_cast<int32_t*>(w + L.rank);
   d.miss_bt = reinterpret_cast<int32_t*>(w + L.miss_bt);
-  d.part_err = reinterpret_cast<float*>(w + L.part_err);
-  d.part_del = reinterpret_cast<float*>(w + L.part_del);
+  d.acc = reinterpret_cast<double*>(w + L.acc);
   d.red_err = reinterpret_cast<float*>(w + L.red_err);
   d.red_del = reinterpret_cast<float*>(w + L.red_del);
   d.iter_log = reinterpret_cast<int32_t*>(w + L.iter_log);
@@ -262,9 +262,15 @@ pa_status pa_init(pa_solver* s, const float* x_init) {
                                     (size_t)d.D * sizeof(float), (size_t)d.D * sizeof(float), d.B,
                                     cudaMemcpyDefault, s->st);
   if (e != cudaSuccess) return cuda_fail("pa_init: copy x_init", e);
+  // both accumulator sets of the reductions start at zero
+  e = cudaMemsetAsync(d.acc, 0, (size_t)2 * 2 * d.B * d.P * sizeof(double), s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_init: clear sums", e);
+  // the first plan (every timestep a first entry) and its batch
   e = pa::launch_init_plan(d, s->st);
-  s->launches++;
+  if (e == cudaSuccess) e = pa::launch_gather(d, 0, s->st);
+  s->launches += 2;
   if (e != cudaSuccess) return cuda_fail("pa_init: launch", e);
+  s->k = 0;
   s->state = St::Ready;
   return PA_OK;
 }
@@ -273,9 +279,7 @@ pa_status pa_step_async(pa_solver* s, const float** batch_x_dev, const int32_t**
                         const int32_t** n_miss_dev) {
   if (!s) return arg_fail("pa_step_async: solver is NULL");
   if (s->state != St::Ready) return state_fail("pa_step_async");
-  const cudaError_t e = pa::launch_gather(s->d, s->st);
-  s->launches++;
-  if (e != cudaSuccess) return cuda_fail("pa_step_async: gather", e);
+  // the batch was gathered by the kernel that planned this iteration
   if (batch_x_dev) *batch_x_dev = s->d.batch_x;
   if (miss_bt_dev) *miss_bt_dev = s->d.miss_bt;
   if (n_miss_dev) *n_miss_dev = &s->d.ctl->n_miss;
@@ -310,7 +314,7 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
   if (!s) return arg_fail("pa_submit_eps: solver is NULL");
   if (s->state != St::Stepped) return state_fail("pa_submit_eps");
   if (!batch_eps_dev) return arg_fail("pa_submit_eps: batch_eps is NULL");
-  int nchunk = 0;
+  const int par = (int)(s->k & 1);
   cudaError_t e = cudaSuccess;
   if (s->timing) {
     if (s->ev_next * 2 + 2 > s->ev.size()) {
@@ -324,10 +328,10 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
   }
   if (s->update_kind == 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
-    e = pa::launch_update_bulk(s->d, batch_eps_dev, s->st, &nchunk);
+    e = pa::launch_update_bulk(s->d, batch_eps_dev, par, s->st);
     s->last_kind = 1;
   } else {
-    e = pa::launch_update_plain(s->d, batch_eps_dev, s->st, &nchunk);
+    e = pa::launch_update_plain(s->d, batch_eps_dev, par, s->st);
     s->last_kind = 0;
   }
   s->launches++;
@@ -337,10 +341,11 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
     s->ev_next++;
   }
-  s->last_nchunk = nchunk;
-  e = pa::launch_decide(s->d, nchunk, s->st);
-  s->launches++;
-  if (e != cudaSuccess) return cuda_fail("pa_submit_eps: decide", e);
+  int nl = 0;
+  e = pa::launch_plan(s->d, par, s->st, &nl);
+  s->launches += nl;
+  if (e != cudaSuccess) return cuda_fail("pa_submit_eps: plan", e);
+  s->k++;
   s->state = St::Ready;
   return PA_OK;
 }
