@@ -295,7 +295,9 @@ __global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
       nxt[npair + q] = 0.0;
     }
   }
-  decide_run<kPlanThreads>(d, ds, RedShared{s_e, s_d}, par, publish, (int)blockIdx.y);
+  __syncthreads();  // the sums and decide_load's state are staged
+  decide_warp(d, ds, RedShared{s_e, s_d}, par, publish, (int)blockIdx.y);
+  __syncthreads();  // the plan (batch row of this CTA) is known
   if ((int)blockIdx.y < ds.total && ds.target_b >= 0) {
     const int b = ds.target_b;
     copy_row<VEC>(d, b, min(ds.target_i, ds.en[b]), blockIdx.y);

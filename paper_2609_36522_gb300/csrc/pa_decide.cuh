@@ -221,4 +221,137 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const Red& red, int p
   }
 }
 
+// The same decision taken by one warp (warp 0 of the calling CTA; the other
+// warps skip it), for the planning kernel in which every CTA decides: with
+// B*P small the ballots and population counts of one warp replace the block
+// scan and its barriers. Reads what decide_load staged (after a barrier that
+// the caller provides) and gives the same plan, ranks and counters as
+// decide_run. The caller synchronises the CTA afterwards.
+template <typename Red>
+__device__ void decide_warp(const Dev& d, DecideShared& sh, const Red& red, int par, bool publish, int target) {
+  if (threadIdx.x >= 32) return;
+  const int lane = threadIdx.x;
+  const int B = d.B, P = d.P, T = d.T;
+  Traj* out_traj = d.traj + (par ^ 1) * B;
+  if (sh.active == 0) {  // finished: the plan carries over
+    if (publish) {
+      const Traj* in_traj = d.traj + par * B;
+      for (int b = lane; b < B; b += 32) out_traj[b] = in_traj[b];
+      if (lane == 0) d.pc[par ^ 1] = d.pc[par];
+    }
+    for (int b = lane; b < B; b += 32) sh.en[b] = sh.e[b];
+    __syncwarp();
+    return;
+  }
+  const int iter = sh.iter;
+  // 1. window advance
+  for (int b = 0; b < B; ++b) {
+    const int t = sh.t[b], p = sh.p[b];
+    int stride = 0;
+    if (p > 0) {
+      int lead = p;
+      for (int j0 = 0; j0 < p; j0 += 32) {
+        const int j = j0 + lane;
+        const unsigned m = __ballot_sync(0xffffffffu, (j < p) && !(red.err(b * P + j) <= d.tol));
+        if (m) {
+          lead = j0 + __ffs(m) - 1;
+          break;
+        }
+      }
+      stride = min(p, 1 + lead);
+    }
+    if (lane == 0) {
+      const int tn = t + stride;
+      sh.tn[b] = tn;
+      sh.pn[b] = p > 0 ? min(P, T - tn) : 0;
+      sh.en[b] = p > 0 ? t + p : sh.e[b];
+      if (publish) {
+        int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
+        if (p > 0) {
+          lg[0] = t; lg[1] = p; lg[2] = sh.om[b]; lg[3] = stride;
+          lg[4] = sh.e[b]; lg[5] = sh.oh1[b]; lg[6] = 0; lg[7] = 0;
+        } else {
+          for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
+          lg[0] = t;
+        }
+      }
+    }
+  }
+  __syncwarp();
+  // 2. hit/miss plan of the next iteration, compacted 32 positions at a time
+  const int N = B * P;
+  int base = 0;
+  int pts = 0;
+  for (int q0 = 0; q0 < N; q0 += 32) {
+    const int q = q0 + lane;
+    int miss = 0, inwin = 0;
+    int b = 0, j = 0;
+    if (q < N) {
+      b = q / P;
+      j = q % P;
+      if (j < sh.pn[b]) {
+        inwin = 1;
+        const int i = sh.tn[b] + j;
+        const int en = sh.t[b] + sh.p[b];  // new frontier
+        if (i >= en) {
+          miss = 1;                        // first entry
+        } else {
+          const int jo = i - sh.t[b] - 1;  // delta of timestep i was computed at old position jo
+          miss = (red.del(b * P + jo) < d.cache_thresh) ? 0 : 1;
+        }
+      }
+    }
+    const unsigned mm = __ballot_sync(0xffffffffu, miss);
+    const int r = base + __popc(mm & ((1u << lane) - 1u));
+    if (miss && r == target) {
+      sh.target_b = b;
+      sh.target_i = sh.tn[b] + j;
+    }
+    if (publish && q < N) {
+      if (miss) {
+        d.rank[q] = r;
+        d.miss_bt[2 * r] = b;
+        d.miss_bt[2 * r + 1] = sh.tn[b] + j;
+        atomicAdd(&sh.m[b], 1);
+      } else {
+        d.rank[q] = -1;
+        if (inwin && j >= 1) atomicAdd(&sh.h1[b], 1);
+      }
+    }
+    base += __popc(mm);
+    pts += __popc(__ballot_sync(0xffffffffu, inwin));
+  }
+  if (lane == 0) sh.total = base;
+  __syncwarp();
+  // 3. trajectories and counters of the next iteration
+  if (publish) {
+    for (int b = lane; b < B; b += 32) {
+      Traj tr{};
+      tr.t = sh.tn[b];
+      tr.p = sh.pn[b];
+      tr.e = sh.en[b];
+      tr.done = (sh.pn[b] == 0);
+      tr.m = sh.m[b];
+      tr.h1 = sh.h1[b];
+      if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
+      out_traj[b] = tr;
+    }
+    if (lane == 0) {
+      int act = 0;
+      for (int b = 0; b < B; ++b) act += (sh.pn[b] > 0);
+      PlanCtr c;
+      c.n_active = act;
+      c.iter = iter + 1;
+      c.nfe = sh.nfe + base;
+      c.hits = sh.hits + (pts - base);
+      d.pc[par ^ 1] = c;
+      d.ctl->n_miss = base;
+      d.ctl->n_active = act;
+      d.ctl->iter = c.iter;
+      d.ctl->nfe = c.nfe;
+      d.ctl->hits = c.hits;
+    }
+  }
+}
+
 }  // namespace pa
