@@ -48,11 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {
-    ("6a9f5cdb0de0680f", "sd15"): 6247488.0,
-    ("6a9f5cdb0de0680f", "batched"): 24649984.0,
-    ("6a9f5cdb0de0680f", "large"): 71753838.0,
-}
+NCU_TRAFFIC = {("e14e0e14b3b3bf7a", "sd15"): 6276224.0,
+               ("e14e0e14b3b3bf7a", "batched"): 24550698.7,
+               ("e14e0e14b3b3bf7a", "large"): 70852681.1}
 
 
 def parse_args(argv=None):
@@ -452,7 +450,7 @@ def run_ours(args):
     traffic = NCU_TRAFFIC.get((sha, args.workload))
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "Picard update (" + ("bulk-copy kernel" if st1["update_kernel"] == 1
+                "kernel": "Picard update (" + ("register-resident or staged form, by shape" if st1["update_kernel"] == 1
                                                else "plain loads") + ")",
                 "traffic_note": "ncu dram read+write bytes per launch, averaged over one generation",
                 "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
