@@ -93,6 +93,11 @@ def test_large_latent():
                tol=1e-3, cache_thresh=0.05, seed=9),
     W.Workload("tight tol", T=24, window=10, batch=2, latent_shape=(4, 16, 16), K=6,
                tol=1e-6, cache_thresh=0.02, seed=10),
+    # more than 1024 (trajectory, position) pairs: one CTA plans, a separate gather follows
+    W.Workload("9 x 128 pairs", T=200, window=128, batch=9, latent_shape=(4, 4, 4), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=13),
+    W.Workload("64 trajectories", T=40, window=32, batch=64, latent_shape=(4, 4, 4), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=14),
 ], ids=lambda w: w.name)
 def test_edge_shapes(w):
     _check(w)
