@@ -13,9 +13,13 @@
 //                 block boundaries); a converged trajectory is frozen; Parareal is exact at k = N.
 // Every evaluation stage: cache distance of each live row against its index's
 // entry (Eq. 4), hit iff entry && delta < tau_cache (Eq. 5), misses compacted
-// trajectory-major (k_srds_plan) and gathered for the denoiser; then the step
-// (k_srds_apply) takes eps from the batch (miss, updating the entry, Eq. 7) or
-// from the cache (hit, Eq. 6).
+// trajectory-major and gathered for the denoiser (k_srds_plan_gather); then
+// the step (k_srds_apply) takes eps from the batch (miss, updating the entry,
+// Eq. 7) or from the cache (hit, Eq. 6). The distances of a stage's rows are
+// summed by the kernel that produced those rows (the previous stage's
+// k_srds_apply, or k_srds_err for the first fine stage of an iteration) into
+// fp64 accumulators, one set per stage parity, while the new values are in
+// registers.
 //
 // Data (rows of D): U, Up [B][N+1][D] fp64 boundaries now and before this
 // iteration; Y [B][N][D] fp64 fine states (F after the sweep); G [B][N][D]
@@ -40,7 +44,6 @@ namespace {
 constexpr int kSThreads = 256;
 constexpr int kSStrip = 4096;        // columns per distance / error CTA
 constexpr int kSMaxRows = 2048;      // B * N
-constexpr int kSPlanPer = kSMaxRows / kSThreads;
 
 enum StageKind : int32_t { kCoarseInit = 0, kFine = 1, kCoarse = 2 };
 
@@ -62,7 +65,8 @@ struct SDev {
   float* batch_x;    // [B*N][D]
   int32_t* miss_bt;  // [B*N][2]
   int32_t* rank;     // [B*N]: miss rank, -1 hit, -2 not live
-  double* part;      // [B*N][nstrip]
+  double* part;      // [B*N][nstrip] Eq. 2 partials of the block boundaries
+  double* sacc;      // [2][B*N] Eq. 4 sums of the next stage's rows, set = stage number mod 2
   int32_t* active;   // [B]
   int32_t* iters;    // [B]
   float* err_log;    // [N][B]
@@ -113,116 +117,81 @@ __device__ __forceinline__ double block_sum(double v, double* s_w) {
   return t;
 }
 
-// Eq. 4 partial sums: sum |x - xhat_i| over one strip of one row with an entry.
-__global__ void __launch_bounds__(kSThreads) k_srds_dist(SDev d, Stage st) {
-  __shared__ double s_w[kSThreads / 32];
-  const int r = blockIdx.y;
+// One stage's plan and batch, one launch. Warp 0 of every CTA takes the
+// stage's decision over its rows (at most 2048, 32 at a time): a live row
+// with an entry hits iff its distance sum / D < tau_cache (Eq. 5); misses get
+// ranks in row order (trajectory-major) by ballots and population counts. The
+// same inputs give the same plan in every CTA; CTA (0, 0) publishes it (ranks,
+// miss list, counters) and clears the distance set the coming apply adds into.
+// Then every CTA narrows its column range of the batch row whose rank is its
+// blockIdx.y, if that row holds a miss.
+__global__ void __launch_bounds__(kSThreads) k_srds_plan_gather(SDev d, Stage st, int set) {
+  __shared__ int s_total, s_row;
+  const int tid = threadIdx.x;
+  const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
+  const int rows = stage_rows(d, st);
+  const int R = d.B * d.N;
+  if (tid < 32) {
+    const int lane = tid;
+    int base = 0, hits = 0, target_row = -1;
+    for (int q0 = 0; q0 < rows; q0 += 32) {
+      const int r = q0 + lane;
+      int b = 0, n = 0, i = 0;
+      double* x = nullptr;
+      const bool live = r < rows && row_info(d, st, r, b, n, i, x);
+      bool hit = false;
+      if (live && d.has[(int64_t)b * d.T + i]) hit = d.sacc[(size_t)set * R + r] / (double)d.D < d.cache_thresh;
+      const bool miss = live && !hit;
+      const unsigned mm = __ballot_sync(0xffffffffu, miss);
+      const int rank = base + __popc(mm & ((1u << lane) - 1u));
+      if (miss && rank == (int)blockIdx.y) target_row = r;
+      if (publish && r < rows) {
+        d.rank[r] = miss ? rank : (live ? -1 : -2);
+        if (miss) {
+          d.miss_bt[2 * rank] = b;
+          d.miss_bt[2 * rank + 1] = i;
+        }
+      }
+      base += __popc(mm);
+      hits += __popc(__ballot_sync(0xffffffffu, live && hit));
+    }
+    // the lane that saw the target row reports it
+    const unsigned tm = __ballot_sync(0xffffffffu, target_row >= 0);
+    if (tm && lane == __ffs(tm) - 1) s_row = target_row;
+    if (lane == 0) {
+      s_total = base;
+      if (!tm) s_row = -1;
+      if (publish) {
+        d.ctl->n_miss = base;
+        d.ctl->nfe += base;
+        d.ctl->hits += hits;
+      }
+    }
+    if (publish)
+      for (int q = lane; q < R; q += 32) d.sacc[(size_t)(set ^ 1) * R + q] = 0.0;
+  }
+  __syncthreads();
+  const int m = blockIdx.y, r = s_row;
+  if (m >= s_total || r < 0) return;
   int b, n, i;
   double* x;
-  if (!row_info(d, st, r, b, n, i, x) || !d.has[(int64_t)b * d.T + i]) return;
-  const double* xh = d.Xh + ((int64_t)b * d.T + i) * d.D;
-  const int64_t c0 = (int64_t)blockIdx.x * kSStrip;
-  const int64_t c1 = (c0 + kSStrip < d.D) ? c0 + kSStrip : d.D;
-  double acc = 0.0;
-  for (int64_t c = c0 + threadIdx.x; c < c1; c += kSThreads) acc += fabs(x[c] - xh[c]);
-  const double t = block_sum(acc, s_w);
-  if (threadIdx.x == 0) d.part[(int64_t)r * d.nstrip + blockIdx.x] = t;
-}
-
-// Hit/miss of every live row (Eq. 5, first entry = miss) and the compaction of
-// the misses in row order (trajectory-major), one CTA.
-__global__ void __launch_bounds__(kSThreads) k_srds_plan(SDev d, Stage st) {
-  __shared__ int s_warp[kSThreads / 32];
-  __shared__ int s_total, s_hits;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  const int rows = stage_rows(d, st);
-  if (tid == 0) s_hits = 0;
-  __syncthreads();
-  int flag[kSPlanPer];  // 1 miss, 0 hit, -1 not live
-  int cnt = 0, hits = 0;
-  const int q0 = tid * kSPlanPer;
-#pragma unroll
-  for (int u = 0; u < kSPlanPer; ++u) {
-    const int r = q0 + u;
-    flag[u] = -1;
-    if (r >= rows) continue;
-    int b, n, i;
-    double* x;
-    if (!row_info(d, st, r, b, n, i, x)) continue;
-    bool hit = false;
-    if (d.has[(int64_t)b * d.T + i]) {
-      double sum = 0.0;
-      for (int k = 0; k < d.nstrip; ++k) sum += d.part[(int64_t)r * d.nstrip + k];
-      hit = sum / (double)d.D < d.cache_thresh;
-    }
-    flag[u] = hit ? 0 : 1;
-    cnt += hit ? 0 : 1;
-    hits += hit ? 1 : 0;
-  }
-  int incl = cnt;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int v = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += v;
-  }
-  if (lane == 31) s_warp[warp] = incl;
-  atomicAdd(&s_hits, hits);
-  __syncthreads();
-  if (warp == 0) {
-    const int w = lane < kSThreads / 32 ? s_warp[lane] : 0;
-    int wi = w;
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-      const int v = __shfl_up_sync(0xffffffffu, wi, o);
-      if (lane >= o) wi += v;
-    }
-    if (lane < kSThreads / 32) s_warp[lane] = wi - w;
-    if (lane == 31) s_total = wi;
-  }
-  __syncthreads();
-  int m = s_warp[warp] + incl - cnt;
-#pragma unroll
-  for (int u = 0; u < kSPlanPer; ++u) {
-    const int r = q0 + u;
-    if (r >= rows) continue;
-    if (flag[u] == 1) {
-      int b, n, i;
-      double* x;
-      row_info(d, st, r, b, n, i, x);
-      d.rank[r] = m;
-      d.miss_bt[2 * m] = b;
-      d.miss_bt[2 * m + 1] = i;
-      ++m;
-    } else {
-      d.rank[r] = flag[u] == 0 ? -1 : -2;
-    }
-  }
-  if (tid == 0) {
-    d.ctl->n_miss = s_total;
-    d.ctl->nfe += s_total;
-    d.ctl->hits += s_hits;
-  }
-}
-
-// batch_x[m] <- the input row of miss m.
-__global__ void __launch_bounds__(kSThreads) k_srds_gather(SDev d, Stage st) {
-  const int n_miss = d.ctl->n_miss;
-  for (int m = blockIdx.y; m < n_miss; m += gridDim.y) {
-    const int b = d.miss_bt[2 * m], i = d.miss_bt[2 * m + 1];
-    const int n = i / d.s;
-    const double* x = st.kind == kFine ? d.Y + ((int64_t)b * d.N + n) * d.D
-                                       : d.U + ((int64_t)b * (d.N + 1) + n) * d.D;
-    float* to = d.batch_x + (int64_t)m * d.D;
-    for (int64_t c = (int64_t)blockIdx.x * kSThreads + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * kSThreads)
-      to[c] = (float)x[c];
-  }
+  row_info(d, st, r, b, n, i, x);
+  float* to = d.batch_x + (int64_t)m * d.D;
+  for (int64_t c = (int64_t)blockIdx.x * kSThreads + tid; c < d.D; c += (int64_t)gridDim.x * kSThreads)
+    to[c] = (float)x[c];
 }
 
 // The step of every live row: eps from the batch (miss: the entry becomes
 // (x, eps), Eq. 7) or the cache (hit, Eq. 6); then a fine step
 // Y <- Y + (c_i - 1) Y + e_i eps, or a coarse jump g = x + (c - 1) x + e eps
 // with U_{n+1} = g (iteration 0) or g + F_n - G_n (later), G_n <- g.
-__global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, const float* __restrict__ beps) {
+// The next stage's rows that this stage produced also get their Eq. 4
+// distance here, added into set `nset`: a fine step feeds the next fine step
+// of its block; the last fine step of block 0 feeds the first coarse block,
+// whose input U_0 does not change; a coarse block feeds the next one.
+__global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, const float* __restrict__ beps,
+                                                         int nset) {
+  __shared__ double s_w[kSThreads / 32];
   const int r = blockIdx.y;
   int b, n, i;
   double* x;
@@ -236,6 +205,24 @@ __global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, cons
   double* Un1 = d.U + ((int64_t)b * (d.N + 1) + n + 1) * d.D;
   double* Gn = d.G + ((int64_t)b * d.N + n) * d.D;
   const double* Fn = d.Y + ((int64_t)b * d.N + n) * d.D;
+  // the next stage's row fed by this one, if any: its row index, timestep and input
+  int nrow = -1, i1 = 0;
+  const double* nx0 = nullptr;  // the next input when it is not the value computed here
+  if (st.kind == kFine) {
+    if (st.j + 1 < d.s) {
+      const int end = min((n + 1) * d.s, d.T);
+      if (i + 1 < end) { nrow = r; i1 = i + 1; }
+    } else if (n == 0) {
+      nrow = b; i1 = 0; nx0 = d.U + (int64_t)b * (d.N + 1) * d.D;
+    }
+  } else if (n + 1 < d.N) {
+    nrow = b; i1 = (n + 1) * d.s;
+  }
+  // an entry for timestep i1 exists if an earlier stage made it, or this row
+  // (same timestep: one step per block) is a miss making it now
+  const bool nhas = nrow >= 0 && ((i1 == i && rk >= 0) || d.has[(int64_t)b * d.T + i1] != 0);
+  const double* xh1 = d.Xh + ((int64_t)b * d.T + i1) * d.D;
+  double dist = 0.0;
   for (int64_t c = (int64_t)blockIdx.x * kSThreads + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * kSThreads) {
     const double xv = x[c];
     const float ev = eps[c];
@@ -244,21 +231,32 @@ __global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, cons
       d.Eh[e_off + c] = ev;
     }
     const double g = xv + fma(cm1, xv, ec * (double)ev);
+    double nv;
     if (st.kind == kFine) {
       x[c] = g;
+      nv = g;
     } else if (st.kind == kCoarseInit) {
       Gn[c] = g;
       Un1[c] = g;
+      nv = g;
     } else {
-      Un1[c] = g + (Fn[c] - Gn[c]);
+      nv = g + (Fn[c] - Gn[c]);
+      Un1[c] = nv;
       Gn[c] = g;
     }
+    if (nhas) dist += fabs((nx0 ? nx0[c] : nv) - xh1[c]);
+  }
+  if (nhas) {
+    const double t = block_sum(dist, s_w);
+    if (threadIdx.x == 0) atomicAdd(d.sacc + (size_t)nset * d.B * d.N + nrow, t);
   }
 }
 
 // End of an iteration: partial sums of (U_{n+1} - Up_{n+1})^2 per strip
 // (iterations >= 1), then Up <- U and Y_n <- U_n for the next fine sweep.
-__global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter) {
+// The next fine sweep starts from Y_n = U_n: the Eq. 4 distance of its first
+// stage's rows (timestep n s) is added into set `nset` here.
+__global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter, int nset) {
   __shared__ double s_w[kSThreads / 32];
   const int r = blockIdx.y, b = r / d.N, n = r % d.N;
   if (!d.active[b]) return;
@@ -268,15 +266,24 @@ __global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter) {
   double* p1 = d.Up + ((int64_t)b * (d.N + 1) + n + 1) * d.D;
   const double* u0 = d.U + ((int64_t)b * (d.N + 1) + n) * d.D;
   double* y = d.Y + ((int64_t)b * d.N + n) * d.D;
-  double acc = 0.0;
+  const bool nhas = d.has[(int64_t)b * d.T + n * d.s] != 0;
+  const double* xh = d.Xh + ((int64_t)b * d.T + n * d.s) * d.D;
+  double acc = 0.0, dist = 0.0;
   for (int64_t c = c0 + threadIdx.x; c < c1; c += kSThreads) {
     const double df = u1[c] - p1[c];
     acc = fma(df, df, acc);
     p1[c] = u1[c];
-    y[c] = u0[c];
+    const double v = u0[c];
+    y[c] = v;
+    if (nhas) dist += fabs(v - xh[c]);
   }
   const double t = block_sum(acc, s_w);
   if (threadIdx.x == 0) d.part[(int64_t)r * d.nstrip + blockIdx.x] = iter > 0 ? t : 0.0;
+  if (nhas) {
+    __syncthreads();  // s_w is reused
+    const double t2 = block_sum(dist, s_w);
+    if (threadIdx.x == 0) atomicAdd(d.sacc + (size_t)nset * d.B * d.N + r, t2);
+  }
 }
 
 // Convergence of every trajectory after iteration `iter` (one CTA).
@@ -342,7 +349,7 @@ __global__ void k_srds_reset(SDev d) {
 }
 
 struct SLayout {
-  size_t U, Up, Y, G, Xh, Eh, has, batch_x, miss_bt, rank, part, active, iters, err_log, coef, ctl, total;
+  size_t U, Up, Y, G, Xh, Eh, has, batch_x, miss_bt, rank, part, sacc, active, iters, err_log, coef, ctl, total;
 };
 
 SLayout s_layout(int T, int64_t D, int B, int N, int nstrip) {
@@ -361,6 +368,7 @@ SLayout s_layout(int T, int64_t D, int B, int N, int nstrip) {
   L.miss_bt = take((size_t)B * N * 2 * sizeof(int32_t));
   L.rank = take((size_t)B * N * sizeof(int32_t));
   L.part = take((size_t)B * N * nstrip * sizeof(double));
+  L.sacc = take((size_t)2 * B * N * sizeof(double));
   L.active = take((size_t)B * sizeof(int32_t));
   L.iters = take((size_t)B * sizeof(int32_t));
   L.err_log = take((size_t)N * B * sizeof(float));
@@ -387,6 +395,8 @@ struct pa_srds {
   int phase;      // -1 created, 0 ready for a step, 1 stepped (waiting for eps), 2 done
   int iter;       // current iteration (0 = coarse initialisation)
   int stage;      // index within the iteration: fine stages first (iter >= 1), then coarse
+  int64_t g;      // stages since pa_srds_init: the distance set of stage g is g mod 2
+  int nsm;        // SMs of the device
   int64_t launches;
   SCtl* host_ctl;
 };
@@ -472,6 +482,7 @@ extern "C" pa_status pa_srds_create(pa_srds** out, int T, const int64_t* latent_
   d.miss_bt = reinterpret_cast<int32_t*>(w + L.miss_bt);
   d.rank = reinterpret_cast<int32_t*>(w + L.rank);
   d.part = reinterpret_cast<double*>(w + L.part);
+  d.sacc = reinterpret_cast<double*>(w + L.sacc);
   d.active = reinterpret_cast<int32_t*>(w + L.active);
   d.iters = reinterpret_cast<int32_t*>(w + L.iters);
   d.err_log = reinterpret_cast<float*>(w + L.err_log);
@@ -496,7 +507,10 @@ extern "C" pa_status pa_srds_create(pa_srds** out, int T, const int64_t* latent_
     const int a0 = n * s, a1 = (n + 1) * s < T ? (n + 1) * s : T;
     jump(alphas_cumprod[a0], alphas_cumprod[a1], &hc[2 * T + n], &hc[2 * T + N + n]);
   }
-  cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&h->host_ctl), sizeof(SCtl), cudaHostAllocDefault);
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&h->nsm, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess) e = cudaHostAlloc(reinterpret_cast<void**>(&h->host_ctl), sizeof(SCtl), cudaHostAllocDefault);
   if (e == cudaSuccess) e = cudaMemcpyAsync(coef, hc.data(), hc.size() * sizeof(double), cudaMemcpyHostToDevice, h->st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d.ctl, 0, sizeof(SCtl), h->st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
@@ -519,9 +533,11 @@ extern "C" pa_status pa_srds_init(pa_srds* h, const float* x_init) {
   k_srds_reset<<<1, 256, 0, h->st>>>(d);
   h->launches += 2;
   e = cudaGetLastError();
+  if (e == cudaSuccess) e = cudaMemsetAsync(d.sacc, 0, (size_t)2 * d.B * d.N * sizeof(double), h->st);
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_init: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   h->iter = 0;
   h->stage = 0;
+  h->g = 0;
   h->phase = 0;
   return PA_OK;
 }
@@ -534,11 +550,14 @@ extern "C" pa_status pa_srds_step_async(pa_srds* h, const float** batch_x, const
   const SDev& d = h->d;
   const Stage st = current_stage(h);
   const int rows = st.kind == kFine ? d.B * d.N : d.B;
-  k_srds_dist<<<dim3(d.nstrip, rows), kSThreads, 0, h->st>>>(d, st);
-  k_srds_plan<<<1, kSThreads, 0, h->st>>>(d, st);
-  const int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
-  k_srds_gather<<<dim3(gx < 32 ? gx : 32, rows), kSThreads, 0, h->st>>>(d, st);
-  h->launches += 3;
+  // every CTA plans: about two CTAs per SM in all, each narrowing a longer part of its row
+  int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
+  const int gcap = (2 * h->nsm + rows - 1) / rows;
+  if (gx > gcap) gx = gcap;
+  if (gx > 32) gx = 32;
+  if (gx < 1) gx = 1;
+  k_srds_plan_gather<<<dim3(gx, rows), kSThreads, 0, h->st>>>(d, st, (int)(h->g & 1));
+  h->launches += 1;
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_step_async: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   if (batch_x) *batch_x = d.batch_x;
@@ -577,16 +596,18 @@ extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
   const Stage st = current_stage(h);
   const int rows = st.kind == kFine ? d.B * d.N : d.B;
   const int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
-  k_srds_apply<<<dim3(gx < 32 ? gx : 32, rows), kSThreads, 0, h->st>>>(d, st, batch_eps);
+  const int nset = (int)((h->g + 1) & 1);  // the next stage's distance set
+  k_srds_apply<<<dim3(gx < 32 ? gx : 32, rows), kSThreads, 0, h->st>>>(d, st, batch_eps, nset);
   h->launches++;
   const int nstages = (h->iter == 0 ? 0 : d.s) + d.N;
   if (++h->stage == nstages) {  // the iteration is complete
-    k_srds_err<<<dim3(d.nstrip, d.B * d.N), kSThreads, 0, h->st>>>(d, h->iter);
+    k_srds_err<<<dim3(d.nstrip, d.B * d.N), kSThreads, 0, h->st>>>(d, h->iter, nset);
     k_srds_finish<<<1, kSThreads, 0, h->st>>>(d, h->iter);
     h->launches += 2;
     h->stage = 0;
     h->iter++;
   }
+  h->g++;
   const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_submit_eps: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   h->phase = (h->iter > d.N) ? 2 : 0;
