@@ -69,7 +69,8 @@ class PicardResult:
 
 
 def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
-               use_cache=True, max_iters=None, record=True, eta=0.0, noise=None):
+               use_cache=True, max_iters=None, record=True, eta=0.0, noise=None,
+               cache_store=None):
     """Cached (or uncached) sliding-window Picard sampling of B trajectories.
 
     alphas       : fp64 [T+1] sampling-order alpha-bar (alphas[T] == 1).
@@ -83,6 +84,9 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
     eta, noise   : stochastic steps (eta > 0): noise [B][T][D] holds the draws
                    z_i; the drift of step i gains sigma_i z_i (the same draw in
                    every iteration).
+    cache_store  : how a cache entry is stored (step 5): None keeps the value,
+                   oracle.storage.round_bf16 stores bfloat16 entries (states
+                   and the fresh eps of a miss keep full precision).
     """
     a = np.asarray(alphas, dtype=np.float64)
     T = len(a) - 1
@@ -161,8 +165,12 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
                 for j in range(pb):
                     if not hitflags[b][j]:
                         i = tb + j
-                        Xhat[b, i] = X[b, i]
-                        Ehat[b, i] = eps_w[j]
+                        if cache_store is None:
+                            Xhat[b, i] = X[b, i]
+                            Ehat[b, i] = eps_w[j]
+                        else:
+                            Xhat[b, i] = cache_store(X[b, i])
+                            Ehat[b, i] = cache_store(eps_w[j])
                         has_entry[b, i] = True
             # 6. drift at the current latents
             idx = np.arange(tb, tb + pb)
