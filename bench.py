@@ -65,6 +65,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-kernel", type=int, default=None)
     ap.add_argument("--gmm-form", type=int, default=None, help="denoiser dot products: 1 tensor cores, 0 CUDA cores")
+    ap.add_argument("--cache-bits", type=int, default=32, choices=[16, 32],
+                    help="storage of the cache entries: 32 fp32, 16 bfloat16")
     ap.add_argument("--oracle-sample", type=float, default=None, help=argparse.SUPPRESS)
     return ap.parse_args(argv)
 
@@ -123,17 +125,19 @@ def kernel_source_sha():
     return h.hexdigest()[:16]
 
 
-def iteration_bytes(log, w: W.Workload):
+def iteration_bytes(log, w: W.Workload, entry_bytes=4):
     """Algorithmic bytes per Picard iteration, from the solver's iteration log.
 
     Per trajectory with window start t, p points, m misses, frontier e and h1
-    hits at positions >= 1 (rows of D fp32 values):
-      update : x_t, the p - lazy materialised old states, p eps rows, m ehat
-               and m xhat writes, h1 xhat reads (next distances), p new states,
-               and p draws z_i for stochastic steps (eta > 0)
+    hits at positions >= 1 (rows of D fp32 values; cache-entry rows of D
+    values of entry_bytes each):
+      update : x_t, the p - lazy materialised old states, m batch eps rows and
+               p - m ehat rows, m ehat and m xhat writes, h1 xhat reads (next
+               distances), p new states, and p draws z_i for stochastic steps
       gather : m reads + m writes;  denoiser: m reads + m writes (+ K means)
     """
     row = w.D * 4
+    ent = w.D * entry_bytes
     upd, other = [], []
     for k in range(log.shape[0]):
         u = o = 0
@@ -142,7 +146,7 @@ def iteration_bytes(log, w: W.Workload):
             if p == 0:
                 continue
             lazy = max(0, t + p - e)
-            u += (1 + (p - lazy) + p + 2 * m + h1 + p + (p if w.eta != 0.0 else 0)) * row
+            u += (1 + (p - lazy) + m + p + (p if w.eta != 0.0 else 0)) * row + ((p - m) + 2 * m + h1) * ent
             o += 4 * m * row
         upd.append(u)
         other.append(o + w.K * row)
@@ -309,6 +313,8 @@ def run_ours(args):
     s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=stream)
     if args.update_kernel is not None:
         s.set_update_kernel(args.update_kernel)
+    if args.cache_bits == 16:
+        s.set_cache_precision(16)
     if w.eta != 0.0:  # stochastic steps: the draws stay resident on the device
         s.set_noise(w.eta, torch.from_numpy(W.noise(w)).to(dev))
     max_rows = w.batch * s.window
@@ -338,7 +344,7 @@ def run_ours(args):
     st0 = s.stats()
     log = s.iter_log()
     nfe, hits = st0["nfe"], st0["hits"]
-    upd_bytes, other_bytes = iteration_bytes(log, w)
+    upd_bytes, other_bytes = iteration_bytes(log, w, 2 if args.cache_bits == 16 else 4)
 
     # One generation (n_iters Picard iterations: denoiser, update and planning
     # kernels each -- the planning kernel decides and gathers the next batch;
@@ -447,7 +453,7 @@ def run_ours(args):
     n_upd = args.steps * n_iters
     achieved = upd_bytes.sum() * args.steps / (upd_ms / 1000.0) / 1e9
     sha = kernel_source_sha()
-    traffic = NCU_TRAFFIC.get((sha, args.workload))
+    traffic = NCU_TRAFFIC.get((sha, args.workload + ("-bf16" if args.cache_bits == 16 else "")))
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic,
                 "kernel": "Picard update (" + ("register-resident or staged form, by shape" if st1["update_kernel"] == 1
@@ -510,6 +516,7 @@ def run_ours(args):
                        "seq_len": w.T, "window": w.window, "latent": "x".join(map(str, w.latent_shape)),
                        "mixture_components": w.K, "tol": w.tol, "cache_thresh": w.cache_thresh,
                        "eta": w.eta,
+                       "cache_entries": "bf16" if args.cache_bits == 16 else "fp32",
                        "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
                                                  if g.form() == 1 else "CUDA cores (fp32 FMA)"),
                        "parallelism": f"replicas x{world} (independent trajectories)",

@@ -187,6 +187,17 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
  * tiled pipeline). Returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
 
+/* Storage precision of the cache entries (xhat, ehat of Eq. 3): 32 = fp32
+ * (default), 16 = bfloat16, rounded to nearest even when an entry is written
+ * (Eq. 7) and widened exactly when read. Not from the paper: a storage option
+ * that halves the entries' bytes; the states, the fresh eps of a miss and all
+ * arithmetic stay fp32, so a hit reuses the rounded eps and Eq. 4 measures the
+ * distance to the rounded input. With 16 the update runs in the register form
+ * (windows up to 104, deterministic steps) or the plain-load kernel. Any time
+ * except between pa_step and pa_submit_eps; the next call must be pa_init.
+ * Returns PA_ERR_ARG for another value, PA_ERR_STATE in the wrong state. */
+PA_API pa_status pa_set_cache_precision(pa_solver* s, int bits);
+
 /* Fault-handling test hook: the number of tries (each may suspend for about
  * 10 us) after which an mbarrier wait of the bulk-copy update kernel counts
  * as timed out (default 2^17, about a second). With 0

@@ -70,6 +70,7 @@ _PROTOS = {
     "pa_iter_log": (C.c_int, [VP, C.POINTER(C.c_int32), C.c_int, C.POINTER(C.c_int)]),
     "pa_last_reductions": (C.c_int, [VP, VP, VP]),
     "pa_set_update_kernel": (C.c_int, [VP, C.c_int]),
+    "pa_set_cache_precision": (C.c_int, [VP, C.c_int]),
     "pa_debug_set_wait_limit": (C.c_int, [VP, C.c_uint32]),
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
     "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.c_int]),
@@ -237,6 +238,10 @@ def pa_last_reductions(h, batch, window):
 
 def pa_set_update_kernel(h, kind):
     return _check("pa_set_update_kernel", lib().pa_set_update_kernel(h, int(kind)))
+
+
+def pa_set_cache_precision(h, bits):
+    return _check("pa_set_cache_precision", lib().pa_set_cache_precision(h, int(bits)))
 
 
 def pa_debug_set_wait_limit(h, polls):

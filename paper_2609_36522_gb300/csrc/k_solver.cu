@@ -153,9 +153,40 @@ __device__ __forceinline__ void stv(float* p, const V<VEC>& v) {
   }
 }
 
+// A cache entry row (xhat or ehat) at element offset `off`: fp32, or bfloat16 when CB.
+template <int VEC, bool CB>
+__device__ __forceinline__ V<VEC> ld_entry(const float* base, int64_t off) {
+  if constexpr (CB) {
+    V<VEC> r;
+    Bf16Row<VEC>::load(reinterpret_cast<const uint16_t*>(base) + off, r.a);
+    return r;
+  } else {
+    return ldv<VEC>(base + off);
+  }
+}
+template <int VEC, bool CB>
+__device__ __forceinline__ void st_entry(float* base, int64_t off, const V<VEC>& v) {
+  if constexpr (CB) {
+    Bf16Row<VEC>::store(reinterpret_cast<uint16_t*>(base) + off, v.a);
+  } else {
+    stv<VEC>(base + off, v);
+  }
+}
+template <int VEC, bool CB>
+__device__ __forceinline__ V<VEC> as_entry(const V<VEC>& v) {
+  if constexpr (CB) {
+    V<VEC> r;
+#pragma unroll
+    for (int k = 0; k < VEC; ++k) r.a[k] = __bfloat162float(__float2bfloat16_rn(v.a[k]));
+    return r;
+  } else {
+    return v;
+  }
+}
+
 constexpr int kPlainThreads = 128;
 
-template <int VEC>
+template <int VEC, bool CB>
 __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const float* __restrict__ beps, int par) {
   extern __shared__ float red[];  // [2][nwarps][P]
   const int b = blockIdx.y;
@@ -169,8 +200,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
   const int64_t col = ((int64_t)blockIdx.x * kPlainThreads + threadIdx.x) * VEC;
   const bool live = col < D;
   float* Xb = d.X + (int64_t)b * (P + 1) * D + col;
-  float* Xh = d.Xhat + (int64_t)b * P * D + col;
-  float* Eh = d.Ehat + (int64_t)b * P * D + col;
+  const int64_t cbase = (int64_t)b * P * D + col;  // element offset of this column in the cache rows
   const int32_t* rk = d.rank + b * P;
   const int n_miss = d.ctl->n_miss;
 
@@ -187,10 +217,11 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
     const int slot = i % P;
     float ev = 0.f, dv = 0.f;
     if (live) {
-      V<VEC> eps = (r >= 0) ? ldv<VEC>(beps + (int64_t)r * D + col) : ldv<VEC>(Eh + (int64_t)slot * D);
+      V<VEC> eps = (r >= 0) ? ldv<VEC>(beps + (int64_t)r * D + col)
+                            : ld_entry<VEC, CB>(d.Ehat, cbase + (int64_t)slot * D);
       if (r >= 0) {
-        stv<VEC>(Eh + (int64_t)slot * D, eps);
-        stv<VEC>(Xh + (int64_t)slot * D, xcur);
+        st_entry<VEC, CB>(d.Ehat, cbase + (int64_t)slot * D, eps);
+        st_entry<VEC, CB>(d.Xhat, cbase + (int64_t)slot * D, xcur);
       }
       V<VEC> xo;
       if (i + 1 <= e) {
@@ -216,7 +247,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
       stv<VEC>(Xb + (int64_t)((i + 1) % (P + 1)) * D, xn);
       if (j + 1 < p) {
         const int r1 = rk[j + 1];
-        V<VEC> xh = (r1 >= 0) ? xo : ldv<VEC>(Xh + (int64_t)((i + 1) % P) * D);
+        V<VEC> xh = (r1 >= 0) ? as_entry<VEC, CB>(xo) : ld_entry<VEC, CB>(d.Xhat, cbase + (int64_t)((i + 1) % P) * D);
 #pragma unroll
         for (int v = 0; v < VEC; ++v) dv += fabsf(xn.a[v] - xh.a[v]);
       }
@@ -383,10 +414,14 @@ cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, int par, c
                        (reinterpret_cast<uintptr_t>(d.noise) & 15) == 0;
   if (d.D % 4 == 0 && aligned) {
     const int nchunk = (int)((d.D + kPlainThreads * 4 - 1) / (kPlainThreads * 4));
-    return launch_ex(k_update_plain<4>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
+    if (d.cache_bf16)
+      return launch_ex(k_update_plain<4, true>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
+    return launch_ex(k_update_plain<4, false>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
   }
   const int nchunk = (int)((d.D + kPlainThreads - 1) / kPlainThreads);
-  return launch_ex(k_update_plain<1>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
+  if (d.cache_bf16)
+    return launch_ex(k_update_plain<1, true>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
+  return launch_ex(k_update_plain<1, false>, dim3(nchunk, d.B), dim3(kPlainThreads), smem, st, 0, d, batch_eps, par);
 }
 
 }  // namespace pa

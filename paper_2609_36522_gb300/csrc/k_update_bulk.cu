@@ -103,6 +103,38 @@ __device__ __forceinline__ void stv(float* p, const Vec<V>& v) {
   }
 }
 
+// A cache entry row (xhat or ehat) as stored: fp32, or bfloat16 when CB.
+template <int V, bool CB>
+__device__ __forceinline__ Vec<V> ld_entry(const float* base, int64_t off) {
+  if constexpr (CB) {
+    Vec<V> r;
+    Bf16Row<V>::load(reinterpret_cast<const uint16_t*>(base) + off, r.a);
+    return r;
+  } else {
+    return ldv<V>(base + off);
+  }
+}
+template <int V, bool CB>
+__device__ __forceinline__ void st_entry(float* base, int64_t off, const Vec<V>& v) {
+  if constexpr (CB) {
+    Bf16Row<V>::store(reinterpret_cast<uint16_t*>(base) + off, v.a);
+  } else {
+    stv<V>(base + off, v);
+  }
+}
+// The value an entry holds once stored.
+template <int V, bool CB>
+__device__ __forceinline__ Vec<V> as_entry(const Vec<V>& v) {
+  if constexpr (CB) {
+    Vec<V> r;
+#pragma unroll
+    for (int k = 0; k < V; ++k) r.a[k] = __bfloat162float(__float2bfloat16_rn(v.a[k]));
+    return r;
+  } else {
+    return v;
+  }
+}
+
 template <int V, int NW, int S>
 struct TileShape {
   static constexpr int SEG = 32 * V;                  // columns per strip
@@ -716,7 +748,7 @@ struct RegShape {
   __host__ __device__ static size_t smem_bytes(int P) { return rank_bytes(P) + kTotBytes + red_bytes(P); }
 };
 
-template <int V, int NW, int LMAX, bool NOISE>
+template <int V, int NW, int LMAX, bool NOISE, bool CB = false>
 __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* __restrict__ beps, int par) {
   using Sh = RegShape<V, NW>;
   constexpr int SEG = Sh::SEG;
@@ -784,9 +816,9 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
         if (sl1 >= P) sl1 -= P;
         int nx = nx0 + g;
         if (nx >= P + 1) nx -= P + 1;
-        if (rk[g] < 0) eps[g] = ldv<V>(Eh + (int64_t)sl * D + mycol);
+        if (rk[g] < 0) eps[g] = ld_entry<V, CB>(Eh, (int64_t)sl * D + mycol);
         if (t + j + 1 <= e) xo[g] = ldv<V>(Xb + (int64_t)nx * D + mycol);
-        if (j + 1 < p && rk[g + 1] < 0) xh[g] = ldv<V>(Xh + (int64_t)sl1 * D + mycol);
+        if (j + 1 < p && rk[g + 1] < 0) xh[g] = ld_entry<V, CB>(Xh, (int64_t)sl1 * D + mycol);
         if (NOISE) zn[g] = ldv<V>(d.noise + ((int64_t)b * d.T + t + j) * D + mycol);
       }
     }
@@ -813,8 +845,8 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
           int sl = sl0 + g;
           if (sl >= P) sl -= P;
           const int64_t o = (int64_t)sl * D + mycol;
-          stv<V>(Eh + o, eps[g]);
-          stv<V>(Xh + o, xc);
+          st_entry<V, CB>(Eh, o, eps[g]);
+          st_entry<V, CB>(Xh, o, xc);
         }
 #pragma unroll
         for (int v = 0; v < V; ++v) {
@@ -867,7 +899,7 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
         if (j + 1 < p) {
           // the next timestep's cache input: its entry if it is a hit, else
           // this iteration's x_{i+1} (the entry it is about to receive)
-          const Vec<V> xc1 = rk[g + 1] < 0 ? xh[g] : xold;
+          const Vec<V> xc1 = rk[g + 1] < 0 ? xh[g] : as_entry<V, CB>(xold);
 #pragma unroll
           for (int v = 0; v < V; ++v) dv += fabsf(xn.a[v] - xc1.a[v]);
         }
@@ -894,12 +926,12 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
   }
 }
 
-template <int V, int NW, int LMAX, bool NOISE>
+template <int V, int NW, int LMAX, bool NOISE, bool CB = false>
 cudaError_t launch_reg(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = RegShape<V, NW>;
   const int nstrip = (int)((d.D + Sh::SEG - 1) / Sh::SEG);
   const size_t smem = Sh::smem_bytes(d.P);
-  auto kern = k_update_reg<V, NW, LMAX, NOISE>;
+  auto kern = k_update_reg<V, NW, LMAX, NOISE, CB>;
   static size_t configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -926,6 +958,11 @@ int reg_lmax(const Dev& d) {
 
 cudaError_t launch_reg_auto(const Dev& d, const float* beps, int par, cudaStream_t st) {
   const int lm = reg_lmax(d);
+  if (d.cache_bf16) {  // bfloat16 entries: deterministic steps only (update_bulk_supported)
+    if (lm == 4) return launch_reg<4, 8, 4, false, true>(d, beps, par, st);
+    if (lm == 8) return launch_reg<4, 8, 8, false, true>(d, beps, par, st);
+    return launch_reg<4, 8, kRegMaxL, false, true>(d, beps, par, st);
+  }
   if (d.noise) {
     if (lm == 4) return launch_reg<4, 8, 4, true>(d, beps, par, st);
     return launch_reg<4, 8, kRegMaxLNoise, true>(d, beps, par, st);
@@ -970,8 +1007,10 @@ cudaError_t launch_tile(const Dev& d, const float* beps, int par, cudaStream_t s
 bool update_bulk_supported(const Dev& d, const float* batch_eps) {
   // 16-byte granularity of bulk copies: every row segment must start on a
   // 16-byte boundary and be a multiple of 16 bytes long. Stochastic steps
-  // stage the draws too, in the segment form only.
+  // stage the draws too, in the segment form only. bfloat16 cache entries:
+  // the register form only, deterministic steps.
   const bool ok = d.D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps) & 15) == 0;
+  if (d.cache_bf16) return ok && !d.noise && reg_lmax(d) > 0;
   if (!d.noise) return ok;
   return ok && (reinterpret_cast<uintptr_t>(d.noise) & 15) == 0 && seg_fits<2, 8, true>(d);
 }
@@ -998,6 +1037,7 @@ bool prefer_wide_strips(const Dev& d) {
 }
 
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, int par, cudaStream_t st) {
+  if (d.cache_bf16) return launch_reg_auto(d, batch_eps, par, st);  // update_bulk_supported
   if (d.bulk_cfg == 12 && reg_lmax(d)) return launch_reg_auto(d, batch_eps, par, st);
   if (d.noise) {  // stochastic steps: the segment forms with the draws (update_bulk_supported)
     if (prefer_wide_strips<true>(d)) {

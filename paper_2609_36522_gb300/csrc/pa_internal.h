@@ -2,6 +2,7 @@
 // kernels (k_solver.cu, k_update_bulk.cu). Not part of the public ABI.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 #include <stddef.h>
 #include <stdint.h>
@@ -106,6 +107,7 @@ struct Dev {
   int64_t D;
   double tol, cache_thresh;   // compared against the fp64 sums divided by D
   int bulk_cfg;               // launch shape of the bulk-copy update kernel
+  int cache_bf16;             // 1: xhat and ehat rows hold bfloat16 values (row pitch D elements)
   uint32_t wait_limit;        // polls before an mbarrier wait counts as timed out
 };
 constexpr uint32_t kWaitLimit = 1u << 17;  // tries of an mbarrier wait (~1.3 s with the suspend hint)
@@ -151,6 +153,37 @@ cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem
   cfg.numAttrs = n;
   return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
 }
+
+// Cache entries stored as bfloat16 (a storage option, not from the paper):
+// loads widen exactly, stores round to nearest even.
+template <int V>
+struct Bf16Row;
+template <>
+struct Bf16Row<4> {
+  __device__ static void load(const uint16_t* p, float* a) {
+    const uint2 q = *reinterpret_cast<const uint2*>(p);
+    a[0] = __uint_as_float(q.x << 16);
+    a[1] = __uint_as_float(q.x & 0xffff0000u);
+    a[2] = __uint_as_float(q.y << 16);
+    a[3] = __uint_as_float(q.y & 0xffff0000u);
+  }
+  __device__ static void store(uint16_t* p, const float* a) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(a[0], a[1]);
+    const __nv_bfloat162 hi = __floats2bfloat162_rn(a[2], a[3]);
+    uint2 q;
+    q.x = *reinterpret_cast<const uint32_t*>(&lo);
+    q.y = *reinterpret_cast<const uint32_t*>(&hi);
+    *reinterpret_cast<uint2*>(p) = q;
+  }
+};
+template <>
+struct Bf16Row<1> {
+  __device__ static void load(const uint16_t* p, float* a) { a[0] = __uint_as_float((uint32_t)*p << 16); }
+  __device__ static void store(uint16_t* p, const float* a) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(a[0]);
+    *p = *reinterpret_cast<const uint16_t*>(&h);
+  }
+};
 
 // One CTA's share of the Eq. 2 error (which = 0) or Eq. 4 distance (which =
 // 1) of window position q = b*P + j, added into the accumulator set of the

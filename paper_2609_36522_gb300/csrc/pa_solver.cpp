@@ -215,6 +215,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.tol = tol;
   d.cache_thresh = cache_thresh;
   d.wait_limit = pa::kWaitLimit;
+  d.cache_bf16 = 0;
   s->update_kind = (D % 4 == 0) ? 1 : 0;
 
   const std::vector<float> hc = step_coefficients(s->alphas, 0.0);  // DDIM (eta = 0)
@@ -437,6 +438,15 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   } else {
     return arg_fail("pa_set_update_kernel: kind must be 0, 1 or 100 + launch shape");
   }
+  return PA_OK;
+}
+
+pa_status pa_set_cache_precision(pa_solver* s, int bits) {
+  if (!s) return arg_fail("pa_set_cache_precision: solver is NULL");
+  if (bits != 16 && bits != 32) return arg_fail("pa_set_cache_precision: bits must be 16 or 32");
+  if (s->state == St::Stepped) return state_fail("pa_set_cache_precision");
+  s->d.cache_bf16 = bits == 16 ? 1 : 0;
+  s->state = St::Created;  // the entries change meaning: pa_init starts over
   return PA_OK;
 }
 

@@ -121,6 +121,10 @@ class Solver:
     def set_update_kernel(self, kind):
         abi.pa_set_update_kernel(self.h, kind)
 
+    def set_cache_precision(self, bits):
+        """16: bfloat16 cache entries, 32: fp32 (default). pa_init must follow."""
+        abi.pa_set_cache_precision(self.h, bits)
+
     def close(self):
         if getattr(self, "h", None) is not None:
             abi.pa_destroy(self.h)

@@ -9,15 +9,15 @@ from oracle import run_picard
 from oracle.gmm import make_eps_fn, gmm_eps
 
 
-def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True):
+def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True, cache_store=None):
     a, x0, mu = W.inputs(w)
     thr = w.cache_thresh if cache_thresh is None else cache_thresh
     return run_picard(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr,
-                      use_cache=use_cache, eta=w.eta, noise=W.noise(w))
+                      use_cache=use_cache, eta=w.eta, noise=W.noise(w), cache_store=cache_store)
 
 
 def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=None,
-            mode="sync", x_init_host=False, gmm_form=None):
+            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None):
     """Run one generation on the GPU.
 
     eps_source: "gmm" (the CUDA mixture kernel) or "oracle" (fp64 mixture
@@ -33,6 +33,8 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
     s = Solver(w.T, w.window, w.latent_shape, a, w.tol, thr, batch=w.batch)
     if update_kernel is not None:
         s.set_update_kernel(update_kernel)
+    if cache_bits is not None:
+        s.set_cache_precision(cache_bits)
     max_rows = w.batch * s.window
     means = torch.from_numpy(mu).to(dev)
     g = GmmDenoiser(means, w.gmm_std, a, max_rows)

@@ -85,6 +85,7 @@ def test_null_handles_are_rejected(lib):
     assert L.pa_nfe(None) == -1
     assert L.pa_n_miss_dev(None) is None
     assert L.pa_set_update_kernel(None, 0) == abi.PA_ERR_ARG
+    assert L.pa_set_cache_precision(None, 16) == abi.PA_ERR_ARG
     L.pa_destroy(None)
     L.pa_gmm_destroy(None)
     assert L.pa_gmm_launches(None) == -1

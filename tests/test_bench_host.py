@@ -63,3 +63,6 @@ def test_iteration_bytes_counts_rows():
     row = w.D * 4
     assert upd[0] == (1 + 0 + 8 + 16 + 0 + 8) * row
     assert other[0] == (4 * 8 + w.K) * row
+    # bfloat16 entries: the 16 entry writes count half a row each
+    upd16, _ = bench.iteration_bytes(log, w, entry_bytes=2)
+    assert upd16[0] == (1 + 0 + 8 + 8) * row + 16 * (row // 2)

@@ -302,3 +302,61 @@ def test_eta_zero_restores_ddim():
     plain = gpu_run(w)
     again = gpu_run(w.with_(eta=0.0))
     assert np.array_equal(plain["x_final"], again["x_final"])
+
+
+# ---- bfloat16 cache entries (a storage option, not from the paper) ----------
+
+def bf16_tolerance(w, orc):
+    """Where the GPU's fp32 value and the oracle's fp64 value of a cache entry
+    element straddle a bfloat16 rounding boundary, the two store neighbouring
+    bfloat16 values: one ulp apart, at most 2^(floor(log2 max|ehat|) - 7). A
+    reuse of that element moves one drift by |e_i| times that ulp, which the
+    window sum carries to the final state. Two such events at the largest DDIM
+    coefficient, relative to the smallest max|x_T|."""
+    from oracle.ddim import step_coefficients
+    _, e, _ = step_coefficients(W.alphas_cumprod(w.T), w.eta)
+    ulp = 2.0 ** (np.floor(np.log2(np.abs(orc.ehat[orc.has_entry]).max())) - 7)
+    return 2.0 * np.abs(e).max() * ulp / np.abs(orc.x_final).max(axis=1).min()
+
+
+@pytest.mark.parametrize("w", [
+    W.SD15, W.BATCHED,
+    W.Workload("multi-strip", T=40, window=24, batch=3, latent_shape=(4, 20, 20), K=6,
+               tol=1e-3, cache_thresh=0.05, seed=16),
+    W.Workload("ragged odd D", T=30, window=12, batch=2, latent_shape=(3, 5, 7), K=3,
+               tol=1e-3, cache_thresh=0.05, seed=3),
+    W.Workload("window 128", T=150, window=128, batch=1, latent_shape=(4, 16, 16), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=15),
+], ids=lambda w: w.name)
+def test_bf16_cache_entries(w):
+    """Entries stored as bfloat16 on both sides: decisions, miss lists and NFE
+    exact (inputs guarded at 1e-3 relative, since an entry element can round to
+    a neighbouring bfloat16 value when the GPU's fp32 value and the oracle's
+    fp64 value straddle a rounding boundary), final latents within the bound of
+    bf16_tolerance (about 1.6e-3 at T = 100). The register form runs where it
+    applies, the plain-load kernel elsewhere (odd D, window 128)."""
+    from oracle.storage import round_bf16
+    orc = oracle_run(w, cache_store=round_bf16)
+    assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-3), decision_margins(orc, w.tol, w.cache_thresh)
+    gpu = gpu_run(w, cache_bits=16)
+    rel = compare(w, orc, gpu)
+    assert rel.max() <= bf16_tolerance(w, orc), (rel, bf16_tolerance(w, orc))
+
+
+def test_bf16_cache_rejected_while_stepped():
+    from paper_2609_36522_gb300 import abi
+    import torch
+    from paper_2609_36522_gb300.solver import Solver
+    w = W.TINY
+    a, x0, _ = W.inputs(w)
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch)
+    s.init(torch.from_numpy(x0).cuda())
+    s.step()
+    with pytest.raises(abi.PaError) as e:
+        s.set_cache_precision(16)
+    assert e.value.status == abi.PA_ERR_STATE
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_set_cache_precision(s.h, 8)
+    assert e.value.status == abi.PA_ERR_ARG
+    s.close()
+
