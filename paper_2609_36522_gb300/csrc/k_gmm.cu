@@ -224,12 +224,9 @@ __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__
                                                        bool bulk, long long* __restrict__ gacc2,
                                                        GmmEpoch* ep, int32_t* status) {
   extern __shared__ __align__(128) unsigned char smem_raw[];
-  __shared__ __align__(8) uint64_t bar;
+  __shared__ __align__(8) uint64_t bar_m, bar_x;
   long long* gacc = begin_dots(gacc2, ep, (int64_t)max_rows * K);
-  const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
   const int r0 = blockIdx.y * kDotRows;
-  if (r0 >= n_rows) return;
-  const int nr = min(kDotRows, n_rows - r0);
   const int64_t c0 = (int64_t)blockIdx.x * chunk;
   const int ncol = (int)(((D - c0) < chunk) ? (D - c0) : chunk);
   const int ld = chunk + 4;  // padded row stride, keeps 16-byte alignment
@@ -237,16 +234,27 @@ __global__ void __launch_bounds__(kThreads) k_gmm_dots(const float* __restrict__
   float* ms = xs + (size_t)kDotRows * ld;
   const int tid = threadIdx.x;
   if (tid == 0) {
-    mbar_init(&bar, 1);
+    mbar_init(&bar_m, 1);
+    mbar_init(&bar_x, 1);
     fence_barrier_init();
-    if (bulk) mbar_arrive_expect_tx(&bar, (uint32_t)ncol * sizeof(float) * (uint32_t)(nr + K));
+    if (bulk) mbar_arrive_expect_tx(&bar_m, (uint32_t)ncol * sizeof(float) * (uint32_t)K);
+  }
+  __syncthreads();
+  stage_rows(ms, ld, mu, D, c0, ncol, K, bulk, &bar_m);  // the means do not depend on the predecessor
+  pdl_wait();  // the rows and their count come from the kernel just before
+  pdl_trigger();  // the successor may now run its prologue
+  const int n_rows = min(*n_rows_dev, max_rows);
+  const int nr = min(kDotRows, n_rows - r0);
+  if (nr <= 0) {  // no rows for this CTA: the means copy lands before it exits
+    wait_staged(bulk, &bar_m, status);
+    return;
   }
   for (int q = tid; q < (kDotRows - nr) * ld; q += kThreads) xs[(size_t)nr * ld + q] = 0.f;  // rows past nr
+  if (tid == 0 && bulk) mbar_arrive_expect_tx(&bar_x, (uint32_t)ncol * sizeof(float) * (uint32_t)nr);
   __syncthreads();
-  stage_rows(ms, ld, mu, D, c0, ncol, K, bulk, &bar);  // the means do not depend on the predecessor
-  pdl_wait();  // the rows come from the gather (or the caller) just before
-  stage_rows(xs, ld, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar);
-  const bool ok = wait_staged(bulk, &bar, status);
+  stage_rows(xs, ld, X + (int64_t)r0 * D, D, c0, ncol, nr, bulk, &bar_x);
+  const bool ok_m = wait_staged(bulk, &bar_m, status);
+  const bool ok = wait_staged(bulk, &bar_x, status) && ok_m;
   __syncthreads();
   if (!ok) return;
 
@@ -324,7 +332,10 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   __shared__ float s_sa[kOutRows], s_q[kOutRows];
   const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
   const int r0 = blockIdx.y * kOutRows;
-  if (r0 >= n_rows) return;
+  if (r0 >= n_rows) {  // every CTA passes the dependency wait before it exits
+    pdl_wait();
+    return;
+  }
   const int nr = min(kOutRows, n_rows - r0);
   const int64_t c0 = (int64_t)blockIdx.x * kOutCols;
   const int ncol = (int)(((D - c0) < kOutCols) ? (D - c0) : kOutCols);
@@ -348,6 +359,7 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
     s_c[2 * rr + 1] = coef[2 * T + i] * coef[i];
   }
   pdl_wait();  // the dot products come from the kernel just before
+  pdl_trigger();  // the successor may now run its prologue
   // both accumulator sets are read together with the set index (one round trip)
   const uint32_t cur = ep->cur;
   const int64_t set_size = (int64_t)max_rows * K;
@@ -473,10 +485,7 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
   __shared__ uint32_t s_taddr;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   long long* gacc = begin_dots(gacc2, ep, (int64_t)max_rows * K);
-  const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
   const int r0 = blockIdx.y * kTcRows;
-  if (r0 >= n_rows) return;
-  const int nr = min(kTcRows, n_rows - r0);
   const int Kp = tc_npad(K);
   const uint32_t ncols = 2 * Kp < 32 ? 32u : (uint32_t)(2 * Kp);  // TMEM columns: a power of two >= 32
   const int64_t c0 = (int64_t)blockIdx.x * kTcCols;
@@ -500,7 +509,18 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
     mbar_arrive_expect_tx(&bar_mu, bytes);
     bulk_g2s(B_img, mu_img + (size_t)blockIdx.x * tc_mu_chunk_floats(K), bytes, &bar_mu);
   }
-  pdl_wait();  // the rows come from the gather just before
+  pdl_wait();  // the rows and their count come from the kernel just before
+  pdl_trigger();  // the successor may now run its prologue
+  const int n_rows = min(*n_rows_dev, max_rows);
+  const int nr = min(kTcRows, n_rows - r0);
+  if (nr <= 0) {  // no rows for this block (the whole cluster alike): the means copy
+                  // lands and TMEM is freed before the CTA exits
+    if (!mbar_wait_bounded(&bar_mu, 0, pa::kDrainLimit) && tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    tc_fence_before_sync();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(taddr, ncols);
+    return;
+  }
 
   // rows -> (hi, lo) in core-matrix order: a warp step covers 8 rows x 16
   // columns; lanes 8q..8q+7 write one 128-byte core matrix (conflict-free).

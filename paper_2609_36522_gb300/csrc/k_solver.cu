@@ -100,6 +100,7 @@ __device__ __forceinline__ void copy_row(const Dev& d, int b, int src_state, int
 template <int VEC>
 __global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d, int par) {
   pdl_wait();  // everything read here comes from the kernel that planned
+  pdl_trigger();  // the successor may now run its prologue
   const int n = d.ctl->n_miss;
   const Traj* tr = d.traj + par * d.B;
   for (int r = blockIdx.y; r < n; r += gridDim.y) {
@@ -191,6 +192,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
   extern __shared__ float red[];  // [2][nwarps][P]
   const int b = blockIdx.y;
   pdl_wait();
+  pdl_trigger();  // the successor may now run its prologue
   const Traj tr = d.traj[par * d.B + b];
   if (tr.p == 0) return;
   const int t = tr.t, p = tr.p, e = tr.e, P = d.P;
@@ -311,6 +313,7 @@ __global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
   const int npair = d.B * d.P;
   decide_load<kPlanThreads>(d, ds, par);
   pdl_wait();  // the sums and the new states come from the update kernel
+  pdl_trigger();  // the successor may now run its prologue
   const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair;
   const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair;
   const double inv_d = 1.0 / (double)d.D;
@@ -344,6 +347,7 @@ __global__ void __launch_bounds__(kPlanOneThreads) k_plan_one(Dev d, int par) {
   const int npair = d.B * d.P;
   decide_load<kPlanOneThreads>(d, ds, par);
   pdl_wait();  // the sums come from the update kernel
+  pdl_trigger();  // the successor may now run its prologue
   const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair;
   const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair;
   const RedSums red{acc_e, acc_d, 1.0 / (double)d.D};

@@ -193,7 +193,10 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   const Traj tr = d.traj[par * d.B + b];
   const int n_miss = d.ctl->n_miss;
   for (int j = tid; j < P; j += NW * 32) s_rank[j] = d.rank[b * P + j];
-  if (tr.p == 0) return;
+  if (tr.p == 0) {  // finished trajectory; every CTA passes the dependency wait before it exits
+    pdl_wait();
+    return;
+  }
   const int t = tr.t, p = tr.p, e = tr.e;
   for (int j = tid; j < p; j += NW * 32) {
     s_slot[j] = (t + j) % P;
@@ -218,6 +221,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_tile(Dev d, const float* __r
   // Everything above came from the decision kernel and earlier; the eps rows
   // below come from the denoiser that ran just before this kernel.
   pdl_wait();
+  pdl_trigger();  // the successor may now run its prologue
 
   const int strip = blockIdx.x;          // the grid is padded to whole clusters
   const bool active = strip < nstrip;
@@ -524,7 +528,10 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
   // from the denoiser just before.
   const Traj tr = d.traj[par * d.B + b];
   const int n_miss = d.ctl->n_miss;
-  if (tr.p == 0) return;
+  if (tr.p == 0) {  // finished trajectory; every CTA passes the dependency wait before it exits
+    pdl_wait();
+    return;
+  }
   const int t = tr.t, p = tr.p, e = tr.e;
   for (int j = tid; j < p; j += NW * 32) {
     int r = d.rank[b * P + j];
@@ -577,6 +584,7 @@ __global__ void __launch_bounds__(NW * 32) k_update_seg(Dev d, const float* __re
       if (NOISE) bulk_g2s(rowp + 3 * SEG, d.noise + ((int64_t)b * d.T + t + j) * D + c0, seg_bytes, &bar[warp]);
     }
     pdl_wait();  // the batch eps rows come from the denoiser that ran just before
+    pdl_trigger();  // the successor may now run its prologue
     for (int j = j0 + lane; j < j1; j += 32) {
       const int r = s_rank[j];
       if (r >= 0) bulk_g2s(s_rows + (size_t)j * NR * SEG, beps + (int64_t)r * D + c0, seg_bytes, &bar[warp]);
@@ -775,7 +783,10 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
     }
     s_rank[j] = r;
   }
-  if (tr.p == 0) return;
+  if (tr.p == 0) {  // finished trajectory; every CTA passes the dependency wait before it exits
+    pdl_wait();
+    return;
+  }
   __syncthreads();
   const int t = tr.t, p = tr.p, e = tr.e;
   const int strip = blockIdx.x;
@@ -824,6 +835,7 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
     }
   }
   pdl_wait();  // the batch eps rows come from the denoiser that ran just before
+  pdl_trigger();  // the successor may now run its prologue
   if (live) {
 #pragma unroll
     for (int g = 0; g < LMAX; ++g)

@@ -113,13 +113,16 @@ struct Dev {
 constexpr uint32_t kWaitLimit = 1u << 17;  // tries of an mbarrier wait (~1.3 s with the suspend hint)
 
 // Programmatic dependent launch (PDL). Every kernel of an iteration is
-// launched with programmatic stream serialization, so it may be scheduled as
-// soon as its predecessor's CTAs have exited, before the predecessor's grid is
-// retired: it does the work that does not read the predecessor's output, then
-// executes pdl_wait() (predecessor complete, its writes visible). No kernel
-// triggers its successor early (pdl_trigger is available but unused: early
-// triggers let waiting CTAs hold shared memory the predecessor still needs),
-// so a kernel's prologue may read anything written two or more kernels back.
+// launched with programmatic stream serialization: it does the work that does
+// not read its predecessor's output, then executes pdl_wait() (predecessor
+// complete, its writes visible). Each kernel triggers its successor
+// (pdl_trigger) right after its own pdl_wait, never before: when a kernel
+// starts, every CTA of its predecessor has passed its wait, so the kernel two
+// back has completed. A kernel's prologue may therefore read anything written
+// two or more kernels back, and must not write anything its predecessor reads.
+// The successor is scheduled only once all of the predecessor's CTAs have
+// triggered, i.e. are resident, so its waiting CTAs never keep a predecessor
+// CTA from an SM.
 __device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
 __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 

@@ -121,6 +121,51 @@ def test_async_equals_sync_and_is_deterministic():
     assert a["nfe"] == b["nfe"]
 
 
+@pytest.mark.parametrize("w,form", [
+    (W.SD15, 0),
+    (W.LARGE.with_(T=60), 1),
+    (W.BATCHED.with_(T=40), 0),
+], ids=["sd15-cuda-cores", "large-tensor-cores", "batched"])
+def test_graph_replay_equals_sync(w, form):
+    """A whole generation captured as one CUDA graph (pa_init and every
+    iteration's denoiser, update and planning kernels, chained by programmatic
+    dependent launches with early triggers) and replayed twice gives the
+    synchronous run's states and iteration log bit for bit: every kernel reads
+    its predecessor's output only after its dependency wait."""
+    import torch
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+    sync = gpu_run(w, gmm_form=form)
+    n_iters = len(sync["log"])
+    a, x0, mu = W.inputs(w)
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=st)
+        g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, w.batch * s.window, stream=st)
+        g.set_form(form)
+        eps = torch.empty(w.batch * s.window, w.D, dtype=torch.float32, device="cuda")
+        x_dev = torch.from_numpy(x0).cuda()
+        s.init(x_dev)
+        out = s.step_async()                       # eager warm-up of every launch path
+        g.eps(*out, eps)
+        s.submit_eps(eps)
+        st.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=st):
+            s.init(x_dev)
+            for _ in range(n_iters):
+                out = s.step_async()
+                g.eps(*out, eps)
+                s.submit_eps(eps)
+        for _ in range(2):
+            graph.replay()
+            st.synchronize()
+            assert s.poll() == 0
+            assert np.array_equal(s.result().cpu().numpy(), sync["x_final"])
+            assert np.array_equal(s.iter_log(), sync["log"])
+    s.close()
+    g.close()
+
+
 def test_host_x_init_equals_device_x_init():
     a = gpu_run(W.TINY)
     b = gpu_run(W.TINY, x_init_host=True)
