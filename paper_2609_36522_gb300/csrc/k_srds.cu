@@ -126,6 +126,8 @@ __device__ __forceinline__ double block_sum(double v, double* s_w) {
 // Then every CTA narrows its column range of the batch row whose rank is its
 // blockIdx.y, if that row holds a miss.
 __global__ void __launch_bounds__(kSThreads) k_srds_plan_gather(SDev d, Stage st, int set) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   __shared__ int s_total, s_row;
   const int tid = threadIdx.x;
   const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
@@ -191,6 +193,8 @@ __global__ void __launch_bounds__(kSThreads) k_srds_plan_gather(SDev d, Stage st
 // whose input U_0 does not change; a coarse block feeds the next one.
 __global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, const float* __restrict__ beps,
                                                          int nset) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   __shared__ double s_w[kSThreads / 32];
   const int r = blockIdx.y;
   int b, n, i;
@@ -257,6 +261,8 @@ __global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, cons
 // The next fine sweep starts from Y_n = U_n: the Eq. 4 distance of its first
 // stage's rows (timestep n s) is added into set `nset` here.
 __global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter, int nset) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   __shared__ double s_w[kSThreads / 32];
   const int r = blockIdx.y, b = r / d.N, n = r % d.N;
   if (!d.active[b]) return;
@@ -288,6 +294,8 @@ __global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter, int ns
 
 // Convergence of every trajectory after iteration `iter` (one CTA).
 __global__ void __launch_bounds__(kSThreads) k_srds_finish(SDev d, int iter) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   __shared__ int s_act;
   if (threadIdx.x == 0) s_act = 0;
   __syncthreads();
@@ -319,6 +327,8 @@ __global__ void __launch_bounds__(kSThreads) k_srds_finish(SDev d, int iter) {
 
 // fp32 rows (pitch D) -> fp64 rows of the boundary array (pitch (N+1) D), and back.
 __global__ void k_srds_load(SDev d, const float* __restrict__ src, int slot) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   const int b = blockIdx.y;
   double* to = d.U + ((int64_t)b * (d.N + 1) + slot) * d.D;
   double* to2 = d.Up + ((int64_t)b * (d.N + 1) + slot) * d.D;
@@ -329,6 +339,8 @@ __global__ void k_srds_load(SDev d, const float* __restrict__ src, int slot) {
 }
 
 __global__ void k_srds_store(SDev d, float* __restrict__ dst, int slot) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   const int b = blockIdx.y;
   const double* from = d.U + ((int64_t)b * (d.N + 1) + slot) * d.D;
   for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < d.D; c += (int64_t)gridDim.x * blockDim.x)
@@ -336,6 +348,8 @@ __global__ void k_srds_store(SDev d, float* __restrict__ dst, int slot) {
 }
 
 __global__ void k_srds_reset(SDev d) {
+  pa::pdl_wait();     // everything read here comes from earlier kernels
+  pa::pdl_trigger();  // the successor may now be scheduled
   for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
     d.active[b] = 1;
     d.iters[b] = 0;
@@ -529,10 +543,9 @@ extern "C" pa_status pa_srds_init(pa_srds* h, const float* x_init) {
   // x_init (host or device) is staged in batch_x, then widened into U_0 and Up_0
   cudaError_t e = cudaMemcpyAsync(d.batch_x, x_init, (size_t)d.B * d.D * sizeof(float), cudaMemcpyDefault, h->st);
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_init: ") + cudaGetErrorString(e), PA_ERR_CUDA);
-  k_srds_load<<<dim3(32, d.B), 256, 0, h->st>>>(d, d.batch_x, 0);
-  k_srds_reset<<<1, 256, 0, h->st>>>(d);
+  e = pa::launch_ex(k_srds_load, dim3(32, d.B), dim3(256), 0, h->st, 0, d, (const float*)d.batch_x, 0);
+  if (e == cudaSuccess) e = pa::launch_ex(k_srds_reset, dim3(1), dim3(256), 0, h->st, 0, d);
   h->launches += 2;
-  e = cudaGetLastError();
   if (e == cudaSuccess) e = cudaMemsetAsync(d.sacc, 0, (size_t)2 * d.B * d.N * sizeof(double), h->st);
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_init: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   h->iter = 0;
@@ -556,9 +569,9 @@ extern "C" pa_status pa_srds_step_async(pa_srds* h, const float** batch_x, const
   if (gx > gcap) gx = gcap;
   if (gx > 32) gx = 32;
   if (gx < 1) gx = 1;
-  k_srds_plan_gather<<<dim3(gx, rows), kSThreads, 0, h->st>>>(d, st, (int)(h->g & 1));
+  const cudaError_t e =
+      pa::launch_ex(k_srds_plan_gather, dim3(gx, rows), dim3(kSThreads), 0, h->st, 0, d, st, (int)(h->g & 1));
   h->launches += 1;
-  const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_step_async: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   if (batch_x) *batch_x = d.batch_x;
   if (miss_bt) *miss_bt = d.miss_bt;
@@ -597,18 +610,19 @@ extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
   const int rows = st.kind == kFine ? d.B * d.N : d.B;
   const int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
   const int nset = (int)((h->g + 1) & 1);  // the next stage's distance set
-  k_srds_apply<<<dim3(gx < 32 ? gx : 32, rows), kSThreads, 0, h->st>>>(d, st, batch_eps, nset);
+  cudaError_t e =
+      pa::launch_ex(k_srds_apply, dim3(gx < 32 ? gx : 32, rows), dim3(kSThreads), 0, h->st, 0, d, st, batch_eps, nset);
   h->launches++;
   const int nstages = (h->iter == 0 ? 0 : d.s) + d.N;
   if (++h->stage == nstages) {  // the iteration is complete
-    k_srds_err<<<dim3(d.nstrip, d.B * d.N), kSThreads, 0, h->st>>>(d, h->iter, nset);
-    k_srds_finish<<<1, kSThreads, 0, h->st>>>(d, h->iter);
+    if (e == cudaSuccess)
+      e = pa::launch_ex(k_srds_err, dim3(d.nstrip, d.B * d.N), dim3(kSThreads), 0, h->st, 0, d, h->iter, nset);
+    if (e == cudaSuccess) e = pa::launch_ex(k_srds_finish, dim3(1), dim3(kSThreads), 0, h->st, 0, d, h->iter);
     h->launches += 2;
     h->stage = 0;
     h->iter++;
   }
   h->g++;
-  const cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_submit_eps: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   h->phase = (h->iter > d.N) ? 2 : 0;
   return PA_OK;
@@ -629,9 +643,8 @@ extern "C" pa_status pa_srds_result(pa_srds* h, float* x_out) {
   if (h->phase != 2) return s_fail("pa_srds_result: not finished", PA_ERR_STATE);
   const SDev& d = h->d;
   // U_N narrowed to fp32 in batch_x (free once sampling is done), then copied out
-  k_srds_store<<<dim3(32, d.B), 256, 0, h->st>>>(d, d.batch_x, d.N);
+  cudaError_t e = pa::launch_ex(k_srds_store, dim3(32, d.B), dim3(256), 0, h->st, 0, d, d.batch_x, d.N);
   h->launches++;
-  cudaError_t e = cudaGetLastError();
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(x_out, d.batch_x, (size_t)d.B * d.D * sizeof(float), cudaMemcpyDefault, h->st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(h->st);
