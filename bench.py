@@ -355,6 +355,9 @@ def run_ours(args):
     one_iteration()                       # eager warm-up of every launch path
     stream.synchronize()
 
+    den_events = []   # (before, after) the denoiser call of every iteration, timed graph only
+    den_ms = [0.0]    # their total over the timed replays
+
     def capture(timed):
         """-> (graph, kernels launched per iteration inside it)"""
         abi.pa_set_kernel_timing(s.h, timed)
@@ -365,7 +368,18 @@ def run_ours(args):
         with torch.cuda.graph(gr, stream=stream):
             s.init(x_dev)                 # x_init copy, sums cleared, first plan and its gather
             for _ in range(n_iters):
-                one_iteration()
+                if not timed:
+                    one_iteration()
+                    continue
+                bx, mb, nm = s.step_async()
+                # recorded inside the capture: external events keep their timestamps
+                ev = (torch.cuda.Event(enable_timing=True, external=True),
+                      torch.cuda.Event(enable_timing=True, external=True))
+                ev[0].record(stream)
+                g.eps(bx, mb, nm, eps)
+                ev[1].record(stream)
+                den_events.append(ev)
+                s.submit_eps(eps)
         abi.pa_set_kernel_timing(s.h, False)
         l1 = s.stats()["launches"] + g.launches()
         return gr, (l1 - l0 - init_launches) // n_iters
@@ -386,6 +400,8 @@ def run_ours(args):
         e1.synchronize()
         ms = e0.elapsed_time(e1)
         upd = abi.pa_kernel_timing(s.h, reset=False)[0] if timed else 0.0
+        if timed:
+            den_ms[0] += sum(a.elapsed_time(b) for a, b in den_events)
         return ms, upd
 
     def cold_iterations(reps):
@@ -426,6 +442,7 @@ def run_ours(args):
     stream.synchronize()
     wall0 = time.perf_counter()
     dev_ms = upd_ms = timed_ms = 0.0
+    den_ms[0] = 0.0
     for _ in range(args.steps):
         a_ms, _ = generation(graph_plain, False)
         dev_ms += a_ms
@@ -531,6 +548,12 @@ def run_ours(args):
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
             "solver_step_gbps": gb_step,
+            "denoiser_us_per_iteration": 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
+            "solver_us_per_iteration": 1000.0 * dev_ms / max(1, args.steps * n_iters)
+                                       - 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
+            "solver_note": ("denoiser time from CUDA events around each denoiser call in the timed graph "
+                            "(its event nodes cut the dependent-launch overlap there, so it is an upper "
+                            "bound); solver = the plain graph's iteration time minus it"),
             "cold_iteration_us": cold_us,
             "cold_iteration_note": "one Picard iteration with L2 flushed before every iteration, "
                                    "CUDA events around each (conservative; includes one event pair per iteration)",
