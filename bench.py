@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {("a1a7792eae7961cc", "sd15"): 6274432.0,
-               ("a1a7792eae7961cc", "batched"): 24556970.7,
-               ("a1a7792eae7961cc", "large"): 70854582.9}
+NCU_TRAFFIC = {("822b9d6f9a31094c", "sd15"): 6274432.0,
+               ("822b9d6f9a31094c", "batched"): 24556970.7,
+               ("822b9d6f9a31094c", "large"): 70854582.9}
 
 
 def parse_args(argv=None):

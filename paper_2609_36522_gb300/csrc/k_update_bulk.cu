@@ -43,12 +43,6 @@ namespace cg = cooperative_groups;
 constexpr int kCluster = 8;
 
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
-
 // s = fl(a + b) and s + err == a + b exactly (Knuth's TwoSum).
 __device__ __forceinline__ void two_sum(float a, float b, float& s, float& err) {
   s = a + b;
