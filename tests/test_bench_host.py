@@ -66,3 +66,25 @@ def test_iteration_bytes_counts_rows():
     # bfloat16 entries: the 16 entry writes count half a row each
     upd16, _ = bench.iteration_bytes(log, w, entry_bytes=2)
     assert upd16[0] == (1 + 0 + 8 + 8) * row + 16 * (row // 2)
+
+
+@pytest.mark.parametrize("workload", ["tiny", "srds"])
+def test_reference_arm_json_line(workload):
+    """bench.py --impl reference times the fp64 oracle on the host and prints
+    one JSON line with the contract's keys (CPU only, no GPU involved)."""
+    import json
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    r = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference",
+                        "--workload", workload, "--steps", "1", "--warmup", "0"],
+                       capture_output=True, text=True, timeout=600, cwd=root)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    for key in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+                "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config", "e2e",
+                "cpu_baseline"):
+        assert key in line, key
+    assert line["impl"] == "reference" and line["value"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
