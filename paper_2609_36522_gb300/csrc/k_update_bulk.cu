@@ -58,6 +58,21 @@ __device__ __forceinline__ void acc_add(float& hi, float& lo, float v) {
   lo += e;
 }
 
+// Two lanes of fp32 at once (sm_100 and later: one instruction for both,
+// each rounded to nearest as the scalar operation would be).
+__device__ __forceinline__ float2 x2_add(float2 a, float2 b) { return __fadd2_rn(a, b); }
+__device__ __forceinline__ float2 x2_sub(float2 a, float2 b) {
+  return __ffma2_rn(b, make_float2(-1.f, -1.f), a);  // -b exact, one rounding: a - b
+}
+// (hi, lo) += v for two columns, the TwoSum above per component
+__device__ __forceinline__ void acc_add_x2(float2& hi, float2& lo, float2 v) {
+  const float2 s = x2_add(hi, v);
+  const float2 bb = x2_sub(s, hi);
+  const float2 err = x2_add(x2_sub(hi, x2_sub(s, bb)), x2_sub(v, bb));
+  hi = s;
+  lo = x2_add(lo, err);
+}
+
 // (hi, lo) += (h2, l2)
 __device__ __forceinline__ void acc_add2(float& hi, float& lo, float h2, float l2) {
   float s, e;
@@ -854,12 +869,19 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
           st_entry<V, CB>(Eh, o, eps[g]);
           st_entry<V, CB>(Xh, o, xc);
         }
+        const float2 cm2 = make_float2(cm1[g], cm1[g]), ec2 = make_float2(ec[g], ec[g]);
 #pragma unroll
-        for (int v = 0; v < V; ++v) {
-          float dr = fmaf(cm1[g], xc.a[v], ec[g] * eps[g].a[v]);
-          if (NOISE) dr = fmaf(sg[g], zn[g].a[v], dr);
-          acc_add(rh[v], rl[v], dr);
-          eps[g].a[v] = dr;
+        for (int v = 0; v < V; v += 2) {  // two columns per instruction
+          float2 dr = __ffma2_rn(cm2, make_float2(xc.a[v], xc.a[v + 1]),
+                                 __fmul2_rn(ec2, make_float2(eps[g].a[v], eps[g].a[v + 1])));
+          if (NOISE)
+            dr = __ffma2_rn(make_float2(sg[g], sg[g]), make_float2(zn[g].a[v], zn[g].a[v + 1]), dr);
+          float2 h = make_float2(rh[v], rh[v + 1]), l = make_float2(rl[v], rl[v + 1]);
+          acc_add_x2(h, l, dr);
+          rh[v] = h.x; rh[v + 1] = h.y;
+          rl[v] = l.x; rl[v + 1] = l.y;
+          eps[g].a[v] = dr.x;
+          eps[g].a[v + 1] = dr.y;
         }
         xc = (t + j + 1 <= e) ? xo[g] : xfill;
       }
@@ -893,11 +915,17 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
         const Vec<V> xold = (t + j + 1 <= e) ? xo[g] : xfill;
         Vec<V> xn;
 #pragma unroll
-        for (int v = 0; v < V; ++v) {
-          acc_add(ch[v], cl[v], eps[g].a[v]);
-          xn.a[v] = ch[v] + cl[v];
-          const float df = xn.a[v] - xold.a[v];
-          ev = fmaf(df, df, ev);
+        for (int v = 0; v < V; v += 2) {  // two columns per instruction
+          float2 h = make_float2(ch[v], ch[v + 1]), l = make_float2(cl[v], cl[v + 1]);
+          acc_add_x2(h, l, make_float2(eps[g].a[v], eps[g].a[v + 1]));
+          ch[v] = h.x; ch[v + 1] = h.y;
+          cl[v] = l.x; cl[v + 1] = l.y;
+          const float2 n = x2_add(h, l);
+          const float2 df = x2_sub(n, make_float2(xold.a[v], xold.a[v + 1]));
+          xn.a[v] = n.x;
+          xn.a[v + 1] = n.y;
+          ev = fmaf(df.x, df.x, ev);  // the error terms keep their column order
+          ev = fmaf(df.y, df.y, ev);
         }
         int nx = nx0 + g;
         if (nx >= P + 1) nx -= P + 1;
@@ -907,7 +935,11 @@ __global__ void __launch_bounds__(NW * 32, 1) k_update_reg(Dev d, const float* _
           // this iteration's x_{i+1} (the entry it is about to receive)
           const Vec<V> xc1 = rk[g + 1] < 0 ? xh[g] : as_entry<V, CB>(xold);
 #pragma unroll
-          for (int v = 0; v < V; ++v) dv += fabsf(xn.a[v] - xc1.a[v]);
+          for (int v = 0; v < V; v += 2) {
+            const float2 dd = x2_sub(make_float2(xn.a[v], xn.a[v + 1]), make_float2(xc1.a[v], xc1.a[v + 1]));
+            dv += fabsf(dd.x);
+            dv += fabsf(dd.y);
+          }
         }
       }
       s_red[(size_t)j * 33 + lane] = ev;
