@@ -723,6 +723,8 @@ def run_srds_bench(args, w):
         print(json.dumps(line))
     s.close()
     g.close()
+    if world > 1:
+        dist.destroy_process_group()
     return 0
 
 
