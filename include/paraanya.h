@@ -121,15 +121,18 @@ PA_API pa_status pa_set_noise(pa_solver* s, double eta, const float* noise_dev);
 /* Start a generation: x_init [batch][D] fp32, HOST or DEVICE pointer (the copy
  * direction is inferred from the address). All states of the first window are
  * x_init (Sec. 2.1 initial trajectory estimate); every first-window timestep is
- * a first entry, hence a miss (Sec. 2.2). Clears the cache and counters.
- * May be called again at any time to restart. */
+ * a first entry, hence a miss (Sec. 2.2). Clears the cache and counters,
+ * plans the first iteration and gathers its batch (two kernels), all
+ * asynchronous on the solver's stream. May be called again at any time to
+ * restart. */
 PA_API pa_status pa_init(pa_solver* s, const float* x_init);
 
-/* Plan the next iteration: returns in *n_miss the number of misses M
- * (Eq. 5), in *batch_x_dev the contiguous batch [M][D] of their latents
- * (gathered on the device), and in *miss_bt_dev the (b, i) list [M][2].
- * Synchronises the solver's stream once (to read M). Returns PA_DONE (and
- * M = 0) when every trajectory has finished. */
+/* The planned iteration: returns in *n_miss the number of misses M (Eq. 5),
+ * in *batch_x_dev the contiguous batch [M][D] of their latents and in
+ * *miss_bt_dev the (b, i) list [M][2]. The plan and the batch were made on
+ * the device by pa_init (first iteration) or by the previous pa_submit_eps;
+ * pa_step launches nothing and synchronises the solver's stream once (to read
+ * M). Returns PA_DONE (and M = 0) when every trajectory has finished. */
 PA_API pa_status pa_step(pa_solver* s, int* n_miss, const float** batch_x_dev,
                   const int32_t** miss_bt_dev);
 
@@ -146,9 +149,11 @@ PA_API const int32_t* pa_n_miss_dev(const pa_solver* s);
 /* Hand back eps_theta for the planned misses: batch_eps_dev [M][D] fp32,
  * DEVICE pointer, 16-byte alignment for the bulk-copy pipeline (otherwise the
  * plain-load kernel runs). Runs Eq. 6 (assembly), Eq. 7 (cache update),
- * the drift and the Picard prefix sum (Eq. 1), the errors of Eq. 2, the window
- * advance, and the cache distances / hit-miss plan of the next iteration
- * (Eq. 4, Eq. 5). Asynchronous on the solver's stream. */
+ * the drift and the Picard prefix sum (Eq. 1), the errors of Eq. 2 and the
+ * cache distances of the next iteration (Eq. 4) in the update kernel, then the
+ * window advance, the hit-miss plan of the next iteration (Eq. 5) and the
+ * gather of its batch in the planning kernel. Asynchronous on the solver's
+ * stream; batch_eps_dev must stay valid until the update kernel has run. */
 PA_API pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev);
 
 /* Synchronise and report: *n_active = trajectories not yet at t = T.
