@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {("822b9d6f9a31094c", "sd15"): 6274432.0,
-               ("822b9d6f9a31094c", "batched"): 24556970.7,
-               ("822b9d6f9a31094c", "large"): 70854582.9}
+NCU_TRAFFIC = {("8360bfbccff37bdc", "sd15"): 6267136.0,
+               ("8360bfbccff37bdc", "batched"): 24557952.0,
+               ("8360bfbccff37bdc", "large"): 70762496.0}
 
 
 def parse_args(argv=None):
