@@ -608,10 +608,17 @@ extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
   const SDev& d = h->d;
   const Stage st = current_stage(h);
   const int rows = st.kind == kFine ? d.B * d.N : d.B;
-  const int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
+  // column blocks per row: four columns per thread (at most 32 blocks), or
+  // more blocks when the stage has few rows (a coarse stage has only B), up to
+  // about two CTAs per SM in all and one column per thread
+  int gx = (int)((d.D + kSThreads * 4 - 1) / (kSThreads * 4));
+  if (gx > 32) gx = 32;
+  const int gsm = (2 * h->nsm + rows - 1) / rows;
+  const int gmax = (int)((d.D + kSThreads - 1) / kSThreads);
+  if (gsm > gx) gx = gsm < gmax ? gsm : gmax;
+  if (gx < 1) gx = 1;
   const int nset = (int)((h->g + 1) & 1);  // the next stage's distance set
-  cudaError_t e =
-      pa::launch_ex(k_srds_apply, dim3(gx < 32 ? gx : 32, rows), dim3(kSThreads), 0, h->st, 0, d, st, batch_eps, nset);
+  cudaError_t e = pa::launch_ex(k_srds_apply, dim3(gx, rows), dim3(kSThreads), 0, h->st, 0, d, st, batch_eps, nset);
   h->launches++;
   const int nstages = (h->iter == 0 ? 0 : d.s) + d.N;
   if (++h->stage == nstages) {  // the iteration is complete
