@@ -42,7 +42,7 @@ void set_error(const std::string& msg);  // pa_solver.cpp
 namespace {
 
 constexpr int kSThreads = 256;
-constexpr int kSStrip = 4096;        // columns per distance / error CTA
+constexpr int kSStrip = 1024;        // columns per error CTA
 constexpr int kSMaxRows = 2048;      // B * N
 
 enum StageKind : int32_t { kCoarseInit = 0, kFine = 1, kCoarse = 2 };
