@@ -1,33 +1,38 @@
-// Tile-parallel Picard update with bulk-copy staging, for sm_103a.
+// Picard update kernels for sm_103a, three forms of the same arithmetic.
 //
 // Same mathematics as the plain-load kernel (k_solver.cu): per window position
 // j (timestep i = t + j) Eq. 6 assembly, Eq. 7 cache update for misses, the
 // drift d_j = (c_i - 1) x_i + e_i eps_i at the current latent, the window
 // prefix sum of Eq. 1, the Eq. 2 error of state i+1 and the Eq. 4 distance of
-// timestep i+1 for the next iteration.
+// timestep i+1 for the next iteration. Every form reduces the per-lane Eq. 2
+// and Eq. 4 terms over its CTA in a fixed order and adds the CTA's sums into
+// the iteration's fp64 accumulators (red_add, pa_internal.h).
 //
 // Parallel structure. A CTA owns a strip of SEG = 32*V adjacent columns of one
-// trajectory and walks the window in tiles of TW = NW*S positions. The drifts
-// of different positions are independent; only their prefix sum couples them.
-// So within a tile warp w takes positions w*S .. w*S+S-1, forms its S drifts
-// and their local prefix, publishes its segment total, and after one CTA
-// barrier adds the carry (the running sum from x_t plus the totals of the
-// warps before it). All sums are carried as fp32 (hi, lo) pairs (TwoSum), so
-// the blocked order loses nothing against a sequential compensated sum.
+// trajectory. The drifts of different positions are independent; only their
+// prefix sum couples them. So warps take contiguous runs of positions, form
+// their drifts and the runs' totals, and after one CTA barrier add the carry
+// (the running sum from x_t plus the totals of the runs before theirs). All
+// sums are carried as fp32 (hi, lo) pairs (TwoSum), so the blocked order loses
+// nothing against a sequential compensated sum.
 //
-// Staging. Rows of a tile (per position: the eps row segment, from batch_eps
-// for a miss or ehat_i for a hit; the old state x_{i+1} unless it is a lazy
-// tail copy; xhat_{i+1} when timestep i+1 is a hit) are fetched with
-// cp.async.bulk (TMA engine, global -> shared) into one of nbuf tile buffers;
-// completion is counted on the buffer's mbarrier. Warp 0 issues a whole tile
-// at once, one lane per position. When the whole window fits in shared memory
-// (nbuf >= number of tiles) every copy is in flight right after the prologue;
-// otherwise the buffers are refilled as tiles retire.
+//   k_update_reg   each warp's run (at most LMAX positions) is loaded straight
+//                  into registers; no staging, no waits (default for four
+//                  columns per lane)
+//   k_update_seg   each warp's run is staged in shared memory by cp.async.bulk
+//                  (TMA engine) onto the warp's mbarrier (whole window per CTA)
+//   k_update_tile  the window walks in tiles of TW = NW*S positions through up
+//                  to 16 shared-memory tile buffers (windows too large for the
+//                  other two)
 //
-// Every mbarrier wait is bounded. A wait that runs out records kDevTimeout in
-// the solver's status word and stops further issues; the CTA finishes its
-// (now meaningless) arithmetic with in-bounds accesses only, drains the
-// copies already issued with bounded waits, and returns.
+// Staging (seg, tile). Rows (per position: the eps row segment, from
+// batch_eps for a miss or ehat_i for a hit; the old state x_{i+1} unless it is
+// a lazy tail copy; xhat_{i+1} when timestep i+1 is a hit) are fetched with
+// cp.async.bulk, one lane per row; completion is counted on mbarriers. Every
+// mbarrier wait is bounded. A wait that runs out records kDevTimeout in the
+// solver's status word and stops further issues; the CTA finishes its (now
+// meaningless) arithmetic with in-bounds accesses only, drains the copies
+// already issued with bounded waits, and returns.
 #include <cooperative_groups.h>
 
 #include "pa_bulk.cuh"
