@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {("8360bfbccff37bdc", "sd15"): 6267136.0,
-               ("8360bfbccff37bdc", "batched"): 24557952.0,
-               ("8360bfbccff37bdc", "large"): 70762496.0}
+NCU_TRAFFIC = {("fbf31a285cad9699", "sd15"): 6267136.0,
+               ("fbf31a285cad9699", "batched"): 24557952.0,
+               ("fbf31a285cad9699", "large"): 70762496.0}
 
 
 def parse_args(argv=None):
@@ -117,11 +117,17 @@ UPDATE_KERNEL_SOURCES = ("k_update_bulk.cu", "pa_bulk.cuh", "pa_internal.h")
 
 
 def kernel_source_sha():
+    """sha256-16 of the update kernel's sources with comments and whitespace
+    removed: it changes when the code changes, not when a comment does."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for name in UPDATE_KERNEL_SOURCES:
-        with open(os.path.join(ROOT, "paper_2609_36522_gb300", "csrc", name), "rb") as f:
-            h.update(f.read())
+        with open(os.path.join(ROOT, "paper_2609_36522_gb300", "csrc", name)) as f:
+            src = f.read()
+        src = re.sub(r"/\*.*?\*/", " ", src, flags=re.S)
+        src = re.sub(r"//[^\n]*", " ", src)
+        h.update("".join(src.split()).encode())
     return h.hexdigest()[:16]
 
 
