@@ -65,6 +65,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-kernel", type=int, default=None)
     ap.add_argument("--gmm-form", type=int, default=None, help="denoiser dot products: 1 tensor cores, 0 CUDA cores")
+    ap.add_argument("--cache-thresh", type=float, default=None,
+                    help="override the workload's tau_cache (the threshold sweep)")
     ap.add_argument("--cache-bits", type=int, default=32, choices=[16, 32],
                     help="storage of the cache entries: 32 fp32, 16 bfloat16")
     ap.add_argument("--oracle-sample", type=float, default=None, help=argparse.SUPPRESS)
@@ -310,6 +312,8 @@ def run_ours(args):
         pa_build.build()
     barrier()
     w = rank_workload(W.ALL[args.workload], rank)
+    if args.cache_thresh is not None:
+        w = w.with_(cache_thresh=args.cache_thresh)
     if w.sampler == "srds":
         return run_srds_bench(args, w)
     a, x0, mu = W.inputs(w)
@@ -467,6 +471,27 @@ def run_ours(args):
     launches = 2 * args.steps * (n_iters * kernels_per_iter + init_launches)   # both graphs, pa_init each
     cold_us = cold_iterations(max(1, min(args.steps, 10)))
 
+    # Quality check of the paper's kind with latents in place of CLIP scores:
+    # the cached result against serial DDIM, which is the same library with a
+    # window of one point and no cache (every step evaluated in order).
+    graph_plain.replay()
+    stream.synchronize()
+    assert s.poll() == 0
+    x_cached = s.result().cpu().numpy()
+    ser = Solver(w.T, 1, w.latent_shape, a, 0.0, 0.0, batch=w.batch, stream=stream)
+    if w.eta != 0.0:
+        ser.set_noise(w.eta, torch.from_numpy(W.noise(w)).to(dev))
+    ser.init(x_dev)
+    while True:
+        out = ser.step()
+        if out is None:
+            break
+        g.eps(out.batch_x_ptr, out.miss_bt_ptr, ser.n_miss_dev(), eps)
+        ser.submit_eps(eps)
+    x_serial = ser.result().cpu().numpy()
+    ser.close()
+    deviation = float((np.abs(x_cached - x_serial).max(axis=1) / np.abs(x_serial).max(axis=1)).max())
+
     units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
     value = units / secs
     gb_step = (upd_bytes.sum() + other_bytes.sum()) * args.steps / (dev_ms / 1000.0) / 1e9
@@ -553,6 +578,7 @@ def run_ours(args):
                                  "of the same generation, replayed alternately"},
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
+            "deviation_from_serial_ddim": deviation,
             "solver_step_gbps": gb_step,
             "denoiser_us_per_iteration": 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
             "solver_us_per_iteration": 1000.0 * dev_ms / max(1, args.steps * n_iters)
