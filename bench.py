@@ -719,6 +719,24 @@ def run_srds_bench(args, w):
                "d2h_bytes_per_step": int(w.batch * w.D * 4 + (polls // reps) * 24), "steps": reps,
                "api": f"pa_srds_init (host x_init), pa_srds_step_async + pa_gmm_eps + pa_srds_submit_eps in "
                       f"chunks of {E2E_CHUNK} stages, pa_srds_poll per chunk, pa_srds_result (host x_T)"}
+    # the sampled latents against serial DDIM (the Picard solver with a window
+    # of one point and no cache, same inputs and denoiser)
+    graph.replay()
+    stream.synchronize()
+    assert s.poll() == 0
+    x_srds = s.result().cpu().numpy()
+    from paper_2609_36522_gb300.solver import Solver
+    ser = Solver(w.T, 1, w.latent_shape, a, 0.0, 0.0, batch=w.batch, stream=stream)
+    ser.init(x_dev)
+    while True:
+        out = ser.step()
+        if out is None:
+            break
+        g.eps(out.batch_x_ptr, out.miss_bt_ptr, ser.n_miss_dev(), eps)
+        ser.submit_eps(eps)
+    x_serial = ser.result().cpu().numpy()
+    ser.close()
+    deviation = float((np.abs(x_srds - x_serial).max(axis=1) / np.abs(x_serial).max(axis=1)).max())
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         cpu = cpu_baseline(args.workload)
@@ -742,6 +760,7 @@ def run_srds_bench(args, w):
                        "timing": "CUDA events around each generation: one CUDA-graph replay of "
                                  "pa_srds_init and its stages"},
             "nfe_per_step": nfe, "hits_per_step": hits, "hit_rate": hits / max(1, hits + nfe),
+            "deviation_from_serial_ddim": deviation,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                          "frac": achieved / peak, "traffic": None,
                          "kernel": "whole evaluation stages (solver kernels and denoiser, one graph)",
