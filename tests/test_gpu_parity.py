@@ -98,6 +98,9 @@ def test_large_latent():
                tol=1e-3, cache_thresh=0.05, seed=13),
     W.Workload("64 trajectories", T=40, window=32, batch=64, latent_shape=(4, 4, 4), K=4,
                tol=1e-3, cache_thresh=0.05, seed=14),
+    # a 1000-point window: tiled update kernel, one-CTA planner (2 x 1000 pairs)
+    W.Workload("window 1000", T=1000, window=1000, batch=2, latent_shape=(4, 4, 4), K=3,
+               tol=1e-3, cache_thresh=0.05, seed=16),
 ], ids=lambda w: w.name)
 def test_edge_shapes(w):
     _check(w)

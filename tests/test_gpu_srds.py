@@ -103,3 +103,17 @@ def test_srds_async_equals_sync():
     b = gpu_srds(w, mode="async")
     assert np.array_equal(a["x_final"], b["x_final"])
     assert a["stats"]["nfe"] == b["stats"]["nfe"]
+
+
+@pytest.mark.parametrize("T,batch,shape", [(1, 2, (4, 4, 4)), (2, 1, (4, 8, 8)), (5, 3, (3, 5, 7)),
+                                           (17, 64, (4, 4, 4))])
+def test_srds_edge_shapes(T, batch, shape):
+    """Blocks of one step (T = 1, 2: a coarse jump and the fine step of its
+    block share a timestep, so the fine stage's new entry feeds the coarse
+    stage's distance in the same kernel), ragged blocks and odd D (T = 5), and
+    64 trajectories x 5 blocks of rows."""
+    w = W.TINY.with_(T=T, latent_shape=shape, K=3, sampler="srds", batch=batch, seed=31)
+    orc = oracle_srds(w)
+    compare_srds(w, orc, gpu_srds(w))
+    g = gpu_srds(w, mode="async")
+    assert g["stats"]["nfe"] == orc.nfe
