@@ -375,6 +375,7 @@ def bf16_tolerance(w, orc):
                tol=1e-3, cache_thresh=0.05, seed=3),
     W.Workload("window 128", T=150, window=128, batch=1, latent_shape=(4, 16, 16), K=4,
                tol=1e-3, cache_thresh=0.05, seed=15),
+    W.TINY.with_(T=60, window=16, latent_shape=(4, 8, 8), eta=1.0, seed=3, name="stochastic steps"),
 ], ids=lambda w: w.name)
 def test_bf16_cache_entries(w):
     """Entries stored as bfloat16 on both sides: decisions, miss lists and NFE
@@ -382,7 +383,8 @@ def test_bf16_cache_entries(w):
     a neighbouring bfloat16 value when the GPU's fp32 value and the oracle's
     fp64 value straddle a rounding boundary), final latents within the bound of
     bf16_tolerance (about 1.6e-3 at T = 100). The register form runs where it
-    applies, the plain-load kernel elsewhere (odd D, window 128)."""
+    applies, the plain-load kernel elsewhere (odd D, window 128, stochastic
+    steps)."""
     from oracle.storage import round_bf16
     orc = oracle_run(w, cache_store=round_bf16)
     assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-3), decision_margins(orc, w.tol, w.cache_thresh)
