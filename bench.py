@@ -115,7 +115,7 @@ def measured_hbm_gbs():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-UPDATE_KERNEL_SOURCES = ("k_update_bulk.cu", "pa_bulk.cuh", "pa_internal.h")
+UPDATE_KERNEL_SOURCES = ("k_update_bulk.cu", "k_update_lean.cu", "pa_bulk.cuh", "pa_internal.h")
 
 
 def kernel_source_sha():
@@ -504,8 +504,8 @@ def run_ours(args):
     traffic = NCU_TRAFFIC.get((sha, args.workload + ("-bf16" if args.cache_bits == 16 else "")))
     roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "traffic": traffic,
-                "kernel": "Picard update (" + ("register-resident or staged form, by shape" if st1["update_kernel"] == 1
-                                               else "plain loads") + ")",
+                "kernel": "Picard update (" + {2: "lean register form", 1: "register-resident or staged form, by shape"}
+                .get(st1["update_kernel"], "plain loads") + ")",
                 "traffic_note": "ncu dram read+write bytes per launch, averaged over one generation",
                 "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
                 "alg_bytes_per_launch": float(upd_bytes.mean()),

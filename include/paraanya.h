@@ -74,8 +74,8 @@ typedef struct {
   int32_t n_active;      /* trajectories with t < T */
   int32_t n_miss;        /* misses planned for the next iteration */
   int32_t device_status; /* 0, or the first device-side error code */
-  int32_t update_kernel; /* kernel of the last pa_submit_eps: 0 plain loads, 1 bulk-copy
-                            pipeline, -1 none yet */
+  int32_t update_kernel; /* kernel of the last pa_submit_eps: 0 plain loads, 1 bulk forms,
+                            2 lean register form, -1 none yet */
 } pa_stats_t;
 
 /* ---- solver ------------------------------------------------------------ */
@@ -183,13 +183,24 @@ PA_API pa_status pa_iter_log(pa_solver* s, int32_t* out, int max_iters, int* n_i
  * Either pointer may be NULL. Synchronises. */
 PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out);
 
-/* Select the Picard-update kernel: 0 = plain loads, 1 = bulk-copy pipeline
- * (default when D % 4 == 0; it falls back to plain loads for a batch_eps
- * pointer that is not 16-byte aligned), 100 + n = bulk-copy pipeline with
- * launch shape n (0..11; columns per lane, warps per CTA, pipeline depth --
- * a tuning aid), 112 = the register-resident form (rows loaded straight into
- * registers; windows up to 104 points, 64 with stochastic steps, else the
- * tiled pipeline). Returns PA_ERR_ARG for an unknown value. */
+/* Select the Picard-update kernel (all forms compute Eq. 1, 2, 4, 6 and 7 of
+ * one iteration; they differ in rounding order only, never in a decision
+ * beyond the decision-margin guard):
+ *   0       plain loads (one thread per column; any D);
+ *   1       the bulk forms: register-resident rows, or rows staged in shared
+ *           memory by bulk copies for windows the registers cannot hold;
+ *   2       the lean register form (default when D % 4 == 0): 16-byte rows
+ *           straight into registers, plain fp32 prefix sums, coefficients and
+ *           ranks staged in shared memory; windows up to 112 points with
+ *           deterministic steps, else it falls back to 1;
+ *   100 + n bulk forms with launch shape n (0..12; columns per lane, warps per
+ *           CTA, pipeline depth; 112 = the register-resident form);
+ *   200 + n lean form with launch shape n: 0 by window, 1 = 16 warps x 7
+ *           positions, 2 = 12 x 9, 3 = 8 x 4 and 4 = 8 x 8 (two CTAs per SM);
+ *           210 + n the same with compensated (TwoSum) sums, deterministic
+ *           steps only. A shape that cannot hold the window falls back to 1.
+ * Forms 1 and 2 fall back to plain loads for a batch_eps pointer that is not
+ * 16-byte aligned. A tuning aid; returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
 
 /* Storage precision of the cache entries (xhat, ehat of Eq. 3): 32 = fp32

@@ -300,8 +300,8 @@ struct RedSums {
   const double* e;
   const double* dl;
   double inv_d;
-  __device__ double err(int q) const { return __ldcg(e + q) * inv_d; }
-  __device__ double del(int q) const { return __ldcg(dl + q) * inv_d; }
+  __device__ double err(int q) const { return __ldcg(e + (size_t)q * kAccStride) * inv_d; }
+  __device__ double del(int q) const { return __ldcg(dl + (size_t)q * kAccStride) * inv_d; }
 };
 
 template <int VEC>
@@ -314,19 +314,20 @@ __global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
   decide_load<kPlanThreads>(d, ds, par);
   pdl_wait();  // the sums and the new states come from the update kernel
   pdl_trigger();  // the successor may now run its prologue
-  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair;
-  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair;
+  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
+  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
   const double inv_d = 1.0 / (double)d.D;
   for (int q = tid; q < npair; q += kPlanThreads) {
-    const double ve = __ldcg(acc_e + q) * inv_d, vd = __ldcg(acc_d + q) * inv_d;
+    const size_t o = (size_t)q * kAccStride;
+    const double ve = __ldcg(acc_e + o) * inv_d, vd = __ldcg(acc_d + o) * inv_d;
     s_e[q] = ve;
     s_d[q] = vd;
     if (publish) {
       d.red_err[q] = (float)ve;
       d.red_del[q] = (float)vd;
-      double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair;  // iteration k+1 adds into these
-      nxt[q] = 0.0;
-      nxt[npair + q] = 0.0;
+      double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;  // iteration k+1 adds into these
+      nxt[o] = 0.0;
+      nxt[(size_t)npair * kAccStride + o] = 0.0;
     }
   }
   __syncthreads();  // the sums and decide_load's state are staged
@@ -348,16 +349,16 @@ __global__ void __launch_bounds__(kPlanOneThreads) k_plan_one(Dev d, int par) {
   decide_load<kPlanOneThreads>(d, ds, par);
   pdl_wait();  // the sums come from the update kernel
   pdl_trigger();  // the successor may now run its prologue
-  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair;
-  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair;
+  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
+  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
   const RedSums red{acc_e, acc_d, 1.0 / (double)d.D};
   decide_run<kPlanOneThreads>(d, ds, red, par, true, -1);
-  double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair;
+  double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;
   for (int q = threadIdx.x; q < npair; q += kPlanOneThreads) {
     d.red_err[q] = (float)red.err(q);
     d.red_del[q] = (float)red.del(q);
-    nxt[q] = 0.0;
-    nxt[npair + q] = 0.0;
+    nxt[(size_t)q * kAccStride] = 0.0;
+    nxt[((size_t)npair + q) * kAccStride] = 0.0;
   }
 }
 

@@ -12,7 +12,12 @@ namespace pa {
 constexpr int kMaxWindow = 1024;
 constexpr int kMaxBatch = 64;
 constexpr size_t kAlign = 256;
+// Doubles from one fp64 accumulator (Eq. 2 / Eq. 4 sums) to the next: each
+// sits on its own 128-byte line, so the atomic adds of many CTAs into
+// different window positions do not queue behind one another on a line.
+constexpr int kAccStride = 16;
 constexpr int kBulkConfigs = 13;    // launch shapes of the bulk-copy update kernel
+constexpr int kLeanConfigs = 15;    // launch shapes of the lean register update kernel (0..4, 10..14)
 
 // Device status codes written by kernels (first error wins, atomicCAS from 0).
 constexpr int kDevOk = 0;
@@ -76,7 +81,7 @@ inline Layout make_layout(int T, int P, int64_t D, int B) {
   L.ctl = take(sizeof(Ctl));
   L.rank = take((size_t)B * P * sizeof(int32_t));
   L.miss_bt = take((size_t)B * P * 2 * sizeof(int32_t));
-  L.acc = take((size_t)2 * 2 * B * P * sizeof(double));  // [set][err, dist][B][P]
+  L.acc = take((size_t)2 * 2 * B * P * kAccStride * sizeof(double));  // [set][err, dist][B][P], strided
   L.red_err = take((size_t)B * P * sizeof(float));
   L.red_del = take((size_t)B * P * sizeof(float));
   L.iter_log = take((size_t)(T + 1) * B * kLogFields * sizeof(int32_t));
@@ -99,7 +104,7 @@ struct Dev {
   Ctl* ctl;
   int32_t* rank;      // [B][P] rank of window position j among the misses, -1 = hit
   int32_t* miss_bt;   // [B*P][2]
-  double* acc;        // [2][2][B][P]: sums of Eq. 2 and Eq. 4 terms; set k mod 2 in iteration k
+  double* acc;        // [2][2][B][P] x kAccStride: sums of Eq. 2 and Eq. 4 terms; set k mod 2 in iteration k
   float* red_err;     // [B][P] the last decision's reductions (divided by D), for the host
   float* red_del;
   int32_t* iter_log;  // [T+1][B][kLogFields]
@@ -193,7 +198,7 @@ struct Bf16Row<1> {
 // iteration's parity. fp64 sums of fp32 CTA partials: the rounding of the
 // order in which CTAs arrive is far below the fp32 partials' own.
 __device__ __forceinline__ void red_add(const Dev& d, int par, int which, int q, float v) {
-  atomicAdd(d.acc + ((size_t)(par * 2 + which) * d.B * d.P + q), (double)v);
+  atomicAdd(d.acc + ((size_t)(par * 2 + which) * d.B * d.P + q) * kAccStride, (double)v);
 }
 
 // Kernel launchers (k_solver.cu). Each returns the launch error. par = k mod 2
@@ -207,5 +212,9 @@ cudaError_t launch_plan(const Dev& d, int par, cudaStream_t st, int* launches);
 // k_update_bulk.cu
 cudaError_t launch_update_bulk(const Dev& d, const float* batch_eps, int par, cudaStream_t st);
 bool update_bulk_supported(const Dev& d, const float* batch_eps);
+// k_update_lean.cu; shape: see launch_update_lean (cudaErrorNotSupported when
+// the shape cannot hold the window)
+cudaError_t launch_update_lean(const Dev& d, const float* batch_eps, int par, int shape, cudaStream_t st);
+bool update_lean_supported(const Dev& d, const float* batch_eps);
 
 }  // namespace pa

@@ -40,7 +40,8 @@ struct pa_solver {
   char* ws;
   cudaStream_t st;
   St state;
-  int update_kind;   // requested: 0 plain, 1 bulk pipeline
+  int update_kind;   // requested: 0 plain, 1 bulk pipeline, 2 lean register form
+  int lean_shape;    // launch shape of the lean register form
   int last_kind;     // kernel the last pa_submit_eps actually launched (-1: none yet)
   int64_t k;         // pa_submit_eps calls since pa_init: the plan of iteration k is copy k mod 2
   int64_t launches;
@@ -189,6 +190,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   s->launches = 0;
   s->k = 0;
   s->last_kind = -1;
+  s->lean_shape = 0;
   char* w = s->ws;
   pa::Dev& d = s->d;
   d.X = reinterpret_cast<float*>(w + L.X);
@@ -216,7 +218,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.cache_thresh = cache_thresh;
   d.wait_limit = pa::kWaitLimit;
   d.cache_bf16 = 0;
-  s->update_kind = (D % 4 == 0) ? 1 : 0;
+  s->update_kind = (D % 4 == 0) ? 2 : 0;  // lean register form, else the bulk forms, else plain loads
 
   const std::vector<float> hc = step_coefficients(s->alphas, 0.0);  // DDIM (eta = 0)
   cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), sizeof(pa::Ctl), cudaHostAllocDefault);
@@ -264,7 +266,7 @@ pa_status pa_init(pa_solver* s, const float* x_init) {
                                     cudaMemcpyDefault, s->st);
   if (e != cudaSuccess) return cuda_fail("pa_init: copy x_init", e);
   // both accumulator sets of the reductions start at zero
-  e = cudaMemsetAsync(d.acc, 0, (size_t)2 * 2 * d.B * d.P * sizeof(double), s->st);
+  e = cudaMemsetAsync(d.acc, 0, (size_t)2 * 2 * d.B * d.P * pa::kAccStride * sizeof(double), s->st);
   if (e != cudaSuccess) return cuda_fail("pa_init: clear sums", e);
   // the first plan (every timestep a first entry) and its batch
   e = pa::launch_init_plan(d, s->st);
@@ -328,7 +330,18 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
     if (e == cudaSuccess) e = record_timing_event(s->ev[2 * s->ev_next], s->st);
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
   }
-  if (s->update_kind == 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
+  bool done = false;
+  if (s->update_kind == 2 && pa::update_lean_supported(s->d, batch_eps_dev)) {
+    e = pa::launch_update_lean(s->d, batch_eps_dev, par, s->lean_shape, s->st);
+    if (e == cudaErrorNotSupported) {
+      e = cudaSuccess;  // this shape cannot hold the window: the bulk forms below
+    } else {
+      s->last_kind = 2;
+      done = true;
+    }
+  }
+  if (done) {
+  } else if (s->update_kind >= 1 && pa::update_bulk_supported(s->d, batch_eps_dev)) {
     e = pa::launch_update_bulk(s->d, batch_eps_dev, par, s->st);
     s->last_kind = 1;
   } else {
@@ -429,14 +442,19 @@ pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out) {
 
 pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   if (!s) return arg_fail("pa_set_update_kernel: solver is NULL");
-  if (kind == 0 || kind == 1) {
+  if (kind == 0 || kind == 1 || kind == 2) {
     s->update_kind = kind;
+    s->lean_shape = 0;
     s->d.bulk_cfg = 0;
   } else if (kind >= 100 && kind < 100 + pa::kBulkConfigs) {
     s->update_kind = 1;
     s->d.bulk_cfg = kind - 100;
+  } else if (kind >= 200 && kind < 200 + pa::kLeanConfigs && (kind - 200) % 10 <= 4) {
+    s->update_kind = 2;
+    s->lean_shape = kind - 200;
+    s->d.bulk_cfg = 0;
   } else {
-    return arg_fail("pa_set_update_kernel: kind must be 0, 1 or 100 + launch shape");
+    return arg_fail("pa_set_update_kernel: kind must be 0, 1, 2, 100 + bulk launch shape or 200 + lean launch shape");
   }
   return PA_OK;
 }
