@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {("fbf31a285cad9699", "sd15"): 6267136.0,
-               ("fbf31a285cad9699", "batched"): 24557952.0,
-               ("fbf31a285cad9699", "large"): 70762496.0}
+NCU_TRAFFIC = {("0f3c656eafda7fd5", "sd15"): 6251072.0,
+               ("0f3c656eafda7fd5", "batched"): 24608597.0,
+               ("0f3c656eafda7fd5", "large"): 70587502.0}
 
 
 def parse_args(argv=None):

@@ -66,7 +66,7 @@ struct SDev {
   int32_t* miss_bt;  // [B*N][2]
   int32_t* rank;     // [B*N]: miss rank, -1 hit, -2 not live
   double* part;      // [B*N][nstrip] Eq. 2 partials of the block boundaries
-  double* sacc;      // [2][B*N] Eq. 4 sums of the next stage's rows, set = stage number mod 2
+  double* sacc;      // [2][B*N] x kAccStride: Eq. 4 sums of the next stage's rows, set = stage number mod 2
   int32_t* active;   // [B]
   int32_t* iters;    // [B]
   float* err_log;    // [N][B]
@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(kSThreads) k_srds_plan_gather(SDev d, Stage st
       double* x = nullptr;
       const bool live = r < rows && row_info(d, st, r, b, n, i, x);
       bool hit = false;
-      if (live && d.has[(int64_t)b * d.T + i]) hit = d.sacc[(size_t)set * R + r] / (double)d.D < d.cache_thresh;
+      if (live && d.has[(int64_t)b * d.T + i]) hit = d.sacc[((size_t)set * R + r) * pa::kAccStride] / (double)d.D < d.cache_thresh;
       const bool miss = live && !hit;
       const unsigned mm = __ballot_sync(0xffffffffu, miss);
       const int rank = base + __popc(mm & ((1u << lane) - 1u));
@@ -170,7 +170,7 @@ __global__ void __launch_bounds__(kSThreads) k_srds_plan_gather(SDev d, Stage st
       }
     }
     if (publish)
-      for (int q = lane; q < R; q += 32) d.sacc[(size_t)(set ^ 1) * R + q] = 0.0;
+      for (int q = lane; q < R; q += 32) d.sacc[((size_t)(set ^ 1) * R + q) * pa::kAccStride] = 0.0;
   }
   __syncthreads();
   const int m = blockIdx.y, r = s_row;
@@ -252,7 +252,7 @@ __global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, cons
   }
   if (nhas) {
     const double t = block_sum(dist, s_w);
-    if (threadIdx.x == 0) atomicAdd(d.sacc + (size_t)nset * d.B * d.N + nrow, t);
+    if (threadIdx.x == 0) atomicAdd(d.sacc + ((size_t)nset * d.B * d.N + nrow) * pa::kAccStride, t);
   }
 }
 
@@ -288,7 +288,7 @@ __global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter, int ns
   if (nhas) {
     __syncthreads();  // s_w is reused
     const double t2 = block_sum(dist, s_w);
-    if (threadIdx.x == 0) atomicAdd(d.sacc + (size_t)nset * d.B * d.N + r, t2);
+    if (threadIdx.x == 0) atomicAdd(d.sacc + ((size_t)nset * d.B * d.N + r) * pa::kAccStride, t2);
   }
 }
 
@@ -382,7 +382,7 @@ SLayout s_layout(int T, int64_t D, int B, int N, int nstrip) {
   L.miss_bt = take((size_t)B * N * 2 * sizeof(int32_t));
   L.rank = take((size_t)B * N * sizeof(int32_t));
   L.part = take((size_t)B * N * nstrip * sizeof(double));
-  L.sacc = take((size_t)2 * B * N * sizeof(double));
+  L.sacc = take((size_t)2 * B * N * pa::kAccStride * sizeof(double));  // one 128-byte line per sum
   L.active = take((size_t)B * sizeof(int32_t));
   L.iters = take((size_t)B * sizeof(int32_t));
   L.err_log = take((size_t)N * B * sizeof(float));
@@ -546,7 +546,7 @@ extern "C" pa_status pa_srds_init(pa_srds* h, const float* x_init) {
   e = pa::launch_ex(k_srds_load, dim3(32, d.B), dim3(256), 0, h->st, 0, d, (const float*)d.batch_x, 0);
   if (e == cudaSuccess) e = pa::launch_ex(k_srds_reset, dim3(1), dim3(256), 0, h->st, 0, d);
   h->launches += 2;
-  if (e == cudaSuccess) e = cudaMemsetAsync(d.sacc, 0, (size_t)2 * d.B * d.N * sizeof(double), h->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(d.sacc, 0, (size_t)2 * d.B * d.N * pa::kAccStride * sizeof(double), h->st);
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_init: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   h->iter = 0;
   h->stage = 0;

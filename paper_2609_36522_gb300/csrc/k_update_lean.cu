@@ -226,14 +226,27 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
     if (warp == 0) {
       c = x[0];
     } else {
-      for (int w = 0; w < warp; ++w) {
-        const float4 v = s_tot[w * 32 + lane];
-        if constexpr (COMP) {
-          const float4 u = s_lo[w * 32 + lane];
-          two_sum2p(c.l, cl.l, make_float2(v.x, v.y), make_float2(u.x, u.y));
-          two_sum2p(c.h, cl.h, make_float2(v.z, v.w), make_float2(u.z, u.w));
-        } else {
-          c = qadd(c, Q{make_float2(v.x, v.y), make_float2(v.z, v.w)});
+      // earlier runs' totals in order, fetched four at a time so that the
+      // shared-memory latency is paid once per group, not once per run
+      for (int w0 = 0; w0 < warp; w0 += 4) {
+        float4 v[4], u[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (w0 + q < warp) {
+            v[q] = s_tot[(w0 + q) * 32 + lane];
+            if constexpr (COMP) u[q] = s_lo[(w0 + q) * 32 + lane];
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          if (w0 + q < warp) {
+            if constexpr (COMP) {
+              two_sum2p(c.l, cl.l, make_float2(v[q].x, v[q].y), make_float2(u[q].x, u[q].y));
+              two_sum2p(c.h, cl.h, make_float2(v[q].z, v[q].w), make_float2(u[q].z, u[q].w));
+            } else {
+              c = qadd(c, Q{make_float2(v[q].x, v[q].y), make_float2(v[q].z, v[q].w)});
+            }
+          }
         }
       }
     }
