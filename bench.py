@@ -439,6 +439,29 @@ def run_ours(args):
                 n += 1
         return 1000.0 * tot / max(n, 1)
 
+    def timing_floor(reps=50):
+        """Event-pair time around a kernel that does no work (a one-element
+        fill), captured between two kernels in a graph like the update kernel's
+        events: the launch and completion latency inside every event-timed
+        launch."""
+        t1 = torch.zeros(1, device=dev)
+        ev = (torch.cuda.Event(enable_timing=True, external=True),
+              torch.cuda.Event(enable_timing=True, external=True))
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=stream):
+            t1.add_(1.0)
+            ev[0].record(stream)
+            t1.fill_(0.0)
+            ev[1].record(stream)
+            t1.add_(1.0)
+        tot = 0.0
+        for r in range(reps + 3):
+            gr.replay()
+            stream.synchronize()
+            if r >= 3:
+                tot += ev[0].elapsed_time(ev[1])
+        return 1000.0 * tot / reps
+
     for _ in range(args.warmup):
         generation(graph_plain, False)
         generation(graph_timed, True)
@@ -470,6 +493,7 @@ def run_ours(args):
     clk = clocks.stop()
     launches = 2 * args.steps * (n_iters * kernels_per_iter + init_launches)   # both graphs, pa_init each
     cold_us = cold_iterations(max(1, min(args.steps, 10)))
+    floor_us = timing_floor()
 
     # Quality check of the paper's kind with latents in place of CLIP scores:
     # the cached result against serial DDIM, which is the same library with a
@@ -509,7 +533,13 @@ def run_ours(args):
                 "traffic_note": "ncu dram read+write bytes per launch, averaged over one generation",
                 "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
                 "alg_bytes_per_launch": float(upd_bytes.mean()),
-                "avg_launch_us": 1000.0 * upd_ms / max(n_upd, 1)}
+                "avg_launch_us": 1000.0 * upd_ms / max(n_upd, 1),
+                "timing_floor_us": floor_us,
+                "timing_floor_note": "event-pair time of a one-element fill at the same place in a graph: "
+                                     "launch and completion latency that every event-timed launch includes; "
+                                     "frac_excl_floor divides the bytes by avg_launch_us minus it"}
+    net_us = roofline["avg_launch_us"] - floor_us
+    roofline["frac_excl_floor"] = (float(upd_bytes.mean()) / (net_us * 1e-6) / 1e9 / peak) if net_us > 0 else None
 
     # End to end through the public API with host buffers (no graph, no flush):
     # x_init copied in from pinned host memory, iterations issued with the
