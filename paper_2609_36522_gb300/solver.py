@@ -119,6 +119,9 @@ class Solver:
         return abi.pa_last_reductions(self.h, self.batch, self.window)
 
     def set_update_kernel(self, kind):
+        """Picard-update kernel: 0 plain loads, 1 bulk forms, 2 lean register
+        form (the default), 100 + n / 200 + n launch shapes of the bulk / lean
+        forms (a tuning aid; pa_set_update_kernel documents them)."""
         abi.pa_set_update_kernel(self.h, kind)
 
     def set_cache_precision(self, bits):

@@ -52,6 +52,7 @@ def test_tiny_with_oracle_eps():
 def test_sd15_full_size():
     orc, gpu = _check(W.SD15)
     assert gpu["stats"]["hits"] > 0
+    assert gpu["stats"]["update_kernel"] == 2  # the lean register form is the default
 
 
 def test_sd15_uncached_equals_oracle_uncached():
@@ -328,6 +329,20 @@ def test_lean_update(kind, window, eta):
     assert np.array_equal(ref["log"], got["log"])
     scale = np.abs(ref["x_final"]).max()
     assert np.abs(ref["x_final"] - got["x_final"]).max() <= 1e-5 * scale
+
+
+@pytest.mark.parametrize("kind,eta", [(200, 0.0), (204, 0.0), (201, 1.0), (204, 1.0)])
+def test_lean_update_long_schedule(kind, eta):
+    """A 1000-step schedule: every CTA stages 1000 coefficient sets (two per
+    thread and more) before the plan is known; decisions exact, latents
+    within 1e-5 of the oracle."""
+    w = W.Workload("lean-long", T=1000, window=64, batch=1, latent_shape=(4, 16, 16), K=4,
+                   tol=1e-3, cache_thresh=0.05, seed=3, eta=eta)
+    orc = oracle_run(w)
+    assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-6), decision_margins(orc, w.tol, w.cache_thresh)
+    got = gpu_run(w, update_kernel=kind)
+    assert got["stats"]["update_kernel"] == 2
+    assert compare(w, orc, got).max() <= REL_TOL
 
 
 # ---- stochastic steps (eta > 0): DDPM over the full 1000-step schedule -------
