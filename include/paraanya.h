@@ -113,8 +113,9 @@ PA_API pa_status pa_create(pa_solver** out, int T, int window,
  * that long. eta = 0 (noise_dev may be NULL) restores plain DDIM. eta must be
  * in [0, 1]. Not allowed between pa_step and pa_submit_eps (PA_ERR_STATE);
  * takes effect from the next iteration (call pa_init to restart cleanly).
- * The bulk-copy update kernel stages the draws when D % 4 == 0 and the window
- * fits its shared memory; otherwise the plain-load kernel runs.
+ * With draws the default update is the register-resident bulk form (or the
+ * staged bulk form, which copies the draws into shared memory) when
+ * D % 4 == 0 and the window fits; otherwise the plain-load kernel runs.
  * Synchronises the solver's stream. */
 PA_API pa_status pa_set_noise(pa_solver* s, double eta, const float* noise_dev);
 
@@ -147,8 +148,8 @@ PA_API pa_status pa_step_async(pa_solver* s, const float** batch_x_dev,
 PA_API const int32_t* pa_n_miss_dev(const pa_solver* s);
 
 /* Hand back eps_theta for the planned misses: batch_eps_dev [M][D] fp32,
- * DEVICE pointer, 16-byte alignment for the bulk-copy pipeline (otherwise the
- * plain-load kernel runs). Runs Eq. 6 (assembly), Eq. 7 (cache update),
+ * DEVICE pointer, 16-byte aligned for the lean and bulk update forms
+ * (otherwise the plain-load kernel runs). Runs Eq. 6 (assembly), Eq. 7 (cache update),
  * the drift and the Picard prefix sum (Eq. 1), the errors of Eq. 2 and the
  * cache distances of the next iteration (Eq. 4) in the update kernel, then the
  * window advance, the hit-miss plan of the next iteration (Eq. 5) and the
