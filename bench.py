@@ -48,9 +48,9 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {("0f3c656eafda7fd5", "sd15"): 6251072.0,
-               ("0f3c656eafda7fd5", "batched"): 24608597.0,
-               ("0f3c656eafda7fd5", "large"): 70587502.0}
+NCU_TRAFFIC = {("c44ead84a091f784", "sd15"): 6248768.0,
+               ("c44ead84a091f784", "batched"): 24594133.0,
+               ("c44ead84a091f784", "large"): 70679881.0}
 
 
 def parse_args(argv=None):

@@ -197,9 +197,11 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
  *   100 + n bulk forms with launch shape n (0..12; columns per lane, warps per
  *           CTA, pipeline depth; 112 = the register-resident form);
  *   200 + n lean form with launch shape n: 0 by window, 1 = 16 warps x 7
- *           positions, 2 = 12 x 9, 3 = 8 x 4 and 4 = 8 x 8 (two CTAs per SM);
- *           210 + n the same with compensated (TwoSum) sums, deterministic
- *           steps only. A shape that cannot hold the window falls back to 1.
+ *           positions, 2 = 12 x 9, 3 = 8 x 4 and 4 = 8 x 8 (two CTAs per SM),
+ *           5 = 8 x 4 (three CTAs per SM), 6 = 4 x 8 (four CTAs per SM);
+ *           210 + n (n <= 4) the same with compensated (TwoSum) sums,
+ *           deterministic steps only. Shapes 5 and 6 take deterministic steps
+ *           only. A shape that cannot hold the window falls back to 1.
  * Forms 1 and 2 fall back to plain loads for a batch_eps pointer that is not
  * 16-byte aligned. A tuning aid; returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);

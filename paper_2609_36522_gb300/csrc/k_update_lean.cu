@@ -323,23 +323,27 @@ constexpr size_t kLeanSmemMax = 200 * 1024;
 }  // namespace
 
 // Lean launch shapes (shape % 10): 0 = by window (deterministic steps only),
-// 1 = 16 warps x 7 positions,
-// 2 = 12 x 9, 3 = 8 x 4 (two CTAs per SM), 4 = 8 x 8 (two CTAs per SM);
-// shape >= 10: compensated sums (deterministic steps only).
-// Returns cudaErrorNotSupported when the shape cannot hold the window.
+// 1 = 16 warps x 7 positions (one CTA per SM), 2 = 12 x 9, 3 = 8 x 4 and
+// 4 = 8 x 8 (two CTAs per SM), 5 = 8 x 4 (three CTAs per SM), 6 = 4 x 8 (four
+// CTAs per SM); shape >= 10: compensated sums (shapes 1-4, deterministic steps
+// only). Returns cudaErrorNotSupported when the shape cannot hold the window.
 cudaError_t launch_update_lean(const Dev& d, const float* batch_eps, int par, int shape, cudaStream_t st) {
   const bool comp = shape >= 10;
   int s = shape % 10;
   if (s == 0) {
-    // by window: two CTAs per SM while a warp's run of the window stays short,
-    // else 16 warps of at most 7 positions (one CTA per SM). Stochastic steps
-    // keep the register-resident bulk form, measured faster for them.
+    // by window: as many CTAs per SM as the registers allow without spilling
+    // (three of 8 x 4, two of 8 x 8), else 16 warps of at most 7 positions
+    // (one CTA per SM). Stochastic steps keep the register-resident bulk form,
+    // measured faster for them.
     if (d.noise) return cudaErrorNotSupported;
-    s = d.P <= 32 ? 3 : d.P <= 64 ? 4 : 1;
+    s = d.P <= 32 ? (comp ? 3 : 5) : d.P <= 64 ? 4 : 1;
   }
-  const int nw = s == 1 ? 16 : s == 2 ? 12 : 8;
-  const int lmax = s == 1 ? 7 : s == 2 ? 9 : s == 3 ? 4 : 8;
-  if (s > 4 || d.P > nw * lmax) return cudaErrorNotSupported;
+  static const int kWarps[7] = {0, 16, 12, 8, 8, 8, 4};
+  static const int kRun[7] = {0, 7, 9, 4, 8, 4, 8};
+  if (s > 6 || d.P > kWarps[s] * kRun[s]) return cudaErrorNotSupported;
+  if (s >= 5 && (comp || d.noise)) return cudaErrorNotSupported;
+  if (s == 5) return launch_lean<8, 4, 3, false, false>(d, batch_eps, par, st);
+  if (s == 6) return launch_lean<4, 8, 4, false, false>(d, batch_eps, par, st);
   if (d.noise) {
     if (comp) return cudaErrorNotSupported;
     if (s == 1) return launch_lean<16, 7, 1, true, false>(d, batch_eps, par, st);

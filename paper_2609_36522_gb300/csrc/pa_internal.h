@@ -17,7 +17,7 @@ constexpr size_t kAlign = 256;
 // different window positions do not queue behind one another on a line.
 constexpr int kAccStride = 16;
 constexpr int kBulkConfigs = 13;    // launch shapes of the bulk-copy update kernel
-constexpr int kLeanConfigs = 15;    // launch shapes of the lean register update kernel (0..4, 10..14)
+constexpr int kLeanConfigs = 17;    // launch shapes of the lean register update kernel (0..6, 10..16)
 
 // Device status codes written by kernels (first error wins, atomicCAS from 0).
 constexpr int kDevOk = 0;

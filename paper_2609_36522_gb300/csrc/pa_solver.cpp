@@ -449,7 +449,7 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   } else if (kind >= 100 && kind < 100 + pa::kBulkConfigs) {
     s->update_kind = 1;
     s->d.bulk_cfg = kind - 100;
-  } else if (kind >= 200 && kind < 200 + pa::kLeanConfigs && (kind - 200) % 10 <= 4) {
+  } else if (kind >= 200 && kind < 200 + pa::kLeanConfigs && (kind - 200) % 10 <= 6) {
     s->update_kind = 2;
     s->lean_shape = kind - 200;
     s->d.bulk_cfg = 0;

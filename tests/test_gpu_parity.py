@@ -302,11 +302,11 @@ def test_register_update_matches_staged(window, eta):
 
 # ---- lean register update kernel (launch shapes 200 + n) ---------------------
 
-LEAN_SHAPES = {0: None, 1: (16, 7), 2: (12, 9), 3: (8, 4), 4: (8, 8)}
+LEAN_SHAPES = {0: None, 1: (16, 7), 2: (12, 9), 3: (8, 4), 4: (8, 8), 5: (8, 4), 6: (4, 8)}
 _LEAN_REF = {}
 
 
-@pytest.mark.parametrize("kind", [200, 201, 202, 203, 204, 210, 211, 212, 213, 214])
+@pytest.mark.parametrize("kind", [200, 201, 202, 203, 204, 205, 206, 210, 211, 212, 213, 214])
 @pytest.mark.parametrize("T,window,eta", [(100, 24, 0.0), (100, 64, 0.0), (100, 100, 0.0), (100, 32, 1.0),
                                           (100, 64, 0.5), (150, 112, 0.0), (150, 113, 0.0)])
 def test_lean_update(kind, T, window, eta):
@@ -315,8 +315,9 @@ def test_lean_update(kind, T, window, eta):
     with the plain-load kernel within 1e-5 of the latents' scale, on a ragged
     last strip; a shape that cannot hold the window (or, with stochastic
     steps, compensated sums or the by-window choice) falls back to the bulk
-    forms. Windows of 112 and 113 points are the 16 x 7 shape's capacity and
-    one past it."""
+    forms, as do shapes 5 and 6 (three and four CTAs per SM) with draws.
+    Windows of 112 and 113 points are the 16 x 7 shape's capacity and one
+    past it."""
     w = W.Workload("lean", T=T, window=window, batch=2, latent_shape=(4, 20, 20), K=6,
                    tol=1e-3, cache_thresh=0.05, seed=5, eta=eta)
     if (T, window, eta) not in _LEAN_REF:  # the oracle and the plain-load run, once per case
@@ -326,7 +327,7 @@ def test_lean_update(kind, T, window, eta):
     P = min(window, T)
     shape = LEAN_SHAPES[kind % 10] or ((8, 4) if P <= 32 else (8, 8) if P <= 64 else (16, 7))
     # stochastic steps: compensated sums and the by-window choice keep the bulk forms
-    fits = P <= shape[0] * shape[1] and not (eta != 0.0 and (kind >= 210 or kind == 200))
+    fits = P <= shape[0] * shape[1] and not (eta != 0.0 and (kind >= 210 or kind in (200, 205, 206)))
     assert got["stats"]["update_kernel"] == (2 if fits else 1)
     assert compare(w, orc, got).max() <= REL_TOL
     assert np.array_equal(ref["log"], got["log"])
