@@ -541,43 +541,69 @@ def run_ours(args):
     net_us = roofline["avg_launch_us"] - floor_us
     roofline["frac_excl_floor"] = (float(upd_bytes.mean()) / (net_us * 1e-6) / 1e9 / peak) if net_us > 0 else None
 
-    # End to end through the public API with host buffers (no graph, no flush):
-    # x_init copied in from pinned host memory, iterations issued with the
-    # asynchronous calls in chunks of E2E_CHUNK, pa_poll after each chunk (one
-    # host synchronisation per chunk; iterations issued after the last
-    # trajectory finished do nothing), x_T copied out to pinned host memory.
+    # End to end through the public API with host buffers (no flush): every
+    # step copies x_init in from pinned host memory (pa_init), runs the
+    # generation and copies x_T out to pinned host memory (pa_result), with
+    # host time and device events around the whole loop. Headline: one
+    # Solver.generate call per step (E2E_CHUNK iterations captured once as a
+    # CUDA graph, replayed with one pa_poll per replay). Beside it, the same
+    # through eager calls: pa_step_async + pa_gmm_eps + pa_submit_eps issued
+    # from Python in chunks of E2E_CHUNK, pa_poll per chunk.
     e2e = None
     if not args.no_e2e:
         x_host = torch.from_numpy(x0).pin_memory()
         out_host = torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory()
-        polls = 0
-        stream.synchronize()
         reps = max(3, min(args.steps, 50))
-        e0 = torch.cuda.Event(enable_timing=True)
-        e1 = torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        t0 = time.perf_counter()
-        for _ in range(reps):
-            s.init(x_host)
-            while True:
-                for _ in range(E2E_CHUNK):
-                    bx, mb, nm = s.step_async()
-                    g.eps(bx, mb, nm, eps)
-                    s.submit_eps(eps)
-                polls += 1
-                if s.poll() == 0:
-                    break
-            s.result(out_host)
-        e1.record(stream)
-        stream.synchronize()
-        e2e_s = max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0)
+
+        def denoise(bx, mb, nm):
+            g.eps(bx, mb, nm, eps)
+            return eps
+
+        def timed(run):
+            stream.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            t0 = time.perf_counter()
+            polls = run()
+            e1.record(stream)
+            stream.synchronize()
+            return max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0), polls
+
+        def run_generate():
+            for _ in range(reps):
+                s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK)
+            return reps * -(-n_iters // E2E_CHUNK)
+
+        def run_eager():
+            polls = 0
+            for _ in range(reps):
+                s.init(x_host)
+                while True:
+                    for _ in range(E2E_CHUNK):
+                        bx, mb, nm = s.step_async()
+                        g.eps(bx, mb, nm, eps)
+                        s.submit_eps(eps)
+                    polls += 1
+                    if s.poll() == 0:
+                        break
+                s.result(out_host)
+            return polls
+
+        s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK)   # capture outside the timed loop
+        assert np.array_equal(out_host.numpy(), x_cached), "generate() differs from the graph-replayed generation"
+        e2e_s, polls = timed(run_generate)
+        eager_s, eager_polls = timed(run_eager)
         units_e, secs_e = aggregate(reps * n_iters, e2e_s)
+        units_g, secs_g = aggregate(reps * n_iters, eager_s)
         e2e = {"value": units_e / secs_e, "unit": UNIT,
                "h2d_bytes_per_step": int(w.batch * w.D * 4),
                "d2h_bytes_per_step": int(w.batch * w.D * 4 + (polls // reps) * 32),
                "steps": reps,
-               "api": f"pa_init (host x_init), pa_step_async + pa_gmm_eps + pa_submit_eps in chunks of "
-                      f"{E2E_CHUNK} iterations, pa_poll per chunk, pa_result (host x_T)"}
+               "api": f"Solver.generate: pa_init (host x_init), {E2E_CHUNK} iterations of pa_step_async + "
+                      f"pa_gmm_eps + pa_submit_eps captured once as a CUDA graph and replayed, pa_poll per "
+                      f"replay, pa_result (host x_T)",
+               "eager_value": units_g / secs_g,
+               "eager_api": f"the same calls issued from Python in chunks of {E2E_CHUNK}, pa_poll per chunk"}
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

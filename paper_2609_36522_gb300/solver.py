@@ -106,6 +106,44 @@ class Solver:
         abi.pa_result(self.h, out.data_ptr())
         return out
 
+    def generate(self, x_init, denoise, out=None, chunk=4):
+        """One whole generation in one call: x_init [batch][D] (CUDA tensor or
+        pinned host tensor) in, x_T out (into ``out``, a CUDA or pinned host
+        tensor, else a new CUDA tensor).
+
+        ``denoise(batch_x_ptr, miss_bt_ptr, n_miss_dev_ptr)`` enqueues eps_theta
+        of the planned misses on this solver's stream, reading the miss count
+        on the device (as ``GmmDenoiser.eps`` does), and returns the CUDA eps
+        tensor it wrote; it must write the same buffer on every call and be
+        capturable in a CUDA graph. ``chunk`` (even) iterations are captured
+        once per (denoise, chunk) and the graph is replayed, one ``pa_poll``
+        per replay, until every trajectory has reached T; iterations issued
+        after that do nothing on the device."""
+        if chunk < 2 or chunk % 2:
+            raise ValueError("chunk must be a positive even number (iterations alternate two plan copies)")
+        graphs = self.__dict__.setdefault("_gen_graphs", {})
+        key = (denoise, chunk)
+        self.init(x_init)
+        gr = graphs.get(key)
+        if gr is None:
+            # one eager iteration first: launch-time set-up (kernel attributes)
+            # happens outside the capture
+            bx, mb, nm = self.step_async()
+            self.submit_eps(denoise(bx, mb, nm))
+            self.init(x_init)
+            gr = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gr, stream=self.stream):
+                for _ in range(chunk):
+                    bx, mb, nm = self.step_async()
+                    self.submit_eps(denoise(bx, mb, nm))
+            graphs[key] = gr
+            self.init(x_init)  # the capture advanced the host state without running anything
+        for _ in range(self.T // chunk + 2):
+            gr.replay()
+            if self.poll() == 0:
+                return self.result(out)
+        raise RuntimeError("generate: trajectories did not reach T within T iterations")
+
     def nfe(self):
         return abi.pa_nfe(self.h)
 
@@ -129,6 +167,7 @@ class Solver:
         abi.pa_set_cache_precision(self.h, bits)
 
     def close(self):
+        self.__dict__.pop("_gen_graphs", None)  # captured launches refer to this workspace
         if getattr(self, "h", None) is not None:
             abi.pa_destroy(self.h)
             self.h = None

@@ -170,6 +170,37 @@ def test_graph_replay_equals_sync(w, form):
     g.close()
 
 
+@pytest.mark.parametrize("wname,chunk", [("sd15", 4), ("batched", 2), ("tiny", 6)])
+def test_generate_equals_async_path(wname, chunk):
+    """Solver.generate (captured chunks of iterations replayed until done,
+    host x_init in and host x_T out) gives the asynchronous path's latents,
+    log and counters bit for bit, on its first call (capture) and again on
+    the second (replay only)."""
+    import torch
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+    w = {"sd15": W.SD15, "batched": W.BATCHED.with_(T=40), "tiny": W.TINY}[wname]
+    ref = gpu_run(w, mode="async")
+    a, x0, mu = W.inputs(w)
+    st = torch.cuda.Stream()
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=st)
+    g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, w.batch * s.window, stream=st)
+    eps = torch.empty(w.batch * s.window, w.D, dtype=torch.float32, device="cuda")
+
+    def denoise(bx, mb, nm):
+        g.eps(bx, mb, nm, eps)
+        return eps
+
+    x_host = torch.from_numpy(x0).pin_memory()
+    for _ in range(2):
+        out = torch.full((w.batch, w.D), float("nan"), dtype=torch.float32).pin_memory()
+        s.generate(x_host, denoise, out=out, chunk=chunk)
+        assert np.array_equal(out.numpy(), ref["x_final"])
+        assert np.array_equal(s.iter_log(), ref["log"])
+        assert s.stats()["nfe"] == ref["nfe"]
+    s.close()
+    g.close()
+
+
 def test_host_x_init_equals_device_x_init():
     a = gpu_run(W.TINY)
     b = gpu_run(W.TINY, x_init_host=True)
