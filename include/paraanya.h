@@ -211,8 +211,9 @@ PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
  * (Eq. 7) and widened exactly when read. Not from the paper: a storage option
  * that halves the entries' bytes; the states, the fresh eps of a miss and all
  * arithmetic stay fp32, so a hit reuses the rounded eps and Eq. 4 measures the
- * distance to the rounded input. With 16 the update runs in the register form
- * (windows up to 104, deterministic steps) or the plain-load kernel. Any time
+ * distance to the rounded input. With 16 the update runs in the lean register
+ * form (windows up to 112, deterministic steps; selecting 1 or 112 gives the
+ * register-resident bulk form) or the plain-load kernel. Any time
  * except between pa_step and pa_submit_eps; the next call must be pa_init.
  * Returns PA_ERR_ARG for another value, PA_ERR_STATE in the wrong state. */
 PA_API pa_status pa_set_cache_precision(pa_solver* s, int bits);

@@ -45,6 +45,40 @@ __device__ __forceinline__ float2 sub2(float2 a, float2 b) {
 __device__ __forceinline__ Q qadd(const Q& a, const Q& b) { return {__fadd2_rn(a.l, b.l), __fadd2_rn(a.h, b.h)}; }
 __device__ __forceinline__ Q qsub(const Q& a, const Q& b) { return {sub2(a.l, b.l), sub2(a.h, b.h)}; }
 
+// A cache entry row piece (xhat or ehat, four columns) as stored: fp32, or
+// bfloat16 when CB (rounded to nearest even when written, widened exactly when
+// read). The trajectory's rows start where its fp32 rows would; within them
+// the row pitch is D entries.
+template <bool CB>
+__device__ __forceinline__ Q ld_ent(const float* traj_base, int off) {
+  if constexpr (CB) {
+    float a[4];
+    Bf16Row<4>::load(reinterpret_cast<const uint16_t*>(traj_base) + off, a);
+    return {make_float2(a[0], a[1]), make_float2(a[2], a[3])};
+  } else {
+    return ldq(traj_base + off);
+  }
+}
+template <bool CB>
+__device__ __forceinline__ void st_ent(float* traj_base, int off, const Q& q) {
+  if constexpr (CB) {
+    const float a[4] = {q.l.x, q.l.y, q.h.x, q.h.y};
+    Bf16Row<4>::store(reinterpret_cast<uint16_t*>(traj_base) + off, a);
+  } else {
+    stq(traj_base + off, q);
+  }
+}
+// The value an fp32 row piece takes once stored as an entry.
+template <bool CB>
+__device__ __forceinline__ Q as_ent(const Q& q) {
+  if constexpr (CB) {
+    auto r = [](float v) { return __bfloat162float(__float2bfloat16_rn(v)); };
+    return {make_float2(r(q.l.x), r(q.l.y)), make_float2(r(q.h.x), r(q.h.y))};
+  } else {
+    return q;
+  }
+}
+
 // (hi, lo) += v per component: s = fl(hi + v), s + err == hi + v exactly
 // (Knuth's TwoSum), lo accumulates err.
 __device__ __forceinline__ void two_sum2(float2& hi, float2& lo, float2 v) {
@@ -84,7 +118,7 @@ struct LeanShape {
   }
 };
 
-template <int NW, int LMAX, int MINB, bool NOISE, bool COMP>
+template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
 __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const float* __restrict__ beps, int par) {
   using Sh = LeanShape<NW, NOISE>;
   using CT = typename Coef<NOISE>::T;
@@ -131,8 +165,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   const bool live = mycol < D;
   const float* Xr = d.X + (int64_t)b * (P + 1) * D + mycol;  // this lane's column of each ring
   float* Xw = d.X + (int64_t)b * (P + 1) * D + mycol;
-  float* Xh = d.Xhat + (int64_t)b * P * D + mycol;
-  float* Eh = d.Ehat + (int64_t)b * P * D + mycol;
+  float* Xh = d.Xhat + (int64_t)b * P * D;  // entries: column mycol of row slot s at s * D + mycol
+  float* Eh = d.Ehat + (int64_t)b * P * D;
   const float* Zr = NOISE ? d.noise + (int64_t)b * T * D + mycol : nullptr;
   const float* Br = beps + mycol;
   const int L = (p + NW - 1) / NW;  // <= LMAX (launcher)
@@ -171,8 +205,8 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
 #pragma unroll
     for (int g = 0; g < LMAX; ++g) {
       if (g >= nj) break;
-      if (!(miss >> g & 1)) ep[g] = ldq(Eh + cslot(g) * D);
-      if (!(miss >> (g + 1) & 1)) xh[g] = ldq(Xh + cslot(g + 1) * D);
+      if (!(miss >> g & 1)) ep[g] = ld_ent<CB>(Eh, cslot(g) * D + mycol);
+      if (!(miss >> (g + 1) & 1)) xh[g] = ld_ent<CB>(Xh, cslot(g + 1) * D + mycol);
       if constexpr (NOISE) z[g] = ldq(Zr + (t + j0 + g) * D);
     }
   }
@@ -194,9 +228,9 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
     for (int g = 0; g < LMAX; ++g) {
       if (g >= nj) break;
       if (miss >> g & 1) {
-        const int o = cslot(g) * D;
-        stq(Eh + o, ep[g]);
-        stq(Xh + o, x[g]);
+        const int o = cslot(g) * D + mycol;
+        st_ent<CB>(Eh, o, ep[g]);
+        st_ent<CB>(Xh, o, x[g]);
       }
       const CT c = s_coef[t + j0 + g];
       const float2 cm = make_float2(c.x, c.x), ec = make_float2(c.y, c.y);
@@ -274,7 +308,11 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
         if (j + 1 < p) {
           // the next timestep's cache input: its entry if it is a hit, else
           // the old state i+1, the entry it receives in this kernel
-          if (!(miss >> (g + 1) & 1)) df = qsub(n, xh[g]);
+          if (!(miss >> (g + 1) & 1)) {
+            df = qsub(n, xh[g]);
+          } else if constexpr (CB) {
+            df = qsub(n, as_ent<CB>(x[g + 1]));
+          }
           dv = (fabsf(df.l.x) + fabsf(df.l.y)) + (fabsf(df.h.x) + fabsf(df.h.y));
         }
       }
@@ -300,12 +338,12 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   }
 }
 
-template <int NW, int LMAX, int MINB, bool NOISE, bool COMP>
+template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
 cudaError_t launch_lean(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = LeanShape<NW, NOISE>;
   const int nstrip = (int)((d.D + 127) / 128);
   const size_t smem = Sh::smem_bytes(d.T, d.P, COMP);
-  auto kern = k_update_lean<NW, LMAX, MINB, NOISE, COMP>;
+  auto kern = k_update_lean<NW, LMAX, MINB, NOISE, COMP, CB>;
   static size_t configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -341,6 +379,13 @@ cudaError_t launch_update_lean(const Dev& d, const float* batch_eps, int par, in
   static const int kWarps[7] = {0, 16, 12, 8, 8, 8, 4};
   static const int kRun[7] = {0, 7, 9, 4, 8, 4, 8};
   if (s > 6 || d.P > kWarps[s] * kRun[s]) return cudaErrorNotSupported;
+  if (d.cache_bf16) {  // bfloat16 entries: shapes 1, 4 and 5, plain sums, deterministic steps
+    if (comp || d.noise) return cudaErrorNotSupported;
+    if (s == 5) return launch_lean<8, 4, 3, false, false, true>(d, batch_eps, par, st);
+    if (s == 4) return launch_lean<8, 8, 2, false, false, true>(d, batch_eps, par, st);
+    if (s == 1) return launch_lean<16, 7, 1, false, false, true>(d, batch_eps, par, st);
+    return cudaErrorNotSupported;
+  }
   if (s >= 5 && (comp || d.noise)) return cudaErrorNotSupported;
   if (s == 5) return launch_lean<8, 4, 3, false, false>(d, batch_eps, par, st);
   if (s == 6) return launch_lean<4, 8, 4, false, false>(d, batch_eps, par, st);
@@ -364,7 +409,7 @@ cudaError_t launch_update_lean(const Dev& d, const float* batch_eps, int par, in
 }
 
 bool update_lean_supported(const Dev& d, const float* batch_eps) {
-  if (d.cache_bf16 || d.D % 4 != 0) return false;
+  if (d.D % 4 != 0 || (d.cache_bf16 && d.noise)) return false;
   if ((reinterpret_cast<uintptr_t>(batch_eps) & 15) != 0) return false;
   if (d.noise && (reinterpret_cast<uintptr_t>(d.noise) & 15) != 0) return false;
   if (d.P > 16 * 7) return false;

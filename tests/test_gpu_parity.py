@@ -452,6 +452,8 @@ def bf16_tolerance(w, orc):
     W.SD15, W.BATCHED,
     W.Workload("multi-strip", T=40, window=24, batch=3, latent_shape=(4, 20, 20), K=6,
                tol=1e-3, cache_thresh=0.05, seed=16),
+    W.Workload("window 64", T=100, window=64, batch=2, latent_shape=(4, 20, 20), K=6,
+               tol=1e-3, cache_thresh=0.05, seed=16),
     W.Workload("ragged odd D", T=30, window=12, batch=2, latent_shape=(3, 5, 7), K=3,
                tol=1e-3, cache_thresh=0.05, seed=3),
     W.Workload("window 128", T=150, window=128, batch=1, latent_shape=(4, 16, 16), K=4,
@@ -463,8 +465,8 @@ def test_bf16_cache_entries(w):
     exact (inputs guarded at 1e-3 relative, since an entry element can round to
     a neighbouring bfloat16 value when the GPU's fp32 value and the oracle's
     fp64 value straddle a rounding boundary), final latents within the bound of
-    bf16_tolerance (about 1.6e-3 at T = 100). The register form runs where it
-    applies, the plain-load kernel elsewhere (odd D, window 128, stochastic
+    bf16_tolerance (about 1.6e-3 at T = 100). The lean register form runs where
+    it applies, the plain-load kernel elsewhere (odd D, window 128, stochastic
     steps)."""
     from oracle.storage import round_bf16
     orc = oracle_run(w, cache_store=round_bf16)
@@ -472,6 +474,18 @@ def test_bf16_cache_entries(w):
     gpu = gpu_run(w, cache_bits=16)
     rel = compare(w, orc, gpu)
     assert rel.max() <= bf16_tolerance(w, orc), (rel, bf16_tolerance(w, orc))
+
+
+@pytest.mark.parametrize("kind", [112, 0])
+def test_bf16_cache_entries_other_forms(kind):
+    """The register-resident bulk form and the plain-load kernel with
+    bfloat16 entries, on the SD-shaped workload."""
+    from oracle.storage import round_bf16
+    w = W.SD15
+    orc = oracle_run(w, cache_store=round_bf16)
+    gpu = gpu_run(w, cache_bits=16, update_kernel=kind)
+    assert gpu["stats"]["update_kernel"] == (1 if kind == 112 else 0)
+    assert compare(w, orc, gpu).max() <= bf16_tolerance(w, orc)
 
 
 def test_bf16_cache_rejected_while_stepped():
