@@ -48,9 +48,10 @@ FALLBACK_HBM_GBS = 6800.0
 # one generation's launches, keyed by the sha256 of the kernel's source files at
 # capture time and the workload (profiles/ has the capture); reported as null when the kernel
 # source has changed since.
-NCU_TRAFFIC = {("c44ead84a091f784", "sd15"): 6248768.0,
-               ("c44ead84a091f784", "batched"): 24594133.0,
-               ("c44ead84a091f784", "large"): 70679881.0}
+NCU_TRAFFIC = {("acdd184ab975544a", "sd15"): 6247616.0,
+               ("acdd184ab975544a", "batched"): 24608469.0,
+               ("acdd184ab975544a", "large"): 70562414.0,
+               ("acdd184ab975544a", "sd15-bf16"): 6047104.0}
 
 
 def parse_args(argv=None):
