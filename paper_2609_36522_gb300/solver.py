@@ -55,6 +55,7 @@ class Solver:
     def set_noise(self, eta, noise=None):
         """Stochastic steps: noise is a CUDA float32 [batch][T][D] tensor of
         N(0, 1) draws (kept alive by this object); eta = 0 restores DDIM."""
+        self._drop_graphs()
         if eta == 0.0:
             self._noise_keepalive = None
             abi.pa_set_noise(self.h, 0.0, None)
@@ -118,7 +119,10 @@ class Solver:
         capturable in a CUDA graph. ``chunk`` (even) iterations are captured
         once per (denoise, chunk) and the graph is replayed, one ``pa_poll``
         per replay, until every trajectory has reached T; iterations issued
-        after that do nothing on the device."""
+        after that do nothing on the device. The captured launches carry the
+        solver's settings of the capture: the setters of this class drop them;
+        a denoiser's own settings must stay as they were captured (or pass a
+        new callable)."""
         if chunk < 2 or chunk % 2:
             raise ValueError("chunk must be a positive even number (iterations alternate two plan copies)")
         graphs = self.__dict__.setdefault("_gen_graphs", {})
@@ -139,7 +143,8 @@ class Solver:
             graphs[key] = gr
             self.init(x_init)  # the capture advanced the host state without running anything
         for _ in range(self.T // chunk + 2):
-            gr.replay()
+            with torch.cuda.stream(self.stream):  # replay() launches on the current stream
+                gr.replay()
             if self.poll() == 0:
                 return self.result(out)
         raise RuntimeError("generate: trajectories did not reach T within T iterations")
@@ -160,14 +165,19 @@ class Solver:
         """Picard-update kernel: 0 plain loads, 1 bulk forms, 2 lean register
         form (the default), 100 + n / 200 + n launch shapes of the bulk / lean
         forms (a tuning aid; pa_set_update_kernel documents them)."""
+        self._drop_graphs()
         abi.pa_set_update_kernel(self.h, kind)
 
     def set_cache_precision(self, bits):
         """16: bfloat16 cache entries, 32: fp32 (default). pa_init must follow."""
+        self._drop_graphs()
         abi.pa_set_cache_precision(self.h, bits)
 
+    def _drop_graphs(self):
+        self.__dict__.pop("_gen_graphs", None)
+
     def close(self):
-        self.__dict__.pop("_gen_graphs", None)  # captured launches refer to this workspace
+        self._drop_graphs()  # captured launches refer to this workspace
         if getattr(self, "h", None) is not None:
             abi.pa_destroy(self.h)
             self.h = None

@@ -197,6 +197,13 @@ def test_generate_equals_async_path(wname, chunk):
         assert np.array_equal(out.numpy(), ref["x_final"])
         assert np.array_equal(s.iter_log(), ref["log"])
         assert s.stats()["nfe"] == ref["nfe"]
+    # a setting changed after capture takes effect: the captured graph is dropped
+    s.set_update_kernel(0)
+    out = s.generate(x_host, denoise, chunk=chunk)
+    assert s.stats()["update_kernel"] == 0
+    assert np.array_equal(s.iter_log(), ref["log"])
+    assert compare(w, oracle_run(w), dict(x_final=out.cpu().numpy(), nfe=s.nfe(), stats=s.stats(),
+                                          log=s.iter_log(), misses=[])).max() <= REL_TOL
     s.close()
     g.close()
 
