@@ -17,8 +17,10 @@
 // nothing against a sequential compensated sum.
 //
 //   k_update_reg   each warp's run (at most LMAX positions) is loaded straight
-//                  into registers; no staging, no waits (default for four
-//                  columns per lane)
+//                  into registers; no staging, no waits (the bulk forms'
+//                  choice for four columns per lane; the library's default
+//                  with stochastic steps -- k_update_lean.cu has the default
+//                  for deterministic steps)
 //   k_update_seg   each warp's run is staged in shared memory by cp.async.bulk
 //                  (TMA engine) onto the warp's mbarrier (whole window per CTA)
 //   k_update_tile  the window walks in tiles of TW = NW*S positions through up
