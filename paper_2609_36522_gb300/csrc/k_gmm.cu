@@ -79,7 +79,7 @@ constexpr float kDotScale = 4294967296.f;  // 2^32: fixed-point scale of the dot
 
 // tensor-core dot products: rows per CTA (the MMA's M), columns per CTA
 constexpr int kTcRows = 128;
-constexpr int kTcCols = 128;  // 16 MMA steps of 8
+constexpr int kTcCols = 64;   // 8 MMA steps of 8 (98 KB of shared memory at K = 64: two CTAs per SM)
 constexpr int kTcThreads = 256;
 constexpr int kTcCluster = 8;            // column chunks per thread-block cluster ...
 constexpr int kTcClusterMinChunks = 256;  // ... when there are this many chunks (fewer atomics per accumulator)

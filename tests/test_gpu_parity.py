@@ -228,15 +228,19 @@ def _gmm_rows(w, n, seed=0):
 @pytest.mark.parametrize("form", [1, 0])
 @pytest.mark.parametrize("wname,n,max_rows", [("sd15", 48, 48), ("sd15", 1, 100), ("sd15", 37, 100),
                                               ("sd15", 100, 100), ("batched", 256, 256),
-                                              ("large", 48, 48), ("tiny", 5, 8)])
+                                              ("large", 48, 48), ("large", 1, 128), ("large", 70, 128),
+                                              ("large", 128, 128), ("k32", 100, 100), ("tiny", 5, 8)])
 def test_gmm_kernel_against_oracle(wname, n, max_rows, form):
     """The mixture denoiser alone, with the dot products on the tensor cores
     (form 1) and on the CUDA cores (form 0), on rows spread over the whole
     schedule, with the device row count below the capacity, and over three
-    calls in a row (the fixed-point accumulators and the tickets are reused)."""
+    calls in a row (the fixed-point accumulators and the tickets are reused).
+    With 64 components: one row, 70 rows (a ragged second 64-row block of the
+    tensor-core form's row tiles is not reached; rows past 48 are), and full
+    128-row tiles; exactly 32 components."""
     import torch
     from paper_2609_36522_gb300.solver import GmmDenoiser
-    w = W.ALL[wname]
+    w = W.SD15.with_(K=32, name="k32") if wname == "k32" else W.ALL[wname]
     a, mu, idx, x, miss = _gmm_rows(w, n)
     dev = torch.device("cuda")
     g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows)
