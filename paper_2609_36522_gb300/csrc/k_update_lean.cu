@@ -22,7 +22,11 @@
 //  - the window start x_t enters the run totals of warp 0, so later warps
 //    need no copy of it;
 //  - COMP carries every sum as an fp32 (hi, lo) pair (TwoSum); without it the
-//    sums are plain fp32 (fewer instructions, rounding of a 100-term fp32 sum).
+//    sums are plain fp32 (fewer instructions, rounding of a 100-term fp32 sum);
+//  - CB stores the cache entries as bfloat16 (rounded to nearest even when
+//    written, widened exactly when read).
+// MINB CTAs per SM bound the registers: one CTA of 16 warps for windows up to
+// 112 positions, two of 8 warps up to 64, three of 8 warps up to 32.
 #include "pa_internal.h"
 
 namespace pa {
