@@ -102,8 +102,13 @@ class Solver:
         return n
 
     def result(self, out=None):
+        """x_T [batch][D] into ``out`` (a contiguous float32 CUDA or host
+        tensor of batch x D elements), else into a new CUDA tensor."""
         if out is None:
             out = torch.empty(self.batch, self.D, dtype=torch.float32, device=self.workspace.device)
+        elif (not isinstance(out, torch.Tensor) or out.dtype != torch.float32 or not out.is_contiguous()
+              or out.numel() != self.batch * self.D):
+            raise ValueError("out must be a contiguous float32 tensor of batch x D elements")
         abi.pa_result(self.h, out.data_ptr())
         return out
 
@@ -282,15 +287,24 @@ class SrdsSolver:
         return bx, mb, nm
 
     def submit_eps(self, eps):
-        abi.pa_srds_submit_eps(self.h, eps.data_ptr() if isinstance(eps, torch.Tensor) else eps)
+        if isinstance(eps, torch.Tensor):
+            if eps.dtype != torch.float32 or not eps.is_cuda or not eps.is_contiguous():
+                raise ValueError("eps must be a contiguous CUDA float32 tensor")
+            eps = eps.data_ptr()
+        abi.pa_srds_submit_eps(self.h, eps)
 
     def poll(self):
         st, n = abi.pa_srds_poll(self.h)
         return n
 
     def result(self, out=None):
+        """x_T [batch][D] into ``out`` (a contiguous float32 CUDA or host
+        tensor of batch x D elements), else into a new CUDA tensor."""
         if out is None:
             out = torch.empty(self.batch, self.D, dtype=torch.float32, device=self.workspace.device)
+        elif (not isinstance(out, torch.Tensor) or out.dtype != torch.float32 or not out.is_contiguous()
+              or out.numel() != self.batch * self.D):
+            raise ValueError("out must be a contiguous float32 tensor of batch x D elements")
         abi.pa_srds_result(self.h, out.data_ptr())
         return out
 
