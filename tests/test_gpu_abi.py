@@ -138,3 +138,22 @@ def test_bounded_wait_reports_timeout_and_context_survives(kind):
     _run(s, g, eps)
     assert np.array_equal(clean, s.result().cpu().numpy())
     assert s.stats()["device_status"] == 0
+
+
+def test_update_kernel_selector_rejects_unknown_shapes():
+    """pa_set_update_kernel takes 0, 1, 2, 100 + bulk shape and 200 + lean
+    shape (0-6, 10-16); anything else is PA_ERR_ARG and leaves the choice as
+    it was."""
+    w = W.TINY
+    s, g, eps, x0 = _solver(w)
+    for kind in (2, 0, 1, 100, 112, 200, 206, 210, 216):
+        abi.pa_set_update_kernel(s.h, kind)
+    for kind in (-1, 3, 99, 113, 199, 207, 209, 217, 300):
+        with pytest.raises(abi.PaError) as e:
+            abi.pa_set_update_kernel(s.h, kind)
+        assert e.value.status == abi.PA_ERR_ARG
+    s.init(x0)
+    _run(s, g, eps)
+    # the last accepted choice, 216, stays: shape 6 has no compensated form,
+    # so the update falls back to the bulk forms
+    assert s.stats()["update_kernel"] == 1
