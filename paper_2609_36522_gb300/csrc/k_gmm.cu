@@ -393,7 +393,9 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   const bool ok = wait_staged(bulk, &bar, status);
   __syncthreads();
   if (!ok) return;
-  const int cg = tid % (kOutCols / 4), rg = tid / (kOutCols / 4);  // 64 column groups x 4 row groups
+  // kOutCols / 4 column groups of 4 x kThreads / (kOutCols / 4) row groups of 4
+  static_assert(kThreads / (kOutCols / 4) * 4 == kOutRows, "the threads cover the tile's rows");
+  const int cg = tid % (kOutCols / 4), rg = tid / (kOutCols / 4);
   const int cc = cg * 4;
   if (cc >= ncol) return;
   float acc[4][4];
@@ -770,7 +772,7 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
   if (e == cudaSuccess)
     e = pa::launch_ex(k_gmm_out,
                       dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
-                      dim3(kOutCols), out_smem, g->st, 0, batch_x_dev, g->means, (const long long*)gacc2, ep, coef,
+                      dim3(kThreads), out_smem, g->st, 0, batch_x_dev, g->means, (const long long*)gacc2, ep, coef,
                       g->T, miss_bt_dev, mnorm, n_rows_dev, g->K, g->D, g->max_rows, bulk, vec_out, batch_eps_dev,
                       status);
   g->launches += 2;
@@ -951,7 +953,7 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   const bool vec_out = D % 4 == 0 && (reinterpret_cast<uintptr_t>(batch_eps_dev) & 15) == 0;
   k_gmm_dots<<<dim3(nchunk, (n_rows + kDotRows - 1) / kDotRows), kThreads, dots_smem, st>>>(
       batch_x_dev, means_dev, nrows_dev, K, D, chunk, nchunk, n_rows, bulk, gacc2, ep, status);
-  k_gmm_out<<<dim3((unsigned)((D + kOutCols - 1) / kOutCols), (n_rows + kOutRows - 1) / kOutRows), kOutCols,
+  k_gmm_out<<<dim3((unsigned)((D + kOutCols - 1) / kOutCols), (n_rows + kOutRows - 1) / kOutRows), kThreads,
               out_smem, st>>>(batch_x_dev, means_dev, gacc2, ep, coef, T, miss_bt_dev, mnorm, nrows_dev, K, D,
                               n_rows, bulk, vec_out, batch_eps_dev, status);
   e = cudaGetLastError();
