@@ -157,3 +157,20 @@ def test_update_kernel_selector_rejects_unknown_shapes():
     # the last accepted choice, 216, stays: shape 6 has no compensated form,
     # so the update falls back to the bulk forms
     assert s.stats()["update_kernel"] == 1
+
+
+def test_result_buffer_is_checked():
+    """Solver.result refuses an output buffer of the wrong size, type or
+    layout before the library writes batch x D values into it."""
+    import torch
+    w = W.TINY
+    s, g, eps, x0 = _solver(w)
+    s.init(x0)
+    _run(s, g, eps)
+    for bad in (torch.empty(w.batch * w.D - 1, dtype=torch.float32, device="cuda"),
+                torch.empty(w.batch, w.D, dtype=torch.float64, device="cuda"),
+                torch.empty(w.batch, 2 * w.D, dtype=torch.float32, device="cuda")[:, ::2]):
+        with pytest.raises(ValueError):
+            s.result(bad)
+    good = torch.empty(w.batch * w.D, dtype=torch.float32, device="cuda")
+    assert torch.equal(s.result(good).view(w.batch, w.D), s.result())
