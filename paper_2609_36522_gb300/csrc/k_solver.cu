@@ -333,7 +333,7 @@ __global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
     }
   }
   __syncthreads();  // the sums and decide_load's state are staged
-  decide_warp(d, ds, RedShared{s_e, s_d}, par, publish, (int)blockIdx.y);
+  decide_par(d, ds, RedShared{s_e, s_d}, par, publish, (int)blockIdx.y);
   __syncthreads();  // the plan (batch row of this CTA) is known
   if ((int)blockIdx.y < ds.total && ds.target_b >= 0) {
     const int b = ds.target_b;

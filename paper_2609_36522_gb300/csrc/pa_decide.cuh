@@ -15,6 +15,9 @@ struct DecideShared {
   int tn[kMaxBatch], pn[kMaxBatch], en[kMaxBatch], m[kMaxBatch], h1[kMaxBatch];
   int om[kMaxBatch], oh1[kMaxBatch];
   int warp_tot[32];
+  unsigned cmiss[32], cwin[32];  // decide_par: miss / in-window bits of each 32-position chunk
+  int cbase[32];                 // decide_par: misses before each chunk
+  int pts;                       // decide_par: window positions planned
   int total, active, iter;
   long long nfe, hits;
   int target_b, target_i;  // the miss of the requested batch row, if any
@@ -221,31 +224,33 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const Red& red, int p
   }
 }
 
-// The same decision taken by one warp (warp 0 of the calling CTA; the other
-// warps skip it), for the planning kernel in which every CTA decides: with
-// B*P small the ballots and population counts of one warp replace the block
-// scan and its barriers. Reads what decide_load staged (after a barrier that
-// the caller provides) and gives the same plan, ranks and counters as
-// decide_run. The caller synchronises the CTA afterwards.
+// The same decision with all warps of the CTA at work, for the planning
+// kernel in which every CTA decides (B*P <= 32 * 32): warp w advances the
+// windows of trajectories w, w + NW, ...; warp w tests the 32-position chunks
+// w, w + NW, ... of the next windows; one warp turns the chunks' miss counts
+// into each chunk's first rank; the chunks then place their misses. Gives the
+// same plan, ranks and counters as decide_run. Every thread of
+// the CTA calls it (it holds CTA barriers); the caller synchronises the CTA
+// afterwards.
 template <typename Red>
-__device__ void decide_warp(const Dev& d, DecideShared& sh, const Red& red, int par, bool publish, int target) {
-  if (threadIdx.x >= 32) return;
-  const int lane = threadIdx.x;
+__device__ void decide_par(const Dev& d, DecideShared& sh, const Red& red, int par, bool publish, int target) {
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
   const int B = d.B, P = d.P, T = d.T;
   Traj* out_traj = d.traj + (par ^ 1) * B;
-  if (sh.active == 0) {  // finished: the plan carries over
-    if (publish) {
-      const Traj* in_traj = d.traj + par * B;
-      for (int b = lane; b < B; b += 32) out_traj[b] = in_traj[b];
-      if (lane == 0) d.pc[par ^ 1] = d.pc[par];
+  if (sh.active == 0) {  // finished: the plan carries over (uniform across the CTA)
+    if (warp == 0) {
+      if (publish) {
+        const Traj* in_traj = d.traj + par * B;
+        for (int b = lane; b < B; b += 32) out_traj[b] = in_traj[b];
+        if (lane == 0) d.pc[par ^ 1] = d.pc[par];
+      }
+      for (int b = lane; b < B; b += 32) sh.en[b] = sh.e[b];
     }
-    for (int b = lane; b < B; b += 32) sh.en[b] = sh.e[b];
-    __syncwarp();
     return;
   }
   const int iter = sh.iter;
-  // 1. window advance
-  for (int b = 0; b < B; ++b) {
+  // 1. window advance, one warp per trajectory
+  for (int b = warp; b < B; b += nw) {
     const int t = sh.t[b], p = sh.p[b];
     int stride = 0;
     if (p > 0) {
@@ -277,18 +282,14 @@ __device__ void decide_warp(const Dev& d, DecideShared& sh, const Red& red, int 
       }
     }
   }
-  __syncwarp();
-  // 2. hit/miss plan of the next iteration, compacted 32 positions at a time
-  const int N = B * P;
-  int base = 0;
-  int pts = 0;
-  for (int q0 = 0; q0 < N; q0 += 32) {
-    const int q = q0 + lane;
+  __syncthreads();
+  // 2. hit/miss tests of the next windows, one warp per 32-position chunk
+  const int N = B * P, nchunk = (N + 31) / 32;
+  for (int c = warp; c < nchunk; c += nw) {
+    const int q = c * 32 + lane;
     int miss = 0, inwin = 0;
-    int b = 0, j = 0;
     if (q < N) {
-      b = q / P;
-      j = q % P;
+      const int b = q / P, j = q % P;
       if (j < sh.pn[b]) {
         inwin = 1;
         const int i = sh.tn[b] + j;
@@ -301,13 +302,42 @@ __device__ void decide_warp(const Dev& d, DecideShared& sh, const Red& red, int 
         }
       }
     }
-    const unsigned mm = __ballot_sync(0xffffffffu, miss);
-    const int r = base + __popc(mm & ((1u << lane) - 1u));
+    const unsigned mm = __ballot_sync(0xffffffffu, miss), wm = __ballot_sync(0xffffffffu, inwin);
+    if (lane == 0) {
+      sh.cmiss[c] = mm;
+      sh.cwin[c] = wm;
+    }
+  }
+  __syncthreads();
+  // each chunk's first rank: an exclusive scan of the chunks' miss counts
+  if (warp == 0) {
+    const int cnt = lane < nchunk ? __popc(sh.cmiss[lane]) : 0;
+    const int win = lane < nchunk ? __popc(sh.cwin[lane]) : 0;
+    int incl = cnt;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    if (lane < nchunk) sh.cbase[lane] = incl - cnt;
+    const int pts = __reduce_add_sync(0xffffffffu, win);
+    if (lane == 31) sh.total = incl;
+    if (lane == 0) sh.pts = pts;
+  }
+  __syncthreads();
+  // 3. the misses' ranks (trajectory-major, ascending t), the requested row
+  for (int c = warp; c < nchunk; c += nw) {
+    const int q = c * 32 + lane;
+    if (q >= N) continue;
+    const unsigned mm = sh.cmiss[c];
+    const int miss = (mm >> lane) & 1u;
+    const int b = q / P, j = q % P;
+    const int r = sh.cbase[c] + __popc(mm & ((1u << lane) - 1u));
     if (miss && r == target) {
       sh.target_b = b;
       sh.target_i = sh.tn[b] + j;
     }
-    if (publish && q < N) {
+    if (publish) {
       if (miss) {
         d.rank[q] = r;
         d.miss_bt[2 * r] = b;
@@ -315,17 +345,14 @@ __device__ void decide_warp(const Dev& d, DecideShared& sh, const Red& red, int 
         atomicAdd(&sh.m[b], 1);
       } else {
         d.rank[q] = -1;
-        if (inwin && j >= 1) atomicAdd(&sh.h1[b], 1);
+        if (((sh.cwin[c] >> lane) & 1u) && j >= 1) atomicAdd(&sh.h1[b], 1);
       }
     }
-    base += __popc(mm);
-    pts += __popc(__ballot_sync(0xffffffffu, inwin));
   }
-  if (lane == 0) sh.total = base;
-  __syncwarp();
-  // 3. trajectories and counters of the next iteration
   if (publish) {
-    for (int b = lane; b < B; b += 32) {
+    __syncthreads();
+    // 4. trajectories and counters of the next iteration
+    for (int b = tid; b < B; b += blockDim.x) {
       Traj tr{};
       tr.t = sh.tn[b];
       tr.p = sh.pn[b];
@@ -336,20 +363,21 @@ __device__ void decide_warp(const Dev& d, DecideShared& sh, const Red& red, int 
       if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
       out_traj[b] = tr;
     }
-    if (lane == 0) {
+    if (tid == 0) {
       int act = 0;
       for (int b = 0; b < B; ++b) act += (sh.pn[b] > 0);
-      PlanCtr c;
-      c.n_active = act;
-      c.iter = iter + 1;
-      c.nfe = sh.nfe + base;
-      c.hits = sh.hits + (pts - base);
-      d.pc[par ^ 1] = c;
+      const int base = sh.total;
+      PlanCtr cc;
+      cc.n_active = act;
+      cc.iter = iter + 1;
+      cc.nfe = sh.nfe + base;
+      cc.hits = sh.hits + (sh.pts - base);
+      d.pc[par ^ 1] = cc;
       d.ctl->n_miss = base;
       d.ctl->n_active = act;
-      d.ctl->iter = c.iter;
-      d.ctl->nfe = c.nfe;
-      d.ctl->hits = c.hits;
+      d.ctl->iter = cc.iter;
+      d.ctl->nfe = cc.nfe;
+      d.ctl->hits = cc.hits;
     }
   }
 }
