@@ -117,10 +117,11 @@ __device__ __forceinline__ double block_sum(double v, double* s_w) {
   return t;
 }
 
-// One stage's plan and batch, one launch. Warp 0 of every CTA takes the
-// stage's decision over its rows (at most 2048, 32 at a time): a live row
-// with an entry hits iff its distance sum / D < tau_cache (Eq. 5); misses get
-// ranks in row order (trajectory-major) by ballots and population counts. The
+// One stage's plan and batch, one launch. Every CTA takes the stage's
+// decision over its rows (at most 2048) with all of its warps, one 32-row chunk
+// per warp at a time: a live row with an entry hits iff its distance sum / D <
+// tau_cache (Eq. 5); misses get ranks in row order (trajectory-major) from the
+// chunks' ballots and one scan of their miss counts. The
 // same inputs give the same plan in every CTA; CTA (0, 0) publishes it (ranks,
 // miss list, counters) and clears the distance set the coming apply adds into.
 // Then every CTA narrows its column range of the batch row whose rank is its
@@ -128,49 +129,83 @@ __device__ __forceinline__ double block_sum(double v, double* s_w) {
 __global__ void __launch_bounds__(kSThreads) k_srds_plan_gather(SDev d, Stage st, int set) {
   pa::pdl_wait();     // everything read here comes from earlier kernels
   pa::pdl_trigger();  // the successor may now be scheduled
+  constexpr int kChunks = kSMaxRows / 32, kWarps = kSThreads / 32;
   __shared__ int s_total, s_row;
-  const int tid = threadIdx.x;
+  __shared__ unsigned s_mm[kChunks], s_hm[kChunks];  // miss / hit bits of each 32-row chunk
+  __shared__ int s_base[kChunks];                     // misses before each chunk
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
   const int rows = stage_rows(d, st);
   const int R = d.B * d.N;
-  if (tid < 32) {
-    const int lane = tid;
-    int base = 0, hits = 0, target_row = -1;
-    for (int q0 = 0; q0 < rows; q0 += 32) {
-      const int r = q0 + lane;
-      int b = 0, n = 0, i = 0;
-      double* x = nullptr;
-      const bool live = r < rows && row_info(d, st, r, b, n, i, x);
-      bool hit = false;
-      if (live && d.has[(int64_t)b * d.T + i]) hit = d.sacc[((size_t)set * R + r) * pa::kAccStride] / (double)d.D < d.cache_thresh;
-      const bool miss = live && !hit;
-      const unsigned mm = __ballot_sync(0xffffffffu, miss);
-      const int rank = base + __popc(mm & ((1u << lane) - 1u));
-      if (miss && rank == (int)blockIdx.y) target_row = r;
-      if (publish && r < rows) {
-        d.rank[r] = miss ? rank : (live ? -1 : -2);
-        if (miss) {
-          d.miss_bt[2 * rank] = b;
-          d.miss_bt[2 * rank + 1] = i;
-        }
-      }
-      base += __popc(mm);
-      hits += __popc(__ballot_sync(0xffffffffu, live && hit));
+  const int nchunk = (rows + 31) / 32;
+  // 1. hit/miss of every row, one warp per chunk; a row's trajectory flag, entry
+  //    flag and distance sum are read together
+  for (int c = warp; c < nchunk; c += kWarps) {
+    const int r = c * 32 + lane;
+    bool live = false, hit = false;
+    if (r < rows) {
+      int b, n, i;
+      double* x;
+      live = row_info(d, st, r, b, n, i, x);
+      const bool has = i < d.T && d.has[(int64_t)b * d.T + i];
+      const double sv = d.sacc[((size_t)set * R + r) * pa::kAccStride];
+      hit = live && has && sv / (double)d.D < d.cache_thresh;
     }
-    // the lane that saw the target row reports it
-    const unsigned tm = __ballot_sync(0xffffffffu, target_row >= 0);
-    if (tm && lane == __ffs(tm) - 1) s_row = target_row;
+    const unsigned mm = __ballot_sync(0xffffffffu, live && !hit), hm = __ballot_sync(0xffffffffu, hit);
     if (lane == 0) {
-      s_total = base;
-      if (!tm) s_row = -1;
+      s_mm[c] = mm;
+      s_hm[c] = hm;
+    }
+  }
+  __syncthreads();
+  // 2. each chunk's first rank (exclusive scan of the chunk miss counts, two
+  //    chunks per lane), the totals, the counters
+  if (warp == 0) {
+    const int c0 = 2 * lane, c1 = 2 * lane + 1;
+    const int n0 = c0 < nchunk ? __popc(s_mm[c0]) : 0, n1 = c1 < nchunk ? __popc(s_mm[c1]) : 0;
+    int incl = n0 + n1;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int v = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += v;
+    }
+    const int excl = incl - (n0 + n1);
+    if (c0 < nchunk) s_base[c0] = excl;
+    if (c1 < nchunk) s_base[c1] = excl + n0;
+    const int hits = __reduce_add_sync(0xffffffffu, (c0 < nchunk ? __popc(s_hm[c0]) : 0) +
+                                                        (c1 < nchunk ? __popc(s_hm[c1]) : 0));
+    const int total = __shfl_sync(0xffffffffu, incl, 31);
+    if (lane == 0) {
+      s_total = total;
+      s_row = -1;
       if (publish) {
-        d.ctl->n_miss = base;
-        d.ctl->nfe += base;
+        d.ctl->n_miss = total;
+        d.ctl->nfe += total;
         d.ctl->hits += hits;
       }
     }
     if (publish)
       for (int q = lane; q < R; q += 32) d.sacc[((size_t)(set ^ 1) * R + q) * pa::kAccStride] = 0.0;
+  }
+  __syncthreads();
+  // 3. ranks in row order; the row of this CTA's rank
+  for (int c = warp; c < nchunk; c += kWarps) {
+    const int r = c * 32 + lane;
+    if (r >= rows) continue;
+    const unsigned mm = s_mm[c];
+    const bool miss = (mm >> lane) & 1u;
+    const int rank = s_base[c] + __popc(mm & ((1u << lane) - 1u));
+    if (miss && rank == (int)blockIdx.y) s_row = r;  // one row holds each rank
+    if (publish) {
+      d.rank[r] = miss ? rank : (((s_hm[c] >> lane) & 1u) ? -1 : -2);
+      if (miss) {
+        int b, n, i;
+        double* x;
+        row_info(d, st, r, b, n, i, x);
+        d.miss_bt[2 * rank] = b;
+        d.miss_bt[2 * rank + 1] = i;
+      }
+    }
   }
   __syncthreads();
   const int m = blockIdx.y, r = s_row;
