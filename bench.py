@@ -455,13 +455,13 @@ def run_ours(args):
             t1.fill_(0.0)
             ev[1].record(stream)
             t1.add_(1.0)
-        tot = 0.0
+        times = []
         for r in range(reps + 3):
             gr.replay()
             stream.synchronize()
             if r >= 3:
-                tot += ev[0].elapsed_time(ev[1])
-        return 1000.0 * tot / reps
+                times.append(ev[0].elapsed_time(ev[1]))
+        return 1000.0 * float(np.median(times))  # the median: single replays can stall
 
     for _ in range(args.warmup):
         generation(graph_plain, False)
@@ -536,7 +536,7 @@ def run_ours(args):
                 "alg_bytes_per_launch": float(upd_bytes.mean()),
                 "avg_launch_us": 1000.0 * upd_ms / max(n_upd, 1),
                 "timing_floor_us": floor_us,
-                "timing_floor_note": "event-pair time of a one-element fill at the same place in a graph: "
+                "timing_floor_note": "median event-pair time of a one-element fill at the same place in a graph: "
                                      "launch and completion latency that every event-timed launch includes; "
                                      "frac_excl_floor divides the bytes by avg_launch_us minus it"}
     net_us = roofline["avg_launch_us"] - floor_us
