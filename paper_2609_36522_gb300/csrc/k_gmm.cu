@@ -146,11 +146,6 @@ __device__ __forceinline__ float warp_sum(float v) {
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
   return v;
 }
-__device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
-  return v;
-}
 
 // ||mu_k||^2, one CTA per component, fixed-order tree.
 __global__ void __launch_bounds__(256) k_gmm_norms(const float* __restrict__ mu, int64_t D,
@@ -377,17 +372,27 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
     s_r[q] = l;
   }
   __syncthreads();
-  for (int rr = warp; rr < nr; rr += kThreads / 32) {
-    float* l = s_r + rr * K;
-    float mx = -INFINITY;
-    for (int k = lane; k < K; k += 32) mx = fmaxf(mx, l[k]);
-    mx = warp_max(mx);
-    float sum = 0.f;
-    for (int k = lane; k < K; k += 32) sum += expf(l[k] - mx);
-    sum = warp_sum(sum);
-    const float inv = 1.f / sum;
-    __syncwarp();
-    for (int k = lane; k < K; k += 32) l[k] = expf(l[k] - mx) * inv;
+  // softmax per row: a half-warp per row when K <= 16 (two rows per warp and
+  // pass), else a warp; the reductions are the same trees either way
+  {
+    const int width = K <= 16 ? 16 : 32, sub = lane / width, sl = lane % width;
+    for (int rr0 = warp * (32 / width); rr0 < nr; rr0 += (kThreads / 32) * (32 / width)) {
+      const int rr = rr0 + sub;
+      const bool ok = rr < nr;
+      float* l = s_r + (ok ? rr : 0) * K;
+      float mx = -INFINITY;
+      if (ok)
+        for (int k = sl; k < K; k += width) mx = fmaxf(mx, l[k]);
+      for (int o = width / 2; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      float sum = 0.f;
+      if (ok)
+        for (int k = sl; k < K; k += width) sum += expf(l[k] - mx);
+      for (int o = width / 2; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      const float inv = 1.f / sum;
+      __syncwarp();
+      if (ok)
+        for (int k = sl; k < K; k += width) l[k] = expf(l[k] - mx) * inv;
+    }
   }
   if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) ep->epoch = cur + 1u;  // the next call's set
   const bool ok = wait_staged(bulk, &bar, status);
