@@ -290,6 +290,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 // CTAs read copy par of the plan, which no CTA writes in this launch.
 constexpr int kPlanThreads = 256;
 constexpr int kFusedMaxPairs = 1024;  // B*P planned in every CTA; beyond, one CTA plans
+static_assert(kFusedMaxPairs <= 32 * 32, "decide_par keeps one miss mask per 32-position chunk, 32 of them");
 
 struct RedShared {
   const double* e;
