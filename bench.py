@@ -4,16 +4,28 @@
 Workload (default): SD-v1.5-shaped cached Picard DDIM -- T=100, window 100,
 batch 1, 4x64x64 fp32 latents, 16-component mixture denoiser, tol 1e-3,
 tau_cache 0.05 (synthetic seeded inputs). One bench step = one complete
-generation (every Picard iteration until t = T). ``value`` is Picard solver
-steps (iterations) per second, whole job: the iterations all ranks ran divided
-by the slowest rank's device time, measured with CUDA events around every
-iteration (gather, mixture denoiser, update, decision). L2 (129 MB) is flushed
-before every iteration by writing a 256 MiB buffer, outside the timed events,
-because the whole working set (~35 MB) would otherwise stay L2-resident.
+generation (every Picard iteration until t = T), replayed as one CUDA graph
+with one pair of CUDA events around it on the launch stream; L2 (129 MB) is
+flushed before every generation by writing a 256 MiB buffer, outside the
+events. ``value`` is Picard iterations per second of device time, denoiser
+included, whole job (the iterations all ranks ran over the slowest rank's time).
 
-Also reported: the roofline of the dominant kernel (the Picard update), the
-end-to-end rate through the public API with host buffers (``e2e``), the fp64
-oracle timed on the host cores (``cpu_baseline``), NFE and hit rate.
+Also reported:
+  solver_step   the cache + Picard solver step alone: a graph of the solver's
+                kernels with the eps rows recorded from the same generation and
+                an empty stand-in kernel where the denoiser ran, no event nodes
+                inside; microseconds per iteration and its algorithmic bytes
+                per microsecond against the measured HBM copy bandwidth (and
+                the nominal 8 TB/s), with L2 flushed per generation, L2 warm,
+                and L2 flushed before every iteration;
+  roofline      the solver step's kernel (the fused step where it runs) from
+                the solver-only graph;
+  uncached      the same generation with tau_cache = 0 (no hits): NFE,
+                iterations and time;
+  e2e           the public API with host buffers (copies inside the timing);
+  cpu_baseline  the fp64 oracle on the host cores, one thread and all cores,
+                whole iterations and the solver step with the denoiser's time
+                taken out.
 
 ``--impl reference`` times the fp64 CPU oracle (the only reference this
 method has: the paper ships no code) on the same workload.
@@ -44,14 +56,14 @@ FLUSH_BYTES = 256 << 20
 E2E_CHUNK = 4      # Picard iterations issued between two pa_poll calls in the end-to-end run
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
-# ncu DRAM bytes (read + write) of the update kernel per launch, averaged over
-# one generation's launches, keyed by the sha256 of the kernel's source files at
-# capture time and the workload (profiles/ has the capture); reported as null when the kernel
+NOMINAL_HBM_GBS = 8000.0
+# ncu DRAM bytes (read + write) per launch of the solver step's kernel(s),
+# averaged over one generation's launches, keyed by the sha256 of the solver
+# kernels' source files at capture time and the workload. These are stored
+# figures from an earlier ncu capture of this bench command (profiles/ has it),
+# not a measurement of the current run; reported as null once the kernel
 # source has changed since.
-NCU_TRAFFIC = {("acdd184ab975544a", "sd15"): 6247616.0,
-               ("acdd184ab975544a", "batched"): 24608469.0,
-               ("acdd184ab975544a", "large"): 70562414.0,
-               ("acdd184ab975544a", "sd15-bf16"): 6047104.0}
+NCU_TRAFFIC = {}
 
 
 def parse_args(argv=None):
@@ -116,7 +128,8 @@ def measured_hbm_gbs():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-UPDATE_KERNEL_SOURCES = ("k_update_bulk.cu", "k_update_lean.cu", "pa_bulk.cuh", "pa_internal.h")
+UPDATE_KERNEL_SOURCES = ("k_update_bulk.cu", "k_update_lean.cu", "k_solver.cu", "pa_decide.cuh", "pa_bulk.cuh",
+                         "pa_internal.h")
 
 
 def kernel_source_sha():
@@ -134,7 +147,7 @@ def kernel_source_sha():
     return h.hexdigest()[:16]
 
 
-def iteration_bytes(log, w: W.Workload, entry_bytes=4):
+def iteration_bytes(log, w: W.Workload, entry_bytes=4, fused=False):
     """Algorithmic bytes per Picard iteration, from the solver's iteration log.
 
     Per trajectory with window start t, p points, m misses, frontier e and h1
@@ -143,23 +156,28 @@ def iteration_bytes(log, w: W.Workload, entry_bytes=4):
       update : x_t, the p - lazy materialised old states, m batch eps rows and
                p - m ehat rows, m ehat and m xhat writes, h1 xhat reads (next
                distances), p new states, and p draws z_i for stochastic steps
-      gather : m reads + m writes;  denoiser: m reads + m writes (+ K means)
+      gather : the next iteration's m' batch rows: read and written by the
+               planning kernel, written only by the fused step (the new states
+               are still in its registers)
+      denoiser: m reads + m writes (+ K means)
+    Returns (update, gather, denoiser) arrays over the iterations.
     """
     row = w.D * 4
     ent = w.D * entry_bytes
-    upd, other = [], []
-    for k in range(log.shape[0]):
-        u = o = 0
+    n = log.shape[0]
+    upd, gat, den = np.zeros(n), np.zeros(n), np.zeros(n)
+    for k in range(n):
         for b in range(log.shape[1]):
             t, p, m, stride, e, h1 = (int(v) for v in log[k, b, :6])
             if p == 0:
                 continue
             lazy = max(0, t + p - e)
-            u += (1 + (p - lazy) + m + p + (p if w.eta != 0.0 else 0)) * row + ((p - m) + 2 * m + h1) * ent
-            o += 4 * m * row
-        upd.append(u)
-        other.append(o + w.K * row)
-    return np.array(upd, dtype=np.float64), np.array(other, dtype=np.float64)
+            upd[k] += (1 + (p - lazy) + m + p + (p if w.eta != 0.0 else 0)) * row + ((p - m) + 2 * m + h1) * ent
+            den[k] += 2 * m * row
+            if k + 1 < n:
+                gat[k] += (1 if fused else 2) * int(log[k + 1, b, 2]) * row
+        den[k] += w.K * row
+    return upd, gat, den
 
 
 class ClockSampler:
@@ -215,81 +233,138 @@ class ClockSampler:
 
 # --------------------------------------------------------- oracle timing ----
 
-def oracle_sample(workload_name, budget_s):
+def oracle_sample(workload_name, budget_s, cache_thresh=None):
     """Time the fp64 oracle on whole generations of the workload for about
-    budget_s seconds (at least one generation). Runs in a fresh process."""
+    budget_s seconds (at least one generation), and within that the time its
+    denoiser calls took (the solver step = the rest). Runs in a fresh process."""
     from oracle import run_picard, run_srds
     from oracle.gmm import make_eps_fn
     w = W.ALL[workload_name]
+    if cache_thresh is not None:
+        w = w.with_(cache_thresh=cache_thresh)
     a, x0, mu = W.inputs(w)
     f = make_eps_fn(a, mu, w.gmm_std)
+    t_eps = [0.0]
+
+    def f_timed(rows, idx):
+        t0 = time.perf_counter()
+        r = f(rows, idx)
+        t_eps[0] += time.perf_counter() - t0
+        return r
+
     iters = gens = 0
     t0 = time.perf_counter()
     while True:
         if w.sampler == "srds":   # a solver step is one evaluation stage
-            r = run_srds(a, x0, f, w.tol, w.cache_thresh)
+            r = run_srds(a, x0, f_timed, w.tol, w.cache_thresh)
             iters += len(r.batches)
         else:
-            r = run_picard(a, x0, f, w.window, w.tol, w.cache_thresh, record=False,
+            r = run_picard(a, x0, f_timed, w.window, w.tol, w.cache_thresh, record=False,
                            eta=w.eta, noise=W.noise(w))
             iters += r.iters
         gens += 1
         if time.perf_counter() - t0 >= budget_s:
             break
     dt = time.perf_counter() - t0
-    return {"iters": iters, "generations": gens, "seconds": dt, "nfe_per_gen": r.nfe,
-            "iters_per_gen": r.iters}
+    return {"iters": iters, "generations": gens, "seconds": dt, "denoiser_seconds": t_eps[0],
+            "nfe_per_gen": r.nfe, "iters_per_gen": r.iters}
 
 
-def time_oracle_subprocess(workload_name, budget_s):
+def cpu_model():
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else platform)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.split(":")[0].strip() == "Model name":
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+def time_oracle_subprocess(workload_name, budget_s, threads=1, cache_thresh=None):
     env = dict(os.environ)
     for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
-        env[k] = "1"
+        env[k] = str(threads)
     env["CUDA_VISIBLE_DEVICES"] = ""
+    extra = [] if cache_thresh is None else ["--cache-thresh", repr(float(cache_thresh))]
     r = subprocess.run([sys.executable, os.path.abspath(__file__), "--workload", workload_name,
-                        "--oracle-sample", str(budget_s)], capture_output=True, text=True, env=env)
+                        "--oracle-sample", str(budget_s), *extra], capture_output=True, text=True, env=env)
     if r.returncode != 0:
         raise RuntimeError(f"oracle sample failed: {r.stderr[-2000:]}")
     return json.loads(r.stdout.strip().splitlines()[-1])
 
 
-def cpu_baseline(workload_name, budget_s=12.0):
-    s = time_oracle_subprocess(workload_name, budget_s)
-    return {"value": s["iters"] / s["seconds"], "unit": UNIT, "cores": 1, "kind": "oracle",
-            "sample": f"{s['generations']} full generation(s) of the workload "
-                      f"({s['iters']} solver steps, {s['seconds']:.1f} s) by the fp64 NumPy "
-                      f"oracle, single-threaded (BLAS/OpenMP threads = 1)"}
+def cpu_baseline(workload_name, budget_s=10.0, cache_thresh=None):
+    """The oracle on one host thread (the line's value) and on all of them
+    (BLAS/OpenMP threads = os.cpu_count(); NumPy's element-wise work stays on
+    one thread), with the solver step's share (the denoiser's time taken out)."""
+    ncpu = os.cpu_count() or 1
+    legs = {}
+    for name, thr in (("one_thread", 1), ("all_cores", ncpu)):
+        s = time_oracle_subprocess(workload_name, budget_s, threads=thr, cache_thresh=cache_thresh)
+        solver_s = max(s["seconds"] - s["denoiser_seconds"], 1e-12)
+        legs[name] = {"value": s["iters"] / s["seconds"], "threads": thr,
+                      "solver_step_us_per_iteration": 1e6 * solver_s / s["iters"],
+                      "solver_steps_per_s_denoiser_excluded": s["iters"] / solver_s,
+                      "sample": f"{s['generations']} full generation(s), {s['iters']} solver steps, "
+                                f"{s['seconds']:.1f} s ({s['denoiser_seconds']:.1f} s in the denoiser)"}
+    one = legs["one_thread"]
+    return {"value": one["value"], "unit": UNIT, "cores": 1, "kind": "oracle",
+            "sample": f"fp64 NumPy oracle, single-threaded (BLAS/OpenMP threads = 1): {one['sample']}",
+            "cpu_model": cpu_model(), "host_cores": ncpu,
+            "solver_step_us_per_iteration": one["solver_step_us_per_iteration"],
+            "all_cores": legs["all_cores"]}
 
 
 # ------------------------------------------------------------ reference ----
+
+def workload_config(w: W.Workload, world, steps_per_gen):
+    """The ``config`` of a bench line: the workload only, the same for both arms."""
+    return {"workload": w.name,
+            "step": ("one full cached Parareal generation (solver step = evaluation stage)"
+                     if w.sampler == "srds" else "one full cached-Picard generation"),
+            "solver_steps_per_step": int(steps_per_gen), "global_batch": w.batch * world, "seq_len": w.T,
+            "window": w.window, "latent": "x".join(map(str, w.latent_shape)), "mixture_components": w.K,
+            "tol": w.tol, "cache_thresh": w.cache_thresh, "eta": w.eta}
+
 
 def run_reference(args):
     rank, world, _ = rank_info()
     if rank != 0:
         return 0
     w = W.ALL[args.workload]
+    if args.cache_thresh is not None:
+        w = w.with_(cache_thresh=args.cache_thresh)
     # each step: one whole generation by the oracle, in its own process
     for _ in range(args.warmup):
-        time_oracle_subprocess(args.workload, 0.0)
+        time_oracle_subprocess(args.workload, 0.0, cache_thresh=args.cache_thresh)
     iters = 0
     secs = 0.0
+    per_gen = 0
     for _ in range(args.steps):
-        s = time_oracle_subprocess(args.workload, 0.0)
+        s = time_oracle_subprocess(args.workload, 0.0, cache_thresh=args.cache_thresh)
         iters += s["iters"]
         secs += s["seconds"]
+        per_gen = s["iters_per_gen"] if w.sampler != "srds" else s["iters"] // max(1, s["generations"])
     value = iters / secs
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000.0 * secs / args.steps, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": w.name,
-                   "step": ("one full cached Parareal generation (solver step = evaluation stage)"
-                            if w.sampler == "srds" else "one full cached-Picard generation"),
-                   "global_batch": w.batch, "seq_len": w.T, "window": w.window},
+        "config": workload_config(w, 1, per_gen),
         "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle",
                          "sample": f"{args.steps} full generation(s), fp64 NumPy oracle, "
-                                   f"single-threaded"},
+                                   f"single-threaded", "cpu_model": cpu_model(),
+                         "host_cores": os.cpu_count()},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -321,13 +396,19 @@ def run_ours(args):
     dev = torch.device("cuda", local)
     stream = torch.cuda.Stream(device=dev)
     torch.cuda.set_stream(stream)
-    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=stream)
-    if args.update_kernel is not None:
-        s.set_update_kernel(args.update_kernel)
-    if args.cache_bits == 16:
-        s.set_cache_precision(16)
-    if w.eta != 0.0:  # stochastic steps: the draws stay resident on the device
-        s.set_noise(w.eta, torch.from_numpy(W.noise(w)).to(dev))
+    noise_dev = torch.from_numpy(W.noise(w)).to(dev) if w.eta != 0.0 else None
+
+    def make_solver(cache_thresh):
+        sv = Solver(w.T, w.window, w.latent_shape, a, w.tol, cache_thresh, batch=w.batch, stream=stream)
+        if args.update_kernel is not None:
+            sv.set_update_kernel(args.update_kernel)
+        if args.cache_bits == 16:
+            sv.set_cache_precision(16)
+        if noise_dev is not None:  # stochastic steps: the draws stay resident on the device
+            sv.set_noise(w.eta, noise_dev)
+        return sv
+
+    s = make_solver(w.cache_thresh)
     max_rows = w.batch * s.window
     g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows, stream=stream)
     if args.gmm_form is not None:
@@ -337,30 +418,42 @@ def run_ours(args):
     flush = None if args.no_flush else torch.empty(FLUSH_BYTES, dtype=torch.uint8, device=dev)
     stream.synchronize()
 
-    def one_iteration():
-        bx, mb, nm = s.step_async()
+    def one_iteration(sv=None):
+        sv = s if sv is None else sv
+        bx, mb, nm = sv.step_async()
         g.eps(bx, mb, nm, eps)
-        s.submit_eps(eps)
+        sv.submit_eps(eps)
 
-    # learn the iteration count with the synchronous API (also a warm-up)
-    s.init(x_dev)
-    n_iters = 0
-    while True:
-        out = s.step()
-        if out is None:
-            break
-        g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
-        s.submit_eps(eps)
-        n_iters += 1
+    def run_sync(sv, record=None):
+        """One generation through the synchronous API; -> iterations. With a
+        list in `record`, the denoiser's eps rows of every iteration are kept."""
+        sv.init(x_dev)
+        n = 0
+        while True:
+            out = sv.step()
+            if out is None:
+                return n
+            g.eps(out.batch_x_ptr, out.miss_bt_ptr, sv.n_miss_dev(), eps)
+            if record is not None:
+                record.append(eps[: max(out.n_miss, 1)].clone())
+            sv.submit_eps(eps)
+            n += 1
+
+    # learn the iteration count with the synchronous API (also a warm-up),
+    # keeping the eps rows for the solver-only graph
+    eps_rec = []
+    n_iters = run_sync(s, eps_rec)
     st0 = s.stats()
     log = s.iter_log()
     nfe, hits = st0["nfe"], st0["hits"]
-    upd_bytes, other_bytes = iteration_bytes(log, w, 2 if args.cache_bits == 16 else 4)
+    fused = st0["update_kernel"] == 3
+    upd_bytes, gat_bytes, den_bytes = iteration_bytes(log, w, 2 if args.cache_bits == 16 else 4, fused)
+    step_bytes = upd_bytes + gat_bytes          # the solver step of each iteration
 
-    # One generation (n_iters Picard iterations: denoiser, update and planning
-    # kernels each -- the planning kernel decides and gathers the next batch;
-    # pa_init gathers the first) as a CUDA graph. The timed graph also records CUDA
-    # events around every update-kernel launch (the roofline's kernel time); the
+    # One generation (pa_init, then n_iters Picard iterations: the denoiser's
+    # two kernels and the solver step -- the fused step kernel, or the update
+    # and planning kernels) as a CUDA graph. The timed graph also records CUDA
+    # events around every denoiser call and every solver-step launch; the
     # plain graph has no event nodes and gives the iteration rate.
     s.init(x_dev)
     one_iteration()                       # eager warm-up of every launch path
@@ -368,6 +461,7 @@ def run_ours(args):
 
     den_events = []   # (before, after) the denoiser call of every iteration, timed graph only
     den_ms = [0.0]    # their total over the timed replays
+    init_launches = 2                     # pa_init: first plan and its gather
 
     def capture(timed):
         """-> (graph, kernels launched per iteration inside it)"""
@@ -395,8 +489,6 @@ def run_ours(args):
         l1 = s.stats()["launches"] + g.launches()
         return gr, (l1 - l0 - init_launches) // n_iters
 
-    # denoiser, update and planning (decision + next gather) kernels of one iteration
-    init_launches = 2                     # pa_init: first plan and its gather
     graph_plain, kernels_per_iter = capture(False)
     graph_timed, _ = capture(True)
 
@@ -415,54 +507,6 @@ def run_ours(args):
             den_ms[0] += sum(a.elapsed_time(b) for a, b in den_events)
         return ms, upd
 
-    def cold_iterations(reps):
-        """Per-iteration time with L2 flushed before every Picard iteration.
-        Iterations alternate between the two copies of the plan, so an even
-        and an odd iteration are captured and replayed in turn."""
-        single = [torch.cuda.CUDAGraph(), torch.cuda.CUDAGraph()]
-        s.init(x_dev)
-        stream.synchronize()
-        for k in range(2):
-            with torch.cuda.graph(single[k], stream=stream):
-                one_iteration()
-        tot, n = 0.0, 0
-        for _ in range(reps):
-            s.init(x_dev)
-            for it in range(n_iters):
-                if flush is not None:
-                    flush.zero_()
-                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-                e0.record(stream)
-                single[it % 2].replay()
-                e1.record(stream)
-                e1.synchronize()
-                tot += e0.elapsed_time(e1)
-                n += 1
-        return 1000.0 * tot / max(n, 1)
-
-    def timing_floor(reps=50):
-        """Event-pair time around a kernel that does no work (a one-element
-        fill), captured between two kernels in a graph like the update kernel's
-        events: the launch and completion latency inside every event-timed
-        launch."""
-        t1 = torch.zeros(1, device=dev)
-        ev = (torch.cuda.Event(enable_timing=True, external=True),
-              torch.cuda.Event(enable_timing=True, external=True))
-        gr = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(gr, stream=stream):
-            t1.add_(1.0)
-            ev[0].record(stream)
-            t1.fill_(0.0)
-            ev[1].record(stream)
-            t1.add_(1.0)
-        times = []
-        for r in range(reps + 3):
-            gr.replay()
-            stream.synchronize()
-            if r >= 3:
-                times.append(ev[0].elapsed_time(ev[1]))
-        return 1000.0 * float(np.median(times))  # the median: single replays can stall
-
     for _ in range(args.warmup):
         generation(graph_plain, False)
         generation(graph_timed, True)
@@ -475,14 +519,13 @@ def run_ours(args):
     barrier()
     stream.synchronize()
     wall0 = time.perf_counter()
-    dev_ms = upd_ms = timed_ms = 0.0
+    dev_ms = upd_ms = 0.0
     den_ms[0] = 0.0
     for _ in range(args.steps):
         a_ms, _ = generation(graph_plain, False)
         dev_ms += a_ms
         assert s.poll() == 0
-        t_ms, u_ms = generation(graph_timed, True)     # same work, update kernel bracketed by events
-        timed_ms += t_ms
+        _, u_ms = generation(graph_timed, True)     # same work, solver-step launches bracketed by events
         upd_ms += u_ms
         assert s.poll() == 0
     stream.synchronize()
@@ -493,54 +536,177 @@ def run_ours(args):
     time.sleep(0.2)
     clk = clocks.stop()
     launches = 2 * args.steps * (n_iters * kernels_per_iter + init_launches)   # both graphs, pa_init each
-    cold_us = cold_iterations(max(1, min(args.steps, 10)))
-    floor_us = timing_floor()
-
-    # Quality check of the paper's kind with latents in place of CLIP scores:
-    # the cached result against serial DDIM, which is the same library with a
-    # window of one point and no cache (every step evaluated in order).
     graph_plain.replay()
     stream.synchronize()
     assert s.poll() == 0
     x_cached = s.result().cpu().numpy()
+
+    # ---- the solver step alone ------------------------------------------
+    # The same generation with the recorded eps rows fed to pa_submit_eps and
+    # pa_debug_gap (an empty kernel with the same dependent-launch attribute)
+    # where the denoiser ran, so every solver kernel sees the dependency
+    # structure it has in a generation. pa_init is its own graph, replayed
+    # before the timed one; events around the iterations only.
+    g_init = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_init, stream=stream):
+        s.init(x_dev)
+    g_iter = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_iter, stream=stream):
+        for k in range(n_iters):
+            s.step_async()
+            s.submit_eps(eps_rec[k])
+            abi.pa_debug_gap(s.stream_ptr)
+    # one graph per iteration, for the L2-cold-before-every-iteration figure
+    # (captured from a fresh pa_init so that iteration k uses plan copy k mod 2,
+    # as after g_init)
+    s.init(x_dev)
+    stream.synchronize()
+    g_each = []
+    for k in range(n_iters):
+        gk = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gk, stream=stream):
+            s.step_async()
+            s.submit_eps(eps_rec[k])
+            abi.pa_debug_gap(s.stream_ptr)
+        g_each.append(gk)
+
+    def solver_only(do_flush, reps):
+        tot = 0.0
+        for _ in range(reps):
+            if do_flush and flush is not None:
+                flush.zero_()
+            g_init.replay()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            g_iter.replay()
+            e1.record(stream)
+            e1.synchronize()
+            tot += e0.elapsed_time(e1)
+        return 1000.0 * tot / (reps * n_iters)    # us per iteration
+
+    def solver_cold(reps):
+        """L2 flushed before every iteration, events around each iteration's graph."""
+        per = np.zeros(n_iters)
+        for _ in range(reps):
+            g_init.replay()
+            for k in range(n_iters):
+                if flush is not None:
+                    flush.zero_()
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record(stream)
+                g_each[k].replay()
+                e1.record(stream)
+                e1.synchronize()
+                per[k] += e0.elapsed_time(e1)
+        return 1000.0 * per / reps                 # us per iteration, per iteration index
+
+    solver_only(True, 3)                           # warm-up
+    so_reps = max(10, min(args.steps * 5, 200))
+    so_us = solver_only(True, so_reps)
+    so_warm_us = solver_only(False, so_reps)
+    cold_per = solver_cold(max(3, min(args.steps, 20)))
+    assert s.poll() == 0
+    so_log_ok = bool(np.array_equal(s.iter_log(), log))
+    so_x_ok = bool(np.array_equal(s.result().cpu().numpy(), x_cached))
+    assert so_log_ok and so_x_ok, "the solver-only replay diverged from the generation it was recorded from"
+    peak, peak_kind = measured_hbm_gbs()
+    alg_it = float(step_bytes.mean())
+    so_gbps = alg_it / (so_us * 1e-6) / 1e9
+    so_warm_gbps = alg_it / (so_warm_us * 1e-6) / 1e9
+    cold_gbps = float(step_bytes.sum()) / (float(cold_per.sum()) * 1e-6) / 1e9
+    sha = kernel_source_sha()
+    tkey = args.workload + ("-bf16" if args.cache_bits == 16 else "")
+    traffic = NCU_TRAFFIC.get((sha, tkey))
+    step_kernel = {3: "fused step (update, grid barrier, decision, next batch from registers)",
+                   2: "lean register update + planning kernel",
+                   1: "register-resident or staged update + planning kernel"}.get(st1["update_kernel"],
+                                                                                 "plain-load update + planning kernel")
+    solver_step = {
+        "kernels": step_kernel,
+        "us_per_iteration": so_us,
+        "alg_bytes_per_iteration": alg_it,
+        "gbps": so_gbps, "frac_of_measured_hbm": so_gbps / peak, "frac_of_nominal_8tbs": so_gbps / NOMINAL_HBM_GBS,
+        "us_per_iteration_warm_l2": so_warm_us, "gbps_warm_l2": so_warm_gbps,
+        "frac_warm_l2_of_measured_hbm": so_warm_gbps / peak,
+        "cold_l2_us_per_iteration": float(cold_per.mean()), "cold_l2_gbps": cold_gbps,
+        "cold_l2_frac_of_measured_hbm": cold_gbps / peak,
+        "cold_l2_us_by_iteration": [round(float(v), 2) for v in cold_per],
+        "steps_per_s": 1e6 / so_us,
+        "event_timed_launch_us": 1000.0 * upd_ms / max(1, args.steps * n_iters),
+        "timing": ("a CUDA graph of the generation's solver-step launches fed the eps rows recorded "
+                   "from the same generation, with pa_debug_gap (an empty kernel with the same "
+                   "dependent-launch attribute) where the denoiser ran; pa_init replayed before it, "
+                   "one event pair around the iterations, L2 flushed before each replay (warm_l2: "
+                   "not flushed). cold_l2: L2 flushed before every iteration, one graph and one event "
+                   "pair per iteration. event_timed_launch_us: events around each solver-step launch "
+                   "inside the full generation graph (the events cut the dependent-launch overlap)"),
+        "checks": "iteration log and x_T bitwise equal to the generation with the denoiser",
+    }
+    roofline = {"bound": "hbm", "achieved": so_gbps, "peak": peak, "unit": "GB/s",
+                "frac": so_gbps / peak, "traffic": traffic,
+                "kernel": "solver step: " + step_kernel,
+                "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
+                "alg_bytes_per_launch": alg_it,
+                "avg_launch_us": so_us,
+                "avg_launch_note": ("per iteration of the solver-only graph (one solver step and one empty "
+                                    "stand-in kernel per iteration, events around the whole graph): an upper "
+                                    "bound of the step's own launch time"),
+                "traffic_note": ("ncu dram read+write bytes per solver step, averaged over one generation; a "
+                                 "stored figure from an earlier capture of this command, keyed by the kernel "
+                                 "sources' hash (null: not captured for these sources)")}
+
+    # ---- uncached run alongside (tau_cache = 0: every window point evaluated)
+    su = make_solver(0.0)
+    un_iters = run_sync(su)
+    un_st = su.stats()
+    su.init(x_dev)
+    one_iteration(su)
+    stream.synchronize()
+    gu = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gu, stream=stream):
+        su.init(x_dev)
+        for _ in range(un_iters):
+            one_iteration(su)
+    un_ms = 0.0
+    un_reps = max(5, min(args.steps, 50))
+    for r in range(un_reps + 2):
+        if flush is not None:
+            flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        gu.replay()
+        e1.record(stream)
+        e1.synchronize()
+        if r >= 2:
+            un_ms += e0.elapsed_time(e1)
+    assert su.poll() == 0
+    x_uncached = su.result().cpu().numpy()
+    del gu
+    su.close()
+    un_ms /= un_reps
+    uncached = {"nfe_per_step": un_st["nfe"], "iters_per_step": un_iters, "ms_per_step": un_ms,
+                "value": un_iters / (un_ms / 1000.0),
+                "cached_speedup_per_generation": un_ms / (dev_ms / args.steps),
+                "nfe_reduction": 1.0 - nfe / max(1, un_st["nfe"])}
+
+    # Quality check of the paper's kind with latents in place of CLIP scores:
+    # the cached result against serial DDIM, which is the same library with a
+    # window of one point and no cache (every step evaluated in order).
     ser = Solver(w.T, 1, w.latent_shape, a, 0.0, 0.0, batch=w.batch, stream=stream)
-    if w.eta != 0.0:
-        ser.set_noise(w.eta, torch.from_numpy(W.noise(w)).to(dev))
-    ser.init(x_dev)
-    while True:
-        out = ser.step()
-        if out is None:
-            break
-        g.eps(out.batch_x_ptr, out.miss_bt_ptr, ser.n_miss_dev(), eps)
-        ser.submit_eps(eps)
+    if noise_dev is not None:
+        ser.set_noise(w.eta, noise_dev)
+    run_sync(ser)
     x_serial = ser.result().cpu().numpy()
     ser.close()
-    deviation = float((np.abs(x_cached - x_serial).max(axis=1) / np.abs(x_serial).max(axis=1)).max())
+
+    def dev_from_serial(x):
+        return float((np.abs(x - x_serial).max(axis=1) / np.abs(x_serial).max(axis=1)).max())
+
+    deviation = dev_from_serial(x_cached)
+    uncached["deviation_from_serial_ddim"] = dev_from_serial(x_uncached)
 
     units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
     value = units / secs
-    gb_step = (upd_bytes.sum() + other_bytes.sum()) * args.steps / (dev_ms / 1000.0) / 1e9
-
-    # roofline of the dominant kernel (Picard update)
-    peak, peak_kind = measured_hbm_gbs()
-    n_upd = args.steps * n_iters
-    achieved = upd_bytes.sum() * args.steps / (upd_ms / 1000.0) / 1e9
-    sha = kernel_source_sha()
-    traffic = NCU_TRAFFIC.get((sha, args.workload + ("-bf16" if args.cache_bits == 16 else "")))
-    roofline = {"bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
-                "frac": achieved / peak, "traffic": traffic,
-                "kernel": "Picard update (" + {2: "lean register form", 1: "register-resident or staged form, by shape"}
-                .get(st1["update_kernel"], "plain loads") + ")",
-                "traffic_note": "ncu dram read+write bytes per launch, averaged over one generation",
-                "peak_kind": f"{peak_kind} HBM copy bandwidth (of {peak_kind})",
-                "alg_bytes_per_launch": float(upd_bytes.mean()),
-                "avg_launch_us": 1000.0 * upd_ms / max(n_upd, 1),
-                "timing_floor_us": floor_us,
-                "timing_floor_note": "median event-pair time of a one-element fill at the same place in a graph: "
-                                     "launch and completion latency that every event-timed launch includes; "
-                                     "frac_excl_floor divides the bytes by avg_launch_us minus it"}
-    net_us = roofline["avg_launch_us"] - floor_us
-    roofline["frac_excl_floor"] = (float(upd_bytes.mean()) / (net_us * 1e-6) / 1e9 / peak) if net_us > 0 else None
 
     # End to end through the public API with host buffers (no flush): every
     # step copies x_init in from pinned host memory (pa_init), runs the
@@ -608,7 +774,7 @@ def run_ours(args):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(args.workload)
+        cpu = cpu_baseline(args.workload, cache_thresh=args.cache_thresh)
 
     if rank == 0:
         line = {
@@ -616,36 +782,28 @@ def run_ours(args):
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": dev_ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": w.name, "step": "one full cached-Picard generation",
-                       "picard_iters_per_step": n_iters, "global_batch": w.batch * world,
-                       "seq_len": w.T, "window": w.window, "latent": "x".join(map(str, w.latent_shape)),
-                       "mixture_components": w.K, "tol": w.tol, "cache_thresh": w.cache_thresh,
-                       "eta": w.eta,
-                       "cache_entries": "bf16" if args.cache_bits == 16 else "fp32",
+            "config": workload_config(w, world, n_iters),
+            "method": {"cache_entries": "bf16" if args.cache_bits == 16 else "fp32",
+                       "solver_step_kernels": step_kernel,
+                       "kernels_per_iteration": kernels_per_iter,
                        "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
                                                  if g.form() == 1 else "CUDA cores (fp32 FMA)"),
-                       "parallelism": f"replicas x{world} (independent trajectories)",
-                       "l2": ("not flushed" if args.no_flush else
+                       "parallelism": f"replicas x{world} (independent trajectories)"},
+            "timing": {"l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every generation (between timed steps), outside the "
                               "timed events"),
-                       "timing": "CUDA events around each generation: pa_init outside, then one CUDA-graph "
-                                 "replay of its Picard iterations (denoiser, update and planning kernels each; "
-                                 "the planning kernel decides and gathers the next batch) on the "
-                                 "launch stream; the update kernel's own events come from a second graph "
-                                 "of the same generation, replayed alternately"},
+                       "value": "CUDA events around each generation: one CUDA-graph replay of pa_init and its "
+                                "Picard iterations (denoiser and solver-step kernels each) on the launch "
+                                "stream"},
             "nfe_per_step": nfe, "hits_per_step": hits,
             "hit_rate": hits / max(1, hits + nfe),
             "deviation_from_serial_ddim": deviation,
-            "solver_step_gbps": gb_step,
+            "solver_step": solver_step,
+            "uncached": uncached,
             "denoiser_us_per_iteration": 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
-            "solver_us_per_iteration": 1000.0 * dev_ms / max(1, args.steps * n_iters)
-                                       - 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
-            "solver_note": ("denoiser time from CUDA events around each denoiser call in the timed graph "
-                            "(its event nodes cut the dependent-launch overlap there, so it is an upper "
-                            "bound); solver = the plain graph's iteration time minus it"),
-            "cold_iteration_us": cold_us,
-            "cold_iteration_note": "one Picard iteration with L2 flushed before every iteration, "
-                                   "CUDA events around each (conservative; includes one event pair per iteration)",
+            "denoiser_note": ("CUDA events around each denoiser call in the timed graph (its event nodes cut "
+                              "the dependent-launch overlap there, so it is an upper bound)"),
+            "denoiser_alg_bytes_per_iteration": float(den_bytes.mean()),
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,
@@ -654,6 +812,7 @@ def run_ours(args):
             "wall_s_timed_region": wall,
         }
         print(json.dumps(line))
+    del g_iter, g_init, g_each, graph_plain, graph_timed
     s.close()
     g.close()
     if world > 1:
@@ -839,7 +998,7 @@ def run_srds_bench(args, w):
 def main(argv=None):
     args = parse_args(argv)
     if args.oracle_sample is not None:
-        print(json.dumps(oracle_sample(args.workload, args.oracle_sample)))
+        print(json.dumps(oracle_sample(args.workload, args.oracle_sample, args.cache_thresh)))
         return 0
     if args.impl == "reference":
         return run_reference(args)

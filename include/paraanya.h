@@ -75,7 +75,7 @@ typedef struct {
   int32_t n_miss;        /* misses planned for the next iteration */
   int32_t device_status; /* 0, or the first device-side error code */
   int32_t update_kernel; /* kernel of the last pa_submit_eps: 0 plain loads, 1 bulk forms,
-                            2 lean register form, -1 none yet */
+                            2 lean register form, 3 fused step, -1 none yet */
 } pa_stats_t;
 
 /* ---- solver ------------------------------------------------------------ */
@@ -148,27 +148,39 @@ PA_API pa_status pa_step_async(pa_solver* s, const float** batch_x_dev,
 PA_API const int32_t* pa_n_miss_dev(const pa_solver* s);
 
 /* Hand back eps_theta for the planned misses: batch_eps_dev [M][D] fp32,
- * DEVICE pointer, 16-byte aligned for the lean and bulk update forms
+ * DEVICE pointer, 16-byte aligned for the fused, lean and bulk update forms
  * (otherwise the plain-load kernel runs). Runs Eq. 6 (assembly), Eq. 7 (cache update),
  * the drift and the Picard prefix sum (Eq. 1), the errors of Eq. 2 and the
- * cache distances of the next iteration (Eq. 4) in the update kernel, then the
- * window advance, the hit-miss plan of the next iteration (Eq. 5) and the
- * gather of its batch in the planning kernel. Asynchronous on the solver's
- * stream; batch_eps_dev must stay valid until the update kernel has run. */
+ * cache distances of the next iteration (Eq. 4), then the window advance
+ * (Sec. 2.1), the hit-miss plan of the next iteration (Eq. 5) and the gather
+ * of its batch (Sec. 2.2, one batched pass): by default in one fused kernel
+ * when all of its CTAs (one per 128 columns of each trajectory) fit on the
+ * GPU at once -- a cooperative launch with a bounded grid barrier --, else
+ * in an update kernel followed by a planning kernel. Asynchronous on the
+ * solver's stream; batch_eps_dev must stay valid until the update has run. */
 PA_API pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev);
 
 /* Synchronise and report: *n_active = trajectories not yet at t = T.
  * Returns PA_DONE when it is 0, or a device error status. */
 PA_API pa_status pa_poll(pa_solver* s, int* n_active);
 
-/* Final states x_T [batch][D] fp32 into a HOST or DEVICE pointer. Valid once
- * pa_step/pa_poll returned PA_DONE; PA_ERR_STATE before. Synchronises. */
+/* Final states x_T [batch][D] fp32 into a HOST or DEVICE pointer: the end
+ * point of Eq. 1's trajectory once the sliding window has reached T
+ * (Sec. 2.1: the window advances until every state has converged by Eq. 2).
+ * Valid once pa_step/pa_poll returned PA_DONE; PA_ERR_STATE before.
+ * Synchronises. */
 PA_API pa_status pa_result(pa_solver* s, float* x_out);
 
-/* Network evaluations so far (sum of misses). Synchronises; -1 on error. */
+/* Network evaluations so far: the sum over iterations of the misses, i.e. of
+ * |M| of Eq. 5 (hits reuse the cached eps of Eq. 6 and cost no evaluation),
+ * the NFE that Table 1 and Table 3 count per image. Synchronises; -1 on
+ * error. */
 PA_API int64_t pa_nfe(pa_solver* s);
 
-/* Counters, see pa_stats_t. Synchronises. */
+/* Counters, see pa_stats_t: the iterations, NFE and cache hits that the
+ * paper reports (Table 1: NFE; Table 3: iterations, NFE and hits per image),
+ * plus bookkeeping (launches, active trajectories, device status).
+ * Synchronises. */
 PA_API pa_status pa_stats(pa_solver* s, pa_stats_t* out);
 
 /* Per-iteration log, HOST buffer out[max_iters][batch][8] int32:
@@ -187,6 +199,13 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
 /* Select the Picard-update kernel (all forms compute Eq. 1, 2, 4, 6 and 7 of
  * one iteration; they differ in rounding order only, never in a decision
  * beyond the decision-margin guard):
+ *   3       the fused step (default when D % 4 == 0): the lean register form's
+ *           update, a grid barrier, the decision in every CTA and the next
+ *           batch written from registers, one kernel per iteration; used when
+ *           every CTA of its grid (ceil(D / 128) x batch) is resident at once
+ *           and batch * window <= 1024, else form 2 runs;
+ *   300 + n the fused step with lean launch shape n (0, 1, 4, 5 below; with
+ *           stochastic steps 0, 1, 3, 4);
  *   0       plain loads (one thread per column; any D);
  *   1       the bulk forms: register-resident rows, or rows staged in shared
  *           memory by bulk copies for windows the registers cannot hold;
@@ -220,10 +239,11 @@ PA_API pa_status pa_set_cache_precision(pa_solver* s, int bits);
 
 /* Fault-handling test hook: the number of tries (each may suspend for about
  * 10 us) after which an mbarrier wait of the bulk-copy update kernel counts
- * as timed out (default 2^17, about a second). With 0
- * every such wait gives up at once: the kernel records PA_ERR_TIMEOUT (read by
- * the next synchronising call), still drains its in-flight copies with the
- * default bound, and leaves the solver's numbers meaningless until pa_init. */
+ * as timed out (default 2^17, about a second); the fused step's grid barrier
+ * polls 16 times this many times. With 0 every such wait gives up at once:
+ * the kernel records PA_ERR_TIMEOUT (read by the next synchronising call),
+ * still drains its in-flight copies with the default bound, and leaves the
+ * solver's numbers meaningless until pa_init. */
 PA_API pa_status pa_debug_set_wait_limit(pa_solver* s, uint32_t polls);
 
 /* Enable (1) or disable (0) CUDA-event timing of every Picard-update kernel
@@ -238,6 +258,19 @@ PA_API pa_status pa_set_kernel_timing(pa_solver* s, int enable);
  * replay's times. Synchronises. */
 PA_API pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches, int reset);
 
+/* Timing aid: launches one kernel that does no work, with the programmatic
+ * dependent launch attribute that the library's own kernels carry, on a
+ * cudaStream_t (may be NULL). Placed between pa_submit_eps calls where the
+ * denoiser would run (eps replayed from a recorded run), it keeps the solver
+ * kernels' dependency structure -- each kernel reads before its dependency
+ * wait only what was written two or more kernels back -- so that the solver
+ * step can be timed alone. Not part of the method. */
+PA_API pa_status pa_debug_gap(void* stream);
+
+/* Release the solver handle (the host-side state machine of Sec. 2.1-2.2's
+ * iteration: the window, the plan and the counters). The caller-owned
+ * workspace, and with it the cache of Eq. 3, is not freed. Synchronises the
+ * solver's stream first; NULL is a no-op. */
 PA_API void pa_destroy(pa_solver* s);
 
 /* ---- Parareal (SRDS-style) sampling with the same cache ------------------

@@ -74,6 +74,7 @@ _PROTOS = {
     "pa_debug_set_wait_limit": (C.c_int, [VP, C.c_uint32]),
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
     "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.c_int]),
+    "pa_debug_gap": (C.c_int, [VP]),
     "pa_destroy": (None, [VP]),
     "pa_srds_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int64, C.c_int]),
     "pa_srds_create": (C.c_int, [PVP, C.c_int, C.POINTER(C.c_int64), C.c_int, C.POINTER(C.c_double),
@@ -258,6 +259,10 @@ def pa_kernel_timing(h, reset=True):
     n = C.c_int64()
     _check("pa_kernel_timing", lib().pa_kernel_timing(h, C.byref(ms), C.byref(n), int(bool(reset))))
     return ms.value, n.value
+
+
+def pa_debug_gap(stream_ptr):
+    return _check("pa_debug_gap", lib().pa_debug_gap(_dptr(stream_ptr)))
 
 
 def pa_destroy(h):

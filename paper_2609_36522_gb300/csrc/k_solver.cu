@@ -367,6 +367,17 @@ __global__ void __launch_bounds__(kPlanOneThreads) k_plan_one(Dev d, int par) {
 
 }  // namespace
 
+namespace {
+// No work: waits for its predecessor and lets its successor start, like the
+// library's other kernels (programmatic dependent launch).
+__global__ void k_gap() {
+  pdl_wait();
+  pdl_trigger();
+}
+}  // namespace
+
+cudaError_t launch_gap(cudaStream_t st) { return launch_ex(k_gap, dim3(1), dim3(32), 0, st, 0); }
+
 cudaError_t launch_init_plan(const Dev& d, cudaStream_t st) {
   k_init_plan<<<1, 256, 0, st>>>(d);
   return cudaGetLastError();

@@ -27,6 +27,17 @@
 //    written, widened exactly when read).
 // MINB CTAs per SM bound the registers: one CTA of 16 warps for windows up to
 // 112 positions, two of 8 warps up to 64, three of 8 warps up to 32.
+//
+// FUSE makes it the whole solver step of one iteration (launch_step_fused):
+// after the strip sums are added, a grid barrier (every CTA resident, a
+// cooperative launch) makes the Eq. 2 / Eq. 4 sums complete; every CTA then
+// reads them and takes the decision that ends the iteration (window advance,
+// hit/miss plan and ranks of the next iteration, pa_decide.cuh) -- the same
+// inputs and arithmetic give the same plan everywhere, CTA (0, 0) publishes it
+// and writes its strip of the next batch (a4) straight from the new states
+// still in its registers: the gather reads nothing. One kernel per iteration
+// instead of the update and planning kernels.
+#include "pa_decide.cuh"
 #include "pa_internal.h"
 
 namespace pa {
@@ -117,12 +128,94 @@ struct LeanShape {
   __host__ __device__ static size_t rank_bytes(int P) { return ((size_t)P * 4 + 127) / 128 * 128; }
   __host__ __device__ static size_t red_bytes(int P) { return ((size_t)2 * P * 33 * sizeof(float) + 127) / 128 * 128; }
   static constexpr size_t kTotBytes = (size_t)NW * 32 * 16;  // run totals, one float4 per lane and warp
-  __host__ __device__ static size_t smem_bytes(int T, int P, bool comp) {
-    return coef_bytes(T) + rank_bytes(P) + red_bytes(P) + kTotBytes * (comp ? 2 : 1);
+  // the fused step's complete sums, err and distance of every (b, j), fp64
+  __host__ __device__ static size_t sum_bytes(int B, int P) { return (size_t)2 * B * P * sizeof(double); }
+  __host__ __device__ static size_t smem_bytes(int T, int P, bool comp, int B = 0) {
+    return sum_bytes(B, P) + coef_bytes(T) + rank_bytes(P) + red_bytes(P) + kTotBytes * (comp ? 2 : 1);
   }
 };
 
-template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
+// The complete sums as the decision reads them (shared memory, divided by D).
+struct LeanRed {
+  const double* e;
+  const double* dl;
+  __device__ double err(int q) const { return e[q]; }
+  __device__ double del(int q) const { return dl[q]; }
+};
+
+
+// The fused step after the update: grid barrier, the complete sums, the
+// decision in every CTA, and the warp's share of the next batch from the new
+// states in `xn` (states t + j0 + 1 .. t + j0 + nj of trajectory tr; NULL for a
+// finished trajectory). Every thread of every CTA calls it.
+template <int NW, int LMAX>
+__device__ __forceinline__ void step_tail(const Dev& d, DecideShared& ds, double* s_sum, int par, const Traj& tr,
+                                          const Q* xn, int j0, int nj, int mycol, int D, bool live) {
+  const int tid = threadIdx.x;
+  const int B = d.B, P = d.P, npair = B * P;
+  const unsigned long long ncta = (unsigned long long)gridDim.x * gridDim.y;
+  // the spin polls an L2 line (about half a microsecond each): 16 x the
+  // mbarrier limit keeps the same order of time, about a second
+  const uint32_t spin = d.wait_limit > (0xffffffffu >> 4) ? 0xffffffffu : d.wait_limit << 4;
+  if (!grid_sync(d.gbar, ncta, spin)) {
+    if (tid == 0) atomicCAS(&d.ctl->status, kDevOk, kDevTimeout);
+    return;  // the plan is not published; the host reports PA_ERR_TIMEOUT
+  }
+  const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
+  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
+  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
+  const double inv_d = 1.0 / (double)d.D;
+  double* s_e = s_sum;
+  double* s_d = s_sum + npair;
+  for (int q = tid; q < npair; q += NW * 32) {
+    const size_t o = (size_t)q * kAccStride;
+    const double ve = __ldcg(acc_e + o) * inv_d, vd = __ldcg(acc_d + o) * inv_d;
+    s_e[q] = ve;
+    s_d[q] = vd;
+    if (publish) {
+      d.red_err[q] = (float)ve;
+      d.red_del[q] = (float)vd;
+      double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;  // iteration k+1 adds into these
+      nxt[o] = 0.0;
+      nxt[(size_t)npair * kAccStride + o] = 0.0;
+    }
+  }
+  __syncthreads();
+  decide_par(d, ds, LeanRed{s_e, s_d}, par, publish, -1);
+  __syncthreads();  // the next plan (ds.tn, ds.pn, chunk masks and bases) is known
+  if (xn == nullptr || !live || nj <= 0) return;
+  // a4 of the next iteration: its timestep i (tn <= i < tn + pn) reads state
+  // min(i, t + p) -- states past the frontier t + p are lazy copies of it --
+  // which this warp holds if it is one of t + j0 + 1 .. t + j0 + nj
+  const int b = blockIdx.y;
+  const int tn = ds.tn[b], pn = ds.pn[b];
+  const int s_end = tr.t + tr.p;  // the new frontier (last computed state)
+  auto miss_rank = [&](int i) -> int {  // rank of next-window timestep i, -1 for a hit
+    const int q = b * P + (i - tn);
+    const unsigned mm = ds.cmiss[q >> 5];
+    const unsigned bit = 1u << (q & 31);
+    return (mm & bit) ? ds.cbase[q >> 5] + __popc(mm & (bit - 1u)) : -1;
+  };
+  Q last = xn[0];
+#pragma unroll
+  for (int g = 0; g < LMAX; ++g) {
+    if (g >= nj) break;
+    const int s = tr.t + j0 + g + 1;  // the state xn[g] holds
+    last = xn[g];
+    if (s < s_end && s >= tn && s < tn + pn) {
+      const int r = miss_rank(s);
+      if (r >= 0) stq(d.batch_x + (int64_t)r * D + mycol, xn[g]);
+    }
+  }
+  if (j0 + nj == tr.p) {  // this warp holds the frontier state: it also serves the lazy timesteps
+    for (int i = max(tn, s_end); i < tn + pn; ++i) {
+      const int r = miss_rank(i);
+      if (r >= 0) stq(d.batch_x + (int64_t)r * D + mycol, last);
+    }
+  }
+}
+
+template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false, bool FUSE = false>
 __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const float* __restrict__ beps, int par) {
   using Sh = LeanShape<NW, NOISE>;
   using CT = typename Coef<NOISE>::T;
@@ -130,17 +223,22 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int T = d.T, P = d.P, b = blockIdx.y;
   const int D = (int)d.D;  // (P + 1) * D and T * D fit in int32 (launcher)
-  CT* s_coef = reinterpret_cast<CT*>(smem_raw);
-  int32_t* s_rank = reinterpret_cast<int32_t*>(smem_raw + Sh::coef_bytes(T));
-  float* s_red = reinterpret_cast<float*>(smem_raw + Sh::coef_bytes(T) + Sh::rank_bytes(P));  // [2][P][33]
-  float4* s_tot = reinterpret_cast<float4*>(smem_raw + Sh::coef_bytes(T) + Sh::rank_bytes(P) + Sh::red_bytes(P));
+  const size_t o_sum = FUSE ? Sh::sum_bytes(d.B, P) : 0;
+  double* s_sum = reinterpret_cast<double*>(smem_raw);  // FUSE: [2][B][P]
+  CT* s_coef = reinterpret_cast<CT*>(smem_raw + o_sum);
+  int32_t* s_rank = reinterpret_cast<int32_t*>(smem_raw + o_sum + Sh::coef_bytes(T));
+  float* s_red = reinterpret_cast<float*>(smem_raw + o_sum + Sh::coef_bytes(T) + Sh::rank_bytes(P));  // [2][P][33]
+  float4* s_tot =
+      reinterpret_cast<float4*>(smem_raw + o_sum + Sh::coef_bytes(T) + Sh::rank_bytes(P) + Sh::red_bytes(P));
   float4* s_lo = s_tot + NW * 32;  // COMP only
+  __shared__ DecideShared ds;      // FUSE only (the compiler drops it otherwise)
 
   // Prologue: everything here was written two or more kernels back (plan,
   // ranks, n_miss by the planning kernel; coefficients at creation). None of
   // it depends on the plan, so all of it is in flight at once.
   const Traj tr = d.traj[par * d.B + b];
   const int n_miss = d.ctl->n_miss;
+  if constexpr (FUSE) decide_load<NW * 32>(d, ds, par);  // the plan of every trajectory, for the decision
   for (int i = tid; i < T; i += NW * 32) {
     CT c;
     if constexpr (NOISE) {
@@ -160,7 +258,13 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   }
   if (tr.p == 0) {  // finished trajectory; every CTA passes the dependency wait before it exits
     pdl_wait();
-    return;
+    if constexpr (!FUSE) {
+      return;
+    } else {  // the fused step still meets the barrier and takes the decision
+      pdl_trigger();
+      step_tail<NW, LMAX>(d, ds, s_sum, par, tr, nullptr, 0, 0, 0, 0, false);
+      return;
+    }
   }
   __syncthreads();
 
@@ -307,6 +411,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
         }
         stq(Xw + so * D, n);
         Q df = qsub(n, x[g + 1]);  // against the old state i+1 (lazy-resolved)
+        if constexpr (FUSE) ep[g] = n;  // the drift is spent: keep the new state for the next batch
         const float2 e2 = __ffma2_rn(df.h, df.h, __fmul2_rn(df.l, df.l));
         ev = e2.x + e2.y;
         if (j + 1 < p) {
@@ -340,6 +445,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
     }
     red_add(d, par, which, b * P + j, (a0 + a1) + (a2 + a3));
   }
+  if constexpr (FUSE) step_tail<NW, LMAX>(d, ds, s_sum, par, tr, ep, j0, nj, mycol, D, live);
 }
 
 template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
@@ -361,6 +467,43 @@ cudaError_t launch_lean(const Dev& d, const float* beps, int par, cudaStream_t s
 }
 
 constexpr size_t kLeanSmemMax = 200 * 1024;
+
+// The fused step: launched cooperatively, so only when every CTA of the grid
+// (a strip of 128 columns of each trajectory) can be resident at once;
+// cudaErrorNotSupported otherwise (the caller then launches the update and
+// planning kernels).
+template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
+cudaError_t launch_fused(const Dev& d, const float* beps, int par, cudaStream_t st) {
+  using Sh = LeanShape<NW, NOISE>;
+  const int nstrip = (int)((d.D + 127) / 128);
+  const size_t smem = Sh::smem_bytes(d.T, d.P, COMP, d.B);
+  if (smem > kLeanSmemMax) return cudaErrorNotSupported;
+  auto kern = k_update_lean<NW, LMAX, MINB, NOISE, COMP, CB, true>;
+  // per device: the dynamic shared memory configured and the resident CTAs
+  // the whole GPU holds at that size
+  static size_t configured[64] = {};
+  static size_t cap_smem[64] = {};
+  static int capacity[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= 64) return cudaErrorNotSupported;
+  if (smem > configured[dev]) {
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    configured[dev] = smem;
+  }
+  if (smem != cap_smem[dev]) {
+    int per_sm = 0, nsm = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, NW * 32, smem);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&nsm, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    capacity[dev] = per_sm * nsm;
+    cap_smem[dev] = smem;
+  }
+  if ((int64_t)nstrip * d.B > capacity[dev]) return cudaErrorNotSupported;
+  return launch_ex_coop(kern, dim3(nstrip, d.B, 1), dim3(NW * 32), smem, st, 0, true, d, beps, par);
+}
 
 }  // namespace
 
@@ -410,6 +553,41 @@ cudaError_t launch_update_lean(const Dev& d, const float* batch_eps, int par, in
   if (s == 2) return launch_lean<12, 9, 1, false, false>(d, batch_eps, par, st);
   if (s == 3) return launch_lean<8, 4, 2, false, false>(d, batch_eps, par, st);
   return launch_lean<8, 8, 2, false, false>(d, batch_eps, par, st);
+}
+
+// Fused step shapes: as launch_update_lean's (0 = by window, also with
+// stochastic steps); compensated sums are not offered.
+cudaError_t launch_step_fused(const Dev& d, const float* batch_eps, int par, int shape, cudaStream_t st) {
+  if (!step_fused_supported(d, batch_eps, shape)) return cudaErrorNotSupported;
+  int s = shape % 10;
+  // by window, as the lean form; with draws 16 x 7 above 32 positions (8 x 8
+  // would spill)
+  if (s == 0) s = d.P <= 32 ? (d.noise ? 3 : 5) : (d.P <= 64 && !d.noise) ? 4 : 1;
+  static const int kWarps[7] = {0, 16, 12, 8, 8, 8, 4};
+  static const int kRun[7] = {0, 7, 9, 4, 8, 4, 8};
+  if (s > 6 || d.P > kWarps[s] * kRun[s]) return cudaErrorNotSupported;
+  if (d.cache_bf16) {
+    if (s == 5) return launch_fused<8, 4, 3, false, false, true>(d, batch_eps, par, st);
+    if (s == 4) return launch_fused<8, 8, 2, false, false, true>(d, batch_eps, par, st);
+    if (s == 1) return launch_fused<16, 7, 1, false, false, true>(d, batch_eps, par, st);
+    return cudaErrorNotSupported;
+  }
+  if (d.noise) {
+    if (s == 1) return launch_fused<16, 7, 1, true, false>(d, batch_eps, par, st);
+    if (s == 3) return launch_fused<8, 4, 2, true, false>(d, batch_eps, par, st);
+    if (s == 4) return launch_fused<8, 8, 2, true, false>(d, batch_eps, par, st);
+    return cudaErrorNotSupported;
+  }
+  if (s == 1) return launch_fused<16, 7, 1, false, false>(d, batch_eps, par, st);
+  if (s == 4) return launch_fused<8, 8, 2, false, false>(d, batch_eps, par, st);
+  if (s == 5) return launch_fused<8, 4, 3, false, false>(d, batch_eps, par, st);
+  return cudaErrorNotSupported;
+}
+
+bool step_fused_supported(const Dev& d, const float* batch_eps, int shape) {
+  // every CTA decides in shared memory from one miss mask per 32-position chunk
+  if (shape >= 10 || (int64_t)d.B * d.P > 32 * 32) return false;
+  return update_lean_supported(d, batch_eps);
 }
 
 bool update_lean_supported(const Dev& d, const float* batch_eps) {

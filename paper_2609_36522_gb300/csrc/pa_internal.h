@@ -61,7 +61,7 @@ struct PlanCtr {
 
 struct Layout {
   size_t X, Xhat, Ehat, batch_x, coef, traj, pc, ctl, rank, miss_bt;
-  size_t acc, red_err, red_del, iter_log, total;
+  size_t acc, red_err, red_del, iter_log, gbar, total;
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -85,6 +85,7 @@ inline Layout make_layout(int T, int P, int64_t D, int B) {
   L.red_err = take((size_t)B * P * sizeof(float));
   L.red_del = take((size_t)B * P * sizeof(float));
   L.iter_log = take((size_t)(T + 1) * B * kLogFields * sizeof(int32_t));
+  L.gbar = take(128);                              // arrival counter of the fused step's grid barrier
   L.total = o;
   return L;
 }
@@ -108,6 +109,7 @@ struct Dev {
   float* red_err;     // [B][P] the last decision's reductions (divided by D), for the host
   float* red_del;
   int32_t* iter_log;  // [T+1][B][kLogFields]
+  unsigned long long* gbar;  // arrivals at the fused step's grid barrier (cleared by pa_init)
   int T, P, B;
   int64_t D;
   double tol, cache_thresh;   // compared against the fp64 sums divided by D
@@ -133,17 +135,18 @@ __device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.lau
 
 bool pdl_enabled();  // false when the environment sets PA_DISABLE_PDL=1
 
-// cudaLaunchKernelEx with the PDL attribute (when enabled) and an optional
-// cluster width along x (0 = no cluster attribute).
+// cudaLaunchKernelEx with the PDL attribute (when enabled), an optional
+// cluster width along x (0 = no cluster attribute) and, with `coop`, the
+// cooperative attribute (every CTA resident at once, for a grid barrier).
 template <typename... KArgs, typename... Args>
-cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
-                      unsigned cluster_x, Args&&... args) {
+cudaError_t launch_ex_coop(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                           unsigned cluster_x, bool coop, Args&&... args) {
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = grid;
   cfg.blockDim = block;
   cfg.dynamicSmemBytes = smem;
   cfg.stream = st;
-  cudaLaunchAttribute attr[2];
+  cudaLaunchAttribute attr[3];
   unsigned n = 0;
   if (pdl_enabled()) {
     attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
@@ -157,9 +160,20 @@ cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem
     attr[n].val.clusterDim.z = 1;
     ++n;
   }
+  if (coop) {
+    attr[n].id = cudaLaunchAttributeCooperative;
+    attr[n].val.cooperative = 1;
+    ++n;
+  }
   cfg.attrs = attr;
   cfg.numAttrs = n;
   return cudaLaunchKernelEx(&cfg, kern, static_cast<Args&&>(args)...);
+}
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_ex(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                      unsigned cluster_x, Args&&... args) {
+  return launch_ex_coop(kern, grid, block, smem, st, cluster_x, false, static_cast<Args&&>(args)...);
 }
 
 // Cache entries stored as bfloat16 (a storage option, not from the paper):
@@ -193,12 +207,58 @@ struct Bf16Row<1> {
   }
 };
 
+// A CTA's partial of an Eq. 2 / Eq. 4 sum (non-negative fp32) as it enters the
+// fp64 accumulators: rounded up to a multiple of 2^-32. Every term is then a
+// multiple of 2^-32 and every partial sum of such terms below 2^21 is exactly
+// representable in fp64 (2^21 / 2^-32 = 2^53), so the accumulated sum is exact
+// -- the same whatever order the CTAs arrive in -- as long as it stays below
+// 2^21; above that the sum divided by D is at least 2^21 / D (>= 32 for rows of
+// up to 65536 values), far beyond any tolerance the decision compares it
+// with. Rounding up keeps a nonzero partial nonzero (tol = 0 stays exact) and
+// moves a sum by at most one 2^-32 per CTA.
+__device__ __forceinline__ double quantize_partial(float v) {
+  return ceil((double)v * 4294967296.0) * (1.0 / 4294967296.0);
+}
+
 // One CTA's share of the Eq. 2 error (which = 0) or Eq. 4 distance (which =
 // 1) of window position q = b*P + j, added into the accumulator set of the
-// iteration's parity. fp64 sums of fp32 CTA partials: the rounding of the
-// order in which CTAs arrive is far below the fp32 partials' own.
+// iteration's parity (exact, see quantize_partial).
 __device__ __forceinline__ void red_add(const Dev& d, int par, int which, int q, float v) {
-  atomicAdd(d.acc + ((size_t)(par * 2 + which) * d.B * d.P + q) * kAccStride, (double)v);
+  atomicAdd(d.acc + ((size_t)(par * 2 + which) * d.B * d.P + q) * kAccStride, quantize_partial(v));
+}
+
+// Grid-wide barrier of a launch whose CTAs are all resident at once (the
+// fused step kernel, launched cooperatively). Thread 0 of each CTA publishes
+// the CTA's writes (fence), adds one to the counter and waits until the count
+// reaches the next multiple of the grid size: launches of one solver never
+// overlap at the barrier (each starts its arrivals after the previous one
+// completed), so the count before an arrival identifies the launch. The wait
+// polls at most `limit` times; false = it ran out (the caller records
+// PA_ERR_TIMEOUT and returns). Every thread of the CTA must call it.
+__device__ __forceinline__ bool grid_sync(unsigned long long* ctr, unsigned long long n, uint32_t limit) {
+  __shared__ int s_ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    const unsigned long long old = atomicAdd(ctr, 1ull);
+    const unsigned long long target = (old / n + 1ull) * n;
+    int ok = 1;
+    if (old + 1ull != target) {
+      for (uint32_t polls = 0;; ++polls) {
+        if (polls >= limit) {  // limit 0: every CTA but the last to arrive gives up at once
+          ok = 0;
+          break;
+        }
+        unsigned long long v;
+        asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(ctr) : "memory");
+        if (v >= target) break;
+      }
+    }
+    __threadfence();
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
 }
 
 // Kernel launchers (k_solver.cu). Each returns the launch error. par = k mod 2
@@ -216,5 +276,13 @@ bool update_bulk_supported(const Dev& d, const float* batch_eps);
 // the shape cannot hold the window)
 cudaError_t launch_update_lean(const Dev& d, const float* batch_eps, int par, int shape, cudaStream_t st);
 bool update_lean_supported(const Dev& d, const float* batch_eps);
+// The fused step (k_update_lean.cu): the lean update, a grid barrier, the
+// decision in every CTA and the next batch written from registers -- one
+// kernel per iteration in place of the update and planning kernels. Only for
+// grids that are resident in one wave; cudaErrorNotSupported otherwise.
+cudaError_t launch_step_fused(const Dev& d, const float* batch_eps, int par, int shape, cudaStream_t st);
+bool step_fused_supported(const Dev& d, const float* batch_eps, int shape);
+// An empty kernel with programmatic dependent launch (k_solver.cu)
+cudaError_t launch_gap(cudaStream_t st);
 
 }  // namespace pa

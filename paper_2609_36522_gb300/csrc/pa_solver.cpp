@@ -40,7 +40,7 @@ struct pa_solver {
   char* ws;
   cudaStream_t st;
   St state;
-  int update_kind;   // requested: 0 plain, 1 bulk pipeline, 2 lean register form
+  int update_kind;   // requested: 0 plain, 1 bulk pipeline, 2 lean register form, 3 fused step
   int lean_shape;    // launch shape of the lean register form
   int last_kind;     // kernel the last pa_submit_eps actually launched (-1: none yet)
   int64_t k;         // pa_submit_eps calls since pa_init: the plan of iteration k is copy k mod 2
@@ -213,12 +213,15 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.red_err = reinterpret_cast<float*>(w + L.red_err);
   d.red_del = reinterpret_cast<float*>(w + L.red_del);
   d.iter_log = reinterpret_cast<int32_t*>(w + L.iter_log);
+  d.gbar = reinterpret_cast<unsigned long long*>(w + L.gbar);
   d.T = T; d.P = P; d.B = batch; d.D = D;
   d.tol = tol;
   d.cache_thresh = cache_thresh;
   d.wait_limit = pa::kWaitLimit;
   d.cache_bf16 = 0;
-  s->update_kind = (D % 4 == 0) ? 2 : 0;  // lean register form, else the bulk forms, else plain loads
+  // the fused step where its grid is resident in one wave, else the lean
+  // register form and the planning kernel, else the bulk forms, else plain loads
+  s->update_kind = (D % 4 == 0) ? 3 : 0;
 
   const std::vector<float> hc = step_coefficients(s->alphas, 0.0);  // DDIM (eta = 0)
   cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), sizeof(pa::Ctl), cudaHostAllocDefault);
@@ -267,6 +270,7 @@ pa_status pa_init(pa_solver* s, const float* x_init) {
   if (e != cudaSuccess) return cuda_fail("pa_init: copy x_init", e);
   // both accumulator sets of the reductions start at zero
   e = cudaMemsetAsync(d.acc, 0, (size_t)2 * 2 * d.B * d.P * pa::kAccStride * sizeof(double), s->st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(d.gbar, 0, sizeof(unsigned long long), s->st);  // barrier arrivals
   if (e != cudaSuccess) return cuda_fail("pa_init: clear sums", e);
   // the first plan (every timestep a first entry) and its batch
   e = pa::launch_init_plan(d, s->st);
@@ -330,8 +334,17 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
     if (e == cudaSuccess) e = record_timing_event(s->ev[2 * s->ev_next], s->st);
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
   }
-  bool done = false;
-  if (s->update_kind == 2 && pa::update_lean_supported(s->d, batch_eps_dev)) {
+  bool done = false, planned = false;
+  if (s->update_kind == 3) {
+    e = pa::launch_step_fused(s->d, batch_eps_dev, par, s->lean_shape, s->st);
+    if (e == cudaErrorNotSupported) {
+      e = cudaSuccess;  // the grid is not resident in one wave: update and planning kernels
+    } else {
+      s->last_kind = 3;
+      done = planned = true;
+    }
+  }
+  if (!done && s->update_kind >= 2 && pa::update_lean_supported(s->d, batch_eps_dev)) {
     e = pa::launch_update_lean(s->d, batch_eps_dev, par, s->lean_shape, s->st);
     if (e == cudaErrorNotSupported) {
       e = cudaSuccess;  // this shape cannot hold the window: the bulk forms below
@@ -355,10 +368,12 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
     s->ev_next++;
   }
-  int nl = 0;
-  e = pa::launch_plan(s->d, par, s->st, &nl);
-  s->launches += nl;
-  if (e != cudaSuccess) return cuda_fail("pa_submit_eps: plan", e);
+  if (!planned) {  // the fused step took the decision and gathered the next batch itself
+    int nl = 0;
+    e = pa::launch_plan(s->d, par, s->st, &nl);
+    s->launches += nl;
+    if (e != cudaSuccess) return cuda_fail("pa_submit_eps: plan", e);
+  }
   s->k++;
   s->state = St::Ready;
   return PA_OK;
@@ -442,7 +457,7 @@ pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out) {
 
 pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   if (!s) return arg_fail("pa_set_update_kernel: solver is NULL");
-  if (kind == 0 || kind == 1 || kind == 2) {
+  if (kind == 0 || kind == 1 || kind == 2 || kind == 3) {
     s->update_kind = kind;
     s->lean_shape = 0;
     s->d.bulk_cfg = 0;
@@ -453,8 +468,13 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
     s->update_kind = 2;
     s->lean_shape = kind - 200;
     s->d.bulk_cfg = 0;
+  } else if (kind >= 300 && kind <= 306) {
+    s->update_kind = 3;
+    s->lean_shape = kind - 300;
+    s->d.bulk_cfg = 0;
   } else {
-    return arg_fail("pa_set_update_kernel: kind must be 0, 1, 2, 100 + bulk launch shape or 200 + lean launch shape");
+    return arg_fail("pa_set_update_kernel: kind must be 0, 1, 2, 3, 100 + bulk launch shape, "
+                    "200 + lean launch shape or 300 + fused-step launch shape");
   }
   return PA_OK;
 }
@@ -496,6 +516,12 @@ pa_status pa_kernel_timing(pa_solver* s, double* update_ms, int64_t* n_launches,
   *update_ms = tot;
   *n_launches = (int64_t)s->ev_next;
   if (reset) s->ev_next = 0;
+  return PA_OK;
+}
+
+pa_status pa_debug_gap(void* stream) {
+  const cudaError_t e = pa::launch_gap(static_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) return cuda_fail("pa_debug_gap", e);
   return PA_OK;
 }
 

@@ -17,12 +17,13 @@ def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True, cache_store=Non
 
 
 def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=None,
-            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None):
+            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None, reductions=False):
     """Run one generation on the GPU.
 
     eps_source: "gmm" (the CUDA mixture kernel) or "oracle" (fp64 mixture
     posterior evaluated on the host for the gathered batch, rounded to fp32).
     mode: "sync" (pa_step) or "async" (pa_step_async, device-side counts).
+    reductions: keep every iteration's Eq. 2 / Eq. 4 reductions (sync mode).
     """
     import torch
     from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
@@ -55,6 +56,7 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
     s.init(x_init)
     misses = []
     batches = []
+    reds = []
     if mode == "sync":
         while True:
             out = s.step()
@@ -71,6 +73,8 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
                 eps_buf[:n].copy_(torch.from_numpy(e.astype(np.float32)))
             batches.append(n)
             s.submit_eps(eps_buf)
+            if reductions:
+                reds.append(s.last_reductions())
     else:
         if eps_source != "gmm":
             raise ValueError("async mode needs the device-side denoiser")
@@ -81,7 +85,7 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
         s.poll()
     xT = s.result().cpu().numpy()
     res = dict(x_final=xT, nfe=s.nfe(), stats=s.stats(), log=s.iter_log(), misses=misses,
-               batches=batches, gmm_launches=g.launches())
+               batches=batches, gmm_launches=g.launches(), reductions=reds)
     s.close()
     g.close()
     return res

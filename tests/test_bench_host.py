@@ -56,16 +56,55 @@ def test_iteration_bytes_counts_rows():
     import numpy as np
     import bench
     w = W.TINY
-    # one trajectory: t=0, p=8, 8 misses, stride 4, frontier 0 (all lazy), no hits
-    log = np.zeros((1, 1, 8), dtype=np.int32)
+    # iteration 0: t=0, p=8, 8 misses, stride 4, frontier 0 (all lazy), no hits;
+    # iteration 1: t=4, p=8, 5 misses, stride 8, frontier 8, 3 hits at j >= 1
+    log = np.zeros((2, 1, 8), dtype=np.int32)
     log[0, 0, :6] = (0, 8, 8, 4, 0, 0)
-    upd, other = bench.iteration_bytes(log, w)
+    log[1, 0, :6] = (4, 8, 5, 8, 8, 3)
+    upd, gat, den = bench.iteration_bytes(log, w)
     row = w.D * 4
     assert upd[0] == (1 + 0 + 8 + 16 + 0 + 8) * row
-    assert other[0] == (4 * 8 + w.K) * row
+    # iteration 1: lazy = 4 + 8 - 8 = 4; 3 ehat hits; 10 entry writes; 3 xhat reads
+    assert upd[1] == (1 + 4 + 5 + 8) * row + (3 + 10 + 3) * row
+    # the planning kernel gathers iteration 1's 5 rows after iteration 0 (read
+    # and write), nothing after the last iteration; the fused step only writes
+    assert gat[0] == 2 * 5 * row and gat[1] == 0
+    _, gat_f, _ = bench.iteration_bytes(log, w, fused=True)
+    assert gat_f[0] == 5 * row and gat_f[1] == 0
+    assert den[0] == (2 * 8 + w.K) * row and den[1] == (2 * 5 + w.K) * row
     # bfloat16 entries: the 16 entry writes count half a row each
-    upd16, _ = bench.iteration_bytes(log, w, entry_bytes=2)
+    upd16, _, _ = bench.iteration_bytes(log, w, entry_bytes=2)
     assert upd16[0] == (1 + 0 + 8 + 8) * row + 16 * (row // 2)
+
+
+def test_cpu_baseline_legs(monkeypatch):
+    """cpu_baseline reports the one-thread leg as its value, an all-cores leg
+    beside it, the CPU model and the solver step with the denoiser excluded."""
+    import bench
+    calls = []
+
+    def fake(name, budget, threads=1, cache_thresh=None):
+        calls.append(threads)
+        return {"iters": 8, "generations": 2, "seconds": 2.0, "denoiser_seconds": 1.5,
+                "nfe_per_gen": 10, "iters_per_gen": 4}
+
+    monkeypatch.setattr(bench, "time_oracle_subprocess", fake)
+    cb = bench.cpu_baseline("tiny", budget_s=0.0)
+    assert calls == [1, os.cpu_count() or 1]
+    assert cb["cores"] == 1 and cb["value"] == 4.0 and cb["kind"] == "oracle"
+    assert cb["host_cores"] == (os.cpu_count() or 1) and cb["cpu_model"]
+    assert abs(cb["solver_step_us_per_iteration"] - 1e6 * 0.5 / 8) < 1e-6
+    assert cb["all_cores"]["threads"] == (os.cpu_count() or 1)
+    assert abs(cb["all_cores"]["solver_steps_per_s_denoiser_excluded"] - 16.0) < 1e-9
+
+
+def test_reference_config_matches_ours():
+    """Both arms carry the same workload-only config for the same workload."""
+    import bench
+    w = W.SD15
+    c = bench.workload_config(w, 1, 4)
+    assert c["workload"] == w.name and c["solver_steps_per_step"] == 4 and c["window"] == 100
+    assert set(c) >= {"workload", "global_batch", "seq_len"}
 
 
 @pytest.mark.parametrize("workload", ["tiny", "srds"])
@@ -88,3 +127,5 @@ def test_reference_arm_json_line(workload):
     assert line["impl"] == "reference" and line["value"] > 0
     assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] == 1
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+    assert line["config"]["workload"] == W.ALL[workload].name
+    assert line["config"]["solver_steps_per_step"] >= 1

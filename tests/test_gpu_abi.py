@@ -112,13 +112,13 @@ def test_nonblocking_stream():
     assert np.array_equal(a, s2.result().cpu().numpy())
 
 
-@pytest.mark.parametrize("kind", [110, 101])
+@pytest.mark.parametrize("kind", [110, 101, 3])
 def test_bounded_wait_reports_timeout_and_context_survives(kind):
     """Force every mbarrier wait of a bulk-copy update kernel (the staged
-    segment form, the tiled pipeline) to give up at once: the kernel records a
-    timeout (no hang, no fault), drains its copies, and the next synchronising
-    call reports PA_ERR_TIMEOUT. After pa_init the same solver reproduces a
-    clean run bit for bit."""
+    segment form, the tiled pipeline), or the fused step's grid barrier, to
+    give up at once: the kernel records a timeout (no hang, no fault), drains
+    its copies, and the next synchronising call reports PA_ERR_TIMEOUT. After
+    pa_init the same solver reproduces a clean run bit for bit."""
     w = W.SD15.with_(T=30, window=30)
     s, g, eps, x0 = _solver(w)
     s.set_update_kernel(kind)
@@ -138,17 +138,18 @@ def test_bounded_wait_reports_timeout_and_context_survives(kind):
     _run(s, g, eps)
     assert np.array_equal(clean, s.result().cpu().numpy())
     assert s.stats()["device_status"] == 0
+    assert s.stats()["update_kernel"] == (3 if kind == 3 else 1)
 
 
 def test_update_kernel_selector_rejects_unknown_shapes():
-    """pa_set_update_kernel takes 0, 1, 2, 100 + bulk shape and 200 + lean
-    shape (0-6, 10-16); anything else is PA_ERR_ARG and leaves the choice as
-    it was."""
+    """pa_set_update_kernel takes 0, 1, 2, 3, 100 + bulk shape, 200 + lean
+    shape (0-6, 10-16) and 300 + fused shape (0-6); anything else is
+    PA_ERR_ARG and leaves the choice as it was."""
     w = W.TINY
     s, g, eps, x0 = _solver(w)
-    for kind in (2, 0, 1, 100, 112, 200, 206, 210, 216):
+    for kind in (3, 300, 306, 2, 0, 1, 100, 112, 200, 206, 210, 216):
         abi.pa_set_update_kernel(s.h, kind)
-    for kind in (-1, 3, 99, 113, 199, 207, 209, 217, 300):
+    for kind in (-1, 4, 99, 113, 199, 207, 209, 217, 299, 307, 310):
         with pytest.raises(abi.PaError) as e:
             abi.pa_set_update_kernel(s.h, kind)
         assert e.value.status == abi.PA_ERR_ARG

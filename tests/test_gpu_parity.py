@@ -52,7 +52,7 @@ def test_tiny_with_oracle_eps():
 def test_sd15_full_size():
     orc, gpu = _check(W.SD15)
     assert gpu["stats"]["hits"] > 0
-    assert gpu["stats"]["update_kernel"] == 2  # the lean register form is the default
+    assert gpu["stats"]["update_kernel"] == 3  # the fused step is the default where it fits
 
 
 def test_sd15_uncached_equals_oracle_uncached():
@@ -389,6 +389,65 @@ def test_lean_update_long_schedule(kind, eta):
     got = gpu_run(w, update_kernel=kind)
     assert got["stats"]["update_kernel"] == 2
     assert compare(w, orc, got).max() <= REL_TOL
+
+
+# ---- fused solver step: update, grid barrier, decision, batch from registers --
+
+FUSED_CASES = [
+    W.SD15,
+    W.TINY,
+    W.SD15.with_(window=64, name="SD window 64"),
+    W.SD15.with_(T=150, window=112, latent_shape=(4, 32, 32), name="window 112"),
+    W.Workload("ragged strips B3", T=40, window=24, batch=3, latent_shape=(4, 20, 20), K=6,
+               tol=1e-3, cache_thresh=0.05, seed=12),
+    # every error below tol: the window slides by p and the next window is all
+    # lazy tail states, which the warp holding the frontier state writes
+    W.Workload("huge tol", T=40, window=16, batch=2, latent_shape=(4, 8, 8), K=4,
+               tol=1e3, cache_thresh=0.05, seed=2),
+    W.Workload("cache 0.1", T=60, window=60, batch=1, latent_shape=(4, 32, 32), K=8,
+               tol=1e-3, cache_thresh=0.1, seed=4),
+]
+
+
+@pytest.mark.parametrize("w", FUSED_CASES, ids=lambda w: w.name)
+def test_fused_step_equals_update_and_planning(w):
+    """The fused step (one kernel per iteration) against the update kernel +
+    planning kernel pair of the same launch shape: the same arithmetic, so the
+    iteration log, the final states and every iteration's reductions are
+    bitwise equal -- the Eq. 2 / Eq. 4 sums are exact whatever order the CTAs
+    add their partials in --, and both take the oracle's decisions."""
+    orc = oracle_run(w)
+    assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-6), decision_margins(orc, w.tol, w.cache_thresh)
+    fused = gpu_run(w, reductions=True)
+    split = gpu_run(w, update_kernel=2, reductions=True)
+    assert fused["stats"]["update_kernel"] == 3 and split["stats"]["update_kernel"] == 2
+    assert compare(w, orc, fused).max() <= REL_TOL
+    assert np.array_equal(fused["log"], split["log"])
+    assert np.array_equal(fused["x_final"], split["x_final"])
+    assert len(fused["reductions"]) == len(split["reductions"]) > 0
+    for (ef, df), (es, dss) in zip(fused["reductions"], split["reductions"]):
+        assert np.array_equal(ef, es) and np.array_equal(df, dss)
+
+
+def test_fused_step_falls_back_beyond_one_wave():
+    """The batched workload's grid (128 strips x 8 trajectories) is not
+    resident in one wave: the update and planning kernels run instead."""
+    orc, gpu = _check(W.BATCHED.with_(T=40))
+    assert gpu["stats"]["update_kernel"] == 2
+
+
+@pytest.mark.parametrize("window", [24, 64])
+def test_fused_step_stochastic(window):
+    """Stochastic steps through the fused step (8 x 4 and 16 x 7 shapes)
+    against the oracle and against the register-resident bulk form."""
+    w = W.Workload("fused eta", T=100, window=window, batch=1, latent_shape=(4, 32, 32), K=6,
+                   tol=1e-3, cache_thresh=0.05, seed=5, eta=1.0)
+    orc = oracle_run(w)
+    fused = gpu_run(w)
+    assert fused["stats"]["update_kernel"] == 3
+    assert compare(w, orc, fused).max() <= REL_TOL
+    bulk = gpu_run(w, update_kernel=112)
+    assert np.array_equal(fused["log"], bulk["log"])
 
 
 # ---- stochastic steps (eta > 0): DDPM over the full 1000-step schedule -------
