@@ -153,11 +153,11 @@ PA_API const int32_t* pa_n_miss_dev(const pa_solver* s);
  * the drift and the Picard prefix sum (Eq. 1), the errors of Eq. 2 and the
  * cache distances of the next iteration (Eq. 4), then the window advance
  * (Sec. 2.1), the hit-miss plan of the next iteration (Eq. 5) and the gather
- * of its batch (Sec. 2.2, one batched pass): by default in one fused kernel
- * when all of its CTAs (one per 128 columns of each trajectory) fit on the
- * GPU at once -- a cooperative launch with a bounded grid barrier --, else
- * in an update kernel followed by a planning kernel. Asynchronous on the
- * solver's stream; batch_eps_dev must stay valid until the update has run. */
+ * of its batch (Sec. 2.2, one batched pass): by default in an update kernel
+ * followed by a planning kernel, or (pa_set_update_kernel 3) in one fused
+ * kernel when all of its CTAs fit on the GPU at once -- a cooperative launch
+ * with a bounded grid barrier. Asynchronous on the solver's stream;
+ * batch_eps_dev must stay valid until the update has run. */
 PA_API pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev);
 
 /* Synchronise and report: *n_active = trajectories not yet at t = T.
@@ -199,17 +199,18 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
 /* Select the Picard-update kernel (all forms compute Eq. 1, 2, 4, 6 and 7 of
  * one iteration; they differ in rounding order only, never in a decision
  * beyond the decision-margin guard):
- *   3       the fused step (default when D % 4 == 0): the lean register form's
- *           update, a grid barrier, the decision in every CTA and the next
- *           batch written from registers, one kernel per iteration; used when
- *           every CTA of its grid (ceil(D / 128) x batch) is resident at once
- *           and batch * window <= 1024, else form 2 runs;
+ *   3       the fused step: the lean register form's update, a grid barrier,
+ *           the decision in every CTA and the next batch written from
+ *           registers, one kernel per iteration; used when every CTA of its
+ *           grid (ceil(D / 128) x batch) is resident at once and
+ *           batch * window <= 1024, else form 2 runs;
  *   300 + n the fused step with lean launch shape n (0, 1, 4, 5 below; with
  *           stochastic steps 0, 1, 3, 4);
  *   0       plain loads (one thread per column; any D);
  *   1       the bulk forms: register-resident rows, or rows staged in shared
  *           memory by bulk copies for windows the registers cannot hold;
- *   2       the lean register form (default when D % 4 == 0): 16-byte rows
+ *   2       the lean register form followed by the planning kernel (default
+ *           when D % 4 == 0): 16-byte rows
  *           straight into registers, plain fp32 prefix sums, coefficients and
  *           ranks staged in shared memory; windows up to 112 points with
  *           deterministic steps, else it falls back to 1;
@@ -377,7 +378,11 @@ PA_API pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32_t* 
                      const int32_t* n_rows_dev, float* batch_eps_dev);
 
 /* Synchronise the handle's stream and report a device-side failure of the
- * denoiser kernels (a bounded bulk-copy wait that ran out): PA_ERR_TIMEOUT. */
+ * denoiser kernels (a bounded bulk-copy wait that ran out): PA_ERR_TIMEOUT.
+ * The failure also shows in the output: the output kernel writes NaN into
+ * every tile of a call whose waits ran out, and, the handle's accumulators
+ * being incomplete from then on, into every later call's output; create a
+ * new handle after a timeout. */
 PA_API pa_status pa_gmm_check(pa_gmm* g);
 
 /* Kernels launched by this handle since pa_gmm_create. */
@@ -420,15 +425,20 @@ PA_API void pa_gmm_destroy(pa_gmm* g);
  * accumulators) would exceed 4 MiB are rejected with PA_ERR_ARG and a message
  * naming the bytes needed; use pa_gmm_create/pa_gmm_eps then.
  *
- * The first call on a device looks up the array's device address
- * (cudaGetSymbolAddress) with that device current; make that first call
- * before any stream capture. Every call on a device shares the one array and
- * overwrites it (the status word is cleared at the start of each call), so
- * calls whose work overlaps on the GPU -- on different streams, or from
- * different host threads without ordering -- race and give wrong results.
- * The call is asynchronous on `stream`; it calls no cudaMalloc, cudaFree or
- * other allocating routine. A bounded-wait timeout inside its kernels is
- * recorded in the array's status word only (not reported). */
+ * Every call looks up the array's device address (cudaGetSymbolAddress) with
+ * the caller's device current; the first call on a device also makes the
+ * library's device code resident there, so make that first call before any
+ * stream capture. Every call on a device shares the one array and overwrites
+ * it (the status word, the accumulators and the row count are set afresh at
+ * the start of each call), so calls whose work overlaps on the GPU -- on
+ * different streams, or from different host threads without ordering -- race
+ * and give wrong results. The call is asynchronous on `stream`: the
+ * per-timestep scalars are formed on the device from alphas that travel in
+ * the parameters of small set-up launches (one per 3000 timesteps), so
+ * nothing on the host has to outlive the call and no host-to-device copy
+ * blocks it. It calls no cudaMalloc, cudaFree or other allocating routine. A
+ * bounded-wait timeout inside its kernels is recorded in the array's status
+ * word, and the output rows of the tiles it affected are written as NaN. */
 PA_API pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D, double std,
                                     const double* alphas_cumprod, int T,
                                     const float* batch_x_dev, const int32_t* miss_bt_dev,

@@ -32,7 +32,6 @@
 #include <cmath>
 #include <cstdlib>
 #include <cstring>
-#include <mutex>
 #include <string>
 #include <vector>
 
@@ -355,8 +354,11 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   }
   pdl_wait();  // the dot products come from the kernel just before
   pdl_trigger();  // the successor may now run its prologue
-  // both accumulator sets are read together with the set index (one round trip)
+  // both accumulator sets are read together with the set index and the
+  // status word (one round trip): a dot-product kernel that timed out left
+  // the sums incomplete
   const uint32_t cur = ep->cur;
+  const int dots_status = __ldcg(status);
   const int64_t set_size = (int64_t)max_rows * K;
   __syncthreads();
   for (int q = tid; q < kOutRows * K; q += kThreads) {
@@ -396,8 +398,13 @@ __global__ void __launch_bounds__(kThreads) k_gmm_out(const float* __restrict__ 
   }
   if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) ep->epoch = cur + 1u;  // the next call's set
   const bool ok = wait_staged(bulk, &bar, status);
-  __syncthreads();
-  if (!ok) return;
+  if (__syncthreads_or(!ok || dots_status != 0)) {
+    // a bounded wait ran out here or in the dot products: the tile is written
+    // as NaN, so the failure shows in the output as well as in the status word
+    for (int q = tid; q < nr * ncol; q += kThreads)
+      eps[(int64_t)(r0 + q / ncol) * D + c0 + q % ncol] = __int_as_float(0x7fc00000);
+    return;
+  }
   // kOutCols / 4 column groups of 4 x kThreads / (kOutCols / 4) row groups of 4
   static_assert(kThreads / (kOutCols / 4) * 4 == kOutRows, "the threads cover the tile's rows");
   const int cg = tid % (kOutCols / 4), rg = tid / (kOutCols / 4);
@@ -834,41 +841,47 @@ extern "C" void pa_gmm_destroy(pa_gmm* g) { delete g; }
 constexpr size_t kNoAllocScratchBytes = (size_t)4 << 20;  // 4 MiB, held by every device that loads this library
 
 // The fixed scratch. In host code `g_gmm_scratch` is only a stand-in name:
-// its device address comes from cudaGetSymbolAddress, looked up per device.
+// its device address comes from cudaGetSymbolAddress, looked up on each call
+// with the caller's device current.
 static __device__ __align__(256) unsigned char g_gmm_scratch[kNoAllocScratchBytes];
 
 namespace {
 
-constexpr int kNoAllocMaxDevices = 64;
-constexpr int kNoAllocCoefChunk = 512;                    // host coefficients staged in chunks on the stack
+// Per-timestep scalars of the allocation-free path, formed on the device in
+// fp64 from alpha-bar values that travel in the launch's own parameters (no
+// host buffer, no host-to-device copy); the launch with i0 = 0 also stores the
+// row count. Same expressions as pa_gmm_create's host loop, with no fused
+// multiply-add, so the values round to fp32 alike.
+constexpr int kNoAllocCoefChunk = 3000;  // alphas per launch: 24 KB of kernel parameters
+struct AlphaChunk {
+  int i0, n;
+  double std;
+  double a[kNoAllocCoefChunk];
+};
 
-std::mutex g_scratch_mu;
-unsigned char* g_scratch_dev[kNoAllocMaxDevices] = {};
+__global__ void __launch_bounds__(256) k_noalloc_coef(AlphaChunk c, int T, int n_rows, float* __restrict__ coef,
+                                                      int32_t* __restrict__ nrows_dev) {
+  for (int u = threadIdx.x; u < c.n; u += blockDim.x) {
+    const double a = c.a[u];
+    const double v = __dadd_rn(__dmul_rn(__dmul_rn(a, c.std), c.std), 1.0 - a);
+    coef[c.i0 + u] = (float)sqrt(a);
+    coef[T + c.i0 + u] = (float)(1.0 / (2.0 * v));
+    coef[2 * T + c.i0 + u] = (float)(sqrt(1.0 - a) / v);
+  }
+  if (c.i0 == 0 && threadIdx.x == 0) *nrows_dev = n_rows;
+}
 
-// Device address of g_gmm_scratch for the current device, looked up once per
-// device (the host-side name is only a stand-in for the device array).
+// Device address of g_gmm_scratch for the current device, looked up on every
+// call (cheap, not a stream operation; a cached address could go stale if the
+// device's context were torn down and the module reloaded elsewhere).
 pa_status scratch_for_current_device(unsigned char** out) {
-  int dev = -1;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) {
-    pa::set_error(std::string("pa_gmm_eps_noalloc: cudaGetDevice: ") + cudaGetErrorString(e));
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_gmm_scratch);
+  if (e != cudaSuccess || !p) {
+    pa::set_error(std::string("pa_gmm_eps_noalloc: cudaGetSymbolAddress: ") + cudaGetErrorString(e));
     return PA_ERR_CUDA;
   }
-  if (dev < 0 || dev >= kNoAllocMaxDevices) {
-    pa::set_error("pa_gmm_eps_noalloc: device index beyond the supported 64");
-    return PA_ERR_ARG;
-  }
-  std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_dev[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_gmm_scratch);
-    if (e != cudaSuccess || !p) {
-      pa::set_error(std::string("pa_gmm_eps_noalloc: cudaGetSymbolAddress: ") + cudaGetErrorString(e));
-      return PA_ERR_CUDA;
-    }
-    g_scratch_dev[dev] = static_cast<unsigned char*>(p);
-  }
-  *out = g_scratch_dev[dev];
+  *out = static_cast<unsigned char*>(p);
   return PA_OK;
 }
 
@@ -920,24 +933,20 @@ extern "C" pa_status pa_gmm_eps_noalloc(const float* means_dev, int K, int64_t D
   int32_t* nrows_dev = reinterpret_cast<int32_t*>(scratch + o_n);
   int32_t* status = reinterpret_cast<int32_t*>(scratch + o_status);
 
-  // Per-timestep scalars, formed in fp64 on the host in stack-sized chunks;
-  // each pageable copy returns once its source has been staged.
+  // Per-timestep scalars and the row count: small launches whose parameters
+  // carry the alphas (asynchronous, nothing on the host to outlive the call).
   cudaError_t e = cudaSuccess;
-  float buf[kNoAllocCoefChunk];
-  for (int part = 0; part < 3 && e == cudaSuccess; ++part) {
+  {
+    AlphaChunk c;
+    c.std = std;
     for (int i0 = 0; i0 < T && e == cudaSuccess; i0 += kNoAllocCoefChunk) {
-      const int n = (T - i0) < kNoAllocCoefChunk ? (T - i0) : kNoAllocCoefChunk;
-      for (int u = 0; u < n; ++u) {
-        const double a = alphas_cumprod[i0 + u];
-        const double v = a * std * std + (1.0 - a);
-        buf[u] = (float)(part == 0 ? std::sqrt(a) : part == 1 ? 1.0 / (2.0 * v) : std::sqrt(1.0 - a) / v);
-      }
-      e = cudaMemcpyAsync(coef + (size_t)part * T + i0, buf, (size_t)n * sizeof(float),
-                          cudaMemcpyHostToDevice, st);
+      c.i0 = i0;
+      c.n = (T - i0) < kNoAllocCoefChunk ? (T - i0) : kNoAllocCoefChunk;
+      for (int u = 0; u < c.n; ++u) c.a[u] = alphas_cumprod[i0 + u];
+      k_noalloc_coef<<<1, 256, 0, st>>>(c, T, n_rows, coef, nrows_dev);
+      e = cudaGetLastError();
     }
   }
-  const int32_t nr = n_rows;
-  if (e == cudaSuccess) e = cudaMemcpyAsync(nrows_dev, &nr, sizeof(nr), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(status, 0, sizeof(int32_t), st);  // starts at zero every call
   if (e == cudaSuccess)  // the epoch and both accumulator sets start at zero every call too
     e = cudaMemsetAsync(ep, 0, sizeof(GmmEpoch), st);

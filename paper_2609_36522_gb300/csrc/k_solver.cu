@@ -292,49 +292,27 @@ constexpr int kPlanThreads = 256;
 constexpr int kFusedMaxPairs = 1024;  // B*P planned in every CTA; beyond, one CTA plans
 static_assert(kFusedMaxPairs <= 32 * 32, "decide_par keeps one miss mask per 32-position chunk, 32 of them");
 
-struct RedShared {
-  const double* e;
-  const double* dl;
-  __device__ double err(int q) const { return e[q]; }
-  __device__ double del(int q) const { return dl[q]; }
-};
-
+// The complete sums read from global memory (one-CTA planner).
 struct RedSums {
   const double* e;
   const double* dl;
-  double inv_d;
+  double inv_d, tol_d, thr_d;
   __device__ double err(int q) const { return __ldcg(e + (size_t)q * kAccStride) * inv_d; }
   __device__ double del(int q) const { return __ldcg(dl + (size_t)q * kAccStride) * inv_d; }
+  __device__ bool conv(int q) const { return sum_le(__ldcg(e + (size_t)q * kAccStride), tol_d); }
+  __device__ bool near(int q) const { return sum_lt(__ldcg(dl + (size_t)q * kAccStride), thr_d); }
 };
 
 template <int VEC>
 __global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
   __shared__ DecideShared ds;
-  __shared__ double s_e[kFusedMaxPairs], s_d[kFusedMaxPairs];
-  const int tid = threadIdx.x;
   const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
-  const int npair = d.B * d.P;
   decide_load<kPlanThreads>(d, ds, par);
   pdl_wait();  // the sums and the new states come from the update kernel
   pdl_trigger();  // the successor may now run its prologue
-  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
-  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
-  const double inv_d = 1.0 / (double)d.D;
-  for (int q = tid; q < npair; q += kPlanThreads) {
-    const size_t o = (size_t)q * kAccStride;
-    const double ve = __ldcg(acc_e + o) * inv_d, vd = __ldcg(acc_d + o) * inv_d;
-    s_e[q] = ve;
-    s_d[q] = vd;
-    if (publish) {
-      d.red_err[q] = (float)ve;
-      d.red_del[q] = (float)vd;
-      double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;  // iteration k+1 adds into these
-      nxt[o] = 0.0;
-      nxt[(size_t)npair * kAccStride + o] = 0.0;
-    }
-  }
-  __syncthreads();  // the sums and decide_load's state are staged
-  decide_par(d, ds, RedShared{s_e, s_d}, par, publish, (int)blockIdx.y);
+  stage_decision_bits(d, ds, par, publish ? 0 : -1, 1);
+  __syncthreads();  // the decision's input bits and decide_load's state are staged
+  decide_par(d, ds, par, publish ? 0 : -1, 1, (int)blockIdx.y);
   __syncthreads();  // the plan (batch row of this CTA) is known
   if ((int)blockIdx.y < ds.total && ds.target_b >= 0) {
     const int b = ds.target_b;
@@ -354,7 +332,7 @@ __global__ void __launch_bounds__(kPlanOneThreads) k_plan_one(Dev d, int par) {
   pdl_trigger();  // the successor may now run its prologue
   const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
   const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
-  const RedSums red{acc_e, acc_d, 1.0 / (double)d.D};
+  const RedSums red{acc_e, acc_d, d.inv_d, d.tol_d, d.thr_d};
   decide_run<kPlanOneThreads>(d, ds, red, par, true, -1);
   double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;
   for (int q = threadIdx.x; q < npair; q += kPlanOneThreads) {

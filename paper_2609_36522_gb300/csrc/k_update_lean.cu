@@ -128,31 +128,20 @@ struct LeanShape {
   __host__ __device__ static size_t rank_bytes(int P) { return ((size_t)P * 4 + 127) / 128 * 128; }
   __host__ __device__ static size_t red_bytes(int P) { return ((size_t)2 * P * 33 * sizeof(float) + 127) / 128 * 128; }
   static constexpr size_t kTotBytes = (size_t)NW * 32 * 16;  // run totals, one float4 per lane and warp
-  // the fused step's complete sums, err and distance of every (b, j), fp64
-  __host__ __device__ static size_t sum_bytes(int B, int P) { return (size_t)2 * B * P * sizeof(double); }
-  __host__ __device__ static size_t smem_bytes(int T, int P, bool comp, int B = 0) {
-    return sum_bytes(B, P) + coef_bytes(T) + rank_bytes(P) + red_bytes(P) + kTotBytes * (comp ? 2 : 1);
+  __host__ __device__ static size_t smem_bytes(int T, int P, bool comp) {
+    return coef_bytes(T) + rank_bytes(P) + red_bytes(P) + kTotBytes * (comp ? 2 : 1);
   }
 };
-
-// The complete sums as the decision reads them (shared memory, divided by D).
-struct LeanRed {
-  const double* e;
-  const double* dl;
-  __device__ double err(int q) const { return e[q]; }
-  __device__ double del(int q) const { return dl[q]; }
-};
-
 
 // The fused step after the update: grid barrier, the complete sums, the
 // decision in every CTA, and the warp's share of the next batch from the new
 // states in `xn` (states t + j0 + 1 .. t + j0 + nj of trajectory tr; NULL for a
 // finished trajectory). Every thread of every CTA calls it.
 template <int NW, int LMAX>
-__device__ __forceinline__ void step_tail(const Dev& d, DecideShared& ds, double* s_sum, int par, const Traj& tr,
-                                          const Q* xn, int j0, int nj, int mycol, int D, bool live) {
+__device__ __forceinline__ void step_tail(const Dev& d, DecideShared& ds, int par, const Traj& tr, const Q* xn,
+                                          int j0, int nj, int mycol, int D, bool live) {
   const int tid = threadIdx.x;
-  const int B = d.B, P = d.P, npair = B * P;
+  const int P = d.P;
   const unsigned long long ncta = (unsigned long long)gridDim.x * gridDim.y;
   // the spin polls an L2 line (about half a microsecond each): 16 x the
   // mbarrier limit keeps the same order of time, about a second
@@ -161,27 +150,12 @@ __device__ __forceinline__ void step_tail(const Dev& d, DecideShared& ds, double
     if (tid == 0) atomicCAS(&d.ctl->status, kDevOk, kDevTimeout);
     return;  // the plan is not published; the host reports PA_ERR_TIMEOUT
   }
-  const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
-  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
-  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
-  const double inv_d = 1.0 / (double)d.D;
-  double* s_e = s_sum;
-  double* s_d = s_sum + npair;
-  for (int q = tid; q < npair; q += NW * 32) {
-    const size_t o = (size_t)q * kAccStride;
-    const double ve = __ldcg(acc_e + o) * inv_d, vd = __ldcg(acc_d + o) * inv_d;
-    s_e[q] = ve;
-    s_d[q] = vd;
-    if (publish) {
-      d.red_err[q] = (float)ve;
-      d.red_del[q] = (float)vd;
-      double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;  // iteration k+1 adds into these
-      nxt[o] = 0.0;
-      nxt[(size_t)npair * kAccStride + o] = 0.0;
-    }
-  }
+  // every CTA publishes a share: CTA c writes the reductions and ranks of the
+  // positions and chunks congruent to c, CTA 0 the trajectories and counters
+  const int cta = blockIdx.y * gridDim.x + blockIdx.x;
+  stage_decision_bits(d, ds, par, cta, (int)ncta);
   __syncthreads();
-  decide_par(d, ds, LeanRed{s_e, s_d}, par, publish, -1);
+  decide_par(d, ds, par, cta, (int)ncta, -1);
   __syncthreads();  // the next plan (ds.tn, ds.pn, chunk masks and bases) is known
   if (xn == nullptr || !live || nj <= 0) return;
   // a4 of the next iteration: its timestep i (tn <= i < tn + pn) reads state
@@ -223,13 +197,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int T = d.T, P = d.P, b = blockIdx.y;
   const int D = (int)d.D;  // (P + 1) * D and T * D fit in int32 (launcher)
-  const size_t o_sum = FUSE ? Sh::sum_bytes(d.B, P) : 0;
-  double* s_sum = reinterpret_cast<double*>(smem_raw);  // FUSE: [2][B][P]
-  CT* s_coef = reinterpret_cast<CT*>(smem_raw + o_sum);
-  int32_t* s_rank = reinterpret_cast<int32_t*>(smem_raw + o_sum + Sh::coef_bytes(T));
-  float* s_red = reinterpret_cast<float*>(smem_raw + o_sum + Sh::coef_bytes(T) + Sh::rank_bytes(P));  // [2][P][33]
-  float4* s_tot =
-      reinterpret_cast<float4*>(smem_raw + o_sum + Sh::coef_bytes(T) + Sh::rank_bytes(P) + Sh::red_bytes(P));
+  CT* s_coef = reinterpret_cast<CT*>(smem_raw);
+  int32_t* s_rank = reinterpret_cast<int32_t*>(smem_raw + Sh::coef_bytes(T));
+  float* s_red = reinterpret_cast<float*>(smem_raw + Sh::coef_bytes(T) + Sh::rank_bytes(P));  // [2][P][33]
+  float4* s_tot = reinterpret_cast<float4*>(smem_raw + Sh::coef_bytes(T) + Sh::rank_bytes(P) + Sh::red_bytes(P));
   float4* s_lo = s_tot + NW * 32;  // COMP only
   __shared__ DecideShared ds;      // FUSE only (the compiler drops it otherwise)
 
@@ -262,7 +233,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
       return;
     } else {  // the fused step still meets the barrier and takes the decision
       pdl_trigger();
-      step_tail<NW, LMAX>(d, ds, s_sum, par, tr, nullptr, 0, 0, 0, 0, false);
+      step_tail<NW, LMAX>(d, ds, par, tr, nullptr, 0, 0, 0, 0, false);
       return;
     }
   }
@@ -305,10 +276,20 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
 
   Q x[LMAX + 1], ep[LMAX], xh[LMAX], z[NOISE ? LMAX : 1];
   if (live && nj > 0) {
+    // states past the frontier e are lazy copies of state e: one load of
+    // row e serves all of this warp's lazy positions
+    const int nreal = e - (t + j0);  // positions g <= nreal hold materialised states
+    Q xe = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+    if (nreal < 0) xe = ldq(Xr + se * D);
 #pragma unroll
     for (int g = 0; g <= LMAX; ++g) {
       if (g > nj) break;
-      x[g] = ldq(Xr + xslot(g) * D);
+      if (g <= nreal) {
+        x[g] = ldq(Xr + xslot(g) * D);
+        xe = x[g];
+      } else {
+        x[g] = xe;
+      }
     }
 #pragma unroll
     for (int g = 0; g < LMAX; ++g) {
@@ -445,7 +426,7 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
     }
     red_add(d, par, which, b * P + j, (a0 + a1) + (a2 + a3));
   }
-  if constexpr (FUSE) step_tail<NW, LMAX>(d, ds, s_sum, par, tr, ep, j0, nj, mycol, D, live);
+  if constexpr (FUSE) step_tail<NW, LMAX>(d, ds, par, tr, ep, j0, nj, mycol, D, live);
 }
 
 template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
@@ -476,7 +457,7 @@ template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
 cudaError_t launch_fused(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = LeanShape<NW, NOISE>;
   const int nstrip = (int)((d.D + 127) / 128);
-  const size_t smem = Sh::smem_bytes(d.T, d.P, COMP, d.B);
+  const size_t smem = Sh::smem_bytes(d.T, d.P, COMP);
   if (smem > kLeanSmemMax) return cudaErrorNotSupported;
   auto kern = k_update_lean<NW, LMAX, MINB, NOISE, COMP, CB, true>;
   // per device: the dynamic shared memory configured and the resident CTAs

@@ -14,8 +14,10 @@ struct DecideShared {
   int t[kMaxBatch], p[kMaxBatch], e[kMaxBatch];
   int tn[kMaxBatch], pn[kMaxBatch], en[kMaxBatch], m[kMaxBatch], h1[kMaxBatch];
   int om[kMaxBatch], oh1[kMaxBatch];
+  int stride[kMaxBatch], nh[kMaxBatch];  // decide_par: window advance and next-window positions with an entry
   int warp_tot[32];
   unsigned cmiss[32], cwin[32];  // decide_par: miss / in-window bits of each 32-position chunk
+  unsigned conv[32], near[32];   // decide_par's inputs as bits: Eq. 2 error <= tol, Eq. 4 distance < tau_cache
   int cbase[32];                 // decide_par: misses before each chunk
   int pts;                       // decide_par: window positions planned
   int total, active, iter;
@@ -104,7 +106,7 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const Red& red, int p
     int lead = p;
     for (int j0 = 0; j0 < p; j0 += 32) {
       const int j = j0 + lane;
-      const bool fail = (j < p) && !(red.err(b * P + j) <= d.tol);
+      const bool fail = (j < p) && !red.conv(b * P + j);
       const unsigned m = __ballot_sync(0xffffffffu, fail);
       if (m) {
         lead = j0 + __ffs(m) - 1;
@@ -136,7 +138,7 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const Red& red, int p
     const int en = s_t[b] + s_p[b];  // new frontier
     if (i >= en) return 1;           // first entry
     const int jo = i - s_t[b] - 1;   // delta of timestep i was computed at old position jo
-    return (red.del(b * P + jo) < d.cache_thresh) ? 0 : 1;
+    return red.near(b * P + jo) ? 0 : 1;
   };
   int cnt = 0;
   for (int q = q0; q < q1; ++q) cnt += is_miss(q);
@@ -224,22 +226,57 @@ __device__ void decide_run(const Dev& d, DecideShared& sh, const Red& red, int p
   }
 }
 
-// The same decision with all warps of the CTA at work, for the planning
-// kernel in which every CTA decides (B*P <= 32 * 32): warp w advances the
-// windows of trajectories w, w + NW, ...; warp w tests the 32-position chunks
-// w, w + NW, ... of the next windows; one warp turns the chunks' miss counts
-// into each chunk's first rank; the chunks then place their misses. Gives the
-// same plan, ranks and counters as decide_run. Every thread of
-// the CTA calls it (it holds CTA barriers); the caller synchronises the CTA
-// afterwards.
-template <typename Red>
-__device__ void decide_par(const Dev& d, DecideShared& sh, const Red& red, int par, bool publish, int target) {
+// Set bits of the bit string w (bit q of the string = bit q & 31 of word
+// q >> 5) in positions [lo, hi).
+__device__ __forceinline__ int range_popc(const unsigned* w, int lo, int hi) {
+  int n = 0;
+  while (lo < hi) {
+    const int c = lo >> 5, o = lo & 31;
+    const int take = min(32 - o, hi - lo);
+    const unsigned m = (take == 32 ? 0xffffffffu : ((1u << take) - 1u)) << o;
+    n += __popc(w[c] & m);
+    lo += take;
+  }
+  return n;
+}
+
+// Bits [pos, pos + 32) of a bit string of 32 words (bits past the last word read as 0).
+__device__ __forceinline__ unsigned bits32(const unsigned* w, int pos) {
+  const int c = pos >> 5, o = pos & 31;
+  unsigned v = c < 32 ? w[c] >> o : 0u;
+  if (o && c + 1 < 32) v |= w[c + 1] << (32 - o);
+  return v;
+}
+
+// The decision that ends an iteration, for kernels in which every CTA decides
+// (B*P <= 32 * 32), from the bit strings that stage_decision_bits left in
+// sh.conv (bit b*P + j: the Eq. 2 error of window position j of trajectory b
+// is <= tol) and sh.near (bit b*P + j: the Eq. 4 distance of timestep
+// t_b + j + 1 is < tau_cache). Warp 0 alone takes it with bit operations:
+//  1. lane b advances trajectory b: stride = min(p, 1 + leading ones of its
+//     conv bits), t' = t + stride, p' = min(P, T - t'), frontier e' = t + p;
+//  2. lane c builds 32-position word c of the next windows' bits: position
+//     j' of trajectory b (timestep i = t' + j') is in the window for j' < p';
+//     it has an entry iff i < t + p, i.e. j' < p - stride, and then hits iff
+//     near bit j' + stride - 1 (where its distance was computed) is set
+//     (Eq. 5, strict); all other window positions miss;
+//  3. lane c turns the miss counts of 32-position chunk c into its first rank
+//     (an exclusive scan): misses are ranked trajectory-major, ascending t.
+// Then, after one CTA barrier, every warp handles chunks: the ranks and the
+// miss list are written by publishing CTAs (chunk c by the CTA whose pub_id is
+// c mod pub_count; pub_id < 0 writes nothing) and every CTA notes the miss of
+// batch row `target` (target_b, target_i); the CTA with pub_id 0 also writes
+// the trajectories, counters and iteration log. Gives the same plan, ranks and
+// counters as decide_run. Every thread of the CTA calls it; the caller
+// synchronises the CTA afterwards.
+__device__ inline void decide_par(const Dev& d, DecideShared& sh, int par, int pub_id, int pub_count, int target) {
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
   const int B = d.B, P = d.P, T = d.T;
+  const int N = B * P, nchunk = (N + 31) / 32;
   Traj* out_traj = d.traj + (par ^ 1) * B;
   if (sh.active == 0) {  // finished: the plan carries over (uniform across the CTA)
     if (warp == 0) {
-      if (publish) {
+      if (pub_id == 0) {
         const Traj* in_traj = d.traj + par * B;
         for (int b = lane; b < B; b += 32) out_traj[b] = in_traj[b];
         if (lane == 0) d.pc[par ^ 1] = d.pc[par];
@@ -249,28 +286,27 @@ __device__ void decide_par(const Dev& d, DecideShared& sh, const Red& red, int p
     return;
   }
   const int iter = sh.iter;
-  // 1. window advance, one warp per trajectory
-  for (int b = warp; b < B; b += nw) {
-    const int t = sh.t[b], p = sh.p[b];
-    int stride = 0;
-    if (p > 0) {
-      int lead = p;
-      for (int j0 = 0; j0 < p; j0 += 32) {
-        const int j = j0 + lane;
-        const unsigned m = __ballot_sync(0xffffffffu, (j < p) && !(red.err(b * P + j) <= d.tol));
-        if (m) {
-          lead = j0 + __ffs(m) - 1;
-          break;
+  if (warp == 0) {
+    for (int b = lane; b < B; b += 32) {
+      const int t = sh.t[b], p = sh.p[b];
+      int stride = 0;
+      if (p > 0) {
+        int lead = 0;
+        while (lead < p) {
+          const unsigned w = bits32(sh.conv, b * P + lead);
+          const int ones = w == 0xffffffffu ? 32 : __ffs(~w) - 1;
+          lead += ones;
+          if (ones < 32) break;
         }
+        stride = min(p, 1 + min(lead, p));
       }
-      stride = min(p, 1 + lead);
-    }
-    if (lane == 0) {
-      const int tn = t + stride;
+      const int tn = t + stride, pn = p > 0 ? min(P, T - tn) : 0;
       sh.tn[b] = tn;
-      sh.pn[b] = p > 0 ? min(P, T - tn) : 0;
+      sh.pn[b] = pn;
       sh.en[b] = p > 0 ? t + p : sh.e[b];
-      if (publish) {
+      sh.stride[b] = stride;
+      sh.nh[b] = p > 0 ? p - stride : 0;  // next-window positions with a cache entry
+      if (pub_id == 0) {
         int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
         if (p > 0) {
           lg[0] = t; lg[1] = p; lg[2] = sh.om[b]; lg[3] = stride;
@@ -281,36 +317,29 @@ __device__ void decide_par(const Dev& d, DecideShared& sh, const Red& red, int p
         }
       }
     }
-  }
-  __syncthreads();
-  // 2. hit/miss tests of the next windows, one warp per 32-position chunk
-  const int N = B * P, nchunk = (N + 31) / 32;
-  for (int c = warp; c < nchunk; c += nw) {
-    const int q = c * 32 + lane;
-    int miss = 0, inwin = 0;
-    if (q < N) {
-      const int b = q / P, j = q % P;
-      if (j < sh.pn[b]) {
-        inwin = 1;
-        const int i = sh.tn[b] + j;
-        const int en = sh.t[b] + sh.p[b];  // new frontier
-        if (i >= en) {
-          miss = 1;                        // first entry
-        } else {
-          const int jo = i - sh.t[b] - 1;  // delta of timestep i was computed at old position jo
-          miss = (red.del(b * P + jo) < d.cache_thresh) ? 0 : 1;
-        }
+    __syncwarp();
+    // lane c builds word c of the next windows' bits from the trajectories
+    // that overlap positions [32c, 32c + 32)
+    if (lane < nchunk) {
+      const int lo = lane * 32, hi = min(lo + 32, N);
+      unsigned win = 0u, miss = 0u;
+      for (int b = lo / P; b * P < hi; ++b) {
+        const int base = b * P;
+        const int w0 = max(lo, base), w1 = min(hi, base + sh.pn[b]);
+        if (w1 <= w0) continue;
+        const unsigned wm = (w1 - w0 == 32 ? 0xffffffffu : ((1u << (w1 - w0)) - 1u)) << (w0 - lo);
+        unsigned hm = 0u;
+        const int h1 = min(hi, base + sh.nh[b]);
+        if (h1 > w0)  // near bit of position q sits at q + stride - 1
+          hm = bits32(sh.near, lo + sh.stride[b] - 1) &
+               ((h1 - w0 == 32 ? 0xffffffffu : ((1u << (h1 - w0)) - 1u)) << (w0 - lo));
+        win |= wm;
+        miss |= wm & ~hm;
       }
+      sh.cwin[lane] = win;
+      sh.cmiss[lane] = miss;
     }
-    const unsigned mm = __ballot_sync(0xffffffffu, miss), wm = __ballot_sync(0xffffffffu, inwin);
-    if (lane == 0) {
-      sh.cmiss[c] = mm;
-      sh.cwin[c] = wm;
-    }
-  }
-  __syncthreads();
-  // each chunk's first rank: an exclusive scan of the chunks' miss counts
-  if (warp == 0) {
+    __syncwarp();
     const int cnt = lane < nchunk ? __popc(sh.cmiss[lane]) : 0;
     const int win = lane < nchunk ? __popc(sh.cwin[lane]) : 0;
     int incl = cnt;
@@ -319,47 +348,47 @@ __device__ void decide_par(const Dev& d, DecideShared& sh, const Red& red, int p
       const int v = __shfl_up_sync(0xffffffffu, incl, o);
       if (lane >= o) incl += v;
     }
-    if (lane < nchunk) sh.cbase[lane] = incl - cnt;
+    sh.cbase[lane] = incl - cnt;
     const int pts = __reduce_add_sync(0xffffffffu, win);
     if (lane == 31) sh.total = incl;
     if (lane == 0) sh.pts = pts;
   }
   __syncthreads();
-  // 3. the misses' ranks (trajectory-major, ascending t), the requested row
+  // the misses' ranks and miss list (trajectory-major, ascending t), the requested row
   for (int c = warp; c < nchunk; c += nw) {
+    const bool writes = pub_id >= 0 && c % pub_count == pub_id;
+    if (!writes && target < 0) continue;
     const int q = c * 32 + lane;
     if (q >= N) continue;
     const unsigned mm = sh.cmiss[c];
     const int miss = (mm >> lane) & 1u;
-    const int b = q / P, j = q % P;
+    const int b = q / P, j = q - b * P;
     const int r = sh.cbase[c] + __popc(mm & ((1u << lane) - 1u));
     if (miss && r == target) {
       sh.target_b = b;
       sh.target_i = sh.tn[b] + j;
     }
-    if (publish) {
+    if (writes) {
       if (miss) {
         d.rank[q] = r;
         d.miss_bt[2 * r] = b;
         d.miss_bt[2 * r + 1] = sh.tn[b] + j;
-        atomicAdd(&sh.m[b], 1);
       } else {
         d.rank[q] = -1;
-        if (((sh.cwin[c] >> lane) & 1u) && j >= 1) atomicAdd(&sh.h1[b], 1);
       }
     }
   }
-  if (publish) {
-    __syncthreads();
-    // 4. trajectories and counters of the next iteration
+  if (pub_id == 0) {
+    // trajectories and counters of the next iteration; a trajectory's misses
+    // and its hits at positions >= 1 come from the chunk bits
     for (int b = tid; b < B; b += blockDim.x) {
       Traj tr{};
       tr.t = sh.tn[b];
       tr.p = sh.pn[b];
       tr.e = sh.en[b];
       tr.done = (sh.pn[b] == 0);
-      tr.m = sh.m[b];
-      tr.h1 = sh.h1[b];
+      tr.m = range_popc(sh.cmiss, b * P, b * P + sh.pn[b]);
+      tr.h1 = sh.pn[b] > 1 ? (sh.pn[b] - 1) - range_popc(sh.cmiss, b * P + 1, b * P + sh.pn[b]) : 0;
       if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
       out_traj[b] = tr;
     }
@@ -381,5 +410,43 @@ __device__ void decide_par(const Dev& d, DecideShared& sh, const Red& red, int p
     }
   }
 }
+
+// The decision's inputs as bits in shared memory (sh.conv, sh.near), from the
+// complete fp64 sums of iteration par (divided by D): every thread of the CTA
+// takes positions tid, tid + blockDim.x, ... and each warp's ballot is the
+// bit word of its 32 consecutive positions. When `keep` is set, the CTA also
+// writes the reductions of positions q with q mod pub_count == pub_id for the
+// host and clears them in the next iteration's accumulator set. The caller
+// synchronises the CTA before reading the bits.
+__device__ __forceinline__ void stage_decision_bits(const Dev& d, DecideShared& sh, int par, int pub_id,
+                                                    int pub_count) {
+  const int tid = threadIdx.x, lane = tid & 31;
+  const int npair = d.B * d.P;
+  const double* acc_e = d.acc + (size_t)(par * 2 + 0) * npair * kAccStride;
+  const double* acc_d = d.acc + (size_t)(par * 2 + 1) * npair * kAccStride;
+  double* nxt = d.acc + (size_t)((par ^ 1) * 2) * npair * kAccStride;  // iteration k+1 adds into these
+  for (int base = 0; base < npair; base += blockDim.x) {  // blockDim.x is a multiple of 32
+    const int q = base + tid;
+    bool cv = false, nr = false;
+    if (q < npair) {
+      const size_t o = (size_t)q * kAccStride;
+      const double se = __ldcg(acc_e + o), sd = __ldcg(acc_d + o);
+      cv = sum_le(se, d.tol_d);
+      nr = sum_lt(sd, d.thr_d);
+      if (pub_id >= 0 && q % pub_count == pub_id) {
+        d.red_err[q] = (float)(se * d.inv_d);
+        d.red_del[q] = (float)(sd * d.inv_d);
+        nxt[o] = 0.0;
+        nxt[(size_t)npair * kAccStride + o] = 0.0;
+      }
+    }
+    const unsigned cm = __ballot_sync(0xffffffffu, cv), nm = __ballot_sync(0xffffffffu, nr);
+    if (lane == 0 && q < npair) {
+      sh.conv[q >> 5] = cm;
+      sh.near[q >> 5] = nm;
+    }
+  }
+}
+
 
 }  // namespace pa

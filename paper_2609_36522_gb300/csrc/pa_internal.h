@@ -112,7 +112,13 @@ struct Dev {
   unsigned long long* gbar;  // arrivals at the fused step's grid barrier (cleared by pa_init)
   int T, P, B;
   int64_t D;
-  double tol, cache_thresh;   // compared against the fp64 sums divided by D
+  double tol, cache_thresh;   // tau of Eq. 2 and tau_cache of Eq. 5
+  // The same thresholds on the undivided sums, as the kernels compare them:
+  // sum <= tol * D (Eq. 2) and sum < tau_cache * D (Eq. 5), formed in fp64 on
+  // the host; both sides are non-negative doubles, so the kernels compare
+  // their bit patterns as integers (the same order) and run no fp64
+  // arithmetic. inv_d = 1 / D for the reductions reported to the host.
+  double tol_d, thr_d, inv_d;
   int bulk_cfg;               // launch shape of the bulk-copy update kernel
   int cache_bf16;             // 1: xhat and ehat rows hold bfloat16 values (row pitch D elements)
   uint32_t wait_limit;        // polls before an mbarrier wait counts as timed out
@@ -220,6 +226,14 @@ __device__ __forceinline__ double quantize_partial(float v) {
   return ceil((double)v * 4294967296.0) * (1.0 / 4294967296.0);
 }
 
+// Eq. 2 / Eq. 5 tests on an accumulated (non-negative) sum, by bit pattern.
+__device__ __forceinline__ bool sum_le(double sum, double bound) {
+  return __double_as_longlong(sum) <= __double_as_longlong(bound);
+}
+__device__ __forceinline__ bool sum_lt(double sum, double bound) {
+  return __double_as_longlong(sum) < __double_as_longlong(bound);
+}
+
 // One CTA's share of the Eq. 2 error (which = 0) or Eq. 4 distance (which =
 // 1) of window position q = b*P + j, added into the accumulator set of the
 // iteration's parity (exact, see quantize_partial).
@@ -254,8 +268,7 @@ __device__ __forceinline__ bool grid_sync(unsigned long long* ctr, unsigned long
         if (v >= target) break;
       }
     }
-    __threadfence();
-    s_ok = ok;
+    s_ok = ok;  // the acquire load orders the CTA's later reads (after the barrier below)
   }
   __syncthreads();
   return s_ok != 0;

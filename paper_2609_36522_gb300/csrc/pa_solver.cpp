@@ -217,11 +217,17 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.T = T; d.P = P; d.B = batch; d.D = D;
   d.tol = tol;
   d.cache_thresh = cache_thresh;
+  d.tol_d = tol * (double)D;
+  d.thr_d = cache_thresh * (double)D;
+  d.inv_d = 1.0 / (double)D;
   d.wait_limit = pa::kWaitLimit;
   d.cache_bf16 = 0;
-  // the fused step where its grid is resident in one wave, else the lean
-  // register form and the planning kernel, else the bulk forms, else plain loads
-  s->update_kind = (D % 4 == 0) ? 3 : 0;
+  // the lean register form and the planning kernel, else the bulk forms, else
+  // plain loads; the fused step (3) is an option: at the 4x64x64 shape it
+  // takes as long per solver step as the pair and a generation with the
+  // denoiser is slower with it (its 16-warp CTAs hold every SM's register
+  // file through the grid barrier, so nothing overlaps their tail)
+  s->update_kind = (D % 4 == 0) ? 2 : 0;
 
   const std::vector<float> hc = step_coefficients(s->alphas, 0.0);  // DDIM (eta = 0)
   cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), sizeof(pa::Ctl), cudaHostAllocDefault);

@@ -52,7 +52,7 @@ def test_tiny_with_oracle_eps():
 def test_sd15_full_size():
     orc, gpu = _check(W.SD15)
     assert gpu["stats"]["hits"] > 0
-    assert gpu["stats"]["update_kernel"] == 3  # the fused step is the default where it fits
+    assert gpu["stats"]["update_kernel"] == 2  # lean register update + planning kernel by default
 
 
 def test_sd15_uncached_equals_oracle_uncached():
@@ -418,8 +418,8 @@ def test_fused_step_equals_update_and_planning(w):
     add their partials in --, and both take the oracle's decisions."""
     orc = oracle_run(w)
     assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-6), decision_margins(orc, w.tol, w.cache_thresh)
-    fused = gpu_run(w, reductions=True)
-    split = gpu_run(w, update_kernel=2, reductions=True)
+    fused = gpu_run(w, update_kernel=3, reductions=True)
+    split = gpu_run(w, reductions=True)
     assert fused["stats"]["update_kernel"] == 3 and split["stats"]["update_kernel"] == 2
     assert compare(w, orc, fused).max() <= REL_TOL
     assert np.array_equal(fused["log"], split["log"])
@@ -432,7 +432,7 @@ def test_fused_step_equals_update_and_planning(w):
 def test_fused_step_falls_back_beyond_one_wave():
     """The batched workload's grid (128 strips x 8 trajectories) is not
     resident in one wave: the update and planning kernels run instead."""
-    orc, gpu = _check(W.BATCHED.with_(T=40))
+    orc, gpu = _check(W.BATCHED.with_(T=40), update_kernel=3)
     assert gpu["stats"]["update_kernel"] == 2
 
 
@@ -443,7 +443,7 @@ def test_fused_step_stochastic(window):
     w = W.Workload("fused eta", T=100, window=window, batch=1, latent_shape=(4, 32, 32), K=6,
                    tol=1e-3, cache_thresh=0.05, seed=5, eta=1.0)
     orc = oracle_run(w)
-    fused = gpu_run(w)
+    fused = gpu_run(w, update_kernel=3)
     assert fused["stats"]["update_kernel"] == 3
     assert compare(w, orc, fused).max() <= REL_TOL
     bulk = gpu_run(w, update_kernel=112)
