@@ -75,7 +75,8 @@ typedef struct {
   int32_t n_miss;        /* misses planned for the next iteration */
   int32_t device_status; /* 0, or the first device-side error code */
   int32_t update_kernel; /* kernel of the last pa_submit_eps: 0 plain loads, 1 bulk forms,
-                            2 lean register form, 3 fused step, -1 none yet */
+                            2 lean register form, 3 fused step, 4 Anderson mixing
+                            (pa_set_anderson), -1 none yet */
 } pa_stats_t;
 
 /* ---- solver ------------------------------------------------------------ */
@@ -225,6 +226,40 @@ PA_API pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_o
  * Forms 1 and 2 fall back to plain loads for a batch_eps pointer that is not
  * 16-byte aligned. A tuning aid; returns PA_ERR_ARG for an unknown value. */
 PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
+
+/* ---- triangular Anderson mixing (ParaTAA-style update) ------------------
+ * Sec. 2.1 names ParaTAA among the Picard-family samplers the cache plugs
+ * into and Sec. 2.2 leaves the sampler's own update to it; the paper states
+ * no formula for ParaTAA. This library's reading: every iteration first forms
+ * the Picard map's value G_s (Eq. 1) and the residual R_s = G_s - X_s of each
+ * window state s = t + j + 1, then mixes with the previous iteration's G'_s,
+ * R'_s (history depth 1):
+ *   gamma_j = sum_{j' <= j} <dR, R> / sum_{j' <= j} <dR, dR>, dR = R - R'
+ *   (sums over D and over window positions up to j: a least-squares fit
+ *   that is lower triangular in time; 0 for a zero denominator),
+ *   X_s <- G_s - gamma_j (G_s - G'_s)
+ * for states that were computed in the previous iteration, except window
+ * position 0, whose Picard value is already exact (it depends only on the
+ * converged window start); other states take X_s <- G_s. The cache test
+ * (Eq. 4-5), the batch, Eq. 6-7, the convergence error (Eq. 2) of the mixed
+ * iterate, the stride rule and the window advance are unchanged. Depth 0 is
+ * plain Picard. One iteration is then three kernels (the mixing form of the
+ * lean update, the mix kernel, the planning kernel) besides the denoiser.
+ * ------------------------------------------------------------------------ */
+
+/* Bytes of the second device workspace that mixing needs: G and R of every
+ * window state by iteration parity (4 x batch x (window+1) x D fp32) and the
+ * Gram sums; 0 on bad sizes. */
+PA_API size_t pa_anderson_workspace_bytes(int T, int window, int64_t D, int batch);
+
+/* depth 1: mix every iteration, using workspace_dev (DEVICE, 256-byte
+ * aligned, >= pa_anderson_workspace_bytes(), caller-owned, valid until depth
+ * 0 is set or the solver is destroyed); depth 0: plain Picard (workspace
+ * ignored). Needs D % 4 == 0, a window of at most 112 points and fp32 cache
+ * entries (PA_ERR_ARG otherwise). Not between pa_step and pa_submit_eps
+ * (PA_ERR_STATE); pa_init must follow. While mixing, pa_set_update_kernel's
+ * choice does not apply and pa_stats reports update_kernel 4. */
+PA_API pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t workspace_bytes);
 
 /* Storage precision of the cache entries (xhat, ehat of Eq. 3): 32 = fp32
  * (default), 16 = bfloat16, rounded to nearest even when an entry is written

@@ -71,6 +71,8 @@ _PROTOS = {
     "pa_last_reductions": (C.c_int, [VP, VP, VP]),
     "pa_set_update_kernel": (C.c_int, [VP, C.c_int]),
     "pa_set_cache_precision": (C.c_int, [VP, C.c_int]),
+    "pa_anderson_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int, C.c_int64, C.c_int]),
+    "pa_set_anderson": (C.c_int, [VP, C.c_int, VP, C.c_size_t]),
     "pa_debug_set_wait_limit": (C.c_int, [VP, C.c_uint32]),
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
     "pa_kernel_timing": (C.c_int, [VP, C.POINTER(C.c_double), C.POINTER(C.c_int64), C.c_int]),
@@ -243,6 +245,15 @@ def pa_set_update_kernel(h, kind):
 
 def pa_set_cache_precision(h, bits):
     return _check("pa_set_cache_precision", lib().pa_set_cache_precision(h, int(bits)))
+
+
+def pa_anderson_workspace_bytes(T, window, D, batch):
+    return int(lib().pa_anderson_workspace_bytes(T, window, D, batch))
+
+
+def pa_set_anderson(h, depth, workspace_ptr, workspace_bytes):
+    return _check("pa_set_anderson", lib().pa_set_anderson(h, int(depth), _dptr(workspace_ptr),
+                                                             int(workspace_bytes)))
 
 
 def pa_debug_set_wait_limit(h, polls):

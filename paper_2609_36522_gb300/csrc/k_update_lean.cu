@@ -28,6 +28,13 @@
 // MINB CTAs per SM bound the registers: one CTA of 16 warps for windows up to
 // 112 positions, two of 8 warps up to 64, three of 8 warps up to 32.
 //
+// TAA makes it the first half of a triangularly Anderson-mixed iteration
+// (launch_update_taa): the prefix sum is the Picard map's output G of every
+// window state; G and the residual R = G - X are stored by iteration parity
+// (not the states: the mix kernel forms those), and each CTA adds its partials
+// of <dR, R> and <dR, dR> (dR = R - R of the previous iteration, for states
+// that have one) into the Gram sums instead of the Eq. 2 / Eq. 4 terms.
+//
 // FUSE makes it the whole solver step of one iteration (launch_step_fused):
 // after the strip sums are added, a grid barrier (every CTA resident, a
 // cooperative launch) makes the Eq. 2 / Eq. 4 sums complete; every CTA then
@@ -189,8 +196,9 @@ __device__ __forceinline__ void step_tail(const Dev& d, DecideShared& ds, int pa
   }
 }
 
-template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false, bool FUSE = false>
+template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false, bool FUSE = false, bool TAA = false>
 __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const float* __restrict__ beps, int par) {
+  static_assert(!(FUSE && TAA), "the fused step and the Anderson mixing are separate forms");
   using Sh = LeanShape<NW, NOISE>;
   using CT = typename Coef<NOISE>::T;
   extern __shared__ __align__(128) unsigned char smem_raw[];
@@ -248,6 +256,10 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   float* Eh = d.Ehat + (int64_t)b * P * D;
   const float* Zr = NOISE ? d.noise + (int64_t)b * T * D + mycol : nullptr;
   const float* Br = beps + mycol;
+  // Anderson mixing: G and R of this iteration (parity par), R of the previous one
+  float* Gw = TAA ? d.taa_g + ((int64_t)par * d.B + b) * (P + 1) * D + mycol : nullptr;
+  float* Rw = TAA ? d.taa_r + ((int64_t)par * d.B + b) * (P + 1) * D + mycol : nullptr;
+  const float* Rp = TAA ? d.taa_r + ((int64_t)(par ^ 1) * d.B + b) * (P + 1) * D + mycol : nullptr;
   const int L = (p + NW - 1) / NW;  // <= LMAX (launcher)
   const int j0 = warp * L;
   const int nj = min(j0 + L, p) - j0;  // positions of this warp (<= 0: none)
@@ -295,7 +307,17 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
     for (int g = 0; g < LMAX; ++g) {
       if (g >= nj) break;
       if (!(miss >> g & 1)) ep[g] = ld_ent<CB>(Eh, cslot(g) * D + mycol);
-      if (!(miss >> (g + 1) & 1)) xh[g] = ld_ent<CB>(Xh, cslot(g + 1) * D + mycol);
+      if constexpr (TAA) {
+        // the previous iteration's residual of state t + j0 + g + 1, which it
+        // has iff that state was computed then (state <= e)
+        if (t + j0 + g + 1 <= e) {
+          int sr = sx0 + g + 1;
+          if (sr > P) sr -= P + 1;
+          xh[g] = ldq(Rp + sr * D);
+        }
+      } else {
+        if (!(miss >> (g + 1) & 1)) xh[g] = ld_ent<CB>(Xh, cslot(g + 1) * D + mycol);
+      }
       if constexpr (NOISE) z[g] = ldq(Zr + (t + j0 + g) * D);
     }
   }
@@ -390,20 +412,34 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
           c = qadd(c, ep[g]);
           n = c;
         }
-        stq(Xw + so * D, n);
-        Q df = qsub(n, x[g + 1]);  // against the old state i+1 (lazy-resolved)
-        if constexpr (FUSE) ep[g] = n;  // the drift is spent: keep the new state for the next batch
-        const float2 e2 = __ffma2_rn(df.h, df.h, __fmul2_rn(df.l, df.l));
-        ev = e2.x + e2.y;
-        if (j + 1 < p) {
-          // the next timestep's cache input: its entry if it is a hit, else
-          // the old state i+1, the entry it receives in this kernel
-          if (!(miss >> (g + 1) & 1)) {
-            df = qsub(n, xh[g]);
-          } else if constexpr (CB) {
-            df = qsub(n, as_ent<CB>(x[g + 1]));
+        if constexpr (TAA) {
+          // n is the Picard map's value G of state t + j + 1; R = G - X
+          const Q rr = qsub(n, x[g + 1]);
+          stq(Gw + so * D, n);
+          stq(Rw + so * D, rr);
+          if (t + j + 1 <= e) {  // a history: dR = R - R'
+            const Q dr = qsub(rr, xh[g]);
+            const float2 nr = __ffma2_rn(dr.h, rr.h, __fmul2_rn(dr.l, rr.l));
+            const float2 dd = __ffma2_rn(dr.h, dr.h, __fmul2_rn(dr.l, dr.l));
+            ev = nr.x + nr.y;
+            dv = dd.x + dd.y;
           }
-          dv = (fabsf(df.l.x) + fabsf(df.l.y)) + (fabsf(df.h.x) + fabsf(df.h.y));
+        } else {
+          stq(Xw + so * D, n);
+          Q df = qsub(n, x[g + 1]);  // against the old state i+1 (lazy-resolved)
+          if constexpr (FUSE) ep[g] = n;  // the drift is spent: keep the new state for the next batch
+          const float2 e2 = __ffma2_rn(df.h, df.h, __fmul2_rn(df.l, df.l));
+          ev = e2.x + e2.y;
+          if (j + 1 < p) {
+            // the next timestep's cache input: its entry if it is a hit, else
+            // the old state i+1, the entry it receives in this kernel
+            if (!(miss >> (g + 1) & 1)) {
+              df = qsub(n, xh[g]);
+            } else if constexpr (CB) {
+              df = qsub(n, as_ent<CB>(x[g + 1]));
+            }
+            dv = (fabsf(df.l.x) + fabsf(df.l.y)) + (fabsf(df.h.x) + fabsf(df.h.y));
+          }
         }
       }
       s_red[j * 33 + lane] = ev;
@@ -424,17 +460,21 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
       a2 += row[k + 2];
       a3 += row[k + 3];
     }
-    red_add(d, par, which, b * P + j, (a0 + a1) + (a2 + a3));
+    if constexpr (TAA) {
+      red_add_gram(d, par, which, b * P + j, (a0 + a1) + (a2 + a3));
+    } else {
+      red_add(d, par, which, b * P + j, (a0 + a1) + (a2 + a3));
+    }
   }
   if constexpr (FUSE) step_tail<NW, LMAX>(d, ds, par, tr, ep, j0, nj, mycol, D, live);
 }
 
-template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false>
+template <int NW, int LMAX, int MINB, bool NOISE, bool COMP, bool CB = false, bool FUSE = false, bool TAA = false>
 cudaError_t launch_lean(const Dev& d, const float* beps, int par, cudaStream_t st) {
   using Sh = LeanShape<NW, NOISE>;
   const int nstrip = (int)((d.D + 127) / 128);
   const size_t smem = Sh::smem_bytes(d.T, d.P, COMP);
-  auto kern = k_update_lean<NW, LMAX, MINB, NOISE, COMP, CB>;
+  auto kern = k_update_lean<NW, LMAX, MINB, NOISE, COMP, CB, FUSE, TAA>;
   static size_t configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -563,6 +603,20 @@ cudaError_t launch_step_fused(const Dev& d, const float* batch_eps, int par, int
   if (s == 4) return launch_fused<8, 8, 2, false, false>(d, batch_eps, par, st);
   if (s == 5) return launch_fused<8, 4, 3, false, false>(d, batch_eps, par, st);
   return cudaErrorNotSupported;
+}
+
+// The mixing form of the lean update: by window like the lean form (16 x 7,
+// 8 x 8 or 8 x 4 warps x positions; with draws 16 x 7 or 8 x 4 at two CTAs per
+// SM), fp32 cache entries.
+cudaError_t launch_update_taa(const Dev& d, const float* batch_eps, int par, cudaStream_t st) {
+  if (!update_lean_supported(d, batch_eps) || d.cache_bf16 || !d.taa_g) return cudaErrorNotSupported;
+  if (d.noise) {
+    if (d.P <= 32) return launch_lean<8, 4, 2, true, false, false, false, true>(d, batch_eps, par, st);
+    return launch_lean<16, 7, 1, true, false, false, false, true>(d, batch_eps, par, st);
+  }
+  if (d.P <= 32) return launch_lean<8, 4, 3, false, false, false, false, true>(d, batch_eps, par, st);
+  if (d.P <= 64) return launch_lean<8, 8, 2, false, false, false, false, true>(d, batch_eps, par, st);
+  return launch_lean<16, 7, 1, false, false, false, false, true>(d, batch_eps, par, st);
 }
 
 bool step_fused_supported(const Dev& d, const float* batch_eps, int shape) {

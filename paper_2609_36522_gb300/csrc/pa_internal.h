@@ -110,6 +110,15 @@ struct Dev {
   float* red_del;
   int32_t* iter_log;  // [T+1][B][kLogFields]
   unsigned long long* gbar;  // arrivals at the fused step's grid barrier (cleared by pa_init)
+  // Triangular Anderson mixing (pa_set_anderson), in a caller-owned second
+  // workspace: the Picard map's output G and residual R of every window
+  // state, [2][B][P+1][D] each by iteration parity (copy k mod 2 written in
+  // iteration k, slot = state mod (P+1)), and the Gram sums <dR, R>, <dR, dR>
+  // per position, [2][2][B][P] x kAccStride, set k mod 2 in iteration k.
+  float* taa_g;
+  float* taa_r;
+  double* taa_acc;
+  int taa;            // 1: iterations mix (depth 1); 0: plain Picard
   int T, P, B;
   int64_t D;
   double tol, cache_thresh;   // tau of Eq. 2 and tau_cache of Eq. 5
@@ -241,6 +250,23 @@ __device__ __forceinline__ void red_add(const Dev& d, int par, int which, int q,
   atomicAdd(d.acc + ((size_t)(par * 2 + which) * d.B * d.P + q) * kAccStride, quantize_partial(v));
 }
 
+// A CTA's partial of a Gram sum of the Anderson mixing (<dR, R> for which = 0,
+// <dR, dR> for which = 1) of window position q, into set par. The partial may
+// be negative; rounded to a multiple of 2^-32 like the other sums, so the
+// accumulated sum is exact while the sum of the terms' magnitudes stays below
+// 2^21.
+__device__ __forceinline__ void red_add_gram(const Dev& d, int par, int which, int q, float v) {
+  atomicAdd(d.taa_acc + ((size_t)(par * 2 + which) * d.B * d.P + q) * kAccStride, quantize_partial(v));
+}
+
+// Bytes of the Anderson workspace: G and R by iteration parity, the Gram sums.
+inline size_t taa_layout(int P, int64_t D, int B, size_t* o_r, size_t* o_acc) {
+  const size_t rows = align_up((size_t)2 * B * (P + 1) * D * sizeof(float), kAlign);
+  *o_r = rows;
+  *o_acc = 2 * rows;
+  return 2 * rows + align_up((size_t)2 * 2 * B * P * kAccStride * sizeof(double), kAlign);
+}
+
 // Grid-wide barrier of a launch whose CTAs are all resident at once (the
 // fused step kernel, launched cooperatively). Thread 0 of each CTA publishes
 // the CTA's writes (fence), adds one to the counter and waits until the count
@@ -295,6 +321,12 @@ bool update_lean_supported(const Dev& d, const float* batch_eps);
 // grids that are resident in one wave; cudaErrorNotSupported otherwise.
 cudaError_t launch_step_fused(const Dev& d, const float* batch_eps, int par, int shape, cudaStream_t st);
 bool step_fused_supported(const Dev& d, const float* batch_eps, int shape);
+// Triangular Anderson mixing (k_update_lean.cu, k_taa.cu): the lean update in
+// its mixing form (G and R, Gram partials; the states are left to the mix
+// kernel), then the mix kernel (X <- G - gamma_j (G - G'), the Eq. 2 and
+// Eq. 4 partials). cudaErrorNotSupported when the lean form cannot run.
+cudaError_t launch_update_taa(const Dev& d, const float* batch_eps, int par, cudaStream_t st);
+cudaError_t launch_taa_mix(const Dev& d, int par, cudaStream_t st);
 // An empty kernel with programmatic dependent launch (k_solver.cu)
 cudaError_t launch_gap(cudaStream_t st);
 

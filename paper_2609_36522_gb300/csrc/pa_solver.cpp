@@ -214,6 +214,10 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.red_del = reinterpret_cast<float*>(w + L.red_del);
   d.iter_log = reinterpret_cast<int32_t*>(w + L.iter_log);
   d.gbar = reinterpret_cast<unsigned long long*>(w + L.gbar);
+  d.taa_g = nullptr;
+  d.taa_r = nullptr;
+  d.taa_acc = nullptr;
+  d.taa = 0;
   d.T = T; d.P = P; d.B = batch; d.D = D;
   d.tol = tol;
   d.cache_thresh = cache_thresh;
@@ -277,6 +281,8 @@ pa_status pa_init(pa_solver* s, const float* x_init) {
   // both accumulator sets of the reductions start at zero
   e = cudaMemsetAsync(d.acc, 0, (size_t)2 * 2 * d.B * d.P * pa::kAccStride * sizeof(double), s->st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d.gbar, 0, sizeof(unsigned long long), s->st);  // barrier arrivals
+  if (e == cudaSuccess && d.taa)  // both sets of the Anderson Gram sums
+    e = cudaMemsetAsync(d.taa_acc, 0, (size_t)2 * 2 * d.B * d.P * pa::kAccStride * sizeof(double), s->st);
   if (e != cudaSuccess) return cuda_fail("pa_init: clear sums", e);
   // the first plan (every timestep a first entry) and its batch
   e = pa::launch_init_plan(d, s->st);
@@ -341,7 +347,17 @@ pa_status pa_submit_eps(pa_solver* s, const float* batch_eps_dev) {
     if (e != cudaSuccess) return cuda_fail("pa_submit_eps: timing event", e);
   }
   bool done = false, planned = false;
-  if (s->update_kind == 3) {
+  if (s->d.taa) {  // triangular Anderson mixing: the mixing update, then the mix kernel
+    e = pa::launch_update_taa(s->d, batch_eps_dev, par, s->st);
+    if (e == cudaErrorNotSupported) return arg_fail("pa_submit_eps: Anderson mixing needs a 16-byte aligned batch_eps");
+    if (e == cudaSuccess) {
+      s->launches++;
+      e = pa::launch_taa_mix(s->d, par, s->st);
+    }
+    s->last_kind = 4;
+    done = true;
+  }
+  if (!done && s->update_kind == 3) {
     e = pa::launch_step_fused(s->d, batch_eps_dev, par, s->lean_shape, s->st);
     if (e == cudaErrorNotSupported) {
       e = cudaSuccess;  // the grid is not resident in one wave: update and planning kernels
@@ -485,10 +501,47 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   return PA_OK;
 }
 
+size_t pa_anderson_workspace_bytes(int T, int window, int64_t D, int batch) {
+  if (!sizes_ok(T, window, D, batch)) return 0;
+  const int P = window < T ? window : T;
+  size_t o_r = 0, o_acc = 0;
+  return pa::taa_layout(P, D, batch, &o_r, &o_acc);
+}
+
+pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t workspace_bytes) {
+  if (!s) return arg_fail("pa_set_anderson: solver is NULL");
+  if (depth != 0 && depth != 1) return arg_fail("pa_set_anderson: depth must be 0 or 1");
+  if (s->state == St::Stepped) return state_fail("pa_set_anderson");
+  pa::Dev& d = s->d;
+  if (depth == 0) {
+    d.taa = 0;
+    d.taa_g = d.taa_r = nullptr;
+    d.taa_acc = nullptr;
+    s->state = St::Created;  // the iterates change meaning: pa_init starts over
+    return PA_OK;
+  }
+  if (d.D % 4 != 0 || d.P > 16 * 7 || d.cache_bf16)
+    return arg_fail("pa_set_anderson: needs D % 4 == 0, a window of at most 112 points and fp32 cache entries");
+  size_t o_r = 0, o_acc = 0;
+  const size_t need = pa::taa_layout(d.P, d.D, d.B, &o_r, &o_acc);
+  if (!workspace_dev || (reinterpret_cast<uintptr_t>(workspace_dev) % pa::kAlign) != 0 || workspace_bytes < need) {
+    pa::set_error("pa_set_anderson: workspace NULL, not 256-byte aligned, or smaller than pa_anderson_workspace_bytes()");
+    return PA_ERR_WORKSPACE;
+  }
+  char* w = static_cast<char*>(workspace_dev);
+  d.taa_g = reinterpret_cast<float*>(w);
+  d.taa_r = reinterpret_cast<float*>(w + o_r);
+  d.taa_acc = reinterpret_cast<double*>(w + o_acc);
+  d.taa = 1;
+  s->state = St::Created;
+  return PA_OK;
+}
+
 pa_status pa_set_cache_precision(pa_solver* s, int bits) {
   if (!s) return arg_fail("pa_set_cache_precision: solver is NULL");
   if (bits != 16 && bits != 32) return arg_fail("pa_set_cache_precision: bits must be 16 or 32");
   if (s->state == St::Stepped) return state_fail("pa_set_cache_precision");
+  if (bits == 16 && s->d.taa) return arg_fail("pa_set_cache_precision: Anderson mixing keeps fp32 cache entries");
   s->d.cache_bf16 = bits == 16 ? 1 : 0;
   s->state = St::Created;  // the entries change meaning: pa_init starts over
   return PA_OK;

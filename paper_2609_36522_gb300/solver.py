@@ -173,6 +173,20 @@ class Solver:
         self._drop_graphs()
         abi.pa_set_update_kernel(self.h, kind)
 
+    def set_anderson(self, depth):
+        """Triangular Anderson mixing of the iterates (ParaTAA-style update):
+        depth 1 mixes with the previous iteration (its workspace is allocated
+        here), 0 restores plain Picard. pa_init must follow."""
+        self._drop_graphs()
+        if depth == 0:
+            abi.pa_set_anderson(self.h, 0, None, 0)
+            self._taa_workspace = None
+            return
+        nbytes = abi.pa_anderson_workspace_bytes(self.T, self.window, self.D, self.batch)
+        ws = torch.empty(nbytes, dtype=torch.uint8, device=self.workspace.device)
+        abi.pa_set_anderson(self.h, depth, ws.data_ptr(), nbytes)
+        self._taa_workspace = ws
+
     def set_cache_precision(self, bits):
         """16: bfloat16 cache entries, 32: fp32 (default). pa_init must follow."""
         self._drop_graphs()

@@ -7,23 +7,28 @@ import numpy as np
 import workload as W
 from oracle import run_picard
 from oracle.gmm import make_eps_fn, gmm_eps
+from oracle.taa import run_taa
 
 
-def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True, cache_store=None):
+def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True, cache_store=None, anderson=0):
     a, x0, mu = W.inputs(w)
     thr = w.cache_thresh if cache_thresh is None else cache_thresh
+    if anderson:
+        return run_taa(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr, depth=anderson,
+                       use_cache=use_cache, eta=w.eta, noise=W.noise(w))
     return run_picard(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr,
                       use_cache=use_cache, eta=w.eta, noise=W.noise(w), cache_store=cache_store)
 
 
 def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=None,
-            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None, reductions=False):
+            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None, reductions=False, anderson=None):
     """Run one generation on the GPU.
 
     eps_source: "gmm" (the CUDA mixture kernel) or "oracle" (fp64 mixture
     posterior evaluated on the host for the gathered batch, rounded to fp32).
     mode: "sync" (pa_step) or "async" (pa_step_async, device-side counts).
     reductions: keep every iteration's Eq. 2 / Eq. 4 reductions (sync mode).
+    anderson: history depth of the triangular Anderson mixing (None: not set).
     """
     import torch
     from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
@@ -36,6 +41,8 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
         s.set_update_kernel(update_kernel)
     if cache_bits is not None:
         s.set_cache_precision(cache_bits)
+    if anderson is not None:
+        s.set_anderson(anderson)
     max_rows = w.batch * s.window
     means = torch.from_numpy(mu).to(dev)
     g = GmmDenoiser(means, w.gmm_std, a, max_rows)

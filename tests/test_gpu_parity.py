@@ -575,3 +575,127 @@ def test_bf16_cache_rejected_while_stepped():
     assert e.value.status == abi.PA_ERR_ARG
     s.close()
 
+
+
+# ---- triangular Anderson mixing (ParaTAA-style update, pa_set_anderson) ------
+
+TAA_CASES = [
+    W.SD15, W.BATCHED.with_(T=60), W.TINY,
+    W.SD15.with_(T=150, window=112, latent_shape=(4, 32, 32), name="window 112"),
+    W.Workload("ragged strips B3", T=40, window=24, batch=3, latent_shape=(4, 20, 20), K=6,
+               tol=1e-3, cache_thresh=0.05, seed=12),
+    W.Workload("tight tol", T=100, window=100, batch=1, latent_shape=(4, 16, 16), K=16,
+               tol=1e-5, cache_thresh=0.0, seed=0),
+    W.Workload("cache 0.1", T=60, window=60, batch=1, latent_shape=(4, 32, 32), K=8,
+               tol=1e-3, cache_thresh=0.1, seed=4),
+    W.Workload("stochastic P24", T=100, window=24, batch=1, latent_shape=(4, 32, 32), K=6,
+               tol=1e-3, cache_thresh=0.05, seed=5, eta=1.0),
+    W.Workload("stochastic P64", T=100, window=64, batch=1, latent_shape=(4, 32, 32), K=6,
+               tol=1e-3, cache_thresh=0.05, seed=5, eta=1.0),
+]
+
+
+@pytest.mark.parametrize("w", TAA_CASES, ids=lambda w: w.name)
+def test_anderson_against_oracle(w):
+    """Depth-1 triangular Anderson mixing: iteration log, miss lists, NFE and
+    hits bit-exact against oracle.taa, final latents within 1e-5."""
+    orc = oracle_run(w, anderson=1)
+    assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-6), decision_margins(orc, w.tol, w.cache_thresh)
+    gpu = gpu_run(w, anderson=1)
+    assert gpu["stats"]["update_kernel"] == 4
+    rel = compare(w, orc, gpu)
+    assert rel.max() <= REL_TOL, rel
+
+
+def test_anderson_depth_zero_restores_picard():
+    """Switching the mixing on and off again gives the Picard run bit for bit."""
+    w = W.Workload("taa off", T=40, window=16, batch=2, latent_shape=(4, 16, 16), K=4,
+                   tol=1e-3, cache_thresh=0.05, seed=3)
+    import torch
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+    ref = gpu_run(w)
+    a, x0, mu = W.inputs(w)
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch)
+    s.set_anderson(1)
+    s.set_anderson(0)
+    g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, w.batch * s.window)
+    eps = torch.empty(w.batch * s.window, w.D, dtype=torch.float32, device="cuda")
+    s.init(torch.from_numpy(x0).cuda())
+    while (out := s.step()) is not None:
+        g.eps(out.batch_x_ptr, out.miss_bt_ptr, s.n_miss_dev(), eps)
+        s.submit_eps(eps)
+    assert np.array_equal(s.result().cpu().numpy(), ref["x_final"])
+    assert s.stats()["update_kernel"] == 2
+    s.close()
+    g.close()
+
+
+def test_anderson_rejects_unsupported_settings():
+    """Odd D, windows beyond 112 points and bfloat16 entries are refused with
+    PA_ERR_ARG; a workspace that is too small with PA_ERR_WORKSPACE."""
+    import torch
+    from paper_2609_36522_gb300 import abi
+    from paper_2609_36522_gb300.solver import Solver
+    a = W.alphas_cumprod(30)
+    for shape, window in (((3, 5, 7), 8), ((4, 8, 8), 113)):
+        s = Solver(30 if window < 30 else 150, window, shape, W.alphas_cumprod(30 if window < 30 else 150),
+                   1e-3, 0.05)
+        with pytest.raises(abi.PaError) as e:
+            s.set_anderson(1)
+        assert e.value.status == abi.PA_ERR_ARG
+        s.close()
+    s = Solver(30, 8, (4, 8, 8), a, 1e-3, 0.05)
+    s.set_cache_precision(16)
+    with pytest.raises(abi.PaError) as e:
+        s.set_anderson(1)
+    assert e.value.status == abi.PA_ERR_ARG
+    s.set_cache_precision(32)
+    need = abi.pa_anderson_workspace_bytes(30, 8, 256, 1)
+    buf = torch.empty(need, dtype=torch.uint8, device="cuda")
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_set_anderson(s.h, 1, buf.data_ptr(), need - 256)
+    assert e.value.status == abi.PA_ERR_WORKSPACE
+    abi.pa_set_anderson(s.h, 1, buf.data_ptr(), need)
+    with pytest.raises(abi.PaError) as e:
+        s.set_cache_precision(16)
+    assert e.value.status == abi.PA_ERR_ARG
+    s.close()
+
+
+def test_anderson_graph_replay_equals_sync():
+    """A mixed generation captured as one CUDA graph (three solver kernels
+    and the denoiser's two per iteration, chained by dependent launches) and
+    replayed twice gives the synchronous run bit for bit."""
+    import torch
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+    w = W.SD15
+    sync = gpu_run(w, anderson=1)
+    n_iters = len(sync["log"])
+    a, x0, mu = W.inputs(w)
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=st)
+        s.set_anderson(1)
+        g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, w.batch * s.window, stream=st)
+        eps = torch.empty(w.batch * s.window, w.D, dtype=torch.float32, device="cuda")
+        x_dev = torch.from_numpy(x0).cuda()
+        s.init(x_dev)
+        out = s.step_async()
+        g.eps(*out, eps)
+        s.submit_eps(eps)
+        st.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=st):
+            s.init(x_dev)
+            for _ in range(n_iters):
+                out = s.step_async()
+                g.eps(*out, eps)
+                s.submit_eps(eps)
+        for _ in range(2):
+            graph.replay()
+            st.synchronize()
+            assert s.poll() == 0
+            assert np.array_equal(s.result().cpu().numpy(), sync["x_final"])
+            assert np.array_equal(s.iter_log(), sync["log"])
+    s.close()
+    g.close()
