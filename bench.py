@@ -72,7 +72,8 @@ def parse_args(argv=None):
     ap.add_argument("--steps", type=int, default=200)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=sorted(W.ALL), default="sd15")
+    ap.add_argument("--workload", choices=sorted(W.ALL), default="sd15",
+                    help="sd15 is the headline; *_taa run the triangular Anderson (ParaTAA-style) update")
     ap.add_argument("--no-flush", action="store_true", help="do not flush L2 between iterations")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -172,7 +173,17 @@ def iteration_bytes(log, w: W.Workload, entry_bytes=4, fused=False):
             if p == 0:
                 continue
             lazy = max(0, t + p - e)
-            upd[k] += (1 + (p - lazy) + m + p + (p if w.eta != 0.0 else 0)) * row + ((p - m) + 2 * m + h1) * ent
+            zr = p if w.eta != 0.0 else 0
+            if w.sampler == "taa":
+                # mixing update: x_t, old states, eps rows, the previous R of
+                # states with a history (nh); entries of the misses, G and R
+                # written. mix kernel: G, G' of mixed positions, old states,
+                # next-hit entries read; the new states written
+                nh = max(0, min(p, e - t))
+                upd[k] += ((1 + (p - lazy) + m + nh + zr + 2 * p) + (p + max(0, nh - 1) + (p - lazy) + h1 + p)) \
+                    * row + ((p - m) + 2 * m) * ent
+            else:
+                upd[k] += (1 + (p - lazy) + m + p + zr) * row + ((p - m) + 2 * m + h1) * ent
             den[k] += 2 * m * row
             if k + 1 < n:
                 gat[k] += (1 if fused else 2) * int(log[k + 1, b, 2]) * row
@@ -239,6 +250,7 @@ def oracle_sample(workload_name, budget_s, cache_thresh=None):
     denoiser calls took (the solver step = the rest). Runs in a fresh process."""
     from oracle import run_picard, run_srds
     from oracle.gmm import make_eps_fn
+    from oracle.taa import run_taa
     w = W.ALL[workload_name]
     if cache_thresh is not None:
         w = w.with_(cache_thresh=cache_thresh)
@@ -258,6 +270,10 @@ def oracle_sample(workload_name, budget_s, cache_thresh=None):
         if w.sampler == "srds":   # a solver step is one evaluation stage
             r = run_srds(a, x0, f_timed, w.tol, w.cache_thresh)
             iters += len(r.batches)
+        elif w.sampler == "taa":
+            r = run_taa(a, x0, f_timed, w.window, w.tol, w.cache_thresh, depth=1, record=False,
+                        eta=w.eta, noise=W.noise(w))
+            iters += r.iters
         else:
             r = run_picard(a, x0, f_timed, w.window, w.tol, w.cache_thresh, record=False,
                            eta=w.eta, noise=W.noise(w))
@@ -406,6 +422,8 @@ def run_ours(args):
             sv.set_cache_precision(16)
         if noise_dev is not None:  # stochastic steps: the draws stay resident on the device
             sv.set_noise(w.eta, noise_dev)
+        if w.sampler == "taa":     # triangular Anderson mixing of depth 1
+            sv.set_anderson(1)
         return sv
 
     s = make_solver(w.cache_thresh)
@@ -617,7 +635,8 @@ def run_ours(args):
     sha = kernel_source_sha()
     tkey = args.workload + ("-bf16" if args.cache_bits == 16 else "")
     traffic = NCU_TRAFFIC.get((sha, tkey))
-    step_kernel = {3: "fused step (update, grid barrier, decision, next batch from registers)",
+    step_kernel = {4: "Anderson-mixing update + mix kernel + planning kernel",
+                   3: "fused step (update, grid barrier, decision, next batch from registers)",
                    2: "lean register update + planning kernel",
                    1: "register-resident or staged update + planning kernel"}.get(st1["update_kernel"],
                                                                                  "plain-load update + planning kernel")

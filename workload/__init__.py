@@ -54,7 +54,8 @@ class Workload:
     seed: int = 0               # trajectory b uses noise seed (seed + b)
     gmm_std: float = GMM_STD
     eta: float = 0.0            # stochastic steps (eta = 1: DDPM); 0 = DDIM
-    sampler: str = "picard"     # "picard" (sliding window) or "srds" (Parareal blocks; window unused)
+    sampler: str = "picard"     # "picard" (sliding window), "taa" (the same with triangular
+                                # Anderson mixing of depth 1) or "srds" (Parareal blocks; window unused)
     extra: dict = field(default_factory=dict, compare=False)
 
     @property
@@ -81,6 +82,9 @@ DDPM = Workload("DDPM T1000 P64 B1 4x64x64 K16", T=1000, window=64, batch=1,
 # Parareal (SRDS-style) sampling with the cache, on the SD-shaped and batched inputs.
 SRDS = SD15.with_(name="SRDS T100 B1 4x64x64 K16", sampler="srds")
 SRDS_BATCHED = BATCHED.with_(name="SRDS T100 B8 4x64x64 K16", sampler="srds")
+# Triangular Anderson mixing (a ParaTAA-style update) on the SD-shaped and batched inputs.
+SD15_TAA = SD15.with_(name="SD-v1.5-shaped T100 P100 B1 4x64x64 K16 TAA", sampler="taa")
+BATCHED_TAA = BATCHED.with_(name="batched T100 P32 B8 4x64x64 K16 TAA", sampler="taa")
 SWEEP_THRESHOLDS = (0.0, 0.01, 0.02, 0.05, 0.1)
 
 
@@ -91,7 +95,7 @@ def sweep(base: Workload = SD15):
 
 
 ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM,
-       "srds": SRDS, "srds_batched": SRDS_BATCHED}
+       "srds": SRDS, "srds_batched": SRDS_BATCHED, "sd15_taa": SD15_TAA, "batched_taa": BATCHED_TAA}
 
 
 def train_alphas_cumprod() -> np.ndarray:
