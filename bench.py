@@ -250,10 +250,12 @@ def oracle_sample(workload_name, budget_s, cache_thresh=None):
     denoiser calls took (the solver step = the rest). Runs in a fresh process."""
     from oracle import run_picard, run_srds
     from oracle.gmm import make_eps_fn
+    from oracle.picard import CacheAdaptation
     from oracle.taa import run_taa
     w = W.ALL[workload_name]
     if cache_thresh is not None:
         w = w.with_(cache_thresh=cache_thresh)
+    adapt = CacheAdaptation(*w.extra["adapt"]) if w.extra.get("adapt") else None
     a, x0, mu = W.inputs(w)
     f = make_eps_fn(a, mu, w.gmm_std)
     t_eps = [0.0]
@@ -272,11 +274,11 @@ def oracle_sample(workload_name, budget_s, cache_thresh=None):
             iters += len(r.batches)
         elif w.sampler == "taa":
             r = run_taa(a, x0, f_timed, w.window, w.tol, w.cache_thresh, depth=1, record=False,
-                        eta=w.eta, noise=W.noise(w))
+                        eta=w.eta, noise=W.noise(w), adapt=adapt)
             iters += r.iters
         else:
             r = run_picard(a, x0, f_timed, w.window, w.tol, w.cache_thresh, record=False,
-                           eta=w.eta, noise=W.noise(w))
+                           eta=w.eta, noise=W.noise(w), adapt=adapt)
             iters += r.iters
         gens += 1
         if time.perf_counter() - t0 >= budget_s:
@@ -344,7 +346,9 @@ def cpu_baseline(workload_name, budget_s=10.0, cache_thresh=None):
 
 def workload_config(w: W.Workload, world, steps_per_gen):
     """The ``config`` of a bench line: the workload only, the same for both arms."""
-    return {"workload": w.name,
+    extra = {"cache_adaptation": dict(zip(("rate", "target", "tau_min", "tau_max"), w.extra["adapt"]))} \
+        if w.extra.get("adapt") else {}
+    return {**extra, "workload": w.name,
             "step": ("one full cached Parareal generation (solver step = evaluation stage)"
                      if w.sampler == "srds" else "one full cached-Picard generation"),
             "solver_steps_per_step": int(steps_per_gen), "global_batch": w.batch * world, "seq_len": w.T,
@@ -424,6 +428,8 @@ def run_ours(args):
             sv.set_noise(w.eta, noise_dev)
         if w.sampler == "taa":     # triangular Anderson mixing of depth 1
             sv.set_anderson(1)
+        if w.extra.get("adapt") and cache_thresh > 0.0:   # tau_cache adapted online
+            sv.set_cache_adaptation(*w.extra["adapt"])
         return sv
 
     s = make_solver(w.cache_thresh)

@@ -187,7 +187,8 @@ PA_API pa_status pa_stats(pa_solver* s, pa_stats_t* out);
 /* Per-iteration log, HOST buffer out[max_iters][batch][8] int32:
  * (window start t, evaluation points p, misses of trajectory b, stride,
  *  evaluated frontier e before the iteration (states > e were lazy copies of
- *  state e), hits among window positions 1..p-1, 0, 0).
+ *  state e), hits among window positions 1..p-1, window positions that had a
+ *  cache entry, hits among them).
  * *n_iters receives the number of logged iterations. Synchronises. */
 PA_API pa_status pa_iter_log(pa_solver* s, int32_t* out, int max_iters, int* n_iters);
 
@@ -260,6 +261,33 @@ PA_API size_t pa_anderson_workspace_bytes(int T, int window, int64_t D, int batc
  * (PA_ERR_STATE); pa_init must follow. While mixing, pa_set_update_kernel's
  * choice does not apply and pa_stats reports update_kernel 4. */
 PA_API pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t workspace_bytes);
+
+/* ---- online adaptation of tau_cache ---------------------------------------
+ * The paper's conclusion names an online adaptive tau_cache as future work and
+ * states no rule. This library's reading: every trajectory keeps its own
+ * tau_cache, starting at pa_create's cache_thresh; after each iteration, with
+ * n_e of its window positions that had a cache entry and n_h hits among them
+ * (Eq. 5):
+ *   n_h / n_e <  target:  tau <- min(tau * (1 + rate), tau_max) if the window
+ *                         advanced beyond its first position (stride > 1),
+ *                         else tau holds (reuse is not raised while the window
+ *                         stalls);
+ *   n_h / n_e >= target:  tau <- max(tau / (1 + rate), tau_min);
+ *   n_e = 0:              tau holds;
+ * and the next iteration's hit test (Eq. 5) uses the new tau. All of it runs
+ * in the planning kernel's decision (fp64 on the device, exactly as on the
+ * host). rate = 0 switches adaptation off (tau_cache fixed, the default).
+ * ------------------------------------------------------------------------ */
+
+/* rate >= 0 (0: off), 0 <= target <= 1, 0 <= tau_min <= tau_max (tau_max may
+ * be +inf). Needs batch * window <= 1024 when rate > 0. PA_ERR_ARG otherwise;
+ * PA_ERR_STATE between pa_step and pa_submit_eps; pa_init must follow. */
+PA_API pa_status pa_set_cache_adaptation(pa_solver* s, double rate, double target, double tau_min, double tau_max);
+
+/* The tau_cache of the planned iteration's hit test, per trajectory, into a
+ * HOST array of batch doubles (cache_thresh for every trajectory when
+ * adaptation is off). PA_ERR_STATE before pa_init. Synchronises. */
+PA_API pa_status pa_cache_thresholds(pa_solver* s, double* tau_out);
 
 /* Storage precision of the cache entries (xhat, ehat of Eq. 3): 32 = fp32
  * (default), 16 = bfloat16, rounded to nearest even when an entry is written

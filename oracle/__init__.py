@@ -16,7 +16,10 @@ ddim    -- DDIM step (eta = 0, and eta > 0 with draws fixed before sampling),
 gmm     -- posterior-mean noise of an isotropic Gaussian mixture, the synthetic
            stand-in for the SD v1.5 UNet eps_theta.
 picard  -- sliding-window Picard iteration (Eq. 1, Eq. 2) with ParaAnya's
-           output cache (Eq. 3-7), for a batch of independent trajectories.
+           output cache (Eq. 3-7), for a batch of independent trajectories,
+           optionally with tau_cache adapted online (CacheAdaptation).
+taa     -- the same with triangular Anderson mixing of the iterates
+           (a ParaTAA-style update, depth 0 or 1).
 srds    -- Parareal (SRDS-style) DDIM sampling with the same cache on the
            coarse and fine evaluations (Sec. 2.1, Sec. 2.2).
 guard   -- decision-margin guard used to reject generated inputs whose
@@ -31,7 +34,7 @@ scalar pure-Python implementation for tiny T in ``tests/scalar_picard.py``.
 Every function here carries a pin; none is "parity unpinned".
 """
 from . import ddim, gmm, picard, guard, srds  # noqa: F401
-from .picard import run_picard, PicardResult  # noqa: F401
+from .picard import run_picard, PicardResult, CacheAdaptation  # noqa: F401
 from .srds import run_srds, SrdsResult  # noqa: F401
 from .ddim import serial_ddim, drift_coefficients  # noqa: F401
 from .gmm import gmm_eps  # noqa: F401

@@ -5,7 +5,8 @@ The GPU keeps fp32 states while the oracle runs in fp64, so a cache distance
 could be decided differently by the two. Inputs are therefore rejected when any
 decision the oracle actually took lies within ``rel`` (relative) of its
 threshold: every delta of a point that had a cache entry (it decides hit or
-miss), and every err_j that the stride depends on (the leading run up to and
+miss, against the tau_cache of that iteration and trajectory when tau_cache
+adapts), and every err_j that the stride depends on (the leading run up to and
 including the first err_j > tau, excluding the last window position, whose
 error never changes the stride).
 """
@@ -24,10 +25,11 @@ def decision_margins(result, tol, cache_thresh):
     m_err = math.inf
     for rec in result.records:
         for b, deltas in enumerate(rec.delta):
-            if cache_thresh > 0:
+            thr = rec.tau[b] if rec.tau is not None else cache_thresh   # adapted per iteration
+            if thr > 0:
                 for d in deltas:
                     if d is not None:
-                        m_delta = min(m_delta, abs(d - cache_thresh) / cache_thresh)
+                        m_delta = min(m_delta, abs(d - thr) / thr)
             errs = rec.err[b]
             p = len(errs)
             if tol > 0 and p > 1:

@@ -41,6 +41,33 @@ from .ddim import drift, step_coefficients
 
 
 @dataclass
+class CacheAdaptation:
+    """Online adaptation of tau_cache (the paper names it as future work in
+    its conclusion and states no rule; this is the reading written down in the
+    design notes). Per trajectory, after every iteration: with n_e of its
+    window positions that had a cache entry and n_h hits among them,
+      n_h / n_e <  target: tau <- min(tau * (1 + rate), tau_max), but only if
+                           the window advanced beyond its first position
+                           (stride > 1); with stride 1 tau holds;
+      n_h / n_e >= target: tau <- max(tau / (1 + rate), tau_min);
+    no entries (n_e = 0): tau holds. The next iteration's hit test (Eq. 5)
+    uses the new tau. rate = 0 keeps tau_cache fixed."""
+
+    rate: float
+    target: float
+    tau_min: float = 0.0
+    tau_max: float = float("inf")
+
+    def step(self, tau, n_e, n_h, stride):
+        if n_e == 0:
+            return tau
+        up = 1.0 + self.rate
+        if n_h / n_e < self.target:
+            return min(tau * up, self.tau_max) if stride > 1 else tau
+        return max(tau / up, self.tau_min)
+
+
+@dataclass
 class IterRecord:
     """What one Picard iteration decided, per trajectory and globally."""
 
@@ -52,6 +79,7 @@ class IterRecord:
     miss_bt: List[tuple]              # canonical miss order (b, i)
     err: List[List[float]]            # Eq. 2 error per window position
     stride: List[int]
+    tau: Optional[List[float]] = None  # tau_cache per trajectory used by this iteration's hit test
 
 
 @dataclass
@@ -70,7 +98,7 @@ class PicardResult:
 
 def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
                use_cache=True, max_iters=None, record=True, eta=0.0, noise=None,
-               cache_store=None):
+               cache_store=None, adapt=None):
     """Cached (or uncached) sliding-window Picard sampling of B trajectories.
 
     alphas       : fp64 [T+1] sampling-order alpha-bar (alphas[T] == 1).
@@ -87,6 +115,9 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
     cache_store  : how a cache entry is stored (step 5): None keeps the value,
                    oracle.storage.round_bf16 stores bfloat16 entries (states
                    and the fresh eps of a miss keep full precision).
+    adapt        : a CacheAdaptation: tau_cache per trajectory, starting at
+                   cache_thresh and adapted after every iteration; None keeps
+                   cache_thresh fixed.
     """
     a = np.asarray(alphas, dtype=np.float64)
     T = len(a) - 1
@@ -113,6 +144,7 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
     active = np.ones(B, dtype=bool)
     iters_per = [0] * B
     nfe = hits = 0
+    tau = [float(cache_thresh)] * B
     records: List[IterRecord] = []
     k = 0
     while active.any():
@@ -120,6 +152,7 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
             break
         k += 1
         p = [int(min(P, T - t[b])) if active[b] else 0 for b in range(B)]
+        tau_k = list(tau)
 
         # 1-2. cache distance (Eq. 4) and hit/miss partition (Eq. 5)
         deltas, hitflags = [], []
@@ -130,7 +163,7 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
                 if use_cache and has_entry[b, i]:
                     d_bi = float(np.sum(np.abs(X[b, i] - Xhat[b, i])) / D)
                     db.append(d_bi)
-                    hb.append(d_bi < cache_thresh)
+                    hb.append(d_bi < tau[b])
                 else:
                     db.append(None)          # first entry (or no cache): miss
                     hb.append(False)
@@ -196,6 +229,9 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
                 active[b] = False
             errs.append([float(v) for v in err])
             strides.append(stride)
+            if adapt is not None:   # tau_cache for the next iteration's hit test
+                n_e = sum(1 for dv in deltas[b] if dv is not None)
+                tau[b] = adapt.step(tau[b], n_e, sum(hitflags[b]), stride)
 
         n_miss = len(miss_bt)
         nfe += n_miss
@@ -205,7 +241,7 @@ def run_picard(alphas, x_init, eps_fn, window, tol, cache_thresh,
                 k=k,
                 t=[int(t[b] - strides[b]) if p[b] else -1 for b in range(B)],
                 p=p, delta=deltas, hit=hitflags, miss_bt=miss_bt,
-                err=errs, stride=strides))
+                err=errs, stride=strides, tau=tau_k))
 
     return PicardResult(x_final=X[:, T].copy(), states=X, iters=k,
                         iters_per_traj=iters_per, nfe=nfe, hits=hits,

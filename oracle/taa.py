@@ -48,11 +48,12 @@ from .picard import IterRecord, PicardResult
 
 
 def run_taa(alphas, x_init, eps_fn, window, tol, cache_thresh, depth=1,
-            use_cache=True, record=True, eta=0.0, noise=None, gammas=None):
+            use_cache=True, record=True, eta=0.0, noise=None, gammas=None, adapt=None):
     """Cached (or uncached) sliding-window Picard sampling with triangular
     Anderson mixing of history depth ``depth`` (0 or 1), for B trajectories.
 
-    Arguments as ``oracle.picard.run_picard``; ``gammas``, if a list, receives
+    Arguments as ``oracle.picard.run_picard`` (``adapt``: tau_cache adapted per
+    trajectory after every iteration, oracle.picard.CacheAdaptation); ``gammas``, if a list, receives
     per iteration the list over trajectories of the mixing coefficients of the
     window positions (0.0 where a position has no history).
     """
@@ -87,11 +88,13 @@ def run_taa(alphas, x_init, eps_fn, window, tol, cache_thresh, depth=1,
     active = np.ones(B, dtype=bool)
     iters_per = [0] * B
     nfe = hits = 0
+    tau = [float(cache_thresh)] * B
     records: List[IterRecord] = []
     k = 0
     while active.any():
         k += 1
         p = [int(min(P, T - t[b])) if active[b] else 0 for b in range(B)]
+        tau_k = list(tau)
 
         # 1-2. cache distance (Eq. 4) and hit/miss partition (Eq. 5)
         deltas, hitflags = [], []
@@ -102,7 +105,7 @@ def run_taa(alphas, x_init, eps_fn, window, tol, cache_thresh, depth=1,
                 if use_cache and has_entry[b, i]:
                     d_bi = float(np.sum(np.abs(X[b, i] - Xhat[b, i])) / D)
                     db.append(d_bi)
-                    hb.append(d_bi < cache_thresh)
+                    hb.append(d_bi < tau[b])
                 else:
                     db.append(None)
                     hb.append(False)
@@ -182,6 +185,9 @@ def run_taa(alphas, x_init, eps_fn, window, tol, cache_thresh, depth=1,
             errs.append([float(v) for v in err])
             strides.append(stride)
             gam_k.append([float(v) for v in gam])
+            if adapt is not None:   # tau_cache for the next iteration's hit test
+                n_e = sum(1 for dv in deltas[b] if dv is not None)
+                tau[b] = adapt.step(tau[b], n_e, sum(hitflags[b]), stride)
 
         n_miss = len(miss_bt)
         nfe += n_miss
@@ -191,7 +197,7 @@ def run_taa(alphas, x_init, eps_fn, window, tol, cache_thresh, depth=1,
         if record:
             records.append(IterRecord(
                 k=k, t=[int(t[b] - strides[b]) if p[b] else -1 for b in range(B)],
-                p=p, delta=deltas, hit=hitflags, miss_bt=miss_bt, err=errs, stride=strides))
+                p=p, delta=deltas, hit=hitflags, miss_bt=miss_bt, err=errs, stride=strides, tau=tau_k))
 
     return PicardResult(x_final=X[:, T].copy(), states=X, iters=k, iters_per_traj=iters_per,
                         nfe=nfe, hits=hits, records=records, xhat=Xhat, ehat=Ehat,

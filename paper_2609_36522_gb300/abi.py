@@ -72,6 +72,8 @@ _PROTOS = {
     "pa_set_update_kernel": (C.c_int, [VP, C.c_int]),
     "pa_set_cache_precision": (C.c_int, [VP, C.c_int]),
     "pa_anderson_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int, C.c_int64, C.c_int]),
+    "pa_set_cache_adaptation": (C.c_int, [VP, C.c_double, C.c_double, C.c_double, C.c_double]),
+    "pa_cache_thresholds": (C.c_int, [VP, C.POINTER(C.c_double)]),
     "pa_set_anderson": (C.c_int, [VP, C.c_int, VP, C.c_size_t]),
     "pa_debug_set_wait_limit": (C.c_int, [VP, C.c_uint32]),
     "pa_set_kernel_timing": (C.c_int, [VP, C.c_int]),
@@ -219,7 +221,7 @@ def pa_stats(h):
     return s.as_dict()
 
 
-LOG_FIELDS = 8   # t, p, misses, stride, e, hits at positions >= 1, 0, 0
+LOG_FIELDS = 8   # t, p, misses, stride, e, hits at positions >= 1, positions with an entry, hits among them
 
 
 def pa_iter_log(h, max_iters, batch):
@@ -245,6 +247,17 @@ def pa_set_update_kernel(h, kind):
 
 def pa_set_cache_precision(h, bits):
     return _check("pa_set_cache_precision", lib().pa_set_cache_precision(h, int(bits)))
+
+
+def pa_set_cache_adaptation(h, rate, target, tau_min=0.0, tau_max=float("inf")):
+    return _check("pa_set_cache_adaptation", lib().pa_set_cache_adaptation(h, float(rate), float(target),
+                                                                             float(tau_min), float(tau_max)))
+
+
+def pa_cache_thresholds(h, batch):
+    buf = (C.c_double * batch)()
+    _check("pa_cache_thresholds", lib().pa_cache_thresholds(h, buf))
+    return [buf[b] for b in range(batch)]
 
 
 def pa_anderson_workspace_bytes(T, window, D, batch):

@@ -33,8 +33,9 @@ __global__ void k_init_plan(Dev d) {
   const int p0 = min(d.P, d.T);
   for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
     Traj tr{};
-    tr.t = 0; tr.p = p0; tr.e = 0; tr.done = 0; tr.m = p0; tr.h1 = 0;
+    tr.t = 0; tr.p = p0; tr.e = 0; tr.done = 0; tr.m = p0; tr.h1 = 0;  // no entries yet: ne = nh = 0
     d.traj[b] = tr;  // copy 0: the plan of iteration 0
+    if (d.adapt) d.tau[b] = d.cache_thresh;  // tau_cache starts at the configured value
   }
   for (int q = threadIdx.x; q < d.B * d.P; q += blockDim.x) {
     const int b = q / d.P, j = q % d.P;

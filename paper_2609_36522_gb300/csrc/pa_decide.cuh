@@ -15,6 +15,10 @@ struct DecideShared {
   int tn[kMaxBatch], pn[kMaxBatch], en[kMaxBatch], m[kMaxBatch], h1[kMaxBatch];
   int om[kMaxBatch], oh1[kMaxBatch];
   int stride[kMaxBatch], nh[kMaxBatch];  // decide_par: window advance and next-window positions with an entry
+  int one[kMaxBatch], onh[kMaxBatch];    // the planned iteration's positions with an entry, and hits among them
+  double tau[kMaxBatch];                 // tau_cache per trajectory: of the planned iteration, then of the next
+  double thr[kMaxBatch];                 // the next hit test's bound on the undivided sums, tau * D
+  double del[32 * 32];                   // with adaptation: the Eq. 4 sums themselves
   int warp_tot[32];
   unsigned cmiss[32], cwin[32];  // decide_par: miss / in-window bits of each 32-position chunk
   unsigned conv[32], near[32];   // decide_par's inputs as bits: Eq. 2 error <= tol, Eq. 4 distance < tau_cache
@@ -46,8 +50,10 @@ __device__ void decide_load(const Dev& d, DecideShared& sh, int par) {
     const Traj tr = tr0[b];
     sh.t[b] = tr.t; sh.p[b] = tr.p; sh.e[b] = tr.e;
     sh.om[b] = tr.m; sh.oh1[b] = tr.h1;
+    sh.one[b] = tr.ne; sh.onh[b] = tr.nh;
     sh.m[b] = 0;
     sh.h1[b] = 0;
+    sh.tau[b] = d.adapt ? d.tau[par * d.B + b] : d.cache_thresh;
   }
 }
 
@@ -255,11 +261,14 @@ __device__ __forceinline__ unsigned bits32(const unsigned* w, int pos) {
 // t_b + j + 1 is < tau_cache). Warp 0 alone takes it with bit operations:
 //  1. lane b advances trajectory b: stride = min(p, 1 + leading ones of its
 //     conv bits), t' = t + stride, p' = min(P, T - t'), frontier e' = t + p;
-//  2. lane c builds 32-position word c of the next windows' bits: position
-//     j' of trajectory b (timestep i = t' + j') is in the window for j' < p';
+//     with adaptation on, lane b also forms trajectory b's tau_cache for the
+//     next hit test from the planned iteration's hit rate and the stride;
+//  2. the next windows' bits, one ballot per 32-position chunk: position j'
+//     of trajectory b (timestep i = t' + j') is in the window for j' < p';
 //     it has an entry iff i < t + p, i.e. j' < p - stride, and then hits iff
-//     near bit j' + stride - 1 (where its distance was computed) is set
-//     (Eq. 5, strict); all other window positions miss;
+//     the distance computed at position j' + stride - 1 is below tau_cache
+//     (Eq. 5, strict; the near bit, or the sum against tau * D when tau
+//     adapts); all other window positions miss;
 //  3. lane c turns the miss counts of 32-position chunk c into its first rank
 //     (an exclusive scan): misses are ranked trajectory-major, ascending t.
 // Then, after one CTA barrier, every warp handles chunks: the ranks and the
@@ -278,7 +287,10 @@ __device__ inline void decide_par(const Dev& d, DecideShared& sh, int par, int p
     if (warp == 0) {
       if (pub_id == 0) {
         const Traj* in_traj = d.traj + par * B;
-        for (int b = lane; b < B; b += 32) out_traj[b] = in_traj[b];
+        for (int b = lane; b < B; b += 32) {
+          out_traj[b] = in_traj[b];
+          if (d.adapt) d.tau[(par ^ 1) * B + b] = d.tau[par * B + b];
+        }
         if (lane == 0) d.pc[par ^ 1] = d.pc[par];
       }
       for (int b = lane; b < B; b += 32) sh.en[b] = sh.e[b];
@@ -306,11 +318,29 @@ __device__ inline void decide_par(const Dev& d, DecideShared& sh, int par, int p
       sh.en[b] = p > 0 ? t + p : sh.e[b];
       sh.stride[b] = stride;
       sh.nh[b] = p > 0 ? p - stride : 0;  // next-window positions with a cache entry
+      if (d.adapt) {
+        // tau_cache of the next hit test, from the planned iteration's hit
+        // rate among positions with an entry and its stride: below the
+        // target rate tau rises by (1 + rate) if the window advanced beyond
+        // its first position, else holds; at or above it falls by (1 + rate);
+        // kept within [tau_min, tau_max]; no entries: tau holds
+        double tau = sh.tau[b];
+        const int ne = sh.one[b], nh = sh.onh[b];
+        if (p > 0 && ne > 0) {
+          if ((double)nh / (double)ne < d.adapt_target) {
+            if (stride > 1) tau = fmin(tau * d.adapt_up, d.tau_max);
+          } else {
+            tau = fmax(tau / d.adapt_up, d.tau_min);
+          }
+        }
+        sh.tau[b] = tau;
+        sh.thr[b] = tau * (double)d.D;
+      }
       if (pub_id == 0) {
         int32_t* lg = d.iter_log + ((int64_t)iter * B + b) * kLogFields;
         if (p > 0) {
           lg[0] = t; lg[1] = p; lg[2] = sh.om[b]; lg[3] = stride;
-          lg[4] = sh.e[b]; lg[5] = sh.oh1[b]; lg[6] = 0; lg[7] = 0;
+          lg[4] = sh.e[b]; lg[5] = sh.oh1[b]; lg[6] = sh.one[b]; lg[7] = sh.onh[b];
         } else {
           for (int f = 0; f < kLogFields; ++f) lg[f] = 0;
           lg[0] = t;
@@ -318,26 +348,30 @@ __device__ inline void decide_par(const Dev& d, DecideShared& sh, int par, int p
       }
     }
     __syncwarp();
-    // lane c builds word c of the next windows' bits from the trajectories
-    // that overlap positions [32c, 32c + 32)
-    if (lane < nchunk) {
-      const int lo = lane * 32, hi = min(lo + 32, N);
-      unsigned win = 0u, miss = 0u;
-      for (int b = lo / P; b * P < hi; ++b) {
-        const int base = b * P;
-        const int w0 = max(lo, base), w1 = min(hi, base + sh.pn[b]);
-        if (w1 <= w0) continue;
-        const unsigned wm = (w1 - w0 == 32 ? 0xffffffffu : ((1u << (w1 - w0)) - 1u)) << (w0 - lo);
-        unsigned hm = 0u;
-        const int h1 = min(hi, base + sh.nh[b]);
-        if (h1 > w0)  // near bit of position q sits at q + stride - 1
-          hm = bits32(sh.near, lo + sh.stride[b] - 1) &
-               ((h1 - w0 == 32 ? 0xffffffffu : ((1u << (h1 - w0)) - 1u)) << (w0 - lo));
-        win |= wm;
-        miss |= wm & ~hm;
+    // the next windows' bits, one 32-position chunk per ballot: position j'
+    // of trajectory b is in the window for j' < p', has an entry for
+    // j' < nh (= p - stride) and then hits iff the Eq. 4 distance computed at
+    // position j' + stride - 1 is below the bound (Eq. 5, strict)
+    for (int c = 0; c < nchunk; ++c) {
+      const int q = c * 32 + lane;
+      bool win = false, miss = false;
+      if (q < N) {
+        const int b = q / P, jn = q - b * P;
+        if (jn < sh.pn[b]) {
+          win = true;
+          bool hit = false;
+          if (jn < sh.nh[b]) {
+            const int qo = b * P + jn + sh.stride[b] - 1;
+            hit = d.adapt ? sum_lt(sh.del[qo], sh.thr[b]) : ((sh.near[qo >> 5] >> (qo & 31)) & 1u);
+          }
+          miss = !hit;
+        }
       }
-      sh.cwin[lane] = win;
-      sh.cmiss[lane] = miss;
+      const unsigned wm = __ballot_sync(0xffffffffu, win), mm = __ballot_sync(0xffffffffu, miss);
+      if (lane == 0) {
+        sh.cwin[c] = wm;
+        sh.cmiss[c] = mm;
+      }
     }
     __syncwarp();
     const int cnt = lane < nchunk ? __popc(sh.cmiss[lane]) : 0;
@@ -389,6 +423,9 @@ __device__ inline void decide_par(const Dev& d, DecideShared& sh, int par, int p
       tr.done = (sh.pn[b] == 0);
       tr.m = range_popc(sh.cmiss, b * P, b * P + sh.pn[b]);
       tr.h1 = sh.pn[b] > 1 ? (sh.pn[b] - 1) - range_popc(sh.cmiss, b * P + 1, b * P + sh.pn[b]) : 0;
+      tr.ne = sh.nh[b];
+      tr.nh = sh.nh[b] - range_popc(sh.cmiss, b * P, b * P + sh.nh[b]);
+      if (d.adapt) d.tau[(par ^ 1) * B + b] = sh.tau[b];
       if (tr.t > T || tr.e < tr.t) atomicCAS(&d.ctl->status, kDevOk, kDevBadState);
       out_traj[b] = tr;
     }
@@ -433,6 +470,7 @@ __device__ __forceinline__ void stage_decision_bits(const Dev& d, DecideShared& 
       const double se = __ldcg(acc_e + o), sd = __ldcg(acc_d + o);
       cv = sum_le(se, d.tol_d);
       nr = sum_lt(sd, d.thr_d);
+      if (d.adapt) sh.del[q] = sd;  // the bound is known only once the windows have advanced
       if (pub_id >= 0 && q % pub_count == pub_id) {
         d.red_err[q] = (float)(se * d.inv_d);
         d.red_del[q] = (float)(sd * d.inv_d);

@@ -34,10 +34,12 @@ constexpr int kDevBadState = 3;     // trajectory bookkeeping inconsistent
 //  m : misses of trajectory b in the planned iteration (for the iteration log)
 //  h1: hits among window positions 1..p-1 of the planned iteration (their xhat
 //      rows are read for the next iteration's distances; for the byte count)
+//  ne: window positions of the planned iteration that have a cache entry
+//  nh: hits among them (the adaptation of tau_cache reads ne and nh)
 struct Traj {
-  int32_t t, p, e, done, m, h1, pad0, pad1;
+  int32_t t, p, e, done, m, h1, ne, nh;
 };
-constexpr int kLogFields = 8;  // iteration log entry: t, p, misses, stride, e, h1, 0, 0
+constexpr int kLogFields = 8;  // iteration log entry: t, p, misses, stride, e, h1, ne, nh
 
 // Counters read by the host (one copy, written by whichever kernel publishes
 // a plan) and by the denoiser (n_miss, through its device pointer).
@@ -61,7 +63,7 @@ struct PlanCtr {
 
 struct Layout {
   size_t X, Xhat, Ehat, batch_x, coef, traj, pc, ctl, rank, miss_bt;
-  size_t acc, red_err, red_del, iter_log, gbar, total;
+  size_t acc, red_err, red_del, iter_log, gbar, tau, total;
 };
 
 inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
@@ -86,6 +88,7 @@ inline Layout make_layout(int T, int P, int64_t D, int B) {
   L.red_del = take((size_t)B * P * sizeof(float));
   L.iter_log = take((size_t)(T + 1) * B * kLogFields * sizeof(int32_t));
   L.gbar = take(128);                              // arrival counter of the fused step's grid barrier
+  L.tau = take((size_t)2 * B * sizeof(double));    // tau_cache per trajectory, by plan parity
   L.total = o;
   return L;
 }
@@ -119,6 +122,12 @@ struct Dev {
   float* taa_r;
   double* taa_acc;
   int taa;            // 1: iterations mix (depth 1); 0: plain Picard
+  // Online adaptation of tau_cache (pa_set_cache_adaptation): tau of every
+  // trajectory, [2][B] by plan parity (copy k mod 2 is the tau of iteration
+  // k's hit test); adapt = 0 keeps tau_cache fixed (thr_d is then used).
+  double* tau;
+  int adapt;
+  double adapt_up, adapt_target, tau_min, tau_max;
   int T, P, B;
   int64_t D;
   double tol, cache_thresh;   // tau of Eq. 2 and tau_cache of Eq. 5

@@ -218,6 +218,12 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.taa_r = nullptr;
   d.taa_acc = nullptr;
   d.taa = 0;
+  d.tau = reinterpret_cast<double*>(w + L.tau);
+  d.adapt = 0;
+  d.adapt_up = 1.0;
+  d.adapt_target = 0.0;
+  d.tau_min = 0.0;
+  d.tau_max = 0.0;
   d.T = T; d.P = P; d.B = batch; d.D = D;
   d.tol = tol;
   d.cache_thresh = cache_thresh;
@@ -498,6 +504,39 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
     return arg_fail("pa_set_update_kernel: kind must be 0, 1, 2, 3, 100 + bulk launch shape, "
                     "200 + lean launch shape or 300 + fused-step launch shape");
   }
+  return PA_OK;
+}
+
+pa_status pa_set_cache_adaptation(pa_solver* s, double rate, double target, double tau_min, double tau_max) {
+  if (!s) return arg_fail("pa_set_cache_adaptation: solver is NULL");
+  if (s->state == St::Stepped) return state_fail("pa_set_cache_adaptation");
+  if (!(rate >= 0.0) || !std::isfinite(rate) || !(target >= 0.0 && target <= 1.0) || !(tau_min >= 0.0) ||
+      !std::isfinite(tau_min) || std::isnan(tau_max) || !(tau_max >= tau_min))
+    return arg_fail("pa_set_cache_adaptation: need rate >= 0, 0 <= target <= 1, 0 <= tau_min <= tau_max");
+  pa::Dev& d = s->d;
+  if (rate > 0.0 && d.B * d.P > 32 * 32)
+    return arg_fail("pa_set_cache_adaptation: batch * window must be at most 1024");
+  d.adapt = rate > 0.0 ? 1 : 0;
+  d.adapt_up = 1.0 + rate;
+  d.adapt_target = target;
+  d.tau_min = tau_min;
+  d.tau_max = tau_max;
+  s->state = St::Created;  // pa_init restarts from tau_cache
+  return PA_OK;
+}
+
+pa_status pa_cache_thresholds(pa_solver* s, double* tau_out) {
+  if (!s || !tau_out) return arg_fail("pa_cache_thresholds: NULL argument");
+  if (s->state == St::Created) return state_fail("pa_cache_thresholds");
+  const pa::Dev& d = s->d;
+  if (!d.adapt) {
+    for (int b = 0; b < d.B; ++b) tau_out[b] = d.cache_thresh;
+    return PA_OK;
+  }
+  cudaError_t e = cudaMemcpyAsync(tau_out, d.tau + (s->k & 1) * d.B, (size_t)d.B * sizeof(double),
+                                  cudaMemcpyDeviceToHost, s->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_cache_thresholds", e);
   return PA_OK;
 }
 

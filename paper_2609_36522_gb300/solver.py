@@ -173,6 +173,15 @@ class Solver:
         self._drop_graphs()
         abi.pa_set_update_kernel(self.h, kind)
 
+    def set_cache_adaptation(self, rate, target, tau_min=0.0, tau_max=float("inf")):
+        """Online adaptation of tau_cache per trajectory (rate 0: off); pa_init must follow."""
+        self._drop_graphs()
+        abi.pa_set_cache_adaptation(self.h, rate, target, tau_min, tau_max)
+
+    def cache_thresholds(self):
+        """tau_cache of the planned iteration's hit test, per trajectory."""
+        return abi.pa_cache_thresholds(self.h, self.batch)
+
     def set_anderson(self, depth):
         """Triangular Anderson mixing of the iterates (ParaTAA-style update):
         depth 1 mixes with the previous iteration (its workspace is allocated

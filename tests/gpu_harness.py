@@ -7,21 +7,25 @@ import numpy as np
 import workload as W
 from oracle import run_picard
 from oracle.gmm import make_eps_fn, gmm_eps
+from oracle.picard import CacheAdaptation
 from oracle.taa import run_taa
 
 
-def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True, cache_store=None, anderson=0):
+def oracle_run(w: W.Workload, cache_thresh=None, use_cache=True, cache_store=None, anderson=0, adapt=None):
+    """adapt: None or (rate, target, tau_min, tau_max) of the tau_cache adaptation."""
     a, x0, mu = W.inputs(w)
     thr = w.cache_thresh if cache_thresh is None else cache_thresh
+    ad = None if adapt is None else CacheAdaptation(*adapt)
     if anderson:
         return run_taa(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr, depth=anderson,
-                       use_cache=use_cache, eta=w.eta, noise=W.noise(w))
+                       use_cache=use_cache, eta=w.eta, noise=W.noise(w), adapt=ad)
     return run_picard(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr,
-                      use_cache=use_cache, eta=w.eta, noise=W.noise(w), cache_store=cache_store)
+                      use_cache=use_cache, eta=w.eta, noise=W.noise(w), cache_store=cache_store, adapt=ad)
 
 
 def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=None,
-            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None, reductions=False, anderson=None):
+            mode="sync", x_init_host=False, gmm_form=None, cache_bits=None, reductions=False, anderson=None,
+            adapt=None):
     """Run one generation on the GPU.
 
     eps_source: "gmm" (the CUDA mixture kernel) or "oracle" (fp64 mixture
@@ -29,6 +33,8 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
     mode: "sync" (pa_step) or "async" (pa_step_async, device-side counts).
     reductions: keep every iteration's Eq. 2 / Eq. 4 reductions (sync mode).
     anderson: history depth of the triangular Anderson mixing (None: not set).
+    adapt: None or (rate, target, tau_min, tau_max): tau_cache adapted online;
+    every planned iteration's tau_cache per trajectory is kept (sync mode).
     """
     import torch
     from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
@@ -43,6 +49,8 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
         s.set_cache_precision(cache_bits)
     if anderson is not None:
         s.set_anderson(anderson)
+    if adapt is not None:
+        s.set_cache_adaptation(*adapt)
     max_rows = w.batch * s.window
     means = torch.from_numpy(mu).to(dev)
     g = GmmDenoiser(means, w.gmm_std, a, max_rows)
@@ -64,11 +72,14 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
     misses = []
     batches = []
     reds = []
+    taus = []
     if mode == "sync":
         while True:
             out = s.step()
             if out is None:
                 break
+            if adapt is not None:
+                taus.append(s.cache_thresholds())
             n, bx, mb = out.n_miss, out.batch_x, out.miss_bt
             mbh = mb.cpu().numpy().copy()
             misses.append([tuple(int(v) for v in row) for row in mbh])
@@ -92,7 +103,7 @@ def gpu_run(w: W.Workload, cache_thresh=None, eps_source="gmm", update_kernel=No
         s.poll()
     xT = s.result().cpu().numpy()
     res = dict(x_final=xT, nfe=s.nfe(), stats=s.stats(), log=s.iter_log(), misses=misses,
-               batches=batches, gmm_launches=g.launches(), reductions=reds)
+               batches=batches, gmm_launches=g.launches(), reductions=reds, taus=taus)
     s.close()
     g.close()
     return res

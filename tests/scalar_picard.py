@@ -52,11 +52,17 @@ def _eps(x, a, means, std):
     return out
 
 
-def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh, noise=None):
+def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh, noise=None, adapt=None, taus=None):
     """Returns (final states per trajectory, per-iteration (misses, strides, distances)).
 
     noise: None for DDIM; else the draws noise[b][i] of every trajectory and
-    step, and every step is an ancestral DDPM step (eta = 1)."""
+    step, and every step is an ancestral DDPM step (eta = 1).
+    adapt: None, or (rate, target, lo, hi): each trajectory's threshold moves
+    after every iteration -- up by the factor 1 + rate when fewer than
+    target of its points with an entry hit and its window moved by more than
+    one point, down by that factor when at least target of them hit, never
+    outside [lo, hi], unchanged when no point had an entry. taus, if a list,
+    receives every iteration's thresholds."""
     T = len(alphas) - 1
     B = len(x_init)
     D = len(x_init[0])
@@ -69,7 +75,10 @@ def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh, noise=None)
     cache = [dict() for _ in range(B)]          # i -> (xhat, ehat)
     start = [0] * B
     log = []
+    thr_b = [thresh] * B
     while any(s < T for s in start):
+        if taus is not None:
+            taus.append(list(thr_b))
         # decide hits and misses, trajectory by trajectory, point by point
         plan = []
         misses = []
@@ -89,7 +98,7 @@ def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh, noise=None)
                 if i in cache[b]:
                     xh = cache[b][i][0]
                     dist = sum(abs(u - w) for u, w in zip(states[b][i], xh)) / D
-                    hit = dist < thresh
+                    hit = dist < thr_b[b]
                 row.append(hit)
                 drow.append(dist)
                 if not hit:
@@ -142,6 +151,16 @@ def scalar_cached_picard(alphas, x_init, means, std, P, tol, thresh, noise=None)
                 states[b][i] = list(states[b][t + p])
             start[b] = nt
             strides.append(stride)
+            if adapt is not None:
+                rate, target, lo, hi = adapt
+                had = [dv for dv in dists[b] if dv is not None]
+                if had:
+                    n_hit = sum(1 for h in plan[b] if h)
+                    if n_hit / len(had) < target:
+                        if stride > 1:
+                            thr_b[b] = min(thr_b[b] * (1.0 + rate), hi)
+                    else:
+                        thr_b[b] = max(thr_b[b] / (1.0 + rate), lo)
         log.append((misses, strides, dists))
     finals = [states[b][T] for b in range(B)]
     return finals, log

@@ -699,3 +699,57 @@ def test_anderson_graph_replay_equals_sync():
             assert np.array_equal(s.iter_log(), sync["log"])
     s.close()
     g.close()
+
+
+# ---- online adaptation of tau_cache (pa_set_cache_adaptation) -----------------
+
+ADAPT_CASES = [
+    (W.SD15.with_(cache_thresh=0.02, name="SD tau0 0.02"), (0.5, 0.5, 0.0, 0.2), {}),
+    (W.SD15.with_(cache_thresh=0.1, name="SD tau0 0.1"), (0.5, 0.3, 0.01, 0.2), {}),
+    (W.BATCHED.with_(T=60, cache_thresh=0.05), (1.0, 0.6, 0.0, 1.0), {}),
+    (W.TINY, (1.0, 0.9, 0.0, 1.0), {}),
+    (W.SD15.with_(cache_thresh=0.02, name="SD fused"), (0.5, 0.5, 0.0, 0.2), {"update_kernel": 3}),
+    (W.SD15.with_(cache_thresh=0.02, name="SD anderson"), (0.5, 0.5, 0.0, 0.2), {"anderson": 1}),
+]
+
+
+@pytest.mark.parametrize("w,adapt,kw", ADAPT_CASES, ids=lambda v: v.name if isinstance(v, W.Workload) else "")
+def test_cache_adaptation_against_oracle(w, adapt, kw):
+    """tau_cache adapted online on the device: the same tau per trajectory and
+    iteration as the oracle (fp64, bit for bit), the same decisions, miss lists,
+    NFE and hits; final latents within 1e-5. Also through the fused step and
+    with Anderson mixing."""
+    orc = oracle_run(w, adapt=adapt, anderson=kw.get("anderson", 0))
+    assert margins_ok(orc, w.tol, w.cache_thresh, rel=1e-6), decision_margins(orc, w.tol, w.cache_thresh)
+    gpu = gpu_run(w, adapt=adapt, **kw)
+    rel = compare(w, orc, gpu)
+    assert rel.max() <= REL_TOL, rel
+    assert [r.tau for r in orc.records] == gpu["taus"]
+    assert len({t for r in orc.records for t in r.tau}) > 1   # tau did move
+
+
+def test_cache_adaptation_rate_zero_is_fixed():
+    """Rate 0 (adaptation off) gives the fixed-threshold run bit for bit."""
+    w = W.SD15
+    fixed = gpu_run(w)
+    off = gpu_run(w, adapt=(0.0, 0.5, 0.0, 1.0))
+    assert np.array_equal(fixed["x_final"], off["x_final"])
+    assert np.array_equal(fixed["log"], off["log"])
+    assert all(t == [w.cache_thresh] for t in off["taus"])
+
+
+def test_cache_adaptation_rejects_bad_arguments():
+    from paper_2609_36522_gb300 import abi
+    from paper_2609_36522_gb300.solver import Solver
+    w = W.TINY
+    s = Solver(w.T, w.window, w.latent_shape, W.alphas_cumprod(w.T), w.tol, w.cache_thresh)
+    for args in ((-0.1, 0.5, 0.0, 1.0), (0.5, 1.5, 0.0, 1.0), (0.5, 0.5, 0.2, 0.1), (float("nan"), 0.5, 0.0, 1.0)):
+        with pytest.raises(abi.PaError) as e:
+            s.set_cache_adaptation(*args)
+        assert e.value.status == abi.PA_ERR_ARG
+    s.close()
+    big = Solver(200, 128, (4, 4, 4), W.alphas_cumprod(200), 1e-3, 0.05, batch=9)
+    with pytest.raises(abi.PaError) as e:
+        big.set_cache_adaptation(0.5, 0.5)
+    assert e.value.status == abi.PA_ERR_ARG
+    big.close()

@@ -171,3 +171,64 @@ def test_guard_reports_margins():
     assert 0 < md < np.inf and 0 < me < np.inf
     assert margins_ok(r, w.tol, w.cache_thresh)
     assert not margins_ok(r, w.tol, w.cache_thresh, rel=1.0)
+
+
+# ---- online adaptation of tau_cache (CacheAdaptation) -----------------------
+
+from oracle.picard import CacheAdaptation  # noqa: E402
+
+ADAPT_W = W.Workload("adapt", T=40, window=16, batch=2, latent_shape=(2, 4, 4), K=3, tol=1e-3,
+                     cache_thresh=0.02, seed=6)
+
+
+def _adapt_run(w, adapt, thr=None):
+    a, x0, mu = W.inputs(w)
+    return run_picard(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol,
+                      w.cache_thresh if thr is None else thr, adapt=adapt)
+
+
+def test_adaptation_with_rate_zero_is_fixed_tau():
+    fixed = _adapt_run(ADAPT_W, None)
+    off = _adapt_run(ADAPT_W, CacheAdaptation(rate=0.0, target=0.5))
+    assert np.array_equal(fixed.states, off.states)
+    assert [r.miss_bt for r in fixed.records] == [r.miss_bt for r in off.records]
+    assert all(t == ADAPT_W.cache_thresh for r in off.records for t in r.tau)
+
+
+def test_adaptation_limits():
+    """tau_cache 0 stays 0 (uncached); a floor of +inf-like size hits every
+    point with an entry (NFE = B * T); tau never leaves [tau_min, tau_max]."""
+    zero = _adapt_run(ADAPT_W, CacheAdaptation(rate=0.5, target=1.0), thr=0.0)
+    assert zero.hits == 0 and all(t == 0.0 for r in zero.records for t in r.tau)
+    always = _adapt_run(ADAPT_W, CacheAdaptation(rate=0.5, target=0.0, tau_min=1e30), thr=1e30)
+    assert always.nfe == ADAPT_W.batch * ADAPT_W.T
+    bounded = _adapt_run(ADAPT_W, CacheAdaptation(rate=0.5, target=0.9, tau_min=0.01, tau_max=0.04))
+    taus = [t for r in bounded.records for t in r.tau]
+    assert min(taus[ADAPT_W.batch:]) >= 0.01 and max(taus) <= 0.04
+    assert len(set(taus)) > 1   # it did move
+
+
+def test_adaptation_raises_reuse_toward_the_target():
+    """Starting where the fixed threshold gives no hits, a high target raises
+    tau and the run reuses more cache entries than the fixed run."""
+    fixed = _adapt_run(ADAPT_W, None, thr=0.005)
+    adapt = _adapt_run(ADAPT_W, CacheAdaptation(rate=1.0, target=0.9), thr=0.005)
+    assert adapt.hits > fixed.hits
+
+
+@pytest.mark.parametrize("rate,target,lo,hi,thr,seed", [(0.5, 0.8, 0.0, 1.0, 0.02, 0), (1.0, 0.3, 0.005, 0.2, 0.05, 1),
+                                                        (0.25, 1.0, 0.0, 0.5, 0.01, 2)])
+def test_adaptation_scalar_second_implementation_agrees(rate, target, lo, hi, thr, seed):
+    w = W.Workload("adapt scalar", T=8, window=4, batch=2, latent_shape=(1, 2, 3), K=3, tol=1e-3,
+                   cache_thresh=thr, seed=seed)
+    a, x0, mu = W.inputs(w)
+    r = run_picard(a, x0, make_eps_fn(a, mu, w.gmm_std), w.window, w.tol, thr,
+                   adapt=CacheAdaptation(rate=rate, target=target, tau_min=lo, tau_max=hi))
+    taus = []
+    finals, log = scalar_cached_picard(list(a), x0.astype(np.float64).tolist(), mu.astype(np.float64).tolist(),
+                                       0.5, w.window, w.tol, thr, adapt=(rate, target, lo, hi), taus=taus)
+    assert len(log) == r.iters
+    for rec, (misses, strides, _), tk in zip(r.records, log, taus):
+        assert rec.miss_bt == misses and rec.stride == strides
+        assert rec.tau == tk
+    assert np.abs(np.array(finals) - r.x_final).max() <= 1e-12 * np.abs(r.x_final).max()

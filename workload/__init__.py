@@ -85,6 +85,11 @@ SRDS_BATCHED = BATCHED.with_(name="SRDS T100 B8 4x64x64 K16", sampler="srds")
 # Triangular Anderson mixing (a ParaTAA-style update) on the SD-shaped and batched inputs.
 SD15_TAA = SD15.with_(name="SD-v1.5-shaped T100 P100 B1 4x64x64 K16 TAA", sampler="taa")
 BATCHED_TAA = BATCHED.with_(name="batched T100 P32 B8 4x64x64 K16 TAA", sampler="taa")
+# Online adaptation of tau_cache on the SD-shaped inputs: tau starts at 0.02 and
+# tracks a 50 % hit rate among points with an entry, by factors of 1.5, within
+# [0, 0.2] (extra["adapt"] = (rate, target, tau_min, tau_max)).
+SD15_ADAPT = SD15.with_(name="SD-v1.5-shaped T100 P100 B1 4x64x64 K16 adaptive tau_cache",
+                        cache_thresh=0.02, extra={"adapt": (0.5, 0.5, 0.0, 0.2)})
 SWEEP_THRESHOLDS = (0.0, 0.01, 0.02, 0.05, 0.1)
 
 
@@ -95,7 +100,7 @@ def sweep(base: Workload = SD15):
 
 
 ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM,
-       "srds": SRDS, "srds_batched": SRDS_BATCHED, "sd15_taa": SD15_TAA, "batched_taa": BATCHED_TAA}
+       "srds": SRDS, "srds_batched": SRDS_BATCHED, "sd15_taa": SD15_TAA, "batched_taa": BATCHED_TAA, "sd15_adapt": SD15_ADAPT}
 
 
 def train_alphas_cumprod() -> np.ndarray:
