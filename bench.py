@@ -54,6 +54,10 @@ METRIC = "Picard+cache solver steps/s and HBM GB/s vs peak at T=100, 4x64x64; NF
 UNIT = "solver steps/s"
 FLUSH_BYTES = 256 << 20
 E2E_CHUNK = 4      # Picard iterations issued between two pa_poll calls in the end-to-end run
+GMM_FORMS = {2: "one kernel: clusters of 16 CTAs per 8 rows, CUDA-core dot products summed through "
+                "distributed shared memory",
+             1: "tensor-core dot products (tcgen05 kind::tf32, split operands) + output kernel",
+             0: "CUDA-core dot products (fp32 FMA) + output kernel"}
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
@@ -78,7 +82,8 @@ def parse_args(argv=None):
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--update-kernel", type=int, default=None)
-    ap.add_argument("--gmm-form", type=int, default=None, help="denoiser dot products: 1 tensor cores, 0 CUDA cores")
+    ap.add_argument("--gmm-form", type=int, default=None,
+                    help="denoiser: 2 one cluster kernel, 1 tensor-core dots + output kernel, 0 CUDA-core dots + output kernel")
     ap.add_argument("--cache-thresh", type=float, default=None,
                     help="override the workload's tau_cache (the threshold sweep)")
     ap.add_argument("--cache-bits", type=int, default=32, choices=[16, 32],
@@ -448,15 +453,21 @@ def run_ours(args):
         g.eps(bx, mb, nm, eps)
         sv.submit_eps(eps)
 
-    def run_sync(sv, record=None):
+    def run_sync(sv, record=None, record_in=None):
         """One generation through the synchronous API; -> iterations. With a
-        list in `record`, the denoiser's eps rows of every iteration are kept."""
+        list in `record`, the denoiser's eps rows of every iteration are kept;
+        with a list in `record_in`, its inputs (batch rows, miss list, count)."""
         sv.init(x_dev)
         n = 0
         while True:
             out = sv.step()
             if out is None:
                 return n
+            if record_in is not None:
+                m = max(out.n_miss, 1)
+                record_in.append((out.batch_x[:out.n_miss].clone() if out.n_miss else torch.zeros(1, w.D, device=dev),
+                                  out.miss_bt[:out.n_miss].clone() if out.n_miss else torch.zeros(1, 2, dtype=torch.int32, device=dev),
+                                  torch.tensor([out.n_miss], dtype=torch.int32, device=dev), m))
             g.eps(out.batch_x_ptr, out.miss_bt_ptr, sv.n_miss_dev(), eps)
             if record is not None:
                 record.append(eps[: max(out.n_miss, 1)].clone())
@@ -465,8 +476,8 @@ def run_ours(args):
 
     # learn the iteration count with the synchronous API (also a warm-up),
     # keeping the eps rows for the solver-only graph
-    eps_rec = []
-    n_iters = run_sync(s, eps_rec)
+    eps_rec, den_in = [], []
+    n_iters = run_sync(s, eps_rec, den_in)
     st0 = s.stats()
     log = s.iter_log()
     nfe, hits = st0["nfe"], st0["hits"]
@@ -680,6 +691,30 @@ def run_ours(args):
                                  "stored figure from an earlier capture of this command, keyed by the kernel "
                                  "sources' hash (null: not captured for these sources)")}
 
+    # ---- the denoiser alone -----------------------------------------------
+    # Its calls of the same generation on the recorded batches (rows, miss
+    # list, count), each followed by pa_debug_gap as the solver step's stand-in,
+    # as one graph; events around it, L2 flushed before each replay.
+    g_den = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_den, stream=stream):
+        for bx_k, mb_k, nm_k, _ in den_in:
+            g.eps(bx_k.data_ptr(), mb_k.data_ptr(), nm_k.data_ptr(), eps)
+            abi.pa_debug_gap(s.stream_ptr)
+    den_only = 0.0
+    den_reps = max(10, min(args.steps * 5, 200))
+    for r in range(den_reps + 3):
+        if flush is not None:
+            flush.zero_()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        g_den.replay()
+        e1.record(stream)
+        e1.synchronize()
+        if r >= 3:
+            den_only += e0.elapsed_time(e1)
+    den_only_us = 1000.0 * den_only / (den_reps * n_iters)
+    del g_den
+
     # ---- uncached run alongside (tau_cache = 0: every window point evaluated)
     su = make_solver(0.0)
     un_iters = run_sync(su)
@@ -811,8 +846,7 @@ def run_ours(args):
             "method": {"cache_entries": "bf16" if args.cache_bits == 16 else "fp32",
                        "solver_step_kernels": step_kernel,
                        "kernels_per_iteration": kernels_per_iter,
-                       "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
-                                                 if g.form() == 1 else "CUDA cores (fp32 FMA)"),
+                       "denoiser": GMM_FORMS.get(g.form(), "?"),
                        "parallelism": f"replicas x{world} (independent trajectories)"},
             "timing": {"l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every generation (between timed steps), outside the "
@@ -825,9 +859,10 @@ def run_ours(args):
             "deviation_from_serial_ddim": deviation,
             "solver_step": solver_step,
             "uncached": uncached,
-            "denoiser_us_per_iteration": 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
-            "denoiser_note": ("CUDA events around each denoiser call in the timed graph (its event nodes cut "
-                              "the dependent-launch overlap there, so it is an upper bound)"),
+            "denoiser_us_per_iteration": den_only_us,
+            "denoiser_note": ("the denoiser alone: a graph of its calls on the generation's recorded batches, "
+                              "each followed by pa_debug_gap, events around the graph, L2 flushed per replay"),
+            "denoiser_event_timed_us": 1000.0 * den_ms[0] / max(1, args.steps * n_iters),
             "denoiser_alg_bytes_per_iteration": float(den_bytes.mean()),
             "roofline": roofline,
             "cpu_baseline": cpu,
@@ -992,8 +1027,7 @@ def run_srds_bench(args, w):
                        "global_batch": w.batch * world, "seq_len": w.T,
                        "latent": "x".join(map(str, w.latent_shape)), "mixture_components": w.K,
                        "tol": w.tol, "cache_thresh": w.cache_thresh,
-                       "denoiser_dot_products": ("tensor cores (tcgen05 kind::tf32, split operands)"
-                                                 if g.form() == 1 else "CUDA cores (fp32 FMA)"),
+                       "denoiser": GMM_FORMS.get(g.form(), "?"),
                        "parallelism": f"replicas x{world} (independent trajectories)",
                        "l2": ("not flushed" if args.no_flush else
                               "256 MiB write before every generation (between timed steps), outside the "

@@ -451,20 +451,24 @@ PA_API pa_status pa_gmm_check(pa_gmm* g);
 /* Kernels launched by this handle since pa_gmm_create. */
 PA_API int64_t pa_gmm_launches(const pa_gmm* g);
 
-/* How pa_gmm_eps forms the dot products x . mu_k (a choice of this library;
- * the paper has no counterpart). form 1: on the tensor cores (tcgen05,
- * kind::tf32, every operand split into two tf32 parts and three products
- * summed, which keeps fp32 accuracy), 128 rows x 128 columns per CTA;
- * available when the GPU is of the sm_100 family, D % 4 == 0 and the means
- * are 16-byte aligned, and selected by pa_gmm_create when also K > 16.
- * form 0: fp32 FMA on the CUDA cores (the default for K <= 16, where the
- * contraction is too small for the tensor cores to pay off). A
- * call whose batch_x is not 16-byte aligned uses form 0. The forms agree to
- * fp32 rounding; each is bitwise reproducible. Returns PA_ERR_ARG for form 1
- * when it is not available. */
+/* How pa_gmm_eps computes (a choice of this library; the paper has no
+ * counterpart). form 2 (the default for K <= 16 when D is a multiple of 64):
+ * one kernel -- a thread-block cluster of 16 CTAs per block of 8 rows, each CTA
+ * one sixteenth of the columns; the partial dot products x . mu_k are summed
+ * across the cluster through distributed shared memory and every CTA writes
+ * its columns of eps from the row and mean tiles it staged once. form 1: the
+ * dot products on the tensor cores (tcgen05, kind::tf32, every operand split
+ * into two tf32 parts and three products summed, which keeps fp32 accuracy),
+ * 128 rows x 64 columns per CTA, then an output kernel; available when the GPU
+ * is of the sm_100 family, D % 4 == 0 and the means are 16-byte aligned, and
+ * the default when K > 16. form 0: fp32 FMA dot products on the CUDA cores,
+ * then the output kernel. A call whose batch_x or batch_eps is not 16-byte
+ * aligned uses form 0 (form 2 falls back to it). The forms agree to fp32
+ * rounding; each is bitwise reproducible. Returns PA_ERR_ARG for a form that
+ * is not available. */
 PA_API pa_status pa_gmm_set_form(pa_gmm* g, int form);
 
-/* The form pa_gmm_eps uses: 1 or 0, -1 for NULL. */
+/* The form pa_gmm_eps uses: 2, 1 or 0, -1 for NULL. */
 PA_API int pa_gmm_form(const pa_gmm* g);
 
 PA_API void pa_gmm_destroy(pa_gmm* g);

@@ -646,6 +646,221 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
   }
 }
 
+// ---------------------------------------------------------------------------
+// Single-kernel form for up to 16 components (form 2): a thread-block cluster
+// of CL CTAs takes a block of RB rows; CTA q of the cluster owns columns
+// [q * chunk, (q + 1) * chunk) with chunk = D / CL. Each CTA stages its chunk of
+// the means (before the dependency wait: the means do not change) and of the
+// rows, forms the rows' partial dot products x . mu_k over its columns in
+// registers (4 rows x 4 components per warp, packed fp32 pairs, 16-byte
+// shared loads), and the CL partials are summed through distributed shared
+// memory in rank order -- the same sums in every CTA of the cluster. Every CTA then
+// takes the logits and the max-subtracted softmax of the block's rows and
+// writes eps = a x - a sqrt(a) R M for its columns from the tiles it already
+// holds: no second kernel, no global accumulators, nothing read twice. The
+// cluster's barriers are hardware barriers; its CTAs are co-scheduled.
+constexpr int kClThreads = 256;
+constexpr int kClMaxK = 16;
+
+constexpr int kClCoefT = 2048;  // per-timestep scalars staged in shared memory up to this many timesteps
+
+template <int CL, int RB>
+struct ClShape {
+  static int ld(int chunk) { return chunk + 4; }  // padded row stride: the two half-warps' rows on other banks
+  static size_t coef_bytes(int T) { return T <= kClCoefT ? (size_t)3 * T * sizeof(float) : 0; }
+  static size_t smem_bytes(int chunk, int T) {
+    return (size_t)(kClMaxK + RB) * ld(chunk) * sizeof(float) + coef_bytes(T);
+  }
+};
+
+__device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+
+template <int CL, int RB>
+__global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restrict__ X, const float* __restrict__ mu,
+                                                            const float* __restrict__ coef, int T,
+                                                            const int32_t* __restrict__ miss_bt,
+                                                            const float* __restrict__ mnorm,
+                                                            const int32_t* __restrict__ n_rows_dev, int K, int64_t D,
+                                                            int chunk, int max_rows, float* __restrict__ eps,
+                                                            int32_t* status) {
+  static_assert(RB == 8 && kClThreads == 256, "8 warps: 2 row quads x 4 component quads of the 8 x 16 block");
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bar_m, bar_x;
+  __shared__ float s_part[RB * kClMaxK];   // this CTA's partial dot products (read by the cluster)
+  __shared__ float s_r[RB * kClMaxK];      // dot products [row][k], then logits
+  __shared__ __align__(16) float s_rt[kClMaxK * RB];  // responsibilities [k][row]
+  __shared__ float s_sa[RB], s_q[RB], s_c[RB], s_cs[RB];
+  __shared__ int s_bad;
+  cg::cluster_group cluster = cg::this_cluster();
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int rank = (int)cluster.block_rank();
+  const int ld = chunk + 4;
+  const int64_t c0 = (int64_t)rank * chunk;
+  float* ms = reinterpret_cast<float*>(smem_raw);  // [kClMaxK][ld], rows >= K zero
+  float* xs = ms + (size_t)kClMaxK * ld;           // [RB][ld]
+  float* s_coef = xs + (size_t)RB * ld;            // [3][T] when T <= kClCoefT
+  if (tid == 0) {
+    mbar_init(&bar_m, 1);
+    mbar_init(&bar_x, 1);
+    fence_barrier_init();
+    mbar_arrive_expect_tx(&bar_m, (uint32_t)chunk * sizeof(float) * (uint32_t)K);
+    s_bad = 0;
+  }
+  for (int q = tid; q < (kClMaxK - K) * ld; q += kClThreads) ms[(size_t)K * ld + q] = 0.f;
+  const bool coef_staged = T <= kClCoefT;  // constants: staged before the dependency wait
+  if (coef_staged)
+    for (int q = tid; q < 3 * T; q += kClThreads) s_coef[q] = coef[q];
+  __syncthreads();
+  if (warp == 0)  // the means do not depend on the predecessor
+    for (int k = lane; k < K; k += 32) bulk_g2s(ms + (size_t)k * ld, mu + (int64_t)k * D + c0, chunk * 4u, &bar_m);
+  pdl_wait();     // the rows, their count and their timesteps come from the kernel just before
+  pdl_trigger();  // the successor may now run its prologue
+  const int n_rows = min(*n_rows_dev, max_rows);
+  const int r0 = blockIdx.y * RB;
+  const int nr = min(RB, n_rows - r0);
+  if (nr <= 0) {  // the whole cluster has no rows (uniform): the means copy lands first
+    if (!mbar_wait_bounded(&bar_m, 0, pa::kDrainLimit) && tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    return;
+  }
+  if (tid == 0) mbar_arrive_expect_tx(&bar_x, (uint32_t)chunk * sizeof(float) * (uint32_t)nr);
+  for (int q = tid; q < (RB - nr) * ld; q += kClThreads) xs[(size_t)nr * ld + q] = 0.f;  // rows past the count
+  if (tid < nr) {
+    const int i = miss_bt[2 * (r0 + tid) + 1];
+    const float* cf = coef_staged ? s_coef : coef;
+    s_sa[tid] = cf[i];
+    s_q[tid] = cf[T + i];
+    s_c[tid] = cf[2 * T + i];
+    s_cs[tid] = cf[2 * T + i] * cf[i];
+  }
+  __syncthreads();  // expect_tx precedes the copies
+  if (warp == 0)
+    for (int r = lane; r < nr; r += 32) bulk_g2s(xs + (size_t)r * ld, X + (int64_t)(r0 + r) * D + c0, chunk * 4u, &bar_x);
+  // bounded waits; a CTA whose copies did not land keeps to the cluster's
+  // barriers (its peers wait for it there) and writes NaN
+  bool ok = mbar_wait_bounded(&bar_m, 0, pa::kWaitLimit);
+  ok = mbar_wait_bounded(&bar_x, 0, pa::kWaitLimit) && ok;
+  if (!ok) {
+    if (tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    s_bad = 1;
+    mbar_wait_bounded(&bar_m, 0, pa::kDrainLimit);
+    mbar_wait_bounded(&bar_x, 0, pa::kDrainLimit);
+  }
+  __syncthreads();
+  // partial dot products: warp w takes rows 4 (w & 1) .. + 3 and components
+  // 4 (w >> 1) .. + 3; lane l the columns 4 l + 128 i (16-byte shared loads,
+  // conflict-free), accumulated in packed fp32 pairs (two columns per FMA);
+  // then a shuffle tree over the lanes
+  {
+    const int rq = (warp & 1) * 4, kq = (warp >> 1) * 4;
+    float2 a2[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int u = 0; u < 4; ++u) a2[i][u] = make_float2(0.f, 0.f);
+#pragma unroll 2
+    for (int c = lane * 4; c < chunk; c += 128) {
+      float4 xv[4], mv[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) xv[i] = *reinterpret_cast<const float4*>(xs + (size_t)(rq + i) * ld + c);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) mv[u] = *reinterpret_cast<const float4*>(ms + (size_t)(kq + u) * ld + c);
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          a2[i][u] = __ffma2_rn(make_float2(xv[i].x, xv[i].y), make_float2(mv[u].x, mv[u].y), a2[i][u]);
+          a2[i][u] = __ffma2_rn(make_float2(xv[i].z, xv[i].w), make_float2(mv[u].z, mv[u].w), a2[i][u]);
+        }
+    }
+    float a[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+      for (int u = 0; u < 4; ++u) a[i][u] = a2[i][u].x + a2[i][u].y;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) a[i][u] += __shfl_xor_sync(0xffffffffu, a[i][u], o);
+    if (lane == 0)
+#pragma unroll
+      for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int u = 0; u < 4; ++u) s_part[(rq + i) * kClMaxK + kq + u] = a[i][u];
+  }
+  cluster.sync();  // every CTA's partials are in its shared memory
+  // the complete dot products: the CL partials in rank order
+  if (tid < RB * kClMaxK) {
+    float v[CL];
+#pragma unroll
+    for (int q = 0; q < CL; ++q) v[q] = cluster.map_shared_rank(s_part, q)[tid];  // all in flight at once
+    float sum = 0.f;
+#pragma unroll
+    for (int q = 0; q < CL; ++q) sum += v[q];
+    s_r[tid] = sum;
+  }
+  cluster_arrive();  // this CTA has read its peers' partials (they may exit after the wait below)
+  __syncthreads();
+  // logits and max-subtracted softmax, a half-warp per row
+  {
+    const int rr = warp * 2 + (lane >> 4), k = lane & 15;
+    if (rr < RB) {
+      const bool on = rr < nr && k < K;
+      float l = -INFINITY;
+      if (on) {
+        const float sa = s_sa[rr];
+        l = (2.f * sa * s_r[rr * kClMaxK + k] - sa * sa * mnorm[k]) * s_q[rr];
+      }
+      float mx = l;
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+      const float ex = on ? expf(l - mx) : 0.f;
+      float sum = ex;
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+      s_rt[k * RB + rr] = ex / sum;  // zero for k >= K
+    }
+  }
+  __syncthreads();
+  // eps = a x - a sqrt(a) sum_k R_k mu_k over this CTA's columns, four per thread
+  const bool bad = s_bad != 0;
+  for (int cq = tid * 4; cq < chunk; cq += kClThreads * 4) {
+    float2 acc[RB][2];  // columns cq, cq+1 and cq+2, cq+3 of each row, packed fp32 pairs
+#pragma unroll
+    for (int r = 0; r < RB; ++r) acc[r][0] = acc[r][1] = make_float2(0.f, 0.f);
+#pragma unroll 4
+    for (int k = 0; k < K; ++k) {
+      const float4 m = *reinterpret_cast<const float4*>(ms + (size_t)k * ld + cq);
+      const float2 ml = make_float2(m.x, m.y), mh = make_float2(m.z, m.w);
+#pragma unroll
+      for (int r = 0; r < RB; r += 4) {
+        const float4 v = *reinterpret_cast<const float4*>(s_rt + k * RB + r);  // responsibilities of 4 rows
+        const float w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          const float2 w2 = make_float2(w4[q], w4[q]);
+          acc[r + q][0] = __ffma2_rn(w2, ml, acc[r + q][0]);
+          acc[r + q][1] = __ffma2_rn(w2, mh, acc[r + q][1]);
+        }
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < RB; ++r) {
+      if (r >= nr) break;
+      const float4 x = *reinterpret_cast<const float4*>(xs + (size_t)r * ld + cq);
+      const float ac = s_c[r], acs = s_cs[r];
+      float4 o = make_float4(ac * x.x - acs * acc[r][0].x, ac * x.y - acs * acc[r][0].y, ac * x.z - acs * acc[r][1].x,
+                             ac * x.w - acs * acc[r][1].y);
+      if (bad) o = make_float4(__int_as_float(0x7fc00000), __int_as_float(0x7fc00000), __int_as_float(0x7fc00000),
+                               __int_as_float(0x7fc00000));
+      *reinterpret_cast<float4*>(eps + (int64_t)(r0 + r) * D + c0 + cq) = o;
+    }
+  }
+  cluster_wait();  // no CTA leaves while a peer may still read its partials
+}
+
 }  // namespace
 
 struct pa_gmm {
@@ -658,7 +873,14 @@ struct pa_gmm {
   int64_t launches;
   bool tc_ok;   // the tensor-core dot products fit this device and these sizes
   bool use_tc;  // ... and are selected
+  bool cl_ok;   // the single-kernel cluster form fits these sizes and this device
+  int form;     // 0 CUDA-core dots + output kernel, 1 tensor-core dots + output kernel, 2 cluster form
 };
+
+namespace {
+constexpr int kClSize = 16;   // CTAs per cluster (non-portable size, opted into)
+constexpr int kClRows = 8;    // rows per cluster
+}  // namespace
 
 extern "C" size_t pa_gmm_workspace_bytes(int K, int64_t D, int max_rows, int T) {
   if (K < 1 || K > kMaxK || D < 1 || max_rows < 1 || T < 1 || T > 100000) return 0;
@@ -741,6 +963,42 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
   // Picard iteration); at K = 64 the tensor cores win (151.9 vs 170.4 us at
   // 4x128x128).
   g->use_tc = g->tc_ok && K > kTcMinK;
+  // The single-kernel cluster form for K <= 16 when D splits into kClSize
+  // 16-byte-aligned column chunks whose tiles fit in shared memory and a
+  // cluster of kClSize CTAs can be resident; then the default.
+  g->cl_ok = false;
+  g->form = g->use_tc ? 1 : 0;
+  if (e == cudaSuccess && major == 10 && K <= kClMaxK && D % (4 * kClSize) == 0 &&
+      (reinterpret_cast<uintptr_t>(means_dev) & 15) == 0) {
+    const int chunk = (int)(D / kClSize);
+    const size_t smem = ClShape<kClSize, kClRows>::smem_bytes(chunk, T);
+    auto kern = k_gmm_cluster<kClSize, kClRows>;
+    if (smem + 4096 <= (size_t)optin) {
+      e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+      if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+      if (e == cudaSuccess) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(kClSize, 1, 1);
+        cfg.blockDim = dim3(kClThreads);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute at[1];
+        at[0].id = cudaLaunchAttributeClusterDimension;
+        at[0].val.clusterDim.x = kClSize;
+        at[0].val.clusterDim.y = 1;
+        at[0].val.clusterDim.z = 1;
+        cfg.attrs = at;
+        cfg.numAttrs = 1;
+        int nclusters = 0;
+        e = cudaOccupancyMaxActiveClusters(&nclusters, kern, &cfg);
+        g->cl_ok = e == cudaSuccess && nclusters > 0;
+        if (e != cudaSuccess) {
+          (void)cudaGetLastError();  // the size is not supported here: keep the two-kernel forms
+          e = cudaSuccess;
+        }
+      }
+    }
+    if (g->cl_ok) g->form = 2;
+  }
   if (e == cudaSuccess) e = cudaStreamSynchronize(g->st);
   if (e != cudaSuccess) {
     pa::set_error(std::string("pa_gmm_create: ") + cudaGetErrorString(e));
@@ -770,6 +1028,20 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
   const size_t out_smem = (size_t)(g->K + kOutRows) * kOutCols * sizeof(float);
   const dim3 tc_grid(L.tc_chunks, (g->max_rows + kTcRows - 1) / kTcRows);
   cudaError_t e;
+  if (g->form == 2 && bulk && vec_out) {  // one kernel: cluster of kClSize CTAs per kClRows rows
+    const int chunk = (int)(g->D / kClSize);
+    e = pa::launch_ex(k_gmm_cluster<kClSize, kClRows>, dim3(kClSize, (g->max_rows + kClRows - 1) / kClRows),
+                      dim3(kClThreads), ClShape<kClSize, kClRows>::smem_bytes(chunk, g->T), g->st, kClSize,
+                      batch_x_dev, g->means, coef, g->T, miss_bt_dev, mnorm, n_rows_dev, g->K, g->D, chunk,
+                      g->max_rows, batch_eps_dev, status);
+    g->launches += 1;
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e != cudaSuccess) {
+      pa::set_error(std::string("pa_gmm_eps: ") + cudaGetErrorString(e));
+      return PA_ERR_CUDA;
+    }
+    return PA_OK;
+  }
   if (g->use_tc && bulk && L.tc_chunks >= kTcClusterMinChunks)
     e = pa::launch_ex(k_gmm_dots_tc<kTcCluster>, tc_grid, dim3(kTcThreads), tc_smem_bytes(g->K), g->st,
                       kTcCluster, batch_x_dev, (const float*)(g->ws + L.mu_img), n_rows_dev, g->K, g->D,
@@ -813,17 +1085,23 @@ extern "C" int64_t pa_gmm_launches(const pa_gmm* g) { return g ? g->launches : -
 
 extern "C" pa_status pa_gmm_set_form(pa_gmm* g, int form) {
   if (!g) { pa::set_error("pa_gmm_set_form: NULL handle"); return PA_ERR_ARG; }
-  if (form != 0 && form != 1) { pa::set_error("pa_gmm_set_form: form must be 0 or 1"); return PA_ERR_ARG; }
+  if (form < 0 || form > 2) { pa::set_error("pa_gmm_set_form: form must be 0, 1 or 2"); return PA_ERR_ARG; }
   if (form == 1 && !g->tc_ok) {
     pa::set_error("pa_gmm_set_form: tensor-core dot products need an sm_100-family GPU, D % 4 == 0, "
                   "16-byte aligned means and enough shared memory");
     return PA_ERR_ARG;
   }
+  if (form == 2 && !g->cl_ok) {
+    pa::set_error("pa_gmm_set_form: the cluster form needs K <= 16, D a multiple of 64, an sm_100-family GPU, "
+                  "16-byte aligned means and enough shared memory");
+    return PA_ERR_ARG;
+  }
   g->use_tc = form == 1;
+  g->form = form;
   return PA_OK;
 }
 
-extern "C" int pa_gmm_form(const pa_gmm* g) { return g ? (g->use_tc ? 1 : 0) : -1; }
+extern "C" int pa_gmm_form(const pa_gmm* g) { return g ? g->form : -1; }
 
 extern "C" void pa_gmm_destroy(pa_gmm* g) { delete g; }
 

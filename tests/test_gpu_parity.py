@@ -126,10 +126,12 @@ def test_async_equals_sync_and_is_deterministic():
 
 
 @pytest.mark.parametrize("w,form", [
+    (W.SD15, 2),
     (W.SD15, 0),
     (W.LARGE.with_(T=60), 1),
+    (W.BATCHED.with_(T=40), 2),
     (W.BATCHED.with_(T=40), 0),
-], ids=["sd15-cuda-cores", "large-tensor-cores", "batched"])
+], ids=["sd15-cluster", "sd15-cuda-cores", "large-tensor-cores", "batched-cluster", "batched-cuda-cores"])
 def test_graph_replay_equals_sync(w, form):
     """A whole generation captured as one CUDA graph (pa_init and every
     iteration's denoiser, update and planning kernels, chained by programmatic
@@ -225,26 +227,37 @@ def _gmm_rows(w, n, seed=0):
     return a, mu, idx, x, miss
 
 
-@pytest.mark.parametrize("form", [1, 0])
+@pytest.mark.parametrize("form", [2, 1, 0])
 @pytest.mark.parametrize("wname,n,max_rows", [("sd15", 48, 48), ("sd15", 1, 100), ("sd15", 37, 100),
                                               ("sd15", 100, 100), ("batched", 256, 256),
                                               ("large", 48, 48), ("large", 1, 128), ("large", 70, 128),
-                                              ("large", 128, 128), ("k32", 100, 100), ("tiny", 5, 8)])
+                                              ("large", 128, 128), ("k32", 100, 100), ("tiny", 5, 8),
+                                              ("k3 d64", 11, 16)])
 def test_gmm_kernel_against_oracle(wname, n, max_rows, form):
-    """The mixture denoiser alone, with the dot products on the tensor cores
-    (form 1) and on the CUDA cores (form 0), on rows spread over the whole
-    schedule, with the device row count below the capacity, and over three
-    calls in a row (the fixed-point accumulators and the tickets are reused).
-    With 64 components: one row, 70 rows (a ragged second 64-row block of the
-    tensor-core form's row tiles is not reached; rows past 48 are), and full
-    128-row tiles; exactly 32 components."""
+    """The mixture denoiser alone, in one cluster kernel (form 2), with the dot
+    products on the tensor cores (form 1) and on the CUDA cores (form 0), on
+    rows spread over the whole schedule, with the device row count below the
+    capacity and not a multiple of the cluster form's 8-row blocks, and over
+    three calls in a row (the fixed-point accumulators and the tickets are
+    reused). With 64 components: one row, 70 rows (a ragged second 64-row
+    block of the tensor-core form's row tiles is not reached; rows past 48
+    are), and full 128-row tiles; exactly 32 components; 3 components over 64
+    columns (4 columns per CTA of the cluster form)."""
     import torch
+    from paper_2609_36522_gb300 import abi
     from paper_2609_36522_gb300.solver import GmmDenoiser
-    w = W.SD15.with_(K=32, name="k32") if wname == "k32" else W.ALL[wname]
+    w = {"k32": W.SD15.with_(K=32, name="k32"),
+         "k3 d64": W.TINY.with_(K=3, latent_shape=(4, 4, 4), name="k3 d64")}.get(wname) or W.ALL[wname]
     a, mu, idx, x, miss = _gmm_rows(w, n)
     dev = torch.device("cuda")
     g = GmmDenoiser(torch.from_numpy(mu).to(dev), w.gmm_std, a, max_rows)
-    assert g.form() == (1 if w.K > 16 else 0), "tensor cores by default above 16 components"
+    assert g.form() == (1 if w.K > 16 else 2), "cluster form up to 16 components, tensor cores above"
+    if form == 2 and w.K > 16:
+        with pytest.raises(abi.PaError) as e:
+            g.set_form(2)
+        assert e.value.status == abi.PA_ERR_ARG
+        g.close()
+        return
     g.set_form(form)
     xd = torch.zeros(max_rows, w.D, dtype=torch.float32, device=dev)
     xd[:n] = torch.from_numpy(x).to(dev)
@@ -303,11 +316,13 @@ def test_gmm_in_cuda_graph():
         g.close()
 
 
-def test_sd15_tensor_core_denoiser():
-    """Whole-pipeline parity with the denoiser's dot products on the tensor
-    cores (the default only above 16 components)."""
+@pytest.mark.parametrize("form", [1, 0])
+def test_sd15_other_denoiser_forms(form):
+    """Whole-pipeline parity with the denoiser's two-kernel forms (dot
+    products on the tensor cores, the default only above 16 components, or
+    on the CUDA cores) in place of the cluster form."""
     w = W.SD15
-    compare(w, oracle_run(w), gpu_run(w, gmm_form=1))
+    assert compare(w, oracle_run(w), gpu_run(w, gmm_form=form)).max() <= REL_TOL
 
 
 @pytest.mark.parametrize("kind", [0, 1] + list(range(100, 113)))
