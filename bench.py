@@ -67,7 +67,11 @@ NOMINAL_HBM_GBS = 8000.0
 # figures from an earlier ncu capture of this bench command (profiles/ has it),
 # not a measurement of the current run; reported as null once the kernel
 # source has changed since.
-NCU_TRAFFIC = {}
+NCU_TRAFFIC = {
+    # SD-v1.5-shaped workload: per iteration, k_update_lean 6,247,552 B + k_plan_gather
+    # 2,003,648 B read (no DRAM writes within either launch), averaged over p = 100, 78, 34, 20.
+    ("45c85ee88b35fafd", "sd15"): 8251200,
+}
 
 
 def parse_args(argv=None):
