@@ -654,7 +654,8 @@ def run_ours(args):
     so_warm_gbps = alg_it / (so_warm_us * 1e-6) / 1e9
     cold_gbps = float(step_bytes.sum()) / (float(cold_per.sum()) * 1e-6) / 1e9
     sha = kernel_source_sha()
-    tkey = args.workload + ("-bf16" if args.cache_bits == 16 else "")
+    tkey = args.workload + ("-bf16" if args.cache_bits == 16 else "") + \
+        ("" if args.cache_thresh is None else f"-c{args.cache_thresh:g}")
     traffic = NCU_TRAFFIC.get((sha, tkey))
     step_kernel = {4: "Anderson-mixing update + mix kernel + planning kernel",
                    3: "fused step (update, grid barrier, decision, next batch from registers)",

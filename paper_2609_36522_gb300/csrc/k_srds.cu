@@ -105,6 +105,15 @@ __device__ __forceinline__ bool row_info(const SDev& d, const Stage& st, int r, 
   return d.active[b] != 0;
 }
 
+// A CTA's partial of an Eq. 4 sum (non-negative) as it enters the fp64
+// accumulator that CTAs add into in arrival order: rounded up to a multiple of
+// 2^-32, so every partial sum below 2^21 is exactly representable (2^21 / 2^-32
+// = 2^53) and the accumulated sum is the same whatever the order; above 2^21
+// the mean distance is at least 2^21 / D, far beyond any tau_cache.
+__device__ __forceinline__ double quantize_sum(double v) {
+  return ceil(v * 4294967296.0) * (1.0 / 4294967296.0);
+}
+
 __device__ __forceinline__ double block_sum(double v, double* s_w) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
@@ -287,7 +296,7 @@ __global__ void __launch_bounds__(kSThreads) k_srds_apply(SDev d, Stage st, cons
   }
   if (nhas) {
     const double t = block_sum(dist, s_w);
-    if (threadIdx.x == 0) atomicAdd(d.sacc + ((size_t)nset * d.B * d.N + nrow) * pa::kAccStride, t);
+    if (threadIdx.x == 0) atomicAdd(d.sacc + ((size_t)nset * d.B * d.N + nrow) * pa::kAccStride, quantize_sum(t));
   }
 }
 
@@ -323,7 +332,7 @@ __global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter, int ns
   if (nhas) {
     __syncthreads();  // s_w is reused
     const double t2 = block_sum(dist, s_w);
-    if (threadIdx.x == 0) atomicAdd(d.sacc + ((size_t)nset * d.B * d.N + r) * pa::kAccStride, t2);
+    if (threadIdx.x == 0) atomicAdd(d.sacc + ((size_t)nset * d.B * d.N + r) * pa::kAccStride, quantize_sum(t2));
   }
 }
 

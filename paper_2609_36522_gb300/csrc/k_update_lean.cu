@@ -288,20 +288,15 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
 
   Q x[LMAX + 1], ep[LMAX], xh[LMAX], z[NOISE ? LMAX : 1];
   if (live && nj > 0) {
-    // states past the frontier e are lazy copies of state e: one load of
-    // row e serves all of this warp's lazy positions
-    const int nreal = e - (t + j0);  // positions g <= nreal hold materialised states
-    Q xe = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-    if (nreal < 0) xe = ldq(Xr + se * D);
+    // every row load issued before any is used: a lazy position reads the
+    // row of state e by address (an L1 hit after the first). Copying the
+    // first lazy load's registers to the later positions instead makes each
+    // copy wait for its load, which serialises the loads (measured 44.4
+    // against 36.6 us per update launch at 4x128x128, window 64)
 #pragma unroll
     for (int g = 0; g <= LMAX; ++g) {
       if (g > nj) break;
-      if (g <= nreal) {
-        x[g] = ldq(Xr + xslot(g) * D);
-        xe = x[g];
-      } else {
-        x[g] = xe;
-      }
+      x[g] = ldq(Xr + xslot(g) * D);
     }
 #pragma unroll
     for (int g = 0; g < LMAX; ++g) {
