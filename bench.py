@@ -68,9 +68,11 @@ NOMINAL_HBM_GBS = 8000.0
 # not a measurement of the current run; reported as null once the kernel
 # source has changed since.
 NCU_TRAFFIC = {
-    # SD-v1.5-shaped workload: per iteration, k_update_lean 6,247,552 B + k_plan_gather
-    # 2,003,648 B read (no DRAM writes within either launch), averaged over p = 100, 78, 34, 20.
-    ("45c85ee88b35fafd", "sd15"): 8251200,
+    # per iteration: k_update_lean + k_plan_gather read + write bytes, averaged
+    # over the first generation's launches
+    ("23415a7edd5e7822", "sd15"): 8252224,       # 6,248,704 + 2,003,520 (no DRAM writes)
+    ("23415a7edd5e7822", "batched"): 30268032,   # 24,575,659 + 5,692,373
+    ("23415a7edd5e7822", "large"): 79840365,     # 70,997,211 + 8,843,154
 }
 
 

@@ -723,7 +723,13 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
     if (!mbar_wait_bounded(&bar_m, 0, pa::kDrainLimit) && tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
     return;
   }
-  if (tid == 0) mbar_arrive_expect_tx(&bar_x, (uint32_t)chunk * sizeof(float) * (uint32_t)nr);
+  // the row copies go out first: they need only the count, while each row's
+  // coefficients wait for its timestep (one more trip to memory)
+  if (warp == 0) {
+    if (lane == 0) mbar_arrive_expect_tx(&bar_x, (uint32_t)chunk * sizeof(float) * (uint32_t)nr);
+    __syncwarp();  // expect_tx precedes the copies
+    for (int r = lane; r < nr; r += 32) bulk_g2s(xs + (size_t)r * ld, X + (int64_t)(r0 + r) * D + c0, chunk * 4u, &bar_x);
+  }
   for (int q = tid; q < (RB - nr) * ld; q += kClThreads) xs[(size_t)nr * ld + q] = 0.f;  // rows past the count
   if (tid < nr) {
     const int i = miss_bt[2 * (r0 + tid) + 1];
@@ -733,9 +739,6 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
     s_c[tid] = cf[2 * T + i];
     s_cs[tid] = cf[2 * T + i] * cf[i];
   }
-  __syncthreads();  // expect_tx precedes the copies
-  if (warp == 0)
-    for (int r = lane; r < nr; r += 32) bulk_g2s(xs + (size_t)r * ld, X + (int64_t)(r0 + r) * D + c0, chunk * 4u, &bar_x);
   // bounded waits; a CTA whose copies did not land keeps to the cluster's
   // barriers (its peers wait for it there) and writes NaN
   bool ok = mbar_wait_bounded(&bar_m, 0, pa::kWaitLimit);
@@ -773,22 +776,31 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
           a2[i][u] = __ffma2_rn(make_float2(xv[i].z, xv[i].w), make_float2(mv[u].z, mv[u].w), a2[i][u]);
         }
     }
-    float a[4][4];
+    // the 16 sums (v = 4 i + u) over the 32 lanes by a halving exchange: at
+    // offset o each lane keeps half of its values (the upper half if lane bit
+    // o is set) and adds its partner's copy of them, so after offsets 16, 8,
+    // 4, 2 lane l holds value l >> 1 summed over 16 lanes and offset 1
+    // completes it: 16 shuffles instead of 80
+    float a[16];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
-      for (int u = 0; u < 4; ++u) a[i][u] = a2[i][u].x + a2[i][u].y;
+      for (int u = 0; u < 4; ++u) a[i * 4 + u] = a2[i][u].x + a2[i][u].y;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1)
+    for (int o = 16, n = 8; o > 1; o >>= 1, n >>= 1) {
+      const bool up = (lane & o) != 0;
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int u = 0; u < 4; ++u) a[i][u] += __shfl_xor_sync(0xffffffffu, a[i][u], o);
-    if (lane == 0)
-#pragma unroll
-      for (int i = 0; i < 4; ++i)
-#pragma unroll
-        for (int u = 0; u < 4; ++u) s_part[(rq + i) * kClMaxK + kq + u] = a[i][u];
+      for (int v = 0; v < n; ++v) {
+        const float send = up ? a[v] : a[v + n];
+        const float keep = up ? a[v + n] : a[v];
+        a[v] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+      }
+    }
+    a[0] += __shfl_xor_sync(0xffffffffu, a[0], 1);
+    if ((lane & 1) == 0) {
+      const int v = lane >> 1;
+      s_part[(rq + (v >> 2)) * kClMaxK + kq + (v & 3)] = a[0];
+    }
   }
   cluster.sync();  // every CTA's partials are in its shared memory
   // the complete dot products: the CL partials in rank order
