@@ -674,6 +674,9 @@ struct ClShape {
 };
 
 __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+  asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
 template <int CL, int RB>
@@ -687,8 +690,7 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
   static_assert(RB == 8 && kClThreads == 256, "8 warps: 2 row quads x 4 component quads of the 8 x 16 block");
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t bar_m, bar_x;
-  __shared__ float s_part[RB * kClMaxK];   // this CTA's partial dot products (read by the cluster)
-  __shared__ float s_r[RB * kClMaxK];      // dot products [row][k], then logits
+  __shared__ float s_all[CL][RB * kClMaxK];  // the partial dot products of every CTA, pushed by their owners
   __shared__ __align__(16) float s_rt[kClMaxK * RB];  // responsibilities [k][row]
   __shared__ float s_sa[RB], s_q[RB], s_c[RB], s_cs[RB];
   __shared__ int s_bad;
@@ -723,6 +725,7 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
     if (!mbar_wait_bounded(&bar_m, 0, pa::kDrainLimit) && tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
     return;
   }
+  cluster_arrive_relaxed();  // this CTA runs: its peers may push into its shared memory after their wait
   // the row copies go out first: they need only the count, while each row's
   // coefficients wait for its timestep (one more trip to memory)
   if (warp == 0) {
@@ -797,33 +800,33 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
       }
     }
     a[0] += __shfl_xor_sync(0xffffffffu, a[0], 1);
-    if ((lane & 1) == 0) {
-      const int v = lane >> 1;
-      s_part[(rq + (v >> 2)) * kClMaxK + kq + (v & 3)] = a[0];
-    }
+    // lanes 2v and 2v + 1 both hold value v: each pushes it into half of the
+    // cluster's CTAs (slot [this CTA's rank][row * 16 + k] there); stores
+    // need no round trip, and after the cluster barrier every CTA reads its
+    // own shared memory only
+    cluster_wait();  // every CTA of the cluster is running
+    const int v = lane >> 1;
+    float* slot = &s_all[rank][(rq + (v >> 2)) * kClMaxK + kq + (v & 3)];
+    const int q0 = (lane & 1) * (CL / 2);
+#pragma unroll
+    for (int q = 0; q < CL / 2; ++q) *cluster.map_shared_rank(slot, q0 + q) = a[0];
   }
-  cluster.sync();  // every CTA's partials are in its shared memory
-  // the complete dot products: the CL partials in rank order
+  cluster_arrive();  // release: this CTA's pushes ...
+  cluster_wait();    // acquire: ... and every peer's are visible; no remote access follows
+  // the complete dot products (the CL partials in rank order), the logits and
+  // the max-subtracted softmax: thread t < 128 takes row t / 16, component
+  // t % 16, so each row is a half-warp
   if (tid < RB * kClMaxK) {
-    float v[CL];
+    const int rr = tid >> 4, k = tid & 15;
+    float dot = 0.f;
 #pragma unroll
-    for (int q = 0; q < CL; ++q) v[q] = cluster.map_shared_rank(s_part, q)[tid];  // all in flight at once
-    float sum = 0.f;
-#pragma unroll
-    for (int q = 0; q < CL; ++q) sum += v[q];
-    s_r[tid] = sum;
-  }
-  cluster_arrive();  // this CTA has read its peers' partials (they may exit after the wait below)
-  __syncthreads();
-  // logits and max-subtracted softmax, a half-warp per row
-  {
-    const int rr = warp * 2 + (lane >> 4), k = lane & 15;
-    if (rr < RB) {
+    for (int q = 0; q < CL; ++q) dot += s_all[q][tid];
+    {
       const bool on = rr < nr && k < K;
       float l = -INFINITY;
       if (on) {
         const float sa = s_sa[rr];
-        l = (2.f * sa * s_r[rr * kClMaxK + k] - sa * sa * mnorm[k]) * s_q[rr];
+        l = (2.f * sa * dot - sa * sa * mnorm[k]) * s_q[rr];
       }
       float mx = l;
 #pragma unroll
@@ -870,7 +873,6 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
       *reinterpret_cast<float4*>(eps + (int64_t)(r0 + r) * D + c0 + cq) = o;
     }
   }
-  cluster_wait();  // no CTA leaves while a peer may still read its partials
 }
 
 }  // namespace
