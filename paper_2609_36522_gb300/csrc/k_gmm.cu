@@ -680,17 +680,19 @@ __device__ __forceinline__ void cluster_arrive_relaxed() {
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
 template <int CL, int RB>
-__global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restrict__ X, const float* __restrict__ mu,
+__global__ void __launch_bounds__(kClThreads, 2) k_gmm_cluster(const float* __restrict__ X, const float* __restrict__ mu,
                                                             const float* __restrict__ coef, int T,
                                                             const int32_t* __restrict__ miss_bt,
                                                             const float* __restrict__ mnorm,
                                                             const int32_t* __restrict__ n_rows_dev, int K, int64_t D,
                                                             int chunk, int max_rows, float* __restrict__ eps,
                                                             int32_t* status) {
-  static_assert(RB == 8 && kClThreads == 256, "8 warps: 2 row quads x 4 component quads of the 8 x 16 block");
+  static_assert(RB == 8 && kClThreads == 256 && CL % 2 == 0,
+                "8 warps: 2 row quads x 2 component octets x 2 column halves of the 8 x 16 block");
   extern __shared__ __align__(128) unsigned char smem_raw[];
   __shared__ __align__(8) uint64_t bar_m, bar_x;
   __shared__ float s_all[CL][RB * kClMaxK];  // the partial dot products of every CTA, pushed by their owners
+  __shared__ float s_half[2][RB * kClMaxK];  // this CTA's partials from each half of its columns
   __shared__ __align__(16) float s_rt[kClMaxK * RB];  // responsibilities [k][row]
   __shared__ float s_sa[RB], s_q[RB], s_c[RB], s_cs[RB];
   __shared__ int s_bad;
@@ -753,44 +755,51 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
     mbar_wait_bounded(&bar_x, 0, pa::kDrainLimit);
   }
   __syncthreads();
-  // partial dot products: warp w takes rows 4 (w & 1) .. + 3 and components
-  // 4 (w >> 1) .. + 3; lane l the columns 4 l + 128 i (16-byte shared loads,
-  // conflict-free), accumulated in packed fp32 pairs (two columns per FMA);
-  // then a shuffle tree over the lanes
+  // partial dot products: warp w takes rows 4 (w & 1) .. + 3, components
+  // 8 ((w >> 1) & 1) .. + 7 and half w >> 2 of the CTA's columns; lane l the
+  // columns 4 l + 128 i of that half (16-byte shared loads, conflict-free),
+  // accumulated in packed fp32 pairs (two columns per FMA): each loaded row
+  // vector feeds 8 components and each mean vector 4 rows
   {
-    const int rq = (warp & 1) * 4, kq = (warp >> 1) * 4;
-    float2 a2[4][4];
+    const int rq = (warp & 1) * 4, ko = ((warp >> 1) & 1) * 8, half = warp >> 2;
+    const int hb = ((chunk >> 2) >> 1) << 2;  // where the second half starts: a multiple of 4 columns
+    const int cb = half ? hb : 0, ce = half ? chunk : hb;
+    float2 a2[4][8];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
-      for (int u = 0; u < 4; ++u) a2[i][u] = make_float2(0.f, 0.f);
+      for (int u = 0; u < 8; ++u) a2[i][u] = make_float2(0.f, 0.f);
 #pragma unroll 2
-    for (int c = lane * 4; c < chunk; c += 128) {
-      float4 xv[4], mv[4];
+    for (int c = cb + lane * 4; c < ce; c += 128) {
+      float4 xv[4];
 #pragma unroll
       for (int i = 0; i < 4; ++i) xv[i] = *reinterpret_cast<const float4*>(xs + (size_t)(rq + i) * ld + c);
 #pragma unroll
-      for (int u = 0; u < 4; ++u) mv[u] = *reinterpret_cast<const float4*>(ms + (size_t)(kq + u) * ld + c);
+      for (int uh = 0; uh < 8; uh += 4) {
+        float4 mv[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i)
+        for (int u = 0; u < 4; ++u) mv[u] = *reinterpret_cast<const float4*>(ms + (size_t)(ko + uh + u) * ld + c);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          a2[i][u] = __ffma2_rn(make_float2(xv[i].x, xv[i].y), make_float2(mv[u].x, mv[u].y), a2[i][u]);
-          a2[i][u] = __ffma2_rn(make_float2(xv[i].z, xv[i].w), make_float2(mv[u].z, mv[u].w), a2[i][u]);
-        }
+        for (int i = 0; i < 4; ++i)
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            float2& acc = a2[i][uh + u];
+            acc = __ffma2_rn(make_float2(xv[i].x, xv[i].y), make_float2(mv[u].x, mv[u].y), acc);
+            acc = __ffma2_rn(make_float2(xv[i].z, xv[i].w), make_float2(mv[u].z, mv[u].w), acc);
+          }
+      }
     }
-    // the 16 sums (v = 4 i + u) over the 32 lanes by a halving exchange: at
+    // the 32 sums (v = 8 i + u) over the 32 lanes by a halving exchange: at
     // offset o each lane keeps half of its values (the upper half if lane bit
     // o is set) and adds its partner's copy of them, so after offsets 16, 8,
-    // 4, 2 lane l holds value l >> 1 summed over 16 lanes and offset 1
-    // completes it: 16 shuffles instead of 80
-    float a[16];
+    // 4, 2, 1 lane l holds value l summed over all lanes: 31 shuffles
+    float a[32];
 #pragma unroll
     for (int i = 0; i < 4; ++i)
 #pragma unroll
-      for (int u = 0; u < 4; ++u) a[i * 4 + u] = a2[i][u].x + a2[i][u].y;
+      for (int u = 0; u < 8; ++u) a[i * 8 + u] = a2[i][u].x + a2[i][u].y;
 #pragma unroll
-    for (int o = 16, n = 8; o > 1; o >>= 1, n >>= 1) {
+    for (int o = 16, n = 16; o > 0; o >>= 1, n >>= 1) {
       const bool up = (lane & o) != 0;
 #pragma unroll
       for (int v = 0; v < n; ++v) {
@@ -799,17 +808,21 @@ __global__ void __launch_bounds__(kClThreads) k_gmm_cluster(const float* __restr
         a[v] = keep + __shfl_xor_sync(0xffffffffu, send, o);
       }
     }
-    a[0] += __shfl_xor_sync(0xffffffffu, a[0], 1);
-    // lanes 2v and 2v + 1 both hold value v: each pushes it into half of the
-    // cluster's CTAs (slot [this CTA's rank][row * 16 + k] there); stores
-    // need no round trip, and after the cluster barrier every CTA reads its
-    // own shared memory only
-    cluster_wait();  // every CTA of the cluster is running
-    const int v = lane >> 1;
-    float* slot = &s_all[rank][(rq + (v >> 2)) * kClMaxK + kq + (v & 3)];
-    const int q0 = (lane & 1) * (CL / 2);
+    s_half[half][(rq + (lane >> 3)) * kClMaxK + ko + (lane & 7)] = a[0];
+  }
+  __syncthreads();
+  // this CTA's partial of (row, k) = idx: its two column halves, pushed into
+  // every CTA of the cluster (slot [this CTA's rank][idx] there), half of the
+  // CTAs by each of the two threads that hold it; stores need no round trip,
+  // and after the cluster barrier every CTA reads its own shared memory only
+  cluster_wait();  // every CTA of the cluster is running
+  {
+    const int idx = tid & (RB * kClMaxK - 1);
+    const float pv = s_half[0][idx] + s_half[1][idx];
+    float* slot = &s_all[rank][idx];
+    const int q0 = (tid >> 7) * (CL / 2);
 #pragma unroll
-    for (int q = 0; q < CL / 2; ++q) *cluster.map_shared_rank(slot, q0 + q) = a[0];
+    for (int q = 0; q < CL / 2; ++q) *cluster.map_shared_rank(slot, q0 + q) = pv;
   }
   cluster_arrive();  // release: this CTA's pushes ...
   cluster_wait();    // acquire: ... and every peer's are visible; no remote access follows
@@ -987,7 +1000,9 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
     const int chunk = (int)(D / kClSize);
     const size_t smem = ClShape<kClSize, kClRows>::smem_bytes(chunk, T);
     auto kern = k_gmm_cluster<kClSize, kClRows>;
-    if (smem + 4096 <= (size_t)optin) {
+    cudaFuncAttributes fa = {};
+    e = cudaFuncGetAttributes(&fa, kern);
+    if (e == cudaSuccess && smem + fa.sharedSizeBytes <= (size_t)optin) {
       e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
       if (e == cudaSuccess) e = cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
       if (e == cudaSuccess) {
