@@ -780,7 +780,7 @@ def run_ours(args):
     # generation and copies x_T out to pinned host memory (pa_result), with
     # host time and device events around the whole loop. Headline: one
     # Solver.generate call per step (E2E_CHUNK iterations captured once as a
-    # CUDA graph, replayed with one pa_poll per replay). Beside it, the same
+    # CUDA graph, replayed with one pa_poll_result per replay). Beside it, the same
     # through eager calls: pa_step_async + pa_gmm_eps + pa_submit_eps issued
     # from Python in chunks of E2E_CHUNK, pa_poll per chunk.
     e2e = None
@@ -831,11 +831,11 @@ def run_ours(args):
         units_g, secs_g = aggregate(reps * n_iters, eager_s)
         e2e = {"value": units_e / secs_e, "unit": UNIT,
                "h2d_bytes_per_step": int(w.batch * w.D * 4),
-               "d2h_bytes_per_step": int(w.batch * w.D * 4 + (polls // reps) * 32),
+               "d2h_bytes_per_step": int((polls // reps) * (w.batch * w.D * 4 + 32)),
                "steps": reps,
                "api": f"Solver.generate: pa_init (host x_init), {E2E_CHUNK} iterations of pa_step_async + "
-                      f"pa_gmm_eps + pa_submit_eps captured once as a CUDA graph and replayed, pa_poll per "
-                      f"replay, pa_result (host x_T)",
+                      f"pa_gmm_eps + pa_submit_eps captured once as a CUDA graph and replayed, "
+                      f"pa_poll_result per replay (counters and host x_T behind one synchronisation)",
                "eager_value": units_g / secs_g,
                "eager_api": f"the same calls issued from Python in chunks of {E2E_CHUNK}, pa_poll per chunk"}
 

@@ -172,6 +172,17 @@ PA_API pa_status pa_poll(pa_solver* s, int* n_active);
  * Synchronises. */
 PA_API pa_status pa_result(pa_solver* s, float* x_out);
 
+/* pa_poll and pa_result behind one synchronisation, for callers that poll in
+ * a loop (Solver.generate): enqueues the copy of the counters and the copy of
+ * the states at t = T into x_out (HOST or DEVICE, [batch][D] fp32), waits for
+ * the stream once, then reports like pa_poll. When it returns PA_DONE, x_out
+ * holds x_T (Eq. 1's end point, Sec. 2.1) exactly as pa_result would write it;
+ * with PA_OK (trajectories still active) x_out holds the states then stored
+ * in the slot of x_T, which the caller overwrites by a later call. A device
+ * error status as pa_poll. PA_ERR_STATE before pa_init or between
+ * pa_step_async and pa_submit_eps. */
+PA_API pa_status pa_poll_result(pa_solver* s, float* x_out, int* n_active);
+
 /* Network evaluations so far: the sum over iterations of the misses, i.e. of
  * |M| of Eq. 5 (hits reuse the cached eps of Eq. 6 and cost no evaluation),
  * the NFE that Table 1 and Table 3 count per image. Synchronises; -1 on

@@ -65,6 +65,7 @@ _PROTOS = {
     "pa_submit_eps": (C.c_int, [VP, VP]),
     "pa_poll": (C.c_int, [VP, C.POINTER(C.c_int)]),
     "pa_result": (C.c_int, [VP, VP]),
+    "pa_poll_result": (C.c_int, [VP, VP, C.POINTER(C.c_int)]),
     "pa_nfe": (C.c_int64, [VP]),
     "pa_stats": (C.c_int, [VP, C.POINTER(PaStats)]),
     "pa_iter_log": (C.c_int, [VP, C.POINTER(C.c_int32), C.c_int, C.POINTER(C.c_int)]),
@@ -206,6 +207,13 @@ def pa_poll(h):
 
 def pa_result(h, x_out_ptr):
     return _check("pa_result", lib().pa_result(h, _dptr(x_out_ptr)))
+
+
+def pa_poll_result(h, x_out_ptr):
+    """-> (status, n_active); x_out holds x_T when status is PA_DONE."""
+    n = C.c_int()
+    st = _check("pa_poll_result", lib().pa_poll_result(h, _dptr(x_out_ptr), C.byref(n)))
+    return st, n.value
 
 
 def pa_nfe(h):

@@ -432,6 +432,24 @@ pa_status pa_result(pa_solver* s, float* x_out) {
   return sync_ctl(s, "pa_result");
 }
 
+pa_status pa_poll_result(pa_solver* s, float* x_out, int* n_active) {
+  if (!s) return arg_fail("pa_poll_result: solver is NULL");
+  if (!x_out) return arg_fail("pa_poll_result: x_out is NULL");
+  if (s->state != St::Ready && s->state != St::Done) return state_fail("pa_poll_result");
+  const pa::Dev& d = s->d;
+  const float* src = d.X + (int64_t)(d.T % (d.P + 1)) * d.D;
+  cudaError_t e = cudaMemcpy2DAsync(x_out, (size_t)d.D * sizeof(float), src,
+                                    (size_t)(d.P + 1) * d.D * sizeof(float), (size_t)d.D * sizeof(float),
+                                    d.B, cudaMemcpyDefault, s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_poll_result", e);
+  const pa_status r = sync_ctl(s, "pa_poll_result");
+  if (r != PA_OK) return r;
+  if (n_active) *n_active = s->host_ctl->n_active;
+  if (s->host_ctl->n_active != 0) return PA_OK;
+  s->state = St::Done;
+  return PA_DONE;
+}
+
 int64_t pa_nfe(pa_solver* s) {
   if (!s || s->state == St::Created) return -1;
   if (sync_ctl(s, "pa_nfe") != PA_OK) return -1;

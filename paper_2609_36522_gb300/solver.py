@@ -101,16 +101,26 @@ class Solver:
         st, n = abi.pa_poll(self.h)
         return n
 
+    def _out(self, out):
+        if out is None:
+            return torch.empty(self.batch, self.D, dtype=torch.float32, device=self.workspace.device)
+        if (not isinstance(out, torch.Tensor) or out.dtype != torch.float32 or not out.is_contiguous()
+                or out.numel() != self.batch * self.D):
+            raise ValueError("out must be a contiguous float32 tensor of batch x D elements")
+        return out
+
     def result(self, out=None):
         """x_T [batch][D] into ``out`` (a contiguous float32 CUDA or host
         tensor of batch x D elements), else into a new CUDA tensor."""
-        if out is None:
-            out = torch.empty(self.batch, self.D, dtype=torch.float32, device=self.workspace.device)
-        elif (not isinstance(out, torch.Tensor) or out.dtype != torch.float32 or not out.is_contiguous()
-              or out.numel() != self.batch * self.D):
-            raise ValueError("out must be a contiguous float32 tensor of batch x D elements")
+        out = self._out(out)
         abi.pa_result(self.h, out.data_ptr())
         return out
+
+    def poll_result(self, out):
+        """pa_poll and pa_result behind one synchronisation: the number of
+        trajectories still active; when it is 0, ``out`` holds x_T."""
+        st, n = abi.pa_poll_result(self.h, out.data_ptr())
+        return n
 
     def generate(self, x_init, denoise, out=None, chunk=4):
         """One whole generation in one call: x_init [batch][D] (CUDA tensor or
@@ -122,8 +132,9 @@ class Solver:
         on the device (as ``GmmDenoiser.eps`` does), and returns the CUDA eps
         tensor it wrote; it must write the same buffer on every call and be
         capturable in a CUDA graph. ``chunk`` (even) iterations are captured
-        once per (denoise, chunk) and the graph is replayed, one ``pa_poll``
-        per replay, until every trajectory has reached T; iterations issued
+        once per (denoise, chunk) and the graph is replayed, one
+        ``pa_poll_result`` per replay (the counters and x_T behind one
+        synchronisation), until every trajectory has reached T; iterations issued
         after that do nothing on the device. The captured launches carry the
         solver's settings of the capture: the setters of this class drop them;
         a denoiser's own settings must stay as they were captured (or pass a
@@ -147,11 +158,12 @@ class Solver:
                     self.submit_eps(denoise(bx, mb, nm))
             graphs[key] = gr
             self.init(x_init)  # the capture advanced the host state without running anything
+        out = self._out(out)
         for _ in range(self.T // chunk + 2):
             with torch.cuda.stream(self.stream):  # replay() launches on the current stream
                 gr.replay()
-            if self.poll() == 0:
-                return self.result(out)
+            if self.poll_result(out) == 0:  # one synchronisation: the counters and x_T together
+                return out
         raise RuntimeError("generate: trajectories did not reach T within T iterations")
 
     def nfe(self):

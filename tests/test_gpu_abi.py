@@ -182,3 +182,45 @@ def test_result_buffer_is_checked():
             s.result(bad)
     good = torch.empty(w.batch * w.D, dtype=torch.float32, device="cuda")
     assert torch.equal(s.result(good).view(w.batch, w.D), s.result())
+
+
+def test_poll_result_is_poll_and_result_behind_one_sync():
+    """pa_poll_result: PA_ERR_STATE before pa_init and between pa_step_async
+    and pa_submit_eps; PA_OK with the active count while trajectories run;
+    PA_DONE with x_out bit-equal to pa_result once they are done; and the
+    generate() loop built on it gives the synchronous result."""
+    import torch
+    w = W.BATCHED.with_(T=30)
+    s, g, eps, x0 = _solver(w)
+    out = torch.empty(w.batch, w.D, dtype=torch.float32, device="cuda")
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_poll_result(s.h, out.data_ptr())
+    assert e.value.status == abi.PA_ERR_STATE
+    s.init(x0)
+    bx, mb, nm = s.step_async()
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_poll_result(s.h, out.data_ptr())
+    assert e.value.status == abi.PA_ERR_STATE
+    g.eps(bx, mb, nm, eps)
+    s.submit_eps(eps)
+    st, n = abi.pa_poll_result(s.h, out.data_ptr())
+    assert st == abi.PA_OK and n == w.batch
+    while True:
+        bx, mb, nm = s.step_async()
+        g.eps(bx, mb, nm, eps)
+        s.submit_eps(eps)
+        st, n = abi.pa_poll_result(s.h, out.data_ptr())
+        if st == abi.PA_DONE:
+            break
+        assert n > 0
+    assert n == 0
+    assert torch.equal(out, s.result())
+    host = torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory()
+
+    def denoise(bx, mb, nm):
+        g.eps(bx, mb, nm, eps)
+        return eps
+
+    for _ in range(2):
+        s.generate(x0, denoise, out=host)
+        assert torch.equal(host, out.cpu())
