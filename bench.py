@@ -685,6 +685,10 @@ def run_ours(args):
                    "inside the full generation graph (the events cut the dependent-launch overlap)"),
         "checks": "iteration log and x_T bitwise equal to the generation with the denoiser",
     }
+    if traffic is not None:  # DRAM bytes (stored ncu figure) over the same time
+        solver_step["dram_bytes_per_iteration"] = traffic
+        solver_step["dram_gbps"] = traffic / (so_us * 1e-6) / 1e9
+        solver_step["dram_frac_of_measured_hbm"] = solver_step["dram_gbps"] / peak
     roofline = {"bound": "hbm", "achieved": so_gbps, "peak": peak, "unit": "GB/s",
                 "frac": so_gbps / peak, "traffic": traffic,
                 "kernel": "solver step: " + step_kernel,

@@ -191,7 +191,8 @@ def test_poll_result_is_poll_and_result_behind_one_sync():
     generate() loop built on it gives the synchronous result."""
     import torch
     w = W.BATCHED.with_(T=30)
-    s, g, eps, x0 = _solver(w)
+    st = torch.cuda.Stream()  # generate() captures a CUDA graph: not on the default stream
+    s, g, eps, x0 = _solver(w, stream=st)
     out = torch.empty(w.batch, w.D, dtype=torch.float32, device="cuda")
     with pytest.raises(abi.PaError) as e:
         abi.pa_poll_result(s.h, out.data_ptr())
