@@ -180,8 +180,9 @@ class Solver:
 
     def set_update_kernel(self, kind):
         """Picard-update kernel: 0 plain loads, 1 bulk forms, 2 lean register
-        form (the default), 100 + n / 200 + n launch shapes of the bulk / lean
-        forms (a tuning aid; pa_set_update_kernel documents them)."""
+        form (the default), 3 fused step, 100 + n / 200 + n / 300 + n launch
+        shapes of the bulk / lean / fused forms (a tuning aid;
+        pa_set_update_kernel documents them)."""
         self._drop_graphs()
         abi.pa_set_update_kernel(self.h, kind)
 
