@@ -56,7 +56,8 @@ FLUSH_BYTES = 256 << 20
 E2E_CHUNK = 4      # Picard iterations issued between two pa_poll calls in the end-to-end run
 GMM_FORMS = {2: "one kernel: clusters of 16 CTAs per 8 rows, CUDA-core dot products summed through "
                 "distributed shared memory",
-             1: "tensor-core dot products (tcgen05 kind::tf32, split operands) + output kernel",
+             1: "tensor-core dot products (tcgen05 kind::tf32, split operands), then for 16 < K <= 64 the "
+                "responsibilities and the output contraction on the tensor cores too, else an output kernel",
              0: "CUDA-core dot products (fp32 FMA) + output kernel"}
 PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0

@@ -470,7 +470,10 @@ PA_API int64_t pa_gmm_launches(const pa_gmm* g);
  * its columns of eps from the row and mean tiles it staged once. form 1: the
  * dot products on the tensor cores (tcgen05, kind::tf32, every operand split
  * into two tf32 parts and three products summed, which keeps fp32 accuracy),
- * 128 rows x 64 columns per CTA, then an output kernel; available when the GPU
+ * 128 rows x 64 columns per CTA, then an output kernel -- for 16 < K <= 64
+ * and D % 128 == 0 the output contraction R M on the tensor cores as well (a
+ * kernel that forms the responsibilities' split image, then 128 rows x 128
+ * columns per CTA with the accumulators in TMEM); available when the GPU
  * is of the sm_100 family, D % 4 == 0 and the means are 16-byte aligned, and
  * the default when K > 16. form 0: fp32 FMA dot products on the CUDA cores,
  * then the output kernel. A call whose batch_x or batch_eps is not 16-byte

@@ -92,9 +92,17 @@ __host__ __device__ inline int tc_npad(int K) {
 }
 // floats of one column chunk's means image: hi and lo, Kp rows each
 __host__ __device__ inline size_t tc_mu_chunk_floats(int K) { return (size_t)2 * tc_npad(K) * kTcCols; }
+// The tensor-core output contraction: kOtCols columns per CTA, up to 64
+// (padded) components; its operand images hold 2 x 128 rows (hi, then lo)
+// of tc_npad(K) values in core-matrix order.
+constexpr int kOtCols = 128;
+constexpr int kOtThreads = 256;
+constexpr int kOtMaxKp = 64;
+constexpr int kRespRows = 8;  // rows per k_gmm_resp CTA, a warp each
+__host__ __device__ inline size_t ot_img_floats(int K) { return (size_t)2 * kTcRows * tc_npad(K); }
 
 struct GmmLayout {
-  size_t coef, mnorm, gacc, epoch, status, mu_img, total;
+  size_t coef, mnorm, gacc, epoch, status, mu_img, mut_img, r_img, rcoef, total;
   int tc_chunks;    // column chunks of the tensor-core dot products (whole clusters)
   int nchunk;       // D-chunks of the CUDA-core dots kernel
   int chunk;        // columns per chunk
@@ -136,6 +144,12 @@ GmmLayout gmm_layout(int K, int64_t D, int max_rows, int T) {
   L.status = take(sizeof(int32_t));
   L.tc_chunks = (int)((D + kTcCols - 1) / kTcCols + kTcCluster - 1) / kTcCluster * kTcCluster;  // whole clusters
   L.mu_img = take((size_t)L.tc_chunks * tc_mu_chunk_floats(K) * sizeof(float));
+  // the tensor-core output contraction (16 < K <= 64): the means' transposed
+  // split image, the responsibilities' split image and the rows' scalars
+  const bool ot = K > kTcMinK && tc_npad(K) <= kOtMaxKp;
+  L.mut_img = take(ot ? (size_t)((D + kOtCols - 1) / kOtCols) * ot_img_floats(K) * sizeof(float) : 0);
+  L.r_img = take(ot ? (size_t)((max_rows + kTcRows - 1) / kTcRows) * ot_img_floats(K) * sizeof(float) : 0);
+  L.rcoef = take(ot ? (size_t)2 * max_rows * sizeof(float) : 0);
   L.total = o;
   return L;
 }
@@ -647,6 +661,241 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
 }
 
 // ---------------------------------------------------------------------------
+// Tensor-core form of the output contraction, for 16 < K <= 64 (with the
+// tensor-core dot products, form 1). eps = a x - a sqrt(a) R M, and R M is a
+// dense contraction over the components: rows x K times K x D.
+// k_gmm_resp forms each row's responsibilities once -- the same logits and
+// max-subtracted softmax as k_gmm_out -- and writes them as a split image
+// (hi = tf32(R), lo = tf32(R - hi), in core-matrix order, K-major); then
+// k_gmm_out_tc takes a block of 128 rows (M = 128; rows past the count are
+// zero) and kOtCols columns: one bulk copy brings the responsibilities'
+// image, another the means' transposed split image of its columns (built once
+// per handle, k_gmm_mut_image: the hi rows of the 128 columns followed by
+// their lo rows), one thread issues R_hi [M_hi; M_lo]^T (N = 256, columns
+// [0, 128) hi*hi and [128, 256) hi*lo) and R_lo M_hi^T (accumulated into
+// [0, 128)) per 8-component step into TMEM, and every thread reads its row's
+// accumulators back (tcgen05.ld, one row per TMEM lane) and writes its
+// columns of eps from the row values it loaded before the dependency wait.
+
+// element (r, c) of a K-major tile with Kp columns, in core-matrix order
+__host__ __device__ inline int ot_off(int r, int c, int Kp) {
+  return ((r >> 3) * (Kp >> 2) + (c >> 2)) * 32 + (r & 7) * 4 + (c & 3);
+}
+
+// The means' transposed split image, once per handle: chunk ch of kOtCols
+// columns, rows n (column ch * kOtCols + n; n >= kOtCols: the lo parts) x
+// components.
+__global__ void __launch_bounds__(256) k_gmm_mut_image(const float* __restrict__ mu, int K, int64_t D,
+                                                       float* __restrict__ img) {
+  const int Kp = tc_npad(K);
+  const int64_t ch = blockIdx.x;
+  float* out = img + ch * ot_img_floats(K);
+  for (int q = threadIdx.x; q < Kp * kOtCols; q += 256) {
+    const int k = q / kOtCols, n = q % kOtCols;  // consecutive threads read consecutive columns
+    const int64_t col = ch * kOtCols + n;
+    const float v = (k < K && col < D) ? mu[(int64_t)k * D + col] : 0.f;
+    const float hi = to_tf32(v);
+    out[ot_off(n, k, Kp)] = hi;
+    out[ot_off(n + kOtCols, k, Kp)] = to_tf32(v - hi);
+  }
+}
+
+// The responsibilities of every row (a warp per row) as the split image of
+// its 128-row block, and the row's scalars (a, a sqrt(a)) for the epilogue;
+// rows past the count (up to the end of their block) are zero. Advances the
+// accumulator epoch as k_gmm_out does.
+__global__ void __launch_bounds__(kRespRows * 32) k_gmm_resp(const long long* __restrict__ gacc2, GmmEpoch* ep,
+                                                             const float* __restrict__ coef, int T,
+                                                             const int32_t* __restrict__ miss_bt,
+                                                             const float* __restrict__ mnorm,
+                                                             const int32_t* __restrict__ n_rows_dev, int K,
+                                                             int max_rows, float* __restrict__ rimg,
+                                                             float* __restrict__ rcoef) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r = blockIdx.x * kRespRows + warp;
+  const int Kp = tc_npad(K);
+  const int n_rows = min(*n_rows_dev, max_rows);  // written two kernels back
+  float sa = 0.f, q = 0.f, c = 0.f;
+  if (r < n_rows) {
+    const int i = miss_bt[2 * r + 1];
+    sa = coef[i];
+    q = coef[T + i];
+    c = coef[2 * T + i];
+  }
+  pdl_wait();     // the dot products come from the kernel just before
+  pdl_trigger();  // the successor may now run its prologue
+  const uint32_t cur = ep->cur;
+  float* blk = rimg + (size_t)(r / kTcRows) * ot_img_floats(K);
+  const int rr = r % kTcRows;
+  float rv[2] = {0.f, 0.f};  // components lane and lane + 32
+  if (r < n_rows) {
+    const long long* g = gacc2 + (int64_t)(cur & 1u) * max_rows * K + (int64_t)r * K;
+    float l[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+    for (int u = 0; u < 2; ++u) {
+      const int k = lane + 32 * u;
+      if (k < K) {
+        const float dot = __ll2float_rn(__ldcg(g + k)) * (1.f / kDotScale);  // exact scale
+        l[u] = (2.f * sa * dot - sa * sa * mnorm[k]) * q;
+      }
+    }
+    float mx = fmaxf(l[0], l[1]);  // the order of k_gmm_out's loop: k = lane, then lane + 32
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    float sum = 0.f;
+#pragma unroll
+    for (int u = 0; u < 2; ++u)
+      if (lane + 32 * u < K) sum += expf(l[u] - mx);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const float inv = 1.f / sum;
+#pragma unroll
+    for (int u = 0; u < 2; ++u)
+      if (lane + 32 * u < K) rv[u] = expf(l[u] - mx) * inv;
+    if (lane == 0) {
+      rcoef[2 * r] = c;
+      rcoef[2 * r + 1] = c * sa;
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 2; ++u) {
+    const int k = lane + 32 * u;
+    if (k < Kp) {
+      const float hi = to_tf32(rv[u]);
+      blk[ot_off(rr, k, Kp)] = hi;
+      blk[ot_off(rr + kTcRows, k, Kp)] = to_tf32(rv[u] - hi);
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) ep->epoch = cur + 1u;  // the next call's set
+}
+
+__host__ inline size_t ot_smem_bytes(int K) {
+  // both split images; at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
+  const size_t b = (size_t)2 * ot_img_floats(K) * sizeof(float);
+  return b < 80 * 1024 ? 80 * 1024 : b;
+}
+
+__global__ void __launch_bounds__(kOtThreads, 1) k_gmm_out_tc(const float* __restrict__ X,
+                                                              const float* __restrict__ mut_img,
+                                                              const float* __restrict__ rimg,
+                                                              const float* __restrict__ rcoef,
+                                                              const int32_t* __restrict__ n_rows_dev, int K,
+                                                              int64_t D, int max_rows, float* __restrict__ eps,
+                                                              int32_t* status) {
+  extern __shared__ __align__(128) unsigned char smem_raw[];
+  __shared__ __align__(8) uint64_t bar_b, bar_a, bar_mma;
+  __shared__ uint32_t s_taddr;
+  constexpr uint32_t kTmemCols = 2 * kOtCols;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int Kp = tc_npad(K);
+  const size_t img = ot_img_floats(K);
+  float* A = reinterpret_cast<float*>(smem_raw);  // responsibilities: hi rows, then lo rows
+  float* B = A + img;                              // means of the columns: hi rows, then lo rows
+  const int64_t c0 = (int64_t)blockIdx.x * kOtCols;
+  const int r0 = blockIdx.y * kTcRows;
+  if (tid == 0) {
+    mbar_init(&bar_b, 1);
+    mbar_init(&bar_a, 1);
+    mbar_init(&bar_mma, 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(&s_taddr, kTmemCols);
+    tc_fence_before_sync();
+  }
+  __syncthreads();
+  tc_fence_after_sync();
+  const uint32_t taddr = s_taddr;
+  const uint32_t img_bytes = (uint32_t)(img * sizeof(float));
+  if (tid == 0) {  // the means image does not change
+    mbar_arrive_expect_tx(&bar_b, img_bytes);
+    bulk_g2s(B, mut_img + (size_t)blockIdx.x * img, img_bytes, &bar_b);
+  }
+  // the rows and their count were written three kernels back: thread (warp,
+  // lane) takes row 32 (warp % 4) + lane (its TMEM lane) and the 64 columns
+  // of half warp / 4
+  const int n_rows = min(*n_rows_dev, max_rows);
+  const int nr = min(kTcRows, n_rows - r0);
+  const int row = 32 * (warp & 3) + lane, half = warp >> 2;
+  const int64_t cb0 = c0 + half * (kOtCols / 2);
+  float4 xv[kOtCols / 8];
+  if (row < nr) {
+    const float4* xr = reinterpret_cast<const float4*>(X + (int64_t)(r0 + row) * D + cb0);
+#pragma unroll
+    for (int u = 0; u < kOtCols / 8; ++u) xv[u] = __ldg(xr + u);
+  }
+  pdl_wait();     // the responsibilities and the row scalars come from the kernel just before
+  pdl_trigger();  // the successor may now run its prologue
+  if (nr <= 0) {  // no rows in this block: the means copy lands and TMEM is freed
+    if (!mbar_wait_bounded(&bar_b, 0, pa::kDrainLimit) && tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    tc_fence_before_sync();
+    __syncthreads();
+    if (warp == 0) tmem_dealloc(taddr, kTmemCols);
+    return;
+  }
+  if (tid == 0) {
+    mbar_arrive_expect_tx(&bar_a, img_bytes);
+    bulk_g2s(A, rimg + (size_t)blockIdx.y * img, img_bytes, &bar_a);
+  }
+  const bool dots_bad = __ldcg(status) != 0;  // a dot-product wait ran out: the sums are incomplete
+  bool ok = __syncthreads_and(mbar_wait_bounded(&bar_b, 0, pa::kWaitLimit) &&
+                              mbar_wait_bounded(&bar_a, 0, pa::kWaitLimit));
+  if (!ok) {
+    if (tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    mbar_wait_bounded(&bar_b, 0, pa::kDrainLimit);  // the copies land before the CTA moves on
+    mbar_wait_bounded(&bar_a, 0, pa::kDrainLimit);
+  }
+  if (tid == 0 && ok) {
+    tc_fence_after_sync();
+    const uint32_t idesc2 = tc_idesc_tf32(kTcRows, 2 * kOtCols), idesc1 = tc_idesc_tf32(kTcRows, kOtCols);
+    const uint32_t a_hi = smem_u32(A), a_lo = smem_u32(A + (size_t)kTcRows * Kp), b = smem_u32(B);
+    const uint32_t sbo = (uint32_t)(Kp / 4) * 128;  // next 8-row group
+    for (int ks = 0; ks < Kp / 8; ++ks) {
+      const uint32_t ko = (uint32_t)ks * 256;  // two core matrices along K per step
+      tc_mma_tf32(taddr, tc_smem_desc(a_hi + ko, 128, sbo), tc_smem_desc(b + ko, 128, sbo), idesc2,
+                  ks > 0 ? 1u : 0u);
+      tc_mma_tf32(taddr, tc_smem_desc(a_lo + ko, 128, sbo), tc_smem_desc(b + ko, 128, sbo), idesc1, 1u);
+    }
+    tc_commit(&bar_mma);
+  }
+  if (ok && !__syncthreads_and(mbar_wait_bounded(&bar_mma, 0, pa::kWaitLimit))) {
+    if (tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    mbar_wait_bounded(&bar_mma, 0, pa::kDrainLimit);  // the MMAs finish before TMEM is freed
+    ok = false;
+  }
+  tc_fence_after_sync();
+  const bool live = row < nr;
+  const float ac = live ? rcoef[2 * (r0 + row)] : 0.f, acs = live ? rcoef[2 * (r0 + row) + 1] : 0.f;
+  float* er = eps + (int64_t)(r0 + row) * D + cb0;
+  const uint32_t tl = taddr + ((uint32_t)(32 * (warp & 3)) << 16) + (uint32_t)(half * (kOtCols / 2));
+#pragma unroll
+  for (int cb = 0; cb < kOtCols / 2; cb += 16) {
+    float v[16], w[16];
+    if (ok) {  // uniform across the CTA: every lane of the warp takes part in the loads
+      tmem_ld16(tl + (uint32_t)cb, v);
+      tmem_ld16(tl + (uint32_t)(kOtCols + cb), w);
+    }
+    if (!live) continue;
+#pragma unroll
+    for (int g = 0; g < 4; ++g) {
+      const float4 x = xv[cb / 4 + g];
+      float4 o;
+      if (ok && !dots_bad) {
+        o = make_float4(ac * x.x - acs * (v[4 * g] + w[4 * g]), ac * x.y - acs * (v[4 * g + 1] + w[4 * g + 1]),
+                        ac * x.z - acs * (v[4 * g + 2] + w[4 * g + 2]), ac * x.w - acs * (v[4 * g + 3] + w[4 * g + 3]));
+      } else {  // a bounded wait ran out here or before: the tile shows it
+        const float nan = __int_as_float(0x7fc00000);
+        o = make_float4(nan, nan, nan, nan);
+      }
+      *reinterpret_cast<float4*>(er + cb + 4 * g) = o;
+    }
+  }
+  tc_fence_before_sync();
+  __syncthreads();
+  if (warp == 0) tmem_dealloc(taddr, kTmemCols);
+}
+
+// ---------------------------------------------------------------------------
 // Single-kernel form for up to 16 components (form 2): a thread-block cluster
 // of CL CTAs takes a block of RB rows; CTA q of the cluster owns columns
 // [q * chunk, (q + 1) * chunk) with chunk = D / CL. Each CTA stages its chunk of
@@ -901,6 +1150,7 @@ struct pa_gmm {
   bool tc_ok;   // the tensor-core dot products fit this device and these sizes
   bool use_tc;  // ... and are selected
   bool cl_ok;   // the single-kernel cluster form fits these sizes and this device
+  bool ot_ok;   // form 1 also takes the output contraction on the tensor cores (16 < K <= 64)
   int form;     // 0 CUDA-core dots + output kernel, 1 tensor-core dots + output kernel, 2 cluster form
 };
 
@@ -982,6 +1232,20 @@ extern "C" pa_status pa_gmm_create(pa_gmm** out, int K, int64_t D, const float* 
       g->launches++;
       e = cudaGetLastError();
       g->tc_ok = e == cudaSuccess;
+    }
+  }
+  // The tensor-core output contraction beside them: 16 < K <= 64 (padded
+  // components fit one image of 128 rows x 64), whole kOtCols-column chunks.
+  g->ot_ok = false;
+  if (e == cudaSuccess && g->tc_ok && K > kTcMinK && tc_npad(K) <= kOtMaxKp && D % kOtCols == 0 &&
+      ot_smem_bytes(K) + 4096 <= (size_t)optin) {
+    e = cudaFuncSetAttribute(k_gmm_out_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)ot_smem_bytes(K));
+    if (e == cudaSuccess) {
+      k_gmm_mut_image<<<(unsigned)(D / kOtCols), 256, 0, g->st>>>(means_dev, K, D,
+                                                                    reinterpret_cast<float*>(g->ws + L.mut_img));
+      g->launches++;
+      e = cudaGetLastError();
+      g->ot_ok = e == cudaSuccess;
     }
   }
   // Default: the tensor cores for K > 16. At K <= 16 the contraction is under
@@ -1082,6 +1346,27 @@ extern "C" pa_status pa_gmm_eps(pa_gmm* g, const float* batch_x_dev, const int32
     e = pa::launch_ex(k_gmm_dots, dim3(L.nchunk, (g->max_rows + kDotRows - 1) / kDotRows), dim3(kThreads),
                       dots_smem_bytes(g->K, L.chunk), g->st, 0, batch_x_dev, g->means, n_rows_dev, g->K, g->D,
                       L.chunk, L.nchunk, g->max_rows, bulk, gacc2, ep, status);
+  if (g->use_tc && g->ot_ok && bulk && vec_out) {  // responsibilities, then the contraction on the tensor cores
+    const int blocks = (g->max_rows + kTcRows - 1) / kTcRows;
+    float* rimg = reinterpret_cast<float*>(g->ws + L.r_img);
+    float* rcoef = reinterpret_cast<float*>(g->ws + L.rcoef);
+    if (e == cudaSuccess)
+      e = pa::launch_ex(k_gmm_resp, dim3(blocks * (kTcRows / kRespRows)), dim3(kRespRows * 32), 0, g->st, 0,
+                        (const long long*)gacc2, ep, coef, g->T, miss_bt_dev, mnorm, n_rows_dev, g->K, g->max_rows,
+                        rimg, rcoef);
+    if (e == cudaSuccess)
+      e = pa::launch_ex(k_gmm_out_tc, dim3((unsigned)(g->D / kOtCols), blocks), dim3(kOtThreads),
+                        ot_smem_bytes(g->K), g->st, 0, batch_x_dev, (const float*)(g->ws + L.mut_img),
+                        (const float*)rimg, (const float*)rcoef, n_rows_dev, g->K, g->D, g->max_rows,
+                        batch_eps_dev, status);
+    g->launches += 3;
+    if (e == cudaSuccess) e = cudaGetLastError();
+    if (e != cudaSuccess) {
+      pa::set_error(std::string("pa_gmm_eps: ") + cudaGetErrorString(e));
+      return PA_ERR_CUDA;
+    }
+    return PA_OK;
+  }
   if (e == cudaSuccess)
     e = pa::launch_ex(k_gmm_out,
                       dim3((unsigned)((g->D + kOutCols - 1) / kOutCols), (g->max_rows + kOutRows - 1) / kOutRows),
