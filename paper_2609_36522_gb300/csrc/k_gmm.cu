@@ -92,14 +92,16 @@ __host__ __device__ inline int tc_npad(int K) {
 }
 // floats of one column chunk's means image: hi and lo, Kp rows each
 __host__ __device__ inline size_t tc_mu_chunk_floats(int K) { return (size_t)2 * tc_npad(K) * kTcCols; }
-// The tensor-core output contraction: kOtCols columns per CTA, up to 64
-// (padded) components; its operand images hold 2 x 128 rows (hi, then lo)
-// of tc_npad(K) values in core-matrix order.
-constexpr int kOtCols = 128;
+// The tensor-core output contraction: kOtCols columns per CTA (two CTAs per
+// SM), up to 64 (padded) components; its operand images hold hi rows, then lo
+// rows, of tc_npad(K) values in core-matrix order: 2 x 128 rows of
+// responsibilities, 2 x kOtCols rows (columns of D) of means.
+constexpr int kOtCols = 64;
 constexpr int kOtThreads = 256;
 constexpr int kOtMaxKp = 64;
 constexpr int kRespRows = 8;  // rows per k_gmm_resp CTA, a warp each
 __host__ __device__ inline size_t ot_img_floats(int K) { return (size_t)2 * kTcRows * tc_npad(K); }
+__host__ __device__ inline size_t ot_mut_floats(int K) { return (size_t)2 * kOtCols * tc_npad(K); }
 
 struct GmmLayout {
   size_t coef, mnorm, gacc, epoch, status, mu_img, mut_img, r_img, rcoef, total;
@@ -147,7 +149,7 @@ GmmLayout gmm_layout(int K, int64_t D, int max_rows, int T) {
   // the tensor-core output contraction (16 < K <= 64): the means' transposed
   // split image, the responsibilities' split image and the rows' scalars
   const bool ot = K > kTcMinK && tc_npad(K) <= kOtMaxKp;
-  L.mut_img = take(ot ? (size_t)((D + kOtCols - 1) / kOtCols) * ot_img_floats(K) * sizeof(float) : 0);
+  L.mut_img = take(ot ? (size_t)((D + kOtCols - 1) / kOtCols) * ot_mut_floats(K) * sizeof(float) : 0);
   L.r_img = take(ot ? (size_t)((max_rows + kTcRows - 1) / kTcRows) * ot_img_floats(K) * sizeof(float) : 0);
   L.rcoef = take(ot ? (size_t)2 * max_rows * sizeof(float) : 0);
   L.total = o;
@@ -670,10 +672,11 @@ __global__ void __launch_bounds__(kTcThreads) k_gmm_dots_tc(const float* __restr
 // k_gmm_out_tc takes a block of 128 rows (M = 128; rows past the count are
 // zero) and kOtCols columns: one bulk copy brings the responsibilities'
 // image, another the means' transposed split image of its columns (built once
-// per handle, k_gmm_mut_image: the hi rows of the 128 columns followed by
-// their lo rows), one thread issues R_hi [M_hi; M_lo]^T (N = 256, columns
-// [0, 128) hi*hi and [128, 256) hi*lo) and R_lo M_hi^T (accumulated into
-// [0, 128)) per 8-component step into TMEM, and every thread reads its row's
+// per handle, k_gmm_mut_image: the hi rows of the kOtCols columns followed by
+// their lo rows), one thread issues R_hi [M_hi; M_lo]^T (N = 2 kOtCols,
+// columns [0, kOtCols) hi*hi and [kOtCols, 2 kOtCols) hi*lo) and R_lo M_hi^T
+// (accumulated into [0, kOtCols)) per 8-component step into TMEM, and every
+// thread reads its row's
 // accumulators back (tcgen05.ld, one row per TMEM lane) and writes its
 // columns of eps from the row values it loaded before the dependency wait.
 
@@ -689,7 +692,7 @@ __global__ void __launch_bounds__(256) k_gmm_mut_image(const float* __restrict__
                                                        float* __restrict__ img) {
   const int Kp = tc_npad(K);
   const int64_t ch = blockIdx.x;
-  float* out = img + ch * ot_img_floats(K);
+  float* out = img + ch * ot_mut_floats(K);
   for (int q = threadIdx.x; q < Kp * kOtCols; q += 256) {
     const int k = q / kOtCols, n = q % kOtCols;  // consecutive threads read consecutive columns
     const int64_t col = ch * kOtCols + n;
@@ -770,12 +773,12 @@ __global__ void __launch_bounds__(kRespRows * 32) k_gmm_resp(const long long* __
 }
 
 __host__ inline size_t ot_smem_bytes(int K) {
-  // both split images; at least 80 KB so that at most two CTAs (2 x 256 TMEM columns) share an SM
-  const size_t b = (size_t)2 * ot_img_floats(K) * sizeof(float);
-  return b < 80 * 1024 ? 80 * 1024 : b;
+  // both split images; at least 60 KB so that at most three CTAs (3 x 128 TMEM columns) share an SM
+  const size_t b = (ot_img_floats(K) + ot_mut_floats(K)) * sizeof(float);
+  return b < 60 * 1024 ? 60 * 1024 : b;
 }
 
-__global__ void __launch_bounds__(kOtThreads, 1) k_gmm_out_tc(const float* __restrict__ X,
+__global__ void __launch_bounds__(kOtThreads, 2) k_gmm_out_tc(const float* __restrict__ X,
                                                               const float* __restrict__ mut_img,
                                                               const float* __restrict__ rimg,
                                                               const float* __restrict__ rcoef,
@@ -788,7 +791,7 @@ __global__ void __launch_bounds__(kOtThreads, 1) k_gmm_out_tc(const float* __res
   constexpr uint32_t kTmemCols = 2 * kOtCols;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int Kp = tc_npad(K);
-  const size_t img = ot_img_floats(K);
+  const size_t img = ot_img_floats(K), mimg = ot_mut_floats(K);
   float* A = reinterpret_cast<float*>(smem_raw);  // responsibilities: hi rows, then lo rows
   float* B = A + img;                              // means of the columns: hi rows, then lo rows
   const int64_t c0 = (int64_t)blockIdx.x * kOtCols;
@@ -806,10 +809,10 @@ __global__ void __launch_bounds__(kOtThreads, 1) k_gmm_out_tc(const float* __res
   __syncthreads();
   tc_fence_after_sync();
   const uint32_t taddr = s_taddr;
-  const uint32_t img_bytes = (uint32_t)(img * sizeof(float));
+  const uint32_t img_bytes = (uint32_t)(img * sizeof(float)), mimg_bytes = (uint32_t)(mimg * sizeof(float));
   if (tid == 0) {  // the means image does not change
-    mbar_arrive_expect_tx(&bar_b, img_bytes);
-    bulk_g2s(B, mut_img + (size_t)blockIdx.x * img, img_bytes, &bar_b);
+    mbar_arrive_expect_tx(&bar_b, mimg_bytes);
+    bulk_g2s(B, mut_img + (size_t)blockIdx.x * mimg, mimg_bytes, &bar_b);
   }
   // the rows and their count were written three kernels back: thread (warp,
   // lane) takes row 32 (warp % 4) + lane (its TMEM lane) and the 64 columns
