@@ -18,8 +18,11 @@ Also reported:
                 per microsecond against the measured HBM copy bandwidth (and
                 the nominal 8 TB/s), with L2 flushed per generation, L2 warm,
                 and L2 flushed before every iteration;
-  roofline      the solver step's kernel (the fused step where it runs) from
-                the solver-only graph;
+  roofline      the solver step (update and planning kernels, or the fused
+                step where it runs) from the solver-only graph, with the stored
+                ncu DRAM bytes of those kernels as ``traffic``;
+  denoiser      the denoiser alone: a graph of the same generation's calls on
+                the recorded batches;
   uncached      the same generation with tau_cache = 0 (no hits): NFE,
                 iterations and time;
   e2e           the public API with host buffers (copies inside the timing);
