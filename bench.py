@@ -475,7 +475,9 @@ def run_ours(args):
                 return n
             if record_in is not None:
                 m = max(out.n_miss, 1)
-                record_in.append((out.batch_x[:out.n_miss].clone() if out.n_miss else torch.zeros(1, w.D, device=dev),
+                full = torch.zeros(max_rows, w.D, dtype=torch.float32, device=dev)  # the denoiser may read every row
+                full[:out.n_miss].copy_(out.batch_x)
+                record_in.append((full,
                                   out.miss_bt[:out.n_miss].clone() if out.n_miss else torch.zeros(1, 2, dtype=torch.int32, device=dev),
                                   torch.tensor([out.n_miss], dtype=torch.int32, device=dev), m))
             g.eps(out.batch_x_ptr, out.miss_bt_ptr, sv.n_miss_dev(), eps)

@@ -231,7 +231,8 @@ def _gmm_rows(w, n, seed=0):
 @pytest.mark.parametrize("wname,n,max_rows", [("sd15", 48, 48), ("sd15", 1, 100), ("sd15", 37, 100),
                                               ("sd15", 100, 100), ("batched", 256, 256),
                                               ("large", 48, 48), ("large", 1, 128), ("large", 70, 128),
-                                              ("large", 128, 128), ("k32", 100, 100), ("tiny", 5, 8),
+                                              ("large", 128, 128), ("k32", 100, 100), ("k32", 300, 300),
+                                              ("k32", 129, 200), ("tiny", 5, 8),
                                               ("k3 d64", 11, 16)])
 def test_gmm_kernel_against_oracle(wname, n, max_rows, form):
     """The mixture denoiser alone, in one cluster kernel (form 2), with the dot

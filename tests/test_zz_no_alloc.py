@@ -57,7 +57,11 @@ def test_noalloc_matches_handle_entry_point_on_two_calls(lib):
         nd = torch.tensor([n], dtype=torch.int32, device=dev)
         ref = torch.empty_like(xd)
         got = torch.full_like(xd, float("nan"))
-        g.eps(xd.data_ptr(), md.data_ptr(), nd.data_ptr(), ref)
+        xfull = torch.zeros(100, w.D, dtype=torch.float32, device=dev)  # the handle's batch holds max_rows rows
+        xfull[:n] = xd
+        reff = torch.empty_like(xfull)
+        g.eps(xfull.data_ptr(), md.data_ptr(), nd.data_ptr(), reff)
+        ref.copy_(reff[:n])
         abi.pa_gmm_eps_noalloc(mu_d.data_ptr(), w.K, w.D, w.gmm_std, list(a), xd.data_ptr(),
                                md.data_ptr(), n, got.data_ptr(), stream.cuda_stream)
         torch.cuda.synchronize()
