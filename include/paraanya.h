@@ -260,8 +260,9 @@ PA_API pa_status pa_set_update_kernel(pa_solver* s, int kind);
  * ------------------------------------------------------------------------ */
 
 /* Bytes of the second device workspace that mixing needs: G and R of every
- * window state by iteration parity (4 x batch x (window+1) x D fp32) and the
- * Gram sums; 0 on bad sizes. */
+ * window state by iteration parity (4 x batch x (window+1) x D fp32), the
+ * Gram sums and one row per trajectory (the frontier state before the
+ * iteration); 0 on bad sizes. */
 PA_API size_t pa_anderson_workspace_bytes(int T, int window, int64_t D, int batch);
 
 /* depth 1: mix every iteration, using workspace_dev (DEVICE, 256-byte

@@ -64,11 +64,13 @@ __global__ void __launch_bounds__(kMixThreads) k_taa_mix(Dev d, int par) {
   __syncthreads();
   const float gam = s_gamma;
   const int slot = s % (P + 1);
-  const int slot_old = (s <= e ? s : e) % (P + 1);  // a lazy state reads state e
   const float* G = d.taa_g + ((int64_t)par * d.B + b) * (P + 1) * D + (int64_t)slot * D;
   const float* Gp = d.taa_g + ((int64_t)(par ^ 1) * d.B + b) * (P + 1) * D + (int64_t)slot * D;
   float* Xs = d.X + ((int64_t)b * (P + 1) + slot) * D;
-  const float* Xo = d.X + ((int64_t)b * (P + 1) + slot_old) * D;
+  // the old state: its own slot, which only this CTA's columns write; a lazy
+  // state (past e) is state e, whose slot the CTA of state e overwrites in
+  // this launch, so it reads the copy the update kernel kept
+  const float* Xo = s <= e ? d.X + ((int64_t)b * (P + 1) + slot) * D : d.taa_xe + (int64_t)b * D;
   const float* Xh = d.Xhat + ((int64_t)b * P + s % P) * D;  // entry of timestep s (used when j + 1 < p)
   const bool want_dl = j + 1 < p;
   const bool dl_from_old = rank_next >= 0;  // position j+1 missed: its entry is the old state

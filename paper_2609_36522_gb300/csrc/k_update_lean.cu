@@ -329,6 +329,16 @@ __global__ void __launch_bounds__(NW * 32, MINB) k_update_lean(Dev d, const floa
   // Pass 1: Eq. 7 for the misses, the drifts (kept in ep) and the run total.
   Q tot = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)}, tlo = tot;
   if (live && nj > 0) {
+    if constexpr (TAA) {
+      // the frontier state's value before the iteration, for the mix kernel's
+      // lazy states (the mix overwrites state e's slot): written by the one
+      // warp whose run holds state e, the last warp when e = t + p
+#pragma unroll
+      for (int g = 0; g <= LMAX; ++g) {
+        if (g > nj) break;
+        if (t + j0 + g == e && (g < nj || j0 + nj == p)) stq(d.taa_xe + (int64_t)b * D + mycol, x[g]);
+      }
+    }
     if (warp == 0) tot = x[0];  // the window start x_t begins the sum
 #pragma unroll
     for (int g = 0; g < LMAX; ++g) {

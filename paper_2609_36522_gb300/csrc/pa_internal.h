@@ -117,10 +117,14 @@ struct Dev {
   // workspace: the Picard map's output G and residual R of every window
   // state, [2][B][P+1][D] each by iteration parity (copy k mod 2 written in
   // iteration k, slot = state mod (P+1)), and the Gram sums <dR, R>, <dR, dR>
-  // per position, [2][2][B][P] x kAccStride, set k mod 2 in iteration k.
+  // per position, [2][2][B][P] x kAccStride, set k mod 2 in iteration k,
+  // and the frontier state's value before the iteration, [B][D]: the mix
+  // kernel overwrites state e's slot while the lazy states (past e) still
+  // need its old value.
   float* taa_g;
   float* taa_r;
   double* taa_acc;
+  float* taa_xe;
   int taa;            // 1: iterations mix (depth 1); 0: plain Picard
   // Online adaptation of tau_cache (pa_set_cache_adaptation): tau of every
   // trajectory, [2][B] by plan parity (copy k mod 2 is the tau of iteration
@@ -269,11 +273,12 @@ __device__ __forceinline__ void red_add_gram(const Dev& d, int par, int which, i
 }
 
 // Bytes of the Anderson workspace: G and R by iteration parity, the Gram sums.
-inline size_t taa_layout(int P, int64_t D, int B, size_t* o_r, size_t* o_acc) {
+inline size_t taa_layout(int P, int64_t D, int B, size_t* o_r, size_t* o_acc, size_t* o_xe) {
   const size_t rows = align_up((size_t)2 * B * (P + 1) * D * sizeof(float), kAlign);
   *o_r = rows;
   *o_acc = 2 * rows;
-  return 2 * rows + align_up((size_t)2 * 2 * B * P * kAccStride * sizeof(double), kAlign);
+  *o_xe = *o_acc + align_up((size_t)2 * 2 * B * P * kAccStride * sizeof(double), kAlign);
+  return *o_xe + align_up((size_t)B * D * sizeof(float), kAlign);
 }
 
 // Grid-wide barrier of a launch whose CTAs are all resident at once (the

@@ -217,6 +217,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   d.taa_g = nullptr;
   d.taa_r = nullptr;
   d.taa_acc = nullptr;
+  d.taa_xe = nullptr;
   d.taa = 0;
   d.tau = reinterpret_cast<double*>(w + L.tau);
   d.adapt = 0;
@@ -561,8 +562,8 @@ pa_status pa_cache_thresholds(pa_solver* s, double* tau_out) {
 size_t pa_anderson_workspace_bytes(int T, int window, int64_t D, int batch) {
   if (!sizes_ok(T, window, D, batch)) return 0;
   const int P = window < T ? window : T;
-  size_t o_r = 0, o_acc = 0;
-  return pa::taa_layout(P, D, batch, &o_r, &o_acc);
+  size_t o_r = 0, o_acc = 0, o_xe = 0;
+  return pa::taa_layout(P, D, batch, &o_r, &o_acc, &o_xe);
 }
 
 pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t workspace_bytes) {
@@ -572,15 +573,15 @@ pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t w
   pa::Dev& d = s->d;
   if (depth == 0) {
     d.taa = 0;
-    d.taa_g = d.taa_r = nullptr;
+    d.taa_g = d.taa_r = d.taa_xe = nullptr;
     d.taa_acc = nullptr;
     s->state = St::Created;  // the iterates change meaning: pa_init starts over
     return PA_OK;
   }
   if (d.D % 4 != 0 || d.P > 16 * 7 || d.cache_bf16)
     return arg_fail("pa_set_anderson: needs D % 4 == 0, a window of at most 112 points and fp32 cache entries");
-  size_t o_r = 0, o_acc = 0;
-  const size_t need = pa::taa_layout(d.P, d.D, d.B, &o_r, &o_acc);
+  size_t o_r = 0, o_acc = 0, o_xe = 0;
+  const size_t need = pa::taa_layout(d.P, d.D, d.B, &o_r, &o_acc, &o_xe);
   if (!workspace_dev || (reinterpret_cast<uintptr_t>(workspace_dev) % pa::kAlign) != 0 || workspace_bytes < need) {
     pa::set_error("pa_set_anderson: workspace NULL, not 256-byte aligned, or smaller than pa_anderson_workspace_bytes()");
     return PA_ERR_WORKSPACE;
@@ -589,6 +590,7 @@ pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t w
   d.taa_g = reinterpret_cast<float*>(w);
   d.taa_r = reinterpret_cast<float*>(w + o_r);
   d.taa_acc = reinterpret_cast<double*>(w + o_acc);
+  d.taa_xe = reinterpret_cast<float*>(w + o_xe);
   d.taa = 1;
   s->state = St::Created;
   return PA_OK;
