@@ -929,6 +929,20 @@ __device__ __forceinline__ void cluster_arrive() { asm volatile("barrier.cluster
 __device__ __forceinline__ void cluster_arrive_relaxed() {
   asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
+// The address of this CTA's shared variable at `saddr` in the shared memory of
+// cluster CTA `rank` (a shared::cluster address).
+__device__ __forceinline__ uint32_t cluster_map(uint32_t saddr, int rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+// A 4-byte store into a peer's shared memory that completes on the peer's
+// mbarrier (both shared::cluster addresses): no round trip for the sender.
+__device__ __forceinline__ void st_async_remote(uint32_t raddr, float v, uint32_t rbar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.b32 [%0], %1, [%2];" ::"r"(raddr),
+               "r"(__float_as_uint(v)), "r"(rbar)
+               : "memory");
+}
 __device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 
 template <int CL, int RB>
@@ -942,7 +956,7 @@ __global__ void __launch_bounds__(kClThreads, 2) k_gmm_cluster(const float* __re
   static_assert(RB == 8 && kClThreads == 256 && CL % 2 == 0,
                 "8 warps: 2 row quads x 2 component octets x 2 column halves of the 8 x 16 block");
   extern __shared__ __align__(128) unsigned char smem_raw[];
-  __shared__ __align__(8) uint64_t bar_m, bar_x;
+  __shared__ __align__(8) uint64_t bar_m, bar_x, bar_p;
   __shared__ float s_all[CL][RB * kClMaxK];  // the partial dot products of every CTA, pushed by their owners
   __shared__ float s_half[2][RB * kClMaxK];  // this CTA's partials from each half of its columns
   __shared__ __align__(16) float s_rt[kClMaxK * RB];  // responsibilities [k][row]
@@ -959,10 +973,15 @@ __global__ void __launch_bounds__(kClThreads, 2) k_gmm_cluster(const float* __re
   if (tid == 0) {
     mbar_init(&bar_m, 1);
     mbar_init(&bar_x, 1);
+    mbar_init(&bar_p, 1);
     fence_barrier_init();
     mbar_arrive_expect_tx(&bar_m, (uint32_t)chunk * sizeof(float) * (uint32_t)K);
+    // every CTA of the cluster stores its RB x kClMaxK partials here
+    mbar_arrive_expect_tx(&bar_p, (uint32_t)(CL * RB * kClMaxK * sizeof(float)));
     s_bad = 0;
   }
+  // ||mu_k||^2 of the component this thread takes in the softmax (constant)
+  const float mn = (tid < RB * kClMaxK && (tid & (kClMaxK - 1)) < K) ? mnorm[tid & (kClMaxK - 1)] : 0.f;
   for (int q = tid; q < (kClMaxK - K) * ld; q += kClThreads) ms[(size_t)K * ld + q] = 0.f;
   const bool coef_staged = T <= kClCoefT;  // constants: staged before the dependency wait
   if (coef_staged)
@@ -1063,21 +1082,26 @@ __global__ void __launch_bounds__(kClThreads, 2) k_gmm_cluster(const float* __re
     s_half[half][(rq + (lane >> 3)) * kClMaxK + ko + (lane & 7)] = a[0];
   }
   __syncthreads();
-  // this CTA's partial of (row, k) = idx: its two column halves, pushed into
+  // this CTA's partial of (row, k) = idx: its two column halves, stored into
   // every CTA of the cluster (slot [this CTA's rank][idx] there), half of the
-  // CTAs by each of the two threads that hold it; stores need no round trip,
-  // and after the cluster barrier every CTA reads its own shared memory only
-  cluster_wait();  // every CTA of the cluster is running
+  // CTAs by each of the two threads that hold it, by asynchronous stores that
+  // complete on the receiver's mbarrier: no round trip for the sender and no
+  // cluster barrier; every CTA waits for its own barrier and then reads its
+  // own shared memory only
+  cluster_wait();  // every CTA of the cluster is running (its barrier initialised)
   {
     const int idx = tid & (RB * kClMaxK - 1);
     const float pv = s_half[0][idx] + s_half[1][idx];
-    float* slot = &s_all[rank][idx];
+    const uint32_t slot = smem_u32(&s_all[rank][idx]), bar = smem_u32(&bar_p);
     const int q0 = (tid >> 7) * (CL / 2);
 #pragma unroll
-    for (int q = 0; q < CL / 2; ++q) *cluster.map_shared_rank(slot, q0 + q) = pv;
+    for (int q = 0; q < CL / 2; ++q) st_async_remote(cluster_map(slot, q0 + q), pv, cluster_map(bar, q0 + q));
   }
-  cluster_arrive();  // release: this CTA's pushes ...
-  cluster_wait();    // acquire: ... and every peer's are visible; no remote access follows
+  if (!mbar_wait_bounded(&bar_p, 0, pa::kWaitLimit)) {  // every peer's partials have landed
+    if (tid == 0) atomicCAS(status, 0, pa::kDevTimeout);
+    s_bad = 1;
+  }
+  __syncthreads();
   // the complete dot products (the CL partials in rank order), the logits and
   // the max-subtracted softmax: thread t < 128 takes row t / 16, component
   // t % 16, so each row is a half-warp
@@ -1091,7 +1115,7 @@ __global__ void __launch_bounds__(kClThreads, 2) k_gmm_cluster(const float* __re
       float l = -INFINITY;
       if (on) {
         const float sa = s_sa[rr];
-        l = (2.f * sa * dot - sa * sa * mnorm[k]) * s_q[rr];
+        l = (2.f * sa * dot - sa * sa * mn) * s_q[rr];
       }
       float mx = l;
 #pragma unroll
