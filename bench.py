@@ -74,9 +74,9 @@ NOMINAL_HBM_GBS = 8000.0
 NCU_TRAFFIC = {
     # per iteration: k_update_lean + k_plan_gather read + write bytes, averaged
     # over the first generation's launches
-    ("23415a7edd5e7822", "sd15"): 8252224,       # 6,248,704 + 2,003,520 (no DRAM writes)
-    ("23415a7edd5e7822", "batched"): 30268032,   # 24,575,659 + 5,692,373
-    ("23415a7edd5e7822", "large"): 79840365,     # 70,997,211 + 8,843,154
+    ("2e7808ed5d540455", "sd15"): 8251136,       # 6,246,912 + 2,004,224 (no DRAM writes)
+    ("2e7808ed5d540455", "batched"): 30266923,   # 24,573,568 + 5,693,355
+    ("2e7808ed5d540455", "large"): 79748608,     # 70,906,697 + 8,841,911
 }
 
 
@@ -790,7 +790,8 @@ def run_ours(args):
     # generation and copies x_T out to pinned host memory (pa_result), with
     # host time and device events around the whole loop. Headline: one
     # Solver.generate call per step (E2E_CHUNK iterations captured once as a
-    # CUDA graph, replayed with one pa_poll_result per replay). Beside it, the same
+    # CUDA graph, replayed with one pa_poll_begin per replay, each poll read
+    # after the next replay is enqueued). Beside it, the same
     # through eager calls: pa_step_async + pa_gmm_eps + pa_submit_eps issued
     # from Python in chunks of E2E_CHUNK, pa_poll per chunk.
     e2e = None
@@ -814,9 +815,11 @@ def run_ours(args):
             return max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0), polls
 
         def run_generate():
+            polls = 0
             for _ in range(reps):
                 s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK)
-            return reps * -(-n_iters // E2E_CHUNK)
+                polls += s.generate_polls
+            return polls
 
         def run_eager():
             polls = 0
@@ -845,7 +848,9 @@ def run_ours(args):
                "steps": reps,
                "api": f"Solver.generate: pa_init (host x_init), {E2E_CHUNK} iterations of pa_step_async + "
                       f"pa_gmm_eps + pa_submit_eps captured once as a CUDA graph and replayed, "
-                      f"pa_poll_result per replay (counters and host x_T behind one synchronisation)",
+                      f"pa_poll_begin per replay (copies of the counters and host x_T, no wait), "
+                      f"each poll's pa_poll_end after the next replay is enqueued (one replay past "
+                      f"the end, which changes nothing)",
                "eager_value": units_g / secs_g,
                "eager_api": f"the same calls issued from Python in chunks of {E2E_CHUNK}, pa_poll per chunk"}
 
