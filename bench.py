@@ -789,9 +789,11 @@ def run_ours(args):
     # step copies x_init in from pinned host memory (pa_init), runs the
     # generation and copies x_T out to pinned host memory (pa_result), with
     # host time and device events around the whole loop. Headline: one
-    # Solver.generate call per step (E2E_CHUNK iterations captured once as a
-    # CUDA graph, replayed with one pa_poll_begin per replay, each poll read
-    # after the next replay is enqueued). Beside it, the same
+    # Solver.generate call per step through the device-driven loop (pa_init,
+    # pa_loop_launch, pa_poll_begin: no host round trip inside a generation),
+    # without waiting, so that each generation is queued behind the previous
+    # one's poll (at most two in flight, each checked); finish() at the end.
+    # Beside it: the same calls waiting for every generation, and the
     # through eager calls: pa_step_async + pa_gmm_eps + pa_submit_eps issued
     # from Python in chunks of E2E_CHUNK, pa_poll per chunk.
     e2e = None
@@ -814,12 +816,11 @@ def run_ours(args):
             stream.synchronize()
             return max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0), polls
 
-        def run_generate():
-            polls = 0
+        def run_generate(wait=False):
             for _ in range(reps):
-                s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK)
-                polls += s.generate_polls
-            return polls
+                s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK, wait=wait)
+            s.finish()
+            return reps * (1 if s.generate_path() == "device loop" else -(-n_iters // E2E_CHUNK))
 
         def run_eager():
             polls = 0
@@ -839,18 +840,28 @@ def run_ours(args):
         s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK)   # capture outside the timed loop
         assert np.array_equal(out_host.numpy(), x_cached), "generate() differs from the graph-replayed generation"
         e2e_s, polls = timed(run_generate)
+        assert np.array_equal(out_host.numpy(), x_cached), "pipelined generate() differs"
+        wait_s, _ = timed(lambda: run_generate(wait=True))
         eager_s, eager_polls = timed(run_eager)
         units_e, secs_e = aggregate(reps * n_iters, e2e_s)
+        units_w, secs_w = aggregate(reps * n_iters, wait_s)
         units_g, secs_g = aggregate(reps * n_iters, eager_s)
         e2e = {"value": units_e / secs_e, "unit": UNIT,
                "h2d_bytes_per_step": int(w.batch * w.D * 4),
                "d2h_bytes_per_step": int((polls // reps) * (w.batch * w.D * 4 + 32)),
                "steps": reps,
-               "api": f"Solver.generate: pa_init (host x_init), {E2E_CHUNK} iterations of pa_step_async + "
-                      f"pa_gmm_eps + pa_submit_eps captured once as a CUDA graph and replayed, "
-                      f"pa_poll_begin per replay (copies of the counters and host x_T, no wait), "
-                      f"each poll's pa_poll_end after the next replay is enqueued (one replay past "
-                      f"the end, which changes nothing)",
+               "api": ("Solver.generate(wait=False) per step: pa_init (host x_init), pa_loop_launch (a CUDA "
+                       "graph whose conditional WHILE node repeats two captured iterations -- pa_step_async, "
+                       "pa_gmm_eps, pa_submit_eps -- until every trajectory has reached T), pa_poll_begin "
+                       "(host x_T and the counters); each generation's poll read and checked once the next "
+                       "generation is queued, Solver.finish() after the last"
+                       if s.generate_path() == "device loop" else
+                       f"Solver.generate: {E2E_CHUNK} iterations captured as a CUDA graph, replayed with "
+                       f"pa_poll_result per replay (the driver refused the conditional graph node: "
+                       f"{s.__dict__.get('loop_error')})"),
+               "generate_path": s.generate_path(),
+               "waiting_value": units_w / secs_w,
+               "waiting_api": "the same with generate(wait=True): the host waits for each generation's poll",
                "eager_value": units_g / secs_g,
                "eager_api": f"the same calls issued from Python in chunks of {E2E_CHUNK}, pa_poll per chunk"}
 

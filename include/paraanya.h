@@ -183,6 +183,58 @@ PA_API pa_status pa_result(pa_solver* s, float* x_out);
  * pa_step_async and pa_submit_eps. */
 PA_API pa_status pa_poll_result(pa_solver* s, float* x_out, int* n_active);
 
+/* pa_poll_result split in two so that the caller can enqueue more work
+ * before it waits (Solver.generate without waiting enqueues the next
+ * generation behind the poll of the previous one, so the GPU does not idle
+ * while the host reads the counters). pa_poll_begin enqueues, on the solver's
+ * stream, the copy of the
+ * states at t = T into x_out (HOST or DEVICE, [batch][D] fp32; NULL: no copy)
+ * and of the counters into one of two pinned mirrors, and returns without
+ * waiting; x_out must stay allocated and unread until the matching
+ * pa_poll_end. pa_poll_end waits for the OLDEST pending pa_poll_begin's
+ * copies and reports its counters like pa_poll: PA_DONE when no trajectory
+ * was active at that point (x_out of that poll holds x_T, Eq. 1's end point,
+ * Sec. 2.1, exactly as pa_result writes it), PA_OK otherwise, or a device
+ * error status. Iterations enqueued after every trajectory reached T change
+ * nothing, so a later pending poll copies the same x_T. At most two polls
+ * pending: a third pa_poll_begin returns PA_ERR_STATE, as does pa_poll_end
+ * with none pending, pa_poll_begin before pa_init, between pa_step_async and
+ * pa_submit_eps, or while the stream is being captured. Pending polls
+ * survive pa_init: each reports the counters as they stood at its own
+ * pa_poll_begin in stream order. */
+PA_API pa_status pa_poll_begin(pa_solver* s, float* x_out);
+PA_API pa_status pa_poll_end(pa_solver* s, int* n_active);
+
+/* The device-driven generation loop: Sec. 2.1's outer loop (slide the window
+ * until every trajectory has reached T, Eq. 1 and 2) run by the GPU itself,
+ * with no host round trip per iteration or per chunk. After pa_init (the
+ * iteration count must be even), pa_loop_capture_begin starts capturing the
+ * solver's stream into the body of a CUDA graph's conditional WHILE node; the
+ * caller then issues exactly two iterations (pa_step_async, its denoiser's
+ * launches on the solver's stream reading the miss count on the device,
+ * pa_submit_eps; twice: the iterations alternate two plan copies); and
+ * pa_loop_capture_end appends a one-thread kernel that sets the node's
+ * condition (repeat while a trajectory is active, the device status is clean
+ * and fewer than T / 2 + 2 passes have run: the window advances at least one
+ * step per iteration, so T iterations always suffice, and the pass limit
+ * bounds the loop whatever the counters say), closes the capture and
+ * instantiates the graph. Nothing runs during the capture, and the host
+ * state returns to what it was at pa_loop_capture_begin. pa_loop_launch
+ * enqueues the whole loop after a pa_init (any even iteration count): on
+ * return the host may enqueue pa_poll_begin (or call pa_poll_result); host
+ * stepping (pa_step_async) is refused until the next pa_init. The captured
+ * launches carry the settings of the capture: every setter of this handle
+ * drops the loop (and is refused while a capture is open). One loop per
+ * handle; a new capture replaces it. Errors: PA_ERR_STATE for a call out of
+ * order (no capture open, a body that did not hold exactly two iterations,
+ * kernel timing enabled: its events cannot sit in a loop body, a stream
+ * already being captured); PA_ERR_CUDA where the driver refuses the
+ * conditional node or its instantiation (the capture is closed either way
+ * and the stream stays usable). */
+PA_API pa_status pa_loop_capture_begin(pa_solver* s);
+PA_API pa_status pa_loop_capture_end(pa_solver* s);
+PA_API pa_status pa_loop_launch(pa_solver* s);
+
 /* Network evaluations so far: the sum over iterations of the misses, i.e. of
  * |M| of Eq. 5 (hits reuse the cached eps of Eq. 6 and cost no evaluation),
  * the NFE that Table 1 and Table 3 count per image. Synchronises; -1 on

@@ -66,6 +66,11 @@ _PROTOS = {
     "pa_poll": (C.c_int, [VP, C.POINTER(C.c_int)]),
     "pa_result": (C.c_int, [VP, VP]),
     "pa_poll_result": (C.c_int, [VP, VP, C.POINTER(C.c_int)]),
+    "pa_poll_begin": (C.c_int, [VP, VP]),
+    "pa_poll_end": (C.c_int, [VP, C.POINTER(C.c_int)]),
+    "pa_loop_capture_begin": (C.c_int, [VP]),
+    "pa_loop_capture_end": (C.c_int, [VP]),
+    "pa_loop_launch": (C.c_int, [VP]),
     "pa_nfe": (C.c_int64, [VP]),
     "pa_stats": (C.c_int, [VP, C.POINTER(PaStats)]),
     "pa_iter_log": (C.c_int, [VP, C.POINTER(C.c_int32), C.c_int, C.POINTER(C.c_int)]),
@@ -214,6 +219,30 @@ def pa_poll_result(h, x_out_ptr):
     n = C.c_int()
     st = _check("pa_poll_result", lib().pa_poll_result(h, _dptr(x_out_ptr), C.byref(n)))
     return st, n.value
+
+
+def pa_poll_begin(h, x_out_ptr):
+    """Enqueue the copies of x_T (unless x_out_ptr is None) and the counters; no wait."""
+    return _check("pa_poll_begin", lib().pa_poll_begin(h, _dptr(x_out_ptr)))
+
+
+def pa_poll_end(h):
+    """-> (status, n_active) of the oldest pending pa_poll_begin, after waiting for it."""
+    n = C.c_int()
+    st = _check("pa_poll_end", lib().pa_poll_end(h, C.byref(n)))
+    return st, n.value
+
+
+def pa_loop_capture_begin(h):
+    return _check("pa_loop_capture_begin", lib().pa_loop_capture_begin(h))
+
+
+def pa_loop_capture_end(h):
+    return _check("pa_loop_capture_end", lib().pa_loop_capture_end(h))
+
+
+def pa_loop_launch(h):
+    return _check("pa_loop_launch", lib().pa_loop_launch(h))
 
 
 def pa_nfe(h):

@@ -12,6 +12,7 @@
 
 #include "../../include/paraanya.h"
 #include "pa_internal.h"
+#include "pa_loop.h"
 
 namespace pa {
 
@@ -46,6 +47,18 @@ struct pa_solver {
   int64_t k;         // pa_submit_eps calls since pa_init: the plan of iteration k is copy k mod 2
   int64_t launches;
   pa::Ctl* host_ctl; // pinned mirror of the device Ctl
+  pa::Ctl* host_ring;        // pinned: two more mirrors, one per pending pa_poll_begin
+  cudaEvent_t poll_ev[2];    // recorded behind each pending poll's copies
+  int poll_head, poll_count;  // the oldest pending poll's mirror, polls pending
+  // the device-driven generation loop (pa_loop_*): a graph [clear the pass
+  // counter] -> [WHILE node; body: two iterations and the loop test]
+  cudaGraph_t loop_graph;
+  cudaGraphExec_t loop_exec;
+  cudaGraphConditionalHandle loop_cond;
+  int32_t* loop_passes;    // device: body passes of the running launch
+  bool loop_capturing;     // between pa_loop_capture_begin and _end
+  bool looped;             // a loop was launched since pa_init: host-side stepping is closed
+  int64_t loop_k0, loop_launches0;  // s->k and s->launches when the capture began
   std::vector<double> alphas;  // the schedule, kept for pa_set_noise
   double eta;
   // optional CUDA-event timing of the Picard-update kernel
@@ -98,13 +111,9 @@ bool sizes_ok(int T, int P, int64_t D, int B) {
          D <= ((int64_t)1 << 40);
 }
 
-// Copy the device Ctl into the pinned mirror and wait. Returns a status for
-// a CUDA failure or a device-side error.
-pa_status sync_ctl(pa_solver* s, const char* where) {
-  cudaError_t e = cudaMemcpyAsync(s->host_ctl, s->d.ctl, sizeof(pa::Ctl), cudaMemcpyDeviceToHost, s->st);
-  if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);
-  if (e != cudaSuccess) return cuda_fail(where, e);
-  const int ds = s->host_ctl->status;
+// The device status word of a copied Ctl as a status.
+pa_status check_ctl(const pa::Ctl& c, const char* where) {
+  const int ds = c.status;
   if (ds == pa::kDevTimeout) {
     pa::set_error(std::string(where) + ": a device-side bounded wait ran out");
     return PA_ERR_TIMEOUT;
@@ -116,6 +125,15 @@ pa_status sync_ctl(pa_solver* s, const char* where) {
   return PA_OK;
 }
 
+// Copy the device Ctl into the pinned mirror and wait. Returns a status for
+// a CUDA failure or a device-side error.
+pa_status sync_ctl(pa_solver* s, const char* where) {
+  cudaError_t e = cudaMemcpyAsync(s->host_ctl, s->d.ctl, sizeof(pa::Ctl), cudaMemcpyDeviceToHost, s->st);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);
+  if (e != cudaSuccess) return cuda_fail(where, e);
+  return check_ctl(*s->host_ctl, where);
+}
+
 // Inside a stream capture the event becomes an event-record node of the graph
 // (recorded again at every replay); outside it is an ordinary record.
 cudaError_t record_timing_event(cudaEvent_t ev, cudaStream_t st) {
@@ -124,6 +142,35 @@ cudaError_t record_timing_event(cudaEvent_t ev, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   if (cs == cudaStreamCaptureStatusActive) return cudaEventRecordWithFlags(ev, st, cudaEventRecordExternal);
   return cudaEventRecord(ev, st);
+}
+
+// Enqueue the copy of the states in the slot of t = T ([batch][D]) into x_out.
+cudaError_t copy_xt(pa_solver* s, float* x_out) {
+  const pa::Dev& d = s->d;
+  const float* src = d.X + (int64_t)(d.T % (d.P + 1)) * d.D;
+  return cudaMemcpy2DAsync(x_out, (size_t)d.D * sizeof(float), src, (size_t)(d.P + 1) * d.D * sizeof(float),
+                           (size_t)d.D * sizeof(float), d.B, cudaMemcpyDefault, s->st);
+}
+
+// Forget the captured generation loop (its launches carry the settings of
+// the capture). Not while a capture is open.
+void drop_loop(pa_solver* s) {
+  if (s->loop_exec) cudaGraphExecDestroy(s->loop_exec);
+  if (s->loop_graph) cudaGraphDestroy(s->loop_graph);  // and the body the conditional node owns
+  s->loop_exec = nullptr;
+  s->loop_graph = nullptr;
+  s->loop_cond = 0;
+}
+
+// Setters that change what the captured launches would be drop the loop;
+// none may run while one is being captured.
+bool loop_busy(pa_solver* s, const char* where) {
+  if (!s->loop_capturing) {
+    drop_loop(s);
+    return false;
+  }
+  pa::set_error(std::string(where) + ": a generation loop is being captured");
+  return true;
 }
 
 }  // namespace
@@ -241,16 +288,35 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   s->update_kind = (D % 4 == 0) ? 2 : 0;
 
   const std::vector<float> hc = step_coefficients(s->alphas, 0.0);  // DDIM (eta = 0)
-  cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), sizeof(pa::Ctl), cudaHostAllocDefault);
+  s->poll_ev[0] = s->poll_ev[1] = nullptr;
+  s->poll_head = s->poll_count = 0;
+  s->loop_graph = nullptr;
+  s->loop_exec = nullptr;
+  s->loop_cond = 0;
+  s->loop_passes = nullptr;
+  s->loop_capturing = s->looped = false;
+  s->loop_k0 = s->loop_launches0 = 0;
+  cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), 3 * sizeof(pa::Ctl), cudaHostAllocDefault);
   if (e != cudaSuccess) {
     delete s;
     return cuda_fail("pa_create: cudaHostAlloc", e);
   }
-  std::memset(s->host_ctl, 0, sizeof(pa::Ctl));
+  std::memset(s->host_ctl, 0, 3 * sizeof(pa::Ctl));
+  s->host_ring = s->host_ctl + 1;
+  e = cudaEventCreateWithFlags(&s->poll_ev[0], cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&s->poll_ev[1], cudaEventDisableTiming);
+  if (e != cudaSuccess) {
+    for (cudaEvent_t x : s->poll_ev)
+      if (x) cudaEventDestroy(x);
+    cudaFreeHost(s->host_ctl);
+    delete s;
+    return cuda_fail("pa_create: cudaEventCreate", e);
+  }
   e = cudaMemcpyAsync(coef, hc.data(), hc.size() * sizeof(float), cudaMemcpyHostToDevice, s->st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d.ctl, 0, sizeof(pa::Ctl), s->st);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s->st);
   if (e != cudaSuccess) {
+    for (cudaEvent_t x : s->poll_ev) cudaEventDestroy(x);
     cudaFreeHost(s->host_ctl);
     delete s;
     return cuda_fail("pa_create", e);
@@ -261,6 +327,7 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
 
 pa_status pa_set_noise(pa_solver* s, double eta, const float* noise_dev) {
   if (!s) return arg_fail("pa_set_noise: solver is NULL");
+  if (loop_busy(s, "pa_set_noise")) return PA_ERR_STATE;
   if (s->state == St::Stepped) return state_fail("pa_set_noise");
   if (!(eta >= 0.0 && eta <= 1.0)) return arg_fail("pa_set_noise: eta must be in [0, 1]");
   if (eta > 0.0 && !noise_dev) return arg_fail("pa_set_noise: eta > 0 needs the draws (noise_dev)");
@@ -297,6 +364,7 @@ pa_status pa_init(pa_solver* s, const float* x_init) {
   s->launches += 2;
   if (e != cudaSuccess) return cuda_fail("pa_init: launch", e);
   s->k = 0;
+  s->looped = false;
   s->state = St::Ready;
   return PA_OK;
 }
@@ -304,7 +372,7 @@ pa_status pa_init(pa_solver* s, const float* x_init) {
 pa_status pa_step_async(pa_solver* s, const float** batch_x_dev, const int32_t** miss_bt_dev,
                         const int32_t** n_miss_dev) {
   if (!s) return arg_fail("pa_step_async: solver is NULL");
-  if (s->state != St::Ready) return state_fail("pa_step_async");
+  if (s->state != St::Ready || s->looped) return state_fail("pa_step_async");
   // the batch was gathered by the kernel that planned this iteration
   if (batch_x_dev) *batch_x_dev = s->d.batch_x;
   if (miss_bt_dev) *miss_bt_dev = s->d.miss_bt;
@@ -424,11 +492,7 @@ pa_status pa_result(pa_solver* s, float* x_out) {
   if (!s) return arg_fail("pa_result: solver is NULL");
   if (!x_out) return arg_fail("pa_result: x_out is NULL");
   if (s->state != St::Done) return state_fail("pa_result");
-  const pa::Dev& d = s->d;
-  const float* src = d.X + (int64_t)(d.T % (d.P + 1)) * d.D;
-  cudaError_t e = cudaMemcpy2DAsync(x_out, (size_t)d.D * sizeof(float), src,
-                                    (size_t)(d.P + 1) * d.D * sizeof(float), (size_t)d.D * sizeof(float),
-                                    d.B, cudaMemcpyDefault, s->st);
+  const cudaError_t e = copy_xt(s, x_out);
   if (e != cudaSuccess) return cuda_fail("pa_result", e);
   return sync_ctl(s, "pa_result");
 }
@@ -437,11 +501,7 @@ pa_status pa_poll_result(pa_solver* s, float* x_out, int* n_active) {
   if (!s) return arg_fail("pa_poll_result: solver is NULL");
   if (!x_out) return arg_fail("pa_poll_result: x_out is NULL");
   if (s->state != St::Ready && s->state != St::Done) return state_fail("pa_poll_result");
-  const pa::Dev& d = s->d;
-  const float* src = d.X + (int64_t)(d.T % (d.P + 1)) * d.D;
-  cudaError_t e = cudaMemcpy2DAsync(x_out, (size_t)d.D * sizeof(float), src,
-                                    (size_t)(d.P + 1) * d.D * sizeof(float), (size_t)d.D * sizeof(float),
-                                    d.B, cudaMemcpyDefault, s->st);
+  cudaError_t e = copy_xt(s, x_out);
   if (e != cudaSuccess) return cuda_fail("pa_poll_result", e);
   const pa_status r = sync_ctl(s, "pa_poll_result");
   if (r != PA_OK) return r;
@@ -449,6 +509,151 @@ pa_status pa_poll_result(pa_solver* s, float* x_out, int* n_active) {
   if (s->host_ctl->n_active != 0) return PA_OK;
   s->state = St::Done;
   return PA_DONE;
+}
+
+pa_status pa_poll_begin(pa_solver* s, float* x_out) {
+  if (!s) return arg_fail("pa_poll_begin: solver is NULL");
+  if (s->state != St::Ready && s->state != St::Done) return state_fail("pa_poll_begin");
+  if (s->poll_count == 2) {
+    pa::set_error("pa_poll_begin: two polls are pending (pa_poll_end first)");
+    return PA_ERR_STATE;
+  }
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(s->st, &cs);
+  if (e != cudaSuccess) return cuda_fail("pa_poll_begin", e);
+  if (cs != cudaStreamCaptureStatusNone) {
+    pa::set_error("pa_poll_begin: the solver's stream is being captured");
+    return PA_ERR_STATE;
+  }
+  const int slot = (s->poll_head + s->poll_count) & 1;
+  if (x_out) e = copy_xt(s, x_out);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(&s->host_ring[slot], s->d.ctl, sizeof(pa::Ctl), cudaMemcpyDeviceToHost, s->st);
+  if (e == cudaSuccess) e = cudaEventRecord(s->poll_ev[slot], s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_poll_begin", e);
+  s->poll_count++;
+  return PA_OK;
+}
+
+pa_status pa_poll_end(pa_solver* s, int* n_active) {
+  if (!s) return arg_fail("pa_poll_end: solver is NULL");
+  if (s->poll_count == 0) {
+    pa::set_error("pa_poll_end: no poll is pending");
+    return PA_ERR_STATE;
+  }
+  const int slot = s->poll_head;
+  s->poll_head ^= 1;
+  s->poll_count--;
+  const cudaError_t e = cudaEventSynchronize(s->poll_ev[slot]);
+  if (e != cudaSuccess) return cuda_fail("pa_poll_end", e);
+  const pa::Ctl& c = s->host_ring[slot];
+  const pa_status r = check_ctl(c, "pa_poll_end");
+  if (r != PA_OK) return r;
+  if (n_active) *n_active = c.n_active;
+  if (c.n_active != 0) return PA_OK;
+  if (s->state == St::Ready) s->state = St::Done;
+  return PA_DONE;
+}
+
+pa_status pa_loop_capture_begin(pa_solver* s) {
+  if (!s) return arg_fail("pa_loop_capture_begin: solver is NULL");
+  if (s->loop_capturing) {
+    pa::set_error("pa_loop_capture_begin: a capture is already open");
+    return PA_ERR_STATE;
+  }
+  if (s->state != St::Ready || s->looped || (s->k & 1)) return state_fail("pa_loop_capture_begin");
+  if (s->timing) {
+    pa::set_error("pa_loop_capture_begin: kernel timing records events, which a loop body cannot hold");
+    return PA_ERR_STATE;
+  }
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(s->st, &cs);
+  if (e != cudaSuccess) return cuda_fail("pa_loop_capture_begin", e);
+  if (cs != cudaStreamCaptureStatusNone) {
+    pa::set_error("pa_loop_capture_begin: the solver's stream is already being captured");
+    return PA_ERR_STATE;
+  }
+  drop_loop(s);
+  if (!s->loop_passes) e = cudaMalloc(reinterpret_cast<void**>(&s->loop_passes), sizeof(int32_t));
+  cudaGraphNode_t clear = nullptr, loop = nullptr;
+  cudaGraphNodeParams np = {};
+  if (e == cudaSuccess) e = cudaGraphCreate(&s->loop_graph, 0);
+  // the condition is 1 at every launch: the body runs at least once
+  if (e == cudaSuccess) e = cudaGraphConditionalHandleCreate(&s->loop_cond, s->loop_graph, 1, cudaGraphCondAssignDefault);
+  if (e == cudaSuccess) {
+    cudaMemsetParams mp = {};
+    mp.dst = s->loop_passes;
+    mp.value = 0;
+    mp.elementSize = sizeof(int32_t);
+    mp.width = 1;
+    mp.height = 1;
+    e = cudaGraphAddMemsetNode(&clear, s->loop_graph, nullptr, 0, &mp);
+  }
+  if (e == cudaSuccess) {
+    np.type = cudaGraphNodeTypeConditional;
+    np.conditional.handle = s->loop_cond;
+    np.conditional.type = cudaGraphCondTypeWhile;
+    np.conditional.size = 1;
+    e = cudaGraphAddNode(&loop, s->loop_graph, &clear, nullptr, 1, &np);
+  }
+  if (e == cudaSuccess)
+    e = cudaStreamBeginCaptureToGraph(s->st, np.conditional.phGraph_out[0], nullptr, nullptr, 0,
+                                      cudaStreamCaptureModeThreadLocal);
+  if (e != cudaSuccess) {
+    drop_loop(s);
+    return cuda_fail("pa_loop_capture_begin", e);
+  }
+  s->loop_capturing = true;
+  s->loop_k0 = s->k;
+  s->loop_launches0 = s->launches;
+  return PA_OK;
+}
+
+pa_status pa_loop_capture_end(pa_solver* s) {
+  if (!s) return arg_fail("pa_loop_capture_end: solver is NULL");
+  if (!s->loop_capturing) {
+    pa::set_error("pa_loop_capture_end: no capture is open");
+    return PA_ERR_STATE;
+  }
+  const bool two = s->state == St::Ready && s->k == s->loop_k0 + 2;
+  cudaError_t e = cudaSuccess;
+  // at most T iterations reach t = T (the window advances by at least one
+  // step in each): T / 2 + 2 passes of two iterations cover them
+  if (two) e = pa::launch_loop_cond(s->loop_cond, s->d.ctl, s->loop_passes, s->d.T / 2 + 2, s->st);
+  cudaGraph_t body = nullptr;
+  const cudaError_t e2 = cudaStreamEndCapture(s->st, &body);
+  if (e == cudaSuccess) e = e2;
+  s->loop_capturing = false;
+  s->k = s->loop_k0;  // nothing ran: the host state is the one before the capture
+  s->launches = s->loop_launches0;
+  if (s->state == St::Stepped) s->state = St::Ready;
+  if (e == cudaSuccess && !two) {
+    drop_loop(s);
+    pa::set_error("pa_loop_capture_end: the body must hold exactly two iterations "
+                  "(pa_step_async, the denoiser, pa_submit_eps, twice)");
+    return PA_ERR_STATE;
+  }
+  if (e == cudaSuccess) e = cudaGraphInstantiate(&s->loop_exec, s->loop_graph, 0);
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    drop_loop(s);
+    return cuda_fail("pa_loop_capture_end", e);
+  }
+  return PA_OK;
+}
+
+pa_status pa_loop_launch(pa_solver* s) {
+  if (!s) return arg_fail("pa_loop_launch: solver is NULL");
+  if (!s->loop_exec) {
+    pa::set_error("pa_loop_launch: no generation loop has been captured");
+    return PA_ERR_STATE;
+  }
+  if (s->state != St::Ready || s->looped || s->loop_capturing || ((s->k ^ s->loop_k0) & 1))
+    return state_fail("pa_loop_launch");
+  const cudaError_t e = cudaGraphLaunch(s->loop_exec, s->st);
+  if (e != cudaSuccess) return cuda_fail("pa_loop_launch", e);
+  s->looped = true;
+  return PA_OK;
 }
 
 int64_t pa_nfe(pa_solver* s) {
@@ -504,6 +709,7 @@ pa_status pa_last_reductions(pa_solver* s, float* err_out, float* delta_out) {
 
 pa_status pa_set_update_kernel(pa_solver* s, int kind) {
   if (!s) return arg_fail("pa_set_update_kernel: solver is NULL");
+  if (loop_busy(s, "pa_set_update_kernel")) return PA_ERR_STATE;
   if (kind == 0 || kind == 1 || kind == 2 || kind == 3) {
     s->update_kind = kind;
     s->lean_shape = 0;
@@ -528,6 +734,7 @@ pa_status pa_set_update_kernel(pa_solver* s, int kind) {
 
 pa_status pa_set_cache_adaptation(pa_solver* s, double rate, double target, double tau_min, double tau_max) {
   if (!s) return arg_fail("pa_set_cache_adaptation: solver is NULL");
+  if (loop_busy(s, "pa_set_cache_adaptation")) return PA_ERR_STATE;
   if (s->state == St::Stepped) return state_fail("pa_set_cache_adaptation");
   if (!(rate >= 0.0) || !std::isfinite(rate) || !(target >= 0.0 && target <= 1.0) || !(tau_min >= 0.0) ||
       !std::isfinite(tau_min) || std::isnan(tau_max) || !(tau_max >= tau_min))
@@ -568,6 +775,7 @@ size_t pa_anderson_workspace_bytes(int T, int window, int64_t D, int batch) {
 
 pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t workspace_bytes) {
   if (!s) return arg_fail("pa_set_anderson: solver is NULL");
+  if (loop_busy(s, "pa_set_anderson")) return PA_ERR_STATE;
   if (depth != 0 && depth != 1) return arg_fail("pa_set_anderson: depth must be 0 or 1");
   if (s->state == St::Stepped) return state_fail("pa_set_anderson");
   pa::Dev& d = s->d;
@@ -598,6 +806,7 @@ pa_status pa_set_anderson(pa_solver* s, int depth, void* workspace_dev, size_t w
 
 pa_status pa_set_cache_precision(pa_solver* s, int bits) {
   if (!s) return arg_fail("pa_set_cache_precision: solver is NULL");
+  if (loop_busy(s, "pa_set_cache_precision")) return PA_ERR_STATE;
   if (bits != 16 && bits != 32) return arg_fail("pa_set_cache_precision: bits must be 16 or 32");
   if (s->state == St::Stepped) return state_fail("pa_set_cache_precision");
   if (bits == 16 && s->d.taa) return arg_fail("pa_set_cache_precision: Anderson mixing keeps fp32 cache entries");
@@ -608,12 +817,14 @@ pa_status pa_set_cache_precision(pa_solver* s, int bits) {
 
 pa_status pa_debug_set_wait_limit(pa_solver* s, uint32_t polls) {
   if (!s) return arg_fail("pa_debug_set_wait_limit: solver is NULL");
+  if (loop_busy(s, "pa_debug_set_wait_limit")) return PA_ERR_STATE;
   s->d.wait_limit = polls ? polls : 0u;
   return PA_OK;
 }
 
 pa_status pa_set_kernel_timing(pa_solver* s, int enable) {
   if (!s) return arg_fail("pa_set_kernel_timing: solver is NULL");
+  if (loop_busy(s, "pa_set_kernel_timing")) return PA_ERR_STATE;
   s->timing = (enable != 0);
   return PA_OK;
 }
@@ -647,6 +858,15 @@ void pa_destroy(pa_solver* s) {
   if (!s) return;
   cudaStreamSynchronize(s->st);
   for (cudaEvent_t x : s->ev) cudaEventDestroy(x);
+  for (cudaEvent_t x : s->poll_ev)
+    if (x) cudaEventDestroy(x);
+  if (s->loop_capturing) {  // close the capture so that the stream stays usable
+    cudaGraph_t g = nullptr;
+    cudaStreamEndCapture(s->st, &g);
+    (void)cudaGetLastError();
+  }
+  drop_loop(s);
+  if (s->loop_passes) cudaFree(s->loop_passes);
   if (s->host_ctl) cudaFreeHost(s->host_ctl);
   delete s;
 }

@@ -122,7 +122,7 @@ class Solver:
         st, n = abi.pa_poll_result(self.h, out.data_ptr())
         return n
 
-    def generate(self, x_init, denoise, out=None, chunk=4):
+    def generate(self, x_init, denoise, out=None, chunk=4, wait=True):
         """One whole generation in one call: x_init [batch][D] (CUDA tensor or
         pinned host tensor) in, x_T out (into ``out``, a CUDA or pinned host
         tensor, else a new CUDA tensor).
@@ -130,17 +130,43 @@ class Solver:
         ``denoise(batch_x_ptr, miss_bt_ptr, n_miss_dev_ptr)`` enqueues eps_theta
         of the planned misses on this solver's stream, reading the miss count
         on the device (as ``GmmDenoiser.eps`` does), and returns the CUDA eps
-        tensor it wrote; it must write the same buffer on every call and be
-        capturable in a CUDA graph. ``chunk`` (even) iterations are captured
-        once per (denoise, chunk) and the graph is replayed, one
-        ``pa_poll_result`` per replay (the counters and x_T behind one
-        synchronisation), until every trajectory has reached T; iterations issued
-        after that do nothing on the device. The captured launches carry the
-        solver's settings of the capture: the setters of this class drop them;
-        a denoiser's own settings must stay as they were captured (or pass a
-        new callable)."""
+        tensor it wrote; it must write the same buffer on every call, allocate
+        nothing and be capturable in a CUDA graph.
+
+        The first call per denoiser captures two iterations as the body of a
+        device-side loop (``pa_loop_capture_begin/_end``: a CUDA graph whose
+        conditional WHILE node repeats the body until every trajectory has
+        reached T). Each call then enqueues ``pa_init`` (x_init copied in),
+        ``pa_loop_launch`` and ``pa_poll_begin`` (x_T and the counters copied
+        out): no host round trip inside a generation. With ``wait`` the call
+        returns after that poll; without it, it returns at once with at most
+        two generations in flight (a third call first waits for the oldest and
+        checks it), and ``finish()`` waits for the rest; ``out`` and x_init
+        must then stay untouched until then.
+
+        Where the loop cannot be built (a driver without conditional graph
+        nodes), ``chunk`` (even) iterations are captured as a CUDA graph and
+        replayed with one ``pa_poll_result`` per replay instead (always
+        waiting). The captured launches carry the solver's settings of the
+        capture: the setters of this class drop them; a denoiser's own settings
+        must stay as they were captured (or pass a new callable)."""
         if chunk < 2 or chunk % 2:
             raise ValueError("chunk must be a positive even number (iterations alternate two plan copies)")
+        out = self._out(out)
+        if self.__dict__.get("_loop_for") is not denoise and self.__dict__.get("loop_error") is None:
+            self._capture_loop(x_init, denoise)
+        if self.__dict__.get("_loop_for") is denoise:
+            pending = self.__dict__.setdefault("_pending", [])
+            self.init(x_init)
+            abi.pa_loop_launch(self.h)
+            if len(pending) == 2:
+                self._end_poll()
+            abi.pa_poll_begin(self.h, out.data_ptr())
+            pending.append((out, self._x_init_keepalive))
+            if wait:
+                self.finish()
+            return out
+        self.finish()
         graphs = self.__dict__.setdefault("_gen_graphs", {})
         key = (denoise, chunk)
         self.init(x_init)
@@ -158,13 +184,57 @@ class Solver:
                     self.submit_eps(denoise(bx, mb, nm))
             graphs[key] = gr
             self.init(x_init)  # the capture advanced the host state without running anything
-        out = self._out(out)
         for _ in range(self.T // chunk + 2):
             with torch.cuda.stream(self.stream):  # replay() launches on the current stream
                 gr.replay()
             if self.poll_result(out) == 0:  # one synchronisation: the counters and x_T together
                 return out
         raise RuntimeError("generate: trajectories did not reach T within T iterations")
+
+    def _capture_loop(self, x_init, denoise):
+        self.finish()
+        self.init(x_init)
+        # one eager iteration first: launch-time set-up (kernel attributes)
+        # happens outside the capture
+        bx, mb, nm = self.step_async()
+        self.submit_eps(denoise(bx, mb, nm))
+        self.init(x_init)
+        abi.pa_loop_capture_begin(self.h)
+        try:
+            with torch.cuda.stream(self.stream):  # torch work of the denoiser lands in the body
+                for _ in range(2):
+                    bx, mb, nm = self.step_async()
+                    self.submit_eps(denoise(bx, mb, nm))
+        except BaseException:
+            try:
+                abi.pa_loop_capture_end(self.h)  # closes the capture; the body is incomplete
+            except abi.PaError:
+                pass
+            raise
+        try:
+            abi.pa_loop_capture_end(self.h)
+        except abi.PaError as e:
+            if e.status != abi.PA_ERR_CUDA:
+                raise
+            self.loop_error = str(e)  # this driver cannot run the loop: replay and poll instead
+            return
+        self._loop_for = denoise
+
+    def _end_poll(self):
+        pending = self.__dict__.get("_pending", [])
+        pending.pop(0)
+        st, n = abi.pa_poll_end(self.h)
+        if n != 0:
+            raise RuntimeError(f"generate: {n} trajectories had not reached T when the device loop ended")
+
+    def finish(self):
+        """Wait for every generation still in flight (generate with wait=False) and check it."""
+        while self.__dict__.get("_pending"):
+            self._end_poll()
+
+    def generate_path(self):
+        """How generate runs: 'device loop' or, without conditional graph nodes, 'graph replay + poll'."""
+        return "graph replay + poll" if self.__dict__.get("loop_error") else "device loop"
 
     def nfe(self):
         return abi.pa_nfe(self.h)
@@ -215,13 +285,18 @@ class Solver:
         abi.pa_set_cache_precision(self.h, bits)
 
     def _drop_graphs(self):
+        self.finish()
         self.__dict__.pop("_gen_graphs", None)
+        self.__dict__.pop("_loop_for", None)  # the C setters drop the loop graph itself
 
     def close(self):
-        self._drop_graphs()  # captured launches refer to this workspace
-        if getattr(self, "h", None) is not None:
-            abi.pa_destroy(self.h)
-            self.h = None
+        try:
+            if getattr(self, "h", None) is not None:
+                self._drop_graphs()  # captured launches refer to this workspace
+        finally:
+            if getattr(self, "h", None) is not None:
+                abi.pa_destroy(self.h)
+                self.h = None
 
     def __del__(self):
         try:

@@ -225,3 +225,74 @@ def test_poll_result_is_poll_and_result_behind_one_sync():
     for _ in range(2):
         s.generate(x0, denoise, out=host)
         assert torch.equal(host, out.cpu())
+
+
+def test_poll_begin_end_keeps_one_iteration_queued():
+    """pa_poll_begin / pa_poll_end: PA_ERR_STATE before pa_init, with no poll
+    pending, between pa_step_async and pa_submit_eps, for a third pending poll
+    and inside a stream capture; two polls with no work between them report
+    the same count; a loop that enqueues iteration k + 1 before it waits for
+    the poll of iteration k sees the synchronous loop's active counts, ends
+    with x_T bit-equal to pa_result, and the iteration it ran past the end
+    changes neither the iteration log nor the NFE."""
+    import torch
+    w = W.BATCHED.with_(T=30)
+    st = torch.cuda.Stream()
+    s, g, eps, x0 = _solver(w, stream=st)
+    out = torch.empty(w.batch, w.D, dtype=torch.float32, device="cuda")
+
+    def state_error(f, *a):
+        with pytest.raises(abi.PaError) as e:
+            f(*a)
+        assert e.value.status == abi.PA_ERR_STATE
+
+    state_error(abi.pa_poll_begin, s.h, out.data_ptr())
+    state_error(abi.pa_poll_end, s.h)
+    # the synchronous loop's active counts, log and NFE
+    s.init(x0)
+    counts = []
+    while True:
+        bx, mb, nm = s.step_async()
+        g.eps(bx, mb, nm, eps)
+        s.submit_eps(eps)
+        stt, n = abi.pa_poll_result(s.h, out.data_ptr())
+        counts.append(n)
+        if stt == abi.PA_DONE:
+            break
+    log, nfe, want = s.iter_log(), s.nfe(), out.clone()
+    s.init(x0)
+    bx, mb, nm = s.step_async()
+    state_error(abi.pa_poll_begin, s.h, out.data_ptr())
+    g.eps(bx, mb, nm, eps)
+    s.submit_eps(eps)
+    abi.pa_poll_begin(s.h, None)
+    abi.pa_poll_begin(s.h, out.data_ptr())
+    state_error(abi.pa_poll_begin, s.h, out.data_ptr())
+    assert abi.pa_poll_end(s.h) == (abi.PA_OK, counts[0])
+    assert abi.pa_poll_end(s.h) == (abi.PA_OK, counts[0])
+    state_error(abi.pa_poll_end, s.h)
+    with torch.cuda.stream(st):
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=st):
+            state_error(abi.pa_poll_begin, s.h, out.data_ptr())
+            out.zero_()  # something captured (never replayed)
+    # pipelined: iteration k + 1 is enqueued before the poll of iteration k is read
+    host = torch.full((w.batch, w.D), float("nan"), dtype=torch.float32).pin_memory()
+    s.init(x0)
+    seen = []
+    for k in range(len(counts) + 1):
+        bx, mb, nm = s.step_async()
+        g.eps(bx, mb, nm, eps)
+        s.submit_eps(eps)
+        abi.pa_poll_begin(s.h, host.data_ptr())
+        if k == 0:
+            continue
+        stt, n = abi.pa_poll_end(s.h)
+        seen.append(n)
+        if stt == abi.PA_DONE:
+            assert abi.pa_poll_end(s.h) == (abi.PA_DONE, 0)
+            break
+    assert seen == counts
+    assert torch.equal(host, want.cpu())
+    assert torch.equal(s.result(), want)
+    assert np.array_equal(s.iter_log(), log) and s.nfe() == nfe

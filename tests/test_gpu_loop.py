@@ -1,0 +1,201 @@
+"""The device-driven generation loop (pa_loop_*): a CUDA graph whose
+conditional WHILE node repeats two captured iterations until every trajectory
+has reached T (Sec. 2.1's outer loop, Eq. 1 and 2, run by the GPU). Each case
+compares the loop with the synchronous host-driven run of the same handle bit
+for bit: final states, iteration log, NFE and hits."""
+import numpy as np
+import pytest
+
+import workload as W
+from paper_2609_36522_gb300 import abi
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_36522_gb300 import build as pa_build
+    pa_build.build()
+
+
+def _setup(w, anderson=0, adapt=None, eta=0.0):
+    import torch
+    from paper_2609_36522_gb300.solver import Solver, GmmDenoiser
+    a, x0, mu = W.inputs(w)
+    st = torch.cuda.Stream()
+    s = Solver(w.T, w.window, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=st)
+    g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, w.batch * s.window, stream=st)
+    eps = torch.empty(w.batch * s.window, w.D, dtype=torch.float32, device="cuda")
+    if anderson:
+        s.set_anderson(anderson)
+    if adapt:
+        s.set_cache_adaptation(*adapt)
+    if eta:
+        gen = torch.Generator(device="cuda").manual_seed(7)
+        s.set_noise(eta, torch.randn(w.batch * w.T * w.D, generator=gen, device="cuda"))
+    torch.cuda.synchronize()
+
+    def denoise(bx, mb, nm):
+        g.eps(bx, mb, nm, eps)
+        return eps
+
+    return s, g, eps, torch.from_numpy(x0).cuda(), denoise
+
+
+def _sync(s, x0, denoise):
+    s.init(x0)
+    while True:
+        plan = s.step()
+        if plan is None:
+            break
+        s.submit_eps(denoise(plan.batch_x_ptr, plan.miss_bt_ptr, s.n_miss_dev()))
+    st = s.stats()
+    return s.result().clone(), s.iter_log(), st["nfe"], st["hits"], st["iters"]
+
+
+LOOP_CASES = [
+    ("sd15", W.SD15, {}),
+    ("batched", W.BATCHED.with_(T=40), {}),
+    ("large", W.LARGE.with_(T=60), {}),
+    ("tiny", W.TINY, {}),
+    ("sd15 anderson", W.SD15.with_(T=60), {"anderson": 1}),
+    ("batched adaptive", W.BATCHED.with_(T=40), {"adapt": (0.5, 0.2, 0.0, 1.0)}),
+    ("ddim eta 1", W.SD15.with_(T=50, window=24), {"eta": 1.0}),
+]
+
+
+@pytest.mark.parametrize("name,w,kw", LOOP_CASES, ids=[c[0] for c in LOOP_CASES])
+def test_loop_equals_host_driven_run(name, w, kw):
+    """generate() through the device loop, twice in a row and then with an
+    odd start (eager iterations first, the loop continuing from an even
+    count), gives the host-driven run's x_T, log, NFE and hits."""
+    import torch
+    s, g, eps, x0, denoise = _setup(w, **kw)
+    want, log, nfe, hits, iters = _sync(s, x0, denoise)
+    for _ in range(2):
+        out = s.generate(x0, denoise)
+        assert s.generate_path() == "device loop", s.__dict__.get("loop_error")
+        assert torch.equal(out, want)
+        st = s.stats()
+        assert np.array_equal(s.iter_log(), log)
+        assert (st["nfe"], st["hits"], st["iters"]) == (nfe, hits, iters)
+    # two eager iterations, then the loop from there
+    s.init(x0)
+    for _ in range(2):
+        bx, mb, nm = s.step_async()
+        s.submit_eps(denoise(bx, mb, nm))
+    abi.pa_loop_launch(s.h)
+    stt, n = abi.pa_poll_result(s.h, out.data_ptr())
+    assert stt == abi.PA_DONE and n == 0
+    assert torch.equal(out, want)
+    assert np.array_equal(s.iter_log(), log)
+    s.close()
+    g.close()
+
+
+def test_loop_generations_in_flight():
+    """generate(wait=False) keeps up to two generations queued; each output
+    equals the host-driven run of its own x_init, and finish() checks the
+    rest."""
+    import torch
+    w = W.BATCHED.with_(T=40)
+    s, g, eps, x0, denoise = _setup(w)
+    inits = [x0, x0.flip(0).contiguous(), (0.5 * x0).contiguous(), x0.roll(1, dims=1).contiguous()]
+    wants = [_sync(s, xi, denoise)[0] for xi in inits]
+    outs = [torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory() for _ in inits]
+    s.generate(inits[0], denoise, out=outs[0])  # the capture
+    for xi, o in zip(inits, outs):
+        o.fill_(float("nan"))
+        s.generate(xi, denoise, out=o, wait=False)
+    s.finish()
+    for o, want in zip(outs, wants):
+        assert torch.equal(o, want.cpu())
+    s.close()
+    g.close()
+
+
+def test_loop_call_order_and_settings():
+    """PA_ERR_STATE: pa_loop_capture_end with no capture, a second
+    capture_begin, a launch with nothing captured, a body of one iteration
+    (the capture is closed and the stream works after it), kernel timing
+    enabled, an odd iteration count, a setter during a capture, host
+    stepping after a launch, a launch not preceded by pa_init. A setter
+    drops the loop."""
+    import torch
+    w = W.SD15.with_(T=40)
+    s, g, eps, x0, denoise = _setup(w)
+
+    def state_error(f, *a):
+        with pytest.raises(abi.PaError) as e:
+            f(*a)
+        assert e.value.status == abi.PA_ERR_STATE
+
+    state_error(abi.pa_loop_capture_end, s.h)
+    state_error(abi.pa_loop_launch, s.h)
+    state_error(abi.pa_loop_capture_begin, s.h)   # before pa_init
+    s.init(x0)
+    bx, mb, nm = s.step_async()
+    s.submit_eps(denoise(bx, mb, nm))
+    state_error(abi.pa_loop_capture_begin, s.h)   # odd iteration count
+    s.init(x0)
+    abi.pa_set_kernel_timing(s.h, 1)
+    state_error(abi.pa_loop_capture_begin, s.h)
+    abi.pa_set_kernel_timing(s.h, 0)
+    abi.pa_loop_capture_begin(s.h)
+    state_error(abi.pa_loop_capture_begin, s.h)
+    state_error(abi.pa_set_update_kernel, s.h, 2)
+    with torch.cuda.stream(s.stream):
+        bx, mb, nm = s.step_async()
+        s.submit_eps(denoise(bx, mb, nm))
+    state_error(abi.pa_loop_capture_end, s.h)     # one iteration only: closed, nothing kept
+    state_error(abi.pa_loop_launch, s.h)
+    want, log, nfe, hits, iters = _sync(s, x0, denoise)  # the stream and the handle still work
+    out = s.generate(x0, denoise)
+    assert torch.equal(out, want)
+    state_error(s.step_async)                     # host stepping closed after a launch ...
+    s.init(x0)                                    # ... until pa_init
+    abi.pa_loop_launch(s.h)
+    state_error(abi.pa_loop_launch, s.h)          # a second launch without pa_init
+    stt, n = abi.pa_poll_result(s.h, out.data_ptr())
+    assert stt == abi.PA_DONE and torch.equal(out, want)
+    abi.pa_set_update_kernel(s.h, 2)              # drops the loop
+    s.init(x0)
+    state_error(abi.pa_loop_launch, s.h)
+    s.close()
+    g.close()
+
+
+def test_loop_ends_on_a_device_error():
+    """With the device-side wait limit at zero the staged update kernel's
+    bounded waits (segment form) give up at once: the loop test sees the status and ends
+    the loop (the launch returns); the poll reports PA_ERR_TIMEOUT, and after
+    pa_init the handle reproduces the clean run through the loop."""
+    import torch
+    w = W.SD15.with_(T=30, window=30)
+    s, g, eps, x0, denoise = _setup(w)
+    s.set_update_kernel(101)  # the staged segment form: its row copies wait on mbarriers
+    want = _sync(s, x0, denoise)[0]
+    abi.pa_debug_set_wait_limit(s.h, 0)
+    s.init(x0)
+    for _ in range(2):
+        bx, mb, nm = s.step_async()
+        s.submit_eps(denoise(bx, mb, nm))
+    s.init(x0)
+    abi.pa_loop_capture_begin(s.h)
+    with torch.cuda.stream(s.stream):
+        for _ in range(2):
+            bx, mb, nm = s.step_async()
+            s.submit_eps(denoise(bx, mb, nm))
+    abi.pa_loop_capture_end(s.h)
+    s.init(x0)
+    abi.pa_loop_launch(s.h)
+    out = torch.empty_like(want)
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_poll_result(s.h, out.data_ptr())
+    assert e.value.status == abi.PA_ERR_TIMEOUT
+    abi.pa_debug_set_wait_limit(s.h, 1 << 17)     # drops the loop
+    s._drop_graphs()
+    assert torch.equal(s.generate(x0, denoise), want)
+    assert s.stats()["device_status"] == 0
+    s.close()
+    g.close()
