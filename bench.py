@@ -74,9 +74,9 @@ NOMINAL_HBM_GBS = 8000.0
 NCU_TRAFFIC = {
     # per iteration: k_update_lean + k_plan_gather read + write bytes, averaged
     # over the first generation's launches
-    ("2e7808ed5d540455", "sd15"): 8251136,       # 6,246,912 + 2,004,224 (no DRAM writes)
-    ("2e7808ed5d540455", "batched"): 30266923,   # 24,573,568 + 5,693,355
-    ("2e7808ed5d540455", "large"): 79748608,     # 70,906,697 + 8,841,911
+    ("de8bf09d1e38c9d5", "sd15"): 8257472,       # 6,253,760 + 2,003,712 (no DRAM writes)
+    ("de8bf09d1e38c9d5", "batched"): 30268459,   # 24,576,256 + 5,692,203
+    ("de8bf09d1e38c9d5", "large"): 79785107,     # 70,941,550 + 8,843,557
 }
 
 
@@ -508,7 +508,7 @@ def run_ours(args):
 
     den_events = []   # (before, after) the denoiser call of every iteration, timed graph only
     den_ms = [0.0]    # their total over the timed replays
-    init_launches = 2                     # pa_init: first plan and its gather
+    init_launches = 1                     # pa_init: one kernel (first plan, its batch, cleared sums)
 
     def capture(timed):
         """-> (graph, kernels launched per iteration inside it)"""
@@ -518,7 +518,7 @@ def run_ours(args):
         l0 = s.stats()["launches"] + g.launches()
         gr = torch.cuda.CUDAGraph()
         with torch.cuda.graph(gr, stream=stream):
-            s.init(x_dev)                 # x_init copy, sums cleared, first plan and its gather
+            s.init(x_dev)                 # x_init copy, then the first plan, its batch and the cleared sums
             for _ in range(n_iters):
                 if not timed:
                     one_iteration()
@@ -789,8 +789,9 @@ def run_ours(args):
     # step copies x_init in from pinned host memory (pa_init), runs the
     # generation and copies x_T out to pinned host memory (pa_result), with
     # host time and device events around the whole loop. Headline: one
-    # Solver.generate call per step through the device-driven loop (pa_init,
-    # pa_loop_launch, pa_poll_begin: no host round trip inside a generation),
+    # Solver.generate call per step through the device-driven loop
+    # (pa_loop_launch: x_init copied in, pa_init's kernel, one graph launch; pa_poll_begin:
+    # no host round trip inside a generation),
     # without waiting, so that each generation is queued behind the previous
     # one's poll (at most two in flight, each checked); finish() at the end.
     # Beside it: the same calls waiting for every generation, and the
@@ -818,9 +819,9 @@ def run_ours(args):
 
         def run_generate(wait=False):
             for _ in range(reps):
-                s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK, wait=wait)
+                s.generate(x_host, denoise, out=out_host, wait=wait)
             s.finish()
-            return reps * (1 if s.generate_path() == "device loop" else -(-n_iters // E2E_CHUNK))
+            return reps * (1 if s.generate_path() == "device loop" else -(-n_iters // s.last_chunk))
 
         def run_eager():
             polls = 0
@@ -837,7 +838,7 @@ def run_ours(args):
                 s.result(out_host)
             return polls
 
-        s.generate(x_host, denoise, out=out_host, chunk=E2E_CHUNK)   # capture outside the timed loop
+        s.generate(x_host, denoise, out=out_host)   # body length learned and loop captured outside the timing
         assert np.array_equal(out_host.numpy(), x_cached), "generate() differs from the graph-replayed generation"
         e2e_s, polls = timed(run_generate)
         assert np.array_equal(out_host.numpy(), x_cached), "pipelined generate() differs"
@@ -848,18 +849,22 @@ def run_ours(args):
         units_g, secs_g = aggregate(reps * n_iters, eager_s)
         e2e = {"value": units_e / secs_e, "unit": UNIT,
                "h2d_bytes_per_step": int(w.batch * w.D * 4),
-               "d2h_bytes_per_step": int((polls // reps) * (w.batch * w.D * 4 + 32)),
+               "d2h_bytes_per_step": int((polls // reps) * (w.batch * w.D * 4 + 40)),  # x_T and the 40-byte counters
                "steps": reps,
-               "api": ("Solver.generate(wait=False) per step: pa_init (host x_init), pa_loop_launch (a CUDA "
-                       "graph whose conditional WHILE node repeats two captured iterations -- pa_step_async, "
-                       "pa_gmm_eps, pa_submit_eps -- until every trajectory has reached T), pa_poll_begin "
+               "api": (f"Solver.generate(wait=False) per step: pa_loop_launch (host x_init copied in, "
+                       f"pa_init's kernel, one launch of a CUDA graph whose conditional WHILE node repeats "
+                       f"{s.last_chunk} captured iterations (the iteration count of one host-driven "
+                       f"generation at capture, rounded up to even) -- pa_step_async, pa_gmm_eps, "
+                       f"pa_submit_eps -- until "
+                       f"every trajectory has reached T), pa_poll_begin "
                        "(host x_T and the counters); each generation's poll read and checked once the next "
                        "generation is queued, Solver.finish() after the last"
                        if s.generate_path() == "device loop" else
-                       f"Solver.generate: {E2E_CHUNK} iterations captured as a CUDA graph, replayed with "
+                       f"Solver.generate: {s.last_chunk} iterations captured as a CUDA graph, replayed with "
                        f"pa_poll_result per replay (the driver refused the conditional graph node: "
                        f"{s.__dict__.get('loop_error')})"),
                "generate_path": s.generate_path(),
+               "loop_body_iterations": s.last_chunk,
                "waiting_value": units_w / secs_w,
                "waiting_api": "the same with generate(wait=True): the host waits for each generation's poll",
                "eager_value": units_g / secs_g,

@@ -30,7 +30,10 @@
  *    bytes (256-byte aligned); the library never calls cudaMalloc. Pointers
  *    returned by pa_step stay valid until the next pa_submit_eps/pa_destroy.
  *  - Streams: every kernel and copy of a solver is issued on the stream given
- *    to pa_create (NULL = legacy default stream).
+ *    to pa_create (NULL = legacy default stream). A replay of a CUDA graph
+ *    captured from that stream must be launched on it too: work of one handle
+ *    running on two streams at once races on its workspace (torn plans and
+ *    miss lists, which the kernels do not guard against).
  *  - Errors: every call returns a pa_status; nothing throws across the ABI.
  *    Device-side failures (a bounded wait that ran out, an index check) are
  *    recorded in a device status word and reported by the next call that
@@ -207,33 +210,39 @@ PA_API pa_status pa_poll_end(pa_solver* s, int* n_active);
 
 /* The device-driven generation loop: Sec. 2.1's outer loop (slide the window
  * until every trajectory has reached T, Eq. 1 and 2) run by the GPU itself,
- * with no host round trip per iteration or per chunk. After pa_init (the
- * iteration count must be even), pa_loop_capture_begin starts capturing the
- * solver's stream into the body of a CUDA graph's conditional WHILE node; the
- * caller then issues exactly two iterations (pa_step_async, its denoiser's
+ * with no host round trip per iteration or per chunk. pa_loop_capture_begin
+ * (after pa_init or any even number of iterations) builds a CUDA graph of one
+ * conditional WHILE node and starts capturing the solver's stream into the
+ * node's body; the caller then
+ * issues an even number n >= 2 of iterations (pa_step_async, its denoiser's
  * launches on the solver's stream reading the miss count on the device,
- * pa_submit_eps; twice: the iterations alternate two plan copies); and
- * pa_loop_capture_end appends a one-thread kernel that sets the node's
- * condition (repeat while a trajectory is active, the device status is clean
- * and fewer than T / 2 + 2 passes have run: the window advances at least one
- * step per iteration, so T iterations always suffice, and the pass limit
- * bounds the loop whatever the counters say), closes the capture and
- * instantiates the graph. Nothing runs during the capture, and the host
- * state returns to what it was at pa_loop_capture_begin. pa_loop_launch
- * enqueues the whole loop after a pa_init (any even iteration count): on
- * return the host may enqueue pa_poll_begin (or call pa_poll_result); host
- * stepping (pa_step_async) is refused until the next pa_init. The captured
- * launches carry the settings of the capture: every setter of this handle
- * drops the loop (and is refused while a capture is open). One loop per
- * handle; a new capture replaces it. Errors: PA_ERR_STATE for a call out of
- * order (no capture open, a body that did not hold exactly two iterations,
- * kernel timing enabled: its events cannot sit in a loop body, a stream
- * already being captured); PA_ERR_CUDA where the driver refuses the
- * conditional node or its instantiation (the capture is closed either way
- * and the stream stays usable). */
+ * pa_submit_eps; an even number because the iterations alternate two plan
+ * copies); pa_loop_capture_end appends a one-thread kernel that sets the
+ * node's condition (repeat while a trajectory is active, the device status is
+ * clean and fewer than T / n + 2 passes have run: the window advances at
+ * least one step per iteration, so T iterations always suffice, and the pass
+ * limit bounds the loop whatever the counters say; iterations after the end
+ * do nothing), closes the capture and instantiates the graph. Nothing runs
+ * during the capture, and the host state returns to what it was at
+ * pa_loop_capture_begin. pa_loop_launch(s, x_init) is pa_init followed by the
+ * whole loop: it enqueues the copy of x_init ([batch][D] fp32, HOST or
+ * DEVICE) into state 0, pa_init's kernel (the first plan, its batch, cleared
+ * sums and counters, the loop's pass counter among them) and one launch of
+ * the graph, and returns; then
+ * pa_poll_begin (or pa_poll_result) reads the outcome. Host stepping
+ * (pa_step_async) is refused until the next pa_init. The captured launches
+ * carry the settings of the capture: every setter of this handle drops the
+ * loop (and is refused while a capture is open). One loop per handle; a new
+ * capture replaces it. Errors: PA_ERR_ARG for NULL arguments; PA_ERR_STATE
+ * for a call out of order (no capture open, a body of an odd number of
+ * iterations or none, kernel timing enabled: its events cannot sit in a loop
+ * body, a stream already being captured, a launch between pa_step_async and
+ * pa_submit_eps or with nothing captured); PA_ERR_CUDA where the driver
+ * refuses the conditional node or its instantiation (the capture is closed
+ * either way and the stream stays usable). */
 PA_API pa_status pa_loop_capture_begin(pa_solver* s);
 PA_API pa_status pa_loop_capture_end(pa_solver* s);
-PA_API pa_status pa_loop_launch(pa_solver* s);
+PA_API pa_status pa_loop_launch(pa_solver* s, const float* x_init);
 
 /* Network evaluations so far: the sum over iterations of the misses, i.e. of
  * |M| of Eq. 5 (hits reuse the cached eps of Eq. 6 and cost no evaluation),

@@ -70,7 +70,7 @@ _PROTOS = {
     "pa_poll_end": (C.c_int, [VP, C.POINTER(C.c_int)]),
     "pa_loop_capture_begin": (C.c_int, [VP]),
     "pa_loop_capture_end": (C.c_int, [VP]),
-    "pa_loop_launch": (C.c_int, [VP]),
+    "pa_loop_launch": (C.c_int, [VP, VP]),
     "pa_nfe": (C.c_int64, [VP]),
     "pa_stats": (C.c_int, [VP, C.POINTER(PaStats)]),
     "pa_iter_log": (C.c_int, [VP, C.POINTER(C.c_int32), C.c_int, C.POINTER(C.c_int)]),
@@ -241,8 +241,8 @@ def pa_loop_capture_end(h):
     return _check("pa_loop_capture_end", lib().pa_loop_capture_end(h))
 
 
-def pa_loop_launch(h):
-    return _check("pa_loop_launch", lib().pa_loop_launch(h))
+def pa_loop_launch(h, x_init_ptr):
+    return _check("pa_loop_launch", lib().pa_loop_launch(h, _dptr(x_init_ptr)))
 
 
 def pa_nfe(h):

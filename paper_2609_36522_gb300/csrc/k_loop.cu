@@ -10,20 +10,19 @@
 namespace pa {
 namespace {
 
-__global__ void k_loop_cond(cudaGraphConditionalHandle h, const Ctl* ctl, int32_t* passes, int32_t limit) {
+__global__ void k_loop_cond(cudaGraphConditionalHandle h, Ctl* ctl, int32_t limit) {
+  pdl_wait();  // the counters come from the planning kernel just before
   if (threadIdx.x != 0) return;
-  const int32_t c = *passes + 1;
-  *passes = c;
+  const int32_t c = ctl->loop_passes + 1;  // cleared by the graph's memset node at each launch
+  ctl->loop_passes = c;
   const bool more = ctl->n_active > 0 && ctl->status == kDevOk && c < limit;
   cudaGraphSetConditional(h, more ? 1u : 0u);
 }
 
 }  // namespace
 
-cudaError_t launch_loop_cond(cudaGraphConditionalHandle h, const Ctl* ctl, int32_t* passes, int32_t limit,
-                             cudaStream_t st) {
-  k_loop_cond<<<1, 32, 0, st>>>(h, ctl, passes, limit);
-  return cudaGetLastError();
+cudaError_t launch_loop_cond(cudaGraphConditionalHandle h, Ctl* ctl, int32_t limit, cudaStream_t st) {
+  return launch_ex(k_loop_cond, dim3(1), dim3(32), 0, st, 0, h, ctl, limit);
 }
 
 }  // namespace pa

@@ -26,47 +26,6 @@ __device__ __forceinline__ void set_status(Ctl* c, int code) {
 }
 
 // ---------------------------------------------------------------------------
-// First iteration (after pa_init): every timestep of every first window enters
-// for the first time, hence is a miss (Sec. 2.2). States 1..p are lazy copies
-// of state 0 = x_init, so the frontier e starts at 0.
-__global__ void k_init_plan(Dev d) {
-  const int p0 = min(d.P, d.T);
-  for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
-    Traj tr{};
-    tr.t = 0; tr.p = p0; tr.e = 0; tr.done = 0; tr.m = p0; tr.h1 = 0;  // no entries yet: ne = nh = 0
-    d.traj[b] = tr;  // copy 0: the plan of iteration 0
-    if (d.adapt) d.tau[b] = d.cache_thresh;  // tau_cache starts at the configured value
-  }
-  for (int q = threadIdx.x; q < d.B * d.P; q += blockDim.x) {
-    const int b = q / d.P, j = q % d.P;
-    if (j < p0) {
-      const int r = b * p0 + j;
-      d.rank[q] = r;
-      d.miss_bt[2 * r] = b;
-      d.miss_bt[2 * r + 1] = j;
-    } else {
-      d.rank[q] = -1;
-    }
-  }
-  if (threadIdx.x == 0) {
-    Ctl c{};
-    c.n_miss = d.B * p0;
-    c.n_active = d.B;
-    c.iter = 0;
-    c.status = kDevOk;
-    c.nfe = (long long)d.B * p0;
-    c.hits = 0;
-    *d.ctl = c;
-    PlanCtr pc;
-    pc.n_active = c.n_active;
-    pc.iter = 0;
-    pc.nfe = c.nfe;
-    pc.hits = 0;
-    d.pc[0] = pc;
-  }
-}
-
-// ---------------------------------------------------------------------------
 // a4: batch_x[r] <- x_{miss[r]} for r < n_miss. A lazy state (i > e) reads
 // state e, the value every new tail state was initialised to. Each thread
 // moves kGatherUnroll vectors per row with all loads issued before the stores;
@@ -110,6 +69,67 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d, int par) {
     const int b = d.miss_bt[2 * r], i = d.miss_bt[2 * r + 1];
     copy_row<VEC>(d, b, min(i, tr[b].e), r);
   }
+}
+
+// ---------------------------------------------------------------------------
+// First iteration (after pa_init's copy of x_init into state 0): every
+// timestep of every first window enters for the first time, hence is a miss
+// (Sec. 2.2); states 1..p are lazy copies of state 0 = x_init, so the frontier
+// e starts at 0 and batch row r = b p0 + j is state 0 of trajectory b. One
+// launch on the gather's grid: each CTA copies its part of its batch row; all
+// CTAs together write the ranks and the miss list and clear both sets of the
+// reduction accumulators (the entries that are added into, every
+// kAccStride-th) and the fused step's barrier counter; CTA (0, 0) writes the
+// trajectories, counters and the plan's counter copy 0.
+template <int VEC>
+__global__ void __launch_bounds__(kGatherThreads) k_init(Dev d) {
+  pdl_wait();  // x_init was copied into state 0 just before
+  pdl_trigger();
+  const int p0 = min(d.P, d.T);
+  const int npair = d.B * d.P;
+  const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x;
+  const int64_t step = (int64_t)gridDim.x * gridDim.y * kGatherThreads;
+  for (int64_t q = cta * kGatherThreads + threadIdx.x; q < npair; q += step) {
+    const int b = (int)(q / d.P), j = (int)(q % d.P);
+    if (j < p0) {
+      const int r = b * p0 + j;
+      d.rank[q] = r;
+      d.miss_bt[2 * r] = b;
+      d.miss_bt[2 * r + 1] = j;
+    } else {
+      d.rank[q] = -1;
+    }
+  }
+  for (int64_t q = cta * kGatherThreads + threadIdx.x; q < 4 * (int64_t)npair; q += step) {
+    d.acc[q * kAccStride] = 0.0;  // [set][err, dist][B][P]
+    if (d.taa) d.taa_acc[q * kAccStride] = 0.0;
+  }
+  if (cta == 0) {
+    for (int b = threadIdx.x; b < d.B; b += blockDim.x) {
+      Traj tr{};
+      tr.t = 0; tr.p = p0; tr.e = 0; tr.done = 0; tr.m = p0; tr.h1 = 0;  // no entries yet: ne = nh = 0
+      d.traj[b] = tr;  // copy 0: the plan of iteration 0
+      if (d.adapt) d.tau[b] = d.cache_thresh;  // tau_cache starts at the configured value
+    }
+    if (threadIdx.x == 0) {
+      *d.gbar = 0ull;
+      Ctl c{};
+      c.n_miss = d.B * p0;
+      c.n_active = d.B;
+      c.iter = 0;
+      c.status = kDevOk;
+      c.nfe = (long long)d.B * p0;
+      c.hits = 0;
+      *d.ctl = c;
+      PlanCtr pc;
+      pc.n_active = c.n_active;
+      pc.iter = 0;
+      pc.nfe = c.nfe;
+      pc.hits = 0;
+      d.pc[0] = pc;
+    }
+  }
+  for (int r = blockIdx.y; r < d.B * p0; r += gridDim.y) copy_row<VEC>(d, r / p0, 0, r);
 }
 
 // ---------------------------------------------------------------------------
@@ -357,11 +377,6 @@ __global__ void k_gap() {
 
 cudaError_t launch_gap(cudaStream_t st) { return launch_ex(k_gap, dim3(1), dim3(32), 0, st, 0); }
 
-cudaError_t launch_init_plan(const Dev& d, cudaStream_t st) {
-  k_init_plan<<<1, 256, 0, st>>>(d);
-  return cudaGetLastError();
-}
-
 namespace {
 dim3 gather_grid(const Dev& d) {
   const int rows = min(d.B * d.P, 65535);
@@ -376,6 +391,12 @@ cudaError_t launch_gather(const Dev& d, int par, cudaStream_t st) {
   const dim3 g = gather_grid(d);
   if (d.D % 4 == 0) return launch_ex(k_gather<4>, g, dim3(kGatherThreads), 0, st, 0, d, par);
   return launch_ex(k_gather<1>, g, dim3(kGatherThreads), 0, st, 0, d, par);
+}
+
+cudaError_t launch_init(const Dev& d, cudaStream_t st) {
+  const dim3 g = gather_grid(d);
+  if (d.D % 4 == 0) return launch_ex(k_init<4>, g, dim3(kGatherThreads), 0, st, 0, d);
+  return launch_ex(k_init<1>, g, dim3(kGatherThreads), 0, st, 0, d);
 }
 
 cudaError_t launch_plan(const Dev& d, int par, cudaStream_t st, int* launches) {

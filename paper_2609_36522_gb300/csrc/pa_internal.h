@@ -50,6 +50,8 @@ struct Ctl {
   int32_t status;     // kDev* code
   long long nfe;
   long long hits;
+  int32_t loop_passes;  // body passes of the device-driven loop since its launch
+  int32_t reserved;
 };
 
 // The counters a decision starts from. Kept in two copies, like the
@@ -317,7 +319,7 @@ __device__ __forceinline__ bool grid_sync(unsigned long long* ctr, unsigned long
 // Kernel launchers (k_solver.cu). Each returns the launch error. par = k mod 2
 // for iteration k: the copy of the plan the kernel reads (and the accumulator
 // set the update kernels add into).
-cudaError_t launch_init_plan(const Dev& d, cudaStream_t st);
+cudaError_t launch_init(const Dev& d, cudaStream_t st);  // first plan, its batch, cleared sums
 cudaError_t launch_gather(const Dev& d, int par, cudaStream_t st);
 cudaError_t launch_update_plain(const Dev& d, const float* batch_eps, int par, cudaStream_t st);
 // the decision after iteration k (par = k mod 2) and the gather of iteration k+1

@@ -7,9 +7,8 @@
 
 namespace pa {
 
-// One thread: passes += 1, then the node's condition := n_active > 0 and the
-// device status clean and passes < limit.
-cudaError_t launch_loop_cond(cudaGraphConditionalHandle h, const Ctl* ctl, int32_t* passes, int32_t limit,
-                             cudaStream_t st);
+// One thread: ctl->loop_passes += 1, then the node's condition := n_active > 0
+// and the device status clean and loop_passes < limit.
+cudaError_t launch_loop_cond(cudaGraphConditionalHandle h, Ctl* ctl, int32_t limit, cudaStream_t st);
 
 }  // namespace pa

@@ -55,7 +55,6 @@ struct pa_solver {
   cudaGraph_t loop_graph;
   cudaGraphExec_t loop_exec;
   cudaGraphConditionalHandle loop_cond;
-  int32_t* loop_passes;    // device: body passes of the running launch
   bool loop_capturing;     // between pa_loop_capture_begin and _end
   bool looped;             // a loop was launched since pa_init: host-side stepping is closed
   int64_t loop_k0, loop_launches0;  // s->k and s->launches when the capture began
@@ -171,6 +170,14 @@ bool loop_busy(pa_solver* s, const char* where) {
   }
   pa::set_error(std::string(where) + ": a generation loop is being captured");
   return true;
+}
+
+// Enqueue the copy of x_init ([batch][D], host or device) into state 0 of
+// every trajectory; the rest of the first window is lazy.
+cudaError_t copy_x_init(pa_solver* s, const float* x_init) {
+  const pa::Dev& d = s->d;
+  return cudaMemcpy2DAsync(d.X, (size_t)(d.P + 1) * d.D * sizeof(float), x_init, (size_t)d.D * sizeof(float),
+                           (size_t)d.D * sizeof(float), d.B, cudaMemcpyDefault, s->st);
 }
 
 }  // namespace
@@ -293,7 +300,6 @@ pa_status pa_create(pa_solver** out, int T, int window, const int64_t* latent_sh
   s->loop_graph = nullptr;
   s->loop_exec = nullptr;
   s->loop_cond = 0;
-  s->loop_passes = nullptr;
   s->loop_capturing = s->looped = false;
   s->loop_k0 = s->loop_launches0 = 0;
   cudaError_t e = cudaHostAlloc(reinterpret_cast<void**>(&s->host_ctl), 3 * sizeof(pa::Ctl), cudaHostAllocDefault);
@@ -346,22 +352,12 @@ pa_status pa_set_noise(pa_solver* s, double eta, const float* noise_dev) {
 pa_status pa_init(pa_solver* s, const float* x_init) {
   if (!s) return arg_fail("pa_init: solver is NULL");
   if (!x_init) return arg_fail("pa_init: x_init is NULL");
-  const pa::Dev& d = s->d;
-  // state 0 of every trajectory <- x_init; the rest of the first window is lazy
-  cudaError_t e = cudaMemcpy2DAsync(d.X, (size_t)(d.P + 1) * d.D * sizeof(float), x_init,
-                                    (size_t)d.D * sizeof(float), (size_t)d.D * sizeof(float), d.B,
-                                    cudaMemcpyDefault, s->st);
+  cudaError_t e = copy_x_init(s, x_init);
   if (e != cudaSuccess) return cuda_fail("pa_init: copy x_init", e);
-  // both accumulator sets of the reductions start at zero
-  e = cudaMemsetAsync(d.acc, 0, (size_t)2 * 2 * d.B * d.P * pa::kAccStride * sizeof(double), s->st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(d.gbar, 0, sizeof(unsigned long long), s->st);  // barrier arrivals
-  if (e == cudaSuccess && d.taa)  // both sets of the Anderson Gram sums
-    e = cudaMemsetAsync(d.taa_acc, 0, (size_t)2 * 2 * d.B * d.P * pa::kAccStride * sizeof(double), s->st);
-  if (e != cudaSuccess) return cuda_fail("pa_init: clear sums", e);
-  // the first plan (every timestep a first entry) and its batch
-  e = pa::launch_init_plan(d, s->st);
-  if (e == cudaSuccess) e = pa::launch_gather(d, 0, s->st);
-  s->launches += 2;
+  // the first plan (every timestep a first entry), its batch, both sets of the
+  // reductions' (and the Anderson Gram sums') accumulators cleared: one kernel
+  e = pa::launch_init(s->d, s->st);
+  s->launches += 1;
   if (e != cudaSuccess) return cuda_fail("pa_init: launch", e);
   s->k = 0;
   s->looped = false;
@@ -574,27 +570,19 @@ pa_status pa_loop_capture_begin(pa_solver* s) {
     return PA_ERR_STATE;
   }
   drop_loop(s);
-  if (!s->loop_passes) e = cudaMalloc(reinterpret_cast<void**>(&s->loop_passes), sizeof(int32_t));
-  cudaGraphNode_t clear = nullptr, loop = nullptr;
+  cudaGraphNode_t loop = nullptr;
   cudaGraphNodeParams np = {};
-  if (e == cudaSuccess) e = cudaGraphCreate(&s->loop_graph, 0);
-  // the condition is 1 at every launch: the body runs at least once
+  e = cudaGraphCreate(&s->loop_graph, 0);
+  // the condition is 1 at every launch: the body runs at least once (the
+  // pass counter is cleared by pa_init's kernel, which pa_loop_launch issues
+  // before the graph)
   if (e == cudaSuccess) e = cudaGraphConditionalHandleCreate(&s->loop_cond, s->loop_graph, 1, cudaGraphCondAssignDefault);
-  if (e == cudaSuccess) {
-    cudaMemsetParams mp = {};
-    mp.dst = s->loop_passes;
-    mp.value = 0;
-    mp.elementSize = sizeof(int32_t);
-    mp.width = 1;
-    mp.height = 1;
-    e = cudaGraphAddMemsetNode(&clear, s->loop_graph, nullptr, 0, &mp);
-  }
   if (e == cudaSuccess) {
     np.type = cudaGraphNodeTypeConditional;
     np.conditional.handle = s->loop_cond;
     np.conditional.type = cudaGraphCondTypeWhile;
     np.conditional.size = 1;
-    e = cudaGraphAddNode(&loop, s->loop_graph, &clear, nullptr, 1, &np);
+    e = cudaGraphAddNode(&loop, s->loop_graph, nullptr, nullptr, 0, &np);
   }
   if (e == cudaSuccess)
     e = cudaStreamBeginCaptureToGraph(s->st, np.conditional.phGraph_out[0], nullptr, nullptr, 0,
@@ -615,11 +603,12 @@ pa_status pa_loop_capture_end(pa_solver* s) {
     pa::set_error("pa_loop_capture_end: no capture is open");
     return PA_ERR_STATE;
   }
-  const bool two = s->state == St::Ready && s->k == s->loop_k0 + 2;
+  const int64_t n_body = s->k - s->loop_k0;  // iterations in the body
+  const bool two = s->state == St::Ready && n_body >= 2 && n_body % 2 == 0;
   cudaError_t e = cudaSuccess;
   // at most T iterations reach t = T (the window advances by at least one
-  // step in each): T / 2 + 2 passes of two iterations cover them
-  if (two) e = pa::launch_loop_cond(s->loop_cond, s->d.ctl, s->loop_passes, s->d.T / 2 + 2, s->st);
+  // step in each): T / n_body + 2 passes cover them
+  if (two) e = pa::launch_loop_cond(s->loop_cond, s->d.ctl, (int32_t)(s->d.T / n_body + 2), s->st);
   cudaGraph_t body = nullptr;
   const cudaError_t e2 = cudaStreamEndCapture(s->st, &body);
   if (e == cudaSuccess) e = e2;
@@ -629,8 +618,8 @@ pa_status pa_loop_capture_end(pa_solver* s) {
   if (s->state == St::Stepped) s->state = St::Ready;
   if (e == cudaSuccess && !two) {
     drop_loop(s);
-    pa::set_error("pa_loop_capture_end: the body must hold exactly two iterations "
-                  "(pa_step_async, the denoiser, pa_submit_eps, twice)");
+    pa::set_error("pa_loop_capture_end: the body must hold an even number of iterations, at least two "
+                  "(pa_step_async, the denoiser, pa_submit_eps each)");
     return PA_ERR_STATE;
   }
   if (e == cudaSuccess) e = cudaGraphInstantiate(&s->loop_exec, s->loop_graph, 0);
@@ -642,17 +631,21 @@ pa_status pa_loop_capture_end(pa_solver* s) {
   return PA_OK;
 }
 
-pa_status pa_loop_launch(pa_solver* s) {
+pa_status pa_loop_launch(pa_solver* s, const float* x_init) {
   if (!s) return arg_fail("pa_loop_launch: solver is NULL");
+  if (!x_init) return arg_fail("pa_loop_launch: x_init is NULL");
   if (!s->loop_exec) {
     pa::set_error("pa_loop_launch: no generation loop has been captured");
     return PA_ERR_STATE;
   }
-  if (s->state != St::Ready || s->looped || s->loop_capturing || ((s->k ^ s->loop_k0) & 1))
-    return state_fail("pa_loop_launch");
-  const cudaError_t e = cudaGraphLaunch(s->loop_exec, s->st);
+  if (s->state == St::Stepped || s->loop_capturing) return state_fail("pa_loop_launch");
+  cudaError_t e = copy_x_init(s, x_init);
+  if (e == cudaSuccess) e = pa::launch_init(s->d, s->st);  // also clears the loop's pass counter
+  if (e == cudaSuccess) e = cudaGraphLaunch(s->loop_exec, s->st);
   if (e != cudaSuccess) return cuda_fail("pa_loop_launch", e);
+  s->k = 0;
   s->looped = true;
+  s->state = St::Ready;
   return PA_OK;
 }
 
@@ -866,7 +859,6 @@ void pa_destroy(pa_solver* s) {
     (void)cudaGetLastError();
   }
   drop_loop(s);
-  if (s->loop_passes) cudaFree(s->loop_passes);
   if (s->host_ctl) cudaFreeHost(s->host_ctl);
   delete s;
 }

@@ -66,13 +66,16 @@ class Solver:
         self._noise_keepalive = noise
         abi.pa_set_noise(self.h, eta, noise.data_ptr())
 
-    def init(self, x_init):
-        """x_init: [batch][D] fp32 tensor (CUDA or CPU, contiguous)."""
+    def _x_init(self, x_init):
         x = x_init if isinstance(x_init, torch.Tensor) else torch.from_numpy(np.ascontiguousarray(x_init))
         if x.dtype != torch.float32 or not x.is_contiguous() or x.numel() != self.batch * self.D:
             raise ValueError("x_init must be a contiguous float32 [batch][D] tensor")
         self._x_init_keepalive = x
-        abi.pa_init(self.h, x.data_ptr())
+        return x
+
+    def init(self, x_init):
+        """x_init: [batch][D] fp32 tensor (CUDA or CPU, contiguous)."""
+        abi.pa_init(self.h, self._x_init(x_init).data_ptr())
 
     def step(self):
         """-> None when done, else a Plan (M, batch_x [M][D], miss_bt [M][2], raw pointers)."""
@@ -122,7 +125,7 @@ class Solver:
         st, n = abi.pa_poll_result(self.h, out.data_ptr())
         return n
 
-    def generate(self, x_init, denoise, out=None, chunk=4, wait=True):
+    def generate(self, x_init, denoise, out=None, chunk=None, wait=True):
         """One whole generation in one call: x_init [batch][D] (CUDA tensor or
         pinned host tensor) in, x_T out (into ``out``, a CUDA or pinned host
         tensor, else a new CUDA tensor).
@@ -133,12 +136,21 @@ class Solver:
         tensor it wrote; it must write the same buffer on every call, allocate
         nothing and be capturable in a CUDA graph.
 
-        The first call per denoiser captures two iterations as the body of a
-        device-side loop (``pa_loop_capture_begin/_end``: a CUDA graph whose
-        conditional WHILE node repeats the body until every trajectory has
-        reached T). Each call then enqueues ``pa_init`` (x_init copied in),
-        ``pa_loop_launch`` and ``pa_poll_begin`` (x_T and the counters copied
-        out): no host round trip inside a generation. With ``wait`` the call
+        The first call per (denoiser, chunk) captures ``chunk`` (even)
+        iterations as the body of a device-side loop
+        (``pa_loop_capture_begin/_end``: a CUDA graph whose conditional WHILE
+        node repeats the body until every trajectory has reached T;
+        iterations after that, up to the end of the pass, do nothing). Each
+        pass of the body costs a few microseconds of loop control and each
+        iteration past the end a few more, so the best body holds the
+        generation's iteration count: with ``chunk=None`` the first call per
+        denoiser runs one host-driven generation of its x_init and takes its
+        iteration count, rounded up to even, as the body (later generations
+        that need more iterations simply take more passes). Each
+        call then enqueues ``pa_loop_launch`` (x_init copied in, pa_init's
+        kernel, one launch of the graph) and ``pa_poll_begin`` (x_T and the
+        counters copied out): no host round trip inside a generation. With
+        ``wait`` the call
         returns after that poll; without it, it returns at once with at most
         two generations in flight (a third call first waits for the oldest and
         checks it), and ``finish()`` waits for the rest; ``out`` and x_init
@@ -150,15 +162,18 @@ class Solver:
         waiting). The captured launches carry the solver's settings of the
         capture: the setters of this class drop them; a denoiser's own settings
         must stay as they were captured (or pass a new callable)."""
+        if chunk is None:
+            chunk = self._auto_chunk(x_init, denoise)
         if chunk < 2 or chunk % 2:
             raise ValueError("chunk must be a positive even number (iterations alternate two plan copies)")
+        self.last_chunk = chunk
         out = self._out(out)
-        if self.__dict__.get("_loop_for") is not denoise and self.__dict__.get("loop_error") is None:
-            self._capture_loop(x_init, denoise)
-        if self.__dict__.get("_loop_for") is denoise:
+        key = (denoise, chunk)
+        if self.__dict__.get("_loop_for") != key and self.__dict__.get("loop_error") is None:
+            self._capture_loop(x_init, denoise, chunk)
+        if self.__dict__.get("_loop_for") == key:
             pending = self.__dict__.setdefault("_pending", [])
-            self.init(x_init)
-            abi.pa_loop_launch(self.h)
+            abi.pa_loop_launch(self.h, self._x_init(x_init).data_ptr())
             if len(pending) == 2:
                 self._end_poll()
             abi.pa_poll_begin(self.h, out.data_ptr())
@@ -168,7 +183,6 @@ class Solver:
             return out
         self.finish()
         graphs = self.__dict__.setdefault("_gen_graphs", {})
-        key = (denoise, chunk)
         self.init(x_init)
         gr = graphs.get(key)
         if gr is None:
@@ -191,7 +205,26 @@ class Solver:
                 return out
         raise RuntimeError("generate: trajectories did not reach T within T iterations")
 
-    def _capture_loop(self, x_init, denoise):
+    def _auto_chunk(self, x_init, denoise):
+        """The loop body for ``generate(chunk=None)``: the iteration count of
+        one host-driven generation of x_init, rounded up to even (learned once
+        per denoiser; 4 where the loop is not available)."""
+        if self.__dict__.get("loop_error") is not None:
+            return 4
+        auto = self.__dict__.setdefault("_auto", {})
+        if denoise not in auto:
+            self.finish()
+            self.init(x_init)
+            while True:
+                plan = self.step()
+                if plan is None:
+                    break
+                self.submit_eps(denoise(plan.batch_x_ptr, plan.miss_bt_ptr, self.n_miss_dev()))
+            n = int(self.stats()["iters"])
+            auto[denoise] = max(2, n + (n & 1))
+        return auto[denoise]
+
+    def _capture_loop(self, x_init, denoise, chunk):
         self.finish()
         self.init(x_init)
         # one eager iteration first: launch-time set-up (kernel attributes)
@@ -202,7 +235,7 @@ class Solver:
         abi.pa_loop_capture_begin(self.h)
         try:
             with torch.cuda.stream(self.stream):  # torch work of the denoiser lands in the body
-                for _ in range(2):
+                for _ in range(chunk):
                     bx, mb, nm = self.step_async()
                     self.submit_eps(denoise(bx, mb, nm))
         except BaseException:
@@ -218,7 +251,7 @@ class Solver:
                 raise
             self.loop_error = str(e)  # this driver cannot run the loop: replay and poll instead
             return
-        self._loop_for = denoise
+        self._loop_for = (denoise, chunk)
 
     def _end_poll(self):
         pending = self.__dict__.get("_pending", [])
@@ -288,6 +321,7 @@ class Solver:
         self.finish()
         self.__dict__.pop("_gen_graphs", None)
         self.__dict__.pop("_loop_for", None)  # the C setters drop the loop graph itself
+        self.__dict__.pop("_auto", None)      # the settings may change the iteration count
 
     def close(self):
         try:

@@ -83,16 +83,17 @@ def test_launch_counter_and_reductions():
     s.init(x0)
     _run(s, g, eps)
     st = s.stats()
-    # first plan and its gather + per iteration: the update and the planning
-    # kernel (decision fused with the next gather), or the fused step
+    # the first plan with its batch (one kernel) + per iteration: the update
+    # and the planning kernel (decision fused with the next gather), or the
+    # fused step
     assert st["update_kernel"] == 2
-    assert st["launches"] == 2 + 2 * st["iters"]
+    assert st["launches"] == 1 + 2 * st["iters"]
     s.set_update_kernel(3)
     s.init(x0)
     _run(s, g, eps)
     st2 = s.stats()
     assert st2["update_kernel"] == 3
-    assert st2["launches"] - st["launches"] == 2 + st2["iters"]
+    assert st2["launches"] - st["launches"] == 1 + st2["iters"]
     err, dl = s.last_reductions()
     assert np.isfinite(err).all() and np.isfinite(dl).all()
 

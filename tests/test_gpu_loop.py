@@ -55,6 +55,9 @@ def _sync(s, x0, denoise):
 
 LOOP_CASES = [
     ("sd15", W.SD15, {}),
+    ("sd15 body 2", W.SD15, {"chunk": 2}),
+    ("large auto body", W.LARGE.with_(T=60), {"chunk": None}),
+    ("batched body 6", W.BATCHED.with_(T=40), {"chunk": 6}),
     ("batched", W.BATCHED.with_(T=40), {}),
     ("large", W.LARGE.with_(T=60), {}),
     ("tiny", W.TINY, {}),
@@ -66,25 +69,29 @@ LOOP_CASES = [
 
 @pytest.mark.parametrize("name,w,kw", LOOP_CASES, ids=[c[0] for c in LOOP_CASES])
 def test_loop_equals_host_driven_run(name, w, kw):
-    """generate() through the device loop, twice in a row and then with an
-    odd start (eager iterations first, the loop continuing from an even
-    count), gives the host-driven run's x_T, log, NFE and hits."""
+    """generate() through the device loop (bodies of 4 iterations unless
+    stated), twice in a row and then after eager iterations (the launch
+    starts over from x_init), gives the host-driven run's x_T, log, NFE and
+    hits: iterations run past the end change nothing."""
     import torch
+    kw = dict(kw)
+    chunk = kw.pop("chunk", 4)
     s, g, eps, x0, denoise = _setup(w, **kw)
     want, log, nfe, hits, iters = _sync(s, x0, denoise)
     for _ in range(2):
-        out = s.generate(x0, denoise)
+        out = s.generate(x0, denoise, chunk=chunk)
         assert s.generate_path() == "device loop", s.__dict__.get("loop_error")
+        assert s.last_chunk == (chunk or iters + (iters & 1))
         assert torch.equal(out, want)
         st = s.stats()
         assert np.array_equal(s.iter_log(), log)
         assert (st["nfe"], st["hits"], st["iters"]) == (nfe, hits, iters)
-    # two eager iterations, then the loop from there
+    # eager iterations first: the launch starts over from x_init
     s.init(x0)
-    for _ in range(2):
+    for _ in range(3):
         bx, mb, nm = s.step_async()
         s.submit_eps(denoise(bx, mb, nm))
-    abi.pa_loop_launch(s.h)
+    abi.pa_loop_launch(s.h, x0.data_ptr())
     stt, n = abi.pa_poll_result(s.h, out.data_ptr())
     assert stt == abi.PA_DONE and n == 0
     assert torch.equal(out, want)
@@ -115,12 +122,13 @@ def test_loop_generations_in_flight():
 
 
 def test_loop_call_order_and_settings():
-    """PA_ERR_STATE: pa_loop_capture_end with no capture, a second
-    capture_begin, a launch with nothing captured, a body of one iteration
-    (the capture is closed and the stream works after it), kernel timing
-    enabled, an odd iteration count, a setter during a capture, host
-    stepping after a launch, a launch not preceded by pa_init. A setter
-    drops the loop."""
+    """PA_ERR_STATE: pa_loop_capture_end with no capture, a launch with
+    nothing captured, capture_begin before pa_init, after an odd number of
+    iterations, with kernel timing enabled and while a capture is open, a
+    setter during a capture, a body of one iteration (the capture is closed
+    and the stream works after it), host stepping after a launch, a launch
+    between pa_step_async and pa_submit_eps. Launches back to back each
+    start over; a setter drops the loop."""
     import torch
     w = W.SD15.with_(T=40)
     s, g, eps, x0, denoise = _setup(w)
@@ -131,7 +139,7 @@ def test_loop_call_order_and_settings():
         assert e.value.status == abi.PA_ERR_STATE
 
     state_error(abi.pa_loop_capture_end, s.h)
-    state_error(abi.pa_loop_launch, s.h)
+    state_error(abi.pa_loop_launch, s.h, x0.data_ptr())   # nothing captured
     state_error(abi.pa_loop_capture_begin, s.h)   # before pa_init
     s.init(x0)
     bx, mb, nm = s.step_async()
@@ -148,19 +156,21 @@ def test_loop_call_order_and_settings():
         bx, mb, nm = s.step_async()
         s.submit_eps(denoise(bx, mb, nm))
     state_error(abi.pa_loop_capture_end, s.h)     # one iteration only: closed, nothing kept
-    state_error(abi.pa_loop_launch, s.h)
+    state_error(abi.pa_loop_launch, s.h, x0.data_ptr())
     want, log, nfe, hits, iters = _sync(s, x0, denoise)  # the stream and the handle still work
     out = s.generate(x0, denoise)
     assert torch.equal(out, want)
     state_error(s.step_async)                     # host stepping closed after a launch ...
     s.init(x0)                                    # ... until pa_init
-    abi.pa_loop_launch(s.h)
-    state_error(abi.pa_loop_launch, s.h)          # a second launch without pa_init
+    bx, mb, nm = s.step_async()
+    state_error(abi.pa_loop_launch, s.h, x0.data_ptr())   # between pa_step_async and pa_submit_eps
+    s.submit_eps(denoise(bx, mb, nm))
+    abi.pa_loop_launch(s.h, x0.data_ptr())
+    abi.pa_loop_launch(s.h, x0.data_ptr())        # back to back: each starts over
     stt, n = abi.pa_poll_result(s.h, out.data_ptr())
     assert stt == abi.PA_DONE and torch.equal(out, want)
     abi.pa_set_update_kernel(s.h, 2)              # drops the loop
-    s.init(x0)
-    state_error(abi.pa_loop_launch, s.h)
+    state_error(abi.pa_loop_launch, s.h, x0.data_ptr())
     s.close()
     g.close()
 
@@ -187,8 +197,7 @@ def test_loop_ends_on_a_device_error():
             bx, mb, nm = s.step_async()
             s.submit_eps(denoise(bx, mb, nm))
     abi.pa_loop_capture_end(s.h)
-    s.init(x0)
-    abi.pa_loop_launch(s.h)
+    abi.pa_loop_launch(s.h, x0.data_ptr())
     out = torch.empty_like(want)
     with pytest.raises(abi.PaError) as e:
         abi.pa_poll_result(s.h, out.data_ptr())
