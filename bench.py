@@ -663,7 +663,8 @@ def run_ours(args):
     cold_gbps = float(step_bytes.sum()) / (float(cold_per.sum()) * 1e-6) / 1e9
     sha = kernel_source_sha()
     tkey = args.workload + ("-bf16" if args.cache_bits == 16 else "") + \
-        ("" if args.cache_thresh is None else f"-c{args.cache_thresh:g}")
+        ("" if args.cache_thresh is None else f"-c{args.cache_thresh:g}") + \
+        ("" if args.update_kernel is None else f"-k{args.update_kernel}")
     traffic = NCU_TRAFFIC.get((sha, tkey))
     step_kernel = {4: "Anderson-mixing update + mix kernel + planning kernel",
                    3: "fused step (update, grid barrier, decision, next batch from registers)",
