@@ -25,6 +25,9 @@ Also reported:
                 the recorded batches;
   uncached      the same generation with tau_cache = 0 (no hits): NFE,
                 iterations and time;
+  hit_heavy     the same generation with tau_cache = 0.1 (the hit path
+                exercised: about a third of the window points hit at the SD
+                shape): NFE, hits, iterations and time;
   e2e           the public API with host buffers (copies inside the timing);
   cpu_baseline  the fp64 oracle on the host cores, one thread and all cores,
                 whole iterations and the solver step with the denoiser's time
@@ -733,39 +736,48 @@ def run_ours(args):
     den_only_us = 1000.0 * den_only / (den_reps * n_iters)
     del g_den
 
-    # ---- uncached run alongside (tau_cache = 0: every window point evaluated)
-    su = make_solver(0.0)
-    un_iters = run_sync(su)
-    un_st = su.stats()
-    su.init(x_dev)
-    one_iteration(su)
-    stream.synchronize()
-    gu = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(gu, stream=stream):
+    # ---- side runs of the same sample: uncached (tau_cache = 0, every window
+    # point evaluated) and hit-heavy (tau_cache = 0.1: the hit path exercised)
+    def side_run(thresh):
+        su = make_solver(thresh)
+        it = run_sync(su)
+        st_ = su.stats()
         su.init(x_dev)
-        for _ in range(un_iters):
-            one_iteration(su)
-    un_ms = 0.0
-    un_reps = max(5, min(args.steps, 50))
-    for r in range(un_reps + 2):
-        if flush is not None:
-            flush.zero_()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        gu.replay()
-        e1.record(stream)
-        e1.synchronize()
-        if r >= 2:
-            un_ms += e0.elapsed_time(e1)
-    assert su.poll() == 0
-    x_uncached = su.result().cpu().numpy()
-    del gu
-    su.close()
-    un_ms /= un_reps
-    uncached = {"nfe_per_step": un_st["nfe"], "iters_per_step": un_iters, "ms_per_step": un_ms,
-                "value": un_iters / (un_ms / 1000.0),
-                "cached_speedup_per_generation": un_ms / (dev_ms / args.steps),
-                "nfe_reduction": 1.0 - nfe / max(1, un_st["nfe"])}
+        one_iteration(su)
+        stream.synchronize()
+        gu = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gu, stream=stream):
+            su.init(x_dev)
+            for _ in range(it):
+                one_iteration(su)
+        ms = 0.0
+        reps = max(5, min(args.steps, 50))
+        for r in range(reps + 2):
+            if flush is not None:
+                flush.zero_()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            gu.replay()
+            e1.record(stream)
+            e1.synchronize()
+            if r >= 2:
+                ms += e0.elapsed_time(e1)
+        assert su.poll() == 0
+        xs = su.result().cpu().numpy()
+        del gu
+        su.close()
+        ms /= reps
+        return {"nfe_per_step": st_["nfe"], "hits_per_step": st_["hits"],
+                "hit_rate": st_["hits"] / max(1, st_["hits"] + st_["nfe"]), "iters_per_step": it,
+                "ms_per_step": ms, "us_per_iteration": 1000.0 * ms / it, "value": it / (ms / 1000.0)}, xs
+
+    uncached, x_uncached = side_run(0.0)
+    for k in ("hits_per_step", "hit_rate"):
+        uncached.pop(k)
+    uncached["cached_speedup_per_generation"] = uncached["ms_per_step"] / (dev_ms / args.steps)
+    uncached["nfe_reduction"] = 1.0 - nfe / max(1, uncached["nfe_per_step"])
+    hit_heavy, x_hit_heavy = side_run(0.1)
+    hit_heavy["cache_thresh"] = 0.1
 
     # Quality check of the paper's kind with latents in place of CLIP scores:
     # the cached result against serial DDIM, which is the same library with a
@@ -782,6 +794,7 @@ def run_ours(args):
 
     deviation = dev_from_serial(x_cached)
     uncached["deviation_from_serial_ddim"] = dev_from_serial(x_uncached)
+    hit_heavy["deviation_from_serial_ddim"] = dev_from_serial(x_hit_heavy)
 
     units, secs = aggregate(args.steps * n_iters, dev_ms / 1000.0)
     value = units / secs
@@ -898,6 +911,7 @@ def run_ours(args):
             "deviation_from_serial_ddim": deviation,
             "solver_step": solver_step,
             "uncached": uncached,
+            "hit_heavy": hit_heavy,
             "denoiser_us_per_iteration": den_only_us,
             "denoiser_note": ("the denoiser alone: a graph of its calls on the generation's recorded batches, "
                               "each followed by pa_debug_gap, events around the graph, L2 flushed per replay"),
