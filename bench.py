@@ -77,9 +77,9 @@ NOMINAL_HBM_GBS = 8000.0
 NCU_TRAFFIC = {
     # per iteration: k_update_lean + k_plan_gather read + write bytes, averaged
     # over the first generation's launches
-    ("de8bf09d1e38c9d5", "sd15"): 8257472,       # 6,253,760 + 2,003,712 (no DRAM writes)
-    ("de8bf09d1e38c9d5", "batched"): 30268459,   # 24,576,256 + 5,692,203
-    ("de8bf09d1e38c9d5", "large"): 79785107,     # 70,941,550 + 8,843,557
+    ("772d428baaa1dd59", "sd15"): 8256576,       # 6,252,672 + 2,003,904 (no DRAM writes)
+    ("772d428baaa1dd59", "batched"): 30269867,   # 24,577,920 + 5,691,947
+    ("772d428baaa1dd59", "large"): 79809462,     # 70,969,051 + 8,840,411
 }
 
 

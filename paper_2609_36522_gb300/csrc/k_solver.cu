@@ -310,6 +310,7 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 // the accumulator set of iteration k+1. Nobody waits for anybody: the other
 // CTAs read copy par of the plan, which no CTA writes in this launch.
 constexpr int kPlanThreads = 256;
+constexpr int kPlanPerSm = 2;   // planning CTAs per SM (three: the launch bound makes the decision spill, slower)
 constexpr int kFusedMaxPairs = 1024;  // B*P planned in every CTA; beyond, one CTA plans
 static_assert(kFusedMaxPairs <= 32 * 32, "decide_par keeps one miss mask per 32-position chunk, 32 of them");
 
@@ -325,7 +326,7 @@ struct RedSums {
 };
 
 template <int VEC>
-__global__ void __launch_bounds__(kPlanThreads) k_plan_gather(Dev d, int par) {
+__global__ void __launch_bounds__(kPlanThreads, kPlanPerSm) k_plan_gather(Dev d, int par) {
   __shared__ DecideShared ds;
   const bool publish = blockIdx.x == 0 && blockIdx.y == 0;
   decide_load<kPlanThreads>(d, ds, par);
@@ -393,8 +394,37 @@ cudaError_t launch_gather(const Dev& d, int par, cudaStream_t st) {
   return launch_ex(k_gather<1>, g, dim3(kGatherThreads), 0, st, 0, d, par);
 }
 
+namespace {
+// The grid of a kernel whose CTA (x, y) copies part x of batch row y: as many
+// parts per row as keep the grid within per_sm CTAs per SM (one wave), each
+// part at least 1024 float4 columns. An error only if the SM count cannot be
+// read.
+cudaError_t split_grid(const Dev& d, int per_sm, dim3* out) {
+  static int nsm[64] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev >= 0 && dev < 64 && nsm[dev] == 0) {
+    e = cudaDeviceGetAttribute(&nsm[dev], cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+  }
+  const int sms = (dev >= 0 && dev < 64 && nsm[dev] > 0) ? nsm[dev] : 148;
+  dim3 g = gather_grid(d);
+  const int64_t nvec = d.D / ((d.D % 4 == 0) ? 4 : 1);
+  const int64_t cap = (nvec + kGatherThreads * 4 - 1) / (kGatherThreads * 4);
+  int64_t gx = (int64_t)per_sm * sms / (int)g.y;
+  if (gx > cap) gx = cap;
+  if (gx > 64) gx = 64;
+  g.x = gx < 1 ? 1 : (unsigned)gx;
+  *out = g;
+  return cudaSuccess;
+}
+}  // namespace
+
 cudaError_t launch_init(const Dev& d, cudaStream_t st) {
-  const dim3 g = gather_grid(d);
+  dim3 g;
+  const cudaError_t e = split_grid(d, kPlanPerSm, &g);
+  if (e != cudaSuccess) return e;
   if (d.D % 4 == 0) return launch_ex(k_init<4>, g, dim3(kGatherThreads), 0, st, 0, d);
   return launch_ex(k_init<1>, g, dim3(kGatherThreads), 0, st, 0, d);
 }
@@ -402,20 +432,10 @@ cudaError_t launch_init(const Dev& d, cudaStream_t st) {
 cudaError_t launch_plan(const Dev& d, int par, cudaStream_t st, int* launches) {
   if (d.B * d.P <= kFusedMaxPairs) {
     *launches = 1;
-    // every CTA plans, so fewer and longer CTAs: about two per SM in all,
-    // each copying a longer part of its row
-    static int nsm[64] = {};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    // every CTA plans and copies a part of its batch row
+    dim3 g;
+    const cudaError_t e = split_grid(d, kPlanPerSm, &g);
     if (e != cudaSuccess) return e;
-    if (dev >= 0 && dev < 64 && nsm[dev] == 0) {
-      e = cudaDeviceGetAttribute(&nsm[dev], cudaDevAttrMultiProcessorCount, dev);
-      if (e != cudaSuccess) return e;
-    }
-    const int sms = (dev >= 0 && dev < 64 && nsm[dev] > 0) ? nsm[dev] : 148;
-    dim3 g = gather_grid(d);
-    const int gx = (2 * sms + (int)g.y - 1) / (int)g.y;
-    if (gx < (int)g.x) g.x = gx < 1 ? 1 : gx;
     if (d.D % 4 == 0) return launch_ex(k_plan_gather<4>, g, dim3(kPlanThreads), 0, st, 0, d, par);
     return launch_ex(k_plan_gather<1>, g, dim3(kPlanThreads), 0, st, 0, d, par);
   }
