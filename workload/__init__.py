@@ -79,6 +79,8 @@ LARGE = Workload("large T200 P64 B2 4x128x128 K64", T=200, window=64, batch=2,
 # over the full 1000-step schedule, window 64 (Table 2's best DDPM window).
 DDPM = Workload("DDPM T1000 P64 B1 4x64x64 K16", T=1000, window=64, batch=1,
                 latent_shape=(4, 64, 64), K=16, tol=1e-3, cache_thresh=0.05, eta=1.0)
+# The same with a 128-point window, the longest window axis of Table 2.
+DDPM128 = DDPM.with_(name="DDPM T1000 P128 B1 4x64x64 K16", window=128)
 # Parareal (SRDS-style) sampling with the cache, on the SD-shaped and batched inputs.
 SRDS = SD15.with_(name="SRDS T100 B1 4x64x64 K16", sampler="srds")
 SRDS_BATCHED = BATCHED.with_(name="SRDS T100 B8 4x64x64 K16", sampler="srds")
@@ -99,7 +101,7 @@ def sweep(base: Workload = SD15):
             for c in SWEEP_THRESHOLDS]
 
 
-ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM,
+ALL = {"tiny": TINY, "sd15": SD15, "batched": BATCHED, "large": LARGE, "ddpm": DDPM, "ddpm128": DDPM128,
        "srds": SRDS, "srds_batched": SRDS_BATCHED, "sd15_taa": SD15_TAA, "batched_taa": BATCHED_TAA, "sd15_adapt": SD15_ADAPT}
 
 
