@@ -1019,35 +1019,64 @@ def run_srds_bench(args, w):
     if not args.no_e2e:
         x_host = torch.from_numpy(x0).pin_memory()
         out_host = torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory()
-        polls = 0
         reps = max(3, min(args.steps, 20))
-        stream.synchronize()
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        e0.record(stream)
-        t0 = time.perf_counter()
-        for _ in range(reps):
-            s.init(x_host)
-            done = False
-            while not done:
-                for _ in range(E2E_CHUNK):
-                    out = s.step_async()
-                    if out is None:
+
+        def denoise(bx, mb, nm):
+            g.eps(bx, mb, nm, eps)
+            return eps
+
+        def timed(run):
+            stream.synchronize()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            t0 = time.perf_counter()
+            polls = run()
+            e1.record(stream)
+            stream.synchronize()
+            return max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0), polls
+
+        def run_generate():
+            for _ in range(reps):
+                s.generate(x_host, denoise, out=out_host)
+            return 0 if s.generate_path() == "device graph" else reps * -(-n_stages // E2E_CHUNK)
+
+        def run_eager():
+            polls = 0
+            for _ in range(reps):
+                s.init(x_host)
+                done = False
+                while not done:
+                    for _ in range(E2E_CHUNK):
+                        out = s.step_async()
+                        if out is None:
+                            done = True
+                            break
+                        g.eps(*out, eps)
+                        s.submit_eps(eps)
+                    polls += 1
+                    if not done and s.poll() == 0:
                         done = True
-                        break
-                    g.eps(*out, eps)
-                    s.submit_eps(eps)
-                polls += 1
-                if not done and s.poll() == 0:
-                    done = True
-            s.result(out_host)
-        e1.record(stream)
-        stream.synchronize()
-        e2e_s = max(e0.elapsed_time(e1) / 1000.0, time.perf_counter() - t0)
+                s.result(out_host)
+            return polls
+
+        s.generate(x_host, denoise, out=out_host)   # the capture, outside the timing
+        e2e_s, polls = timed(run_generate)
+        eager_s, _ = timed(run_eager)
         units_e, secs_e = aggregate(reps * n_stages, e2e_s)
+        units_g, secs_g = aggregate(reps * n_stages, eager_s)
         e2e = {"value": units_e / secs_e, "unit": UNIT, "h2d_bytes_per_step": int(w.batch * w.D * 4),
                "d2h_bytes_per_step": int(w.batch * w.D * 4 + (polls // reps) * 24), "steps": reps,
-               "api": f"pa_srds_init (host x_init), pa_srds_step_async + pa_gmm_eps + pa_srds_submit_eps in "
-                      f"chunks of {E2E_CHUNK} stages, pa_srds_poll per chunk, pa_srds_result (host x_T)"}
+               "api": ("SrdsSolver.generate per step: pa_srds_init (host x_init), pa_srds_loop_launch (every "
+                       "stage of every Parareal iteration captured once as a CUDA graph of IF nodes, one per "
+                       "iteration, the iterations after convergence skipped on the device), pa_srds_result "
+                       "(host x_T, one synchronisation)"
+                       if s.generate_path() == "device graph" else
+                       f"SrdsSolver.generate, stages issued from Python, pa_srds_poll every {E2E_CHUNK} (the "
+                       f"driver refused the conditional graph nodes: {s.__dict__.get('loop_error')})"),
+               "generate_path": s.generate_path(),
+               "eager_value": units_g / secs_g,
+               "eager_api": f"pa_srds_init (host x_init), pa_srds_step_async + pa_gmm_eps + pa_srds_submit_eps "
+                            f"in chunks of {E2E_CHUNK} stages, pa_srds_poll per chunk, pa_srds_result (host x_T)"}
     # the sampled latents against serial DDIM (the Picard solver with a window
     # of one point and no cache, same inputs and denoiser)
     graph.replay()

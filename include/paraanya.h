@@ -487,6 +487,34 @@ PA_API pa_status pa_srds_stats(pa_srds* h, pa_srds_stats_t* out);
  * (rows of iterations not run are unspecified). Synchronises. */
 PA_API pa_status pa_srds_errors(pa_srds* h, float* err_out);
 
+/* A whole Parareal generation as one CUDA graph (the outer loop of Sec. 2.1's
+ * SRDS-style sampler run by the GPU, no host round trip between stages): a
+ * chain of conditional IF nodes, one per Parareal iteration 0..N, each body
+ * that iteration's stages; iteration 0 always runs, iteration k only when the
+ * finishing kernel of iteration k-1 (the convergence test above) found a
+ * trajectory still active. pa_srds_loop_capture_begin, right after
+ * pa_srds_init, starts capturing the sampler's stream; the caller then issues
+ * every stage (pa_srds_step_async, its denoiser's launches on the same stream
+ * reading the miss count on the device, pa_srds_submit_eps) until
+ * pa_srds_step_async returns PA_DONE, i.e. all N + 1 iterations; the library
+ * moves the capture from one IF body to the next at each iteration's end.
+ * pa_srds_loop_capture_end instantiates the graph; nothing runs during the
+ * capture, and the handle is back in its state after pa_srds_init.
+ * pa_srds_loop_launch, after a pa_srds_init, enqueues the graph: on return
+ * pa_srds_result (or pa_srds_poll) reads the outcome. No IF node loops, so
+ * the graph always ends. The captured launches carry the settings of the
+ * capture. Errors: PA_ERR_ARG for a NULL handle; PA_ERR_STATE for a call out
+ * of order (capture_begin not right after pa_srds_init or with a capture
+ * open; capture_end with none open or before every stage was issued: the
+ * capture is then closed and dropped and pa_srds_init must follow; launch
+ * with nothing captured or not right after pa_srds_init); synchronising calls
+ * (pa_srds_step, _poll, _result, _stats, _init) are refused while a capture
+ * is open; PA_ERR_CUDA where the driver refuses a conditional node (the
+ * capture is closed either way). */
+PA_API pa_status pa_srds_loop_capture_begin(pa_srds* h);
+PA_API pa_status pa_srds_loop_capture_end(pa_srds* h);
+PA_API pa_status pa_srds_loop_launch(pa_srds* h);
+
 PA_API void pa_srds_destroy(pa_srds* h);
 
 /* ---- synthetic denoiser: posterior-mean eps of an isotropic Gaussian mixture

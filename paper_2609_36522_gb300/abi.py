@@ -98,6 +98,9 @@ _PROTOS = {
     "pa_srds_result": (C.c_int, [VP, VP]),
     "pa_srds_stats": (C.c_int, [VP, C.POINTER(PaSrdsStats)]),
     "pa_srds_errors": (C.c_int, [VP, VP]),
+    "pa_srds_loop_capture_begin": (C.c_int, [VP]),
+    "pa_srds_loop_capture_end": (C.c_int, [VP]),
+    "pa_srds_loop_launch": (C.c_int, [VP]),
     "pa_srds_destroy": (None, [VP]),
     "pa_gmm_workspace_bytes": (C.c_size_t, [C.c_int, C.c_int64, C.c_int, C.c_int]),
     "pa_gmm_create": (C.c_int, [PVP, C.c_int, C.c_int64, VP, C.c_double,
@@ -243,6 +246,18 @@ def pa_loop_capture_end(h):
 
 def pa_loop_launch(h, x_init_ptr):
     return _check("pa_loop_launch", lib().pa_loop_launch(h, _dptr(x_init_ptr)))
+
+
+def pa_srds_loop_capture_begin(h):
+    return _check("pa_srds_loop_capture_begin", lib().pa_srds_loop_capture_begin(h))
+
+
+def pa_srds_loop_capture_end(h):
+    return _check("pa_srds_loop_capture_end", lib().pa_srds_loop_capture_end(h))
+
+
+def pa_srds_loop_launch(h):
+    return _check("pa_srds_loop_launch", lib().pa_srds_loop_launch(h))
 
 
 def pa_nfe(h):

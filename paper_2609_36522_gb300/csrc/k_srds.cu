@@ -337,7 +337,8 @@ __global__ void __launch_bounds__(kSThreads) k_srds_err(SDev d, int iter, int ns
 }
 
 // Convergence of every trajectory after iteration `iter` (one CTA).
-__global__ void __launch_bounds__(kSThreads) k_srds_finish(SDev d, int iter) {
+__global__ void __launch_bounds__(kSThreads) k_srds_finish(SDev d, int iter, cudaGraphConditionalHandle next,
+                                                           int has_next) {
   pa::pdl_wait();     // everything read here comes from earlier kernels
   pa::pdl_trigger();  // the successor may now be scheduled
   __shared__ int s_act;
@@ -366,6 +367,9 @@ __global__ void __launch_bounds__(kSThreads) k_srds_finish(SDev d, int iter) {
   if (threadIdx.x == 0) {
     d.ctl->n_active = s_act;
     d.ctl->iter = iter;
+    // inside a captured generation: the next iteration's IF node runs only
+    // while a trajectory is still active
+    if (has_next) cudaGraphSetConditional(next, s_act > 0 ? 1u : 0u);
   }
 }
 
@@ -457,6 +461,15 @@ struct pa_srds {
   int nsm;        // SMs of the device
   int64_t launches;
   SCtl* host_ctl;
+  // a whole generation captured as one CUDA graph (pa_srds_loop_*): a chain
+  // of IF nodes, one per Parareal iteration, each body that iteration's
+  // stages; iteration i's finishing kernel sets the condition of i + 1
+  cudaGraph_t loop_graph;
+  cudaGraphExec_t loop_exec;
+  std::vector<cudaGraphConditionalHandle> loop_cond;  // one per iteration 0..N
+  cudaGraphNode_t loop_last;  // the IF node of the iteration being captured
+  bool loop_capturing;
+  int64_t loop_launches0;
 };
 
 namespace {
@@ -464,6 +477,33 @@ namespace {
 pa_status s_fail(const std::string& m, pa_status code) {
   pa::set_error(m);
   return code;
+}
+
+// Forget the captured generation graph.
+void s_drop_loop(pa_srds* h) {
+  if (h->loop_exec) cudaGraphExecDestroy(h->loop_exec);
+  if (h->loop_graph) cudaGraphDestroy(h->loop_graph);  // and the bodies its IF nodes own
+  h->loop_exec = nullptr;
+  h->loop_graph = nullptr;
+  h->loop_cond.clear();
+  h->loop_last = nullptr;
+}
+
+// Append the IF node of iteration it to the chain and point the capture of
+// the sampler's stream at its body.
+cudaError_t s_open_iteration(pa_srds* h, int it) {
+  cudaGraphNodeParams np = {};
+  np.type = cudaGraphNodeTypeConditional;
+  np.conditional.handle = h->loop_cond[it];
+  np.conditional.type = cudaGraphCondTypeIf;
+  np.conditional.size = 1;
+  cudaGraphNode_t node = nullptr;
+  const cudaGraphNode_t dep = h->loop_last;
+  cudaError_t e = cudaGraphAddNode(&node, h->loop_graph, dep ? &dep : nullptr, nullptr, dep ? 1 : 0, &np);
+  if (e != cudaSuccess) return e;
+  h->loop_last = node;
+  return cudaStreamBeginCaptureToGraph(h->st, np.conditional.phGraph_out[0], nullptr, nullptr, 0,
+                                       cudaStreamCaptureModeThreadLocal);
 }
 
 Stage current_stage(const pa_srds* h) {
@@ -583,6 +623,7 @@ extern "C" pa_status pa_srds_create(pa_srds** out, int T, const int64_t* latent_
 
 extern "C" pa_status pa_srds_init(pa_srds* h, const float* x_init) {
   if (!h || !x_init) return s_fail("pa_srds_init: NULL argument", PA_ERR_ARG);
+  if (h->loop_capturing) return s_fail("pa_srds_init: a generation is being captured", PA_ERR_STATE);
   const SDev& d = h->d;
   // x_init (host or device) is staged in batch_x, then widened into U_0 and Up_0
   cudaError_t e = cudaMemcpyAsync(d.batch_x, x_init, (size_t)d.B * d.D * sizeof(float), cudaMemcpyDefault, h->st);
@@ -626,6 +667,8 @@ extern "C" pa_status pa_srds_step_async(pa_srds* h, const float** batch_x, const
 
 extern "C" pa_status pa_srds_step(pa_srds* h, int* n_miss, const float** batch_x, const int32_t** miss_bt) {
   if (!h || !n_miss) return s_fail("pa_srds_step: NULL argument", PA_ERR_ARG);
+  if (h->loop_capturing)
+    return s_fail("pa_srds_step: synchronises; inside a capture use pa_srds_step_async", PA_ERR_STATE);
   if (h->phase == 2) return PA_DONE;
   if (h->phase == 0 && h->stage == 0 && h->iter > 0) {  // a new iteration: anything left to refine?
     cudaError_t e = s_sync_ctl(h);
@@ -666,12 +709,28 @@ extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
   h->launches++;
   const int nstages = (h->iter == 0 ? 0 : d.s) + d.N;
   if (++h->stage == nstages) {  // the iteration is complete
+    const bool next = h->loop_capturing && h->iter + 1 <= d.N;  // captured: set the next IF node's condition
     if (e == cudaSuccess)
       e = pa::launch_ex(k_srds_err, dim3(d.nstrip, d.B * d.N), dim3(kSThreads), 0, h->st, 0, d, h->iter, nset);
-    if (e == cudaSuccess) e = pa::launch_ex(k_srds_finish, dim3(1), dim3(kSThreads), 0, h->st, 0, d, h->iter);
+    if (e == cudaSuccess)
+      e = pa::launch_ex(k_srds_finish, dim3(1), dim3(kSThreads), 0, h->st, 0, d, h->iter,
+                        next ? h->loop_cond[h->iter + 1] : (cudaGraphConditionalHandle)0, next ? 1 : 0);
     h->launches += 2;
     h->stage = 0;
     h->iter++;
+    if (h->loop_capturing) {  // the iteration's body is complete: close it, open the next one's
+      cudaGraph_t body = nullptr;
+      const cudaError_t ec = cudaStreamEndCapture(h->st, &body);
+      if (e == cudaSuccess) e = ec;
+      if (e == cudaSuccess && h->iter <= d.N) e = s_open_iteration(h, h->iter);
+      if (e != cudaSuccess) {  // nothing ran; the capture is closed and dropped
+        (void)cudaGetLastError();
+        h->loop_capturing = false;
+        s_drop_loop(h);
+        h->phase = -1;  // pa_srds_init must follow
+        return s_fail(std::string("pa_srds_submit_eps: capture: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+      }
+    }
   }
   h->g++;
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_submit_eps: ") + cudaGetErrorString(e), PA_ERR_CUDA);
@@ -681,6 +740,7 @@ extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
 
 extern "C" pa_status pa_srds_poll(pa_srds* h, int* n_active) {
   if (!h) return s_fail("pa_srds_poll: NULL handle", PA_ERR_ARG);
+  if (h->loop_capturing) return s_fail("pa_srds_poll: synchronises; not inside a capture", PA_ERR_STATE);
   const cudaError_t e = s_sync_ctl(h);
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_poll: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   const int act = h->host_ctl->n_active;
@@ -691,6 +751,7 @@ extern "C" pa_status pa_srds_poll(pa_srds* h, int* n_active) {
 
 extern "C" pa_status pa_srds_result(pa_srds* h, float* x_out) {
   if (!h || !x_out) return s_fail("pa_srds_result: NULL argument", PA_ERR_ARG);
+  if (h->loop_capturing) return s_fail("pa_srds_result: synchronises; not inside a capture", PA_ERR_STATE);
   if (h->phase != 2) return s_fail("pa_srds_result: not finished", PA_ERR_STATE);
   const SDev& d = h->d;
   // U_N narrowed to fp32 in batch_x (free once sampling is done), then copied out
@@ -703,8 +764,79 @@ extern "C" pa_status pa_srds_result(pa_srds* h, float* x_out) {
   return PA_OK;
 }
 
+extern "C" pa_status pa_srds_loop_capture_begin(pa_srds* h) {
+  if (!h) return s_fail("pa_srds_loop_capture_begin: NULL handle", PA_ERR_ARG);
+  if (h->loop_capturing) return s_fail("pa_srds_loop_capture_begin: a capture is already open", PA_ERR_STATE);
+  if (h->phase != 0 || h->iter != 0 || h->stage != 0 || h->g != 0)
+    return s_fail("pa_srds_loop_capture_begin: call right after pa_srds_init", PA_ERR_STATE);
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  cudaError_t e = cudaStreamIsCapturing(h->st, &cs);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_loop_capture_begin: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  if (cs != cudaStreamCaptureStatusNone)
+    return s_fail("pa_srds_loop_capture_begin: the stream is already being captured", PA_ERR_STATE);
+  s_drop_loop(h);
+  e = cudaGraphCreate(&h->loop_graph, 0);
+  // iteration 0 (the coarse sweep) always runs; every later one only when the
+  // previous one's finishing kernel found a trajectory still active
+  h->loop_cond.assign((size_t)h->d.N + 1, 0);
+  for (int i = 0; i <= h->d.N && e == cudaSuccess; ++i)
+    e = cudaGraphConditionalHandleCreate(&h->loop_cond[i], h->loop_graph, i == 0 ? 1u : 0u,
+                                         cudaGraphCondAssignDefault);
+  if (e == cudaSuccess) e = s_open_iteration(h, 0);
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    s_drop_loop(h);
+    return s_fail(std::string("pa_srds_loop_capture_begin: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  }
+  h->loop_capturing = true;
+  h->loop_launches0 = h->launches;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_loop_capture_end(pa_srds* h) {
+  if (!h) return s_fail("pa_srds_loop_capture_end: NULL handle", PA_ERR_ARG);
+  if (!h->loop_capturing) return s_fail("pa_srds_loop_capture_end: no capture is open", PA_ERR_STATE);
+  h->loop_capturing = false;
+  if (h->phase != 2) {  // a body is still open: close it, keep nothing
+    cudaGraph_t body = nullptr;
+    (void)cudaStreamEndCapture(h->st, &body);
+    (void)cudaGetLastError();
+    s_drop_loop(h);
+    h->phase = -1;  // pa_srds_init must follow
+    return s_fail("pa_srds_loop_capture_end: issue every stage first (pa_srds_step_async until PA_DONE)",
+                  PA_ERR_STATE);
+  }
+  const cudaError_t e = cudaGraphInstantiate(&h->loop_exec, h->loop_graph, 0);
+  if (e != cudaSuccess) {
+    (void)cudaGetLastError();
+    s_drop_loop(h);
+    h->phase = -1;
+    return s_fail(std::string("pa_srds_loop_capture_end: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  }
+  // nothing ran: back to the state right after pa_srds_init
+  h->iter = 0;
+  h->stage = 0;
+  h->g = 0;
+  h->phase = 0;
+  h->launches = h->loop_launches0;
+  return PA_OK;
+}
+
+extern "C" pa_status pa_srds_loop_launch(pa_srds* h) {
+  if (!h) return s_fail("pa_srds_loop_launch: NULL handle", PA_ERR_ARG);
+  if (!h->loop_exec) return s_fail("pa_srds_loop_launch: nothing has been captured", PA_ERR_STATE);
+  if (h->loop_capturing || h->phase != 0 || h->iter != 0 || h->stage != 0 || h->g != 0)
+    return s_fail("pa_srds_loop_launch: call right after pa_srds_init", PA_ERR_STATE);
+  const cudaError_t e = cudaGraphLaunch(h->loop_exec, h->st);
+  if (e != cudaSuccess) return s_fail(std::string("pa_srds_loop_launch: ") + cudaGetErrorString(e), PA_ERR_CUDA);
+  h->phase = 2;  // the graph runs the generation to its end
+  h->iter = h->d.N + 1;
+  return PA_OK;
+}
+
 extern "C" pa_status pa_srds_stats(pa_srds* h, pa_srds_stats_t* out) {
   if (!h || !out) return s_fail("pa_srds_stats: NULL argument", PA_ERR_ARG);
+  if (h->loop_capturing) return s_fail("pa_srds_stats: synchronises; not inside a capture", PA_ERR_STATE);
   const cudaError_t e = s_sync_ctl(h);
   if (e != cudaSuccess) return s_fail(std::string("pa_srds_stats: ") + cudaGetErrorString(e), PA_ERR_CUDA);
   out->iters = h->host_ctl->iter;
@@ -729,6 +861,12 @@ extern "C" pa_status pa_srds_errors(pa_srds* h, float* err_out) {
 
 extern "C" void pa_srds_destroy(pa_srds* h) {
   if (!h) return;
+  if (h->loop_capturing) {  // close the capture so that the stream stays usable
+    cudaGraph_t g = nullptr;
+    cudaStreamEndCapture(h->st, &g);
+    (void)cudaGetLastError();
+  }
+  s_drop_loop(h);
   if (h->host_ctl) cudaFreeHost(h->host_ctl);
   delete h;
 }

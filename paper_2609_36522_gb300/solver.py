@@ -453,6 +453,71 @@ class SrdsSolver:
         abi.pa_srds_result(self.h, out.data_ptr())
         return out
 
+    def generate(self, x_init, denoise, out=None):
+        """One whole Parareal generation in one call: x_init in, x_T out (into
+        ``out``, a CUDA or pinned host tensor, else a new CUDA tensor).
+        ``denoise`` as for ``Solver.generate`` (enqueues on this sampler's
+        stream, reads the miss count on the device, returns the eps buffer it
+        always writes, capturable). The first call per denoiser captures every
+        stage of every Parareal iteration as one CUDA graph of IF nodes
+        (``pa_srds_loop_capture_begin/_end``; iterations after convergence
+        are skipped on the device); each call then enqueues ``pa_srds_init``
+        and ``pa_srds_loop_launch`` and reads x_T with ``pa_srds_result`` (one
+        synchronisation). Where the driver refuses the conditional nodes, the
+        stages are issued from Python with a ``pa_srds_poll`` every 4."""
+        if self.__dict__.get("_loop_for") is not denoise and self.__dict__.get("loop_error") is None:
+            self._capture(x_init, denoise)
+        self.init(x_init)
+        if self.__dict__.get("_loop_for") is denoise:
+            abi.pa_srds_loop_launch(self.h)
+        else:
+            done = False
+            while not done:
+                for _ in range(4):
+                    plan = self.step_async()
+                    if plan is None:
+                        done = True
+                        break
+                    self.submit_eps(denoise(*plan))
+                if not done:
+                    done = self.poll() == 0
+        return self.result(out)
+
+    def _capture(self, x_init, denoise):
+        self.init(x_init)
+        plan = self.step_async()  # one eager stage: launch-time set-up outside the capture
+        self.submit_eps(denoise(*plan))
+        self.init(x_init)
+        abi.pa_srds_loop_capture_begin(self.h)
+        try:
+            with torch.cuda.stream(self.stream):
+                while True:
+                    plan = self.step_async()
+                    if plan is None:
+                        break
+                    self.submit_eps(denoise(*plan))
+        except BaseException as exc:
+            try:
+                abi.pa_srds_loop_capture_end(self.h)  # closes the capture if open; nothing is kept
+            except abi.PaError:
+                pass
+            if isinstance(exc, abi.PaError) and exc.status == abi.PA_ERR_CUDA:
+                self.loop_error = str(exc)  # the driver refused the graph: issue stages from Python
+                return
+            raise
+        try:
+            abi.pa_srds_loop_capture_end(self.h)
+        except abi.PaError as e:
+            if e.status != abi.PA_ERR_CUDA:
+                raise
+            self.loop_error = str(e)
+            return
+        self._loop_for = denoise
+
+    def generate_path(self):
+        """'device graph' or, without conditional graph nodes, 'stages from Python'."""
+        return "stages from Python" if self.__dict__.get("loop_error") else "device graph"
+
     def stats(self):
         return abi.pa_srds_stats(self.h)
 

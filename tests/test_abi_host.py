@@ -88,6 +88,9 @@ def test_null_handles_are_rejected(lib):
     assert L.pa_loop_capture_begin(None) == abi.PA_ERR_ARG
     assert L.pa_loop_capture_end(None) == abi.PA_ERR_ARG
     assert L.pa_loop_launch(None, None) == abi.PA_ERR_ARG
+    assert L.pa_srds_loop_capture_begin(None) == abi.PA_ERR_ARG
+    assert L.pa_srds_loop_capture_end(None) == abi.PA_ERR_ARG
+    assert L.pa_srds_loop_launch(None) == abi.PA_ERR_ARG
     assert L.pa_nfe(None) == -1
     assert L.pa_n_miss_dev(None) is None
     assert L.pa_set_update_kernel(None, 0) == abi.PA_ERR_ARG

@@ -117,3 +117,100 @@ def test_srds_edge_shapes(T, batch, shape):
     compare_srds(w, orc, gpu_srds(w))
     g = gpu_srds(w, mode="async")
     assert g["stats"]["nfe"] == orc.nfe
+
+
+@pytest.mark.parametrize("wname", ["srds", "srds_batched"])
+def test_srds_generation_graph_equals_host_driven(wname):
+    """SrdsSolver.generate through the captured generation (IF nodes, one per
+    Parareal iteration; iterations after convergence skipped on the device),
+    twice and into a pinned host buffer: x_T, NFE, hits and iterations bit for
+    bit those of the host-driven run."""
+    import torch
+    from paper_2609_36522_gb300.solver import SrdsSolver, GmmDenoiser
+    w = W.ALL[wname]
+    a, x0, mu = W.inputs(w)
+    st = torch.cuda.Stream()
+    s = SrdsSolver(w.T, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=st)
+    g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, s.max_rows, stream=st)
+    eps = torch.empty(s.max_rows, w.D, dtype=torch.float32, device="cuda")
+    x0d = torch.from_numpy(x0).cuda()
+    torch.cuda.synchronize()
+
+    def denoise(bx, mb, nm):
+        g.eps(bx, mb, nm, eps)
+        return eps
+
+    s.init(x0d)
+    while True:
+        plan = s.step()
+        if plan is None:
+            break
+        s.submit_eps(denoise(plan.batch_x_ptr, plan.miss_bt_ptr, s.n_miss_dev()))
+    want, st_want = s.result().clone(), s.stats()
+    host = torch.full((w.batch, w.D), float("nan"), dtype=torch.float32).pin_memory()
+    for out in (None, host):
+        got = s.generate(x0d, denoise, out=out)
+        assert s.generate_path() == "device graph", s.__dict__.get("loop_error")
+        assert torch.equal(got.cpu(), want.cpu())
+        st_got = s.stats()
+        assert (st_got["nfe"], st_got["hits"], st_got["iters"]) == (st_want["nfe"], st_want["hits"], st_want["iters"])
+    s.close()
+    g.close()
+
+
+def test_srds_generation_graph_call_order():
+    """PA_ERR_STATE: capture_begin not right after pa_srds_init, capture_end
+    with nothing open or before every stage was issued (the capture is closed,
+    the handle needs pa_srds_init and works after it), launch with nothing
+    captured, synchronising calls inside a capture."""
+    import torch
+    from paper_2609_36522_gb300 import abi
+    from paper_2609_36522_gb300.solver import SrdsSolver, GmmDenoiser
+    w = W.SRDS
+    a, x0, mu = W.inputs(w)
+    st = torch.cuda.Stream()
+    s = SrdsSolver(w.T, w.latent_shape, a, w.tol, w.cache_thresh, batch=w.batch, stream=st)
+    g = GmmDenoiser(torch.from_numpy(mu).cuda(), w.gmm_std, a, s.max_rows, stream=st)
+    eps = torch.empty(s.max_rows, w.D, dtype=torch.float32, device="cuda")
+    x0d = torch.from_numpy(x0).cuda()
+    torch.cuda.synchronize()
+
+    def state_error(f, *args):
+        with pytest.raises(abi.PaError) as e:
+            f(*args)
+        assert e.value.status == abi.PA_ERR_STATE
+
+    state_error(abi.pa_srds_loop_capture_end, s.h)
+    state_error(abi.pa_srds_loop_launch, s.h)
+    s.init(x0d)
+    bx, mb, nm = s.step_async()
+    state_error(abi.pa_srds_loop_capture_begin, s.h)     # not right after pa_srds_init
+    g.eps(bx, mb, nm, eps)
+    s.submit_eps(eps)
+    s.init(x0d)
+    abi.pa_srds_loop_capture_begin(s.h)
+    state_error(abi.pa_srds_loop_capture_begin, s.h)
+    state_error(abi.pa_srds_poll, s.h)
+    state_error(abi.pa_srds_init, s.h, x0d.data_ptr())
+    with torch.cuda.stream(st):
+        bx, mb, nm = s.step_async()
+        g.eps(bx, mb, nm, eps)
+        s.submit_eps(eps)
+    state_error(abi.pa_srds_loop_capture_end, s.h)       # stages left: closed, nothing kept
+    state_error(abi.pa_srds_loop_launch, s.h)
+    s.init(x0d)
+    while True:
+        plan = s.step()
+        if plan is None:
+            break
+        g.eps(plan.batch_x_ptr, plan.miss_bt_ptr, s.n_miss_dev(), eps)
+        s.submit_eps(eps)
+    want = s.result().clone()
+
+    def denoise(bx, mb, nm):
+        g.eps(bx, mb, nm, eps)
+        return eps
+
+    assert torch.equal(s.generate(x0d, denoise), want)
+    s.close()
+    g.close()
