@@ -64,6 +64,14 @@ LOOP_CASES = [
     ("sd15 anderson", W.SD15.with_(T=60), {"anderson": 1}),
     ("batched adaptive", W.BATCHED.with_(T=40), {"adapt": (0.5, 0.2, 0.0, 1.0)}),
     ("ddim eta 1", W.SD15.with_(T=50, window=24), {"eta": 1.0}),
+    ("64 trajectories", W.Workload("64 trajectories", T=40, window=32, batch=64, latent_shape=(4, 4, 4), K=4,
+                                   tol=1e-3, cache_thresh=0.05, seed=14), {"chunk": None}),
+    ("9 x 128 pairs", W.Workload("9 x 128 pairs", T=200, window=128, batch=9, latent_shape=(4, 4, 4), K=4,
+                                 tol=1e-3, cache_thresh=0.05, seed=13), {"chunk": None}),
+    ("window past T, odd T", W.Workload("odd", T=37, window=64, batch=3, latent_shape=(4, 8, 8), K=4,
+                                        tol=1e-3, cache_thresh=0.05, seed=15), {"chunk": 2}),
+    ("ragged D", W.Workload("ragged", T=20, window=7, batch=2, latent_shape=(3, 7, 9), K=4,
+                            tol=1e-3, cache_thresh=0.05, seed=16), {"chunk": 6}),
 ]
 
 
