@@ -1,6 +1,7 @@
 """The C ABI used from plain C: tests/c/abi_generation.c (gcc, no Python and no
 torch in the process) runs cached-Picard generations through libparaanya.so
-with cudaMalloc'd buffers, host x_init in and host x_T out; the results must
+with cudaMalloc'd buffers, host x_init in and host x_T out, step by step and as
+the device-driven loop (pa_loop_*); the results must
 match the fp64 oracle exactly in NFE, iterations and hits and within 1e-5 in
 the final latents."""
 import os
@@ -40,7 +41,8 @@ def _build(tmp):
     W.Workload("C batched", T=24, window=8, batch=3, latent_shape=(4, 8, 8), K=4,
                tol=1e-3, cache_thresh=0.05, seed=21),
 ], ids=lambda w: w.name)
-def test_generation_from_c(w, tmp_path):
+@pytest.mark.parametrize("mode", ["steps", "loop"])
+def test_generation_from_c(w, mode, tmp_path):
     exe = _build(str(tmp_path))
     a, x0, mu = W.inputs(w)
     c, h, wd = w.latent_shape
@@ -49,7 +51,8 @@ def test_generation_from_c(w, tmp_path):
     np.asarray(a, dtype=np.float64).tofile(tmp_path / "alphas.bin")
     np.ascontiguousarray(x0, dtype=np.float32).tofile(tmp_path / "x0.bin")
     np.ascontiguousarray(mu, dtype=np.float32).tofile(tmp_path / "mu.bin")
-    r = subprocess.run([exe, str(tmp_path)], capture_output=True, text=True, timeout=300)
+    r = subprocess.run([exe, str(tmp_path)] + (["loop"] if mode == "loop" else []), capture_output=True,
+                       text=True, timeout=300)
     assert r.returncode == 0, r.stderr
     fields = r.stdout.split()
     nfe, iters, hits = int(fields[1]), int(fields[3]), int(fields[5])
