@@ -502,8 +502,20 @@ cudaError_t s_open_iteration(pa_srds* h, int it) {
   cudaError_t e = cudaGraphAddNode(&node, h->loop_graph, dep ? &dep : nullptr, nullptr, dep ? 1 : 0, &np);
   if (e != cudaSuccess) return e;
   h->loop_last = node;
+  // relaxed: calls this thread makes meanwhile on other work must not
+  // invalidate the capture
   return cudaStreamBeginCaptureToGraph(h->st, np.conditional.phGraph_out[0], nullptr, nullptr, 0,
-                                       cudaStreamCaptureModeThreadLocal);
+                                       cudaStreamCaptureModeRelaxed);
+}
+
+// Let go of a generation graph whose capture the runtime invalidated,
+// without destroying it: destroying such a graph crashed the host process
+// inside the CUDA runtime. The graph leaks; the handle can capture again.
+void s_forget_loop(pa_srds* h) {
+  h->loop_exec = nullptr;
+  h->loop_graph = nullptr;
+  h->loop_cond.clear();
+  h->loop_last = nullptr;
 }
 
 Stage current_stage(const pa_srds* h) {
@@ -726,7 +738,10 @@ extern "C" pa_status pa_srds_submit_eps(pa_srds* h, const float* batch_eps) {
       if (e != cudaSuccess) {  // nothing ran; the capture is closed and dropped
         (void)cudaGetLastError();
         h->loop_capturing = false;
-        s_drop_loop(h);
+        if (ec != cudaSuccess)
+          s_forget_loop(h);  // an invalidated capture: destroy nothing
+        else
+          s_drop_loop(h);
         h->phase = -1;  // pa_srds_init must follow
         return s_fail(std::string("pa_srds_submit_eps: capture: ") + cudaGetErrorString(e), PA_ERR_CUDA);
       }
@@ -799,9 +814,12 @@ extern "C" pa_status pa_srds_loop_capture_end(pa_srds* h) {
   h->loop_capturing = false;
   if (h->phase != 2) {  // a body is still open: close it, keep nothing
     cudaGraph_t body = nullptr;
-    (void)cudaStreamEndCapture(h->st, &body);
+    const cudaError_t ec = cudaStreamEndCapture(h->st, &body);
     (void)cudaGetLastError();
-    s_drop_loop(h);
+    if (ec != cudaSuccess)
+      s_forget_loop(h);  // an invalidated capture: destroy nothing
+    else
+      s_drop_loop(h);
     h->phase = -1;  // pa_srds_init must follow
     return s_fail("pa_srds_loop_capture_end: issue every stage first (pa_srds_step_async until PA_DONE)",
                   PA_ERR_STATE);
@@ -863,7 +881,7 @@ extern "C" void pa_srds_destroy(pa_srds* h) {
   if (!h) return;
   if (h->loop_capturing) {  // close the capture so that the stream stays usable
     cudaGraph_t g = nullptr;
-    cudaStreamEndCapture(h->st, &g);
+    if (cudaStreamEndCapture(h->st, &g) != cudaSuccess) s_forget_loop(h);
     (void)cudaGetLastError();
   }
   s_drop_loop(h);

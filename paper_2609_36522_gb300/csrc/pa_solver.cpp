@@ -151,6 +151,15 @@ cudaError_t copy_xt(pa_solver* s, float* x_out) {
                            (size_t)d.D * sizeof(float), d.B, cudaMemcpyDefault, s->st);
 }
 
+// Let go of a loop graph whose capture the runtime invalidated, without
+// destroying it: destroying such a graph crashed the host process inside the
+// CUDA runtime. The graph leaks; the handle can capture again.
+void forget_loop(pa_solver* s) {
+  s->loop_exec = nullptr;
+  s->loop_graph = nullptr;
+  s->loop_cond = 0;
+}
+
 // Forget the captured generation loop (its launches carry the settings of
 // the capture). Not while a capture is open.
 void drop_loop(pa_solver* s) {
@@ -585,8 +594,10 @@ pa_status pa_loop_capture_begin(pa_solver* s) {
     e = cudaGraphAddNode(&loop, s->loop_graph, nullptr, nullptr, 0, &np);
   }
   if (e == cudaSuccess)
+    // relaxed: calls this thread makes meanwhile on other work (a finalizer
+    // destroying another graph, say) must not invalidate the capture
     e = cudaStreamBeginCaptureToGraph(s->st, np.conditional.phGraph_out[0], nullptr, nullptr, 0,
-                                      cudaStreamCaptureModeThreadLocal);
+                                      cudaStreamCaptureModeRelaxed);
   if (e != cudaSuccess) {
     drop_loop(s);
     return cuda_fail("pa_loop_capture_begin", e);
@@ -613,6 +624,14 @@ pa_status pa_loop_capture_end(pa_solver* s) {
   const cudaError_t e2 = cudaStreamEndCapture(s->st, &body);
   if (e == cudaSuccess) e = e2;
   s->loop_capturing = false;
+  if (e2 != cudaSuccess) {  // the runtime invalidated the capture: keep nothing, destroy nothing
+    (void)cudaGetLastError();
+    forget_loop(s);
+    s->k = s->loop_k0;
+    s->launches = s->loop_launches0;
+    if (s->state == St::Stepped) s->state = St::Ready;
+    return cuda_fail("pa_loop_capture_end", e2);
+  }
   s->k = s->loop_k0;  // nothing ran: the host state is the one before the capture
   s->launches = s->loop_launches0;
   if (s->state == St::Stepped) s->state = St::Ready;
@@ -855,7 +874,7 @@ void pa_destroy(pa_solver* s) {
     if (x) cudaEventDestroy(x);
   if (s->loop_capturing) {  // close the capture so that the stream stays usable
     cudaGraph_t g = nullptr;
-    cudaStreamEndCapture(s->st, &g);
+    if (cudaStreamEndCapture(s->st, &g) != cudaSuccess) forget_loop(s);
     (void)cudaGetLastError();
   }
   drop_loop(s);

@@ -7,6 +7,7 @@ into the workspace, never copied.
 """
 from __future__ import annotations
 
+import gc
 import numpy as np
 import torch
 
@@ -232,24 +233,36 @@ class Solver:
         bx, mb, nm = self.step_async()
         self.submit_eps(denoise(bx, mb, nm))
         self.init(x_init)
-        abi.pa_loop_capture_begin(self.h)
+        # no finalizer of unrelated objects (which may call into CUDA) runs
+        # inside the capture: collect before it, pause the collector during it
+        gc.collect()
+        gc_was_on = gc.isenabled()
+        gc.disable()
         try:
-            with torch.cuda.stream(self.stream):  # torch work of the denoiser lands in the body
-                for _ in range(chunk):
-                    bx, mb, nm = self.step_async()
-                    self.submit_eps(denoise(bx, mb, nm))
-        except BaseException:
+            abi.pa_loop_capture_begin(self.h)
             try:
-                abi.pa_loop_capture_end(self.h)  # closes the capture; the body is incomplete
-            except abi.PaError:
-                pass
-            raise
-        try:
-            abi.pa_loop_capture_end(self.h)
-        except abi.PaError as e:
-            if e.status != abi.PA_ERR_CUDA:
+                with torch.cuda.stream(self.stream):  # torch work of the denoiser lands in the body
+                    for _ in range(chunk):
+                        bx, mb, nm = self.step_async()
+                        self.submit_eps(denoise(bx, mb, nm))
+            except BaseException:
+                try:
+                    abi.pa_loop_capture_end(self.h)  # closes the capture; the body is incomplete
+                except abi.PaError:
+                    pass
                 raise
-            self.loop_error = str(e)  # this driver cannot run the loop: replay and poll instead
+            end_error = None
+            try:
+                abi.pa_loop_capture_end(self.h)
+            except abi.PaError as e:
+                end_error = e
+        finally:
+            if gc_was_on:
+                gc.enable()
+        if end_error is not None:
+            if end_error.status != abi.PA_ERR_CUDA:
+                raise end_error
+            self.loop_error = str(end_error)  # this driver cannot run the loop: replay and poll instead
             return
         self._loop_for = (denoise, chunk)
 
@@ -488,30 +501,37 @@ class SrdsSolver:
         plan = self.step_async()  # one eager stage: launch-time set-up outside the capture
         self.submit_eps(denoise(*plan))
         self.init(x_init)
-        abi.pa_srds_loop_capture_begin(self.h)
+        gc.collect()  # no finalizer of unrelated objects runs inside the capture
+        gc_was_on = gc.isenabled()
+        gc.disable()
         try:
-            with torch.cuda.stream(self.stream):
-                while True:
-                    plan = self.step_async()
-                    if plan is None:
-                        break
-                    self.submit_eps(denoise(*plan))
-        except BaseException as exc:
+            abi.pa_srds_loop_capture_begin(self.h)
             try:
-                abi.pa_srds_loop_capture_end(self.h)  # closes the capture if open; nothing is kept
-            except abi.PaError:
-                pass
-            if isinstance(exc, abi.PaError) and exc.status == abi.PA_ERR_CUDA:
-                self.loop_error = str(exc)  # the driver refused the graph: issue stages from Python
-                return
-            raise
-        try:
-            abi.pa_srds_loop_capture_end(self.h)
-        except abi.PaError as e:
-            if e.status != abi.PA_ERR_CUDA:
+                with torch.cuda.stream(self.stream):
+                    while True:
+                        plan = self.step_async()
+                        if plan is None:
+                            break
+                        self.submit_eps(denoise(*plan))
+            except BaseException as exc:
+                try:
+                    abi.pa_srds_loop_capture_end(self.h)  # closes the capture if open; nothing is kept
+                except abi.PaError:
+                    pass
+                if isinstance(exc, abi.PaError) and exc.status == abi.PA_ERR_CUDA:
+                    self.loop_error = str(exc)  # the driver refused the graph: issue stages from Python
+                    return
                 raise
-            self.loop_error = str(e)
-            return
+            try:
+                abi.pa_srds_loop_capture_end(self.h)
+            except abi.PaError as e:
+                if e.status != abi.PA_ERR_CUDA:
+                    raise
+                self.loop_error = str(e)
+                return
+        finally:
+            if gc_was_on:
+                gc.enable()
         self._loop_for = denoise
 
     def generate_path(self):

@@ -125,6 +125,12 @@ def test_loop_generations_in_flight():
     s.finish()
     for o, want in zip(outs, wants):
         assert torch.equal(o, want.cpu())
+    # pinned host (the poll kernel writes it), device and pageable host (the copy engine) outputs
+    for out in (torch.empty(w.batch, w.D, dtype=torch.float32).pin_memory(),
+                torch.empty(w.batch, w.D, dtype=torch.float32, device="cuda"),
+                torch.empty(w.batch, w.D, dtype=torch.float32)):
+        out.fill_(float("nan"))
+        assert torch.equal(s.generate(inits[1], denoise, out=out).cpu(), wants[1].cpu())
     s.close()
     g.close()
 
@@ -214,5 +220,66 @@ def test_loop_ends_on_a_device_error():
     s._drop_graphs()
     assert torch.equal(s.generate(x0, denoise), want)
     assert s.stats()["device_status"] == 0
+    s.close()
+    g.close()
+
+
+def test_loop_capture_survives_other_cuda_work_and_reports_invalidation():
+    """(a) Another CUDA graph destroyed while the loop is being captured (as a
+    finalizer of an unrelated object may do) leaves the capture valid: it is
+    relaxed, so the loop runs and gives the host-driven x_T. (b) A capture the
+    caller invalidates (a synchronisation of the capturing stream) makes
+    pa_loop_capture_end report PA_ERR_CUDA, keeping and destroying nothing;
+    the handle then captures again and runs."""
+    import torch
+    w = W.SD15.with_(T=40)
+    s, g, eps, x0, denoise = _setup(w)
+    want = _sync(s, x0, denoise)[0]
+    s.init(x0)
+    bx, mb, nm = s.step_async()  # eager warm-up outside the capture
+    s.submit_eps(denoise(bx, mb, nm))
+
+    def other_graph():
+        side = torch.cuda.Stream()
+        buf = torch.zeros(1024, device="cuda")
+        gr = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gr, stream=side):
+            buf.add_(1.0)
+        return gr, buf
+
+    gr, buf = other_graph()
+    torch.cuda.synchronize()
+    s.init(x0)
+    abi.pa_loop_capture_begin(s.h)
+    with torch.cuda.stream(s.stream):
+        for k in range(4):
+            bx, mb, nm = s.step_async()
+            s.submit_eps(denoise(bx, mb, nm))
+            if k == 1:
+                del gr  # destroys that graph (and its executable) mid-capture
+    abi.pa_loop_capture_end(s.h)
+    abi.pa_loop_launch(s.h, x0.data_ptr())
+    out = torch.empty_like(want)
+    stt, n = abi.pa_poll_result(s.h, out.data_ptr())
+    assert stt == abi.PA_DONE and torch.equal(out, want)
+    # (b) invalidated by the caller
+    s.init(x0)
+    abi.pa_loop_capture_begin(s.h)
+    with torch.cuda.stream(s.stream):
+        bx, mb, nm = s.step_async()
+        g.eps(bx, mb, nm, eps)
+        with pytest.raises(RuntimeError):
+            s.stream.synchronize()  # not allowed while capturing: the capture is invalidated
+        with pytest.raises(abi.PaError):
+            s.submit_eps(eps)  # its launches fail on the invalidated capture
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_loop_capture_end(s.h)
+    assert e.value.status == abi.PA_ERR_CUDA
+    with pytest.raises(abi.PaError) as e:
+        abi.pa_loop_launch(s.h, x0.data_ptr())  # nothing was kept
+    assert e.value.status == abi.PA_ERR_STATE
+    torch.cuda.synchronize()
+    s._drop_graphs()
+    assert torch.equal(s.generate(x0, denoise), want)
     s.close()
     g.close()
