@@ -238,8 +238,11 @@ PA_API pa_status pa_poll_end(pa_solver* s, int* n_active);
  * iterations or none, kernel timing enabled: its events cannot sit in a loop
  * body, a stream already being captured, a launch between pa_step_async and
  * pa_submit_eps or with nothing captured); PA_ERR_CUDA where the driver
- * refuses the conditional node or its instantiation (the capture is closed
- * either way and the stream stays usable). */
+ * refuses the conditional node or its instantiation, or where the capture
+ * was invalidated (a synchronisation of the solver's stream during it, say);
+ * the capture is closed either way, nothing is kept, and the stream stays
+ * usable. The capture is relaxed: CUDA calls the thread makes meanwhile on
+ * other work do not invalidate it. */
 PA_API pa_status pa_loop_capture_begin(pa_solver* s);
 PA_API pa_status pa_loop_capture_end(pa_solver* s);
 PA_API pa_status pa_loop_launch(pa_solver* s, const float* x_init);
