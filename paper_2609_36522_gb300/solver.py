@@ -147,20 +147,20 @@ class Solver:
         generation's iteration count: with ``chunk=None`` the first call per
         denoiser runs one host-driven generation of its x_init and takes its
         iteration count, rounded up to even, as the body (later generations
-        that need more iterations simply take more passes). Each
-        call then enqueues ``pa_loop_launch`` (x_init copied in, pa_init's
-        kernel, one launch of the graph) and ``pa_poll_begin`` (x_T and the
-        counters copied out): no host round trip inside a generation. With
-        ``wait`` the call
-        returns after that poll; without it, it returns at once with at most
-        two generations in flight (a third call first waits for the oldest and
-        checks it), and ``finish()`` waits for the rest; ``out`` and x_init
-        must then stay untouched until then.
+        that need more iterations simply take more passes). Each call then
+        enqueues ``pa_loop_launch`` (x_init copied in, pa_init's kernel, one
+        launch of the graph) and ``pa_poll_begin`` (x_T and the counters
+        copied out): no host round trip inside a generation. With ``wait``
+        the call returns after that poll; without it, it returns at once with
+        at most two generations in flight (a third call first waits for the
+        oldest and checks it), and ``finish()`` waits for the rest; ``out``
+        and x_init must then stay untouched until then. The capture runs with
+        the garbage collector paused (no finalizer's CUDA call lands in it).
 
         Where the loop cannot be built (a driver without conditional graph
-        nodes), ``chunk`` (even) iterations are captured as a CUDA graph and
-        replayed with one ``pa_poll_result`` per replay instead (always
-        waiting). The captured launches carry the solver's settings of the
+        nodes, or a capture the runtime invalidated), ``chunk`` (even)
+        iterations are captured as a CUDA graph and replayed with one
+        ``pa_poll_result`` per replay instead (always waiting). The captured launches carry the solver's settings of the
         capture: the setters of this class drop them; a denoiser's own settings
         must stay as they were captured (or pass a new callable)."""
         if chunk is None:
@@ -262,7 +262,7 @@ class Solver:
         if end_error is not None:
             if end_error.status != abi.PA_ERR_CUDA:
                 raise end_error
-            self.loop_error = str(end_error)  # this driver cannot run the loop: replay and poll instead
+            self.loop_error = str(end_error)  # refused or invalidated: replay and poll instead
             return
         self._loop_for = (denoise, chunk)
 
