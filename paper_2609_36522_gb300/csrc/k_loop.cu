@@ -13,7 +13,7 @@ namespace {
 __global__ void k_loop_cond(cudaGraphConditionalHandle h, Ctl* ctl, int32_t limit) {
   pdl_wait();  // the counters come from the planning kernel just before
   if (threadIdx.x != 0) return;
-  const int32_t c = ctl->loop_passes + 1;  // cleared by the graph's memset node at each launch
+  const int32_t c = ctl->loop_passes + 1;  // zeroed by pa_init's kernel before each launch
   ctl->loop_passes = c;
   const bool more = ctl->n_active > 0 && ctl->status == kDevOk && c < limit;
   cudaGraphSetConditional(h, more ? 1u : 0u);
