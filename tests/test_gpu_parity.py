@@ -240,7 +240,8 @@ def test_gmm_kernel_against_oracle(wname, n, max_rows, form):
     rows spread over the whole schedule, with the device row count below the
     capacity and not a multiple of the cluster form's 8-row blocks, and over
     three calls in a row (the fixed-point accumulators and the tickets are
-    reused). With 64 components: one row, 70 rows (a ragged second 64-row
+    reused). Rows past the count hold NaN: the cluster form copies them with
+    the block and must keep them out of every counted row. With 64 components: one row, 70 rows (a ragged second 64-row
     block of the tensor-core form's row tiles is not reached; rows past 48
     are), and full 128-row tiles; exactly 32 components; 3 components over 64
     columns (4 columns per CTA of the cluster form)."""
@@ -260,7 +261,7 @@ def test_gmm_kernel_against_oracle(wname, n, max_rows, form):
         g.close()
         return
     g.set_form(form)
-    xd = torch.zeros(max_rows, w.D, dtype=torch.float32, device=dev)
+    xd = torch.full((max_rows, w.D), float("nan"), dtype=torch.float32, device=dev)
     xd[:n] = torch.from_numpy(x).to(dev)
     md = torch.zeros(max_rows, 2, dtype=torch.int32, device=dev)
     md[:n] = torch.from_numpy(miss).to(dev)
