@@ -102,6 +102,11 @@ def test_large_latent():
     # a 1000-point window: tiled update kernel, one-CTA planner (2 x 1000 pairs)
     W.Workload("window 1000", T=1000, window=1000, batch=2, latent_shape=(4, 4, 4), K=3,
                tol=1e-3, cache_thresh=0.05, seed=16),
+    # the largest problem the limits admit: 64 trajectories (the batch limit)
+    # of the longest schedule, the window asked at its limit of 1024 and
+    # clamped to T = 1000: 64,000 pairs, a 64,000-row denoiser batch
+    W.Workload("64 x 1000", T=1000, window=1024, batch=64, latent_shape=(4, 4, 4), K=3,
+               tol=1e-3, cache_thresh=0.05, seed=18),
 ], ids=lambda w: w.name)
 def test_edge_shapes(w):
     _check(w)
