@@ -82,13 +82,13 @@ NCU_TRAFFIC = {
     ("772d428baaa1dd59", "large"): 79809462,     # 70,969,051 + 8,840,411
 }
 # ncu average duration per launch (cold cache, serialised) of the solver-step
-# and denoiser kernels over one generation's launches, the same key: sd15 and
-# large from the launch lists (`--metrics gpu__time_duration.sum`), batched
-# from the DRAM-bytes capture of the same launches.
+# and denoiser kernels over the launches of a launch list (`--metrics
+# gpu__time_duration.sum`, the launch lists kept under profiles/), the same key.
 NCU_LAUNCH_US = {
     ("772d428baaa1dd59", "sd15"): {"k_update_lean": 8.93, "k_plan_gather": 7.57, "k_gmm_cluster": 10.07,
                                    "k_init": 4.60},
-    ("772d428baaa1dd59", "batched"): {"k_update_lean": 19.91, "k_plan_gather": 11.61, "k_gmm_cluster": 21.80},
+    ("772d428baaa1dd59", "batched"): {"k_update_lean": 18.34, "k_plan_gather": 10.37, "k_gmm_cluster": 20.55,
+                                      "k_init": 6.19},
     ("772d428baaa1dd59", "large"): {"k_update_lean": 34.94, "k_plan_gather": 11.10, "k_gmm_dots_tc": 40.21,
                                     "k_gmm_resp": 4.39, "k_gmm_out_tc": 25.72, "k_init": 9.39},
 }
@@ -699,8 +699,9 @@ def run_ours(args):
         "event_timed_launch_us": 1000.0 * upd_ms / max(1, args.steps * n_iters),
         "ncu_kernel_avg_us": NCU_LAUNCH_US.get((sha, tkey)),
         "ncu_kernel_avg_note": ("ncu gpu__time_duration per launch, cold cache and serialised, averaged over "
-                                "one generation; a stored figure from an earlier capture of this command, keyed "
-                                "by the kernel sources' hash (null: not captured for these sources)"),
+                                "the launches of an earlier ncu launch list of this workload's bench command "
+                                "(several generations); a stored figure keyed by the kernel sources' hash (null: "
+                                "not captured for these sources)"),
         "timing": ("a CUDA graph of the generation's solver-step launches fed the eps rows recorded "
                    "from the same generation, with pa_debug_gap (an empty kernel with the same "
                    "dependent-launch attribute) where the denoiser ran; pa_init replayed before it, "
