@@ -76,7 +76,8 @@ __global__ void __launch_bounds__(kGatherThreads) k_gather(Dev d, int par) {
 // timestep of every first window enters for the first time, hence is a miss
 // (Sec. 2.2); states 1..p are lazy copies of state 0 = x_init, so the frontier
 // e starts at 0 and batch row r = b p0 + j is state 0 of trajectory b. One
-// launch on the gather's grid: each CTA copies its part of its batch row; all
+// launch on the planning kernel's grid: each CTA copies its part of its batch
+// rows; all
 // CTAs together write the ranks and the miss list and clear both sets of the
 // reduction accumulators (the entries that are added into, every
 // kAccStride-th) and the fused step's barrier counter; CTA (0, 0) writes the
@@ -304,7 +305,8 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 // and Eq. 4 distances; every CTA reads them (B*P of each), divides by D and
 // takes the whole decision in shared memory -- the same inputs and the same
 // arithmetic give the same plan in every CTA -- then copies the column range
-// blockIdx.x of batch row blockIdx.y, if that row holds a miss. CTA (0, 0)
+// blockIdx.x of batch rows blockIdx.y, blockIdx.y + gridDim.y, ... that hold
+// a miss (one row per CTA unless the rows outnumber one wave of CTAs). CTA (0, 0)
 // also publishes the plan (copy par ^ 1 of the trajectories and counters,
 // ranks, miss list, iteration log, the reductions for the host) and clears
 // the accumulator set of iteration k+1. Nobody waits for anybody: the other
@@ -325,6 +327,29 @@ struct RedSums {
   __device__ bool near(int q) const { return sum_lt(__ldcg(dl + (size_t)q * kAccStride), thr_d); }
 };
 
+// The miss of batch row r < ds.total from the decision's chunk bits: chunk c
+// holds ranks cbase[c] .. cbase[c] + popc(cmiss[c]) - 1, in bit order. Every
+// lane of a warp calls it and gets the same answer; false if no chunk holds
+// row r (never expected).
+__device__ __forceinline__ bool row_miss(const DecideShared& ds, int B, int P, int r, int* b, int* i) {
+  const int lane = threadIdx.x & 31;
+  const int nchunk = (B * P + 31) / 32;  // <= 32 (kFusedMaxPairs)
+  const unsigned mm = lane < nchunk ? ds.cmiss[lane] : 0u;
+  const int base = lane < nchunk ? ds.cbase[lane] : 0;
+  const unsigned held = __ballot_sync(0xffffffffu, lane < nchunk && r >= base && r < base + __popc(mm));
+  if (held == 0u) return false;
+  const int c = __ffs(held) - 1;
+  const unsigned m = __shfl_sync(0xffffffffu, mm, c);
+  const int n = r - __shfl_sync(0xffffffffu, base, c);  // row r is the n-th miss of chunk c
+  const unsigned at = __ballot_sync(0xffffffffu, ((m >> lane) & 1u) && __popc(m & ((1u << lane) - 1u)) == n);
+  if (at == 0u) return false;
+  const int q = c * 32 + __ffs(at) - 1;
+  if (q >= B * P) return false;
+  *b = q / P;
+  *i = ds.tn[*b] + (q - *b * P);
+  return true;
+}
+
 template <int VEC>
 __global__ void __launch_bounds__(kPlanThreads, kPlanPerSm) k_plan_gather(Dev d, int par) {
   __shared__ DecideShared ds;
@@ -334,11 +359,23 @@ __global__ void __launch_bounds__(kPlanThreads, kPlanPerSm) k_plan_gather(Dev d,
   pdl_trigger();  // the successor may now run its prologue
   stage_decision_bits(d, ds, par, publish ? 0 : -1, 1);
   __syncthreads();  // the decision's input bits and decide_load's state are staged
-  decide_par(d, ds, par, publish ? 0 : -1, 1, (int)blockIdx.y);
-  __syncthreads();  // the plan (batch row of this CTA) is known
-  if ((int)blockIdx.y < ds.total && ds.target_b >= 0) {
-    const int b = ds.target_b;
-    copy_row<VEC>(d, b, min(ds.target_i, ds.en[b]), blockIdx.y);
+  const bool one_row = (int)gridDim.y >= d.B * d.P;  // every batch row has its own CTA
+  decide_par(d, ds, par, publish ? 0 : -1, 1, one_row ? (int)blockIdx.y : -1);
+  __syncthreads();  // the plan (the batch rows of this CTA) is known
+  if (one_row) {
+    if ((int)blockIdx.y < ds.total && ds.target_b >= 0) {
+      const int b = ds.target_b;
+      copy_row<VEC>(d, b, min(ds.target_i, ds.en[b]), blockIdx.y);
+    }
+    return;
+  }
+  for (int r = blockIdx.y; r < ds.total; r += gridDim.y) {
+    int b = 0, i = 0;
+    if (!row_miss(ds, d.B, d.P, r, &b, &i)) {
+      if (threadIdx.x == 0) set_status(d.ctl, kDevBadRank);
+      continue;
+    }
+    copy_row<VEC>(d, b, min(i, ds.en[b]), r);
   }
 }
 
@@ -397,8 +434,9 @@ cudaError_t launch_gather(const Dev& d, int par, cudaStream_t st) {
 namespace {
 // The grid of a kernel whose CTA (x, y) copies part x of batch row y: as many
 // parts per row as keep the grid within per_sm CTAs per SM (one wave), each
-// part at least 1024 float4 columns. An error only if the SM count cannot be
-// read.
+// part at least 1024 float4 columns; with more rows than one wave holds, one
+// wave of whole-row CTAs, CTA y taking rows y, y + gridDim.y, ... An error
+// only if the SM count cannot be read.
 cudaError_t split_grid(const Dev& d, int per_sm, dim3* out) {
   static int nsm[64] = {};
   int dev = 0;
@@ -416,6 +454,9 @@ cudaError_t split_grid(const Dev& d, int per_sm, dim3* out) {
   if (gx > cap) gx = cap;
   if (gx > 64) gx = 64;
   g.x = gx < 1 ? 1 : (unsigned)gx;
+  // more rows than one wave of CTAs: one wave, each CTA taking every
+  // gridDim.y-th row (the planning kernel then plans once per CTA, not per row)
+  if ((int64_t)g.y > (int64_t)per_sm * sms) g.y = (unsigned)(per_sm * sms);
   *out = g;
   return cudaSuccess;
 }

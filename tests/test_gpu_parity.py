@@ -94,6 +94,12 @@ def test_large_latent():
                tol=1e-3, cache_thresh=0.05, seed=9),
     W.Workload("tight tol", T=24, window=10, batch=2, latent_shape=(4, 16, 16), K=6,
                tol=1e-6, cache_thresh=0.02, seed=10),
+    # more batch rows than one wave of planning CTAs (2 per SM): each CTA plans
+    # once and copies every gridDim.y-th row
+    W.Workload("4 x 100 pairs", T=100, window=100, batch=4, latent_shape=(4, 8, 8), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=19),
+    W.Workload("10 x 100 pairs", T=100, window=100, batch=10, latent_shape=(4, 8, 8), K=4,
+               tol=1e-3, cache_thresh=0.05, seed=20),
     # more than 1024 (trajectory, position) pairs: one CTA plans, a separate gather follows
     W.Workload("9 x 128 pairs", T=200, window=128, batch=9, latent_shape=(4, 4, 4), K=4,
                tol=1e-3, cache_thresh=0.05, seed=13),
