@@ -77,20 +77,20 @@ NOMINAL_HBM_GBS = 8000.0
 NCU_TRAFFIC = {
     # per iteration: k_update_lean + k_plan_gather read + write bytes, averaged
     # over the first generation's launches
-    ("772d428baaa1dd59", "sd15"): 8256576,       # 6,252,672 + 2,003,904 (no DRAM writes)
-    ("772d428baaa1dd59", "batched"): 30269867,   # 24,577,920 + 5,691,947
-    ("772d428baaa1dd59", "large"): 79809462,     # 70,969,051 + 8,840,411
+    ("cccff3e1230d7880", "sd15"): 8261056,       # 6,250,944 + 2,010,112 (no DRAM writes)
+    ("cccff3e1230d7880", "batched"): 30269739,   # 24,571,478 + 5,698,261
+    ("cccff3e1230d7880", "large"): 79819739,     # 70,972,270 + 8,847,470
 }
 # ncu average duration per launch (cold cache, serialised) of the solver-step
 # and denoiser kernels over the launches of a launch list (`--metrics
 # gpu__time_duration.sum`, the launch lists kept under profiles/), the same key.
 NCU_LAUNCH_US = {
-    ("772d428baaa1dd59", "sd15"): {"k_update_lean": 8.93, "k_plan_gather": 7.57, "k_gmm_cluster": 10.07,
-                                   "k_init": 4.60},
-    ("772d428baaa1dd59", "batched"): {"k_update_lean": 18.34, "k_plan_gather": 10.37, "k_gmm_cluster": 20.55,
-                                      "k_init": 6.19},
-    ("772d428baaa1dd59", "large"): {"k_update_lean": 34.94, "k_plan_gather": 11.10, "k_gmm_dots_tc": 40.21,
-                                    "k_gmm_resp": 4.39, "k_gmm_out_tc": 25.72, "k_init": 9.39},
+    ("cccff3e1230d7880", "sd15"): {"k_update_lean": 8.77, "k_plan_gather": 7.60, "k_gmm_cluster": 10.02,
+                                   "k_init": 4.56},
+    ("cccff3e1230d7880", "batched"): {"k_update_lean": 18.33, "k_plan_gather": 10.36, "k_gmm_cluster": 20.53,
+                                      "k_init": 6.08},
+    ("cccff3e1230d7880", "large"): {"k_update_lean": 34.56, "k_plan_gather": 10.88, "k_gmm_dots_tc": 40.20,
+                                    "k_gmm_resp": 4.37, "k_gmm_out_tc": 25.55, "k_init": 9.02},
 }
 
 
