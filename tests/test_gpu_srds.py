@@ -1,6 +1,8 @@
 """Parity of the CUDA Parareal (SRDS-style) sampler with the fp64 oracle:
 the per-stage miss lists, NFE, hits and iteration count exactly, final latents
 within 1e-5 (max-abs relative)."""
+import math
+
 import numpy as np
 import pytest
 
@@ -105,15 +107,34 @@ def test_srds_async_equals_sync():
     assert a["stats"]["nfe"] == b["stats"]["nfe"]
 
 
-@pytest.mark.parametrize("T,batch,shape", [(1, 2, (4, 4, 4)), (2, 1, (4, 8, 8)), (5, 3, (3, 5, 7)),
-                                           (17, 64, (4, 4, 4))])
-def test_srds_edge_shapes(T, batch, shape):
+def srds_margin(orc, thresh):
+    """The smallest relative distance of an Eq. 4 mean change from tau_cache
+    over every hit test of the oracle's run."""
+    m = math.inf
+    for batch in orc.batches:
+        for (_b, _i, _hit, dl) in batch:
+            if dl is not None and math.isfinite(dl):
+                m = min(m, abs(dl - thresh) / thresh)
+    return m
+
+
+@pytest.mark.parametrize("T,batch,shape,seed", [(1, 2, (4, 4, 4), 31), (2, 1, (4, 8, 8), 31),
+                                                (5, 3, (3, 5, 7), 31), (17, 64, (4, 4, 4), 31),
+                                                (100, 64, (4, 4, 4), 38)])
+def test_srds_edge_shapes(T, batch, shape, seed):
     """Blocks of one step (T = 1, 2: a coarse jump and the fine step of its
     block share a timestep, so the fine stage's new entry feeds the coarse
     stage's distance in the same kernel), ragged blocks and odd D (T = 5), and
-    64 trajectories x 5 blocks of rows."""
-    w = W.TINY.with_(T=T, latent_shape=shape, K=3, sampler="srds", batch=batch, seed=31)
+    64 trajectories x 5 and x 10 blocks of rows (320 and 640 fine-stage rows:
+    more than one wave of planning CTAs, so each CTA narrows several). The
+    states behind a hit test differ from the oracle's by the fp32 rounding of
+    the denoiser's output, carried through up to T steps and N corrections,
+    so a test within a few 1e-6 of tau_cache can go either way (seed 31 at
+    T = 100 has one at 6e-6); the cases are seeded with every test at least
+    1e-4 away."""
+    w = W.TINY.with_(T=T, latent_shape=shape, K=3, sampler="srds", batch=batch, seed=seed)
     orc = oracle_srds(w)
+    assert srds_margin(orc, w.cache_thresh) > 1e-4
     compare_srds(w, orc, gpu_srds(w))
     g = gpu_srds(w, mode="async")
     assert g["stats"]["nfe"] == orc.nfe
