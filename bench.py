@@ -77,20 +77,20 @@ NOMINAL_HBM_GBS = 8000.0
 NCU_TRAFFIC = {
     # per iteration: k_update_lean + k_plan_gather read + write bytes, averaged
     # over the first generation's launches
-    ("cccff3e1230d7880", "sd15"): 8261056,       # 6,250,944 + 2,010,112 (no DRAM writes)
-    ("cccff3e1230d7880", "batched"): 30269739,   # 24,571,478 + 5,698,261
-    ("cccff3e1230d7880", "large"): 79819739,     # 70,972,270 + 8,847,470
+    ("97d9b1620ebf45c1", "sd15"): 8263616,       # 6,253,184 + 2,010,432 (no DRAM writes)
+    ("97d9b1620ebf45c1", "batched"): 30270037,   # 24,571,861 + 5,698,176
+    ("97d9b1620ebf45c1", "large"): 79946021,     # 71,099,246 + 8,846,775
 }
 # ncu average duration per launch (cold cache, serialised) of the solver-step
 # and denoiser kernels over the launches of a launch list (`--metrics
 # gpu__time_duration.sum`, the launch lists kept under profiles/), the same key.
 NCU_LAUNCH_US = {
-    ("cccff3e1230d7880", "sd15"): {"k_update_lean": 8.77, "k_plan_gather": 7.60, "k_gmm_cluster": 10.02,
-                                   "k_init": 4.56},
-    ("cccff3e1230d7880", "batched"): {"k_update_lean": 18.33, "k_plan_gather": 10.36, "k_gmm_cluster": 20.53,
-                                      "k_init": 6.08},
-    ("cccff3e1230d7880", "large"): {"k_update_lean": 34.56, "k_plan_gather": 10.88, "k_gmm_dots_tc": 40.20,
-                                    "k_gmm_resp": 4.37, "k_gmm_out_tc": 25.55, "k_init": 9.02},
+    ("97d9b1620ebf45c1", "sd15"): {"k_update_lean": 8.77, "k_plan_gather": 7.54, "k_gmm_cluster": 10.01,
+                                   "k_init": 4.58},
+    ("97d9b1620ebf45c1", "batched"): {"k_update_lean": 18.30, "k_plan_gather": 10.35, "k_gmm_cluster": 20.53,
+                                      "k_init": 6.06},
+    ("97d9b1620ebf45c1", "large"): {"k_update_lean": 34.57, "k_plan_gather": 10.92, "k_gmm_dots_tc": 40.10,
+                                    "k_gmm_resp": 4.36, "k_gmm_out_tc": 25.50, "k_init": 8.95},
 }
 
 

@@ -313,7 +313,13 @@ __global__ void __launch_bounds__(kPlainThreads) k_update_plain(Dev d, const flo
 // CTAs read copy par of the plan, which no CTA writes in this launch.
 constexpr int kPlanThreads = 256;
 constexpr int kPlanPerSm = 2;   // planning CTAs per SM (three: the launch bound makes the decision spill, slower)
-constexpr int kFusedMaxPairs = 1024;  // B*P planned in every CTA; beyond, one CTA plans
+constexpr int kFusedMaxPairs = 1024;  // B*P planned in every CTA at most; beyond, one CTA plans
+// Beyond this many pairs one CTA plans and a separate gather follows unless
+// tau_cache adapts (only the every-CTA planner forms the next tau): at the SD
+// latent with 800 and 1000 pairs that measured 49.9 and 59.8 us per solver
+// step against 51.7 and 62.8 us, at 300 and 400 pairs 28.6 and 34.9 against
+// 27.9 and 34.4 us
+constexpr int kFusedPreferPairs = 512;
 static_assert(kFusedMaxPairs <= 32 * 32, "decide_par keeps one miss mask per 32-position chunk, 32 of them");
 
 // The complete sums read from global memory (one-CTA planner).
@@ -379,8 +385,8 @@ __global__ void __launch_bounds__(kPlanThreads, kPlanPerSm) k_plan_gather(Dev d,
   }
 }
 
-// One-CTA planner for B*P beyond kFusedMaxPairs: reads the sums from memory;
-// a separate gather follows.
+// One-CTA planner for B*P beyond kFusedPreferPairs (without adaptation) or
+// kFusedMaxPairs: reads the sums from memory; a separate gather follows.
 constexpr int kPlanOneThreads = 1024;
 
 __global__ void __launch_bounds__(kPlanOneThreads) k_plan_one(Dev d, int par) {
@@ -471,7 +477,8 @@ cudaError_t launch_init(const Dev& d, cudaStream_t st) {
 }
 
 cudaError_t launch_plan(const Dev& d, int par, cudaStream_t st, int* launches) {
-  if (d.B * d.P <= kFusedMaxPairs) {
+  const int npair = d.B * d.P;
+  if (npair <= kFusedPreferPairs || (d.adapt && npair <= kFusedMaxPairs)) {
     *launches = 1;
     // every CTA plans and copies a part of its batch row
     dim3 g;

@@ -69,8 +69,8 @@ LOOP_CASES = [
     ("9 x 128 pairs", W.Workload("9 x 128 pairs", T=200, window=128, batch=9, latent_shape=(4, 4, 4), K=4,
                                  tol=1e-3, cache_thresh=0.05, seed=13), {"chunk": None}),
     # more batch rows than one wave of planning CTAs: each CTA copies several rows
-    ("10 x 100 pairs", W.Workload("10 x 100 pairs", T=100, window=100, batch=10, latent_shape=(4, 8, 8), K=4,
-                                  tol=1e-3, cache_thresh=0.05, seed=20), {"chunk": None}),
+    ("4 x 100 pairs", W.Workload("4 x 100 pairs", T=100, window=100, batch=4, latent_shape=(4, 8, 8), K=4,
+                                 tol=1e-3, cache_thresh=0.05, seed=19), {"chunk": None}),
     ("window past T, odd T", W.Workload("odd", T=37, window=64, batch=3, latent_shape=(4, 8, 8), K=4,
                                         tol=1e-3, cache_thresh=0.05, seed=15), {"chunk": 2}),
     ("ragged D", W.Workload("ragged", T=20, window=7, batch=2, latent_shape=(3, 7, 9), K=4,

@@ -98,6 +98,7 @@ def test_large_latent():
     # once and copies every gridDim.y-th row
     W.Workload("4 x 100 pairs", T=100, window=100, batch=4, latent_shape=(4, 8, 8), K=4,
                tol=1e-3, cache_thresh=0.05, seed=19),
+    # past 512 pairs one CTA plans and a separate gather follows
     W.Workload("10 x 100 pairs", T=100, window=100, batch=10, latent_shape=(4, 8, 8), K=4,
                tol=1e-3, cache_thresh=0.05, seed=20),
     # more than 1024 (trajectory, position) pairs: one CTA plans, a separate gather follows
@@ -741,6 +742,10 @@ ADAPT_CASES = [
     (W.TINY, (1.0, 0.9, 0.0, 1.0), {}),
     (W.SD15.with_(cache_thresh=0.02, name="SD fused"), (0.5, 0.5, 0.0, 0.2), {"update_kernel": 3}),
     (W.SD15.with_(cache_thresh=0.02, name="SD anderson"), (0.5, 0.5, 0.0, 0.2), {"anderson": 1}),
+    # 1000 pairs: without adaptation one CTA would plan; adaptation keeps the
+    # every-CTA planner, here with several batch rows per CTA
+    (W.Workload("10 x 100 adaptive", T=100, window=100, batch=10, latent_shape=(4, 8, 8), K=4,
+                tol=1e-3, cache_thresh=0.02, seed=21), (0.5, 0.5, 0.0, 0.2), {}),
 ]
 
 
